@@ -1,0 +1,125 @@
+"""The Oscars round loop, CPU oracle (test infrastructure only).
+
+Reading of Eq. 4 (its condition ``t mod tau_i = 0`` is per worker while its
+average is global): training proceeds in rounds.  In every round each worker
+i starts from the global model (pull), runs exactly tau_i local SGD steps on
+its own data ("otherwise" branch), pushes its model, and at the barrier T*
+the server replaces the global model with the merge of the pushed models
+(first branch).  Speeds are steady (Section "Problem Formulation"), so T* and
+tau are computed once; synchronisation time is ignored, so the simulated
+clock of worker i advances by tau_i * t_i of compute and mod(T*, t_i) of idle
+time (Eq. 1) per round.
+
+Mini-batches (a reading; the data-partition section of the paper is empty):
+worker i reads its shard sequentially from a cursor that persists across
+rounds and wraps modulo the shard size.
+"""
+from __future__ import annotations
+
+from dataclasses import dataclass, field
+from typing import Callable, List, Optional, Sequence, Tuple
+
+import numpy as np
+
+from . import bf16 as _bf16
+from . import merge as _merge
+from . import model as _model
+from . import schedule as _sched
+
+
+def flatten(layers) -> np.ndarray:
+    """Canonical flat vector W_0, b_0, W_1, b_1, ... (fp32)."""
+    return np.concatenate([np.concatenate([W.reshape(-1), b.reshape(-1)]) for W, b in layers]).astype(np.float32)
+
+
+def unflatten(flat: np.ndarray, dims: Sequence[int]):
+    out, off = [], 0
+    for i, o in zip(dims[:-1], dims[1:]):
+        W = np.asarray(flat[off:off + o * i], dtype=np.float32).reshape(o, i); off += o * i
+        b = np.asarray(flat[off:off + o], dtype=np.float32); off += o
+        out.append((W, b))
+    return out
+
+
+def batch_indices(cursor: int, batch: int, n: int) -> np.ndarray:
+    return (cursor + np.arange(batch, dtype=np.int64)) % n
+
+
+@dataclass
+class RoundRecord:
+    tau: np.ndarray
+    T_star: int
+    worker_loss: np.ndarray          # mean mini-batch loss of each worker this round
+    idle: np.ndarray                 # idle ticks of each worker this round (Eq. 1)
+    x_g: Optional[np.ndarray] = None # global model after the merge (flat, fp32)
+    eval_loss: Optional[float] = None
+
+
+@dataclass
+class OscarsState:
+    dims: List[int]
+    x_g: List[Tuple[np.ndarray, np.ndarray]]
+    cursor: np.ndarray
+    clock: np.ndarray
+    idle: np.ndarray
+    t_iter: np.ndarray
+    T_star: int
+    max_wait: int
+    tau: np.ndarray
+
+
+def init_state(dims, layers0, t_iter, M: int, mode: int = _sched.CAPPED, tau_override=None) -> OscarsState:
+    T_star, mw, tau = _sched.schedule(t_iter, M, mode)
+    if tau_override is not None:
+        tau = np.asarray(tau_override, dtype=np.int32)
+    W = len(t_iter)
+    return OscarsState(list(dims), [(W_.copy(), b.copy()) for W_, b in layers0],
+                       np.zeros(W, np.int64), np.zeros(W, np.int64), np.zeros(W, np.int64),
+                       np.asarray(t_iter, np.int64), T_star, mw, tau)
+
+
+def local_steps(state: OscarsState, worker: int, shard, batch: int, lr: float, rnd: Callable):
+    """Worker ``worker`` pulls the global model and runs tau_i local SGD steps."""
+    X, y = shard
+    layers = [(W.copy(), b.copy()) for W, b in state.x_g]          # pull
+    losses = []
+    for _ in range(int(state.tau[worker])):
+        idx = batch_indices(int(state.cursor[worker]), batch, X.shape[0])
+        state.cursor[worker] = (state.cursor[worker] + batch) % X.shape[0]
+        layers, loss = _model.sgd_step(layers, X[idx], y[idx], lr, rnd)
+        losses.append(loss)
+    return layers, float(np.mean(losses))
+
+
+def run_round(state: OscarsState, shards, batch: int, lr: float, rnd: Callable,
+              weight_rule: str = "uniform", server_lr: float = 1.0, weights=None) -> RoundRecord:
+    W = len(shards)
+    models, wl = [], np.zeros(W)
+    for i in range(W):
+        layers, wl[i] = local_steps(state, i, shards[i], batch, lr, rnd)
+        models.append(flatten(layers))                             # push
+    w = _sched.merge_weights(weight_rule, state.tau, weights)
+    x_new = _merge.merge_models(flatten(state.x_g), models, w, server_lr)
+    state.x_g = unflatten(x_new, state.dims)
+    idle = state.T_star - state.tau.astype(np.int64) * state.t_iter     # = mod(T*, t_i)
+    state.clock += state.tau.astype(np.int64) * state.t_iter + idle
+    state.idle += idle
+    return RoundRecord(state.tau.copy(), state.T_star, wl, idle, x_new)
+
+
+def run(dims, layers0, shards, speeds=None, t_iter=None, M: int = 8, rounds: int = 1,
+        batch: int = 32, lr: float = 0.05, bf16: bool = True, weight_rule: str = "uniform",
+        server_lr: float = 1.0, mode: int = _sched.CAPPED, tau_override=None,
+        eval_set=None, ticks_per_unit: int = 1000):
+    """Run ``rounds`` Oscars rounds; returns (final state, [RoundRecord])."""
+    if t_iter is None:
+        t_iter = _sched.iteration_ticks(speeds, ticks_per_unit)
+    rnd = _bf16.round_bf16 if bf16 else _bf16.identity
+    state = init_state(dims, layers0, t_iter, M, mode, tau_override)
+    records = []
+    for _ in range(rounds):
+        rec = run_round(state, shards, batch, lr, rnd, weight_rule, server_lr)
+        if eval_set is not None:
+            rec.eval_loss = _model.loss_of(state.x_g, eval_set[0], eval_set[1], rnd)
+        records.append(rec)
+    return state, records
