@@ -1,0 +1,409 @@
+#!/usr/bin/env python
+"""Benchmark of the Oscars hot path on one GB300 (or N independent replicas).
+
+A step is one Oscars round of the 784-512-10 MLP workload with W=16 workers
+(batch 64): every worker's tau_i local SGD steps (the schedule of Algorithm 1),
+the push, the server merge and global update (Eq. 4) and the pull.  The
+headline metric is simulated-worker samples per second (sum_i tau_i * B per
+round).  The same JSON line carries the server-merge microbenchmarks (P=25.6M,
+W=64 and P=340M, W=8) as GB/s and fraction of HBM bandwidth.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl oscars|reference]
+
+--impl reference times the CPU oracle (the plain numpy restatement of the
+method) on the same workload and metric.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+import synth  # noqa: E402
+
+WORKLOAD = synth.CFG2
+METRIC = "simulated-worker samples/s (Oscars rounds; merge GB/s alongside)"
+UNIT = "samples/s"
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=30)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", default="oscars", choices=["oscars", "reference"])
+    ap.add_argument("--no-merge", action="store_true", help="skip the merge microbenchmarks")
+    ap.add_argument("--no-cpu", action="store_true", help="skip the CPU oracle baseline")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--merge-reps", type=int, default=20)
+    return ap.parse_args()
+
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        d = json.load(open(p))
+        return d["hbm_gbs"], d["bf16_tflops"], d.get("bf16_tflops_sustained", d["bf16_tflops"]), "measured"
+    return 6800.0, 1900.0, 1700.0, "fallback"
+
+
+def schedule_of(w):
+    from oracle import schedule as S  # schedule inputs only; not timed
+    t = S.iteration_ticks(synth.speeds(w), w.ticks_per_unit)
+    return S.schedule(t, w.M)
+
+
+def workload_config(w, l2):
+    return {"workload": f"{w.name} (W={w.num_workers}, dims={'-'.join(map(str, w.dims))}, batch={w.batch}, "
+                        f"M={w.M}, lognormal(0,0.5) speeds)",
+            "W": w.num_workers, "dims": w.dims, "batch": w.batch, "M": w.M, "lr": w.lr,
+            "samples_per_worker": w.samples_per_worker, "l2": l2}
+
+
+# ------------------------------------------------------------------ clocks
+class ClockSampler:
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_{os.getpid()}.csv")
+
+    def __enter__(self):
+        try:
+            os.makedirs(os.path.dirname(self.path), exist_ok=True)
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index),
+                 "--query-gpu=index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+                 "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+                 "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap",
+                 "--format=csv,noheader,nounits", "-lms", "200"], stdout=self.f, stderr=subprocess.DEVNULL)
+            time.sleep(0.3)
+        except Exception:
+            self.proc = None
+        return self
+
+    def __exit__(self, *a):
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+            self.f.close()
+
+    def summary(self):
+        if not self.proc:
+            return None
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.path):
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx.append(float(f[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower() in ("active", "1", "0x1"):
+                    reasons.add(n)
+        if not sm:
+            return None
+        return {"sm_mhz": float(np.median(sm)), "sm_max_mhz": max(mx), "samples": len(sm),
+                "reasons": sorted(reasons)}
+
+
+# ------------------------------------------------------------------ GPU arm
+def algorithmic_work(w, tau):
+    """Per-round algorithmic FLOPs and bytes of each kernel class."""
+    B, dims = w.batch, w.dims
+    n_steps = int(np.sum(tau))
+    L = len(dims) - 1
+    flops = {}
+    fwd = sum(2.0 * B * dims[l] * dims[l + 1] for l in range(L - 1))
+    dw = sum(2.0 * B * dims[l] * dims[l + 1] for l in range(L - 1))
+    dh = sum(2.0 * B * dims[l] * dims[l + 1] for l in range(1, L - 1))
+    head = 3 * 2.0 * B * dims[L - 1] * dims[L]
+    flops["gemm_fwd"] = fwd * n_steps
+    flops["gemm_dw_sgd"] = dw * n_steps
+    flops["gemm_dh"] = dh * n_steps
+    flops["head_fwd"] = head / 3 * n_steps
+    flops["head_bwd"] = head * 2 / 3 * n_steps
+    P = w.num_params
+    bytes_ = {"merge": (w.num_workers + 2) * P * 4.0}
+    return flops, bytes_
+
+
+def run_gpu(args, rank, world, local_rank):
+    import torch
+    import paper_2102_08550_gb300 as P
+    from paper_2102_08550_gb300 import _build
+
+    _build.build()
+    dev = torch.device(f"cuda:{local_rank}")
+    torch.cuda.set_device(dev)
+    w = WORKLOAD
+    hbm, tf_burst, tf_sus, peak_kind = peaks()
+    T_star, mw, tau = schedule_of(w)
+    samples_per_round = int(np.sum(tau)) * w.batch
+
+    shards = [synth.shard_t(w, k, dev) for k in range(w.num_workers)]
+    layers0 = synth.init_layers_np(w)
+    init = torch.from_numpy(synth.flatten_layers(layers0)).to(dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def make(flags=0):
+        return P.OscarsContext(num_workers=w.num_workers, dims=w.dims, batch=w.batch, lr=w.lr,
+                               speed=synth.speeds(w).tolist(), M=w.M, shards=shards, init_params=init,
+                               stream=stream.cuda_stream, flags=flags)
+
+    ctx = make()
+    flush = torch.empty(512 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)   # > L2 (129 MB)
+
+    def one_round():
+        P.oscars_local_steps(ctx.handle, want_tau=False, want_loss=False)
+        P.oscars_push_merge(ctx.handle)
+
+    for _ in range(args.warmup):
+        one_round()
+    torch.cuda.synchronize()
+    if world > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    with ClockSampler(local_rank) as clk:
+        for i in range(args.steps):
+            flush.fill_(float(i))            # evict the previous round's state from L2 (untimed)
+            evs[i][0].record(stream)
+            one_round()
+            evs[i][1].record(stream)
+        torch.cuda.synchronize()
+    total_ms = sum(a.elapsed_time(b) for a, b in evs)
+    if world > 1:
+        t = torch.tensor([total_ms], device=dev)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        total_ms = float(t.item())
+    torch.cuda.synchronize()
+    value = samples_per_round * args.steps * world / (total_ms / 1e3)
+
+    # ---- per-kernel device time: the same rounds with each launch timed
+    pctx = make(flags=P.FLAG_NO_GRAPH | P.FLAG_PROFILE)
+    for _ in range(2):
+        P.oscars_local_steps(pctx.handle, want_tau=False, want_loss=False)
+        P.oscars_push_merge(pctx.handle)
+    torch.cuda.synchronize()
+    pctx.profile_reset()
+    prof_rounds = max(3, min(args.steps, 10))
+    for i in range(prof_rounds):
+        flush.fill_(float(i))
+        P.oscars_local_steps(pctx.handle, want_tau=False, want_loss=False)
+        P.oscars_push_merge(pctx.handle)
+    prof = pctx.profile()
+    torch.cuda.synchronize()
+    pctx.close()
+    launches_per_round = sum(c for _, c in prof.values()) / prof_rounds
+    flops, bytes_ = algorithmic_work(w, tau)
+    dom = max(prof, key=lambda k: prof[k][0])
+    dom_ms_per_launch = prof[dom][0] / prof[dom][1]
+    launches_dom_per_round = prof[dom][1] / prof_rounds
+    kernels = {k: {"ms_per_round": v[0] / prof_rounds, "launches_per_round": v[1] / prof_rounds,
+                   "share": v[0] / sum(x[0] for x in prof.values())} for k, v in prof.items()}
+    if dom in flops:
+        per_launch = flops[dom] / launches_dom_per_round
+        achieved = per_launch / (dom_ms_per_launch / 1e3) / 1e12
+        roof = {"kernel": dom, "bound": "tensor", "achieved": achieved, "peak": tf_burst, "unit": "TFLOP/s",
+                "frac": achieved / tf_burst, "peak_kind": f"{peak_kind} bf16 dense burst",
+                "work_per_launch": per_launch, "ms_per_launch": dom_ms_per_launch, "traffic": None}
+    elif dom in bytes_:
+        per_launch = bytes_[dom] / launches_dom_per_round
+        achieved = per_launch / (dom_ms_per_launch / 1e3) / 1e9
+        roof = {"kernel": dom, "bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s",
+                "frac": achieved / hbm, "peak_kind": f"{peak_kind} HBM copy", "work_per_launch": per_launch,
+                "ms_per_launch": dom_ms_per_launch, "traffic": None}
+    else:
+        roof = {"kernel": dom, "bound": "alu", "achieved": None, "peak": None, "unit": None, "frac": None,
+                "ms_per_launch": dom_ms_per_launch, "traffic": None}
+
+    # ---- end to end through the C ABI with host-resident inputs
+    e2e = None
+    if not args.no_e2e:
+        e2e = run_e2e(args, ctx, shards, w, tau, dev, stream)
+
+    merge = None if args.no_merge else run_merge(args, dev, stream, hbm, peak_kind)
+    ctx.close()
+    out = {"value": value, "ms_per_step": total_ms / args.steps, "roofline": roof, "kernels": kernels,
+           "gpu_launches": int(round(launches_per_round * args.steps)), "clocks": clk.summary(), "e2e": e2e,
+           "merge": merge, "samples_per_round": samples_per_round, "T_star": int(T_star),
+           "tau": [int(v) for v in tau]}
+    return out
+
+
+def run_e2e(args, ctx, shards, w, tau, dev, stream):
+    """Each round: copy that round's mini-batches from pinned host memory into
+    the device shards, run the round, read the losses back."""
+    import torch
+    import paper_2102_08550_gb300 as P
+    host = [(x.cpu().pin_memory(), y.cpu().pin_memory()) for x, y in shards]
+    n = w.samples_per_worker
+    B = w.batch
+    # the context's cursors after the rounds already run: warmup + steps
+    rounds_done = args.warmup + args.steps
+    cursor = [(rounds_done * int(tau[k]) * B) % n for k in range(w.num_workers)]
+    h2d = 0
+    steps = max(3, args.steps // 2)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for _ in range(steps):
+        for k in range(w.num_workers):
+            rows = int(tau[k]) * B
+            a = cursor[k]
+            segs = [(a, min(n, a + rows))]
+            if a + rows > n:
+                segs.append((0, a + rows - n))
+            for s0, s1 in segs:
+                shards[k][0][s0:s1].copy_(host[k][0][s0:s1], non_blocking=True)
+                shards[k][1][s0:s1].copy_(host[k][1][s0:s1], non_blocking=True)
+                h2d += (s1 - s0) * (w.dims[0] * 4 + 4)
+            cursor[k] = (a + rows) % n
+        _, loss = P.oscars_local_steps(ctx.handle, want_tau=False, want_loss=True)   # D2H of W losses
+        P.oscars_push_merge(ctx.handle)
+    torch.cuda.synchronize()
+    dt = time.perf_counter() - t0
+    samples = int(np.sum(tau)) * B * steps
+    return {"value": samples / dt, "unit": UNIT, "h2d_bytes_per_step": h2d // steps,
+            "d2h_bytes_per_step": 4 * w.num_workers, "steps": steps,
+            "note": "host wall clock; pinned-host mini-batch copies + local steps + merge + loss readback"}
+
+
+def run_merge(args, dev, stream, hbm, peak_kind):
+    import torch
+    import paper_2102_08550_gb300 as P
+    res = {}
+    for m in (synth.CFG4, synth.CFG5):
+        W, Pn = m.num_workers, m.num_params
+        rule = P.W_LOCALSTEPS if m.weight_rule == "localsteps" else P.W_UNIFORM
+        xg0 = synth.merge_xg_t(m, 0, Pn, dev)
+        deltas = [synth.merge_delta_t(m, k, 0, Pn, dev) for k in range(W)]
+        ctx = P.OscarsContext(num_workers=W, dims=[Pn], model=P.MODEL_FLAT, weight_rule=rule, t_ticks=[1] * W,
+                              M=2, init_params=xg0, server_lr=m.server_lr, stream=stream.cuda_stream)
+        del xg0
+        ctx.set_local_steps(synth.merge_taus(m).tolist())
+        ptrs = [d.data_ptr() for d in deltas]
+        for _ in range(3):
+            P.oscars_push_merge(ctx.handle, ptrs)
+        torch.cuda.synchronize()
+        evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+               for _ in range(args.merge_reps)]
+        for a, b in evs:
+            a.record(stream)
+            P.oscars_push_merge(ctx.handle, ptrs)
+            b.record(stream)
+        torch.cuda.synchronize()
+        ts = sorted(a.elapsed_time(b) for a, b in evs)
+        med = ts[len(ts) // 2]
+        alg = (W + 2) * Pn * 4.0
+        gbs = alg / (med / 1e3) / 1e9
+        res[m.name] = {"GB/s": gbs, "frac": gbs / hbm, "ms_median": med, "ms_min": ts[0],
+                       "bytes_per_launch": alg, "weight_rule": m.weight_rule,
+                       "peak": hbm, "peak_kind": f"{peak_kind} HBM copy", "bound": "hbm", "traffic": None,
+                       "l2": "inputs larger than L2"}
+        ctx.close()
+        del deltas
+        torch.cuda.empty_cache()
+    return res
+
+
+# ------------------------------------------------------------------ CPU oracle
+def oracle_rounds(w, rounds, budget_s):
+    """Run up to ``rounds`` oracle rounds (stopping after budget_s seconds);
+    returns (samples, seconds, rounds run)."""
+    from oracle import run as orun
+    from oracle import bf16 as obf16
+    from oracle import schedule as S
+    t = S.iteration_ticks(synth.speeds(w), w.ticks_per_unit)
+    T, mw, tau = S.schedule(t, w.M)
+    rows = min(w.samples_per_worker, rounds * int(tau.max()) * w.batch + w.batch)
+    shards = [synth.shard_np(w, k, n=rows) for k in range(w.num_workers)]
+    state = orun.init_state(w.dims, synth.init_layers_np(w), t, w.M)
+    rnd = obf16.round_bf16 if w.bf16 else obf16.identity
+    t0 = time.perf_counter()
+    done = 0
+    for _ in range(rounds):
+        orun.run_round(state, shards, w.batch, w.lr, rnd)
+        done += 1
+        if time.perf_counter() - t0 > budget_s:
+            break
+    dt = time.perf_counter() - t0
+    return done * int(np.sum(tau)) * w.batch, dt, done
+
+
+def cores_used():
+    try:
+        return len(os.sched_getaffinity(0))
+    except Exception:
+        return os.cpu_count()
+
+
+def run_reference(args):
+    w = WORKLOAD
+    oracle_rounds(w, max(1, min(args.warmup, 2)), 30.0)          # warm-up (imports, caches)
+    samples, dt, done = oracle_rounds(w, args.steps, 120.0)
+    value = samples / dt
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+            "steps": done, "warmup": args.warmup, "ms_per_step": dt / done * 1e3, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64 (bf16 operand emulation)", "data": "synthetic",
+            "config": workload_config(w, "n/a (CPU)"),
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores_used(), "kind": "oracle",
+                             "sample": f"{done} Oscars rounds of {w.name} (numpy fp64, BLAS threads = all cores)"},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line))
+
+
+def main():
+    args = parse()
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+    if args.impl == "reference":
+        if rank == 0:
+            run_reference(args)
+        return
+    if world > 1:
+        import torch
+        torch.cuda.set_device(local_rank)
+        torch.distributed.init_process_group("nccl")
+    res = run_gpu(args, rank, world, local_rank)
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu:
+        samples, dt, done = oracle_rounds(WORKLOAD, 6, 15.0)
+        cpu = {"value": samples / dt, "unit": UNIT, "cores": cores_used(), "kind": "oracle",
+               "sample": f"{done} Oscars rounds of {WORKLOAD.name} (numpy fp64 with bf16 operand emulation)"}
+    if rank == 0:
+        w = WORKLOAD
+        line = {"metric": METRIC, "value": res["value"], "unit": UNIT, "n_gpus": world, "steps": args.steps,
+                "warmup": args.warmup, "ms_per_step": res["ms_per_step"], "higher_is_better": True,
+                "scaling": "weak", "vs_baseline": None, "dtype": "bf16 (fp32 master, fp32 accumulate)",
+                "data": "synthetic (seeded Gaussian-mixture shards, random-init MLP)",
+                "config": workload_config(w, "flushed between timed rounds (512 MB write)"),
+                "roofline": res["roofline"], "cpu_baseline": cpu, "e2e": res["e2e"],
+                "gpu_launches": res["gpu_launches"], "clocks": res["clocks"], "merge": res["merge"],
+                "kernels": res["kernels"], "samples_per_round": res["samples_per_round"],
+                "T_star": res["T_star"], "tau": res["tau"]}
+        print(json.dumps(line))
+    if world > 1:
+        import torch
+        torch.distributed.barrier()
+        torch.distributed.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

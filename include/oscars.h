@@ -1,0 +1,266 @@
+/*
+ * oscars.h - C ABI of the GB300 (sm_103a) Oscars hot path.
+ *
+ * Oscars (arXiv 2102.08550) is semi-synchronous local SGD against a parameter
+ * server: N workers with steady but different iteration times t_i^iter each
+ * run tau_i local SGD steps between global barriers, where the barrier T* and
+ * tau_i = floor(T* / t_i^iter) come from the paper's load-balance search
+ * (Algorithm 1; Eq. 1-3); at the barrier the server merges the workers'
+ * models (Eq. 4, first branch) and the workers pull the result.  This library
+ * simulates the W workers and the server on ONE GPU: worker replicas, the
+ * global model and all activations live in HBM, the workers' compute runs as
+ * grouped kernels, and push / pull are stream-ordered buffer reads.
+ *
+ * Conventions for every entry point:
+ *  - Status: every call returns an oscars_status; nothing throws or aborts
+ *    across this boundary.  On failure the context (if any) keeps a message
+ *    for oscars_last_error().
+ *  - Pointers: "device" pointers are CUDA global-memory addresses of the
+ *    current device; "host" pointers are ordinary process memory.  Where a
+ *    parameter says "host or device" the library copies with
+ *    cudaMemcpyDefault (unified addressing).
+ *  - Ownership: the library never frees caller memory.  Caller buffers passed
+ *    to oscars_create are BORROWED for the context's lifetime and must stay
+ *    valid and unchanged in size until oscars_destroy.  The library owns the
+ *    global model, the worker replicas and all work buffers.
+ *  - Streams: work is ordered on the cuda_stream given at creation (NULL =
+ *    the legacy default stream).  Calls that return values in host memory
+ *    (tau_out, loss_out, schedule queries, pull to host) synchronise that
+ *    stream first.  A context is not thread-safe.
+ *  - Flat parameter vector ("canonical layout"): for layers l = 0..L-1 with
+ *    fan-in d_l = dims[l] and fan-out d_{l+1} = dims[l+1], the weight W_l is
+ *    stored row-major [d_{l+1}][d_l] followed by the bias b_l [d_{l+1}];
+ *    layers follow each other without padding.  P = sum_l d_{l+1}(d_l + 1).
+ */
+#ifndef OSCARS_H
+#define OSCARS_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct oscars_ctx oscars_ctx; /* opaque, library-owned */
+
+typedef enum {
+  OSCARS_OK = 0,
+  OSCARS_EINVAL = 1,   /* bad argument or configuration                         */
+  OSCARS_ENOMEM = 2,   /* host or device allocation failed                      */
+  OSCARS_ECUDA = 3,    /* a CUDA call failed; see oscars_last_error              */
+  OSCARS_ESTATE = 4,   /* call out of protocol order                            */
+  OSCARS_ETIMEOUT = 5, /* a kernel's bounded wait ran out and it returned early */
+  OSCARS_ENOTSUP = 6   /* valid request this build does not implement           */
+} oscars_status;
+
+typedef enum {
+  OSCARS_MODEL_FLAT = 0, /* merge only: dims[0] = P parameters, no local steps */
+  OSCARS_MODEL_MLP = 1   /* ReLU MLP / softmax regression with softmax CE      */
+} oscars_model;
+
+typedef enum {
+  OSCARS_W_UNIFORM = 0,    /* w_k = 1/N: the average of Eq. 4 (first branch)        */
+  OSCARS_W_LOCALSTEPS = 1, /* w_k = tau_k / sum_j tau_j: NOT in the paper            */
+  OSCARS_W_EXPLICIT = 2    /* w_k given to every oscars_push_merge call              */
+} oscars_weight_rule;
+
+typedef enum {
+  OSCARS_SEARCH_CAPPED = 0, /* Algorithm 1, also stopping once T > M * max(t)  */
+  OSCARS_SEARCH_LITERAL = 1 /* Algorithm 1 as printed; needs min(t) < max(t)   */
+} oscars_search_mode;
+
+typedef struct {
+  int32_t num_workers;  /* N = W >= 1 (notation table); <= 256, MLP <= 64       */
+  int32_t model;        /* oscars_model                                          */
+  int32_t num_layers;   /* L >= 1 (MLP); 1 for FLAT                              */
+  const int32_t* dims;  /* host, L+1 entries: input, hidden..., classes.  FLAT:  */
+                        /* dims[0] = P.  MLP: classes <= 32                      */
+  int32_t batch;        /* B, mini-batch rows per local step (MLP)               */
+  float lr;             /* eta of Eq. 4                                          */
+  float server_lr;      /* eta_s of the delta-form merge; 1.0 = Eq. 4's average  */
+  int32_t weight_rule;  /* oscars_weight_rule                                    */
+  int32_t bf16_gemm;    /* 1: GEMM operands rounded to bf16, fp32 accumulate;    */
+                        /* 0: fp32 operands (only L = 1 supported)               */
+  const double* speed;  /* host, W speed factors s_i > 0 (larger = faster), or   */
+                        /* NULL when t_ticks is given                            */
+  const int64_t* t_ticks;  /* host, W iteration times t_i^iter in ticks >= 1;   */
+                           /* overrides speed when non-NULL                      */
+  int64_t ticks_per_unit;  /* Q: t_i = max(1, floor(Q / s_i + 0.5)); 0 = 1000   */
+  int64_t M;               /* local-step spread bound of Eq. 3, >= 1            */
+  int32_t search_mode;     /* oscars_search_mode                                */
+  const float* const* shard_x;   /* host array of W device pointers, worker i's  */
+                                 /* samples [shard_n[i]][dims[0]] fp32 row-major  */
+  const int32_t* const* shard_y; /* host array of W device pointers, labels      */
+                                 /* [shard_n[i]] in [0, classes)                  */
+  const int64_t* shard_n;        /* host, W shard sizes >= 1                      */
+  const float* init_params;      /* host or device, P fp32 canonical layout,     */
+                                 /* copied at creation; NULL = zeros (FLAT only)  */
+  void* cuda_stream;             /* cudaStream_t, borrowed; NULL = default stream */
+  int32_t flags;                 /* bit 0: launch each kernel of a round directly */
+                                 /* instead of replaying a captured CUDA graph;   */
+                                 /* bit 1 (with bit 0): time every launch with    */
+                                 /* CUDA events (see oscars_profile_read)         */
+} oscars_config;
+
+/*
+ * oscars_create - validate cfg, compute the schedule, allocate the model.
+ *
+ * Schedule (host): t_i^iter from speed (or t_ticks), then Algorithm 1 for the
+ * barrier T* (Eq. 3 with its constraint; the search evaluates T = max(t)
+ * first, keeps the first T with the smallest max_i mod(T, t_i) of Eq. 2) and
+ * tau_i = floor(T* / t_i^iter) (the sentence after Eq. 3).
+ * Memory: the global model and W replicas (fp32 master plus bf16 operand
+ * copies in MLP/bf16 mode) and all per-step activations.  The shard pointers
+ * are borrowed.  *out is set only on success.
+ * Errors: EINVAL (bad sizes, NULL pointers, W out of range, t_i < 1, M < 1,
+ * literal search with all t_i equal), ENOTSUP (a model shape outside what the
+ * kernels handle), ENOMEM, ECUDA.
+ */
+oscars_status oscars_create(const oscars_config* cfg, oscars_ctx** out);
+
+/* oscars_destroy - free everything the context owns.  NULL-safe.  Synchronises
+ * the context's stream first. */
+oscars_status oscars_destroy(oscars_ctx* ctx);
+
+/*
+ * oscars_local_steps - one round of worker compute (Eq. 4, "otherwise" branch).
+ *
+ * Every worker i starts from the current global model (the pull of the
+ * parameter-server description, fused into its first step: nothing is copied)
+ * and runs tau_i SGD steps x <- x - lr * g(x), each on the next B samples of
+ * its own shard (a cursor per worker that persists across rounds and wraps
+ * modulo shard_n[i]).  The results stay in the worker replicas, which are the
+ * pushed models.  The simulated clocks advance by tau_i * t_i of compute and
+ * mod(T*, t_i) of idle time (Eq. 1); synchronisation costs nothing.
+ * tau_out: host, W int32 or NULL.  loss_out: host, W floats or NULL: worker
+ * i's mean mini-batch loss over its tau_i steps.  Either being non-NULL
+ * synchronises the stream.
+ * Errors: ESTATE in FLAT mode or when the previous round was not merged yet;
+ * ETIMEOUT if a kernel's bounded wait ran out; ECUDA.
+ */
+oscars_status oscars_local_steps(oscars_ctx* ctx, int32_t* tau_out, float* loss_out);
+
+/*
+ * oscars_push_merge - server merge and global update (Eq. 4, first branch).
+ *
+ * x_g <- x_g + server_lr * sum_k w_k * delta_k, accumulated in fp32 registers
+ * in worker order.  With deltas == NULL, delta_k = x^k - x_g from the worker
+ * replicas of the last oscars_local_steps (MLP mode only); otherwise deltas
+ * is a host array of W device pointers, each to P fp32 values in canonical
+ * layout (any alignment).  w_k follows the weight rule; for OSCARS_W_EXPLICIT
+ * `weights` is a host array of W floats (ignored otherwise, may be NULL).
+ * Errors: ESTATE (deltas == NULL without pending local steps, or in FLAT
+ * mode), EINVAL (NULL delta pointer, NULL weights for the explicit rule),
+ * ECUDA.
+ */
+oscars_status oscars_push_merge(oscars_ctx* ctx, const float* const* deltas, const float* weights);
+
+/*
+ * oscars_pull - serve the global model.
+ * dst != NULL: copy x_g (P fp32, canonical layout) into dst (host or device;
+ * a host dst synchronises).  dst == NULL: write x_g into every worker replica
+ * (an explicit pull; oscars_local_steps does not need it).
+ */
+oscars_status oscars_pull(oscars_ctx* ctx, float* dst);
+
+/*
+ * oscars_get_schedule - the schedule and simulated clocks.  Every output is a
+ * host pointer and may be NULL.  T_star, max_wait: scalars (Eq. 3, Eq. 2 at
+ * T*).  t_iter[W] ticks; tau[W]; wait[W] = mod(T*, t_i) (Eq. 1); clock[W] and
+ * idle[W]: total simulated ticks and idle ticks so far.
+ */
+oscars_status oscars_get_schedule(const oscars_ctx* ctx, int64_t* T_star, int64_t* max_wait,
+                                  int64_t* t_iter, int32_t* tau, int64_t* wait,
+                                  int64_t* clock, int64_t* idle);
+
+/*
+ * oscars_set_local_steps - replace tau (host, W int32 >= 1), e.g. tau = 1 for
+ * BSP or a fixed I for plain local SGD (the comparison schemes of the
+ * paper's Motivation).  The barrier used by the simulated clock becomes
+ * max_i tau_i * t_i.  Errors: EINVAL, ESTATE while a round is pending.
+ */
+oscars_status oscars_set_local_steps(oscars_ctx* ctx, const int32_t* tau);
+
+/*
+ * oscars_eval_loss - mean softmax cross-entropy of the global model on n
+ * samples x [n][dims[0]] fp32 and labels y [n] (both device pointers), with
+ * the same operand precision as training.  MLP mode; n >= 1; *loss is host.
+ */
+oscars_status oscars_eval_loss(oscars_ctx* ctx, const float* x, const int32_t* y, int64_t n,
+                               float* loss);
+
+/*
+ * oscars_read_replica - copy worker k's current model (the model it pushes at
+ * the barrier; Section "Introduction": each worker holds a model copy) in
+ * canonical layout into dst (host or device, P fp32).  MLP mode, 0 <= k < W.
+ */
+oscars_status oscars_read_replica(oscars_ctx* ctx, int32_t k, float* dst);
+
+/*
+ * oscars_profile_read - per-kernel-class device time of the launches made
+ * since the last reset while flag bits 0 and 1 were set (CUDA events recorded
+ * on the context's stream around every launch).  Synchronises on the last
+ * recorded event.  Fills up to `cap` entries: names[i] (library-owned, valid
+ * until the next reset or destroy), ms_total[i], launches[i] (each may be
+ * NULL).  Returns the number of classes, or -1 for a NULL ctx.
+ * oscars_profile_reset clears the totals.
+ */
+int32_t oscars_profile_read(oscars_ctx* ctx, int32_t cap, const char** names, double* ms_total,
+                            int32_t* launches);
+oscars_status oscars_profile_reset(oscars_ctx* ctx);
+
+/* oscars_num_params - P of the context (canonical layout). */
+oscars_status oscars_num_params(const oscars_ctx* ctx, int64_t* P);
+
+/* Message of the last failure on ctx ("" if none).  Valid until the next call. */
+const char* oscars_last_error(const oscars_ctx* ctx);
+
+/* Name of a status code. */
+const char* oscars_status_string(int32_t status);
+
+/*
+ * Host-only helpers (no GPU needed): the scheduler of oscars_create.
+ *
+ * oscars_iteration_ticks: t[i] = max(1, floor(Q / speed[i] + 0.5)) in fp64,
+ * then int64 (Q = ticks_per_unit, 0 = 1000); speed[i] > 0.
+ * oscars_schedule_solve: Algorithm 1 on t_iter[n] with bound M and the given
+ * search mode; outputs T*, the max wait at T* (Eq. 2) and tau[n]
+ * (all host, tau may be NULL).  Errors: EINVAL.
+ * oscars_merge_weights: the fp32 weights of a rule for local-step counts
+ * tau[n] (uniform or local-steps), computed in fp64 and rounded once.
+ */
+oscars_status oscars_iteration_ticks(const double* speed, int32_t n, int64_t ticks_per_unit,
+                                     int64_t* t_iter);
+oscars_status oscars_schedule_solve(const int64_t* t_iter, int32_t n, int64_t M,
+                                    int32_t search_mode, int64_t* T_star, int64_t* max_wait,
+                                    int32_t* tau);
+oscars_status oscars_merge_weights(int32_t rule, const int32_t* tau, int32_t n, float* w);
+
+/*
+ * oscars_merge - the server update of Eq. 4 (first branch) on caller buffers,
+ * without a context: x_g[p] <- x_g[p] + server_lr * sum_k w[k] * deltas[k][p]
+ * for p < P.  x_g: device, P fp32, updated in place.  deltas: host array of W
+ * device pointers to P fp32 each.  w: host, W floats.  Any alignment;
+ * 16-byte aligned pointers take the vector path.  Ordered on `stream`
+ * (cudaStream_t or NULL).  W <= 256.  Errors: EINVAL, ECUDA.
+ */
+oscars_status oscars_merge(float* x_g, const float* const* deltas, const float* w, int32_t W,
+                           int64_t P, float server_lr, void* stream);
+
+/*
+ * oscars_gemm_bf16_nt - C[M][N] = sum_k A[m][k] * B[n][k] on the tcgen05
+ * tensor cores, the contraction of the workers' dense layers (Eq. 4,
+ * "otherwise" branch: forward and backward products) without a fused
+ * epilogue.  A: device, [M][K] bf16 row-major; B: device, [N][K] bf16
+ * row-major; both 16-byte aligned.  C: device, [M][N] fp32 row-major,
+ * overwritten.  M a multiple of 128, K a multiple of 8, N >= 1.  fp32
+ * accumulation.  Ordered on `stream`.  Errors: EINVAL, ECUDA.
+ */
+oscars_status oscars_gemm_bf16_nt(const void* A, const void* B, float* C, int32_t M, int32_t N, int32_t K,
+                                  void* stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* OSCARS_H */

@@ -1,0 +1,1042 @@
+// C ABI of the Oscars hot path: context, schedule, round orchestration.
+//
+// One context simulates the parameter server and its W workers on one GPU
+// (Introduction: parameter-server architecture; Problem Formulation and
+// Algorithm 1: the load-balanced barrier; Eq. 4: local steps and merge).
+//
+// Device memory of a context (MLP mode):
+//   slab    (W+1) slots x P_pad fp32   slots 0..W-1 worker replicas (the
+//                                      pushed models), slot W the global model
+//   shadow  (W+1) x P_pad bf16         bf16 copy of every slot (GEMM operand)
+//   shadowT (W+1) x PT_pad bf16        transposed bf16 copy of the middle
+//                                      layers (K-major operand of dX GEMMs)
+//   per-worker activations, gradients, labels, loss partials, cursors.
+// Inside a slot every W_l and b_l starts on a 64-element boundary; the
+// padding stays zero.
+#include <algorithm>
+#include <cstdio>
+#include <cstring>
+#include <new>
+#include <string>
+#include <vector>
+
+#include "../../include/oscars.h"
+#include "common.cuh"
+#include "internal.h"
+
+using namespace oscars;
+
+namespace {
+
+int64_t round_up(int64_t x, int64_t m) { return (x + m - 1) / m * m; }
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                  const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                  CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+  static EncodeTiledFn fn = nullptr;
+  if (!fn) {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<EncodeTiledFn>(p);
+  }
+  return fn;
+}
+
+// 3-D bf16 tensor map: element (x, y, z) at base + z*stride_z + y*stride_y +
+// 2x bytes; boxes of 64 (x) by box_y rows, 128-byte swizzle, zero fill
+// outside the extents.
+bool make_map(CUtensorMap* m, const void* base, uint64_t dx, uint64_t dy, uint64_t dz, uint64_t stride_y,
+              uint64_t stride_z, uint32_t box_y) {
+  EncodeTiledFn f = encode_fn();
+  if (!f) return false;
+  cuuint64_t dims[3] = {dx, dy, dz};
+  cuuint64_t strides[2] = {stride_y, stride_z};
+  cuuint32_t box[3] = {64, box_y, 1};
+  cuuint32_t es[3] = {1, 1, 1};
+  return f(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(base), dims, strides, box, es,
+           CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+           CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+struct Layer {
+  int in, out;
+  int64_t offW, offB, offT;  // offT < 0: no transposed copy
+};
+
+}  // namespace
+
+struct oscars_ctx {
+  // configuration
+  int W = 0, model = 0, L = 0, B = 0, C = 0;
+  std::vector<int> dims;
+  float lr = 0.f, server_lr = 1.f;
+  int rule = 0, bf16 = 0, flags = 0;
+  int64_t P = 0, P_pad = 0, PT_pad = 0;
+  std::vector<Layer> layers;
+  // schedule (Eq. 1-3, Algorithm 1)
+  std::vector<int64_t> t_iter, clock, idle;
+  std::vector<int32_t> tau;
+  int64_t T_star = 0, max_wait = 0, M = 0, barrier = 0;
+  int search_mode = 0, max_tau = 0;
+  std::vector<int> n_active;  // per local step
+  // data (borrowed)
+  std::vector<const float*> shard_x;
+  std::vector<const int32_t*> shard_y;
+  std::vector<int64_t> shard_n;
+  // device memory
+  std::vector<void*> allocs;
+  float* slab = nullptr;
+  __nv_bfloat16* shadow = nullptr;
+  __nv_bfloat16* shadowT = nullptr;
+  std::vector<__nv_bfloat16*> A, AT, G, GT;  // per layer
+  std::vector<float*> gb;
+  int32_t* labels = nullptr;
+  float* dlog = nullptr;
+  float* loss_part = nullptr;
+  float* loss_dev = nullptr;
+  int64_t* cursor = nullptr;
+  int32_t* tau_dev = nullptr;
+  int* act_wid = nullptr;  // [max_tau][W]
+  int* act_src = nullptr;
+  int* lane_ids = nullptr;   // [W] 0..W-1
+  int* global_src = nullptr; // [W] all = W
+  const float** dx_tab = nullptr;
+  const int32_t** dy_tab = nullptr;
+  int64_t* dn_tab = nullptr;
+  int* err = nullptr;
+  // eval scratch
+  const float** ex_tab = nullptr;
+  const int32_t** ey_tab = nullptr;
+  int64_t* en_tab = nullptr;
+  int64_t* estart = nullptr;
+  int64_t estart_cap = 0;
+  float* eval_part = nullptr;
+  int64_t eval_part_cap = 0;
+  // tensor maps per layer
+  std::vector<CUtensorMap> mShadow, mShadowT, mA, mG, mGT, mAT;
+  // streams / graph
+  cudaStream_t stream = nullptr;
+  cudaStream_t cap = nullptr;
+  cudaGraphExec_t round_exec = nullptr;
+  bool pending = false;
+  std::string last_error;
+  // per-kernel-class CUDA-event profile (flag bit 1, direct launches only)
+  struct ProfEntry {
+    const char* name;
+    cudaEvent_t a, b;
+  };
+  std::vector<ProfEntry> prof_pending;
+  std::vector<cudaEvent_t> prof_pool;
+  std::vector<std::string> prof_names;
+  std::vector<double> prof_ms;
+  std::vector<int> prof_count;
+  bool profiling = false;
+};
+
+namespace {
+
+oscars_status fail(oscars_ctx* c, oscars_status s, const std::string& msg) {
+  if (c) c->last_error = msg;
+  return s;
+}
+
+oscars_status cuda_fail(oscars_ctx* c, cudaError_t e, const char* where) {
+  return fail(c, OSCARS_ECUDA, std::string(where) + ": " + cudaGetErrorString(e));
+}
+
+// ---- profiler: events around each launch on the launching stream
+cudaEvent_t prof_event(oscars_ctx* c) {
+  if (!c->prof_pool.empty()) {
+    cudaEvent_t e = c->prof_pool.back();
+    c->prof_pool.pop_back();
+    return e;
+  }
+  cudaEvent_t e = nullptr;
+  cudaEventCreate(&e);
+  return e;
+}
+
+struct ProfScope {
+  oscars_ctx* c;
+  const char* name;
+  cudaStream_t s;
+  cudaEvent_t a = nullptr;
+  ProfScope(oscars_ctx* c_, const char* n, cudaStream_t s_) : c(c_), name(n), s(s_) {
+    if (c->profiling) {
+      a = prof_event(c);
+      cudaEventRecord(a, s);
+    }
+  }
+  ~ProfScope() {
+    if (a) {
+      cudaEvent_t b = prof_event(c);
+      cudaEventRecord(b, s);
+      c->prof_pending.push_back({name, a, b});
+    }
+  }
+};
+
+// fold finished event pairs into per-name totals (synchronises)
+void prof_collect(oscars_ctx* c) {
+  if (c->prof_pending.empty()) return;
+  cudaEventSynchronize(c->prof_pending.back().b);
+  for (auto& p : c->prof_pending) {
+    float ms = 0.f;
+    cudaEventElapsedTime(&ms, p.a, p.b);
+    size_t i = 0;
+    while (i < c->prof_names.size() && c->prof_names[i] != p.name) ++i;
+    if (i == c->prof_names.size()) {
+      c->prof_names.push_back(p.name);
+      c->prof_ms.push_back(0.0);
+      c->prof_count.push_back(0);
+    }
+    c->prof_ms[i] += ms;
+    c->prof_count[i] += 1;
+    c->prof_pool.push_back(p.a);
+    c->prof_pool.push_back(p.b);
+  }
+  c->prof_pending.clear();
+}
+
+template <typename T>
+bool dev_alloc(oscars_ctx* c, T** p, size_t count) {
+  void* q = nullptr;
+  if (count == 0) count = 1;
+  if (cudaMalloc(&q, count * sizeof(T)) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  c->allocs.push_back(q);
+  *p = static_cast<T*>(q);
+  return true;
+}
+
+void free_all(oscars_ctx* c) {
+  for (auto& p : c->prof_pending) {
+    cudaEventDestroy(p.a);
+    cudaEventDestroy(p.b);
+  }
+  c->prof_pending.clear();
+  for (cudaEvent_t e : c->prof_pool) cudaEventDestroy(e);
+  c->prof_pool.clear();
+  if (c->round_exec) cudaGraphExecDestroy(c->round_exec);
+  c->round_exec = nullptr;
+  for (void* p : c->allocs) cudaFree(p);
+  c->allocs.clear();
+  if (c->cap) cudaStreamDestroy(c->cap);
+  c->cap = nullptr;
+}
+
+// Simulated barrier and idle time per worker for the current tau (Eq. 1).
+void update_barrier(oscars_ctx* c, bool from_search) {
+  if (from_search) {
+    c->barrier = c->T_star;
+  } else {
+    int64_t b = 0;
+    for (int i = 0; i < c->W; ++i) b = std::max(b, static_cast<int64_t>(c->tau[i]) * c->t_iter[i]);
+    c->barrier = b;
+  }
+}
+
+oscars_status build_tables(oscars_ctx* c) {
+  c->max_tau = 0;
+  for (int i = 0; i < c->W; ++i) c->max_tau = std::max(c->max_tau, static_cast<int>(c->tau[i]));
+  c->n_active.assign(c->max_tau, 0);
+  std::vector<int> wid(static_cast<size_t>(c->max_tau) * c->W, 0), src(wid.size(), 0);
+  for (int s = 0; s < c->max_tau; ++s) {
+    int n = 0;
+    for (int i = 0; i < c->W; ++i)
+      if (c->tau[i] > s) {
+        wid[static_cast<size_t>(s) * c->W + n] = i;
+        src[static_cast<size_t>(s) * c->W + n] = s == 0 ? c->W : i;  // first step reads the global model
+        ++n;
+      }
+    c->n_active[s] = n;
+  }
+  if (c->act_wid) {
+    // tables are reallocated when tau changes
+  }
+  if (!dev_alloc(c, &c->act_wid, wid.size()) || !dev_alloc(c, &c->act_src, src.size()) ||
+      !dev_alloc(c, &c->loss_part, static_cast<size_t>(c->W) * c->max_tau * std::max(1, c->B / kRowsPerLossChunk)))
+    return fail(c, OSCARS_ENOMEM, "device allocation failed (schedule tables)");
+  cudaError_t e = cudaMemcpy(c->act_wid, wid.data(), wid.size() * sizeof(int), cudaMemcpyHostToDevice);
+  if (e == cudaSuccess) e = cudaMemcpy(c->act_src, src.data(), src.size() * sizeof(int), cudaMemcpyHostToDevice);
+  if (e == cudaSuccess) e = cudaMemcpy(c->tau_dev, c->tau.data(), c->W * sizeof(int32_t), cudaMemcpyHostToDevice);
+  if (e != cudaSuccess) return cuda_fail(c, e, "schedule upload");
+  if (c->round_exec) {
+    cudaGraphExecDestroy(c->round_exec);
+    c->round_exec = nullptr;
+  }
+  return OSCARS_OK;
+}
+
+cudaError_t refresh_global_shadows(oscars_ctx* c, cudaStream_t s) {
+  if (!c->shadow) return cudaSuccess;
+  const int64_t g = static_cast<int64_t>(c->W) * c->P_pad;
+  cudaError_t e = launch_shadow_refresh(c->slab + g, c->shadow + g, c->P_pad, s);
+  if (e != cudaSuccess) return e;
+  for (const Layer& ly : c->layers) {
+    if (ly.offT < 0) continue;
+    e = launch_transpose_bf16(c->shadow + g + ly.offW,
+                              c->shadowT + static_cast<int64_t>(c->W) * c->PT_pad + ly.offT, ly.out, ly.in, s);
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
+}
+
+GemmArgs gemm_base(oscars_ctx* c, int s) {
+  GemmArgs g;
+  std::memset(&g, 0, sizeof(g));
+  g.wid = c->act_wid + static_cast<size_t>(s) * c->W;
+  g.src = c->act_src + static_cast<size_t>(s) * c->W;
+  g.err = c->err;
+  g.master = c->slab;
+  g.master_w = c->slab;
+  g.shadow = c->shadow;
+  g.slot_stride = c->P_pad;
+  g.slotT_stride = c->PT_pad;
+  g.lr = c->lr;
+  return g;
+}
+
+HeadArgs head_base(oscars_ctx* c) {
+  HeadArgs h;
+  std::memset(&h, 0, sizeof(h));
+  const Layer& ly = c->layers.back();
+  h.H = ly.in;
+  h.C = ly.out;
+  h.B = c->B;
+  h.Ain = c->A[c->L - 1];
+  h.labels = c->labels;
+  h.shadow = c->shadow;
+  h.master = c->slab;
+  h.master_w = c->slab;
+  h.shadow_w = c->shadow;
+  h.slot_stride = c->P_pad;
+  h.offW = ly.offW;
+  h.offB = ly.offB;
+  h.lr = c->lr;
+  h.dlog = c->dlog;
+  if (c->L >= 2) {
+    h.G = c->G[c->L - 2];
+    h.GT = c->GT[c->L - 2];
+    h.gb = c->gb[c->L - 2];
+  }
+  return h;
+}
+
+// forward layers 0..L-2 for `na` lanes (training step or evaluation)
+cudaError_t enqueue_forward(oscars_ctx* c, const int* wid, const int* src, int na, cudaStream_t st) {
+  for (int l = 0; l + 1 < c->L; ++l) {
+    const Layer& ly = c->layers[l];
+    GemmArgs g = gemm_base(c, 0);
+    g.wid = wid;
+    g.src = src;
+    g.M = ly.out;
+    g.N = c->B;
+    g.K = ly.in;
+    g.a_z_src = 1;
+    g.b_z_src = 0;
+    g.offW = ly.offW;
+    g.offB = ly.offB;
+    g.out = c->A[l + 1];
+    g.outT = c->AT[l + 1];
+    ProfScope ps(c, "gemm_fwd", st);
+    cudaError_t e = launch_gemm(kEpiFwd, c->mShadow[l], c->mA[l], g, na, st);
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
+}
+
+cudaError_t enqueue_round_mlp(oscars_ctx* c, cudaStream_t st) {
+  cudaError_t e;
+  for (int s = 0; s < c->max_tau; ++s) {
+    const int na = c->n_active[s];
+    const int* wid = c->act_wid + static_cast<size_t>(s) * c->W;
+    const int* src = c->act_src + static_cast<size_t>(s) * c->W;
+    StageArgs sa;
+    sa.x = c->dx_tab;
+    sa.y = c->dy_tab;
+    sa.n = c->dn_tab;
+    sa.start = c->cursor;
+    sa.row_add = static_cast<int64_t>(s) * c->B;
+    sa.wid = wid;
+    sa.D = c->dims[0];
+    sa.B = c->B;
+    sa.A0 = c->A[0];
+    sa.A0T = c->AT[0];
+    sa.labels = c->labels;
+    {
+      ProfScope ps(c, "stage", st);
+      if ((e = launch_stage(sa, na, st)) != cudaSuccess) return e;
+    }
+    if ((e = enqueue_forward(c, wid, src, na, st)) != cudaSuccess) return e;
+    HeadArgs h = head_base(c);
+    h.wid = wid;
+    h.src = src;
+    h.loss_part = c->loss_part;
+    h.part_mul = c->max_tau;
+    h.part_add = s;
+    {
+      ProfScope ps(c, "head_fwd", st);
+      if ((e = launch_head_fwd(h, na, st)) != cudaSuccess) return e;
+    }
+    {
+      ProfScope ps(c, "head_bwd", st);
+      if ((e = launch_head_bwd(h, na, st)) != cudaSuccess) return e;
+    }
+    for (int l = c->L - 2; l >= 0; --l) {
+      const Layer& ly = c->layers[l];
+      if (l >= 1) {  // input gradient of layer l -> gradient of layer l-1's output
+        GemmArgs g = gemm_base(c, s);
+        g.M = ly.in;
+        g.N = c->B;
+        g.K = ly.out;
+        g.a_z_src = 1;
+        g.b_z_src = 0;
+        g.hmask = c->A[l];
+        g.out = c->G[l - 1];
+        g.outT = c->GT[l - 1];
+        g.gb_out = c->gb[l - 1];
+        ProfScope ps(c, "gemm_dh", st);
+        if ((e = launch_gemm(kEpiDh, c->mShadowT[l], c->mG[l], g, na, st)) != cudaSuccess) return e;
+      }
+      GemmArgs g = gemm_base(c, s);
+      g.M = ly.out;
+      g.N = ly.in;
+      g.K = c->B;
+      g.a_z_src = 0;
+      g.b_z_src = 0;
+      g.offW = ly.offW;
+      g.offB = ly.offB;
+      g.offT = ly.offT;
+      g.shadowT = ly.offT >= 0 ? c->shadowT : nullptr;
+      g.gb_in = c->gb[l];
+      ProfScope ps(c, "gemm_dw_sgd", st);
+      if ((e = launch_gemm(kEpiDw, c->mGT[l], c->mAT[l], g, na, st)) != cudaSuccess) return e;
+    }
+  }
+  const int nc = c->B / kRowsPerLossChunk;
+  ProfScope ps(c, "round_bookkeeping", st);
+  if ((e = launch_loss_finalize(c->loss_part, c->tau_dev, c->W, c->max_tau, nc, c->B, c->loss_dev, st)) != cudaSuccess)
+    return e;
+  return launch_cursor_advance(c->cursor, c->tau_dev, c->dn_tab, c->B, c->W, st);
+}
+
+cudaError_t enqueue_round_softreg(oscars_ctx* c, cudaStream_t st) {
+  SoftregArgs a;
+  a.master = c->slab;
+  a.master_out = c->slab;
+  a.slot_stride = c->P_pad;
+  a.global_slot = c->W;
+  a.offW = c->layers[0].offW;
+  a.offB = c->layers[0].offB;
+  a.D = c->dims[0];
+  a.C = c->dims[1];
+  a.B = c->B;
+  a.lr = c->lr;
+  a.tau = c->tau_dev;
+  a.shard_x = c->dx_tab;
+  a.shard_y = c->dy_tab;
+  a.shard_n = c->dn_tab;
+  a.cursor = c->cursor;
+  a.loss_part = c->loss_part;
+  a.max_tau = c->max_tau;
+  cudaError_t e;
+  {
+    ProfScope ps(c, "softreg_round", st);
+    e = launch_softreg_round(a, c->W, st);
+  }
+  if (e != cudaSuccess) return e;
+  ProfScope ps(c, "round_bookkeeping", st);
+  if ((e = launch_loss_finalize(c->loss_part, c->tau_dev, c->W, c->max_tau, 1, c->B, c->loss_dev, st)) != cudaSuccess)
+    return e;
+  return launch_cursor_advance(c->cursor, c->tau_dev, c->dn_tab, c->B, c->W, st);
+}
+
+cudaError_t enqueue_round(oscars_ctx* c, cudaStream_t st) {
+  return c->L == 1 && !c->bf16 ? enqueue_round_softreg(c, st) : enqueue_round_mlp(c, st);
+}
+
+oscars_status check_err_word(oscars_ctx* c) {
+  if (!c->err) return OSCARS_OK;
+  int h = 0;
+  cudaError_t e = cudaMemcpy(&h, c->err, sizeof(int), cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return cuda_fail(c, e, "reading the kernel error word");
+  if (h != 0) {
+    cudaMemset(c->err, 0, sizeof(int));
+    return fail(c, OSCARS_ETIMEOUT, "a kernel's bounded wait ran out (code " + std::to_string(h) + ")");
+  }
+  return OSCARS_OK;
+}
+
+oscars_status validate_and_layout(oscars_ctx* c, const oscars_config* cfg) {
+  c->W = cfg->num_workers;
+  c->model = cfg->model;
+  if (c->W < 1 || c->W > kMaxMergeWorkers) return fail(c, OSCARS_EINVAL, "num_workers must be in [1, 256]");
+  if (!cfg->dims) return fail(c, OSCARS_EINVAL, "dims is NULL");
+  c->lr = cfg->lr;
+  c->server_lr = cfg->server_lr;
+  c->rule = cfg->weight_rule;
+  c->bf16 = cfg->bf16_gemm;
+  if (c->rule < OSCARS_W_UNIFORM || c->rule > OSCARS_W_EXPLICIT) return fail(c, OSCARS_EINVAL, "bad weight rule");
+  if (!(c->server_lr == c->server_lr)) return fail(c, OSCARS_EINVAL, "server_lr is NaN");
+  if (c->model == OSCARS_MODEL_FLAT) {
+    if (cfg->dims[0] < 1) return fail(c, OSCARS_EINVAL, "FLAT: dims[0] = P must be >= 1");
+    c->L = 0;
+    c->P = cfg->dims[0];
+    c->P_pad = round_up(c->P, 64);
+    return OSCARS_OK;
+  }
+  if (c->model != OSCARS_MODEL_MLP) return fail(c, OSCARS_EINVAL, "unknown model");
+  c->L = cfg->num_layers;
+  if (c->L < 1 || c->L > 16) return fail(c, OSCARS_EINVAL, "num_layers must be in [1, 16]");
+  c->dims.assign(cfg->dims, cfg->dims + c->L + 1);
+  for (int d : c->dims)
+    if (d < 1) return fail(c, OSCARS_EINVAL, "dims must be >= 1");
+  c->B = cfg->batch;
+  c->C = c->dims[c->L];
+  if (c->B < 1) return fail(c, OSCARS_EINVAL, "batch must be >= 1");
+  if (c->C < 2 || c->C > kMaxClasses) return fail(c, OSCARS_ENOTSUP, "classes must be in [2, 32]");
+  if (!(c->lr == c->lr)) return fail(c, OSCARS_EINVAL, "lr is NaN");
+  if (c->L == 1 && !c->bf16) {
+    if (softreg_smem_bytes(c->dims[0], c->C, c->B) > 220 * 1024)
+      return fail(c, OSCARS_ENOTSUP, "softmax regression: weights plus one batch must fit in shared memory");
+  } else if (c->bf16 && c->L >= 2) {
+    if (c->W > kMaxWorkersMLP) return fail(c, OSCARS_ENOTSUP, "MLP mode supports at most 64 workers");
+    if (c->B % 32 != 0 || c->B > 256) return fail(c, OSCARS_ENOTSUP, "bf16 MLP: batch must be a multiple of 32, <= 256");
+    if (c->dims[0] % 8 != 0) return fail(c, OSCARS_ENOTSUP, "bf16 MLP: input dim must be a multiple of 8");
+    for (int l = 1; l < c->L; ++l)
+      if (c->dims[l] % 128 != 0) return fail(c, OSCARS_ENOTSUP, "bf16 MLP: hidden dims must be multiples of 128");
+  } else {
+    return fail(c, OSCARS_ENOTSUP, "supported: fp32 softmax regression (L=1) or bf16 MLP (L>=2)");
+  }
+  int64_t off = 0, offT = 0;
+  c->P = 0;
+  for (int l = 0; l < c->L; ++l) {
+    Layer ly;
+    ly.in = c->dims[l];
+    ly.out = c->dims[l + 1];
+    ly.offW = off;
+    off += round_up(static_cast<int64_t>(ly.in) * ly.out, 64);
+    ly.offB = off;
+    off += round_up(ly.out, 64);
+    ly.offT = -1;
+    if (c->bf16 && l >= 1 && l <= c->L - 2) {
+      ly.offT = offT;
+      offT += round_up(static_cast<int64_t>(ly.in) * ly.out, 64);
+    }
+    c->P += static_cast<int64_t>(ly.in) * ly.out + ly.out;
+    c->layers.push_back(ly);
+  }
+  c->P_pad = round_up(off, 64);
+  c->PT_pad = round_up(offT, 64);
+  return OSCARS_OK;
+}
+
+oscars_status allocate_mlp(oscars_ctx* c) {
+  const int W = c->W, B = c->B, L = c->L;
+  const size_t slots = static_cast<size_t>(W) + 1;
+  if (!dev_alloc(c, &c->slab, slots * c->P_pad)) return fail(c, OSCARS_ENOMEM, "device allocation failed (model slab)");
+  cudaMemset(c->slab, 0, slots * c->P_pad * sizeof(float));
+  if (!dev_alloc(c, &c->cursor, W) || !dev_alloc(c, &c->tau_dev, W) || !dev_alloc(c, &c->loss_dev, std::max(W, 1)) ||
+      !dev_alloc(c, &c->dx_tab, W) || !dev_alloc(c, &c->dy_tab, W) || !dev_alloc(c, &c->dn_tab, W) ||
+      !dev_alloc(c, &c->err, 1) || !dev_alloc(c, &c->lane_ids, W) || !dev_alloc(c, &c->global_src, W) ||
+      !dev_alloc(c, &c->ex_tab, W) || !dev_alloc(c, &c->ey_tab, W) || !dev_alloc(c, &c->en_tab, W))
+    return fail(c, OSCARS_ENOMEM, "device allocation failed (tables)");
+  cudaMemset(c->cursor, 0, W * sizeof(int64_t));
+  cudaMemset(c->err, 0, sizeof(int));
+  std::vector<int> ids(W), gs(W, W);
+  for (int i = 0; i < W; ++i) ids[i] = i;
+  cudaMemcpy(c->lane_ids, ids.data(), W * sizeof(int), cudaMemcpyHostToDevice);
+  cudaMemcpy(c->global_src, gs.data(), W * sizeof(int), cudaMemcpyHostToDevice);
+  cudaMemcpy(c->dx_tab, c->shard_x.data(), W * sizeof(float*), cudaMemcpyHostToDevice);
+  cudaMemcpy(c->dy_tab, c->shard_y.data(), W * sizeof(int32_t*), cudaMemcpyHostToDevice);
+  cudaError_t e = cudaMemcpy(c->dn_tab, c->shard_n.data(), W * sizeof(int64_t), cudaMemcpyHostToDevice);
+  if (e != cudaSuccess) return cuda_fail(c, e, "table upload");
+  if (L == 1 && !c->bf16) return OSCARS_OK;
+
+  if (!dev_alloc(c, &c->shadow, slots * c->P_pad)) return fail(c, OSCARS_ENOMEM, "device allocation failed (bf16 shadow)");
+  cudaMemset(c->shadow, 0, slots * c->P_pad * sizeof(__nv_bfloat16));
+  if (c->PT_pad > 0) {
+    if (!dev_alloc(c, &c->shadowT, slots * c->PT_pad)) return fail(c, OSCARS_ENOMEM, "device allocation failed (bf16 shadow^T)");
+    cudaMemset(c->shadowT, 0, slots * c->PT_pad * sizeof(__nv_bfloat16));
+  }
+  c->A.assign(L, nullptr);
+  c->AT.assign(L, nullptr);
+  c->G.assign(L, nullptr);
+  c->GT.assign(L, nullptr);
+  c->gb.assign(L, nullptr);
+  for (int l = 0; l < L; ++l) {
+    const size_t act = static_cast<size_t>(W) * B * c->dims[l];
+    if (!dev_alloc(c, &c->A[l], act) || !dev_alloc(c, &c->AT[l], act))
+      return fail(c, OSCARS_ENOMEM, "device allocation failed (activations)");
+    if (l + 1 < L) {
+      const size_t gsz = static_cast<size_t>(W) * B * c->dims[l + 1];
+      if (!dev_alloc(c, &c->G[l], gsz) || !dev_alloc(c, &c->GT[l], gsz) ||
+          !dev_alloc(c, &c->gb[l], static_cast<size_t>(W) * c->dims[l + 1]))
+        return fail(c, OSCARS_ENOMEM, "device allocation failed (gradients)");
+    }
+  }
+  if (!dev_alloc(c, &c->labels, static_cast<size_t>(W) * B) || !dev_alloc(c, &c->dlog, static_cast<size_t>(W) * B * c->C))
+    return fail(c, OSCARS_ENOMEM, "device allocation failed (head)");
+
+  // tensor maps
+  c->mShadow.resize(L);
+  c->mShadowT.resize(L);
+  c->mA.resize(L);
+  c->mG.resize(L);
+  c->mGT.resize(L);
+  c->mAT.resize(L);
+  const uint64_t slots64 = slots;
+  for (int l = 0; l + 1 < L; ++l) {
+    const Layer& ly = c->layers[l];
+    bool ok = true;
+    // W_l [out][in] of every slot: A operand of the forward GEMM
+    ok &= make_map(&c->mShadow[l], c->shadow + ly.offW, ly.in, ly.out, slots64, ly.in * 2ull, c->P_pad * 2ull, 128);
+    // layer input [lane][B][in]: B operand of the forward GEMM
+    ok &= make_map(&c->mA[l], c->A[l], ly.in, B, W, ly.in * 2ull, static_cast<uint64_t>(B) * ly.in * 2ull, B);
+    // output gradient^T [lane][out][B]: A operand of the weight-gradient GEMM
+    ok &= make_map(&c->mGT[l], c->GT[l], B, ly.out, W, B * 2ull, static_cast<uint64_t>(B) * ly.out * 2ull, 128);
+    // layer input^T [lane][in][B]: B operand of the weight-gradient GEMM
+    ok &= make_map(&c->mAT[l], c->AT[l], B, ly.in, W, B * 2ull, static_cast<uint64_t>(B) * ly.in * 2ull, 128);
+    if (l >= 1) {
+      // W_l^T [in][out] of every slot: A operand of the input-gradient GEMM
+      ok &= make_map(&c->mShadowT[l], c->shadowT + ly.offT, ly.out, ly.in, slots64, ly.out * 2ull, c->PT_pad * 2ull, 128);
+      // output gradient [lane][B][out]: B operand of the input-gradient GEMM
+      ok &= make_map(&c->mG[l], c->G[l], ly.out, B, W, ly.out * 2ull, static_cast<uint64_t>(B) * ly.out * 2ull, B);
+    }
+    if (!ok) return fail(c, OSCARS_ECUDA, "cuTensorMapEncodeTiled failed (or the driver entry point is missing)");
+  }
+  return OSCARS_OK;
+}
+
+// copy a canonical-layout vector into the padded slot layout (or back)
+cudaError_t copy_canonical(oscars_ctx* c, float* padded, const float* canon, bool to_padded, cudaStream_t s) {
+  if (c->model == OSCARS_MODEL_FLAT) {
+    return to_padded ? cudaMemcpyAsync(padded, canon, c->P * sizeof(float), cudaMemcpyDefault, s)
+                     : cudaMemcpyAsync(const_cast<float*>(canon), padded, c->P * sizeof(float), cudaMemcpyDefault, s);
+  }
+  int64_t co = 0;
+  for (const Layer& ly : c->layers) {
+    const int64_t nw = static_cast<int64_t>(ly.in) * ly.out;
+    cudaError_t e;
+    if (to_padded) {
+      e = cudaMemcpyAsync(padded + ly.offW, canon + co, nw * sizeof(float), cudaMemcpyDefault, s);
+      if (e == cudaSuccess) e = cudaMemcpyAsync(padded + ly.offB, canon + co + nw, ly.out * sizeof(float), cudaMemcpyDefault, s);
+    } else {
+      float* dst = const_cast<float*>(canon);
+      e = cudaMemcpyAsync(dst + co, padded + ly.offW, nw * sizeof(float), cudaMemcpyDefault, s);
+      if (e == cudaSuccess) e = cudaMemcpyAsync(dst + co + nw, padded + ly.offB, ly.out * sizeof(float), cudaMemcpyDefault, s);
+    }
+    if (e != cudaSuccess) return e;
+    co += nw + ly.out;
+  }
+  return cudaSuccess;
+}
+
+bool is_host_ptr(const void* p) {
+  cudaPointerAttributes at;
+  if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
+    cudaGetLastError();
+    return true;
+  }
+  return at.type == cudaMemoryTypeHost || at.type == cudaMemoryTypeUnregistered;
+}
+
+}  // namespace
+
+extern "C" {
+
+oscars_status oscars_create(const oscars_config* cfg, oscars_ctx** out) {
+  if (!cfg || !out) return OSCARS_EINVAL;
+  oscars_ctx* c = new (std::nothrow) oscars_ctx();
+  if (!c) return OSCARS_ENOMEM;
+  oscars_status st = OSCARS_OK;
+  try {
+    st = validate_and_layout(c, cfg);
+    if (st == OSCARS_OK) {
+      c->stream = static_cast<cudaStream_t>(cfg->cuda_stream);
+      c->M = cfg->M;
+      c->search_mode = cfg->search_mode;
+      c->t_iter.assign(c->W, 0);
+      c->tau.assign(c->W, 1);
+      const char* why = "";
+      int r = OSCARS_OK;
+      if (cfg->t_ticks) {
+        for (int i = 0; i < c->W; ++i) c->t_iter[i] = cfg->t_ticks[i];
+      } else if (cfg->speed) {
+        r = iteration_ticks(cfg->speed, c->W, cfg->ticks_per_unit, c->t_iter.data(), &why);
+      } else {
+        for (int i = 0; i < c->W; ++i) c->t_iter[i] = 1;  // homogeneous
+      }
+      if (r == OSCARS_OK)
+        r = schedule_solve(c->t_iter.data(), c->W, c->M, c->search_mode, &c->T_star, &c->max_wait, c->tau.data(), &why);
+      if (r != OSCARS_OK) st = fail(c, static_cast<oscars_status>(r), why);
+    }
+    if (st == OSCARS_OK) {
+      update_barrier(c, true);
+      c->clock.assign(c->W, 0);
+      c->idle.assign(c->W, 0);
+      if (c->model == OSCARS_MODEL_MLP) {
+        if (!cfg->shard_x || !cfg->shard_y || !cfg->shard_n) st = fail(c, OSCARS_EINVAL, "MLP: shard pointers are NULL");
+        for (int i = 0; st == OSCARS_OK && i < c->W; ++i) {
+          if (!cfg->shard_x[i] || !cfg->shard_y[i] || cfg->shard_n[i] < 1)
+            st = fail(c, OSCARS_EINVAL, "MLP: shard " + std::to_string(i) + " is NULL or empty");
+          else {
+            c->shard_x.push_back(cfg->shard_x[i]);
+            c->shard_y.push_back(cfg->shard_y[i]);
+            c->shard_n.push_back(cfg->shard_n[i]);
+          }
+        }
+        if (st == OSCARS_OK && !cfg->init_params) st = fail(c, OSCARS_EINVAL, "MLP: init_params is NULL");
+        if (st == OSCARS_OK) st = allocate_mlp(c);
+        if (st == OSCARS_OK) st = build_tables(c);
+        if (st == OSCARS_OK) {
+          cudaError_t e = copy_canonical(c, c->slab + static_cast<int64_t>(c->W) * c->P_pad, cfg->init_params, true, c->stream);
+          if (e == cudaSuccess) e = refresh_global_shadows(c, c->stream);
+          if (e == cudaSuccess) e = cudaStreamSynchronize(c->stream);
+          if (e != cudaSuccess) st = cuda_fail(c, e, "initial model upload");
+        }
+        if (st == OSCARS_OK && cudaStreamCreateWithFlags(&c->cap, cudaStreamNonBlocking) != cudaSuccess)
+          st = fail(c, OSCARS_ECUDA, "stream creation failed");
+        c->flags = cfg->flags;
+      } else {
+        c->flags = cfg->flags;
+        if (!dev_alloc(c, &c->slab, c->P_pad)) st = fail(c, OSCARS_ENOMEM, "device allocation failed (global model)");
+        if (st == OSCARS_OK) {
+          cudaError_t e = cudaMemsetAsync(c->slab, 0, c->P_pad * sizeof(float), c->stream);
+          if (e == cudaSuccess && cfg->init_params) e = copy_canonical(c, c->slab, cfg->init_params, true, c->stream);
+          if (e == cudaSuccess) e = cudaStreamSynchronize(c->stream);
+          if (e != cudaSuccess) st = cuda_fail(c, e, "initial model upload");
+        }
+      }
+    }
+  } catch (const std::bad_alloc&) {
+    st = OSCARS_ENOMEM;
+  } catch (...) {
+    st = OSCARS_EINVAL;
+  }
+  if (st != OSCARS_OK) {
+    free_all(c);
+    delete c;
+    return st;
+  }
+  *out = c;
+  return OSCARS_OK;
+}
+
+oscars_status oscars_destroy(oscars_ctx* c) {
+  if (!c) return OSCARS_OK;
+  cudaStreamSynchronize(c->stream);
+  free_all(c);
+  delete c;
+  return OSCARS_OK;
+}
+
+oscars_status oscars_local_steps(oscars_ctx* c, int32_t* tau_out, float* loss_out) {
+  if (!c) return OSCARS_EINVAL;
+  if (c->model != OSCARS_MODEL_MLP) return fail(c, OSCARS_ESTATE, "local steps need an MLP context");
+  if (c->pending) return fail(c, OSCARS_ESTATE, "the previous round has not been merged");
+  try {
+    cudaError_t e = cudaSuccess;
+    if (c->flags & 1) {
+      c->profiling = (c->flags & 2) != 0;
+      e = enqueue_round(c, c->stream);
+      c->profiling = false;
+    } else {
+      if (!c->round_exec) {
+        cudaGraph_t g = nullptr;
+        e = cudaStreamBeginCapture(c->cap, cudaStreamCaptureModeThreadLocal);
+        if (e == cudaSuccess) {
+          cudaError_t e2 = enqueue_round(c, c->cap);
+          e = cudaStreamEndCapture(c->cap, &g);
+          if (e2 != cudaSuccess) e = e2;
+        }
+        if (e == cudaSuccess) e = cudaGraphInstantiateWithFlags(&c->round_exec, g, 0);
+        if (g) cudaGraphDestroy(g);
+      }
+      if (e == cudaSuccess) e = cudaGraphLaunch(c->round_exec, c->stream);
+    }
+    if (e != cudaSuccess) return cuda_fail(c, e, "local steps launch");
+    for (int i = 0; i < c->W; ++i) {
+      const int64_t busy = static_cast<int64_t>(c->tau[i]) * c->t_iter[i];
+      c->clock[i] += c->barrier;
+      c->idle[i] += c->barrier - busy;
+    }
+    c->pending = true;
+    if (tau_out) std::memcpy(tau_out, c->tau.data(), c->W * sizeof(int32_t));
+    if (loss_out) {
+      e = cudaStreamSynchronize(c->stream);
+      if (e == cudaSuccess) e = cudaMemcpy(loss_out, c->loss_dev, c->W * sizeof(float), cudaMemcpyDeviceToHost);
+      if (e != cudaSuccess) return cuda_fail(c, e, "local steps");
+      return check_err_word(c);
+    }
+    return OSCARS_OK;
+  } catch (const std::bad_alloc&) {
+    return fail(c, OSCARS_ENOMEM, "host allocation failed");
+  }
+}
+
+oscars_status oscars_push_merge(oscars_ctx* c, const float* const* deltas, const float* weights) {
+  if (!c) return OSCARS_EINVAL;
+  if (c->rule == OSCARS_W_EXPLICIT && !weights) return fail(c, OSCARS_EINVAL, "explicit weight rule needs weights");
+  MergeArgs a;
+  std::memset(&a, 0, sizeof(a));
+  a.W = c->W;
+  if (c->rule == OSCARS_W_EXPLICIT) {
+    for (int k = 0; k < c->W; ++k) a.w[k] = weights[k];
+  } else {
+    merge_weights(c->rule, c->tau.data(), c->W, a.w);
+  }
+  const float eta = c->server_lr;
+  c->profiling = (c->flags & 2) != 0;
+  struct ProfOff {
+    oscars_ctx* c;
+    ~ProfOff() { c->profiling = false; }
+  } prof_off{c};
+  float* xg = c->slab + (c->model == OSCARS_MODEL_MLP ? static_cast<int64_t>(c->W) * c->P_pad : 0);
+  cudaError_t e = cudaSuccess;
+  if (!deltas) {
+    if (c->model != OSCARS_MODEL_MLP || !c->pending)
+      return fail(c, OSCARS_ESTATE, "push_merge without deltas needs pending local steps");
+    for (int k = 0; k < c->W; ++k) a.src[k] = c->slab + static_cast<int64_t>(k) * c->P_pad;
+    ProfScope ps(c, "merge", c->stream);
+    e = launch_merge(a, xg, c->P_pad, eta, true, c->stream);
+  } else {
+    for (int k = 0; k < c->W; ++k)
+      if (!deltas[k]) return fail(c, OSCARS_EINVAL, "NULL delta pointer");
+    if (c->model == OSCARS_MODEL_FLAT) {
+      for (int k = 0; k < c->W; ++k) a.src[k] = deltas[k];
+      ProfScope ps(c, "merge", c->stream);
+      e = launch_merge(a, xg, c->P, eta, false, c->stream);
+    } else {
+      int64_t co = 0;
+      for (const Layer& ly : c->layers) {
+        const int64_t nw = static_cast<int64_t>(ly.in) * ly.out;
+        for (int k = 0; k < c->W; ++k) a.src[k] = deltas[k] + co;
+        e = launch_merge(a, xg + ly.offW, nw, eta, false, c->stream);
+        if (e != cudaSuccess) break;
+        for (int k = 0; k < c->W; ++k) a.src[k] = deltas[k] + co + nw;
+        e = launch_merge(a, xg + ly.offB, ly.out, eta, false, c->stream);
+        if (e != cudaSuccess) break;
+        co += nw + ly.out;
+      }
+    }
+  }
+  if (e == cudaSuccess && c->model == OSCARS_MODEL_MLP) {
+    ProfScope ps(c, "shadow_refresh", c->stream);
+    e = refresh_global_shadows(c, c->stream);
+  }
+  if (e != cudaSuccess) return cuda_fail(c, e, "merge launch");
+  c->pending = false;
+  return OSCARS_OK;
+}
+
+oscars_status oscars_pull(oscars_ctx* c, float* dst) {
+  if (!c) return OSCARS_EINVAL;
+  cudaError_t e = cudaSuccess;
+  const int64_t g = c->model == OSCARS_MODEL_MLP ? static_cast<int64_t>(c->W) * c->P_pad : 0;
+  if (dst) {
+    e = copy_canonical(c, c->slab + g, dst, false, c->stream);
+    if (e == cudaSuccess && is_host_ptr(dst)) e = cudaStreamSynchronize(c->stream);
+  } else if (c->model == OSCARS_MODEL_MLP) {
+    e = launch_broadcast(c->slab + g, c->slab, c->P_pad, c->W, c->P_pad, c->stream);
+    for (int k = 0; e == cudaSuccess && k < c->W && c->shadow; ++k)
+      e = cudaMemcpyAsync(c->shadow + static_cast<int64_t>(k) * c->P_pad, c->shadow + g,
+                          c->P_pad * sizeof(__nv_bfloat16), cudaMemcpyDeviceToDevice, c->stream);
+  }
+  if (e != cudaSuccess) return cuda_fail(c, e, "pull");
+  return OSCARS_OK;
+}
+
+oscars_status oscars_get_schedule(const oscars_ctx* c, int64_t* T_star, int64_t* max_wait, int64_t* t_iter,
+                                  int32_t* tau, int64_t* wait, int64_t* clock, int64_t* idle) {
+  if (!c) return OSCARS_EINVAL;
+  if (T_star) *T_star = c->barrier;
+  if (max_wait) {
+    int64_t m = 0;
+    for (int i = 0; i < c->W; ++i) m = std::max(m, c->barrier - static_cast<int64_t>(c->tau[i]) * c->t_iter[i]);
+    *max_wait = m;
+  }
+  for (int i = 0; i < c->W; ++i) {
+    if (t_iter) t_iter[i] = c->t_iter[i];
+    if (tau) tau[i] = c->tau[i];
+    if (wait) wait[i] = c->barrier - static_cast<int64_t>(c->tau[i]) * c->t_iter[i];
+    if (clock) clock[i] = c->clock[i];
+    if (idle) idle[i] = c->idle[i];
+  }
+  return OSCARS_OK;
+}
+
+oscars_status oscars_set_local_steps(oscars_ctx* c, const int32_t* tau) {
+  if (!c || !tau) return OSCARS_EINVAL;
+  if (c->pending) return fail(c, OSCARS_ESTATE, "cannot change tau while a round is pending");
+  for (int i = 0; i < c->W; ++i)
+    if (tau[i] < 1) return fail(c, OSCARS_EINVAL, "tau must be >= 1");
+  for (int i = 0; i < c->W; ++i) c->tau[i] = tau[i];
+  update_barrier(c, false);
+  if (c->model == OSCARS_MODEL_MLP) {
+    cudaStreamSynchronize(c->stream);
+    return build_tables(c);
+  }
+  return OSCARS_OK;
+}
+
+oscars_status oscars_eval_loss(oscars_ctx* c, const float* x, const int32_t* y, int64_t n, float* loss) {
+  if (!c || !x || !y || !loss || n < 1) return OSCARS_EINVAL;
+  if (c->model != OSCARS_MODEL_MLP) return fail(c, OSCARS_ESTATE, "eval needs an MLP context");
+  cudaError_t e = cudaSuccess;
+  const int64_t g = static_cast<int64_t>(c->W) * c->P_pad;
+  if (c->L == 1 && !c->bf16) {
+    const int blocks = static_cast<int>(std::min<int64_t>(1024, (n + 7) / 8));
+    if (c->eval_part_cap < blocks) {
+      if (!dev_alloc(c, &c->eval_part, blocks)) return fail(c, OSCARS_ENOMEM, "eval scratch");
+      c->eval_part_cap = blocks;
+    }
+    SoftregEvalArgs a;
+    a.master = c->slab + g;
+    a.offW = c->layers[0].offW;
+    a.offB = c->layers[0].offB;
+    a.D = c->dims[0];
+    a.C = c->C;
+    a.x = x;
+    a.y = y;
+    a.n = n;
+    a.loss_sum = c->eval_part;
+    e = launch_softreg_eval(a, blocks, c->stream);
+    if (e == cudaSuccess) e = launch_sum_scaled(c->eval_part, blocks, 1.0 / static_cast<double>(n), c->loss_dev, c->stream);
+  } else {
+    if (n % c->B != 0) return fail(c, OSCARS_ENOTSUP, "MLP eval: n must be a multiple of the batch size");
+    const int64_t chunks = n / c->B;
+    const int nc = c->B / kRowsPerLossChunk;
+    if (c->estart_cap < chunks) {
+      if (!dev_alloc(c, &c->estart, chunks)) return fail(c, OSCARS_ENOMEM, "eval scratch");
+      c->estart_cap = chunks;
+    }
+    if (c->eval_part_cap < chunks * nc) {
+      if (!dev_alloc(c, &c->eval_part, chunks * nc)) return fail(c, OSCARS_ENOMEM, "eval scratch");
+      c->eval_part_cap = chunks * nc;
+    }
+    std::vector<int64_t> starts(chunks), ns(c->W, n);
+    for (int64_t i = 0; i < chunks; ++i) starts[i] = i * c->B;
+    std::vector<const float*> xs(c->W, x);
+    std::vector<const int32_t*> ys(c->W, y);
+    e = cudaStreamSynchronize(c->stream);
+    if (e == cudaSuccess) e = cudaMemcpy(c->estart, starts.data(), chunks * sizeof(int64_t), cudaMemcpyHostToDevice);
+    if (e == cudaSuccess) e = cudaMemcpy(c->ex_tab, xs.data(), c->W * sizeof(float*), cudaMemcpyHostToDevice);
+    if (e == cudaSuccess) e = cudaMemcpy(c->ey_tab, ys.data(), c->W * sizeof(int32_t*), cudaMemcpyHostToDevice);
+    if (e == cudaSuccess) e = cudaMemcpy(c->en_tab, ns.data(), c->W * sizeof(int64_t), cudaMemcpyHostToDevice);
+    for (int64_t base = 0; e == cudaSuccess && base < chunks; base += c->W) {
+      const int na = static_cast<int>(std::min<int64_t>(c->W, chunks - base));
+      StageArgs sa;
+      sa.x = c->ex_tab;
+      sa.y = c->ey_tab;
+      sa.n = c->en_tab;
+      sa.start = c->estart + base;
+      sa.row_add = 0;
+      sa.wid = c->lane_ids;
+      sa.D = c->dims[0];
+      sa.B = c->B;
+      sa.A0 = c->A[0];
+      sa.A0T = c->AT[0];
+      sa.labels = c->labels;
+      e = launch_stage(sa, na, c->stream);
+      if (e == cudaSuccess) e = enqueue_forward(c, c->lane_ids, c->global_src, na, c->stream);
+      if (e == cudaSuccess) {
+        HeadArgs h = head_base(c);
+        h.wid = c->lane_ids;
+        h.src = c->global_src;
+        h.loss_part = c->eval_part;
+        h.part_mul = 1;
+        h.part_add = static_cast<int>(base);
+        e = launch_head_fwd(h, na, c->stream);
+      }
+    }
+    if (e == cudaSuccess)
+      e = launch_sum_scaled(c->eval_part, chunks * nc, 1.0 / static_cast<double>(n), c->loss_dev, c->stream);
+  }
+  if (e == cudaSuccess) e = cudaStreamSynchronize(c->stream);
+  if (e == cudaSuccess) e = cudaMemcpy(loss, c->loss_dev, sizeof(float), cudaMemcpyDeviceToHost);
+  if (e != cudaSuccess) return cuda_fail(c, e, "eval");
+  return check_err_word(c);
+}
+
+oscars_status oscars_read_replica(oscars_ctx* c, int32_t k, float* dst) {
+  if (!c || !dst) return OSCARS_EINVAL;
+  if (c->model != OSCARS_MODEL_MLP) return fail(c, OSCARS_ESTATE, "replicas exist in MLP mode only");
+  if (k < 0 || k >= c->W) return fail(c, OSCARS_EINVAL, "worker index out of range");
+  cudaError_t e = copy_canonical(c, c->slab + static_cast<int64_t>(k) * c->P_pad, dst, false, c->stream);
+  if (e == cudaSuccess && is_host_ptr(dst)) e = cudaStreamSynchronize(c->stream);
+  if (e != cudaSuccess) return cuda_fail(c, e, "read replica");
+  return OSCARS_OK;
+}
+
+oscars_status oscars_gemm_bf16_nt(const void* A, const void* B, float* C, int32_t M, int32_t N, int32_t K,
+                                  void* stream) {
+  if (!A || !B || !C || M < 128 || M % 128 != 0 || N < 1 || K < 8 || K % 8 != 0) return OSCARS_EINVAL;
+  if ((reinterpret_cast<uintptr_t>(A) | reinterpret_cast<uintptr_t>(B)) & 15) return OSCARS_EINVAL;
+  CUtensorMap mA, mB;
+  if (!make_map(&mA, A, K, M, 1, K * 2ull, static_cast<uint64_t>(M) * K * 2ull, 128) ||
+      !make_map(&mB, B, K, N, 1, K * 2ull, static_cast<uint64_t>(N) * K * 2ull, 128))
+    return OSCARS_ECUDA;
+  GemmArgs g;
+  std::memset(&g, 0, sizeof(g));
+  g.M = M;
+  g.N = N;
+  g.K = K;
+  g.c_out = C;
+  return launch_gemm(kEpiStore, mA, mB, g, 1, static_cast<cudaStream_t>(stream)) == cudaSuccess ? OSCARS_OK
+                                                                                               : OSCARS_ECUDA;
+}
+
+int32_t oscars_profile_read(oscars_ctx* c, int32_t cap, const char** names, double* ms_total, int32_t* launches) {
+  if (!c) return -1;
+  prof_collect(c);
+  const int n = static_cast<int>(c->prof_names.size());
+  for (int i = 0; i < n && i < cap; ++i) {
+    if (names) names[i] = c->prof_names[i].c_str();
+    if (ms_total) ms_total[i] = c->prof_ms[i];
+    if (launches) launches[i] = c->prof_count[i];
+  }
+  return n;
+}
+
+oscars_status oscars_profile_reset(oscars_ctx* c) {
+  if (!c) return OSCARS_EINVAL;
+  prof_collect(c);
+  c->prof_names.clear();
+  c->prof_ms.clear();
+  c->prof_count.clear();
+  return OSCARS_OK;
+}
+
+oscars_status oscars_num_params(const oscars_ctx* c, int64_t* P) {
+  if (!c || !P) return OSCARS_EINVAL;
+  *P = c->P;
+  return OSCARS_OK;
+}
+
+const char* oscars_last_error(const oscars_ctx* c) { return c ? c->last_error.c_str() : ""; }
+
+oscars_status oscars_merge(float* x_g, const float* const* deltas, const float* w, int32_t W, int64_t P,
+                           float server_lr, void* stream) {
+  if (!x_g || !deltas || !w || W < 1 || W > kMaxMergeWorkers || P < 0) return OSCARS_EINVAL;
+  MergeArgs a;
+  std::memset(&a, 0, sizeof(a));
+  a.W = W;
+  for (int k = 0; k < W; ++k) {
+    if (!deltas[k]) return OSCARS_EINVAL;
+    a.src[k] = deltas[k];
+    a.w[k] = w[k];
+  }
+  return launch_merge(a, x_g, P, server_lr, false, static_cast<cudaStream_t>(stream)) == cudaSuccess ? OSCARS_OK
+                                                                                                   : OSCARS_ECUDA;
+}
+
+}  // extern "C"

@@ -1,0 +1,316 @@
+// Grouped bf16 GEMM on the 5th-generation tensor cores (tcgen05, sm_103a)
+// for the workers' dense layers (Eq. 4, "otherwise" branch: the forward and
+// backward passes of x - lr * g(x)), with the step's elementwise work fused
+// into the epilogue.
+//
+//   D[m][n] = sum_k A[m][k] * B[n][k]     A, B bf16 K-major, D fp32 in TMEM
+//
+// One CTA computes one 128 x BN tile of one active worker (grid z = worker).
+// Warp 0 lane 0 streams K-blocks of 64 with TMA (128-byte swizzle, 3-D
+// tensor maps whose z coordinate selects the worker's buffer or the
+// parameter slot), warp 1 lane 0 issues tcgen05.mma (M=128, N=BN, K=16) into
+// a TMEM accumulator and frees each stage with tcgen05.commit, warp 2 owns
+// the TMEM allocation; then all four warps read their 32 TMEM lanes
+// (one output row per thread) and run the epilogue:
+//
+//  kEpiFwd  hidden layer forward, m = output feature, n = sample:
+//           h = relu(acc + bias[m]) -> bf16 H[n][m] and H^T[m][n].
+//  kEpiDh   input gradient of a hidden layer, m = input feature, n = sample:
+//           g = acc * (Hmask[n][m] > 0) -> bf16 G[n][m], G^T[m][n] and the
+//           bias gradient gb[m] = sum_n g (fp32, whole batch in one tile).
+//  kEpiDw   weight gradient + SGD, m = output feature, n = input feature:
+//           W[dst] = fmaf(-lr, acc, W[src]) (fp32 master), bf16 shadow,
+//           optional bf16 transposed shadow; column-tile 0 also updates the
+//           bias b[dst] = fmaf(-lr, gb[m], b[src]).
+//  kEpiStore plain C[m][n] = acc in fp32 (a library GEMM for tests and
+//           callers that need one).
+//
+// All waits are bounded (see common.cuh) and report through a device word.
+#include <cstdio>
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace oscars {
+
+namespace {
+
+constexpr int BM = 128;
+constexpr int BK = 64;
+constexpr int kThreads = 128;
+constexpr int kABytes = BM * BK * 2;
+
+template <int BN>
+struct TileCfg {
+  static constexpr int kBBytes = BN * BK * 2;
+  static constexpr int kStageBytes = kABytes + kBBytes;
+  static constexpr uint32_t kTmemCols = BN <= 32 ? 32 : BN <= 64 ? 64 : BN <= 128 ? 128 : 256;
+};
+
+template <int EPI>
+__device__ __forceinline__ void epi_fwd(const GemmArgs& a, int wid, int src, int m, int n0,
+                                        const float (&v)[32]) {
+  const float bias = a.master[static_cast<int64_t>(src) * a.slot_stride + a.offB + m];
+  __nv_bfloat16* out = a.out + static_cast<int64_t>(wid) * a.N * a.M;
+  uint32_t pk[16];
+#pragma unroll
+  for (int c = 0; c < 32; c += 2) {
+    const float h0 = fmaxf(v[c] + bias, 0.f);
+    const float h1 = fmaxf(v[c + 1] + bias, 0.f);
+    const __nv_bfloat162 p = __floats2bfloat162_rn(h0, h1);
+    out[static_cast<int64_t>(n0 + c) * a.M + m] = p.x;
+    out[static_cast<int64_t>(n0 + c + 1) * a.M + m] = p.y;
+    pk[c >> 1] = *reinterpret_cast<const uint32_t*>(&p);
+  }
+  uint4* outT = reinterpret_cast<uint4*>(a.outT + (static_cast<int64_t>(wid) * a.M + m) * a.N + n0);
+#pragma unroll
+  for (int q = 0; q < 4; ++q) outT[q] = make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
+}
+
+__device__ __forceinline__ float epi_dh(const GemmArgs& a, int wid, int m, int n0, const float (&v)[32]) {
+  const __nv_bfloat16* hm = a.hmask + static_cast<int64_t>(wid) * a.N * a.M;
+  __nv_bfloat16* out = a.out + static_cast<int64_t>(wid) * a.N * a.M;
+  uint32_t pk[16];
+  float gsum = 0.f;
+#pragma unroll
+  for (int c = 0; c < 32; c += 2) {
+    const int64_t e0 = static_cast<int64_t>(n0 + c) * a.M + m;
+    const int64_t e1 = e0 + a.M;
+    const float g0 = __bfloat162float(hm[e0]) > 0.f ? v[c] : 0.f;
+    const float g1 = __bfloat162float(hm[e1]) > 0.f ? v[c + 1] : 0.f;
+    gsum += g0;
+    gsum += g1;
+    const __nv_bfloat162 p = __floats2bfloat162_rn(g0, g1);
+    out[e0] = p.x;
+    out[e1] = p.y;
+    pk[c >> 1] = *reinterpret_cast<const uint32_t*>(&p);
+  }
+  uint4* outT = reinterpret_cast<uint4*>(a.outT + (static_cast<int64_t>(wid) * a.M + m) * a.N + n0);
+#pragma unroll
+  for (int q = 0; q < 4; ++q) outT[q] = make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
+  return gsum;
+}
+
+__device__ __forceinline__ void epi_dw(const GemmArgs& a, int wid, int src, int m, int n0,
+                                       const float (&v)[32]) {
+  const int64_t so = static_cast<int64_t>(src) * a.slot_stride + a.offW + static_cast<int64_t>(m) * a.N;
+  const int64_t dof = static_cast<int64_t>(wid) * a.slot_stride + a.offW + static_cast<int64_t>(m) * a.N;
+  float nw[32];
+  if (n0 + 32 <= a.N) {
+    const float4* s4 = reinterpret_cast<const float4*>(a.master + so + n0);
+    float4* d4 = reinterpret_cast<float4*>(a.master_w + dof + n0);
+    uint2* sh = reinterpret_cast<uint2*>(a.shadow + dof + n0);
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+      const float4 o = s4[q];
+      float4 r;
+      r.x = fmaf(-a.lr, v[4 * q + 0], o.x);
+      r.y = fmaf(-a.lr, v[4 * q + 1], o.y);
+      r.z = fmaf(-a.lr, v[4 * q + 2], o.z);
+      r.w = fmaf(-a.lr, v[4 * q + 3], o.w);
+      d4[q] = r;
+      sh[q] = make_uint2(pack_bf16x2(r.x, r.y), pack_bf16x2(r.z, r.w));
+      nw[4 * q + 0] = r.x;
+      nw[4 * q + 1] = r.y;
+      nw[4 * q + 2] = r.z;
+      nw[4 * q + 3] = r.w;
+    }
+  } else {
+#pragma unroll
+    for (int c = 0; c < 32; ++c) {
+      nw[c] = 0.f;
+      if (n0 + c < a.N) {
+        const float r = fmaf(-a.lr, v[c], a.master[so + n0 + c]);
+        a.master_w[dof + n0 + c] = r;
+        a.shadow[dof + n0 + c] = __float2bfloat16_rn(r);
+        nw[c] = r;
+      }
+    }
+  }
+  if (a.shadowT) {
+    __nv_bfloat16* t = a.shadowT + static_cast<int64_t>(wid) * a.slotT_stride + a.offT;
+#pragma unroll
+    for (int c = 0; c < 32; ++c)
+      if (n0 + c < a.N) t[static_cast<int64_t>(n0 + c) * a.M + m] = __float2bfloat16_rn(nw[c]);
+  }
+}
+
+__device__ __forceinline__ void epi_store(const GemmArgs& a, int m, int n0, const float (&v)[32]) {
+  float* c = a.c_out + static_cast<int64_t>(m) * a.N + n0;
+  if (n0 + 32 <= a.N && (a.N & 3) == 0) {
+    float4* c4 = reinterpret_cast<float4*>(c);
+#pragma unroll
+    for (int q = 0; q < 8; ++q) c4[q] = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+  } else {
+#pragma unroll
+    for (int j = 0; j < 32; ++j)
+      if (n0 + j < a.N) c[j] = v[j];
+  }
+}
+
+template <int BN, int EPI>
+__global__ void __launch_bounds__(kThreads) gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA,
+                                                           const __grid_constant__ CUtensorMap mapB,
+                                                           const __grid_constant__ GemmArgs a,
+                                                           int stages) {
+  using Cfg = TileCfg<BN>;
+  extern __shared__ uint8_t smem_raw[];
+  uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+  uint8_t* sA = smem;
+  uint8_t* sB = smem + stages * kABytes;
+  uint64_t* full = reinterpret_cast<uint64_t*>(sB + stages * Cfg::kBBytes);
+  uint64_t* empty = full + stages;
+  uint64_t* accum = empty + stages;
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(accum + 1);
+
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int li = blockIdx.z;
+  const int wid = a.wid ? a.wid[li] : li, src = a.src ? a.src[li] : li;
+  const int m0 = blockIdx.x * BM, n0 = blockIdx.y * BN;
+  const int nk = (a.K + BK - 1) / BK;
+
+  if (threadIdx.x == 0) {
+    prefetch_tmap(&mapA);
+    prefetch_tmap(&mapB);
+    for (int s = 0; s < stages; ++s) {
+      mbar_init(&full[s], 1);
+      mbar_init(&empty[s], 1);
+    }
+    mbar_init(accum, 1);
+    fence_barrier_init();
+    fence_proxy_async_smem();
+  }
+  if (warp == 2) {
+    tmem_alloc(tmem_slot, Cfg::kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tmem_slot;
+
+  if (warp == 0 && lane == 0) {
+    // TMA producer
+    const int za = a.a_z_src ? src : wid;
+    const int zb = a.b_z_src ? src : wid;
+    for (int kb = 0; kb < nk; ++kb) {
+      const int s = kb % stages;
+      if (kb >= stages && !mbar_wait(&empty[s], ((kb / stages) + 1) & 1, a.err, kDevTimeoutEmpty)) break;
+      mbar_arrive_expect_tx(&full[s], kABytes + Cfg::kBBytes);
+      tma_load_3d(sA + s * kABytes, &mapA, kb * BK, m0, za, &full[s]);
+      tma_load_3d(sB + s * Cfg::kBBytes, &mapB, kb * BK, n0, zb, &full[s]);
+    }
+  } else if (warp == 1 && lane == 0) {
+    // MMA issuer
+    constexpr uint32_t idesc = idesc_bf16_f32(BM, BN);
+    for (int kb = 0; kb < nk; ++kb) {
+      const int s = kb % stages;
+      if (!mbar_wait(&full[s], (kb / stages) & 1, a.err, kDevTimeoutFull)) break;
+      tc_fence_after();
+      const uint32_t a_base = smem_u32(sA + s * kABytes);
+      const uint32_t b_base = smem_u32(sB + s * Cfg::kBBytes);
+#pragma unroll
+      for (int j = 0; j < BK / 16; ++j)
+        umma_bf16(tmem, smem_desc_k128(a_base + j * 32), smem_desc_k128(b_base + j * 32), idesc,
+                  (kb | j) != 0 ? 1u : 0u);
+      umma_commit(&empty[s]);
+    }
+    umma_commit(accum);  // arrives once every issued MMA has completed
+  }
+  __syncwarp();
+
+  // epilogue: thread = one accumulator row
+  int acc_ok = 0;
+  if (lane == 0) acc_ok = mbar_wait(accum, 0, a.err, kDevTimeoutAccum) ? 1 : 0;
+  acc_ok = __shfl_sync(0xffffffffu, acc_ok, 0);
+  tc_fence_after();
+  if (acc_ok) {
+    const int m = m0 + warp * 32 + lane;
+    const uint32_t trow = tmem + (static_cast<uint32_t>(warp * 32) << 16);
+    float gsum = 0.f;
+#pragma unroll 1
+    for (int c0 = 0; c0 < BN; c0 += 32) {
+      float v[32];
+      tmem_ld_32x32b_x32(trow + c0, v);
+      if (EPI == kEpiFwd) {
+        epi_fwd<EPI>(a, wid, src, m, n0 + c0, v);
+      } else if (EPI == kEpiDh) {
+        gsum += epi_dh(a, wid, m, n0 + c0, v);
+      } else if (EPI == kEpiStore) {
+        if (n0 + c0 < a.N) epi_store(a, m, n0 + c0, v);
+      } else {
+        if (n0 + c0 < a.N) epi_dw(a, wid, src, m, n0 + c0, v);
+      }
+    }
+    if (EPI == kEpiDh) a.gb_out[static_cast<int64_t>(wid) * a.M + m] = gsum;
+    if (EPI == kEpiDw && blockIdx.y == 0) {
+      const int64_t bo = a.offB + m;
+      a.master_w[static_cast<int64_t>(wid) * a.slot_stride + bo] =
+          fmaf(-a.lr, a.gb_in[static_cast<int64_t>(wid) * a.M + m], a.master[static_cast<int64_t>(src) * a.slot_stride + bo]);
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 2) {
+    tc_fence_after();
+    tmem_dealloc(tmem, Cfg::kTmemCols);
+  }
+}
+
+// Shared memory that keeps the number of resident CTAs per SM at or below
+// 512 / (TMEM columns per CTA), so a tcgen05.alloc never has to wait.
+size_t smem_floor_for_tmem(uint32_t cols) {
+  const size_t per_sm = 233472;  // 228 KB
+  const size_t max_ctas = 512 / cols;
+  return per_sm / (max_ctas + 1) - 1024 + 16;
+}
+
+template <int BN, int EPI>
+cudaError_t launch_tile(const CUtensorMap& mA, const CUtensorMap& mB, const GemmArgs& a, int n_active,
+                        cudaStream_t s) {
+  using Cfg = TileCfg<BN>;
+  const int nk = (a.K + BK - 1) / BK;
+  const int stages = nk < 4 ? nk : 4;
+  size_t smem = 1024 + static_cast<size_t>(stages) * Cfg::kStageBytes + (2 * stages + 2) * 8 + 16;
+  const size_t floor_b = smem_floor_for_tmem(Cfg::kTmemCols);
+  if (smem < floor_b) smem = floor_b;
+  cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<BN, EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       static_cast<int>(smem));
+  if (e != cudaSuccess) return e;
+  dim3 grid(a.M / BM, (a.N + BN - 1) / BN, n_active);
+  gemm_tc_kernel<BN, EPI><<<grid, kThreads, smem, s>>>(mA, mB, a, stages);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+int gemm_bn_for(int epi, int N) {
+  if (epi == kEpiDw || epi == kEpiStore) return 128;
+  return N;  // forward / input gradient: the whole batch in one tile
+}
+
+cudaError_t launch_gemm(int epi, const CUtensorMap& mA, const CUtensorMap& mB, const GemmArgs& a,
+                        int n_active, cudaStream_t s) {
+  if (a.M % BM != 0) return cudaErrorInvalidValue;
+  if (epi == kEpiDw) return launch_tile<128, kEpiDw>(mA, mB, a, n_active, s);
+  if (epi == kEpiStore) return launch_tile<128, kEpiStore>(mA, mB, a, n_active, s);
+  const int bn = gemm_bn_for(epi, a.N);
+  if (epi == kEpiFwd) {
+    switch (bn) {
+      case 32: return launch_tile<32, kEpiFwd>(mA, mB, a, n_active, s);
+      case 64: return launch_tile<64, kEpiFwd>(mA, mB, a, n_active, s);
+      case 128: return launch_tile<128, kEpiFwd>(mA, mB, a, n_active, s);
+      case 256: return launch_tile<256, kEpiFwd>(mA, mB, a, n_active, s);
+      default: return cudaErrorInvalidValue;
+    }
+  }
+  switch (bn) {
+    case 32: return launch_tile<32, kEpiDh>(mA, mB, a, n_active, s);
+    case 64: return launch_tile<64, kEpiDh>(mA, mB, a, n_active, s);
+    case 128: return launch_tile<128, kEpiDh>(mA, mB, a, n_active, s);
+    case 256: return launch_tile<256, kEpiDh>(mA, mB, a, n_active, s);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+}  // namespace oscars

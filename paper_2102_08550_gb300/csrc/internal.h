@@ -1,0 +1,153 @@
+// Internal declarations shared by the translation units of liboscars.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace oscars {
+
+constexpr int kMaxMergeWorkers = 256;   // pointer table of the merge kernel
+constexpr int kMaxWorkersMLP = 64;
+constexpr int kMaxClasses = 32;
+constexpr int kRowsPerLossChunk = 16;   // rows per loss partial in the head kernel
+
+// ---------------------------------------------------------------- merge
+struct MergeArgs {
+  const float* src[kMaxMergeWorkers];  // delta_k, or replica x^k
+  float w[kMaxMergeWorkers];
+  int W;
+};
+
+// x_g <- x_g + eta * sum_k w_k * (replica ? src_k - x_g : src_k), p < P.
+cudaError_t launch_merge(const MergeArgs& a, float* x_g, int64_t P, float eta, bool replica,
+                         cudaStream_t s);
+
+// ---------------------------------------------------------------- scheduler (host)
+int iteration_ticks(const double* speed, int n, int64_t Q, int64_t* t, const char** why);
+int schedule_solve(const int64_t* t, int n, int64_t M, int mode, int64_t* T_star,
+                   int64_t* max_wait, int32_t* tau, const char** why);
+void merge_weights(int rule, const int32_t* tau, int n, float* w);
+
+// ---------------------------------------------------------------- softmax regression (fp32)
+struct SoftregArgs {
+  const float* master;          // slab base (slots of P_pad floats)
+  float* master_out;
+  int64_t slot_stride;          // P_pad
+  int global_slot;              // W
+  int64_t offW, offB;           // element offsets inside a slot
+  int D, C, B;
+  float lr;
+  const int32_t* tau;           // [W]
+  const float* const* shard_x;  // [W] device pointers
+  const int32_t* const* shard_y;
+  const int64_t* shard_n;       // [W]
+  const int64_t* cursor;        // [W]
+  float* loss_part;             // [W][max_tau]  (sum of per-sample losses of one step)
+  int max_tau;
+};
+cudaError_t launch_softreg_round(const SoftregArgs& a, int W, cudaStream_t s);
+size_t softreg_smem_bytes(int D, int C, int B);
+
+struct SoftregEvalArgs {
+  const float* master;  // global slot
+  int64_t offW, offB;
+  int D, C;
+  const float* x;
+  const int32_t* y;
+  int64_t n;
+  float* loss_sum;      // [blocks] partial sums
+};
+cudaError_t launch_softreg_eval(const SoftregEvalArgs& a, int blocks, cudaStream_t s);
+
+// ---------------------------------------------------------------- MLP (bf16 GEMMs)
+// Rows of one step's work: active lane i uses activation buffers of lane
+// `wid[i]` and reads parameters from slot `src[i]` (the global slot on the
+// first local step: the fused pull), writing them to slot `wid[i]`.
+struct StageArgs {
+  const float* const* x;   // [lanes] sample matrix per lane (device pointers)
+  const int32_t* const* y;
+  const int64_t* n;        // [lanes] rows available
+  const int64_t* start;    // [lanes] first row (cursor)
+  int64_t row_add;         // added to start (step * B)
+  const int* wid;          // [n_active]
+  int D, B;
+  __nv_bfloat16* A0;       // [lanes][B][D]
+  __nv_bfloat16* A0T;      // [lanes][D][B]
+  int32_t* labels;         // [lanes][B]
+};
+cudaError_t launch_stage(const StageArgs& a, int n_active, cudaStream_t s);
+
+enum GemmEpi { kEpiFwd = 0, kEpiDh = 1, kEpiDw = 2, kEpiStore = 3 };
+
+struct GemmArgs {
+  const int* wid;     // [n_active]
+  const int* src;     // [n_active]
+  int M, N, K;
+  int a_z_src, b_z_src;  // TMA z coordinate of A / B: 1 = src slot, 0 = lane id
+  int* err;
+  // kEpiFwd: out = relu(acc + bias[m]) -> H [lane][N][M], HT [lane][M][N]
+  // kEpiDh : out = acc * (Hmask[lane][n][m] > 0) -> G, GT, gb[lane][m]
+  // kEpiDw : W[dst] = W[src] - lr * acc (rows m, cols n < N), shadows, bias
+  const float* master;      // fp32 slab base
+  float* master_w;          // same slab (written)
+  __nv_bfloat16* shadow;    // bf16 slab (same layout as master)
+  __nv_bfloat16* shadowT;   // bf16 transposed slab (or null)
+  int64_t slot_stride;      // P_pad
+  int64_t slotT_stride;     // PT_pad
+  int64_t offW, offB, offT; // element offsets of W_l, b_l, W_l^T in a slot
+  float lr;
+  const float* gb_in;       // [lanes][M] bias gradient (kEpiDw)
+  const __nv_bfloat16* hmask;  // [lanes][N][M] (kEpiDh)
+  __nv_bfloat16* out;       // [lanes][N][M]
+  __nv_bfloat16* outT;      // [lanes][M][N]
+  float* gb_out;            // [lanes][M] (kEpiDh)
+  float* c_out;             // kEpiStore: C [M][N] fp32 row-major (lane 0 only)
+};
+cudaError_t launch_gemm(int epi, const CUtensorMap& mapA, const CUtensorMap& mapB,
+                        const GemmArgs& a, int n_active, cudaStream_t s);
+int gemm_bn_for(int epi, int N);
+
+struct HeadArgs {
+  const int* wid;
+  const int* src;
+  int H, C, B;
+  const __nv_bfloat16* Ain;   // [lanes][B][H] input of the last layer
+  const int32_t* labels;      // [lanes][B]
+  const __nv_bfloat16* shadow;
+  const float* master;
+  float* master_w;
+  __nv_bfloat16* shadow_w;
+  int64_t slot_stride;
+  int64_t offW, offB;
+  float lr;
+  float* dlog;                // [lanes][B][C]
+  float* loss_part;           // rows of (B/16) partial sums
+  int part_mul, part_add;     // row = wid * part_mul + part_add
+  __nv_bfloat16* G;           // [lanes][B][H] (head_bwd)
+  __nv_bfloat16* GT;          // [lanes][H][B]
+  float* gb;                  // [lanes][H]
+};
+cudaError_t launch_head_fwd(const HeadArgs& a, int n_active, cudaStream_t s);
+cudaError_t launch_head_bwd(const HeadArgs& a, int n_active, cudaStream_t s);
+
+// loss[w] = sum_{s < tau[w]} sum_c part[(w*max_tau + s)*nc + c] / (B * tau[w])
+cudaError_t launch_loss_finalize(const float* part, const int32_t* tau, int W, int max_tau,
+                                 int nc, int B, float* loss, cudaStream_t s);
+// out[0] = sum_i part[i] / n (fixed order)
+cudaError_t launch_sum_scaled(const float* part, int64_t count, double scale, float* out,
+                              cudaStream_t s);
+// cursor[w] = (cursor[w] + tau[w] * B) % n[w]
+cudaError_t launch_cursor_advance(int64_t* cursor, const int32_t* tau, const int64_t* n, int B,
+                                  int W, cudaStream_t s);
+// shadow[p] = bf16(master[p]) for one slot; shadowT for layers with a transposed copy
+cudaError_t launch_shadow_refresh(const float* master, __nv_bfloat16* shadow, int64_t count,
+                                  cudaStream_t s);
+cudaError_t launch_transpose_bf16(const __nv_bfloat16* src, __nv_bfloat16* dst, int rows,
+                                  int cols, cudaStream_t s);
+// replicas[k] = x_g for k < W (fp32 and bf16 shadows)
+cudaError_t launch_broadcast(const float* xg, float* slab, int64_t stride, int W, int64_t count,
+                             cudaStream_t s);
+
+}  // namespace oscars

@@ -1,0 +1,146 @@
+// Server merge and global update (Eq. 4, first branch; the parameter-server
+// push / combine / pull of the Introduction), delta form:
+//
+//   x_g[p] <- x_g[p] + eta_s * sum_k w_k * delta_k[p],
+//   delta_k = pushed delta, or x^k[p] - x_g[p] for pushed replicas.
+//
+// HBM-bound streaming kernel: every byte of the W pushed buffers is read
+// once with 16-byte streaming loads (ld.global.cs: evict-first, they are
+// never reused), the sum is kept in fp32 registers in worker order
+// k = 0..W-1, and x_g is read and written once.  Algorithmic traffic:
+// (W + 2) * P * 4 bytes.  The pointer table and weights travel in a
+// __grid_constant__ parameter block, so each thread only loads data.
+//
+// Grid: persistent, (SM count) x (resident CTAs per SM) blocks of 256
+// threads striding over 16-byte chunks; each thread keeps 8 independent
+// 16-byte loads in flight per group of 8 workers.
+#include "common.cuh"
+#include "internal.h"
+
+namespace oscars {
+
+namespace {
+
+constexpr int kThreads = 256;
+constexpr int kGroup = 8;
+
+__device__ __forceinline__ float4 ld_stream4(const float4* p) { return __ldcs(p); }
+
+template <bool kReplica>
+__global__ void __launch_bounds__(kThreads) merge_vec4_kernel(const __grid_constant__ MergeArgs a,
+                                                              float* __restrict__ x_g, int64_t n4,
+                                                              float eta) {
+  float4* xg4 = reinterpret_cast<float4*>(x_g);
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n4; i += stride) {
+    const float4 x = __ldcs(xg4 + i);
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    int k = 0;
+    for (; k + kGroup <= a.W; k += kGroup) {
+      float4 v[kGroup];
+#pragma unroll
+      for (int j = 0; j < kGroup; ++j) v[j] = ld_stream4(reinterpret_cast<const float4*>(a.src[k + j]) + i);
+#pragma unroll
+      for (int j = 0; j < kGroup; ++j) {
+        const float w = a.w[k + j];
+        if (kReplica) {
+          acc.x = fmaf(w, v[j].x - x.x, acc.x);
+          acc.y = fmaf(w, v[j].y - x.y, acc.y);
+          acc.z = fmaf(w, v[j].z - x.z, acc.z);
+          acc.w = fmaf(w, v[j].w - x.w, acc.w);
+        } else {
+          acc.x = fmaf(w, v[j].x, acc.x);
+          acc.y = fmaf(w, v[j].y, acc.y);
+          acc.z = fmaf(w, v[j].z, acc.z);
+          acc.w = fmaf(w, v[j].w, acc.w);
+        }
+      }
+    }
+    for (; k < a.W; ++k) {
+      const float4 v = ld_stream4(reinterpret_cast<const float4*>(a.src[k]) + i);
+      const float w = a.w[k];
+      if (kReplica) {
+        acc.x = fmaf(w, v.x - x.x, acc.x);
+        acc.y = fmaf(w, v.y - x.y, acc.y);
+        acc.z = fmaf(w, v.z - x.z, acc.z);
+        acc.w = fmaf(w, v.w - x.w, acc.w);
+      } else {
+        acc.x = fmaf(w, v.x, acc.x);
+        acc.y = fmaf(w, v.y, acc.y);
+        acc.z = fmaf(w, v.z, acc.z);
+        acc.w = fmaf(w, v.w, acc.w);
+      }
+    }
+    float4 out;
+    out.x = fmaf(eta, acc.x, x.x);
+    out.y = fmaf(eta, acc.y, x.y);
+    out.z = fmaf(eta, acc.z, x.z);
+    out.w = fmaf(eta, acc.w, x.w);
+    __stcs(xg4 + i, out);
+  }
+}
+
+// Any alignment: one element per thread and iteration, elements [begin, P).
+template <bool kReplica>
+__global__ void __launch_bounds__(kThreads) merge_scalar_kernel(const __grid_constant__ MergeArgs a,
+                                                                float* __restrict__ x_g,
+                                                                int64_t begin, int64_t P, float eta) {
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
+  for (int64_t p = begin + static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; p < P; p += stride) {
+    const float x = x_g[p];
+    float acc = 0.f;
+    for (int k = 0; k < a.W; ++k) {
+      const float v = __ldcs(a.src[k] + p);
+      acc = fmaf(a.w[k], kReplica ? v - x : v, acc);
+    }
+    x_g[p] = fmaf(eta, acc, x);
+  }
+}
+
+int g_sm_count = 0;
+
+int sm_count() {
+  if (g_sm_count == 0) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&g_sm_count, cudaDevAttrMultiProcessorCount, dev);
+    if (g_sm_count <= 0) g_sm_count = 1;
+  }
+  return g_sm_count;
+}
+
+}  // namespace
+
+cudaError_t launch_merge(const MergeArgs& a, float* x_g, int64_t P, float eta, bool replica,
+                         cudaStream_t s) {
+  if (P <= 0) return cudaSuccess;
+  bool aligned = (reinterpret_cast<uintptr_t>(x_g) & 15) == 0;
+  for (int k = 0; k < a.W && aligned; ++k) aligned = (reinterpret_cast<uintptr_t>(a.src[k]) & 15) == 0;
+  const int ctas_per_sm = 2048 / kThreads;
+  const int64_t n4 = aligned ? P / 4 : 0;
+  if (n4 > 0) {
+    int64_t blocks = static_cast<int64_t>(sm_count()) * ctas_per_sm;
+    const int64_t need = (n4 + kThreads - 1) / kThreads;
+    if (need < blocks) blocks = need;
+    if (replica)
+      merge_vec4_kernel<true><<<static_cast<unsigned>(blocks), kThreads, 0, s>>>(a, x_g, n4, eta);
+    else
+      merge_vec4_kernel<false><<<static_cast<unsigned>(blocks), kThreads, 0, s>>>(a, x_g, n4, eta);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+  }
+  const int64_t begin = n4 * 4;
+  if (begin < P) {
+    int64_t blocks = static_cast<int64_t>(sm_count()) * ctas_per_sm;
+    const int64_t need = (P - begin + kThreads - 1) / kThreads;
+    if (need < blocks) blocks = need;
+    if (replica)
+      merge_scalar_kernel<true><<<static_cast<unsigned>(blocks), kThreads, 0, s>>>(a, x_g, begin, P, eta);
+    else
+      merge_scalar_kernel<false><<<static_cast<unsigned>(blocks), kThreads, 0, s>>>(a, x_g, begin, P, eta);
+    return cudaGetLastError();
+  }
+  return cudaSuccess;
+}
+
+}  // namespace oscars

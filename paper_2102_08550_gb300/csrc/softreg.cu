@@ -1,0 +1,169 @@
+// Local steps of softmax regression in fp32 (one linear layer + softmax
+// cross-entropy): Eq. 4, "otherwise" branch, x <- x - lr * g(x) with g the
+// mean mini-batch gradient.
+//
+// One CTA per worker runs the worker's whole round: it pulls the global
+// model into shared memory (the pull of the parameter-server description,
+// fused: nothing is copied through HBM), runs tau_i SGD steps on successive
+// mini-batches of its shard with the weights resident in shared memory, and
+// writes the result to the worker's replica (the push).  Workers never
+// exchange data inside a round, so the round is one launch.
+//
+// Per step: logits z[b][c] = sum_k x[b][k] W[c][k] + bias[c] (warp-level dot
+// products), p = softmax(z), loss_b = logsumexp(z_b) - z_b[y_b],
+// dz = (p - onehot(y)) / B, dW[c][k] = sum_b dz[b][c] x[b][k],
+// db[c] = sum_b dz[b][c], W <- W - lr dW (fmaf), all fp32.
+#include "common.cuh"
+#include "internal.h"
+
+namespace oscars {
+
+namespace {
+
+constexpr int kThreads = 512;
+constexpr int kWarps = kThreads / 32;
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+__global__ void __launch_bounds__(kThreads) softreg_round_kernel(const __grid_constant__ SoftregArgs a) {
+  extern __shared__ __align__(16) float sm[];
+  const int D = a.D, C = a.C, B = a.B;
+  float* Wsm = sm;                 // [C][D]
+  float* bsm = Wsm + C * D;        // [C] (padded to 32)
+  float* Xsm = bsm + 32;           // [B][D]
+  float* Zsm = Xsm + B * D;        // [B][C] logits, then dz
+  float* Lsm = Zsm + B * C;        // [B] per-sample loss
+  int* Ysm = reinterpret_cast<int*>(Lsm + B);  // [B]
+
+  const int w = blockIdx.x;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int tau = a.tau[w];
+  const float* gsrc = a.master + static_cast<int64_t>(a.global_slot) * a.slot_stride;
+  float* dst = a.master_out + static_cast<int64_t>(w) * a.slot_stride;
+
+  // pull: global model -> shared memory
+  for (int i = tid; i < C * D; i += kThreads) Wsm[i] = gsrc[a.offW + i];
+  for (int i = tid; i < C; i += kThreads) bsm[i] = gsrc[a.offB + i];
+
+  const float* X = a.shard_x[w];
+  const int32_t* Y = a.shard_y[w];
+  const int64_t n = a.shard_n[w];
+  const int64_t cur = a.cursor[w];
+  const float invB = 1.0f / static_cast<float>(B);
+
+  for (int s = 0; s < tau; ++s) {
+    __syncthreads();
+    // mini-batch rows (cursor + s*B + b) mod n
+    for (int i = tid; i < B * D; i += kThreads) {
+      const int b = i / D, k = i - b * D;
+      const int64_t r = (cur + static_cast<int64_t>(s) * B + b) % n;
+      Xsm[i] = X[r * D + k];
+    }
+    for (int b = tid; b < B; b += kThreads) Ysm[b] = Y[(cur + static_cast<int64_t>(s) * B + b) % n];
+    __syncthreads();
+    // logits: one warp per (b, c) dot product
+    for (int q = warp; q < B * C; q += kWarps) {
+      const int b = q / C, c = q - b * C;
+      const float* xr = Xsm + b * D;
+      const float* wr = Wsm + c * D;
+      float acc = 0.f;
+      for (int k = lane; k < D; k += 32) acc = fmaf(xr[k], wr[k], acc);
+      acc = warp_sum(acc);
+      if (lane == 0) Zsm[q] = acc + bsm[c];
+    }
+    __syncthreads();
+    // softmax cross-entropy, one thread per row
+    for (int b = tid; b < B; b += kThreads) {
+      float* z = Zsm + b * C;
+      float m = z[0];
+      for (int c = 1; c < C; ++c) m = fmaxf(m, z[c]);
+      float se = 0.f;
+      for (int c = 0; c < C; ++c) se += expf(z[c] - m);
+      const float lse = m + logf(se);
+      const int y = Ysm[b];
+      Lsm[b] = lse - z[y];
+      for (int c = 0; c < C; ++c) z[c] = (expf(z[c] - lse) - (c == y ? 1.f : 0.f)) * invB;
+    }
+    __syncthreads();
+    if (tid == 0) {
+      float l = 0.f;
+      for (int b = 0; b < B; ++b) l += Lsm[b];
+      a.loss_part[static_cast<int64_t>(w) * a.max_tau + s] = l;
+    }
+    // weight gradient and update, one thread per input feature k
+    for (int k = tid; k < D; k += kThreads) {
+      for (int c = 0; c < C; ++c) {
+        float g = 0.f;
+        for (int b = 0; b < B; ++b) g = fmaf(Zsm[b * C + c], Xsm[b * D + k], g);
+        Wsm[c * D + k] = fmaf(-a.lr, g, Wsm[c * D + k]);
+      }
+    }
+    for (int c = tid; c < C; c += kThreads) {
+      float g = 0.f;
+      for (int b = 0; b < B; ++b) g += Zsm[b * C + c];
+      bsm[c] = fmaf(-a.lr, g, bsm[c]);
+    }
+  }
+  __syncthreads();
+  // push: replica <- shared memory
+  for (int i = tid; i < C * D; i += kThreads) dst[a.offW + i] = Wsm[i];
+  for (int i = tid; i < C; i += kThreads) dst[a.offB + i] = bsm[i];
+}
+
+// Mean cross-entropy of the global model: one warp per sample, partial sums
+// per block (summed afterwards in a fixed order).
+__global__ void __launch_bounds__(256) softreg_eval_kernel(const __grid_constant__ SoftregEvalArgs a) {
+  __shared__ float part[8];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  float mine = 0.f;
+  for (int64_t i = static_cast<int64_t>(blockIdx.x) * 8 + warp; i < a.n; i += static_cast<int64_t>(gridDim.x) * 8) {
+    const float* xr = a.x + i * a.D;
+    float z[kMaxClasses];
+    for (int c = 0; c < a.C; ++c) {
+      const float* wr = a.master + a.offW + static_cast<int64_t>(c) * a.D;
+      float acc = 0.f;
+      for (int k = lane; k < a.D; k += 32) acc = fmaf(xr[k], wr[k], acc);
+      z[c] = warp_sum(acc) + a.master[a.offB + c];
+    }
+    float m = z[0];
+    for (int c = 1; c < a.C; ++c) m = fmaxf(m, z[c]);
+    float se = 0.f;
+    for (int c = 0; c < a.C; ++c) se += expf(z[c] - m);
+    mine += m + logf(se) - z[a.y[i]];
+  }
+  if (lane == 0) part[warp] = mine;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    float s = 0.f;
+    for (int i = 0; i < 8; ++i) s += part[i];
+    a.loss_sum[blockIdx.x] = s;
+  }
+}
+
+}  // namespace
+
+size_t softreg_smem_bytes(int D, int C, int B) {
+  return sizeof(float) * (static_cast<size_t>(C) * D + 32 + static_cast<size_t>(B) * D +
+                          static_cast<size_t>(B) * C + B) +
+         sizeof(int) * B;
+}
+
+cudaError_t launch_softreg_round(const SoftregArgs& a, int W, cudaStream_t s) {
+  const size_t smem = softreg_smem_bytes(a.D, a.C, a.B);
+  cudaError_t e = cudaFuncSetAttribute(softreg_round_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       static_cast<int>(smem));
+  if (e != cudaSuccess) return e;
+  softreg_round_kernel<<<W, kThreads, smem, s>>>(a);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_softreg_eval(const SoftregEvalArgs& a, int blocks, cudaStream_t s) {
+  softreg_eval_kernel<<<blocks, 256, 0, s>>>(a);
+  return cudaGetLastError();
+}
+
+}  // namespace oscars

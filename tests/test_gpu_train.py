@@ -1,0 +1,147 @@
+"""Local steps + merge + pull (Eq. 4, both branches) on the GPU against the
+oracle: schedules bit-exact, merged parameters within 1e-5 (max-abs,
+normalised per tensor), losses within 1e-3 relative.
+
+Cases: the fp32 softmax-regression workload at full size (all rounds), small
+bf16 MLPs that span several tiles, ragged K tails and a middle layer (the
+input-gradient GEMM), the 784-512-10 workload at full size for two rounds,
+and sampled workers of the 3072-1024-1024-10 workload at full size."""
+import dataclasses
+
+import numpy as np
+import pytest
+import torch
+
+import paper_2102_08550_gb300 as P
+import synth
+from oracle import bf16 as obf16
+from oracle import model as omodel
+from oracle import run as orun
+from tests.gpu_util import (LOSS_RTOL, PARAM_RTOL, device_shards, make_context, oracle_inputs, oracle_schedule,
+                            per_tensor_errors, pull_flat, rel_maxabs, replica_flat)
+
+pytestmark = pytest.mark.gpu
+
+
+def run_both(w, rounds, device, rows=None, flags=0, tau_override=None, eval_n=0, oracle_rows=None):
+    """``oracle_rows``: generate only the first rows of each shard for the
+    oracle (enough when the cursor does not wrap within ``rounds``)."""
+    rows = rows or w.samples_per_worker
+    shards_d = device_shards(w, device, n=rows)
+    ctx, layers0 = make_context(w, shards_d, device, flags=flags)
+    if tau_override is not None:
+        ctx.set_local_steps(tau_override)
+    gpu_losses, gpu_x = [], []
+    for _ in range(rounds):
+        tau, loss = ctx.local_steps()
+        ctx.push_merge()
+        gpu_losses.append(np.array(loss))
+        gpu_x.append(pull_flat(ctx, device))
+    shards_h = oracle_inputs(w, oracle_rows or rows)
+    t, T, mw, tau_o = oracle_schedule(w)
+    state, recs = orun.run(w.dims, layers0, shards_h, t_iter=t, M=w.M, rounds=rounds, batch=w.batch, lr=w.lr,
+                           bf16=w.bf16, server_lr=w.server_lr, tau_override=tau_override)
+    sch = ctx.schedule()
+    if tau_override is None:
+        assert sch["tau"] == tau_o.tolist()
+        assert sch["T_star"] == T and sch["max_wait"] == mw
+    assert sch["t_iter"] == t.tolist()
+    assert sch["clock"] == [rounds * sch["T_star"]] * w.num_workers
+    for r in range(rounds):
+        errs = per_tensor_errors(gpu_x[r], recs[r].x_g, w.dims)
+        assert max(errs) <= PARAM_RTOL, (r, errs)
+        np.testing.assert_allclose(gpu_losses[r], recs[r].worker_loss, rtol=LOSS_RTOL)
+    ev = None
+    if eval_n:
+        Xe, ye = synth.eval_np(w, n=eval_n)
+        ge = ctx.eval_loss(torch.from_numpy(Xe).to(device), torch.from_numpy(ye).to(device))
+        oe = omodel.loss_of(state.x_g, Xe, ye, obf16.round_bf16 if w.bf16 else obf16.identity)
+        assert abs(ge - oe) <= LOSS_RTOL * abs(oe), (ge, oe)
+        ev = (ge, oe)
+    ctx.close()
+    return ev
+
+
+def test_softmax_regression_full(cuda_device):
+    w = synth.CFG1
+    run_both(w, w.rounds, cuda_device, eval_n=w.eval_n)
+
+
+def test_softmax_regression_direct_launch(cuda_device):
+    run_both(dataclasses.replace(synth.CFG1, samples_per_worker=200), 3, cuda_device, flags=P.FLAG_NO_GRAPH)
+
+
+SMALL = [
+    # name, dims, W, batch, rows, M
+    ("2layer", [784, 512, 10], 4, 64, 512, 8),
+    ("3layer", [200, 256, 128, 10], 3, 32, 256, 6),       # ragged K tail, middle layer (input-gradient GEMM)
+    ("4layer", [96, 128, 256, 128, 10], 5, 128, 512, 4),
+]
+
+
+@pytest.mark.parametrize("name,dims,W,B,rows,M", SMALL, ids=[s[0] for s in SMALL])
+def test_mlp_small(cuda_device, name, dims, W, B, rows, M):
+    w = synth.TrainWorkload(f"small-{name}", W, dims, B, 0.05, rows, M, 3)
+    run_both(w, 3, cuda_device, rows=rows, eval_n=4 * B)
+
+
+def test_mlp_bsp_override(cuda_device):
+    w = synth.TrainWorkload("small-bsp", 4, [128, 128, 10], 32, 0.1, 128, 4, 2)
+    run_both(w, 2, cuda_device, tau_override=[1, 1, 1, 1])
+
+
+def test_mlp_direct_launch_matches_graph(cuda_device):
+    w = synth.TrainWorkload("small-direct", 3, [256, 128, 10], 64, 0.05, 256, 8, 2)
+    run_both(w, 2, cuda_device, flags=P.FLAG_NO_GRAPH)
+
+
+def test_mlp_784_512_10_w16_full(cuda_device):
+    w = synth.CFG2
+    _, _, _, tau = oracle_schedule(w)
+    need = 2 * int(tau.max()) * w.batch
+    assert need < w.samples_per_worker          # no wrap: a prefix of each shard suffices
+    run_both(w, 2, cuda_device, eval_n=2048, oracle_rows=need + w.batch)
+
+
+def test_mlp_3072_1024_1024_10_w32_sampled_workers(cuda_device):
+    """Full size, one round: the schedule and the local steps of the slowest
+    and the fastest worker (oracle run per worker) before the merge."""
+    w = synth.CFG3
+    shards_d = device_shards(w, cuda_device)
+    ctx, layers0 = make_context(w, shards_d, cuda_device)
+    t, T, mw, tau = oracle_schedule(w)
+    tau_g, loss_g = ctx.local_steps()
+    assert tau_g == tau.tolist()
+    picks = sorted({int(np.argmin(tau)), int(np.argmax(tau))})
+    rows = int(tau.max()) * w.batch
+    for k in picks:
+        got = replica_flat(ctx, k, cuda_device)
+        state = orun.init_state(w.dims, layers0, t, w.M)
+        Xk, yk = synth.shard_np(w, k, n=rows)
+        layers, loss = orun.local_steps(state, k, (Xk, yk), w.batch, w.lr, obf16.round_bf16)
+        errs = per_tensor_errors(got, orun.flatten(layers), w.dims)
+        assert max(errs) <= PARAM_RTOL, (k, int(tau[k]), errs)
+        assert abs(loss_g[k] - loss) <= LOSS_RTOL * abs(loss)
+    ctx.push_merge()
+    ctx.close()
+
+
+def test_protocol_errors(cuda_device):
+    w = synth.TrainWorkload("small-proto", 2, [128, 128, 10], 32, 0.05, 64, 4, 1)
+    ctx, _ = make_context(w, device_shards(w, cuda_device, n=64), cuda_device)
+    with pytest.raises(P.OscarsError) as e:
+        ctx.push_merge()                         # nothing pushed yet
+    assert e.value.status == P.OSCARS_ESTATE
+    ctx.local_steps()
+    with pytest.raises(P.OscarsError) as e:
+        ctx.local_steps()                        # previous round not merged
+    assert e.value.status == P.OSCARS_ESTATE
+    with pytest.raises(P.OscarsError) as e:
+        ctx.set_local_steps([1, 1])
+    assert e.value.status == P.OSCARS_ESTATE
+    ctx.push_merge()
+    ctx.pull(None)                               # explicit broadcast pull
+    x = pull_flat(ctx, cuda_device)
+    for k in range(2):
+        np.testing.assert_array_equal(replica_flat(ctx, k, cuda_device), x)
+    ctx.close()
