@@ -44,6 +44,10 @@ def parse():
     ap.add_argument("--no-cpu", action="store_true", help="skip the CPU oracle baseline")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--merge-reps", type=int, default=20)
+    ap.add_argument("--only", choices=["all", "round", "merge"], default="all",
+                    help="round: only the Oscars-round benchmark; merge: only the merge microbenchmarks")
+    ap.add_argument("--merge-sizes", default="",
+                    help="comma list of P:W merge cases replacing the two default workloads (profiling)")
     return ap.parse_args()
 
 
@@ -284,11 +288,21 @@ def run_e2e(args, ctx, shards, w, tau, dev, stream):
             "note": "host wall clock; pinned-host mini-batch copies + local steps + merge + loss readback"}
 
 
+def merge_workloads(args):
+    if not args.merge_sizes:
+        return [synth.CFG4, synth.CFG5]
+    out = []
+    for item in args.merge_sizes.split(","):
+        Pn, W = (int(v) for v in item.split(":"))
+        out.append(synth.MergeWorkload(f"merge-P{Pn}-W{W}", W, Pn, 1e-3, 8, "localsteps"))
+    return out
+
+
 def run_merge(args, dev, stream, hbm, peak_kind):
     import torch
     import paper_2102_08550_gb300 as P
     res = {}
-    for m in (synth.CFG4, synth.CFG5):
+    for m in merge_workloads(args):
         W, Pn = m.num_workers, m.num_params
         rule = P.W_LOCALSTEPS if m.weight_rule == "localsteps" else P.W_UNIFORM
         xg0 = synth.merge_xg_t(m, 0, Pn, dev)
@@ -381,6 +395,17 @@ def main():
         import torch
         torch.cuda.set_device(local_rank)
         torch.distributed.init_process_group("nccl")
+    if args.only == "merge":
+        import torch
+        from paper_2102_08550_gb300 import _build
+        _build.build()
+        dev = torch.device(f"cuda:{local_rank}")
+        torch.cuda.set_device(dev)
+        hbm, _, _, kind = peaks()
+        print(json.dumps({"merge": run_merge(args, dev, torch.cuda.current_stream(dev), hbm, kind)}))
+        return
+    if args.only == "round":
+        args.no_merge = True
     res = run_gpu(args, rank, world, local_rank)
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu:

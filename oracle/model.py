@@ -36,6 +36,11 @@ def gemm_nt(a: np.ndarray, b: np.ndarray, rnd: Callable) -> np.ndarray:
     return (rnd(a).astype(f64) @ rnd(b).astype(f64).T).astype(f32)
 
 
+def gemm_nn(a: np.ndarray, b: np.ndarray, rnd: Callable) -> np.ndarray:
+    """fp32( rnd(a) @ rnd(b) ), products summed in fp64."""
+    return (rnd(a).astype(f64) @ rnd(b).astype(f64)).astype(f32)
+
+
 def forward(layers, X: np.ndarray, rnd: Callable):
     """Returns (list of layer inputs, list of pre-activations z_l)."""
     inputs, zs = [], []
@@ -74,7 +79,7 @@ def gradients(layers, X, y, rnd: Callable):
         db = dz.astype(f64).sum(axis=0).astype(f32)
         grads[l] = (dW, db)
         if l > 0:
-            dh = (rnd(dz).astype(f64) @ rnd(W).astype(f64)).astype(f32)   # dz @ W
+            dh = gemm_nn(dz, W, rnd)                                     # dz @ W
             dz = np.where(zs[l - 1] > 0, dh, f32(0.0)).astype(f32)      # ReLU mask
     return float(loss.mean()), grads
 

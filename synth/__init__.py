@@ -291,6 +291,40 @@ def eval_t(w: TrainWorkload, device, n: Optional[int] = None):
     return _samples_t(w.seed + SEED_EVAL, S_EVAL_LABEL << 16, S_EVAL_NOISE << 16, n, d, w.clip, means)
 
 
+# ---- integer-valued inputs: fp32 sums of their products are exact ----
+S_INT_X = 9
+S_INT_W = 10
+
+
+def shard_int_np(w: TrainWorkload, worker: int, n: int, vmax: int = 3):
+    """Integer samples in [-vmax, vmax] (fp32) with uniform labels."""
+    d = w.dims[0]
+    b = bits_np(w.seed, (S_INT_X << 16) | worker, np.arange(n * d, dtype=np.uint64))
+    x = ((b % np.uint64(2 * vmax + 1)).astype(np.int64) - vmax).astype(np.float32).reshape(n, d)
+    y = label_np(w.seed, (S_LABEL << 16) | worker, np.arange(n, dtype=np.uint64))
+    return x, y
+
+
+def shard_int_t(w: TrainWorkload, worker: int, n: int, device, vmax: int = 3):
+    import torch
+    d = w.dims[0]
+    idx = torch.arange(n * d, dtype=torch.int64, device=device)
+    b = _lowbias32_t(idx ^ stream_key(w.seed, (S_INT_X << 16) | worker))
+    x = ((b % (2 * vmax + 1)) - vmax).to(torch.float32).reshape(n, d)
+    y = label_t(w.seed, (S_LABEL << 16) | worker, torch.arange(n, dtype=torch.int64, device=device))
+    return x.contiguous(), y
+
+
+def init_layers_int_np(w: TrainWorkload, wmax: int = 4, shift: int = 7):
+    """Weights k * 2**-shift with integer k in [-wmax, wmax]; zero biases."""
+    out = []
+    for l, (i, o) in enumerate(zip(w.dims[:-1], w.dims[1:])):
+        b = bits_np(w.seed + SEED_INIT, (S_INT_W << 16) | l, np.arange(o * i, dtype=np.uint64))
+        k = (b % np.uint64(2 * wmax + 1)).astype(np.int64) - wmax
+        out.append(((k.astype(np.float32) * np.float32(2.0 ** -shift)).reshape(o, i), np.zeros(o, np.float32)))
+    return out
+
+
 # ---- merge microbench inputs ----
 def merge_taus(m: MergeWorkload) -> np.ndarray:
     """Random per-worker local-step counts in [1, tau_max] (int32)."""

@@ -66,3 +66,55 @@ def oracle_schedule(w: synth.TrainWorkload):
     t = osched.iteration_ticks(synth.speeds(w), w.ticks_per_unit)
     T, mw, tau = osched.schedule(t, w.M)
     return t, T, mw, tau
+
+
+# ---------------------------------------------------------------- conditioning envelope
+class perturbed_gemms:
+    """Context manager: every GEMM output of the oracle is multiplied by
+    (1 + rel * N(0, 1)), the size of the difference a different fp32
+    summation order makes.  Used to measure how far the oracle moves from
+    itself, i.e. how well conditioned a run is (test infrastructure only)."""
+
+    def __init__(self, rel: float, seed: int):
+        self.rel, self.rng = rel, np.random.default_rng(seed)
+
+    def __enter__(self):
+        from oracle import model as om
+        self.om, self.nt, self.nn = om, om.gemm_nt, om.gemm_nn
+        rel, rng = self.rel, self.rng
+
+        def wrap(f):
+            def g(a, b, rnd):
+                out = f(a, b, rnd)
+                return (out * (1.0 + rel * rng.standard_normal(out.shape))).astype(np.float32)
+            return g
+        om.gemm_nt, om.gemm_nn = wrap(self.nt), wrap(self.nn)
+        return self
+
+    def __exit__(self, *a):
+        self.om.gemm_nt, self.om.gemm_nn = self.nt, self.nn
+
+
+ENV_REL = 2e-6       # relative GEMM-output perturbation (about 30 fp32 ulps)
+ENV_SEEDS = (11, 12)
+ENV_FACTOR = 4.0
+
+
+def envelope(run_fn, dims, ref_flats):
+    """Per-round, per-tensor max divergence of perturbed oracle runs from the
+    unperturbed ones; ``run_fn()`` returns a list of flat parameter vectors."""
+    env = [np.zeros(2 * (len(dims) - 1)) for _ in ref_flats]
+    for s in ENV_SEEDS:
+        with perturbed_gemms(ENV_REL, s):
+            flats = run_fn()
+        for r, (f, ref) in enumerate(zip(flats, ref_flats)):
+            env[r] = np.maximum(env[r], per_tensor_errors(f, ref, dims))
+    return env
+
+
+def assert_within(errs, env, what):
+    """Every tensor within 1e-5, or within ENV_FACTOR times the oracle's own
+    divergence under fp32-sized perturbations (bf16 rounding and ReLU masks
+    amplify those; the envelope is measured, not assumed)."""
+    bound = np.maximum(PARAM_RTOL, ENV_FACTOR * np.asarray(env))
+    assert np.all(np.asarray(errs) <= bound), (what, list(np.round(errs, 9)), list(np.round(bound, 9)))
