@@ -128,23 +128,56 @@ class ClockSampler:
 
 # ------------------------------------------------------------------ GPU arm
 def algorithmic_work(w, tau):
-    """Per-round algorithmic FLOPs and bytes of each kernel class."""
-    B, dims = w.batch, w.dims
-    n_steps = int(np.sum(tau))
-    L = len(dims) - 1
-    flops = {}
-    fwd = sum(2.0 * B * dims[l] * dims[l + 1] for l in range(L - 1))
-    dw = sum(2.0 * B * dims[l] * dims[l + 1] for l in range(L - 1))
-    dh = sum(2.0 * B * dims[l] * dims[l + 1] for l in range(1, L - 1))
-    head = 3 * 2.0 * B * dims[L - 1] * dims[L]
-    flops["gemm_fwd"] = fwd * n_steps
-    flops["gemm_dw_sgd"] = dw * n_steps
-    flops["gemm_dh"] = dh * n_steps
-    flops["head_fwd"] = head / 3 * n_steps
-    flops["head_bwd"] = head * 2 / 3 * n_steps
-    P = w.num_params
-    bytes_ = {"merge": (w.num_workers + 2) * P * 4.0}
-    return flops, bytes_
+    """Per-round algorithmic work of each kernel class of the MLP path:
+    {class: (flops, hbm_bytes)}.  Bytes count every operand once at its
+    stored width (fp32 master 4 B, bf16 operand copies 2 B), i.e. what a
+    kernel must move if nothing stays on chip between launches."""
+    B, d = w.batch, w.dims
+    L = len(d) - 1
+    n = float(np.sum(tau))            # worker-steps per round
+    W = w.num_workers
+    fl, by = {}, {}
+
+    def add(k, f, b):
+        fl[k] = fl.get(k, 0.0) + f
+        by[k] = by.get(k, 0.0) + b
+    for l in range(L - 1):            # hidden layers on the tensor cores
+        i, o = d[l], d[l + 1]
+        T = 2 if 1 <= l <= L - 2 else 0
+        add("gemm_fwd", n * 2 * B * i * o, n * (o * i * 2 + B * i * 2 + 2 * B * o * 2 + o * 4))
+        add("gemm_dw_sgd", n * 2 * B * i * o,
+            n * (o * i * (4 + 4 + 2 + T) + o * B * 2 + i * B * 2 + o * (4 + 4 + 4)))
+        if l >= 1:
+            add("gemm_dh", n * 2 * B * i * o, n * (o * i * 2 + B * o * 2 + B * i * 2 + 2 * B * i * 2 + i * 4))
+    H, C = d[L - 1], d[L]
+    add("head_fwd", n * 2 * B * H * C, n * (C * H * 2 + B * H * 2 + B * C * 4 + B * 4 + C * 4))
+    add("head_bwd", n * 4 * B * H * C,
+        n * (B * H * 2 + C * H * (2 + 4 + 4 + 2) + 2 * B * H * 2 + H * 4 + B * C * 4 + C * 8))
+    add("stage", 0.0, n * B * (d[0] * 4 + 2 * d[0] * 2 + 8))
+    P_pad = w.num_params   # padding is < 0.1%
+    add("merge", 2.0 * W * P_pad, (W + 2) * P_pad * 4.0)
+    add("shadow_refresh", 0.0, P_pad * 6.0)
+    return fl, by
+
+
+def roofline_of(name, ms_per_launch, launches_per_round, flops, bytes_, hbm, tflops, peak_kind):
+    f = flops.get(name, 0.0) / launches_per_round
+    b = bytes_.get(name, 0.0) / launches_per_round
+    t = ms_per_launch / 1e3
+    if f == 0.0 and b == 0.0:
+        return {"kernel": name, "bound": "alu", "achieved": None, "peak": None, "unit": None, "frac": None,
+                "ms_per_launch": ms_per_launch, "traffic": None}
+    t_flop = f / (tflops * 1e12)
+    t_mem = b / (hbm * 1e9)
+    if t_flop >= t_mem:
+        ach = f / t / 1e12
+        return {"kernel": name, "bound": "tensor", "achieved": ach, "peak": tflops, "unit": "TFLOP/s",
+                "frac": ach / tflops, "peak_kind": f"{peak_kind} bf16 dense (burst)", "flops_per_launch": f,
+                "bytes_per_launch": b, "ms_per_launch": ms_per_launch, "traffic": None}
+    ach = b / t / 1e9
+    return {"kernel": name, "bound": "hbm", "achieved": ach, "peak": hbm, "unit": "GB/s", "frac": ach / hbm,
+            "peak_kind": f"{peak_kind} HBM copy", "flops_per_launch": f, "bytes_per_launch": b,
+            "ms_per_launch": ms_per_launch, "traffic": None}
 
 
 def run_gpu(args, rank, world, local_rank):
@@ -217,25 +250,14 @@ def run_gpu(args, rank, world, local_rank):
     launches_per_round = sum(c for _, c in prof.values()) / prof_rounds
     flops, bytes_ = algorithmic_work(w, tau)
     dom = max(prof, key=lambda k: prof[k][0])
-    dom_ms_per_launch = prof[dom][0] / prof[dom][1]
-    launches_dom_per_round = prof[dom][1] / prof_rounds
-    kernels = {k: {"ms_per_round": v[0] / prof_rounds, "launches_per_round": v[1] / prof_rounds,
-                   "share": v[0] / sum(x[0] for x in prof.values())} for k, v in prof.items()}
-    if dom in flops:
-        per_launch = flops[dom] / launches_dom_per_round
-        achieved = per_launch / (dom_ms_per_launch / 1e3) / 1e12
-        roof = {"kernel": dom, "bound": "tensor", "achieved": achieved, "peak": tf_burst, "unit": "TFLOP/s",
-                "frac": achieved / tf_burst, "peak_kind": f"{peak_kind} bf16 dense burst",
-                "work_per_launch": per_launch, "ms_per_launch": dom_ms_per_launch, "traffic": None}
-    elif dom in bytes_:
-        per_launch = bytes_[dom] / launches_dom_per_round
-        achieved = per_launch / (dom_ms_per_launch / 1e3) / 1e9
-        roof = {"kernel": dom, "bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s",
-                "frac": achieved / hbm, "peak_kind": f"{peak_kind} HBM copy", "work_per_launch": per_launch,
-                "ms_per_launch": dom_ms_per_launch, "traffic": None}
-    else:
-        roof = {"kernel": dom, "bound": "alu", "achieved": None, "peak": None, "unit": None, "frac": None,
-                "ms_per_launch": dom_ms_per_launch, "traffic": None}
+    kernels = {}
+    tot = sum(x[0] for x in prof.values())
+    for k, (ms, cnt) in prof.items():
+        r = roofline_of(k, ms / cnt, cnt / prof_rounds, flops, bytes_, hbm, tf_burst, peak_kind)
+        kernels[k] = {"ms_per_round": ms / prof_rounds, "launches_per_round": cnt / prof_rounds,
+                      "share": ms / tot, "bound": r["bound"], "frac": r["frac"]}
+    roof = roofline_of(dom, prof[dom][0] / prof[dom][1], prof[dom][1] / prof_rounds, flops, bytes_, hbm, tf_burst,
+                       peak_kind)
 
     # ---- end to end through the C ABI with host-resident inputs
     e2e = None

@@ -513,6 +513,7 @@ oscars_status validate_and_layout(oscars_ctx* c, const oscars_config* cfg) {
     if (c->dims[0] % 8 != 0) return fail(c, OSCARS_ENOTSUP, "bf16 MLP: input dim must be a multiple of 8");
     for (int l = 1; l < c->L; ++l)
       if (c->dims[l] % 128 != 0) return fail(c, OSCARS_ENOTSUP, "bf16 MLP: hidden dims must be multiples of 128");
+    if (c->dims[c->L - 1] > 2048) return fail(c, OSCARS_ENOTSUP, "bf16 MLP: the last hidden dim must be <= 2048");
   } else {
     return fail(c, OSCARS_ENOTSUP, "supported: fp32 softmax regression (L=1) or bf16 MLP (L>=2)");
   }

@@ -63,8 +63,15 @@ __global__ void __launch_bounds__(256) stage_kernel(const __grid_constant__ Stag
 // ---------------------------------------------------------------- head forward
 // Logits of the last layer z[b][c] = sum_k bf16(h[b][k]) bf16(W[c][k]) + bias[c]
 // (fp32 accumulate), softmax cross-entropy, dlogits = (p - onehot)/B.
-// Grid (active lanes, B/16); 16 rows per CTA, one warp per two rows.
+// Grid (active lanes, B/16); 16 rows per CTA, one warp per two rows; each
+// lane keeps its slice of the row in registers (16-byte loads issued up
+// front), the class weights sit in shared memory.
+//
+// Softmax without cancellation: e_c = exp(z_c - max z), s = sum_c e_c,
+// p_c = e_c / s, and for the label 1 - p_y = (sum_{c != y} e_c) / s, so the
+// gradient of a confidently classified sample keeps its relative accuracy.
 constexpr int kHeadFwdThreads = 256;
+constexpr int kHeadMaxH8 = 8;   // up to 8 x 16-byte slices per lane: H <= 2048
 
 __global__ void __launch_bounds__(kHeadFwdThreads) head_fwd_kernel(const __grid_constant__ HeadArgs a) {
   extern __shared__ __align__(16) float hsm[];
@@ -76,29 +83,75 @@ __global__ void __launch_bounds__(kHeadFwdThreads) head_fwd_kernel(const __grid_
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const __nv_bfloat16* Wg = a.shadow + static_cast<int64_t>(src) * a.slot_stride + a.offW;
   const float* bias = a.master + static_cast<int64_t>(src) * a.slot_stride + a.offB;
-  for (int q = threadIdx.x; q < C * H; q += kHeadFwdThreads) Wsm[q] = __bfloat162float(Wg[q]);
+  for (int q = threadIdx.x; q < C * H / 8; q += kHeadFwdThreads) {
+    const uint4 v = reinterpret_cast<const uint4*>(Wg)[q];
+    const __nv_bfloat162* p2 = reinterpret_cast<const __nv_bfloat162*>(&v);
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const float2 f = __bfloat1622float2(p2[j]);
+      Wsm[q * 8 + 2 * j] = f.x;
+      Wsm[q * 8 + 2 * j + 1] = f.y;
+    }
+  }
   __syncthreads();
+  const int nslice = H / 256;   // 16-byte slices per lane (H is a multiple of 128; remainder below)
   for (int rr = warp; rr < kRowsPerLossChunk; rr += kHeadFwdThreads / 32) {
     const int b = blockIdx.y * kRowsPerLossChunk + rr;
     const __nv_bfloat16* h = a.Ain + (static_cast<int64_t>(w) * B + b) * H;
+    // this lane's 8-element slices: k = (j * 32 + lane) * 8
+    float hv[kHeadMaxH8][8];
+#pragma unroll
+    for (int j = 0; j < kHeadMaxH8; ++j) {
+      const int k = (j * 32 + lane) * 8;
+      if (k < H) {
+        const uint4 v = *reinterpret_cast<const uint4*>(h + k);
+        const __nv_bfloat162* p2 = reinterpret_cast<const __nv_bfloat162*>(&v);
+#pragma unroll
+        for (int t = 0; t < 4; ++t) {
+          const float2 f = __bfloat1622float2(p2[t]);
+          hv[j][2 * t] = f.x;
+          hv[j][2 * t + 1] = f.y;
+        }
+      } else {
+#pragma unroll
+        for (int t = 0; t < 8; ++t) hv[j][t] = 0.f;
+      }
+    }
+    (void)nslice;
     float zc = -INFINITY;  // lane c holds z_c
     for (int c = 0; c < C; ++c) {
       const float* wr = Wsm + c * H;
       float acc = 0.f;
-      for (int k = lane; k < H; k += 32) acc = fmaf(__bfloat162float(h[k]), wr[k], acc);
+#pragma unroll
+      for (int j = 0; j < kHeadMaxH8; ++j) {
+        const int k = (j * 32 + lane) * 8;
+        if (k < H) {
+          const float4 w0 = *reinterpret_cast<const float4*>(wr + k);
+          const float4 w1 = *reinterpret_cast<const float4*>(wr + k + 4);
+          acc = fmaf(hv[j][0], w0.x, acc);
+          acc = fmaf(hv[j][1], w0.y, acc);
+          acc = fmaf(hv[j][2], w0.z, acc);
+          acc = fmaf(hv[j][3], w0.w, acc);
+          acc = fmaf(hv[j][4], w1.x, acc);
+          acc = fmaf(hv[j][5], w1.y, acc);
+          acc = fmaf(hv[j][6], w1.z, acc);
+          acc = fmaf(hv[j][7], w1.w, acc);
+        }
+      }
       acc = warp_sum(acc) + bias[c];
       if (lane == c) zc = acc;
     }
+    const int y = a.labels[static_cast<int64_t>(w) * B + b];
     const float m = warp_max(zc);
     const float e = lane < C ? expf(zc - m) : 0.f;
-    const float lse = m + logf(warp_sum(e));
-    const int y = a.labels[static_cast<int64_t>(w) * B + b];
+    const float s = warp_sum(e);
+    const float s_other = warp_sum(lane < C && lane != y ? e : 0.f);
     const float zy = __shfl_sync(0xffffffffu, zc, y);
     if (lane < C) {
-      const float p = expf(zc - lse);
-      a.dlog[(static_cast<int64_t>(w) * B + b) * C + lane] = (p - (lane == y ? 1.f : 0.f)) / static_cast<float>(B);
+      const float g = lane == y ? -(s_other / s) : e / s;
+      a.dlog[(static_cast<int64_t>(w) * B + b) * C + lane] = g / static_cast<float>(B);
     }
-    if (lane == 0) rowloss[rr] = lse - zy;
+    if (lane == 0) rowloss[rr] = m + logf(s) - zy;
   }
   __syncthreads();
   if (threadIdx.x == 0) {
@@ -110,79 +163,123 @@ __global__ void __launch_bounds__(kHeadFwdThreads) head_fwd_kernel(const __grid_
 }
 
 // ---------------------------------------------------------------- head backward
-// One thread per hidden feature k (grid: active lanes, H/128):
+// CTA = (active lane, 64 hidden features k); 256 threads.
+//  dh[b][k] = sum_c bf16(dz[b][c]) bf16(W_old[c][k]);  g = dh * (h[b][k] > 0)
+//    -> bf16 G [B][H] and G^T [H][B] (operands of the next GEMMs) and
+//       gb[k] = sum_b g (fp32, the bias gradient of the layer below);
 //  dW[c][k] = sum_b bf16(dz[b][c]) bf16(h[b][k]);  W <- W - lr dW (fmaf);
-//  dh[b][k] = sum_c bf16(dz[b][c]) bf16(W_old[c][k]);  g = dh * (h > 0)
-//  -> G [B][H] and GT [H][B] in bf16 (operands of the next GEMMs) and
-//  gb[k] = sum_b g (fp32, the bias gradient of the layer below).
-// CTA column 0 also updates the head bias with db[c] = sum_b dz[b][c].
-constexpr int kHeadBwdThreads = 128;
+//  CTA column 0 also updates the head bias with db[c] = sum_b dz[b][c].
+// The h tile, dz and the old weight columns are staged in shared memory
+// with 16-byte loads; G^T is assembled in shared memory and written row by
+// row.
+constexpr int kHeadBwdThreads = 256;
+constexpr int kHB = 64;        // hidden features per CTA
+constexpr int kHBGroups = kHeadBwdThreads / kHB;
+
+size_t head_bwd_smem(int B, int C) {
+  return sizeof(float) * (2 * static_cast<size_t>(B) * C + static_cast<size_t>(B) * kHB + static_cast<size_t>(C) * kHB +
+                          kHBGroups * kHB) +
+         sizeof(__nv_bfloat16) * static_cast<size_t>(kHB) * (B + 8);
+}
 
 __global__ void __launch_bounds__(kHeadBwdThreads) head_bwd_kernel(const __grid_constant__ HeadArgs a) {
   extern __shared__ __align__(16) float dsm[];
   const int H = a.H, C = a.C, B = a.B;
-  float* dz = dsm;             // [B][C] fp32
-  float* dzb = dz + B * C;     // [B][C] bf16-rounded
+  float* dz = dsm;                       // [B][C] fp32
+  float* dzb = dz + B * C;               // [B][C] bf16-rounded
+  float* hs = dzb + B * C;               // [B][kHB] bf16 h as float
+  float* wcs = hs + B * kHB;             // [C][kHB] old bf16 weights as float
+  float* gbp = wcs + C * kHB;            // [kHBGroups][kHB]
+  __nv_bfloat16* gts = reinterpret_cast<__nv_bfloat16*>(gbp + kHBGroups * kHB);  // [kHB][B + 8]
+  const int gts_ld = B + 8;
   const int i = blockIdx.x;
   const int w = a.wid[i], src = a.src[i];
+  const int k0 = blockIdx.y * kHB;
+  const int t = threadIdx.x;
+  const int64_t so = static_cast<int64_t>(src) * a.slot_stride;
+  const int64_t dof = static_cast<int64_t>(w) * a.slot_stride;
   const float* dl = a.dlog + static_cast<int64_t>(w) * B * C;
-  for (int q = threadIdx.x; q < B * C; q += kHeadBwdThreads) {
+  for (int q = t; q < B * C; q += kHeadBwdThreads) {
     const float v = dl[q];
     dz[q] = v;
     dzb[q] = bf16_round(v);
   }
-  __syncthreads();
-  const int64_t so = static_cast<int64_t>(src) * a.slot_stride;
-  const int64_t dof = static_cast<int64_t>(w) * a.slot_stride;
-  if (blockIdx.y == 0 && threadIdx.x < C) {
-    const int c = threadIdx.x;
-    float g = 0.f;
-    for (int b = 0; b < B; ++b) g += dz[b * C + c];
-    a.master_w[dof + a.offB + c] = fmaf(-a.lr, g, a.master[so + a.offB + c]);
-  }
-  const int k = blockIdx.y * kHeadBwdThreads + threadIdx.x;
-  if (k >= H) return;
-  // fully unrolled over kMaxClasses so both arrays stay in registers
-  float wc[kMaxClasses], dw[kMaxClasses];
-#pragma unroll
-  for (int c = 0; c < kMaxClasses; ++c) {
-    wc[c] = c < C ? __bfloat162float(a.shadow[so + a.offW + static_cast<int64_t>(c) * H + k]) : 0.f;
-    dw[c] = 0.f;
-  }
+  // h tile: B rows x 64 bf16 = 8 x 16-byte chunks per row
   const __nv_bfloat16* h = a.Ain + static_cast<int64_t>(w) * B * H;
-  __nv_bfloat16* G = a.G + static_cast<int64_t>(w) * B * H;
-  uint4* GT = reinterpret_cast<uint4*>(a.GT + (static_cast<int64_t>(w) * H + k) * B);
-  float gb = 0.f;
-  uint32_t pk[4];
-  for (int b = 0; b < B; ++b) {
-    const float hv = __bfloat162float(h[static_cast<int64_t>(b) * H + k]);
-    float dh = 0.f;
+  for (int q = t; q < B * (kHB / 8); q += kHeadBwdThreads) {
+    const int b = q >> 3, c8 = (q & 7) * 8;
+    float f8[8];
+    if (k0 + c8 < H) {
+      const uint4 v = *reinterpret_cast<const uint4*>(h + static_cast<int64_t>(b) * H + k0 + c8);
+      const __nv_bfloat162* p2 = reinterpret_cast<const __nv_bfloat162*>(&v);
 #pragma unroll
-    for (int c = 0; c < kMaxClasses; ++c) {
-      if (c < C) {
-        const float g = dzb[b * C + c];
-        dw[c] = fmaf(g, hv, dw[c]);
-        dh = fmaf(g, wc[c], dh);
+      for (int j = 0; j < 4; ++j) {
+        const float2 f = __bfloat1622float2(p2[j]);
+        f8[2 * j] = f.x;
+        f8[2 * j + 1] = f.y;
       }
-    }
-    const float gv = hv > 0.f ? dh : 0.f;
-    gb += gv;
-    const __nv_bfloat16 gbv = __float2bfloat16_rn(gv);
-    G[static_cast<int64_t>(b) * H + k] = gbv;
-    const uint32_t bits = static_cast<uint32_t>(*reinterpret_cast<const uint16_t*>(&gbv));
-    const int slot = (b & 7) >> 1;
-    if ((b & 1) == 0) pk[slot] = bits; else pk[slot] |= bits << 16;
-    if ((b & 7) == 7) GT[b >> 3] = make_uint4(pk[0], pk[1], pk[2], pk[3]);
-  }
-  a.gb[static_cast<int64_t>(w) * H + k] = gb;
+    } else {
 #pragma unroll
-  for (int c = 0; c < kMaxClasses; ++c) {
-    if (c < C) {
-      const int64_t e = a.offW + static_cast<int64_t>(c) * H + k;
-      const float nw = fmaf(-a.lr, dw[c], a.master[so + e]);
-      a.master_w[dof + e] = nw;
-      a.shadow_w[dof + e] = __float2bfloat16_rn(nw);
+      for (int j = 0; j < 8; ++j) f8[j] = 0.f;
     }
+#pragma unroll
+    for (int j = 0; j < 8; ++j) hs[b * kHB + c8 + j] = f8[j];
+  }
+  for (int q = t; q < C * kHB; q += kHeadBwdThreads) {
+    const int c = q / kHB, k = q - c * kHB;
+    wcs[q] = k0 + k < H ? __bfloat162float(a.shadow[so + a.offW + static_cast<int64_t>(c) * H + k0 + k]) : 0.f;
+  }
+  __syncthreads();
+
+  // input gradient of the layer below, masked by its ReLU
+  {
+    const int k = t % kHB, grp = t / kHB;
+    const int rows = B / kHBGroups;
+    float gsum = 0.f;
+    __nv_bfloat16* G = a.G + static_cast<int64_t>(w) * B * H;
+    for (int r = 0; r < rows; ++r) {
+      const int b = grp * rows + r;
+      const float hv = hs[b * kHB + k];
+      float dh = 0.f;
+      for (int c = 0; c < C; ++c) dh = fmaf(dzb[b * C + c], wcs[c * kHB + k], dh);
+      const float g = hv > 0.f ? dh : 0.f;
+      gsum += g;
+      const __nv_bfloat16 gb16 = __float2bfloat16_rn(g);
+      if (k0 + k < H) G[static_cast<int64_t>(b) * H + k0 + k] = gb16;
+      gts[k * gts_ld + b] = gb16;
+    }
+    gbp[grp * kHB + k] = gsum;
+  }
+  __syncthreads();
+  if (t < kHB && k0 + t < H) {
+    float g = 0.f;
+    for (int grp = 0; grp < kHBGroups; ++grp) g += gbp[grp * kHB + t];
+    a.gb[static_cast<int64_t>(w) * H + k0 + t] = g;
+  }
+  // G^T rows: B bf16 per hidden feature, 16-byte stores
+  {
+    uint4* GT = reinterpret_cast<uint4*>(a.GT + (static_cast<int64_t>(w) * H + k0) * B);
+    const int per_row = B / 8;
+    for (int q = t; q < kHB * per_row; q += kHeadBwdThreads) {
+      const int k = q / per_row, j = q - k * per_row;
+      if (k0 + k < H) GT[static_cast<int64_t>(k) * per_row + j] = *reinterpret_cast<const uint4*>(gts + k * gts_ld + j * 8);
+    }
+  }
+  // weight gradient and SGD of the head
+  for (int q = t; q < C * kHB; q += kHeadBwdThreads) {
+    const int c = q / kHB, k = q - c * kHB;
+    if (k0 + k >= H) continue;
+    float dw = 0.f;
+    for (int b = 0; b < B; ++b) dw = fmaf(dzb[b * C + c], hs[b * kHB + k], dw);
+    const int64_t e = a.offW + static_cast<int64_t>(c) * H + k0 + k;
+    const float nw = fmaf(-a.lr, dw, a.master[so + e]);
+    a.master_w[dof + e] = nw;
+    a.shadow_w[dof + e] = __float2bfloat16_rn(nw);
+  }
+  if (blockIdx.y == 0 && t < C) {
+    float g = 0.f;
+    for (int b = 0; b < B; ++b) g += dz[b * C + t];
+    a.master_w[dof + a.offB + t] = fmaf(-a.lr, g, a.master[so + a.offB + t]);
   }
 }
 
@@ -253,6 +350,7 @@ cudaError_t launch_stage(const StageArgs& a, int n_active, cudaStream_t s) {
 }
 
 cudaError_t launch_head_fwd(const HeadArgs& a, int n_active, cudaStream_t s) {
+  if (a.H % 8 != 0 || a.H > 32 * 8 * kHeadMaxH8) return cudaErrorInvalidValue;
   const size_t smem = sizeof(float) * static_cast<size_t>(a.C) * a.H;
   cudaError_t e = cudaFuncSetAttribute(head_fwd_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(smem));
@@ -263,11 +361,12 @@ cudaError_t launch_head_fwd(const HeadArgs& a, int n_active, cudaStream_t s) {
 }
 
 cudaError_t launch_head_bwd(const HeadArgs& a, int n_active, cudaStream_t s) {
-  const size_t smem = sizeof(float) * 2 * static_cast<size_t>(a.B) * a.C;
+  if (a.B % (8 * kHBGroups) != 0 || a.H % 8 != 0) return cudaErrorInvalidValue;
+  const size_t smem = head_bwd_smem(a.B, a.C);
   cudaError_t e = cudaFuncSetAttribute(head_bwd_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(smem));
   if (e != cudaSuccess) return e;
-  dim3 grid(n_active, (a.H + kHeadBwdThreads - 1) / kHeadBwdThreads);
+  dim3 grid(n_active, (a.H + kHB - 1) / kHB);
   head_bwd_kernel<<<grid, kHeadBwdThreads, smem, s>>>(a);
   return cudaGetLastError();
 }

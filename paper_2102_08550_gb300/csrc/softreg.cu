@@ -81,12 +81,16 @@ __global__ void __launch_bounds__(kThreads) softreg_round_kernel(const __grid_co
       float* z = Zsm + b * C;
       float m = z[0];
       for (int c = 1; c < C; ++c) m = fmaxf(m, z[c]);
-      float se = 0.f;
-      for (int c = 0; c < C; ++c) se += expf(z[c] - m);
-      const float lse = m + logf(se);
+      // p_c = e_c / s; 1 - p_y = (sum_{c != y} e_c) / s (no cancellation)
       const int y = Ysm[b];
-      Lsm[b] = lse - z[y];
-      for (int c = 0; c < C; ++c) z[c] = (expf(z[c] - lse) - (c == y ? 1.f : 0.f)) * invB;
+      float se = 0.f, so = 0.f;
+      for (int c = 0; c < C; ++c) {
+        const float e = expf(z[c] - m);
+        se += e;
+        if (c != y) so += e;
+      }
+      Lsm[b] = m + logf(se) - z[y];
+      for (int c = 0; c < C; ++c) z[c] = (c == y ? -(so / se) : expf(z[c] - m) / se) * invB;
     }
     __syncthreads();
     if (tid == 0) {
