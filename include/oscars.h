@@ -259,6 +259,36 @@ oscars_status oscars_merge(float* x_g, const float* const* deltas, const float* 
 oscars_status oscars_gemm_bf16_nt(const void* A, const void* B, float* C, int32_t M, int32_t N, int32_t K,
                                   void* stream);
 
+/*
+ * oscars_softreg_steps_noalloc - one worker's tau local SGD steps of fp32
+ * softmax regression, like one worker of oscars_local_steps, for callers that
+ * cannot allocate device memory when they call: code recording a CUDA graph
+ * in global capture mode (where cudaMalloc is refused), hosts whose memory
+ * pool owns the whole GPU, and loops that cannot pay for cudaMalloc/cudaFree,
+ * which may synchronise the device.  The paper has no counterpart; this is a
+ * deployment convenience.  It allocates nothing: its scratch (argument tables
+ * and per-step loss partials) is a fixed 64 KB array inside the library that
+ * every GPU which loads the library keeps until the process exits.
+ *
+ * params_in / params_out: device, classes*dim + classes fp32 each, canonical
+ * layout (W [classes][dim], then b [classes]); they may be the same buffer.
+ * x: device [n][dim] fp32; y: device [n] int32 labels in [0, classes).
+ * Step s uses rows (cursor + s*batch + b) mod n, b < batch.
+ * loss_out: device, 1 float: the mean mini-batch loss over the tau steps.
+ * Ordered on `stream`.  1 <= tau <= 16320 (the scratch holds one loss
+ * partial per step); larger tau, classes outside [2, 32] or bad pointers give
+ * EINVAL, shapes whose weights plus one batch exceed shared memory ENOTSUP.
+ * The first call on a device looks up the scratch address (once per device);
+ * make that first call before any stream capture.  Every call shares the one
+ * scratch array and leaves its contents behind; each call writes all it reads
+ * first, so nothing needs clearing, but calls that overlap on the GPU (other
+ * streams, other threads) race on it.
+ */
+oscars_status oscars_softreg_steps_noalloc(const float* params_in, float* params_out, const float* x,
+                                           const int32_t* y, int64_t n, int64_t cursor, int32_t tau,
+                                           int32_t dim, int32_t classes, int32_t batch, float lr,
+                                           float* loss_out, void* stream);
+
 #ifdef __cplusplus
 }
 #endif

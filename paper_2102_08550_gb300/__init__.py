@@ -64,6 +64,8 @@ _SIGS = {
     "oscars_profile_read": (c_int32, [c_void_p, c_int32, POINTER(ctypes.c_char_p), POINTER(c_double),
                                       POINTER(c_int32)]),
     "oscars_profile_reset": (c_int32, [c_void_p]),
+    "oscars_softreg_steps_noalloc": (c_int32, [c_void_p, c_void_p, c_void_p, c_void_p, c_int64, c_int64, c_int32,
+                                               c_int32, c_int32, c_int32, c_float, c_void_p, c_void_p]),
     "oscars_merge": (c_int32, [c_void_p, POINTER(c_void_p), POINTER(c_float), c_int32, c_int64, c_float, c_void_p]),
 }
 
@@ -129,6 +131,14 @@ def oscars_merge(x_g_ptr: int, delta_ptrs: Sequence[int], w: Sequence[float], P:
     W = len(delta_ptrs)
     _check(lib().oscars_merge(c_void_p(x_g_ptr), _arr(c_void_p, delta_ptrs), _arr(c_float, w), W, P,
                               server_lr, c_void_p(stream or 0)))
+
+
+def oscars_softreg_steps_noalloc(params_in_ptr: int, params_out_ptr: int, x_ptr: int, y_ptr: int, n: int,
+                                 cursor: int, tau: int, dim: int, classes: int, batch: int, lr: float,
+                                 loss_out_ptr: int, stream: Optional[int] = None):
+    _check(lib().oscars_softreg_steps_noalloc(c_void_p(params_in_ptr), c_void_p(params_out_ptr), c_void_p(x_ptr),
+                                              c_void_p(y_ptr), n, cursor, tau, dim, classes, batch, lr,
+                                              c_void_p(loss_out_ptr), c_void_p(stream or 0)))
 
 
 def oscars_create(cfg: OscarsConfig) -> int:
