@@ -37,8 +37,15 @@ namespace {
 
 constexpr int BM = 128;
 constexpr int BK = 64;
-constexpr int kThreads = 128;
 constexpr int kABytes = BM * BK * 2;
+constexpr int kBarrierBytes = 256;          // mbarriers + TMEM address slot
+constexpr int kEpiTileFloats = 32 * 33;     // per-warp staging tile (padded rows)
+
+// Warps per CTA: the weight-gradient epilogue streams the fp32 master and
+// runs two warpgroups (each warp owns its TMEM lane quarter, the two groups
+// split the columns); the others use one warpgroup.
+template <int EPI>
+constexpr int warps_for() { return EPI == kEpiDw ? 8 : 4; }
 
 template <int BN>
 struct TileCfg {
@@ -91,48 +98,47 @@ __device__ __forceinline__ float epi_dh(const GemmArgs& a, int wid, int m, int n
   return gsum;
 }
 
-__device__ __forceinline__ void epi_dw(const GemmArgs& a, int wid, int src, int m, int n0,
-                                       const float (&v)[32]) {
-  const int64_t so = static_cast<int64_t>(src) * a.slot_stride + a.offW + static_cast<int64_t>(m) * a.N;
-  const int64_t dof = static_cast<int64_t>(wid) * a.slot_stride + a.offW + static_cast<int64_t>(m) * a.N;
-  float nw[32];
-  if (n0 + 32 <= a.N) {
-    const float4* s4 = reinterpret_cast<const float4*>(a.master + so + n0);
-    float4* d4 = reinterpret_cast<float4*>(a.master_w + dof + n0);
-    uint2* sh = reinterpret_cast<uint2*>(a.shadow + dof + n0);
+// Weight gradient + SGD for one 32 x 32 block: rows m_base .. m_base + 31
+// (thread `lane` holds row m_base + lane in v), columns n_base .. n_base + 31.
+// The block goes through a padded shared-memory tile so that the fp32
+// master read-modify-write and the bf16 shadow write move full lines (lane =
+// column), while the transposed shadow is written from the row layout
+// (lane = row, consecutive addresses).
+__device__ __forceinline__ void epi_dw_block(const GemmArgs& a, int wid, int src, int m_base, int n_base,
+                                             const float (&v)[32], float* T, int lane) {
 #pragma unroll
-    for (int q = 0; q < 8; ++q) {
-      const float4 o = s4[q];
-      float4 r;
-      r.x = fmaf(-a.lr, v[4 * q + 0], o.x);
-      r.y = fmaf(-a.lr, v[4 * q + 1], o.y);
-      r.z = fmaf(-a.lr, v[4 * q + 2], o.z);
-      r.w = fmaf(-a.lr, v[4 * q + 3], o.w);
-      d4[q] = r;
-      sh[q] = make_uint2(pack_bf16x2(r.x, r.y), pack_bf16x2(r.z, r.w));
-      nw[4 * q + 0] = r.x;
-      nw[4 * q + 1] = r.y;
-      nw[4 * q + 2] = r.z;
-      nw[4 * q + 3] = r.w;
-    }
-  } else {
+  for (int j = 0; j < 32; ++j) T[lane * 33 + j] = v[j];
+  __syncwarp();
+  const int n = n_base + lane;
+  const bool nok = n < a.N;
+  const int64_t so = static_cast<int64_t>(src) * a.slot_stride + a.offW + n;
+  const int64_t dof = static_cast<int64_t>(wid) * a.slot_stride + a.offW + n;
 #pragma unroll
-    for (int c = 0; c < 32; ++c) {
-      nw[c] = 0.f;
-      if (n0 + c < a.N) {
-        const float r = fmaf(-a.lr, v[c], a.master[so + n0 + c]);
-        a.master_w[dof + n0 + c] = r;
-        a.shadow[dof + n0 + c] = __float2bfloat16_rn(r);
-        nw[c] = r;
+  for (int r0 = 0; r0 < 32; r0 += 8) {
+    float old[8];
+#pragma unroll
+    for (int i = 0; i < 8; ++i)
+      old[i] = nok ? a.master[so + static_cast<int64_t>(m_base + r0 + i) * a.N] : 0.f;
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+      const int r = r0 + i;
+      const float nw = fmaf(-a.lr, T[r * 33 + lane], old[i]);
+      if (nok) {
+        const int64_t e = dof + static_cast<int64_t>(m_base + r) * a.N;
+        a.master_w[e] = nw;
+        a.shadow[e] = __float2bfloat16_rn(nw);
       }
+      T[r * 33 + lane] = nw;
     }
   }
+  __syncwarp();
   if (a.shadowT) {
-    __nv_bfloat16* t = a.shadowT + static_cast<int64_t>(wid) * a.slotT_stride + a.offT;
-#pragma unroll
-    for (int c = 0; c < 32; ++c)
-      if (n0 + c < a.N) t[static_cast<int64_t>(n0 + c) * a.M + m] = __float2bfloat16_rn(nw[c]);
+    __nv_bfloat16* t = a.shadowT + static_cast<int64_t>(wid) * a.slotT_stride + a.offT + m_base + lane;
+#pragma unroll 8
+    for (int j = 0; j < 32; ++j)
+      if (n_base + j < a.N) t[static_cast<int64_t>(n_base + j) * a.M] = __float2bfloat16_rn(T[lane * 33 + j]);
   }
+  __syncwarp();
 }
 
 __device__ __forceinline__ void epi_store(const GemmArgs& a, int m, int n0, const float (&v)[32]) {
@@ -149,7 +155,7 @@ __device__ __forceinline__ void epi_store(const GemmArgs& a, int m, int n0, cons
 }
 
 template <int BN, int EPI>
-__global__ void __launch_bounds__(kThreads) gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA,
+__global__ void __launch_bounds__(warps_for<EPI>() * 32) gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA,
                                                            const __grid_constant__ CUtensorMap mapB,
                                                            const __grid_constant__ GemmArgs a,
                                                            int stages) {
@@ -162,6 +168,7 @@ __global__ void __launch_bounds__(kThreads) gemm_tc_kernel(const __grid_constant
   uint64_t* empty = full + stages;
   uint64_t* accum = empty + stages;
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(accum + 1);
+  float* epi_tiles = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(full) + kBarrierBytes);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int li = blockIdx.z;
@@ -220,33 +227,44 @@ __global__ void __launch_bounds__(kThreads) gemm_tc_kernel(const __grid_constant
   __syncwarp();
 
   // epilogue: thread = one accumulator row
-  int acc_ok = 0;
-  if (lane == 0) acc_ok = mbar_wait(accum, 0, a.err, kDevTimeoutAccum) ? 1 : 0;
-  acc_ok = __shfl_sync(0xffffffffu, acc_ok, 0);
+  int acc_ok = mbar_wait(accum, 0, a.err, kDevTimeoutAccum) ? 1 : 0;
+  acc_ok = __all_sync(0xffffffffu, acc_ok);
   tc_fence_after();
   if (acc_ok) {
-    const int m = m0 + warp * 32 + lane;
-    const uint32_t trow = tmem + (static_cast<uint32_t>(warp * 32) << 16);
-    float gsum = 0.f;
+    const int quarter = warp & 3;
+    const int m = m0 + quarter * 32 + lane;
+    const uint32_t trow = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
+    if (EPI == kEpiDw) {
+      constexpr int kHalf = BN / 2;
+      const int c_begin = (warp >> 2) * kHalf;
+      float* T = epi_tiles + warp * kEpiTileFloats;
 #pragma unroll 1
-    for (int c0 = 0; c0 < BN; c0 += 32) {
-      float v[32];
-      tmem_ld_32x32b_x32(trow + c0, v);
-      if (EPI == kEpiFwd) {
-        epi_fwd<EPI>(a, wid, src, m, n0 + c0, v);
-      } else if (EPI == kEpiDh) {
-        gsum += epi_dh(a, wid, m, n0 + c0, v);
-      } else if (EPI == kEpiStore) {
-        if (n0 + c0 < a.N) epi_store(a, m, n0 + c0, v);
-      } else {
-        if (n0 + c0 < a.N) epi_dw(a, wid, src, m, n0 + c0, v);
+      for (int c0 = c_begin; c0 < c_begin + kHalf; c0 += 32) {
+        if (n0 + c0 >= a.N) break;   // uniform in the warp
+        float v[32];
+        tmem_ld_32x32b_x32(trow + c0, v);
+        epi_dw_block(a, wid, src, m0 + quarter * 32, n0 + c0, v, T, lane);
       }
-    }
-    if (EPI == kEpiDh) a.gb_out[static_cast<int64_t>(wid) * a.M + m] = gsum;
-    if (EPI == kEpiDw && blockIdx.y == 0) {
-      const int64_t bo = a.offB + m;
-      a.master_w[static_cast<int64_t>(wid) * a.slot_stride + bo] =
-          fmaf(-a.lr, a.gb_in[static_cast<int64_t>(wid) * a.M + m], a.master[static_cast<int64_t>(src) * a.slot_stride + bo]);
+      if (warp < 4 && blockIdx.y == 0) {
+        const int64_t bo = a.offB + m;
+        a.master_w[static_cast<int64_t>(wid) * a.slot_stride + bo] =
+            fmaf(-a.lr, a.gb_in[static_cast<int64_t>(wid) * a.M + m], a.master[static_cast<int64_t>(src) * a.slot_stride + bo]);
+      }
+    } else {
+      float gsum = 0.f;
+#pragma unroll 1
+      for (int c0 = 0; c0 < BN; c0 += 32) {
+        float v[32];
+        tmem_ld_32x32b_x32(trow + c0, v);
+        if (EPI == kEpiFwd) {
+          epi_fwd<EPI>(a, wid, src, m, n0 + c0, v);
+        } else if (EPI == kEpiDh) {
+          gsum += epi_dh(a, wid, m, n0 + c0, v);
+        } else if (EPI == kEpiStore) {
+          if (n0 + c0 < a.N) epi_store(a, m, n0 + c0, v);
+        }
+      }
+      if (EPI == kEpiDh) a.gb_out[static_cast<int64_t>(wid) * a.M + m] = gsum;
     }
   }
   tc_fence_before();
@@ -271,14 +289,16 @@ cudaError_t launch_tile(const CUtensorMap& mA, const CUtensorMap& mB, const Gemm
   using Cfg = TileCfg<BN>;
   const int nk = (a.K + BK - 1) / BK;
   const int stages = nk < 4 ? nk : 4;
-  size_t smem = 1024 + static_cast<size_t>(stages) * Cfg::kStageBytes + (2 * stages + 2) * 8 + 16;
+  constexpr int kWarps = warps_for<EPI>();
+  size_t smem = 1024 + static_cast<size_t>(stages) * Cfg::kStageBytes + kBarrierBytes +
+                (EPI == kEpiDw ? sizeof(float) * kWarps * kEpiTileFloats : 0);
   const size_t floor_b = smem_floor_for_tmem(Cfg::kTmemCols);
   if (smem < floor_b) smem = floor_b;
   cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<BN, EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(smem));
   if (e != cudaSuccess) return e;
   dim3 grid(a.M / BM, (a.N + BN - 1) / BN, n_active);
-  gemm_tc_kernel<BN, EPI><<<grid, kThreads, smem, s>>>(mA, mB, a, stages);
+  gemm_tc_kernel<BN, EPI><<<grid, kWarps * 32, smem, s>>>(mA, mB, a, stages);
   return cudaGetLastError();
 }
 
