@@ -119,6 +119,12 @@ struct oscars_ctx {
   int64_t eval_part_cap = 0;
   // tensor maps per layer
   std::vector<CUtensorMap> mShadow, mShadowT, mA, mG, mGT, mAT;
+  // per-step input buffers of layer 0 (a round's mini-batches are staged at once)
+  int stage_cap = 0;
+  __nv_bfloat16* A0all = nullptr;
+  __nv_bfloat16* A0Tall = nullptr;
+  int32_t* labels_all = nullptr;
+  std::vector<CUtensorMap> mA0s, mAT0s;
   // streams / graph
   cudaStream_t stream = nullptr;
   cudaStream_t cap = nullptr;
@@ -243,6 +249,33 @@ void update_barrier(oscars_ctx* c, bool from_search) {
   }
 }
 
+// Layer-0 inputs and labels for every local step of a round ([max_tau][W][...])
+// and one pair of tensor maps per step.  Grows when tau grows.
+oscars_status ensure_stage_buffers(oscars_ctx* c) {
+  if (!(c->bf16 && c->L >= 2) || c->stage_cap >= c->max_tau) return OSCARS_OK;
+  const int W = c->W, B = c->B, D = c->dims[0];
+  const size_t per = static_cast<size_t>(W) * B * D;
+  const int cap = c->max_tau;
+  if (!dev_alloc(c, &c->A0all, per * cap) || !dev_alloc(c, &c->A0Tall, per * cap) ||
+      !dev_alloc(c, &c->labels_all, static_cast<size_t>(W) * B * cap))
+    return fail(c, OSCARS_ENOMEM, "device allocation failed (per-step inputs)");
+  c->mA0s.resize(cap);
+  c->mAT0s.resize(cap);
+  for (int s = 0; s < cap; ++s) {
+    if (!make_map(&c->mA0s[s], c->A0all + per * s, D, B, W, D * 2ull, static_cast<uint64_t>(B) * D * 2ull, B) ||
+        !make_map(&c->mAT0s[s], c->A0Tall + per * s, B, D, W, B * 2ull, static_cast<uint64_t>(B) * D * 2ull, 128))
+      return fail(c, OSCARS_ECUDA, "cuTensorMapEncodeTiled failed (per-step inputs)");
+  }
+  // step 0 doubles as the single-step buffers (evaluation)
+  c->A[0] = c->A0all;
+  c->AT[0] = c->A0Tall;
+  c->labels = c->labels_all;
+  c->mA[0] = c->mA0s[0];
+  c->mAT[0] = c->mAT0s[0];
+  c->stage_cap = cap;
+  return OSCARS_OK;
+}
+
 oscars_status build_tables(oscars_ctx* c) {
   c->max_tau = 0;
   for (int i = 0; i < c->W; ++i) c->max_tau = std::max(c->max_tau, static_cast<int>(c->tau[i]));
@@ -272,7 +305,7 @@ oscars_status build_tables(oscars_ctx* c) {
     cudaGraphExecDestroy(c->round_exec);
     c->round_exec = nullptr;
   }
-  return OSCARS_OK;
+  return ensure_stage_buffers(c);
 }
 
 cudaError_t refresh_global_shadows(oscars_ctx* c, cudaStream_t s) {
@@ -331,7 +364,7 @@ HeadArgs head_base(oscars_ctx* c) {
 }
 
 // forward layers 0..L-2 for `na` lanes (training step or evaluation)
-cudaError_t enqueue_forward(oscars_ctx* c, const int* wid, const int* src, int na, cudaStream_t st) {
+cudaError_t enqueue_forward(oscars_ctx* c, const int* wid, const int* src, int na, cudaStream_t st, int step = 0) {
   for (int l = 0; l + 1 < c->L; ++l) {
     const Layer& ly = c->layers[l];
     GemmArgs g = gemm_base(c, 0);
@@ -347,7 +380,7 @@ cudaError_t enqueue_forward(oscars_ctx* c, const int* wid, const int* src, int n
     g.out = c->A[l + 1];
     g.outT = c->AT[l + 1];
     ProfScope ps(c, "gemm_fwd", st);
-    cudaError_t e = launch_gemm(kEpiFwd, c->mShadow[l], c->mA[l], g, na, st);
+    cudaError_t e = launch_gemm(kEpiFwd, c->mShadow[l], l == 0 ? c->mA0s[step] : c->mA[l], g, na, st);
     if (e != cudaSuccess) return e;
   }
   return cudaSuccess;
@@ -355,38 +388,42 @@ cudaError_t enqueue_forward(oscars_ctx* c, const int* wid, const int* src, int n
 
 cudaError_t enqueue_round_mlp(oscars_ctx* c, cudaStream_t st) {
   cudaError_t e;
-  for (int s = 0; s < c->max_tau; ++s) {
-    const int na = c->n_active[s];
-    const int* wid = c->act_wid + static_cast<size_t>(s) * c->W;
-    const int* src = c->act_src + static_cast<size_t>(s) * c->W;
+  {
     StageArgs sa;
     sa.x = c->dx_tab;
     sa.y = c->dy_tab;
     sa.n = c->dn_tab;
     sa.start = c->cursor;
-    sa.row_add = static_cast<int64_t>(s) * c->B;
-    sa.wid = wid;
+    sa.row_add = 0;
+    sa.wid = nullptr;
     sa.D = c->dims[0];
     sa.B = c->B;
-    sa.A0 = c->A[0];
-    sa.A0T = c->AT[0];
-    sa.labels = c->labels;
-    {
-      ProfScope ps(c, "stage", st);
-      if ((e = launch_stage(sa, na, st)) != cudaSuccess) return e;
-    }
-    if ((e = enqueue_forward(c, wid, src, na, st)) != cudaSuccess) return e;
+    sa.A0 = c->A0all;
+    sa.A0T = c->A0Tall;
+    sa.labels = c->labels_all;
+    ProfScope ps(c, "stage", st);
+    if ((e = launch_stage_round(sa, c->tau_dev, c->W, c->max_tau, st)) != cudaSuccess) return e;
+  }
+  for (int s = 0; s < c->max_tau; ++s) {
+    const int na = c->n_active[s];
+    const int* wid = c->act_wid + static_cast<size_t>(s) * c->W;
+    const int* src = c->act_src + static_cast<size_t>(s) * c->W;
+    if ((e = enqueue_forward(c, wid, src, na, st, s)) != cudaSuccess) return e;
     HeadArgs h = head_base(c);
     h.wid = wid;
     h.src = src;
+    h.labels = c->labels_all + static_cast<size_t>(s) * c->W * c->B;
     h.loss_part = c->loss_part;
     h.part_mul = c->max_tau;
     h.part_add = s;
-    {
-      ProfScope ps(c, "head_fwd", st);
-      if ((e = launch_head_fwd(h, na, st)) != cudaSuccess) return e;
-    }
-    {
+    if (head_fused_supported(h.H, h.B, h.C)) {
+      ProfScope ps(c, "head_fused", st);
+      if ((e = launch_head_fused(h, na, st)) != cudaSuccess) return e;
+    } else {
+      {
+        ProfScope ps(c, "head_fwd", st);
+        if ((e = launch_head_fwd(h, na, st)) != cudaSuccess) return e;
+      }
       ProfScope ps(c, "head_bwd", st);
       if ((e = launch_head_bwd(h, na, st)) != cudaSuccess) return e;
     }
@@ -418,7 +455,7 @@ cudaError_t enqueue_round_mlp(oscars_ctx* c, cudaStream_t st) {
       g.shadowT = ly.offT >= 0 ? c->shadowT : nullptr;
       g.gb_in = c->gb[l];
       ProfScope ps(c, "gemm_dw_sgd", st);
-      if ((e = launch_gemm(kEpiDw, c->mGT[l], c->mAT[l], g, na, st)) != cudaSuccess) return e;
+      if ((e = launch_gemm(kEpiDw, c->mGT[l], l == 0 ? c->mAT0s[s] : c->mAT[l], g, na, st)) != cudaSuccess) return e;
     }
   }
   const int nc = c->B / kRowsPerLossChunk;
@@ -575,7 +612,7 @@ oscars_status allocate_mlp(oscars_ctx* c) {
   c->gb.assign(L, nullptr);
   for (int l = 0; l < L; ++l) {
     const size_t act = static_cast<size_t>(W) * B * c->dims[l];
-    if (!dev_alloc(c, &c->A[l], act) || !dev_alloc(c, &c->AT[l], act))
+    if (l > 0 && (!dev_alloc(c, &c->A[l], act) || !dev_alloc(c, &c->AT[l], act)))
       return fail(c, OSCARS_ENOMEM, "device allocation failed (activations)");
     if (l + 1 < L) {
       const size_t gsz = static_cast<size_t>(W) * B * c->dims[l + 1];
@@ -584,7 +621,7 @@ oscars_status allocate_mlp(oscars_ctx* c) {
         return fail(c, OSCARS_ENOMEM, "device allocation failed (gradients)");
     }
   }
-  if (!dev_alloc(c, &c->labels, static_cast<size_t>(W) * B) || !dev_alloc(c, &c->dlog, static_cast<size_t>(W) * B * c->C))
+  if (!dev_alloc(c, &c->dlog, static_cast<size_t>(W) * B * c->C))
     return fail(c, OSCARS_ENOMEM, "device allocation failed (head)");
 
   // tensor maps
@@ -600,12 +637,12 @@ oscars_status allocate_mlp(oscars_ctx* c) {
     bool ok = true;
     // W_l [out][in] of every slot: A operand of the forward GEMM
     ok &= make_map(&c->mShadow[l], c->shadow + ly.offW, ly.in, ly.out, slots64, ly.in * 2ull, c->P_pad * 2ull, 128);
-    // layer input [lane][B][in]: B operand of the forward GEMM
-    ok &= make_map(&c->mA[l], c->A[l], ly.in, B, W, ly.in * 2ull, static_cast<uint64_t>(B) * ly.in * 2ull, B);
+    // layer input [lane][B][in]: B operand of the forward GEMM (layer 0: per step)
+    if (l > 0) ok &= make_map(&c->mA[l], c->A[l], ly.in, B, W, ly.in * 2ull, static_cast<uint64_t>(B) * ly.in * 2ull, B);
     // output gradient^T [lane][out][B]: A operand of the weight-gradient GEMM
     ok &= make_map(&c->mGT[l], c->GT[l], B, ly.out, W, B * 2ull, static_cast<uint64_t>(B) * ly.out * 2ull, 128);
-    // layer input^T [lane][in][B]: B operand of the weight-gradient GEMM
-    ok &= make_map(&c->mAT[l], c->AT[l], B, ly.in, W, B * 2ull, static_cast<uint64_t>(B) * ly.in * 2ull, 128);
+    // layer input^T [lane][in][B]: B operand of the weight-gradient GEMM (layer 0: per step)
+    if (l > 0) ok &= make_map(&c->mAT[l], c->AT[l], B, ly.in, W, B * 2ull, static_cast<uint64_t>(B) * ly.in * 2ull, 128);
     if (l >= 1) {
       // W_l^T [in][out] of every slot: A operand of the input-gradient GEMM
       ok &= make_map(&c->mShadowT[l], c->shadowT + ly.offT, ly.out, ly.in, slots64, ly.out * 2ull, c->PT_pad * 2ull, 128);

@@ -78,6 +78,8 @@ struct StageArgs {
   int32_t* labels;         // [lanes][B]
 };
 cudaError_t launch_stage(const StageArgs& a, int n_active, cudaStream_t s);
+// all mini-batches of a round: step s of worker w (s < tau[w]) at slot s * W + w
+cudaError_t launch_stage_round(const StageArgs& a, const int32_t* tau, int W, int max_tau, cudaStream_t s);
 
 enum GemmEpi { kEpiFwd = 0, kEpiDh = 1, kEpiDw = 2, kEpiStore = 3 };
 
@@ -130,6 +132,10 @@ struct HeadArgs {
   float* gb;                  // [lanes][H]
 };
 cudaError_t launch_head_fwd(const HeadArgs& a, int n_active, cudaStream_t s);
+// forward + backward of the last layer in one launch: one cluster of H/128
+// CTAs per active lane (H <= 1024); false if the shape needs the two-kernel path
+bool head_fused_supported(int H, int B, int C);
+cudaError_t launch_head_fused(const HeadArgs& a, int n_active, cudaStream_t s);
 cudaError_t launch_head_bwd(const HeadArgs& a, int n_active, cudaStream_t s);
 
 // loss[w] = sum_{s < tau[w]} sum_c part[(w*max_tau + s)*nc + c] / (B * tau[w])

@@ -29,16 +29,13 @@ __device__ __forceinline__ float warp_max(float v) {
 // matrix, rounded to bf16 as A0 [B][D] and transposed A0T [D][B] (the
 // K-major operand of the first layer's weight-gradient GEMM).  32 x 32
 // tiles through shared memory so both writes are coalesced.
-__global__ void __launch_bounds__(256) stage_kernel(const __grid_constant__ StageArgs a) {
+__device__ __forceinline__ void stage_tile(const StageArgs& a, int w, int64_t base, __nv_bfloat16* A0,
+                                           __nv_bfloat16* A0T, int32_t* labels) {
   __shared__ __nv_bfloat16 tile[32][34];
-  const int w = a.wid[blockIdx.z];
   const int k0 = blockIdx.x * 32, b0 = blockIdx.y * 32;
   const float* X = a.x[w];
   const int64_t n = a.n[w];
-  const int64_t base = a.start[w] + a.row_add;
   const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;  // 32 x 8
-  __nv_bfloat16* A0 = a.A0 + static_cast<int64_t>(w) * a.B * a.D;
-  __nv_bfloat16* A0T = a.A0T + static_cast<int64_t>(w) * a.B * a.D;
   for (int r = ty; r < 32; r += 8) {
     const int b = b0 + r, k = k0 + tx;
     __nv_bfloat16 v = __float2bfloat16_rn(0.f);
@@ -56,8 +53,27 @@ __global__ void __launch_bounds__(256) stage_kernel(const __grid_constant__ Stag
   }
   if (blockIdx.x == 0 && threadIdx.x < 32) {
     const int b = b0 + threadIdx.x;
-    if (b < a.B) a.labels[static_cast<int64_t>(w) * a.B + b] = a.y[w][(base + b) % n];
+    if (b < a.B) labels[b] = a.y[w][(base + b) % n];
   }
+}
+
+__global__ void __launch_bounds__(256) stage_kernel(const __grid_constant__ StageArgs a) {
+  const int w = a.wid[blockIdx.z];
+  const int64_t off = static_cast<int64_t>(w) * a.B * a.D;
+  stage_tile(a, w, a.start[w] + a.row_add, a.A0 + off, a.A0T + off, a.labels + static_cast<int64_t>(w) * a.B);
+}
+
+// Every mini-batch of a round at once: grid z = step * W + worker; a CTA
+// whose worker has fewer local steps returns at once.  Step s of worker w
+// lands at offset (s * W + w) of the per-step buffers.
+__global__ void __launch_bounds__(256) stage_round_kernel(const __grid_constant__ StageArgs a, const int32_t* tau,
+                                                          int W) {
+  const int z = blockIdx.z;
+  const int s = z / W, w = z - s * W;
+  if (s >= tau[w]) return;
+  const int64_t slot = static_cast<int64_t>(s) * W + w;
+  const int64_t off = slot * a.B * a.D;
+  stage_tile(a, w, a.start[w] + static_cast<int64_t>(s) * a.B, a.A0 + off, a.A0T + off, a.labels + slot * a.B);
 }
 
 // ---------------------------------------------------------------- head forward
@@ -283,6 +299,173 @@ __global__ void __launch_bounds__(kHeadBwdThreads) head_bwd_kernel(const __grid_
   }
 }
 
+// ---------------------------------------------------------------- fused head
+// Forward and backward of the last layer (C <= 32 classes) in one launch.
+// A cluster of H/128 CTAs serves one active lane; CTA r owns hidden features
+// [128 r, 128 r + 128):
+//  1. partial logits over its features, pl[b][c] (warp per row, lanes over k);
+//  2. cluster barrier; every CTA sums the partials of ranks 0..n-1 in that
+//     order from distributed shared memory, so all CTAs hold the same logits,
+//     and runs the softmax cross-entropy (no cancellation: see head_fwd);
+//  3. a second cluster barrier (no CTA leaves while others read its partials);
+//  4. backward for its features exactly as head_bwd: masked input gradient
+//     (bf16 G, G^T, fp32 bias gradient), head weight gradient + SGD.
+// Rank 0 also writes the loss partials and updates the head bias.
+constexpr int kHF = 128;                 // hidden features per CTA
+constexpr int kHFThreads = 256;
+constexpr int kHFGroups = kHFThreads / kHF;
+constexpr int kHFMaxCluster = 8;
+
+size_t head_fused_smem(int B, int C) {
+  return sizeof(float) * (static_cast<size_t>(B) * kHF + static_cast<size_t>(C) * kHF + 3 * static_cast<size_t>(B) * C +
+                          kHFGroups * kHF + B) +
+         sizeof(__nv_bfloat16) * static_cast<size_t>(kHF) * (B + 8);
+}
+
+__global__ void __launch_bounds__(kHFThreads) head_fused_kernel(const __grid_constant__ HeadArgs a) {
+  extern __shared__ __align__(16) float fsm[];
+  const int H = a.H, C = a.C, B = a.B;
+  float* hs = fsm;                         // [B][kHF] bf16 h as float
+  float* wcs = hs + B * kHF;               // [C][kHF] old bf16 head weights as float
+  float* pl = wcs + C * kHF;               // [B][C] partial logits (read by the cluster)
+  float* dz = pl + B * C;                  // [B][C] dlogits fp32
+  float* dzb = dz + B * C;                 // [B][C] bf16-rounded
+  float* gbp = dzb + B * C;                // [kHFGroups][kHF]
+  float* rowloss = gbp + kHFGroups * kHF;  // [B]
+  __nv_bfloat16* gts = reinterpret_cast<__nv_bfloat16*>(rowloss + B);   // [kHF][B + 8]
+  const int gts_ld = B + 8;
+  const int i = blockIdx.x;
+  const int w = a.wid[i], src = a.src[i];
+  const uint32_t rank = cluster_ctarank();
+  const uint32_t ncl = gridDim.y;
+  const int k0 = blockIdx.y * kHF;
+  const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
+  const int64_t so = static_cast<int64_t>(src) * a.slot_stride;
+  const int64_t dof = static_cast<int64_t>(w) * a.slot_stride;
+  const __nv_bfloat16* h = a.Ain + static_cast<int64_t>(w) * B * H;
+
+  // stage this CTA's slice of h and of the head weights
+  for (int q = t; q < B * (kHF / 8); q += kHFThreads) {
+    const int b = q / (kHF / 8), c8 = (q % (kHF / 8)) * 8;
+    const uint4 v = *reinterpret_cast<const uint4*>(h + static_cast<int64_t>(b) * H + k0 + c8);
+    const __nv_bfloat162* p2 = reinterpret_cast<const __nv_bfloat162*>(&v);
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const float2 f = __bfloat1622float2(p2[j]);
+      hs[b * kHF + c8 + 2 * j] = f.x;
+      hs[b * kHF + c8 + 2 * j + 1] = f.y;
+    }
+  }
+  for (int q = t; q < C * (kHF / 8); q += kHFThreads) {
+    const int c = q / (kHF / 8), c8 = (q % (kHF / 8)) * 8;
+    const uint4 v = *reinterpret_cast<const uint4*>(a.shadow + so + a.offW + static_cast<int64_t>(c) * H + k0 + c8);
+    const __nv_bfloat162* p2 = reinterpret_cast<const __nv_bfloat162*>(&v);
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const float2 f = __bfloat1622float2(p2[j]);
+      wcs[c * kHF + c8 + 2 * j] = f.x;
+      wcs[c * kHF + c8 + 2 * j + 1] = f.y;
+    }
+  }
+  __syncthreads();
+  // 1. partial logits: warp per row, each lane 4 features
+  for (int b = warp; b < B; b += kHFThreads / 32) {
+    const float4 hv = *reinterpret_cast<const float4*>(hs + b * kHF + lane * 4);
+    for (int c = 0; c < C; ++c) {
+      const float4 wv = *reinterpret_cast<const float4*>(wcs + c * kHF + lane * 4);
+      float acc = hv.x * wv.x;
+      acc = fmaf(hv.y, wv.y, acc);
+      acc = fmaf(hv.z, wv.z, acc);
+      acc = fmaf(hv.w, wv.w, acc);
+      acc = warp_sum(acc);
+      if (lane == 0) pl[b * C + c] = acc;
+    }
+  }
+  cluster_sync();
+  // 2. logits = sum of the cluster's partials in rank order; softmax CE
+  const float* bias = a.master + so + a.offB;
+  for (int b = t; b < B; b += kHFThreads) {
+    float z[kMaxClasses];
+    float m = -INFINITY;
+    for (int c = 0; c < C; ++c) {
+      float acc = 0.f;
+      for (uint32_t r = 0; r < ncl; ++r) acc += ld_dsmem_f32(pl + b * C + c, r);
+      z[c] = acc + bias[c];
+      m = fmaxf(m, z[c]);
+    }
+    const int y = a.labels[static_cast<int64_t>(w) * B + b];
+    float s = 0.f, so_ = 0.f;
+    for (int c = 0; c < C; ++c) {
+      const float e = expf(z[c] - m);
+      s += e;
+      if (c != y) so_ += e;
+    }
+    for (int c = 0; c < C; ++c) {
+      const float g = (c == y ? -(so_ / s) : expf(z[c] - m) / s) / static_cast<float>(B);
+      dz[b * C + c] = g;
+      dzb[b * C + c] = bf16_round(g);
+    }
+    rowloss[b] = m + logf(s) - z[y];
+  }
+  cluster_sync();   // partials are no longer read remotely; dz is complete locally
+  if (rank == 0) {
+    if (t < B / kRowsPerLossChunk) {
+      float l = 0.f;
+      for (int r = 0; r < kRowsPerLossChunk; ++r) l += rowloss[t * kRowsPerLossChunk + r];
+      const int64_t row = static_cast<int64_t>(w) * a.part_mul + a.part_add;
+      a.loss_part[row * (B / kRowsPerLossChunk) + t] = l;
+    }
+    if (t < C) {
+      float g = 0.f;
+      for (int b = 0; b < B; ++b) g += dz[b * C + t];
+      a.master_w[dof + a.offB + t] = fmaf(-a.lr, g, a.master[so + a.offB + t]);
+    }
+  }
+  // 3. masked input gradient of the layer below for this CTA's features
+  {
+    const int k = t % kHF, grp = t / kHF;
+    const int rows = B / kHFGroups;
+    float gsum = 0.f;
+    __nv_bfloat16* G = a.G + static_cast<int64_t>(w) * B * H;
+    for (int r = 0; r < rows; ++r) {
+      const int b = grp * rows + r;
+      const float hv = hs[b * kHF + k];
+      float dh = 0.f;
+      for (int c = 0; c < C; ++c) dh = fmaf(dzb[b * C + c], wcs[c * kHF + k], dh);
+      const float g = hv > 0.f ? dh : 0.f;
+      gsum += g;
+      const __nv_bfloat16 g16 = __float2bfloat16_rn(g);
+      G[static_cast<int64_t>(b) * H + k0 + k] = g16;
+      gts[k * gts_ld + b] = g16;
+    }
+    gbp[grp * kHF + k] = gsum;
+  }
+  __syncthreads();
+  if (t < kHF) {
+    float g = 0.f;
+    for (int grp = 0; grp < kHFGroups; ++grp) g += gbp[grp * kHF + t];
+    a.gb[static_cast<int64_t>(w) * H + k0 + t] = g;
+  }
+  {
+    uint4* GT = reinterpret_cast<uint4*>(a.GT + (static_cast<int64_t>(w) * H + k0) * B);
+    const int per_row = B / 8;
+    for (int q = t; q < kHF * per_row; q += kHFThreads) {
+      const int k = q / per_row, j = q - k * per_row;
+      GT[static_cast<int64_t>(k) * per_row + j] = *reinterpret_cast<const uint4*>(gts + k * gts_ld + j * 8);
+    }
+  }
+  // 4. head weight gradient and SGD for this CTA's features
+  for (int q = t; q < C * kHF; q += kHFThreads) {
+    const int c = q / kHF, k = q - c * kHF;
+    float dw = 0.f;
+    for (int b = 0; b < B; ++b) dw = fmaf(dzb[b * C + c], hs[b * kHF + k], dw);
+    const int64_t e = a.offW + static_cast<int64_t>(c) * H + k0 + k;
+    const float nw = fmaf(-a.lr, dw, a.master[so + e]);
+    a.master_w[dof + e] = nw;
+    a.shadow_w[dof + e] = __float2bfloat16_rn(nw);
+  }
+}
+
 // ---------------------------------------------------------------- bookkeeping
 __global__ void loss_finalize_kernel(const float* part, const int32_t* tau, int W, int max_tau,
                                      int nc, int B, float* loss) {
@@ -349,6 +532,12 @@ cudaError_t launch_stage(const StageArgs& a, int n_active, cudaStream_t s) {
   return cudaGetLastError();
 }
 
+cudaError_t launch_stage_round(const StageArgs& a, const int32_t* tau, int W, int max_tau, cudaStream_t s) {
+  dim3 grid((a.D + 31) / 32, (a.B + 31) / 32, W * max_tau);
+  stage_round_kernel<<<grid, 256, 0, s>>>(a, tau, W);
+  return cudaGetLastError();
+}
+
 cudaError_t launch_head_fwd(const HeadArgs& a, int n_active, cudaStream_t s) {
   if (a.H % 8 != 0 || a.H > 32 * 8 * kHeadMaxH8) return cudaErrorInvalidValue;
   const size_t smem = sizeof(float) * static_cast<size_t>(a.C) * a.H;
@@ -369,6 +558,32 @@ cudaError_t launch_head_bwd(const HeadArgs& a, int n_active, cudaStream_t s) {
   dim3 grid(n_active, (a.H + kHB - 1) / kHB);
   head_bwd_kernel<<<grid, kHeadBwdThreads, smem, s>>>(a);
   return cudaGetLastError();
+}
+
+bool head_fused_supported(int H, int B, int C) {
+  return H % kHF == 0 && H / kHF <= kHFMaxCluster && B % (8 * kHFGroups) == 0 && B % kRowsPerLossChunk == 0 &&
+         B / kRowsPerLossChunk <= kHFThreads && C <= kMaxClasses && head_fused_smem(B, C) <= 220 * 1024;
+}
+
+cudaError_t launch_head_fused(const HeadArgs& a, int n_active, cudaStream_t s) {
+  if (!head_fused_supported(a.H, a.B, a.C)) return cudaErrorInvalidValue;
+  const size_t smem = head_fused_smem(a.B, a.C);
+  cudaError_t e = cudaFuncSetAttribute(head_fused_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       static_cast<int>(smem));
+  if (e != cudaSuccess) return e;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(n_active, a.H / kHF, 1);
+  cfg.blockDim = dim3(kHFThreads, 1, 1);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 1;
+  attr[0].val.clusterDim.y = a.H / kHF;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, head_fused_kernel, a);
 }
 
 cudaError_t launch_loss_finalize(const float* part, const int32_t* tau, int W, int max_tau, int nc, int B,
