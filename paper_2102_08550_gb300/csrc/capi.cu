@@ -30,6 +30,8 @@ namespace {
 
 int64_t round_up(int64_t x, int64_t m) { return (x + m - 1) / m * m; }
 
+constexpr int kMaxBranches = 16;
+
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
                                   const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
@@ -128,6 +130,16 @@ struct oscars_ctx {
   // streams / graph
   cudaStream_t stream = nullptr;
   cudaStream_t cap = nullptr;
+  // concurrent branches of a round: workers are independent between merges,
+  // so each branch runs the local steps of its own workers on its own stream
+  int n_br = 1;
+  std::vector<cudaStream_t> br_streams;
+  std::vector<cudaEvent_t> br_join;
+  cudaEvent_t br_fork = nullptr;
+  std::vector<int> br_max_tau;          // [n_br]
+  std::vector<int> br_na;               // [n_br][max_tau] active workers per step
+  int* br_wid = nullptr;                // [n_br][max_tau][W]
+  int* br_src = nullptr;
   cudaGraphExec_t round_exec = nullptr;
   bool pending = false;
   std::string last_error;
@@ -236,6 +248,12 @@ void free_all(oscars_ctx* c) {
   c->allocs.clear();
   if (c->cap) cudaStreamDestroy(c->cap);
   c->cap = nullptr;
+  for (cudaStream_t b : c->br_streams) cudaStreamDestroy(b);
+  c->br_streams.clear();
+  for (cudaEvent_t e : c->br_join) cudaEventDestroy(e);
+  c->br_join.clear();
+  if (c->br_fork) cudaEventDestroy(c->br_fork);
+  c->br_fork = nullptr;
 }
 
 // Simulated barrier and idle time per worker for the current tau (Eq. 1).
@@ -294,6 +312,37 @@ oscars_status build_tables(oscars_ctx* c) {
   if (c->act_wid) {
     // tables are reallocated when tau changes
   }
+  // branches: workers sorted by tau (descending), dealt round-robin
+  std::vector<int> order(c->W);
+  for (int i = 0; i < c->W; ++i) order[i] = i;
+  std::stable_sort(order.begin(), order.end(), [&](int x, int y) { return c->tau[x] > c->tau[y]; });
+  std::vector<std::vector<int>> members(c->n_br);
+  for (int j = 0; j < c->W; ++j) members[j % c->n_br].push_back(order[j]);
+  c->br_max_tau.assign(c->n_br, 0);
+  c->br_na.assign(static_cast<size_t>(c->n_br) * c->max_tau, 0);
+  std::vector<int> bw(static_cast<size_t>(c->n_br) * c->max_tau * c->W, 0), bs(bw.size(), 0);
+  for (int g = 0; g < c->n_br; ++g) {
+    std::sort(members[g].begin(), members[g].end());
+    for (int s = 0; s < c->max_tau; ++s) {
+      int n = 0;
+      for (int i : members[g])
+        if (c->tau[i] > s) {
+          const size_t at = (static_cast<size_t>(g) * c->max_tau + s) * c->W + n;
+          bw[at] = i;
+          bs[at] = s == 0 ? c->W : i;
+          ++n;
+        }
+      c->br_na[static_cast<size_t>(g) * c->max_tau + s] = n;
+      if (n > 0) c->br_max_tau[g] = s + 1;
+    }
+  }
+  if (!dev_alloc(c, &c->br_wid, bw.size()) || !dev_alloc(c, &c->br_src, bs.size()))
+    return fail(c, OSCARS_ENOMEM, "device allocation failed (branch tables)");
+  {
+    cudaError_t e = cudaMemcpy(c->br_wid, bw.data(), bw.size() * sizeof(int), cudaMemcpyHostToDevice);
+    if (e == cudaSuccess) e = cudaMemcpy(c->br_src, bs.data(), bs.size() * sizeof(int), cudaMemcpyHostToDevice);
+    if (e != cudaSuccess) return cuda_fail(c, e, "branch table upload");
+  }
   if (!dev_alloc(c, &c->act_wid, wid.size()) || !dev_alloc(c, &c->act_src, src.size()) ||
       !dev_alloc(c, &c->loss_part, static_cast<size_t>(c->W) * c->max_tau * std::max(1, c->B / kRowsPerLossChunk)))
     return fail(c, OSCARS_ENOMEM, "device allocation failed (schedule tables)");
@@ -322,11 +371,11 @@ cudaError_t refresh_global_shadows(oscars_ctx* c, cudaStream_t s) {
   return cudaSuccess;
 }
 
-GemmArgs gemm_base(oscars_ctx* c, int s) {
+GemmArgs gemm_base(oscars_ctx* c, const int* wid, const int* src) {
   GemmArgs g;
   std::memset(&g, 0, sizeof(g));
-  g.wid = c->act_wid + static_cast<size_t>(s) * c->W;
-  g.src = c->act_src + static_cast<size_t>(s) * c->W;
+  g.wid = wid;
+  g.src = src;
   g.err = c->err;
   g.master = c->slab;
   g.master_w = c->slab;
@@ -367,9 +416,7 @@ HeadArgs head_base(oscars_ctx* c) {
 cudaError_t enqueue_forward(oscars_ctx* c, const int* wid, const int* src, int na, cudaStream_t st, int step = 0) {
   for (int l = 0; l + 1 < c->L; ++l) {
     const Layer& ly = c->layers[l];
-    GemmArgs g = gemm_base(c, 0);
-    g.wid = wid;
-    g.src = src;
+    GemmArgs g = gemm_base(c, wid, src);
     g.M = ly.out;
     g.N = c->B;
     g.K = ly.in;
@@ -382,6 +429,62 @@ cudaError_t enqueue_forward(oscars_ctx* c, const int* wid, const int* src, int n
     ProfScope ps(c, "gemm_fwd", st);
     cudaError_t e = launch_gemm(kEpiFwd, c->mShadow[l], l == 0 ? c->mA0s[step] : c->mA[l], g, na, st);
     if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
+}
+
+// One local step of the active workers `wid` (parameters from slots `src`):
+// forward, last layer, and backward of the hidden layers (Eq. 4, "otherwise").
+cudaError_t enqueue_step(oscars_ctx* c, int s, int na, const int* wid, const int* src, cudaStream_t st) {
+  cudaError_t e;
+  if ((e = enqueue_forward(c, wid, src, na, st, s)) != cudaSuccess) return e;
+  HeadArgs h = head_base(c);
+  h.wid = wid;
+  h.src = src;
+  h.labels = c->labels_all + static_cast<size_t>(s) * c->W * c->B;
+  h.loss_part = c->loss_part;
+  h.part_mul = c->max_tau;
+  h.part_add = s;
+  if (head_fused_supported(h.H, h.B, h.C)) {
+    ProfScope ps(c, "head_fused", st);
+    if ((e = launch_head_fused(h, na, st)) != cudaSuccess) return e;
+  } else {
+    {
+      ProfScope ps(c, "head_fwd", st);
+      if ((e = launch_head_fwd(h, na, st)) != cudaSuccess) return e;
+    }
+    ProfScope ps(c, "head_bwd", st);
+    if ((e = launch_head_bwd(h, na, st)) != cudaSuccess) return e;
+  }
+  for (int l = c->L - 2; l >= 0; --l) {
+    const Layer& ly = c->layers[l];
+    if (l >= 1) {  // input gradient of layer l -> gradient of layer l-1's output
+      GemmArgs g = gemm_base(c, wid, src);
+      g.M = ly.in;
+      g.N = c->B;
+      g.K = ly.out;
+      g.a_z_src = 1;
+      g.b_z_src = 0;
+      g.hmask = c->A[l];
+      g.out = c->G[l - 1];
+      g.outT = c->GT[l - 1];
+      g.gb_out = c->gb[l - 1];
+      ProfScope ps(c, "gemm_dh", st);
+      if ((e = launch_gemm(kEpiDh, c->mShadowT[l], c->mG[l], g, na, st)) != cudaSuccess) return e;
+    }
+    GemmArgs g = gemm_base(c, wid, src);
+    g.M = ly.out;
+    g.N = ly.in;
+    g.K = c->B;
+    g.a_z_src = 0;
+    g.b_z_src = 0;
+    g.offW = ly.offW;
+    g.offB = ly.offB;
+    g.offT = ly.offT;
+    g.shadowT = ly.offT >= 0 ? c->shadowT : nullptr;
+    g.gb_in = c->gb[l];
+    ProfScope ps(c, "gemm_dw_sgd", st);
+    if ((e = launch_gemm(kEpiDw, c->mGT[l], l == 0 ? c->mAT0s[s] : c->mAT[l], g, na, st)) != cudaSuccess) return e;
   }
   return cudaSuccess;
 }
@@ -404,58 +507,21 @@ cudaError_t enqueue_round_mlp(oscars_ctx* c, cudaStream_t st) {
     ProfScope ps(c, "stage", st);
     if ((e = launch_stage_round(sa, c->tau_dev, c->W, c->max_tau, st)) != cudaSuccess) return e;
   }
-  for (int s = 0; s < c->max_tau; ++s) {
-    const int na = c->n_active[s];
-    const int* wid = c->act_wid + static_cast<size_t>(s) * c->W;
-    const int* src = c->act_src + static_cast<size_t>(s) * c->W;
-    if ((e = enqueue_forward(c, wid, src, na, st, s)) != cudaSuccess) return e;
-    HeadArgs h = head_base(c);
-    h.wid = wid;
-    h.src = src;
-    h.labels = c->labels_all + static_cast<size_t>(s) * c->W * c->B;
-    h.loss_part = c->loss_part;
-    h.part_mul = c->max_tau;
-    h.part_add = s;
-    if (head_fused_supported(h.H, h.B, h.C)) {
-      ProfScope ps(c, "head_fused", st);
-      if ((e = launch_head_fused(h, na, st)) != cudaSuccess) return e;
-    } else {
-      {
-        ProfScope ps(c, "head_fwd", st);
-        if ((e = launch_head_fwd(h, na, st)) != cudaSuccess) return e;
-      }
-      ProfScope ps(c, "head_bwd", st);
-      if ((e = launch_head_bwd(h, na, st)) != cudaSuccess) return e;
+  if (c->n_br > 1) {
+    cudaError_t e2 = cudaEventRecord(c->br_fork, st);
+    if (e2 != cudaSuccess) return e2;
+  }
+  for (int g = 0; g < c->n_br; ++g) {
+    cudaStream_t sg = c->n_br > 1 ? c->br_streams[g] : st;
+    if (c->n_br > 1 && (e = cudaStreamWaitEvent(sg, c->br_fork, 0)) != cudaSuccess) return e;
+    for (int s = 0; s < c->br_max_tau[g]; ++s) {
+      const size_t at = (static_cast<size_t>(g) * c->max_tau + s);
+      const int na = c->br_na[at];
+      if ((e = enqueue_step(c, s, na, c->br_wid + at * c->W, c->br_src + at * c->W, sg)) != cudaSuccess) return e;
     }
-    for (int l = c->L - 2; l >= 0; --l) {
-      const Layer& ly = c->layers[l];
-      if (l >= 1) {  // input gradient of layer l -> gradient of layer l-1's output
-        GemmArgs g = gemm_base(c, s);
-        g.M = ly.in;
-        g.N = c->B;
-        g.K = ly.out;
-        g.a_z_src = 1;
-        g.b_z_src = 0;
-        g.hmask = c->A[l];
-        g.out = c->G[l - 1];
-        g.outT = c->GT[l - 1];
-        g.gb_out = c->gb[l - 1];
-        ProfScope ps(c, "gemm_dh", st);
-        if ((e = launch_gemm(kEpiDh, c->mShadowT[l], c->mG[l], g, na, st)) != cudaSuccess) return e;
-      }
-      GemmArgs g = gemm_base(c, s);
-      g.M = ly.out;
-      g.N = ly.in;
-      g.K = c->B;
-      g.a_z_src = 0;
-      g.b_z_src = 0;
-      g.offW = ly.offW;
-      g.offB = ly.offB;
-      g.offT = ly.offT;
-      g.shadowT = ly.offT >= 0 ? c->shadowT : nullptr;
-      g.gb_in = c->gb[l];
-      ProfScope ps(c, "gemm_dw_sgd", st);
-      if ((e = launch_gemm(kEpiDw, c->mGT[l], l == 0 ? c->mAT0s[s] : c->mAT[l], g, na, st)) != cudaSuccess) return e;
+    if (c->n_br > 1) {
+      if ((e = cudaEventRecord(c->br_join[g], sg)) != cudaSuccess) return e;
+      if ((e = cudaStreamWaitEvent(st, c->br_join[g], 0)) != cudaSuccess) return e;
     }
   }
   const int nc = c->B / kRowsPerLossChunk;
@@ -733,6 +799,8 @@ oscars_status oscars_create(const oscars_config* cfg, oscars_ctx** out) {
           }
         }
         if (st == OSCARS_OK && !cfg->init_params) st = fail(c, OSCARS_EINVAL, "MLP: init_params is NULL");
+        // bf16 MLP rounds fork into up to 16 concurrent branches (flag bit 2: one stream)
+        c->n_br = (c->bf16 && c->L >= 2 && !(cfg->flags & 4)) ? std::min(c->W, kMaxBranches) : 1;
         if (st == OSCARS_OK) st = allocate_mlp(c);
         if (st == OSCARS_OK) st = build_tables(c);
         if (st == OSCARS_OK) {
@@ -744,6 +812,19 @@ oscars_status oscars_create(const oscars_config* cfg, oscars_ctx** out) {
         if (st == OSCARS_OK && cudaStreamCreateWithFlags(&c->cap, cudaStreamNonBlocking) != cudaSuccess)
           st = fail(c, OSCARS_ECUDA, "stream creation failed");
         c->flags = cfg->flags;
+        for (int g = 1; st == OSCARS_OK && c->n_br > 1 && g <= c->n_br; ++g) {
+          cudaStream_t bs;
+          cudaEvent_t ev;
+          if (cudaStreamCreateWithFlags(&bs, cudaStreamNonBlocking) != cudaSuccess ||
+              cudaEventCreateWithFlags(&ev, cudaEventDisableTiming) != cudaSuccess) {
+            st = fail(c, OSCARS_ECUDA, "stream creation failed");
+            break;
+          }
+          c->br_streams.push_back(bs);
+          c->br_join.push_back(ev);
+        }
+        if (st == OSCARS_OK && c->n_br > 1 && cudaEventCreateWithFlags(&c->br_fork, cudaEventDisableTiming) != cudaSuccess)
+          st = fail(c, OSCARS_ECUDA, "event creation failed");
       } else {
         c->flags = cfg->flags;
         if (!dev_alloc(c, &c->slab, c->P_pad)) st = fail(c, OSCARS_ENOMEM, "device allocation failed (global model)");

@@ -382,17 +382,24 @@ __global__ void __launch_bounds__(kHFThreads) head_fused_kernel(const __grid_con
     }
   }
   cluster_sync();
-  // 2. logits = sum of the cluster's partials in rank order; softmax CE
+  // 2. logits = sum of the cluster's partials in rank order (one thread per
+  // (row, class), independent remote loads), then softmax CE per row
   const float* bias = a.master + so + a.offB;
+  for (int q = t; q < B * C; q += kHFThreads) {
+    float part[kHFMaxCluster];
+#pragma unroll
+    for (int r = 0; r < kHFMaxCluster; ++r) part[r] = r < static_cast<int>(ncl) ? ld_dsmem_f32(pl + q, r) : 0.f;
+    float acc = 0.f;
+#pragma unroll
+    for (int r = 0; r < kHFMaxCluster; ++r)
+      if (r < static_cast<int>(ncl)) acc += part[r];
+    dz[q] = acc + bias[q % C];          // logits, replaced by dlogits below
+  }
+  cluster_sync();   // every remote read of pl is done; no CTA leaves before that
   for (int b = t; b < B; b += kHFThreads) {
-    float z[kMaxClasses];
-    float m = -INFINITY;
-    for (int c = 0; c < C; ++c) {
-      float acc = 0.f;
-      for (uint32_t r = 0; r < ncl; ++r) acc += ld_dsmem_f32(pl + b * C + c, r);
-      z[c] = acc + bias[c];
-      m = fmaxf(m, z[c]);
-    }
+    float* z = dz + b * C;
+    float m = z[0];
+    for (int c = 1; c < C; ++c) m = fmaxf(m, z[c]);
     const int y = a.labels[static_cast<int64_t>(w) * B + b];
     float s = 0.f, so_ = 0.f;
     for (int c = 0; c < C; ++c) {
@@ -400,14 +407,14 @@ __global__ void __launch_bounds__(kHFThreads) head_fused_kernel(const __grid_con
       s += e;
       if (c != y) so_ += e;
     }
+    rowloss[b] = m + logf(s) - z[y];
     for (int c = 0; c < C; ++c) {
       const float g = (c == y ? -(so_ / s) : expf(z[c] - m) / s) / static_cast<float>(B);
-      dz[b * C + c] = g;
+      z[c] = g;
       dzb[b * C + c] = bf16_round(g);
     }
-    rowloss[b] = m + logf(s) - z[y];
   }
-  cluster_sync();   // partials are no longer read remotely; dz is complete locally
+  __syncthreads();
   if (rank == 0) {
     if (t < B / kRowsPerLossChunk) {
       float l = 0.f;
