@@ -316,17 +316,24 @@ constexpr int kHFThreads = 256;
 constexpr int kHFGroups = kHFThreads / kHF;
 constexpr int kHFMaxCluster = 8;
 
+// threads per row in the partial-logit phase and the padded row stride of
+// the h tile (row stride / 4 == threads per row (mod 8): the 16-byte reads of
+// one 8-lane phase hit distinct banks)
+__host__ __device__ constexpr int hf_tpr(int B) { return B >= 256 ? 1 : kHFThreads / B; }
+__host__ __device__ constexpr int hf_stride(int B) { return kHF + 4 * hf_tpr(B); }
+
 size_t head_fused_smem(int B, int C) {
-  return sizeof(float) * (static_cast<size_t>(B) * kHF + static_cast<size_t>(C) * kHF + 3 * static_cast<size_t>(B) * C +
-                          kHFGroups * kHF + B) +
+  return sizeof(float) * (static_cast<size_t>(B) * hf_stride(B) + static_cast<size_t>(C) * kHF +
+                          3 * static_cast<size_t>(B) * C + kHFGroups * kHF + B) +
          sizeof(__nv_bfloat16) * static_cast<size_t>(kHF) * (B + 8);
 }
 
 __global__ void __launch_bounds__(kHFThreads) head_fused_kernel(const __grid_constant__ HeadArgs a) {
   extern __shared__ __align__(16) float fsm[];
   const int H = a.H, C = a.C, B = a.B;
-  float* hs = fsm;                         // [B][kHF] bf16 h as float
-  float* wcs = hs + B * kHF;               // [C][kHF] old bf16 head weights as float
+  const int hsd = hf_stride(B);            // padded row stride of the h tile
+  float* hs = fsm;                         // [B][hsd] bf16 h as float
+  float* wcs = hs + B * hsd;               // [C][kHF] old bf16 head weights as float
   float* pl = wcs + C * kHF;               // [B][C] partial logits (read by the cluster)
   float* dz = pl + B * C;                  // [B][C] dlogits fp32
   float* dzb = dz + B * C;                 // [B][C] bf16-rounded
@@ -352,8 +359,8 @@ __global__ void __launch_bounds__(kHFThreads) head_fused_kernel(const __grid_con
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
       const float2 f = __bfloat1622float2(p2[j]);
-      hs[b * kHF + c8 + 2 * j] = f.x;
-      hs[b * kHF + c8 + 2 * j + 1] = f.y;
+      hs[b * hsd + c8 + 2 * j] = f.x;
+      hs[b * hsd + c8 + 2 * j + 1] = f.y;
     }
   }
   for (int q = t; q < C * (kHF / 8); q += kHFThreads) {
@@ -368,17 +375,36 @@ __global__ void __launch_bounds__(kHFThreads) head_fused_kernel(const __grid_con
     }
   }
   __syncthreads();
-  // 1. partial logits: warp per row, each lane 4 features
-  for (int b = warp; b < B; b += kHFThreads / 32) {
-    const float4 hv = *reinterpret_cast<const float4*>(hs + b * kHF + lane * 4);
-    for (int c = 0; c < C; ++c) {
-      const float4 wv = *reinterpret_cast<const float4*>(wcs + c * kHF + lane * 4);
-      float acc = hv.x * wv.x;
-      acc = fmaf(hv.y, wv.y, acc);
-      acc = fmaf(hv.z, wv.z, acc);
-      acc = fmaf(hv.w, wv.w, acc);
-      acc = warp_sum(acc);
-      if (lane == 0) pl[b * C + c] = acc;
+  // 1. partial logits over this CTA's features: `tpr` threads per row, each
+  // takes every tpr-th 4-feature chunk and keeps all classes in registers;
+  // the tpr partial sums of a row are combined with shuffles.
+  {
+    const int tpr = hf_tpr(B);
+    for (int rb = t / tpr; rb < B; rb += kHFThreads / tpr) {
+      const int q = t % tpr;
+      float acc[kMaxClasses];
+#pragma unroll
+      for (int c = 0; c < kMaxClasses; ++c) acc[c] = 0.f;
+      for (int k = 4 * q; k < kHF; k += 4 * tpr) {
+        const float4 hv = *reinterpret_cast<const float4*>(hs + rb * hsd + k);
+#pragma unroll
+        for (int c = 0; c < kMaxClasses; ++c) {
+          if (c < C) {
+            const float4 wv = *reinterpret_cast<const float4*>(wcs + c * kHF + k);
+            acc[c] = fmaf(hv.x, wv.x, acc[c]);
+            acc[c] = fmaf(hv.y, wv.y, acc[c]);
+            acc[c] = fmaf(hv.z, wv.z, acc[c]);
+            acc[c] = fmaf(hv.w, wv.w, acc[c]);
+          }
+        }
+      }
+#pragma unroll
+      for (int c = 0; c < kMaxClasses; ++c) {
+        if (c < C) {
+          for (int o = tpr / 2; o > 0; o >>= 1) acc[c] += __shfl_xor_sync(0xffffffffu, acc[c], o);
+          if (q == 0) pl[rb * C + c] = acc[c];
+        }
+      }
     }
   }
   cluster_sync();
@@ -436,7 +462,7 @@ __global__ void __launch_bounds__(kHFThreads) head_fused_kernel(const __grid_con
     __nv_bfloat16* G = a.G + static_cast<int64_t>(w) * B * H;
     for (int r = 0; r < rows; ++r) {
       const int b = grp * rows + r;
-      const float hv = hs[b * kHF + k];
+      const float hv = hs[b * hsd + k];
       float dh = 0.f;
       for (int c = 0; c < C; ++c) dh = fmaf(dzb[b * C + c], wcs[c * kHF + k], dh);
       const float g = hv > 0.f ? dh : 0.f;
@@ -465,7 +491,7 @@ __global__ void __launch_bounds__(kHFThreads) head_fused_kernel(const __grid_con
   for (int q = t; q < C * kHF; q += kHFThreads) {
     const int c = q / kHF, k = q - c * kHF;
     float dw = 0.f;
-    for (int b = 0; b < B; ++b) dw = fmaf(dzb[b * C + c], hs[b * kHF + k], dw);
+    for (int b = 0; b < B; ++b) dw = fmaf(dzb[b * C + c], hs[b * hsd + k], dw);
     const int64_t e = a.offW + static_cast<int64_t>(c) * H + k0 + k;
     const float nw = fmaf(-a.lr, dw, a.master[so + e]);
     a.master_w[dof + e] = nw;
