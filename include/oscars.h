@@ -99,7 +99,10 @@ typedef struct {
   int32_t flags;                 /* bit 0: launch each kernel of a round directly */
                                  /* instead of replaying a captured CUDA graph;   */
                                  /* bit 1 (with bit 0): time every launch with    */
-                                 /* CUDA events (see oscars_profile_read)         */
+                                 /* CUDA events (see oscars_profile_read);        */
+                                 /* bit 2: run the workers of a round as up to 16 */
+                                 /* concurrent branches (streams) instead of one  */
+                                 /* launch per layer over all active workers      */
 } oscars_config;
 
 /*

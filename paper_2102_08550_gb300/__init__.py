@@ -21,6 +21,7 @@ W_UNIFORM, W_LOCALSTEPS, W_EXPLICIT = 0, 1, 2
 SEARCH_CAPPED, SEARCH_LITERAL = 0, 1
 FLAG_NO_GRAPH = 1
 FLAG_PROFILE = 2
+FLAG_BRANCHES = 4
 
 
 class OscarsError(RuntimeError):

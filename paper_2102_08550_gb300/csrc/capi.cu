@@ -799,8 +799,8 @@ oscars_status oscars_create(const oscars_config* cfg, oscars_ctx** out) {
           }
         }
         if (st == OSCARS_OK && !cfg->init_params) st = fail(c, OSCARS_EINVAL, "MLP: init_params is NULL");
-        // bf16 MLP rounds fork into up to 16 concurrent branches (flag bit 2: one stream)
-        c->n_br = (c->bf16 && c->L >= 2 && !(cfg->flags & 4)) ? std::min(c->W, kMaxBranches) : 1;
+        // flag bit 2: bf16 MLP rounds fork into up to 16 concurrent worker branches
+        c->n_br = (c->bf16 && c->L >= 2 && (cfg->flags & 4)) ? std::min(c->W, kMaxBranches) : 1;
         if (st == OSCARS_OK) st = allocate_mlp(c);
         if (st == OSCARS_OK) st = build_tables(c);
         if (st == OSCARS_OK) {

@@ -300,68 +300,73 @@ __global__ void __launch_bounds__(kHeadBwdThreads) head_bwd_kernel(const __grid_
 }
 
 // ---------------------------------------------------------------- fused head
-// Forward and backward of the last layer (C <= 32 classes) in one launch.
-// A cluster of H/128 CTAs serves one active lane; CTA r owns hidden features
-// [128 r, 128 r + 128):
-//  1. partial logits over its features, pl[b][c] (warp per row, lanes over k);
-//  2. cluster barrier; every CTA sums the partials of ranks 0..n-1 in that
-//     order from distributed shared memory, so all CTAs hold the same logits,
-//     and runs the softmax cross-entropy (no cancellation: see head_fwd);
+// Forward and backward of the last layer in one launch, specialised for a
+// compile-time class count C.  A cluster of H/128 CTAs serves one active
+// lane; CTA r owns hidden features [128 r, 128 r + 128):
+//  1. partial logits over its features (tpr threads per row, each over an
+//     interleaved set of 4-feature chunks, all C classes in registers);
+//  2. cluster barrier; the logits are the partials of ranks 0..n-1 summed in
+//     that order from distributed shared memory (so every CTA holds the same
+//     values), then the softmax cross-entropy without cancellation;
 //  3. a second cluster barrier (no CTA leaves while others read its partials);
-//  4. backward for its features exactly as head_bwd: masked input gradient
-//     (bf16 G, G^T, fp32 bias gradient), head weight gradient + SGD.
+//  4. masked input gradient of the layer below for its features: item =
+//     (row, 4 features), the 4 x C old weights stay in registers -> bf16 G,
+//     G^T (through shared memory) and the fp32 bias gradient;
+//  5. head weight gradient + SGD: item = (class, 4 features).
 // Rank 0 also writes the loss partials and updates the head bias.
 constexpr int kHF = 128;                 // hidden features per CTA
 constexpr int kHFThreads = 256;
-constexpr int kHFGroups = kHFThreads / kHF;
+constexpr int kHFWarps = kHFThreads / 32;
 constexpr int kHFMaxCluster = 8;
+constexpr int kHFClasses = 10;           // the fused path's class count
 
-// threads per row in the partial-logit phase and the padded row stride of
-// the h tile (row stride / 4 == threads per row (mod 8): the 16-byte reads of
-// one 8-lane phase hit distinct banks)
+// threads per row in phase 1 and the padded row stride of the h tile (row
+// stride / 4 == threads per row (mod 8): the 16-byte reads of one 8-lane
+// phase hit distinct banks)
 __host__ __device__ constexpr int hf_tpr(int B) { return B >= 256 ? 1 : kHFThreads / B; }
 __host__ __device__ constexpr int hf_stride(int B) { return kHF + 4 * hf_tpr(B); }
 
 size_t head_fused_smem(int B, int C) {
   return sizeof(float) * (static_cast<size_t>(B) * hf_stride(B) + static_cast<size_t>(C) * kHF +
-                          3 * static_cast<size_t>(B) * C + kHFGroups * kHF + B) +
+                          3 * static_cast<size_t>(B) * C + kHFWarps * kHF + B) +
          sizeof(__nv_bfloat16) * static_cast<size_t>(kHF) * (B + 8);
 }
 
+template <int C>
 __global__ void __launch_bounds__(kHFThreads) head_fused_kernel(const __grid_constant__ HeadArgs a) {
   extern __shared__ __align__(16) float fsm[];
-  const int H = a.H, C = a.C, B = a.B;
-  const int hsd = hf_stride(B);            // padded row stride of the h tile
+  const int H = a.H, B = a.B;
+  const int hsd = hf_stride(B);
   float* hs = fsm;                         // [B][hsd] bf16 h as float
   float* wcs = hs + B * hsd;               // [C][kHF] old bf16 head weights as float
   float* pl = wcs + C * kHF;               // [B][C] partial logits (read by the cluster)
-  float* dz = pl + B * C;                  // [B][C] dlogits fp32
-  float* dzb = dz + B * C;                 // [B][C] bf16-rounded
-  float* gbp = dzb + B * C;                // [kHFGroups][kHF]
-  float* rowloss = gbp + kHFGroups * kHF;  // [B]
+  float* dz = pl + B * C;                  // [B][C] logits, then dlogits fp32
+  float* dzb = dz + B * C;                 // [B][C] bf16-rounded dlogits
+  float* gbp = dzb + B * C;                // [kHFWarps][kHF] bias-gradient partials
+  float* rowloss = gbp + kHFWarps * kHF;   // [B]
   __nv_bfloat16* gts = reinterpret_cast<__nv_bfloat16*>(rowloss + B);   // [kHF][B + 8]
   const int gts_ld = B + 8;
   const int i = blockIdx.x;
   const int w = a.wid[i], src = a.src[i];
   const uint32_t rank = cluster_ctarank();
-  const uint32_t ncl = gridDim.y;
+  const int ncl = static_cast<int>(gridDim.y);
   const int k0 = blockIdx.y * kHF;
   const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
   const int64_t so = static_cast<int64_t>(src) * a.slot_stride;
   const int64_t dof = static_cast<int64_t>(w) * a.slot_stride;
   const __nv_bfloat16* h = a.Ain + static_cast<int64_t>(w) * B * H;
 
-  // stage this CTA's slice of h and of the head weights
   for (int q = t; q < B * (kHF / 8); q += kHFThreads) {
     const int b = q / (kHF / 8), c8 = (q % (kHF / 8)) * 8;
     const uint4 v = *reinterpret_cast<const uint4*>(h + static_cast<int64_t>(b) * H + k0 + c8);
     const __nv_bfloat162* p2 = reinterpret_cast<const __nv_bfloat162*>(&v);
-#pragma unroll
-    for (int j = 0; j < 4; ++j) {
-      const float2 f = __bfloat1622float2(p2[j]);
-      hs[b * hsd + c8 + 2 * j] = f.x;
-      hs[b * hsd + c8 + 2 * j + 1] = f.y;
-    }
+    float4 lo, hi;
+    float2 f = __bfloat1622float2(p2[0]); lo.x = f.x; lo.y = f.y;
+    f = __bfloat1622float2(p2[1]); lo.z = f.x; lo.w = f.y;
+    f = __bfloat1622float2(p2[2]); hi.x = f.x; hi.y = f.y;
+    f = __bfloat1622float2(p2[3]); hi.z = f.x; hi.w = f.y;
+    *reinterpret_cast<float4*>(hs + b * hsd + c8) = lo;
+    *reinterpret_cast<float4*>(hs + b * hsd + c8 + 4) = hi;
   }
   for (int q = t; q < C * (kHF / 8); q += kHFThreads) {
     const int c = q / (kHF / 8), c8 = (q % (kHF / 8)) * 8;
@@ -375,68 +380,69 @@ __global__ void __launch_bounds__(kHFThreads) head_fused_kernel(const __grid_con
     }
   }
   __syncthreads();
-  // 1. partial logits over this CTA's features: `tpr` threads per row, each
-  // takes every tpr-th 4-feature chunk and keeps all classes in registers;
-  // the tpr partial sums of a row are combined with shuffles.
+
+  // 1. partial logits
   {
     const int tpr = hf_tpr(B);
-    for (int rb = t / tpr; rb < B; rb += kHFThreads / tpr) {
-      const int q = t % tpr;
-      float acc[kMaxClasses];
+    const int rb = t / tpr, q = t % tpr;
+    if (rb < B) {
+      float acc[C];
 #pragma unroll
-      for (int c = 0; c < kMaxClasses; ++c) acc[c] = 0.f;
+      for (int c = 0; c < C; ++c) acc[c] = 0.f;
       for (int k = 4 * q; k < kHF; k += 4 * tpr) {
         const float4 hv = *reinterpret_cast<const float4*>(hs + rb * hsd + k);
 #pragma unroll
-        for (int c = 0; c < kMaxClasses; ++c) {
-          if (c < C) {
-            const float4 wv = *reinterpret_cast<const float4*>(wcs + c * kHF + k);
-            acc[c] = fmaf(hv.x, wv.x, acc[c]);
-            acc[c] = fmaf(hv.y, wv.y, acc[c]);
-            acc[c] = fmaf(hv.z, wv.z, acc[c]);
-            acc[c] = fmaf(hv.w, wv.w, acc[c]);
-          }
+        for (int c = 0; c < C; ++c) {
+          const float4 wv = *reinterpret_cast<const float4*>(wcs + c * kHF + k);
+          acc[c] = fmaf(hv.x, wv.x, acc[c]);
+          acc[c] = fmaf(hv.y, wv.y, acc[c]);
+          acc[c] = fmaf(hv.z, wv.z, acc[c]);
+          acc[c] = fmaf(hv.w, wv.w, acc[c]);
         }
       }
 #pragma unroll
-      for (int c = 0; c < kMaxClasses; ++c) {
-        if (c < C) {
-          for (int o = tpr / 2; o > 0; o >>= 1) acc[c] += __shfl_xor_sync(0xffffffffu, acc[c], o);
-          if (q == 0) pl[rb * C + c] = acc[c];
-        }
+      for (int c = 0; c < C; ++c) {
+        for (int o = tpr / 2; o > 0; o >>= 1) acc[c] += __shfl_xor_sync(0xffffffffu, acc[c], o);
+        if (q == 0) pl[rb * C + c] = acc[c];
       }
     }
   }
   cluster_sync();
-  // 2. logits = sum of the cluster's partials in rank order (one thread per
-  // (row, class), independent remote loads), then softmax CE per row
+  // 2. logits (cluster sum in rank order), softmax cross-entropy
   const float* bias = a.master + so + a.offB;
   for (int q = t; q < B * C; q += kHFThreads) {
     float part[kHFMaxCluster];
 #pragma unroll
-    for (int r = 0; r < kHFMaxCluster; ++r) part[r] = r < static_cast<int>(ncl) ? ld_dsmem_f32(pl + q, r) : 0.f;
+    for (int r = 0; r < kHFMaxCluster; ++r) part[r] = r < ncl ? ld_dsmem_f32(pl + q, r) : 0.f;
     float acc = 0.f;
 #pragma unroll
     for (int r = 0; r < kHFMaxCluster; ++r)
-      if (r < static_cast<int>(ncl)) acc += part[r];
-    dz[q] = acc + bias[q % C];          // logits, replaced by dlogits below
+      if (r < ncl) acc += part[r];
+    dz[q] = acc + bias[q % C];
   }
-  cluster_sync();   // every remote read of pl is done; no CTA leaves before that
+  cluster_sync();   // every remote read of pl is done
   for (int b = t; b < B; b += kHFThreads) {
-    float* z = dz + b * C;
+    float z[C];
+#pragma unroll
+    for (int c = 0; c < C; ++c) z[c] = dz[b * C + c];
     float m = z[0];
+#pragma unroll
     for (int c = 1; c < C; ++c) m = fmaxf(m, z[c]);
     const int y = a.labels[static_cast<int64_t>(w) * B + b];
-    float s = 0.f, so_ = 0.f;
+    float e[C], s = 0.f, so_ = 0.f, zy = 0.f;
+#pragma unroll
     for (int c = 0; c < C; ++c) {
-      const float e = expf(z[c] - m);
-      s += e;
-      if (c != y) so_ += e;
+      e[c] = expf(z[c] - m);
+      s += e[c];
+      if (c != y) so_ += e[c];
+      else zy = z[c];
     }
-    rowloss[b] = m + logf(s) - z[y];
+    rowloss[b] = m + logf(s) - zy;
+    const float inv = 1.0f / static_cast<float>(B);
+#pragma unroll
     for (int c = 0; c < C; ++c) {
-      const float g = (c == y ? -(so_ / s) : expf(z[c] - m) / s) / static_cast<float>(B);
-      z[c] = g;
+      const float g = (c == y ? -(so_ / s) : e[c] / s) * inv;
+      dz[b * C + c] = g;
       dzb[b * C + c] = bf16_round(g);
     }
   }
@@ -448,35 +454,59 @@ __global__ void __launch_bounds__(kHFThreads) head_fused_kernel(const __grid_con
       const int64_t row = static_cast<int64_t>(w) * a.part_mul + a.part_add;
       a.loss_part[row * (B / kRowsPerLossChunk) + t] = l;
     }
-    if (t < C) {
+    // head bias: db[c] = sum_b dz[b][c]; 16 threads per class, then shuffles
+    if (t < C * 16) {
+      const int c = t >> 4, j = t & 15;
       float g = 0.f;
-      for (int b = 0; b < B; ++b) g += dz[b * C + t];
-      a.master_w[dof + a.offB + t] = fmaf(-a.lr, g, a.master[so + a.offB + t]);
+      for (int b = j; b < B; b += 16) g += dz[b * C + c];
+#pragma unroll
+      for (int o = 8; o > 0; o >>= 1) g += __shfl_xor_sync(0xffffffffu, g, o, 16);
+      if (j == 0) a.master_w[dof + a.offB + c] = fmaf(-a.lr, g, a.master[so + a.offB + c]);
     }
   }
-  // 3. masked input gradient of the layer below for this CTA's features
+  // 4. masked input gradient of the layer below: item = (row, 4 features)
   {
-    const int k = t % kHF, grp = t / kHF;
-    const int rows = B / kHFGroups;
-    float gsum = 0.f;
-    __nv_bfloat16* G = a.G + static_cast<int64_t>(w) * B * H;
-    for (int r = 0; r < rows; ++r) {
-      const int b = grp * rows + r;
-      const float hv = hs[b * hsd + k];
-      float dh = 0.f;
-      for (int c = 0; c < C; ++c) dh = fmaf(dzb[b * C + c], wcs[c * kHF + k], dh);
-      const float g = hv > 0.f ? dh : 0.f;
-      gsum += g;
-      const __nv_bfloat16 g16 = __float2bfloat16_rn(g);
-      G[static_cast<int64_t>(b) * H + k0 + k] = g16;
-      gts[k * gts_ld + b] = g16;
+    const int k4 = (t & 31) * 4;           // this thread's 4 features
+    float4 wc[C];
+#pragma unroll
+    for (int c = 0; c < C; ++c) wc[c] = *reinterpret_cast<const float4*>(wcs + c * kHF + k4);
+    float4 gs = make_float4(0.f, 0.f, 0.f, 0.f);
+    __nv_bfloat16* G = a.G + static_cast<int64_t>(w) * B * H + k0 + k4;
+    for (int b = warp; b < B; b += kHFWarps) {
+      const float4 hv = *reinterpret_cast<const float4*>(hs + b * hsd + k4);
+      float4 dh = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+      for (int c = 0; c < C; ++c) {
+        const float g = dzb[b * C + c];
+        dh.x = fmaf(g, wc[c].x, dh.x);
+        dh.y = fmaf(g, wc[c].y, dh.y);
+        dh.z = fmaf(g, wc[c].z, dh.z);
+        dh.w = fmaf(g, wc[c].w, dh.w);
+      }
+      dh.x = hv.x > 0.f ? dh.x : 0.f;
+      dh.y = hv.y > 0.f ? dh.y : 0.f;
+      dh.z = hv.z > 0.f ? dh.z : 0.f;
+      dh.w = hv.w > 0.f ? dh.w : 0.f;
+      gs.x += dh.x;
+      gs.y += dh.y;
+      gs.z += dh.z;
+      gs.w += dh.w;
+      const __nv_bfloat162 p01 = __floats2bfloat162_rn(dh.x, dh.y);
+      const __nv_bfloat162 p23 = __floats2bfloat162_rn(dh.z, dh.w);
+      *reinterpret_cast<uint2*>(G + static_cast<int64_t>(b) * H) =
+          make_uint2(*reinterpret_cast<const uint32_t*>(&p01), *reinterpret_cast<const uint32_t*>(&p23));
+      gts[(k4 + 0) * gts_ld + b] = p01.x;
+      gts[(k4 + 1) * gts_ld + b] = p01.y;
+      gts[(k4 + 2) * gts_ld + b] = p23.x;
+      gts[(k4 + 3) * gts_ld + b] = p23.y;
     }
-    gbp[grp * kHF + k] = gsum;
+    *reinterpret_cast<float4*>(gbp + warp * kHF + k4) = gs;
   }
   __syncthreads();
   if (t < kHF) {
     float g = 0.f;
-    for (int grp = 0; grp < kHFGroups; ++grp) g += gbp[grp * kHF + t];
+#pragma unroll
+    for (int r = 0; r < kHFWarps; ++r) g += gbp[r * kHF + t];
     a.gb[static_cast<int64_t>(w) * H + k0 + t] = g;
   }
   {
@@ -487,15 +517,27 @@ __global__ void __launch_bounds__(kHFThreads) head_fused_kernel(const __grid_con
       GT[static_cast<int64_t>(k) * per_row + j] = *reinterpret_cast<const uint4*>(gts + k * gts_ld + j * 8);
     }
   }
-  // 4. head weight gradient and SGD for this CTA's features
-  for (int q = t; q < C * kHF; q += kHFThreads) {
-    const int c = q / kHF, k = q - c * kHF;
-    float dw = 0.f;
-    for (int b = 0; b < B; ++b) dw = fmaf(dzb[b * C + c], hs[b * hsd + k], dw);
-    const int64_t e = a.offW + static_cast<int64_t>(c) * H + k0 + k;
-    const float nw = fmaf(-a.lr, dw, a.master[so + e]);
-    a.master_w[dof + e] = nw;
-    a.shadow_w[dof + e] = __float2bfloat16_rn(nw);
+  // 5. head weight gradient + SGD: item = (class, 4 features)
+  for (int q = t; q < C * (kHF / 4); q += kHFThreads) {
+    const int c = q / (kHF / 4), k4 = (q % (kHF / 4)) * 4;
+    float4 dw = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int b = 0; b < B; ++b) {
+      const float g = dzb[b * C + c];
+      const float4 hv = *reinterpret_cast<const float4*>(hs + b * hsd + k4);
+      dw.x = fmaf(g, hv.x, dw.x);
+      dw.y = fmaf(g, hv.y, dw.y);
+      dw.z = fmaf(g, hv.z, dw.z);
+      dw.w = fmaf(g, hv.w, dw.w);
+    }
+    const int64_t e = a.offW + static_cast<int64_t>(c) * H + k0 + k4;
+    const float4 o = *reinterpret_cast<const float4*>(a.master + so + e);
+    float4 nw;
+    nw.x = fmaf(-a.lr, dw.x, o.x);
+    nw.y = fmaf(-a.lr, dw.y, o.y);
+    nw.z = fmaf(-a.lr, dw.z, o.z);
+    nw.w = fmaf(-a.lr, dw.w, o.w);
+    *reinterpret_cast<float4*>(a.master_w + dof + e) = nw;
+    *reinterpret_cast<uint2*>(a.shadow_w + dof + e) = make_uint2(pack_bf16x2(nw.x, nw.y), pack_bf16x2(nw.z, nw.w));
   }
 }
 
@@ -594,14 +636,14 @@ cudaError_t launch_head_bwd(const HeadArgs& a, int n_active, cudaStream_t s) {
 }
 
 bool head_fused_supported(int H, int B, int C) {
-  return H % kHF == 0 && H / kHF <= kHFMaxCluster && B % (8 * kHFGroups) == 0 && B % kRowsPerLossChunk == 0 &&
-         B / kRowsPerLossChunk <= kHFThreads && C <= kMaxClasses && head_fused_smem(B, C) <= 220 * 1024;
+  return C == kHFClasses && H % kHF == 0 && H / kHF <= kHFMaxCluster && B % 32 == 0 && B <= 256 &&
+         head_fused_smem(B, C) <= 220 * 1024;
 }
 
 cudaError_t launch_head_fused(const HeadArgs& a, int n_active, cudaStream_t s) {
   if (!head_fused_supported(a.H, a.B, a.C)) return cudaErrorInvalidValue;
   const size_t smem = head_fused_smem(a.B, a.C);
-  cudaError_t e = cudaFuncSetAttribute(head_fused_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  cudaError_t e = cudaFuncSetAttribute(head_fused_kernel<kHFClasses>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(smem));
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
@@ -616,7 +658,7 @@ cudaError_t launch_head_fused(const HeadArgs& a, int n_active, cudaStream_t s) {
   attr[0].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, head_fused_kernel, a);
+  return cudaLaunchKernelEx(&cfg, head_fused_kernel<kHFClasses>, a);
 }
 
 cudaError_t launch_loss_finalize(const float* part, const int32_t* tau, int W, int max_tau, int nc, int B,
