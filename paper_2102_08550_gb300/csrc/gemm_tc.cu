@@ -99,37 +99,29 @@ __device__ __forceinline__ float epi_dh(const GemmArgs& a, int wid, int m, int n
 }
 
 // Weight gradient + SGD for one 32 x 32 block: rows m_base .. m_base + 31
-// (thread `lane` holds row m_base + lane in v), columns n_base .. n_base + 31.
-// The block goes through a padded shared-memory tile so that the fp32
-// master read-modify-write and the bf16 shadow write move full lines (lane =
-// column), while the transposed shadow is written from the row layout
-// (lane = row, consecutive addresses).
-__device__ __forceinline__ void epi_dw_block(const GemmArgs& a, int wid, int src, int m_base, int n_base,
-                                             const float (&v)[32], float* T, int lane) {
+// (thread `lane` holds row m_base + lane in v), columns n_base .. n_base + 31;
+// `old` holds the block's fp32 master values already loaded as
+// old[r] = master[src][m_base + r][n_base + lane] (lane = column).
+// The accumulators go through a padded shared-memory tile so that the fp32
+// master write and the bf16 shadow write move full lines (lane = column),
+// while the transposed shadow is written from the row layout (lane = row).
+__device__ __forceinline__ void epi_dw_block(const GemmArgs& a, int wid, int m_base, int n_base,
+                                             const float (&v)[32], const float (&old)[32], float* T, int lane) {
 #pragma unroll
   for (int j = 0; j < 32; ++j) T[lane * 33 + j] = v[j];
   __syncwarp();
   const int n = n_base + lane;
   const bool nok = n < a.N;
-  const int64_t so = static_cast<int64_t>(src) * a.slot_stride + a.offW + n;
   const int64_t dof = static_cast<int64_t>(wid) * a.slot_stride + a.offW + n;
 #pragma unroll
-  for (int r0 = 0; r0 < 32; r0 += 8) {
-    float old[8];
-#pragma unroll
-    for (int i = 0; i < 8; ++i)
-      old[i] = nok ? a.master[so + static_cast<int64_t>(m_base + r0 + i) * a.N] : 0.f;
-#pragma unroll
-    for (int i = 0; i < 8; ++i) {
-      const int r = r0 + i;
-      const float nw = fmaf(-a.lr, T[r * 33 + lane], old[i]);
-      if (nok) {
-        const int64_t e = dof + static_cast<int64_t>(m_base + r) * a.N;
-        a.master_w[e] = nw;
-        a.shadow[e] = __float2bfloat16_rn(nw);
-      }
-      T[r * 33 + lane] = nw;
+  for (int r = 0; r < 32; ++r) {
+    const float nw = fmaf(-a.lr, T[r * 33 + lane], old[r]);
+    if (nok) {
+      const int64_t e = dof + static_cast<int64_t>(m_base + r) * a.N;
+      a.master_w[e] = nw;
+      a.shadow[e] = __float2bfloat16_rn(nw);
     }
+    T[r * 33 + lane] = nw;
   }
   __syncwarp();
   if (a.shadowT) {
@@ -139,6 +131,17 @@ __device__ __forceinline__ void epi_dw_block(const GemmArgs& a, int wid, int src
       if (n_base + j < a.N) t[static_cast<int64_t>(n_base + j) * a.M] = __float2bfloat16_rn(T[lane * 33 + j]);
   }
   __syncwarp();
+}
+
+// old[r] = master[src][m_base + r][n_base + lane] (0 outside N): one
+// coalesced line per row, all 32 loads issued before any is used
+__device__ __forceinline__ void epi_dw_load(const GemmArgs& a, int src, int m_base, int n_base, int lane,
+                                            float (&old)[32]) {
+  const int n = n_base + lane;
+  const bool nok = n < a.N;
+  const int64_t so = static_cast<int64_t>(src) * a.slot_stride + a.offW + n;
+#pragma unroll
+  for (int r = 0; r < 32; ++r) old[r] = nok ? a.master[so + static_cast<int64_t>(m_base + r) * a.N] : 0.f;
 }
 
 __device__ __forceinline__ void epi_store(const GemmArgs& a, int m, int n0, const float (&v)[32]) {
@@ -234,16 +237,23 @@ __global__ void __launch_bounds__(warps_for<EPI>() * 32) gemm_tc_kernel(const __
     const int quarter = warp & 3;
     const int m = m0 + quarter * 32 + lane;
     const uint32_t trow = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
-    if (EPI == kEpiDw) {
-      constexpr int kHalf = BN / 2;
-      const int c_begin = (warp >> 2) * kHalf;
+    if constexpr (EPI == kEpiDw) {
+      static_assert(BN == 128, "the weight-gradient epilogue covers 2 x 32 columns per warp");
+      const int c_begin = (warp >> 2) * (BN / 2);
+      const int mb = m0 + quarter * 32;
       float* T = epi_tiles + warp * kEpiTileFloats;
-#pragma unroll 1
-      for (int c0 = c_begin; c0 < c_begin + kHalf; c0 += 32) {
-        if (n0 + c0 >= a.N) break;   // uniform in the warp
+      float old0[32], old1[32];
+      epi_dw_load(a, src, mb, n0 + c_begin, lane, old0);        // both chunks' loads in flight
+      epi_dw_load(a, src, mb, n0 + c_begin + 32, lane, old1);
+      if (n0 + c_begin < a.N) {
         float v[32];
-        tmem_ld_32x32b_x32(trow + c0, v);
-        epi_dw_block(a, wid, src, m0 + quarter * 32, n0 + c0, v, T, lane);
+        tmem_ld_32x32b_x32(trow + c_begin, v);
+        epi_dw_block(a, wid, mb, n0 + c_begin, v, old0, T, lane);
+      }
+      if (n0 + c_begin + 32 < a.N) {
+        float v[32];
+        tmem_ld_32x32b_x32(trow + c_begin + 32, v);
+        epi_dw_block(a, wid, mb, n0 + c_begin + 32, v, old1, T, lane);
       }
       if (warp < 4 && blockIdx.y == 0) {
         const int64_t bo = a.offB + m;
@@ -288,7 +298,10 @@ cudaError_t launch_tile(const CUtensorMap& mA, const CUtensorMap& mB, const Gemm
                         cudaStream_t s) {
   using Cfg = TileCfg<BN>;
   const int nk = (a.K + BK - 1) / BK;
-  const int stages = nk < 4 ? nk : 4;
+  // as many stages as K-blocks, within ~200 KB of shared memory: the whole
+  // K extent of these skinny GEMMs is then in flight at once
+  const int max_stages = static_cast<int>((200 * 1024 - (EPI == kEpiDw ? 8 * 32 * 33 * 4 : 0)) / Cfg::kStageBytes);
+  const int stages = nk < max_stages ? nk : (max_stages < 8 ? max_stages : 8);
   constexpr int kWarps = warps_for<EPI>();
   size_t smem = 1024 + static_cast<size_t>(stages) * Cfg::kStageBytes + kBarrierBytes +
                 (EPI == kEpiDw ? sizeof(float) * kWarps * kEpiTileFloats : 0);
