@@ -232,8 +232,9 @@ def run_gpu(args, rank, world, local_rank):
     torch.cuda.synchronize()
     value = samples_per_round * args.steps * world / (total_ms / 1e3)
 
-    # ---- per-kernel device time: the same rounds with each launch timed
-    pctx = make(flags=P.FLAG_NO_GRAPH | P.FLAG_PROFILE)
+    # ---- per-kernel device time: the same round graph with an event node
+    # around every kernel (device timeline, no host launch gaps)
+    pctx = make(flags=P.FLAG_PROFILE)
     for _ in range(2):
         P.oscars_local_steps(pctx.handle, want_tau=False, want_loss=False)
         P.oscars_push_merge(pctx.handle)

@@ -98,8 +98,9 @@ typedef struct {
   void* cuda_stream;             /* cudaStream_t, borrowed; NULL = default stream */
   int32_t flags;                 /* bit 0: launch each kernel of a round directly */
                                  /* instead of replaying a captured CUDA graph;   */
-                                 /* bit 1 (with bit 0): time every launch with    */
-                                 /* CUDA events (see oscars_profile_read);        */
+                                 /* bit 1: time every launch with CUDA events     */
+                                 /* (graph mode: event nodes in the graph; see    */
+                                 /* oscars_profile_read);                         */
                                  /* bit 2: run the workers of a round as up to 16 */
                                  /* concurrent branches (streams) instead of one  */
                                  /* launch per layer over all active workers      */
@@ -201,8 +202,9 @@ oscars_status oscars_read_replica(oscars_ctx* ctx, int32_t k, float* dst);
 
 /*
  * oscars_profile_read - per-kernel-class device time of the launches made
- * since the last reset while flag bits 0 and 1 were set (CUDA events recorded
- * on the context's stream around every launch).  Synchronises on the last
+ * since the last reset while flag bit 1 was set (CUDA events around every
+ * launch on its stream; in graph mode they are event nodes of the captured
+ * graph, so the times exclude host launch gaps).  Synchronises on the last
  * recorded event.  Fills up to `cap` entries: names[i] (library-owned, valid
  * until the next reset or destroy), ms_total[i], launches[i] (each may be
  * NULL).  Returns the number of classes, or -1 for a NULL ctx.

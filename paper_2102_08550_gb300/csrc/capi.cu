@@ -147,8 +147,12 @@ struct oscars_ctx {
   struct ProfEntry {
     const char* name;
     cudaEvent_t a, b;
+    bool graph_owned;   // recorded by an event node of a captured graph: never recycled
   };
   std::vector<ProfEntry> prof_pending;
+  std::vector<ProfEntry> prof_round_graph, prof_merge_graph;   // event nodes of the captured graphs
+  std::vector<ProfEntry>* prof_sink = nullptr;                  // where ProfScope files entries
+  cudaGraphExec_t merge_exec = nullptr;                         // replica-mode merge + shadow refresh
   std::vector<cudaEvent_t> prof_pool;
   std::vector<std::string> prof_names;
   std::vector<double> prof_ms;
@@ -179,6 +183,9 @@ cudaEvent_t prof_event(oscars_ctx* c) {
   return e;
 }
 
+// Events around one launch.  Recorded with cudaEventRecordExternal, so that
+// inside a stream capture they become event nodes of the graph and time the
+// kernel on the device timeline (no host launch gaps).
 struct ProfScope {
   oscars_ctx* c;
   const char* name;
@@ -187,14 +194,17 @@ struct ProfScope {
   ProfScope(oscars_ctx* c_, const char* n, cudaStream_t s_) : c(c_), name(n), s(s_) {
     if (c->profiling) {
       a = prof_event(c);
-      cudaEventRecord(a, s);
+      cudaEventRecordWithFlags(a, s, cudaEventRecordExternal);
     }
   }
   ~ProfScope() {
     if (a) {
       cudaEvent_t b = prof_event(c);
-      cudaEventRecord(b, s);
-      c->prof_pending.push_back({name, a, b});
+      cudaEventRecordWithFlags(b, s, cudaEventRecordExternal);
+      if (c->prof_sink)
+        c->prof_sink->push_back({name, a, b, true});
+      else
+        c->prof_pending.push_back({name, a, b, false});
     }
   }
 };
@@ -215,10 +225,19 @@ void prof_collect(oscars_ctx* c) {
     }
     c->prof_ms[i] += ms;
     c->prof_count[i] += 1;
-    c->prof_pool.push_back(p.a);
-    c->prof_pool.push_back(p.b);
+    if (!p.graph_owned) {
+      c->prof_pool.push_back(p.a);
+      c->prof_pool.push_back(p.b);
+    }
   }
   c->prof_pending.clear();
+}
+
+// after a replay of a profiled graph: queue its event nodes for collection
+void prof_after_replay(oscars_ctx* c, const std::vector<oscars_ctx::ProfEntry>& g) {
+  if (g.empty()) return;
+  for (const auto& e : g) c->prof_pending.push_back(e);
+  prof_collect(c);   // read now: the next replay records the same events again
 }
 
 template <typename T>
@@ -235,11 +254,21 @@ bool dev_alloc(oscars_ctx* c, T** p, size_t count) {
 }
 
 void free_all(oscars_ctx* c) {
-  for (auto& p : c->prof_pending) {
-    cudaEventDestroy(p.a);
-    cudaEventDestroy(p.b);
-  }
+  for (auto& p : c->prof_pending)
+    if (!p.graph_owned) {
+      cudaEventDestroy(p.a);
+      cudaEventDestroy(p.b);
+    }
   c->prof_pending.clear();
+  for (auto* v : {&c->prof_round_graph, &c->prof_merge_graph}) {
+    for (auto& p : *v) {
+      cudaEventDestroy(p.a);
+      cudaEventDestroy(p.b);
+    }
+    v->clear();
+  }
+  if (c->merge_exec) cudaGraphExecDestroy(c->merge_exec);
+  c->merge_exec = nullptr;
   for (cudaEvent_t e : c->prof_pool) cudaEventDestroy(e);
   c->prof_pool.clear();
   if (c->round_exec) cudaGraphExecDestroy(c->round_exec);
@@ -353,6 +382,10 @@ oscars_status build_tables(oscars_ctx* c) {
   if (c->round_exec) {
     cudaGraphExecDestroy(c->round_exec);
     c->round_exec = nullptr;
+  }
+  if (c->merge_exec) {
+    cudaGraphExecDestroy(c->merge_exec);
+    c->merge_exec = nullptr;
   }
   return ensure_stage_buffers(c);
 }
@@ -871,16 +904,26 @@ oscars_status oscars_local_steps(oscars_ctx* c, int32_t* tau_out, float* loss_ou
     } else {
       if (!c->round_exec) {
         cudaGraph_t g = nullptr;
+        for (auto& p : c->prof_round_graph) {
+          cudaEventDestroy(p.a);
+          cudaEventDestroy(p.b);
+        }
+        c->prof_round_graph.clear();
+        c->profiling = (c->flags & 2) != 0;
+        c->prof_sink = &c->prof_round_graph;
         e = cudaStreamBeginCapture(c->cap, cudaStreamCaptureModeThreadLocal);
         if (e == cudaSuccess) {
           cudaError_t e2 = enqueue_round(c, c->cap);
           e = cudaStreamEndCapture(c->cap, &g);
           if (e2 != cudaSuccess) e = e2;
         }
+        c->profiling = false;
+        c->prof_sink = nullptr;
         if (e == cudaSuccess) e = cudaGraphInstantiateWithFlags(&c->round_exec, g, 0);
         if (g) cudaGraphDestroy(g);
       }
       if (e == cudaSuccess) e = cudaGraphLaunch(c->round_exec, c->stream);
+      if (e == cudaSuccess) prof_after_replay(c, c->prof_round_graph);
     }
     if (e != cudaSuccess) return cuda_fail(c, e, "local steps launch");
     for (int i = 0; i < c->W; ++i) {
@@ -925,8 +968,46 @@ oscars_status oscars_push_merge(oscars_ctx* c, const float* const* deltas, const
     if (c->model != OSCARS_MODEL_MLP || !c->pending)
       return fail(c, OSCARS_ESTATE, "push_merge without deltas needs pending local steps");
     for (int k = 0; k < c->W; ++k) a.src[k] = c->slab + static_cast<int64_t>(k) * c->P_pad;
-    ProfScope ps(c, "merge", c->stream);
-    e = launch_merge(a, xg, c->P_pad, eta, true, c->stream);
+    auto enqueue = [&](cudaStream_t st) -> cudaError_t {
+      cudaError_t r;
+      {
+        ProfScope ps(c, "merge", st);
+        r = launch_merge(a, xg, c->P_pad, eta, true, st);
+      }
+      if (r != cudaSuccess) return r;
+      ProfScope ps(c, "shadow_refresh", st);
+      return refresh_global_shadows(c, st);
+    };
+    if (c->flags & 1) {
+      e = enqueue(c->stream);
+    } else {
+      // the weights and buffers of a replica-mode merge never change: one graph
+      if (!c->merge_exec || c->rule == OSCARS_W_EXPLICIT) {
+        if (c->merge_exec) cudaGraphExecDestroy(c->merge_exec);
+        c->merge_exec = nullptr;
+        for (auto& p : c->prof_merge_graph) {
+          cudaEventDestroy(p.a);
+          cudaEventDestroy(p.b);
+        }
+        c->prof_merge_graph.clear();
+        c->prof_sink = &c->prof_merge_graph;
+        cudaGraph_t g = nullptr;
+        e = cudaStreamBeginCapture(c->cap, cudaStreamCaptureModeThreadLocal);
+        if (e == cudaSuccess) {
+          cudaError_t e2 = enqueue(c->cap);
+          e = cudaStreamEndCapture(c->cap, &g);
+          if (e2 != cudaSuccess) e = e2;
+        }
+        c->prof_sink = nullptr;
+        if (e == cudaSuccess) e = cudaGraphInstantiateWithFlags(&c->merge_exec, g, 0);
+        if (g) cudaGraphDestroy(g);
+      }
+      if (e == cudaSuccess) e = cudaGraphLaunch(c->merge_exec, c->stream);
+      if (e == cudaSuccess) prof_after_replay(c, c->prof_merge_graph);
+    }
+    if (e != cudaSuccess) return cuda_fail(c, e, "merge launch");
+    c->pending = false;
+    return OSCARS_OK;
   } else {
     for (int k = 0; k < c->W; ++k)
       if (!deltas[k]) return fail(c, OSCARS_EINVAL, "NULL delta pointer");
