@@ -103,7 +103,9 @@ typedef struct {
                                  /* oscars_profile_read);                         */
                                  /* bit 2: run the workers of a round as up to 16 */
                                  /* concurrent branches (streams) instead of one  */
-                                 /* launch per layer over all active workers      */
+                                 /* launch per layer over all active workers;     */
+                                 /* bit 3: do not use the one-launch round of a   */
+                                 /* 2-layer MLP (per-layer kernels instead)       */
 } oscars_config;
 
 /*

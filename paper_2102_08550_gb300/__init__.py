@@ -22,6 +22,7 @@ SEARCH_CAPPED, SEARCH_LITERAL = 0, 1
 FLAG_NO_GRAPH = 1
 FLAG_PROFILE = 2
 FLAG_BRANCHES = 4
+FLAG_PER_LAYER = 8
 
 
 class OscarsError(RuntimeError):

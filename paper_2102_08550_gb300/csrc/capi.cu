@@ -65,6 +65,20 @@ bool make_map(CUtensorMap* m, const void* base, uint64_t dx, uint64_t dy, uint64
            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// 4-D bf16 tensor map, boxes of 64 x box_y x 1 x 1, 128-byte swizzle
+bool make_map4(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, uint64_t d2, uint64_t d3, uint64_t s1,
+               uint64_t s2, uint64_t s3, uint32_t box_y) {
+  EncodeTiledFn f = encode_fn();
+  if (!f) return false;
+  cuuint64_t dims[4] = {d0, d1, d2, d3};
+  cuuint64_t strides[3] = {s1, s2, s3};
+  cuuint32_t box[4] = {64, box_y, 1, 1};
+  cuuint32_t es[4] = {1, 1, 1, 1};
+  return f(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides, box, es,
+           CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+           CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 struct Layer {
   int in, out;
   int64_t offW, offB, offT;  // offT < 0: no transposed copy
@@ -127,6 +141,8 @@ struct oscars_ctx {
   __nv_bfloat16* A0Tall = nullptr;
   int32_t* labels_all = nullptr;
   std::vector<CUtensorMap> mA0s, mAT0s;
+  bool fused = false;                   // whole-round kernel (2-layer MLP)
+  CUtensorMap mX4, mXT4;                // staged inputs of every step (fused kernel)
   // streams / graph
   cudaStream_t stream = nullptr;
   cudaStream_t cap = nullptr;
@@ -312,6 +328,13 @@ oscars_status ensure_stage_buffers(oscars_ctx* c) {
     if (!make_map(&c->mA0s[s], c->A0all + per * s, D, B, W, D * 2ull, static_cast<uint64_t>(B) * D * 2ull, B) ||
         !make_map(&c->mAT0s[s], c->A0Tall + per * s, B, D, W, B * 2ull, static_cast<uint64_t>(B) * D * 2ull, 128))
       return fail(c, OSCARS_ECUDA, "cuTensorMapEncodeTiled failed (per-step inputs)");
+  }
+  if (c->fused) {
+    const uint64_t per_b = static_cast<uint64_t>(per) * 2;
+    if (!make_map4(&c->mX4, c->A0all, D, B, W, cap, D * 2ull, static_cast<uint64_t>(B) * D * 2ull, per_b, B) ||
+        !make_map4(&c->mXT4, c->A0Tall, B, D, W, cap, B * 2ull, static_cast<uint64_t>(B) * D * 2ull, per_b,
+                   fused_round_xt_rows(B)))
+      return fail(c, OSCARS_ECUDA, "cuTensorMapEncodeTiled failed (fused round inputs)");
   }
   // step 0 doubles as the single-step buffers (evaluation)
   c->A[0] = c->A0all;
@@ -540,21 +563,46 @@ cudaError_t enqueue_round_mlp(oscars_ctx* c, cudaStream_t st) {
     ProfScope ps(c, "stage", st);
     if ((e = launch_stage_round(sa, c->tau_dev, c->W, c->max_tau, st)) != cudaSuccess) return e;
   }
-  if (c->n_br > 1) {
-    cudaError_t e2 = cudaEventRecord(c->br_fork, st);
-    if (e2 != cudaSuccess) return e2;
-  }
-  for (int g = 0; g < c->n_br; ++g) {
-    cudaStream_t sg = c->n_br > 1 ? c->br_streams[g] : st;
-    if (c->n_br > 1 && (e = cudaStreamWaitEvent(sg, c->br_fork, 0)) != cudaSuccess) return e;
-    for (int s = 0; s < c->br_max_tau[g]; ++s) {
-      const size_t at = (static_cast<size_t>(g) * c->max_tau + s);
-      const int na = c->br_na[at];
-      if ((e = enqueue_step(c, s, na, c->br_wid + at * c->W, c->br_src + at * c->W, sg)) != cudaSuccess) return e;
-    }
+  if (c->fused) {
+    FusedRoundArgs f;
+    f.tau = c->tau_dev;
+    f.W = c->W;
+    f.D = c->dims[0];
+    f.H = c->dims[1];
+    f.B = c->B;
+    f.global_slot = c->W;
+    f.lr = c->lr;
+    f.master = c->slab;
+    f.master_w = c->slab;
+    f.shadow = c->shadow;
+    f.slot_stride = c->P_pad;
+    f.offW0 = c->layers[0].offW;
+    f.offB0 = c->layers[0].offB;
+    f.offW1 = c->layers[1].offW;
+    f.offB1 = c->layers[1].offB;
+    f.labels = c->labels_all;
+    f.loss_part = c->loss_part;
+    f.max_tau = c->max_tau;
+    f.err = c->err;
+    ProfScope ps(c, "fused_round", st);
+    if ((e = launch_fused_round(c->mShadow[0], c->mX4, c->mXT4, f, st)) != cudaSuccess) return e;
+  } else {
     if (c->n_br > 1) {
-      if ((e = cudaEventRecord(c->br_join[g], sg)) != cudaSuccess) return e;
-      if ((e = cudaStreamWaitEvent(st, c->br_join[g], 0)) != cudaSuccess) return e;
+      cudaError_t e2 = cudaEventRecord(c->br_fork, st);
+      if (e2 != cudaSuccess) return e2;
+    }
+    for (int g = 0; g < c->n_br; ++g) {
+      cudaStream_t sg = c->n_br > 1 ? c->br_streams[g] : st;
+      if (c->n_br > 1 && (e = cudaStreamWaitEvent(sg, c->br_fork, 0)) != cudaSuccess) return e;
+      for (int s = 0; s < c->br_max_tau[g]; ++s) {
+        const size_t at = (static_cast<size_t>(g) * c->max_tau + s);
+        const int na = c->br_na[at];
+        if ((e = enqueue_step(c, s, na, c->br_wid + at * c->W, c->br_src + at * c->W, sg)) != cudaSuccess) return e;
+      }
+      if (c->n_br > 1) {
+        if ((e = cudaEventRecord(c->br_join[g], sg)) != cudaSuccess) return e;
+        if ((e = cudaStreamWaitEvent(st, c->br_join[g], 0)) != cudaSuccess) return e;
+      }
     }
   }
   const int nc = c->B / kRowsPerLossChunk;
@@ -832,6 +880,9 @@ oscars_status oscars_create(const oscars_config* cfg, oscars_ctx** out) {
           }
         }
         if (st == OSCARS_OK && !cfg->init_params) st = fail(c, OSCARS_EINVAL, "MLP: init_params is NULL");
+        // a 2-layer bf16 MLP runs each round as one fused launch (flag bit 3: per-layer kernels)
+        c->fused = c->bf16 && !(cfg->flags & 8) && !(cfg->flags & 4) &&
+                   fused_round_supported(c->L, c->dims[0], c->L >= 2 ? c->dims[1] : 0, c->C, c->B);
         // flag bit 2: bf16 MLP rounds fork into up to 16 concurrent worker branches
         c->n_br = (c->bf16 && c->L >= 2 && (cfg->flags & 4)) ? std::min(c->W, kMaxBranches) : 1;
         if (st == OSCARS_OK) st = allocate_mlp(c);

@@ -138,6 +138,31 @@ bool head_fused_supported(int H, int B, int C);
 cudaError_t launch_head_fused(const HeadArgs& a, int n_active, cudaStream_t s);
 cudaError_t launch_head_bwd(const HeadArgs& a, int n_active, cudaStream_t s);
 
+// ---------------------------------------------------------------- fused round (2-layer MLP)
+struct FusedRoundArgs {
+  const int32_t* tau;
+  int W, D, H, B;
+  int global_slot;
+  float lr;
+  const float* master;
+  float* master_w;
+  __nv_bfloat16* shadow;
+  int64_t slot_stride;
+  int64_t offW0, offB0, offW1, offB1;
+  const int32_t* labels;
+  float* loss_part;
+  int max_tau;
+  int* err;
+};
+// whole-round kernel for input -> H ReLU -> 10 classes (one cluster per worker)
+bool fused_round_supported(int L, int D, int H, int C, int B);
+int fused_round_xt_rows(int B);   // rows of the X^T box the kernel loads
+// mW0: shadow W0 of every slot {D, H, slots} box {64, 128}; mX: staged inputs
+// {D, B, W, steps} box {64, B}; mXT: staged transposed inputs {B, D, W, steps}
+// box {64, fused_round_xt_rows(B)}
+cudaError_t launch_fused_round(const CUtensorMap& mW0, const CUtensorMap& mX, const CUtensorMap& mXT,
+                               const FusedRoundArgs& a, cudaStream_t s);
+
 // loss[w] = sum_{s < tau[w]} sum_c part[(w*max_tau + s)*nc + c] / (B * tau[w])
 cudaError_t launch_loss_finalize(const float* part, const int32_t* tau, int W, int max_tau,
                                  int nc, int B, float* loss, cudaStream_t s);

@@ -127,6 +127,18 @@ def test_mlp_bsp_override(cuda_device):
     run_both(w, 2, cuda_device, tau_override=[1, 1, 1, 1])
 
 
+def test_mlp_2layer_per_layer_kernels(cuda_device):
+    """The per-layer kernel path for a 2-layer model (the default runs each
+    round of such a model as one fused launch)."""
+    w = synth.TrainWorkload("small-per-layer", 4, [784, 512, 10], 64, 0.05, 512, 8, 2)
+    run_both(w, 2, cuda_device, rows=512, flags=P.FLAG_PER_LAYER)
+
+
+def test_mlp_branches(cuda_device):
+    w = synth.TrainWorkload("small-branches", 5, [256, 128, 128, 10], 32, 0.05, 256, 6, 2)
+    run_both(w, 2, cuda_device, rows=256, flags=P.FLAG_BRANCHES)
+
+
 def test_mlp_direct_launch_matches_graph(cuda_device):
     w = synth.TrainWorkload("small-direct", 3, [256, 128, 10], 64, 0.05, 256, 8, 2)
     run_both(w, 2, cuda_device, flags=P.FLAG_NO_GRAPH)
