@@ -79,6 +79,20 @@ bool make_map4(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, uint6
            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// 3-D fp32 tensor map without swizzle: boxes of box_x x box_y x 1
+bool make_map_f32(CUtensorMap* m, const void* base, uint64_t dx, uint64_t dy, uint64_t dz, uint64_t stride_y,
+                  uint64_t stride_z, uint32_t box_x, uint32_t box_y) {
+  EncodeTiledFn f = encode_fn();
+  if (!f) return false;
+  cuuint64_t dims[3] = {dx, dy, dz};
+  cuuint64_t strides[2] = {stride_y, stride_z};
+  cuuint32_t box[3] = {box_x, box_y, 1};
+  cuuint32_t es[3] = {1, 1, 1};
+  return f(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, const_cast<void*>(base), dims, strides, box, es,
+           CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+           CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 struct Layer {
   int in, out;
   int64_t offW, offB, offT;  // offT < 0: no transposed copy
@@ -143,6 +157,7 @@ struct oscars_ctx {
   std::vector<CUtensorMap> mA0s, mAT0s;
   bool fused = false;                   // whole-round kernel (2-layer MLP)
   CUtensorMap mX4, mXT4;                // staged inputs of every step (fused kernel)
+  CUtensorMap mWm0;                     // fp32 master W0 of every slot (fused kernel)
   // streams / graph
   cudaStream_t stream = nullptr;
   cudaStream_t cap = nullptr;
@@ -333,7 +348,9 @@ oscars_status ensure_stage_buffers(oscars_ctx* c) {
     const uint64_t per_b = static_cast<uint64_t>(per) * 2;
     if (!make_map4(&c->mX4, c->A0all, D, B, W, cap, D * 2ull, static_cast<uint64_t>(B) * D * 2ull, per_b, B) ||
         !make_map4(&c->mXT4, c->A0Tall, B, D, W, cap, B * 2ull, static_cast<uint64_t>(B) * D * 2ull, per_b,
-                   fused_round_xt_rows(B)))
+                   fused_round_xt_rows(B)) ||
+        !make_map_f32(&c->mWm0, c->slab + c->layers[0].offW, D, c->dims[1], static_cast<uint64_t>(W) + 1, D * 4ull,
+                      c->P_pad * 4ull, fused_round_xt_rows(B), 128))
       return fail(c, OSCARS_ECUDA, "cuTensorMapEncodeTiled failed (fused round inputs)");
   }
   // step 0 doubles as the single-step buffers (evaluation)
@@ -585,7 +602,7 @@ cudaError_t enqueue_round_mlp(oscars_ctx* c, cudaStream_t st) {
     f.max_tau = c->max_tau;
     f.err = c->err;
     ProfScope ps(c, "fused_round", st);
-    if ((e = launch_fused_round(c->mShadow[0], c->mX4, c->mXT4, f, st)) != cudaSuccess) return e;
+    if ((e = launch_fused_round(c->mShadow[0], c->mX4, c->mXT4, c->mWm0, f, st)) != cudaSuccess) return e;
   } else {
     if (c->n_br > 1) {
       cudaError_t e2 = cudaEventRecord(c->br_fork, st);

@@ -67,11 +67,13 @@ struct FCfg {
   static constexpr int kStagesF = B >= 128 ? 2 : 4;
   static constexpr int kABytes = kFU * kFBK * 2;            // W0 tile: 128 rows x 64 k
   static constexpr int kBBytes = B * kFBK * 2;              // X tile: B rows x 64 k
-  static constexpr int kND = B >= 128 ? 128 : 256;          // columns (input features) per weight-gradient tile
+  static constexpr int kND = B >= 128 ? 32 : 64;            // columns (input features) per weight-gradient tile
   static constexpr int kKB = (B + kFBK - 1) / kFBK;         // K-blocks of the weight gradient (K = batch)
   static constexpr int kXtBytes = kND * kFBK * 2 * kKB;     // one X^T tile (all K-blocks)
+  static constexpr int kMsBytes = kFU * kND * 4;            // fp32 master tile: 128 rows x kND columns
+  static constexpr int kBufD = kXtBytes + kMsBytes;
   static constexpr int kPipe = kStagesF * (kABytes + kBBytes);
-  static constexpr int kPipeD = 2 * kXtBytes;
+  static constexpr int kPipeD = 2 * kBufD;
   static constexpr int kRegion = kPipe > kPipeD ? kPipe : kPipeD;   // TMA area, reused by both steps
   static constexpr int kDzT = kFU * 128 * kKB;              // dz0^T tile: 128 rows x (64 k per block)
   static constexpr int kTpr = 256 / B;                      // threads per row, partial logits (256 threads)
@@ -120,6 +122,7 @@ template <int B>
 __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_constant__ CUtensorMap mW0,
                                                                  const __grid_constant__ CUtensorMap mX,
                                                                  const __grid_constant__ CUtensorMap mXT,
+                                                                 const __grid_constant__ CUtensorMap mWm,
                                                                  const __grid_constant__ FusedArgs a) {
   using Cfg = FCfg<B>;
   extern __shared__ uint8_t fs_raw[];
@@ -139,9 +142,9 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
   uint64_t* emptyF = fullF + Cfg::kStagesF;    // [kStagesF]
   uint64_t* accF = emptyF + Cfg::kStagesF;     // [1]
   uint64_t* fullD = accF + 1;                  // [2]
-  uint64_t* emptyD = fullD + 2;                // [2] smem X^T buffer free
+  uint64_t* emptyD = fullD + 2;                // [2] (unused: tfreeD covers buffer reuse)
   uint64_t* accD = emptyD + 2;                 // [2] TMEM buffer full
-  uint64_t* tfreeD = accD + 2;                 // [2] TMEM buffer drained (256 arrivals)
+  uint64_t* tfreeD = accD + 2;                 // [2] TMEM + shared buffer drained (256 arrivals)
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(tfreeD + 2);
 
   const int w = blockIdx.x;
@@ -158,6 +161,7 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
     prefetch_tmap(&mW0);
     prefetch_tmap(&mX);
     prefetch_tmap(&mXT);
+    prefetch_tmap(&mWm);
     for (int i = 0; i < Cfg::kStagesF; ++i) {
       mbar_init(&fullF[i], 1);
       mbar_init(&emptyF[i], 1);
@@ -399,12 +403,14 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
     if (warp == 0 && lane == 0) {
       for (int tt = 0; tt < nD; ++tt) {
         const int c = dcount + tt, buf = c & 1, use = c >> 1;
-        if (use >= 1 && !mbar_wait(&emptyD[buf], (use - 1) & 1, a.err, kDevTimeoutEmpty)) break;
-        mbar_arrive_expect_tx(&fullD[buf], Cfg::kXtBytes);
-        uint8_t* dst = region + buf * Cfg::kXtBytes;
+        // the buffer's previous tile must be fully consumed (MMA and epilogue)
+        if (use >= 1 && !mbar_wait(&tfreeD[buf], (use - 1) & 1, a.err, kDevTimeoutEmpty)) break;
+        mbar_arrive_expect_tx(&fullD[buf], Cfg::kBufD);
+        uint8_t* dst = region + buf * Cfg::kBufD;
 #pragma unroll
         for (int kb = 0; kb < Cfg::kKB; ++kb)
           tma_load_4d(dst + kb * Cfg::kND * 128, &mXT, kb * kFBK, tt * Cfg::kND, w, s, &fullD[buf]);
+        tma_load_3d(dst + Cfg::kXtBytes, &mWm, tt * Cfg::kND, u0, src, &fullD[buf]);   // old W0 rows
       }
     } else if (warp == 1 && lane == 0) {
       constexpr uint32_t idesc = idesc_bf16_f32(128, Cfg::kND);
@@ -413,7 +419,7 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
         if (!mbar_wait(&fullD[buf], use & 1, a.err, kDevTimeoutFull)) break;
         if (use >= 1 && !mbar_wait(&tfreeD[buf], (use - 1) & 1, a.err, kDevTimeoutAccum)) break;
         tc_fence_after();
-        const uint32_t xa = smem_u32(region + buf * Cfg::kXtBytes);
+        const uint32_t xa = smem_u32(region + buf * Cfg::kBufD);
         const uint32_t da = smem_u32(dzT);
         const uint32_t dcol = tmem + static_cast<uint32_t>(buf * Cfg::kND);
 #pragma unroll
@@ -422,7 +428,6 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
           for (int j = 0; j < kFBK / 16; ++j)
             umma_bf16(dcol, smem_desc_k128(da + kb * kFU * 128 + j * 32),
                       smem_desc_k128(xa + kb * Cfg::kND * 128 + j * 32), idesc, (kb | j) != 0 ? 1u : 0u);
-        umma_commit(&emptyD[buf]);
         umma_commit(&accD[buf]);
       }
     } else if (warp >= 4) {
@@ -435,25 +440,21 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
         ok = __all_sync(0xffffffffu, ok);
         tc_fence_after();
         if (ok) {
+          const float* Ms = reinterpret_cast<const float*>(region + buf * Cfg::kBufD + Cfg::kXtBytes);
           for (int c0 = grp * 32; c0 < Cfg::kND; c0 += 64) {
             const int n_base = tt * Cfg::kND + c0;        // input feature of lane 0's column
             if (n_base >= D) break;                        // uniform in the warp
             const int n = n_base + lane;
             const bool nok = n < D;
-            // old master values of the 32 rows (lane = column): one line per row
-            float old[32];
-            const int64_t srow = so + a.offW0 + static_cast<int64_t>(u0 + mb) * D + n;
-#pragma unroll
-            for (int r = 0; r < 32; ++r) old[r] = nok ? a.master[srow + static_cast<int64_t>(r) * D] : 0.f;
             float v[32];
             tmem_ld_32x32b_x32(tmem + (static_cast<uint32_t>(quarter * 32) << 16) + buf * Cfg::kND + c0, v);
 #pragma unroll
             for (int j = 0; j < 32; ++j) T[lane * 33 + j] = v[j];
             __syncwarp();
             const int64_t drow = dof + a.offW0 + static_cast<int64_t>(u0 + mb) * D + n;
-#pragma unroll
+#pragma unroll 8
             for (int r = 0; r < 32; ++r) {
-              const float nw = fmaf(-a.lr, T[r * 33 + lane], old[r]);
+              const float nw = fmaf(-a.lr, T[r * 33 + lane], Ms[(mb + r) * Cfg::kND + c0 + lane]);
               if (nok) {
                 a.master_w[drow + static_cast<int64_t>(r) * D] = nw;
                 a.shadow[drow + static_cast<int64_t>(r) * D] = __float2bfloat16_rn(nw);
@@ -482,8 +483,8 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
 }
 
 template <int B>
-cudaError_t launch_b(const CUtensorMap& mW0, const CUtensorMap& mX, const CUtensorMap& mXT, const FusedArgs& a,
-                     cudaStream_t s) {
+cudaError_t launch_b(const CUtensorMap& mW0, const CUtensorMap& mX, const CUtensorMap& mXT, const CUtensorMap& mWm,
+                     const FusedArgs& a, cudaStream_t s) {
   using Cfg = FCfg<B>;
   cudaError_t e = cudaFuncSetAttribute(fused_mlp2_round_kernel<B>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        Cfg::kSmem);
@@ -500,7 +501,7 @@ cudaError_t launch_b(const CUtensorMap& mW0, const CUtensorMap& mX, const CUtens
   attr[0].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, fused_mlp2_round_kernel<B>, mW0, mX, mXT, a);
+  return cudaLaunchKernelEx(&cfg, fused_mlp2_round_kernel<B>, mW0, mX, mXT, mWm, a);
 }
 
 }  // namespace
@@ -512,10 +513,10 @@ bool fused_round_supported(int L, int D, int H, int C, int B) {
   return smem <= 227 * 1024;
 }
 
-int fused_round_xt_rows(int B) { return B >= 128 ? 128 : 256; }
+int fused_round_xt_rows(int B) { return B >= 128 ? 32 : 64; }
 
 cudaError_t launch_fused_round(const CUtensorMap& mW0, const CUtensorMap& mX, const CUtensorMap& mXT,
-                               const FusedRoundArgs& r, cudaStream_t s) {
+                               const CUtensorMap& mWm, const FusedRoundArgs& r, cudaStream_t s) {
   FusedArgs a;
   a.tau = r.tau;
   a.W = r.W;
@@ -536,9 +537,9 @@ cudaError_t launch_fused_round(const CUtensorMap& mW0, const CUtensorMap& mX, co
   a.max_tau = r.max_tau;
   a.err = r.err;
   switch (r.B) {
-    case 32: return launch_b<32>(mW0, mX, mXT, a, s);
-    case 64: return launch_b<64>(mW0, mX, mXT, a, s);
-    case 128: return launch_b<128>(mW0, mX, mXT, a, s);
+    case 32: return launch_b<32>(mW0, mX, mXT, mWm, a, s);
+    case 64: return launch_b<64>(mW0, mX, mXT, mWm, a, s);
+    case 128: return launch_b<128>(mW0, mX, mXT, mWm, a, s);
     default: return cudaErrorInvalidValue;
   }
 }

@@ -159,9 +159,10 @@ bool fused_round_supported(int L, int D, int H, int C, int B);
 int fused_round_xt_rows(int B);   // rows of the X^T box the kernel loads
 // mW0: shadow W0 of every slot {D, H, slots} box {64, 128}; mX: staged inputs
 // {D, B, W, steps} box {64, B}; mXT: staged transposed inputs {B, D, W, steps}
-// box {64, fused_round_xt_rows(B)}
+// box {64, fused_round_xt_rows(B)}; mWm: fp32 master W0 of every slot
+// {D, H, slots} box {fused_round_xt_rows(B), 128}, no swizzle
 cudaError_t launch_fused_round(const CUtensorMap& mW0, const CUtensorMap& mX, const CUtensorMap& mXT,
-                               const FusedRoundArgs& a, cudaStream_t s);
+                               const CUtensorMap& mWm, const FusedRoundArgs& a, cudaStream_t s);
 
 // loss[w] = sum_{s < tau[w]} sum_c part[(w*max_tau + s)*nc + c] / (B * tau[w])
 cudaError_t launch_loss_finalize(const float* part, const int32_t* tau, int W, int max_tau,
