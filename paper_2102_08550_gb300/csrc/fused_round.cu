@@ -88,8 +88,8 @@ struct FCfg {
   static constexpr int oDzb = oDz + B * kFC * 4;             // [B][C] float
   static constexpr int oGbp = oDzb + B * kFC * 4;            // [8][128] float
   static constexpr int oRowLoss = oGbp + 8 * kFU * 4;        // [B] float
-  static constexpr int oEpi = (oRowLoss + B * 4 + 15) / 16 * 16;   // 8 x [32][33] float staging tiles
-  static constexpr int oBar = oEpi + 8 * 32 * 33 * 4;
+  static constexpr int oEpi = (oRowLoss + B * 4 + 15) / 16 * 16;   // 8 x [32][36] float staging tiles
+  static constexpr int oBar = oEpi + 8 * 32 * 36 * 4;
   static constexpr int kBarBytes = 256;
   static constexpr int kSmem = oBar + kBarBytes + 1024;      // + alignment slack
 };
@@ -433,7 +433,7 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
     } else if (warp >= 4) {
       const int quarter = warp & 3, grp = (warp - 4) >> 2;
       const int mb = quarter * 32;                       // local rows of this warp
-      float* T = epi + (warp - 4) * 32 * 33;
+      float* T = epi + (warp - 4) * 32 * 36;   // row stride 36: 16-byte accesses of 8 lanes hit distinct banks
       for (int tt = 0; tt < nD; ++tt) {
         const int c = dcount + tt, buf = c & 1, use = c >> 1;
         int ok = mbar_wait(&accD[buf], use & 1, a.err, kDevTimeoutAccum) ? 1 : 0;
@@ -442,22 +442,31 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
         if (ok) {
           const float* Ms = reinterpret_cast<const float*>(region + buf * Cfg::kBufD + Cfg::kXtBytes);
           for (int c0 = grp * 32; c0 < Cfg::kND; c0 += 64) {
-            const int n_base = tt * Cfg::kND + c0;        // input feature of lane 0's column
+            const int n_base = tt * Cfg::kND + c0;        // first input feature of the chunk
             if (n_base >= D) break;                        // uniform in the warp
-            const int n = n_base + lane;
-            const bool nok = n < D;
             float v[32];
             tmem_ld_32x32b_x32(tmem + (static_cast<uint32_t>(quarter * 32) << 16) + buf * Cfg::kND + c0, v);
 #pragma unroll
-            for (int j = 0; j < 32; ++j) T[lane * 33 + j] = v[j];
+            for (int q = 0; q < 8; ++q)
+              *reinterpret_cast<float4*>(T + lane * 36 + 4 * q) = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
             __syncwarp();
-            const int64_t drow = dof + a.offW0 + static_cast<int64_t>(u0 + mb) * D + n;
-#pragma unroll 8
-            for (int r = 0; r < 32; ++r) {
-              const float nw = fmaf(-a.lr, T[r * 33 + lane], Ms[(mb + r) * Cfg::kND + c0 + lane]);
+            // lane -> (row r0 + lane / 8, columns 4 * (lane % 8) .. + 3): 4 rows per instruction
+            const int cq = (lane & 7) * 4;
+            const bool nok = n_base + cq < D;   // D % 8 == 0: a 4-column group is all in or all out
+#pragma unroll
+            for (int i = 0; i < 8; ++i) {
+              const int r = 4 * i + (lane >> 3);
+              const float4 g = *reinterpret_cast<const float4*>(T + r * 36 + cq);
+              const float4 o = *reinterpret_cast<const float4*>(Ms + (mb + r) * Cfg::kND + c0 + cq);
+              float4 nw;
+              nw.x = fmaf(-a.lr, g.x, o.x);
+              nw.y = fmaf(-a.lr, g.y, o.y);
+              nw.z = fmaf(-a.lr, g.z, o.z);
+              nw.w = fmaf(-a.lr, g.w, o.w);
               if (nok) {
-                a.master_w[drow + static_cast<int64_t>(r) * D] = nw;
-                a.shadow[drow + static_cast<int64_t>(r) * D] = __float2bfloat16_rn(nw);
+                const int64_t e = dof + a.offW0 + static_cast<int64_t>(u0 + mb + r) * D + n_base + cq;
+                *reinterpret_cast<float4*>(a.master_w + e) = nw;
+                *reinterpret_cast<uint2*>(a.shadow + e) = make_uint2(pack_bf16x2(nw.x, nw.y), pack_bf16x2(nw.z, nw.w));
               }
             }
             __syncwarp();

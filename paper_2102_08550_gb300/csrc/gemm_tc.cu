@@ -39,7 +39,7 @@ constexpr int BM = 128;
 constexpr int BK = 64;
 constexpr int kABytes = BM * BK * 2;
 constexpr int kBarrierBytes = 256;          // mbarriers + TMEM address slot
-constexpr int kEpiTileFloats = 32 * 33;     // per-warp staging tile (padded rows)
+constexpr int kEpiTileFloats = 32 * 36;     // per-warp staging tile (row stride 36: conflict-free 16-byte accesses)
 
 // Warps per CTA: the weight-gradient epilogue streams the fp32 master and
 // runs two warpgroups (each warp owns its TMEM lane quarter, the two groups
@@ -99,49 +99,67 @@ __device__ __forceinline__ float epi_dh(const GemmArgs& a, int wid, int m, int n
 }
 
 // Weight gradient + SGD for one 32 x 32 block: rows m_base .. m_base + 31
-// (thread `lane` holds row m_base + lane in v), columns n_base .. n_base + 31;
-// `old` holds the block's fp32 master values already loaded as
-// old[r] = master[src][m_base + r][n_base + lane] (lane = column).
-// The accumulators go through a padded shared-memory tile so that the fp32
-// master write and the bf16 shadow write move full lines (lane = column),
-// while the transposed shadow is written from the row layout (lane = row).
+// (thread `lane` holds row m_base + lane in v), columns n_base .. n_base + 31.
+// `old` holds the block's fp32 master values in the column layout of the
+// store pass: old[i] (i < 8) = 4 columns (n_base + 4 (lane % 8) ..) of row
+// m_base + 4 i + lane / 8.  The accumulators go through a shared-memory tile
+// (row stride 36: 16-byte accesses of 8 lanes hit distinct banks both along
+// rows and along columns) so that the fp32 master and bf16 shadow writes move
+// full lines, 4 rows per instruction; the transposed shadow is written from
+// the row layout (lane = row, consecutive addresses).
 __device__ __forceinline__ void epi_dw_block(const GemmArgs& a, int wid, int m_base, int n_base,
-                                             const float (&v)[32], const float (&old)[32], float* T, int lane) {
+                                             const float (&v)[32], const float4 (&old)[8], float* T, int lane) {
 #pragma unroll
-  for (int j = 0; j < 32; ++j) T[lane * 33 + j] = v[j];
+  for (int q = 0; q < 8; ++q)
+    *reinterpret_cast<float4*>(T + lane * 36 + 4 * q) = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
   __syncwarp();
-  const int n = n_base + lane;
-  const bool nok = n < a.N;
-  const int64_t dof = static_cast<int64_t>(wid) * a.slot_stride + a.offW + n;
+  const int cq = (lane & 7) * 4;
+  const bool nok = n_base + cq < a.N;     // N % 8 == 0: a 4-column group is all in or all out
+  const int64_t dof = static_cast<int64_t>(wid) * a.slot_stride + a.offW + n_base + cq;
 #pragma unroll
-  for (int r = 0; r < 32; ++r) {
-    const float nw = fmaf(-a.lr, T[r * 33 + lane], old[r]);
+  for (int i = 0; i < 8; ++i) {
+    const int r = 4 * i + (lane >> 3);
+    const float4 g = *reinterpret_cast<const float4*>(T + r * 36 + cq);
+    float4 nw;
+    nw.x = fmaf(-a.lr, g.x, old[i].x);
+    nw.y = fmaf(-a.lr, g.y, old[i].y);
+    nw.z = fmaf(-a.lr, g.z, old[i].z);
+    nw.w = fmaf(-a.lr, g.w, old[i].w);
     if (nok) {
       const int64_t e = dof + static_cast<int64_t>(m_base + r) * a.N;
-      a.master_w[e] = nw;
-      a.shadow[e] = __float2bfloat16_rn(nw);
+      *reinterpret_cast<float4*>(a.master_w + e) = nw;
+      *reinterpret_cast<uint2*>(a.shadow + e) = make_uint2(pack_bf16x2(nw.x, nw.y), pack_bf16x2(nw.z, nw.w));
     }
-    T[r * 33 + lane] = nw;
+    *reinterpret_cast<float4*>(T + r * 36 + cq) = nw;
   }
   __syncwarp();
   if (a.shadowT) {
     __nv_bfloat16* t = a.shadowT + static_cast<int64_t>(wid) * a.slotT_stride + a.offT + m_base + lane;
-#pragma unroll 8
-    for (int j = 0; j < 32; ++j)
-      if (n_base + j < a.N) t[static_cast<int64_t>(n_base + j) * a.M] = __float2bfloat16_rn(T[lane * 33 + j]);
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+      const float4 nv = *reinterpret_cast<const float4*>(T + lane * 36 + 4 * q);
+      const float f[4] = {nv.x, nv.y, nv.z, nv.w};
+#pragma unroll
+      for (int j = 0; j < 4; ++j)
+        if (n_base + 4 * q + j < a.N) t[static_cast<int64_t>(n_base + 4 * q + j) * a.M] = __float2bfloat16_rn(f[j]);
+    }
   }
   __syncwarp();
 }
 
-// old[r] = master[src][m_base + r][n_base + lane] (0 outside N): one
-// coalesced line per row, all 32 loads issued before any is used
+// old[i] = master[src][m_base + 4 i + lane / 8][n_base + 4 (lane % 8) ..] as
+// float4 (0 outside N): all 8 loads issued before any is used
 __device__ __forceinline__ void epi_dw_load(const GemmArgs& a, int src, int m_base, int n_base, int lane,
-                                            float (&old)[32]) {
-  const int n = n_base + lane;
-  const bool nok = n < a.N;
-  const int64_t so = static_cast<int64_t>(src) * a.slot_stride + a.offW + n;
+                                            float4 (&old)[8]) {
+  const int cq = (lane & 7) * 4;
+  const bool nok = n_base + cq < a.N;
+  const int64_t so = static_cast<int64_t>(src) * a.slot_stride + a.offW + n_base + cq;
 #pragma unroll
-  for (int r = 0; r < 32; ++r) old[r] = nok ? a.master[so + static_cast<int64_t>(m_base + r) * a.N] : 0.f;
+  for (int i = 0; i < 8; ++i) {
+    const int r = 4 * i + (lane >> 3);
+    old[i] = nok ? *reinterpret_cast<const float4*>(a.master + so + static_cast<int64_t>(m_base + r) * a.N)
+                 : make_float4(0.f, 0.f, 0.f, 0.f);
+  }
 }
 
 __device__ __forceinline__ void epi_store(const GemmArgs& a, int m, int n0, const float (&v)[32]) {
@@ -242,7 +260,7 @@ __global__ void __launch_bounds__(warps_for<EPI>() * 32) gemm_tc_kernel(const __
       const int c_begin = (warp >> 2) * (BN / 2);
       const int mb = m0 + quarter * 32;
       float* T = epi_tiles + warp * kEpiTileFloats;
-      float old0[32], old1[32];
+      float4 old0[8], old1[8];
       epi_dw_load(a, src, mb, n0 + c_begin, lane, old0);        // both chunks' loads in flight
       epi_dw_load(a, src, mb, n0 + c_begin + 32, lane, old1);
       if (n0 + c_begin < a.N) {
