@@ -105,7 +105,9 @@ typedef struct {
                                  /* concurrent branches (streams) instead of one  */
                                  /* launch per layer over all active workers;     */
                                  /* bit 3: do not use the one-launch round of a   */
-                                 /* 2-layer MLP (per-layer kernels instead)       */
+                                 /* 2-layer MLP (per-layer kernels instead);      */
+                                 /* bit 4: stamp the phases of that one-launch    */
+                                 /* round (see oscars_phase_times)                */
 } oscars_config;
 
 /*
@@ -215,6 +217,15 @@ oscars_status oscars_read_replica(oscars_ctx* ctx, int32_t k, float* dst);
 int32_t oscars_profile_read(oscars_ctx* ctx, int32_t cap, const char** names, double* ms_total,
                             int32_t* launches);
 oscars_status oscars_profile_reset(oscars_ctx* ctx);
+
+/*
+ * oscars_phase_times - with flag bit 4, the device time (microseconds, from
+ * %globaltimer) of the three phases of every local step of worker 0 in the
+ * last one-launch round of a 2-layer MLP: forward, last layer, weight
+ * gradient + update, in that order (host us[3 * step + phase], up to cap).
+ * Returns the number of values written, 0 without stamps, -1 on error.
+ */
+int32_t oscars_phase_times(oscars_ctx* ctx, int32_t cap, double* us);
 
 /* oscars_num_params - P of the context (canonical layout). */
 oscars_status oscars_num_params(const oscars_ctx* ctx, int64_t* P);

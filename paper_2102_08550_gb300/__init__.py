@@ -23,6 +23,7 @@ FLAG_NO_GRAPH = 1
 FLAG_PROFILE = 2
 FLAG_BRANCHES = 4
 FLAG_PER_LAYER = 8
+FLAG_PHASE_TIMES = 16
 
 
 class OscarsError(RuntimeError):
@@ -66,6 +67,7 @@ _SIGS = {
     "oscars_profile_read": (c_int32, [c_void_p, c_int32, POINTER(ctypes.c_char_p), POINTER(c_double),
                                       POINTER(c_int32)]),
     "oscars_profile_reset": (c_int32, [c_void_p]),
+    "oscars_phase_times": (c_int32, [c_void_p, c_int32, POINTER(c_double)]),
     "oscars_softreg_steps_noalloc": (c_int32, [c_void_p, c_void_p, c_void_p, c_void_p, c_int64, c_int64, c_int32,
                                                c_int32, c_int32, c_int32, c_float, c_void_p, c_void_p]),
     "oscars_merge": (c_int32, [c_void_p, POINTER(c_void_p), POINTER(c_float), c_int32, c_int64, c_float, c_void_p]),
@@ -216,6 +218,16 @@ def oscars_profile_read(ctx: int):
     if n < 0:
         raise OscarsError(OSCARS_EINVAL, "profile_read")
     return {names[i].decode(): (ms[i], cnt[i]) for i in range(min(n, cap))}
+
+
+def oscars_phase_times(ctx: int):
+    """[(forward, last layer, weight gradient) us per local step] of worker 0."""
+    cap = 3 * 256
+    buf = (c_double * cap)()
+    n = lib().oscars_phase_times(c_void_p(ctx), cap, buf)
+    if n < 0:
+        raise OscarsError(OSCARS_ECUDA, "phase_times")
+    return [tuple(buf[i:i + 3]) for i in range(0, n, 3)]
 
 
 def oscars_profile_reset(ctx: int):

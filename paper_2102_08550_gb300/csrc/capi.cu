@@ -158,6 +158,7 @@ struct oscars_ctx {
   bool fused = false;                   // whole-round kernel (2-layer MLP)
   CUtensorMap mX4, mXT4;                // staged inputs of every step (fused kernel)
   CUtensorMap mWm0;                     // fp32 master W0 of every slot (fused kernel)
+  unsigned long long* phase_ts = nullptr;   // flag bit 4: phase stamps of the fused round
   // streams / graph
   cudaStream_t stream = nullptr;
   cudaStream_t cap = nullptr;
@@ -601,6 +602,12 @@ cudaError_t enqueue_round_mlp(oscars_ctx* c, cudaStream_t st) {
     f.loss_part = c->loss_part;
     f.max_tau = c->max_tau;
     f.err = c->err;
+    f.phase_ts = nullptr;
+    if (c->flags & 16) {
+      if (!c->phase_ts && !dev_alloc(c, &c->phase_ts, static_cast<size_t>(c->max_tau) * 4 + 64))
+        return cudaErrorMemoryAllocation;
+      f.phase_ts = c->phase_ts;
+    }
     ProfScope ps(c, "fused_round", st);
     if ((e = launch_fused_round(c->mShadow[0], c->mX4, c->mXT4, c->mWm0, f, st)) != cudaSuccess) return e;
   } else {
@@ -1261,6 +1268,20 @@ oscars_status oscars_gemm_bf16_nt(const void* A, const void* B, float* C, int32_
   g.c_out = C;
   return launch_gemm(kEpiStore, mA, mB, g, 1, static_cast<cudaStream_t>(stream)) == cudaSuccess ? OSCARS_OK
                                                                                                : OSCARS_ECUDA;
+}
+
+int32_t oscars_phase_times(oscars_ctx* c, int32_t cap, double* us) {
+  if (!c || !us || cap < 1) return -1;
+  if (!c->phase_ts || !c->fused) return 0;
+  std::vector<unsigned long long> h(static_cast<size_t>(c->max_tau) * 4);
+  if (cudaStreamSynchronize(c->stream) != cudaSuccess ||
+      cudaMemcpy(h.data(), c->phase_ts, h.size() * sizeof(unsigned long long), cudaMemcpyDeviceToHost) != cudaSuccess)
+    return -1;
+  const int steps = c->tau[0];
+  int n = 0;
+  for (int s = 0; s < steps && n + 3 <= cap; ++s)
+    for (int p = 0; p < 3; ++p) us[n++] = (h[s * 4 + p + 1] - h[s * 4 + p]) * 1e-3;
+  return n;
 }
 
 int32_t oscars_profile_read(oscars_ctx* c, int32_t cap, const char** names, double* ms_total, int32_t* launches) {

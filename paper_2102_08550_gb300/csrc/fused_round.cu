@@ -108,7 +108,14 @@ struct FusedArgs {
   float* loss_part;         // [(w * max_tau + s) * (B / 16) + chunk]
   int max_tau;
   int* err;
+  unsigned long long* phase_ts;   // [max_tau][4] phase start stamps of worker 0 (or null)
 };
+
+__device__ __forceinline__ unsigned long long global_ns() {
+  unsigned long long v;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(v));
+  return v;
+}
 
 // byte offset of element (row, k) in a K-major 128-byte-swizzled tile of
 // `rows` rows per 64-wide K-block (the layout TMA writes and UMMA reads)
@@ -191,7 +198,9 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
   int kcount = 0;   // F K-blocks issued so far (ring position)
   int dcount = 0;   // D tiles so far (TMEM / X^T double buffer position)
 
+  const bool stamp = a.phase_ts && w == 0 && rank == 0 && t == 0;
   for (int s = 0; s < tau; ++s) {
+    if (stamp) a.phase_ts[s * 4 + 0] = global_ns();
     const int src = s == 0 ? a.global_slot : w;
     const int64_t so = static_cast<int64_t>(src) * a.slot_stride;
     const int64_t dof = static_cast<int64_t>(w) * a.slot_stride;
@@ -255,6 +264,7 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
     }
     tc_fence_before();
     __syncthreads();
+    if (stamp) a.phase_ts[s * 4 + 1] = global_ns();
 
     // ------------------------------------------------------------ H: last layer
     if (t < 256) {   // partial logits: kTpr threads per row, all classes in registers
@@ -399,6 +409,7 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
       *reinterpret_cast<uint2*>(a.shadow + dof + e) = make_uint2(pack_bf16x2(nw.x, nw.y), pack_bf16x2(nw.z, nw.w));
     }
 
+    if (stamp) a.phase_ts[s * 4 + 2] = global_ns();
     // ------------------------------------------------------------ D: weight gradient + SGD of W0 rows
     if (warp == 0 && lane == 0) {
       for (int tt = 0; tt < nD; ++tt) {
@@ -482,6 +493,7 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
     __syncthreads();
     tc_fence_after();
     cluster_sync();               // head bias (rank 0) visible; pl / dz0^T reusable
+    if (stamp) a.phase_ts[s * 4 + 3] = global_ns();
   }
   tc_fence_before();
   __syncthreads();
@@ -545,6 +557,7 @@ cudaError_t launch_fused_round(const CUtensorMap& mW0, const CUtensorMap& mX, co
   a.loss_part = r.loss_part;
   a.max_tau = r.max_tau;
   a.err = r.err;
+  a.phase_ts = r.phase_ts;
   switch (r.B) {
     case 32: return launch_b<32>(mW0, mX, mXT, mWm, a, s);
     case 64: return launch_b<64>(mW0, mX, mXT, mWm, a, s);

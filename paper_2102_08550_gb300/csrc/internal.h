@@ -153,6 +153,7 @@ struct FusedRoundArgs {
   float* loss_part;
   int max_tau;
   int* err;
+  unsigned long long* phase_ts;   // [max_tau][4] phase stamps of worker 0, or null
 };
 // whole-round kernel for input -> H ReLU -> 10 classes (one cluster per worker)
 bool fused_round_supported(int L, int D, int H, int C, int B);
