@@ -345,6 +345,9 @@ oscars_status ensure_stage_buffers(oscars_ctx* c) {
         !make_map(&c->mAT0s[s], c->A0Tall + per * s, B, D, W, B * 2ull, static_cast<uint64_t>(B) * D * 2ull, 128))
       return fail(c, OSCARS_ECUDA, "cuTensorMapEncodeTiled failed (per-step inputs)");
   }
+  if (c->fused && (c->flags & 16) &&
+      !dev_alloc(c, &c->phase_ts, static_cast<size_t>(cap) * 4))   // stamps of every step (flag bit 4)
+    return fail(c, OSCARS_ENOMEM, "device allocation failed (phase stamps)");
   if (c->fused) {
     const uint64_t per_b = static_cast<uint64_t>(per) * 2;
     if (!make_map4(&c->mX4, c->A0all, D, B, W, cap, D * 2ull, static_cast<uint64_t>(B) * D * 2ull, per_b, B) ||
@@ -602,12 +605,7 @@ cudaError_t enqueue_round_mlp(oscars_ctx* c, cudaStream_t st) {
     f.loss_part = c->loss_part;
     f.max_tau = c->max_tau;
     f.err = c->err;
-    f.phase_ts = nullptr;
-    if (c->flags & 16) {
-      if (!c->phase_ts && !dev_alloc(c, &c->phase_ts, static_cast<size_t>(c->max_tau) * 4 + 64))
-        return cudaErrorMemoryAllocation;
-      f.phase_ts = c->phase_ts;
-    }
+    f.phase_ts = (c->flags & 16) ? c->phase_ts : nullptr;
     ProfScope ps(c, "fused_round", st);
     if ((e = launch_fused_round(c->mShadow[0], c->mX4, c->mXT4, c->mWm0, f, st)) != cudaSuccess) return e;
   } else {
@@ -869,6 +867,7 @@ oscars_status oscars_create(const oscars_config* cfg, oscars_ctx** out) {
   oscars_status st = OSCARS_OK;
   try {
     st = validate_and_layout(c, cfg);
+    c->flags = cfg->flags;
     if (st == OSCARS_OK) {
       c->stream = static_cast<cudaStream_t>(cfg->cuda_stream);
       c->M = cfg->M;
