@@ -64,16 +64,17 @@ __device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
 // Per-batch-size configuration (all sizes known at compile time).
 template <int B>
 struct FCfg {
-  static constexpr int kStagesF = B >= 128 ? 2 : 4;
+  static constexpr int kStagesF = 4;
   static constexpr int kABytes = kFU * kFBK * 2;            // W0 tile: 128 rows x 64 k
   static constexpr int kBBytes = B * kFBK * 2;              // X tile: B rows x 64 k
-  static constexpr int kND = B >= 128 ? 32 : 64;            // columns (input features) per weight-gradient tile
+  static constexpr int kND = 32;                            // columns (input features) per weight-gradient tile
+  static constexpr int kNBD = 4;                            // weight-gradient buffers in flight
   static constexpr int kKB = (B + kFBK - 1) / kFBK;         // K-blocks of the weight gradient (K = batch)
   static constexpr int kXtBytes = kND * kFBK * 2 * kKB;     // one X^T tile (all K-blocks)
   static constexpr int kMsBytes = kFU * kND * 4;            // fp32 master tile: 128 rows x kND columns
   static constexpr int kBufD = kXtBytes + kMsBytes;
   static constexpr int kPipe = kStagesF * (kABytes + kBBytes);
-  static constexpr int kPipeD = 2 * kBufD;
+  static constexpr int kPipeD = kNBD * kBufD;
   static constexpr int kRegion = kPipe > kPipeD ? kPipe : kPipeD;   // TMA area, reused by both steps
   static constexpr int kDzT = kFU * 128 * kKB;              // dz0^T tile: 128 rows x (64 k per block)
   static constexpr int kTpr = 256 / B;                      // threads per row, partial logits (256 threads)
@@ -88,7 +89,9 @@ struct FCfg {
   static constexpr int oDzb = oDz + B * kFC * 4;             // [B][C] float
   static constexpr int oGbp = oDzb + B * kFC * 4;            // [8][128] float
   static constexpr int oRowLoss = oGbp + 8 * kFU * 4;        // [B] float
-  static constexpr int oEpi = (oRowLoss + B * 4 + 15) / 16 * 16;   // 8 x [32][36] float staging tiles
+  static constexpr int oPre = (oRowLoss + B * 4 + 15) / 16 * 16;   // H inputs prefetched during F:
+  static constexpr int kPreFloats = kFC * kFU + kFU + 16 + B;       //   W1 master cols, b0, b1, labels
+  static constexpr int oEpi = (oPre + kPreFloats * 4 + 15) / 16 * 16;   // 8 x [32][36] float staging tiles
   static constexpr int oBar = oEpi + 8 * 32 * 36 * 4;
   static constexpr int kBarBytes = 256;
   static constexpr int kSmem = oBar + kBarBytes + 1024;      // + alignment slack
@@ -148,11 +151,15 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
   uint64_t* fullF = bars;                      // [kStagesF]
   uint64_t* emptyF = fullF + Cfg::kStagesF;    // [kStagesF]
   uint64_t* accF = emptyF + Cfg::kStagesF;     // [1]
-  uint64_t* fullD = accF + 1;                  // [2]
-  uint64_t* emptyD = fullD + 2;                // [2] (unused: tfreeD covers buffer reuse)
-  uint64_t* accD = emptyD + 2;                 // [2] TMEM buffer full
-  uint64_t* tfreeD = accD + 2;                 // [2] TMEM + shared buffer drained (256 arrivals)
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(tfreeD + 2);
+  uint64_t* fullD = accF + 1;                  // [kNBD] X^T + master tile landed
+  uint64_t* accD = fullD + Cfg::kNBD;          // [kNBD] TMEM buffer full
+  uint64_t* tfreeD = accD + Cfg::kNBD;         // [kNBD] TMEM + shared buffer drained (128 arrivals)
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(tfreeD + Cfg::kNBD);
+  float* pre = reinterpret_cast<float*>(sm + Cfg::oPre);
+  float* w1m = pre;                            // [C][128] fp32 master W1 columns (src)
+  float* b0m = w1m + kFC * kFU;                // [128] fp32 b0 of own units (src)
+  float* b1m = b0m + kFU;                      // [16] fp32 b1 (src)
+  int* labs = reinterpret_cast<int*>(b1m + 16);   // [B] labels of this step
 
   const int w = blockIdx.x;
   const int rank = static_cast<int>(cluster_ctarank());
@@ -174,11 +181,10 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
       mbar_init(&emptyF[i], 1);
     }
     mbar_init(accF, 1);
-    for (int i = 0; i < 2; ++i) {
+    for (int i = 0; i < Cfg::kNBD; ++i) {
       mbar_init(&fullD[i], 1);
-      mbar_init(&emptyD[i], 1);
       mbar_init(&accD[i], 1);
-      mbar_init(&tfreeD[i], 256);
+      mbar_init(&tfreeD[i], 128);
     }
     fence_barrier_init();
     fence_proxy_async_smem();
@@ -232,10 +238,13 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
       umma_commit(accF);
     }
     kcount += nkF;
-    // head weights of this CTA's columns (old values, bf16 operand) while F runs
+    // every global input of step H, fetched while the tensor core runs F:
+    // head weights of this CTA's columns (bf16 operand and fp32 master), b0 of
+    // its units, the head bias and this step's labels
     for (int q = t; q < kFC * (kFU / 8); q += kFT) {
       const int c = q / (kFU / 8), c8 = (q % (kFU / 8)) * 8;
-      const uint4 v = *reinterpret_cast<const uint4*>(a.shadow + so + a.offW1 + static_cast<int64_t>(c) * H + u0 + c8);
+      const int64_t e = a.offW1 + static_cast<int64_t>(c) * H + u0 + c8;
+      const uint4 v = *reinterpret_cast<const uint4*>(a.shadow + so + e);
       const __nv_bfloat162* p2 = reinterpret_cast<const __nv_bfloat162*>(&v);
 #pragma unroll
       for (int j = 0; j < 4; ++j) {
@@ -243,7 +252,12 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
         wcs[c * kFU + c8 + 2 * j] = f.x;
         wcs[c * kFU + c8 + 2 * j + 1] = f.y;
       }
+      *reinterpret_cast<float4*>(w1m + c * kFU + c8) = *reinterpret_cast<const float4*>(a.master + so + e);
+      *reinterpret_cast<float4*>(w1m + c * kFU + c8 + 4) = *reinterpret_cast<const float4*>(a.master + so + e + 4);
     }
+    if (t < kFU) b0m[t] = a.master[so + a.offB0 + u0 + t];
+    if (t < kFC) b1m[t] = a.master[so + a.offB1 + t];
+    for (int b = t; b < B; b += kFT) labs[b] = a.labels[(static_cast<int64_t>(s) * a.W + w) * B + b];
     __syncwarp();
     if (warp >= 4) {   // epilogue F: thread = hidden unit, columns = samples
       int ok = mbar_wait(accF, s & 1, a.err, kDevTimeoutAccum) ? 1 : 0;
@@ -252,7 +266,7 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
       if (ok) {
         const int quarter = warp & 3, grp = (warp - 4) >> 2;
         const int ul = quarter * 32 + lane;              // local unit
-        const float bias = a.master[so + a.offB0 + u0 + ul];
+        const float bias = b0m[ul];
         const uint32_t trow = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
         for (int c0 = grp * 32; c0 < B; c0 += 64) {
           float v[32];
@@ -290,7 +304,6 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
       }
     }
     cluster_sync();
-    const float* bias1 = a.master + so + a.offB1;
     for (int q = t; q < B * kFC; q += kFT) {
       float part[kFMaxCluster];
 #pragma unroll
@@ -299,10 +312,9 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
 #pragma unroll
       for (int r = 0; r < kFMaxCluster; ++r)
         if (r < ncl) acc += part[r];
-      dz[q] = acc + bias1[q % kFC];
+      dz[q] = acc + b1m[q % kFC];
     }
     cluster_sync();   // all remote reads of pl and all reads of the head bias are done
-    const int32_t* lab = a.labels + (static_cast<int64_t>(s) * a.W + w) * B;
     for (int b = t; b < B; b += kFT) {
       float z[kFC], e[kFC];
 #pragma unroll
@@ -310,7 +322,7 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
       float m = z[0];
 #pragma unroll
       for (int c = 1; c < kFC; ++c) m = fmaxf(m, z[c]);
-      const int y = lab[b];
+      const int y = labs[b];
       float se = 0.f, so_ = 0.f, zy = 0.f;
 #pragma unroll
       for (int c = 0; c < kFC; ++c) {
@@ -341,7 +353,7 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
         for (int b = j; b < B; b += 16) g += dz[b * kFC + c];
 #pragma unroll
         for (int o = 8; o > 0; o >>= 1) g += __shfl_xor_sync(0xffffffffu, g, o, 16);
-        if (j == 0) a.master_w[dof + a.offB1 + c] = fmaf(-a.lr, g, a.master[so + a.offB1 + c]);
+        if (j == 0) a.master_w[dof + a.offB1 + c] = fmaf(-a.lr, g, b1m[c]);
       }
     }
     // masked input gradient dz0[b][u] of this CTA's units: item = (row, 4 units);
@@ -384,7 +396,7 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
       float g = 0.f;
 #pragma unroll
       for (int r = 0; r < 8; ++r) g += gbp[r * kFU + t];
-      a.master_w[dof + a.offB0 + u0 + t] = fmaf(-a.lr, g, a.master[so + a.offB0 + u0 + t]);
+      a.master_w[dof + a.offB0 + u0 + t] = fmaf(-a.lr, g, b0m[t]);
     }
     // head weight gradient + SGD of this CTA's columns: item = (class, 4 units)
     for (int q = t; q < kFC * (kFU / 4); q += kFT) {
@@ -399,7 +411,7 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
         dw.w = fmaf(g, hv.w, dw.w);
       }
       const int64_t e = a.offW1 + static_cast<int64_t>(c) * H + u0 + u4;
-      const float4 o = *reinterpret_cast<const float4*>(a.master + so + e);
+      const float4 o = *reinterpret_cast<const float4*>(w1m + c * kFU + u4);
       float4 nw;
       nw.x = fmaf(-a.lr, dw.x, o.x);
       nw.y = fmaf(-a.lr, dw.y, o.y);
@@ -413,7 +425,7 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
     // ------------------------------------------------------------ D: weight gradient + SGD of W0 rows
     if (warp == 0 && lane == 0) {
       for (int tt = 0; tt < nD; ++tt) {
-        const int c = dcount + tt, buf = c & 1, use = c >> 1;
+        const int c = dcount + tt, buf = c % Cfg::kNBD, use = c / Cfg::kNBD;
         // the buffer's previous tile must be fully consumed (MMA and epilogue)
         if (use >= 1 && !mbar_wait(&tfreeD[buf], (use - 1) & 1, a.err, kDevTimeoutEmpty)) break;
         mbar_arrive_expect_tx(&fullD[buf], Cfg::kBufD);
@@ -426,7 +438,7 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
     } else if (warp == 1 && lane == 0) {
       constexpr uint32_t idesc = idesc_bf16_f32(128, Cfg::kND);
       for (int tt = 0; tt < nD; ++tt) {
-        const int c = dcount + tt, buf = c & 1, use = c >> 1;
+        const int c = dcount + tt, buf = c % Cfg::kNBD, use = c / Cfg::kNBD;
         if (!mbar_wait(&fullD[buf], use & 1, a.err, kDevTimeoutFull)) break;
         if (use >= 1 && !mbar_wait(&tfreeD[buf], (use - 1) & 1, a.err, kDevTimeoutAccum)) break;
         tc_fence_after();
@@ -442,46 +454,44 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
         umma_commit(&accD[buf]);
       }
     } else if (warp >= 4) {
+      // the two warpgroups take alternate tiles; a warp covers 32 rows x 32 columns
       const int quarter = warp & 3, grp = (warp - 4) >> 2;
       const int mb = quarter * 32;                       // local rows of this warp
       float* T = epi + (warp - 4) * 32 * 36;   // row stride 36: 16-byte accesses of 8 lanes hit distinct banks
-      for (int tt = 0; tt < nD; ++tt) {
-        const int c = dcount + tt, buf = c & 1, use = c >> 1;
+      for (int tt = grp; tt < nD; tt += 2) {
+        const int c = dcount + tt, buf = c % Cfg::kNBD, use = c / Cfg::kNBD;
         int ok = mbar_wait(&accD[buf], use & 1, a.err, kDevTimeoutAccum) ? 1 : 0;
         ok = __all_sync(0xffffffffu, ok);
         tc_fence_after();
         if (ok) {
           const float* Ms = reinterpret_cast<const float*>(region + buf * Cfg::kBufD + Cfg::kXtBytes);
-          for (int c0 = grp * 32; c0 < Cfg::kND; c0 += 64) {
-            const int n_base = tt * Cfg::kND + c0;        // first input feature of the chunk
-            if (n_base >= D) break;                        // uniform in the warp
-            float v[32];
-            tmem_ld_32x32b_x32(tmem + (static_cast<uint32_t>(quarter * 32) << 16) + buf * Cfg::kND + c0, v);
+          const int n_base = tt * Cfg::kND;              // first input feature of the tile
+          float v[32];
+          tmem_ld_32x32b_x32(tmem + (static_cast<uint32_t>(quarter * 32) << 16) + buf * Cfg::kND, v);
 #pragma unroll
-            for (int q = 0; q < 8; ++q)
-              *reinterpret_cast<float4*>(T + lane * 36 + 4 * q) = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
-            __syncwarp();
-            // lane -> (row r0 + lane / 8, columns 4 * (lane % 8) .. + 3): 4 rows per instruction
-            const int cq = (lane & 7) * 4;
-            const bool nok = n_base + cq < D;   // D % 8 == 0: a 4-column group is all in or all out
+          for (int q = 0; q < 8; ++q)
+            *reinterpret_cast<float4*>(T + lane * 36 + 4 * q) = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+          __syncwarp();
+          // lane -> (row 4 i + lane / 8, columns 4 (lane % 8) .. + 3): 4 rows per instruction
+          const int cq = (lane & 7) * 4;
+          const bool nok = n_base + cq < D;   // D % 8 == 0: a 4-column group is all in or all out
 #pragma unroll
-            for (int i = 0; i < 8; ++i) {
-              const int r = 4 * i + (lane >> 3);
-              const float4 g = *reinterpret_cast<const float4*>(T + r * 36 + cq);
-              const float4 o = *reinterpret_cast<const float4*>(Ms + (mb + r) * Cfg::kND + c0 + cq);
-              float4 nw;
-              nw.x = fmaf(-a.lr, g.x, o.x);
-              nw.y = fmaf(-a.lr, g.y, o.y);
-              nw.z = fmaf(-a.lr, g.z, o.z);
-              nw.w = fmaf(-a.lr, g.w, o.w);
-              if (nok) {
-                const int64_t e = dof + a.offW0 + static_cast<int64_t>(u0 + mb + r) * D + n_base + cq;
-                *reinterpret_cast<float4*>(a.master_w + e) = nw;
-                *reinterpret_cast<uint2*>(a.shadow + e) = make_uint2(pack_bf16x2(nw.x, nw.y), pack_bf16x2(nw.z, nw.w));
-              }
+          for (int i = 0; i < 8; ++i) {
+            const int r = 4 * i + (lane >> 3);
+            const float4 g = *reinterpret_cast<const float4*>(T + r * 36 + cq);
+            const float4 o = *reinterpret_cast<const float4*>(Ms + (mb + r) * Cfg::kND + cq);
+            float4 nw;
+            nw.x = fmaf(-a.lr, g.x, o.x);
+            nw.y = fmaf(-a.lr, g.y, o.y);
+            nw.z = fmaf(-a.lr, g.z, o.z);
+            nw.w = fmaf(-a.lr, g.w, o.w);
+            if (nok) {
+              const int64_t e = dof + a.offW0 + static_cast<int64_t>(u0 + mb + r) * D + n_base + cq;
+              *reinterpret_cast<float4*>(a.master_w + e) = nw;
+              *reinterpret_cast<uint2*>(a.shadow + e) = make_uint2(pack_bf16x2(nw.x, nw.y), pack_bf16x2(nw.z, nw.w));
             }
-            __syncwarp();
           }
+          __syncwarp();
         }
         tc_fence_before();
         mbar_arrive(&tfreeD[buf]);
@@ -529,12 +539,12 @@ cudaError_t launch_b(const CUtensorMap& mW0, const CUtensorMap& mX, const CUtens
 
 bool fused_round_supported(int L, int D, int H, int C, int B) {
   if (L != 2 || C != kFC || H % kFU != 0 || H / kFU > kFMaxCluster || D % 8 != 0) return false;
-  if (B != 32 && B != 64 && B != 128) return false;
-  const int smem = B == 32 ? FCfg<32>::kSmem : B == 64 ? FCfg<64>::kSmem : FCfg<128>::kSmem;
+  if (B != 32 && B != 64) return false;   // a batch of 128 does not fit the shared-memory budget
+  const int smem = B == 32 ? FCfg<32>::kSmem : FCfg<64>::kSmem;
   return smem <= 227 * 1024;
 }
 
-int fused_round_xt_rows(int B) { return B >= 128 ? 32 : 64; }
+int fused_round_xt_rows(int B) { return FCfg<64>::kND; }
 
 cudaError_t launch_fused_round(const CUtensorMap& mW0, const CUtensorMap& mX, const CUtensorMap& mXT,
                                const CUtensorMap& mWm, const FusedRoundArgs& r, cudaStream_t s) {
@@ -561,7 +571,6 @@ cudaError_t launch_fused_round(const CUtensorMap& mW0, const CUtensorMap& mX, co
   switch (r.B) {
     case 32: return launch_b<32>(mW0, mX, mXT, mWm, a, s);
     case 64: return launch_b<64>(mW0, mX, mXT, mWm, a, s);
-    case 128: return launch_b<128>(mW0, mX, mXT, mWm, a, s);
     default: return cudaErrorInvalidValue;
   }
 }
