@@ -258,7 +258,7 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
     if (t < kFU) b0m[t] = a.master[so + a.offB0 + u0 + t];
     if (t < kFC) b1m[t] = a.master[so + a.offB1 + t];
     for (int b = t; b < B; b += kFT) labs[b] = a.labels[(static_cast<int64_t>(s) * a.W + w) * B + b];
-    __syncwarp();
+    __syncthreads();   // the prefetched b0 is read by the F epilogue below
     if (warp >= 4) {   // epilogue F: thread = hidden unit, columns = samples
       int ok = mbar_wait(accF, s & 1, a.err, kDevTimeoutAccum) ? 1 : 0;
       ok = __all_sync(0xffffffffu, ok);
