@@ -2,31 +2,37 @@
 // ReLU units -> 10 classes) in ONE launch (Eq. 4, "otherwise" branch: each
 // worker runs tau_i SGD steps from the global model).
 //
-// One thread-block cluster serves one worker; its H/128 CTAs split the
-// hidden units, CTA r owning units [128 r, 128 r + 128).  Every step of the
-// worker runs inside the cluster:
+// One thread-block cluster serves one worker.  The hidden units come in
+// groups of 128 (one tensor-core tile of rows); each group is served by S
+// CTAs (S = 1 or 2) that split the INPUT dimension: CTA h of the group owns
+// input columns [c_h, c_{h+1}) of the group's 128 rows of W0 (a split on a
+// 64-column K-block boundary).  Cluster rank = group * S + h.  Every step of
+// the worker runs inside the cluster:
 //
-//  F  forward of the hidden layer for the CTA's units:
-//     z[o][b] = sum_k W0[o][k] X[b][k] on tcgen05 (TMA-fed, TMEM accumulator),
-//     h = relu(z + b0[o]) kept as bf16 in shared memory;
-//  H  last layer: partial logits over the CTA's units, summed over the
+//  F  forward: each CTA computes the partial pre-activation of the group's
+//     128 units over its own input columns on tcgen05 (TMA-fed, TMEM
+//     accumulator).  With S = 2 the pair exchanges partials through
+//     distributed shared memory and each CTA keeps 128/S of the units:
+//     z = (part_0 + part_1) + b0, h = relu(z), bf16, in shared memory;
+//  H  last layer for the CTA's units: partial logits, summed over the whole
 //     cluster in rank order through distributed shared memory, softmax
-//     cross-entropy; the masked input gradient dz0[b][o] of the CTA's units is
-//     written straight into a 128-byte-swizzled K-major shared-memory tile
-//     (the A operand of step D); bias gradient and SGD of b0 (own units), of
-//     the head weights (own columns) and, on rank 0, of the head bias;
-//  D  weight gradient of the hidden layer, dW0[o][k] = sum_b dz0[b][o] X[b][k]
-//     on tcgen05 (X^T tiles by TMA, two TMEM buffers so the MMA of one tile
-//     overlaps the epilogue of the previous), with the SGD update of W0 rows
-//     fused in the epilogue (fp32 master read-modify-write and bf16 shadow,
-//     both through a padded staging tile so every global access is a full
-//     line).
+//     cross-entropy; the masked input gradient dz0[b][u] of its units is
+//     written (as bf16) into the 128-byte-swizzled K-major dz0^T tile of
+//     every CTA of its group (the A operand of step D); bias gradient and SGD
+//     of b0 (own units), of the head weights (own columns) and, on rank 0,
+//     of the head bias;
+//  D  weight gradient of the group's 128 rows over the CTA's own input
+//     columns, dW0[o][k] = sum_b dz0[b][o] X[b][k] on tcgen05 (X^T tiles and
+//     the fp32 master tiles by TMA, four buffers), with the SGD update fused
+//     in the epilogue (16-byte staged accesses, full lines).
 //
-// A CTA only ever rewrites the W0 rows, b0 entries and head-weight columns it
-// owns, so the next step reads its own writes; the head bias, written by rank
-// 0, is ordered by the cluster barriers.  Generic-proxy writes that TMA or
-// the tensor core read afterwards are fenced with fence.proxy.async.
-// Arithmetic and rounding points are those of the multi-kernel path.
+// Ownership: a CTA rewrites only its own (rows x columns) block of W0, its
+// own b0 entries and head-weight columns, so its next step reads its own
+// writes; everything it reads from other CTAs (partials, dz0 rows, logits,
+// the head bias written by rank 0) is ordered by cluster barriers.
+// Generic-proxy writes that TMA or the tensor core read afterwards are
+// fenced with fence.proxy.async.  Arithmetic and rounding points are those of
+// the per-layer path (the pair's two partial sums are added in rank order).
 //
 // Warp roles (384 threads): warp 0 lane 0 issues TMA, warp 1 lane 0 issues
 // tcgen05.mma, warp 2 owns the TMEM allocation (all 512 columns: one CTA per
@@ -39,7 +45,7 @@ namespace oscars {
 namespace {
 
 constexpr int kFT = 384;               // threads
-constexpr int kFU = 128;               // hidden units per CTA
+constexpr int kFU = 128;               // hidden units per group (tensor-core rows)
 constexpr int kFC = 10;                // classes
 constexpr int kFMaxCluster = 8;
 constexpr int kFBK = 64;               // K-block (bf16 elements, 128 bytes)
@@ -61,37 +67,69 @@ __device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
 }
 
-// Per-batch-size configuration (all sizes known at compile time).
-template <int B>
+__device__ __forceinline__ float4 ld_dsmem_f32x4(const float* local, uint32_t rank) {
+  uint32_t remote;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(smem_u32(local)), "r"(rank));
+  float4 v;
+  asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
+               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+               : "r"(remote)
+               : "memory");
+  return v;
+}
+
+__device__ __forceinline__ void st_dsmem_b16(void* local, uint32_t rank, __nv_bfloat16 v) {
+  uint32_t remote;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(smem_u32(local)), "r"(rank));
+  const unsigned short bits = *reinterpret_cast<const unsigned short*>(&v);
+  asm volatile("st.shared::cluster.b16 [%0], %1;" ::"r"(remote), "h"(bits) : "memory");
+}
+
+__device__ __forceinline__ unsigned long long global_ns() {
+  unsigned long long v;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(v));
+  return v;
+}
+
+// Per-shape configuration (all sizes known at compile time).
+template <int B, int S>
 struct FCfg {
+  static_assert(B == 32 || B == 64, "batch of 32 or 64");
+  static_assert(S == 1 || S == 2, "one or two CTAs per group");
+  static constexpr int kUPC = kFU / S;                      // units per CTA in steps F (kept) and H
   static constexpr int kStagesF = 4;
   static constexpr int kABytes = kFU * kFBK * 2;            // W0 tile: 128 rows x 64 k
   static constexpr int kBBytes = B * kFBK * 2;              // X tile: B rows x 64 k
-  static constexpr int kND = 32;                            // columns (input features) per weight-gradient tile
+  static constexpr int kND = 32;                            // columns per weight-gradient tile
   static constexpr int kNBD = 4;                            // weight-gradient buffers in flight
-  static constexpr int kKB = (B + kFBK - 1) / kFBK;         // K-blocks of the weight gradient (K = batch)
-  static constexpr int kXtBytes = kND * kFBK * 2 * kKB;     // one X^T tile (all K-blocks)
-  static constexpr int kMsBytes = kFU * kND * 4;            // fp32 master tile: 128 rows x kND columns
+  static constexpr int kXtBytes = kND * kFBK * 2;           // X^T tile: 32 rows x 64 k (K padded)
+  static constexpr int kMsBytes = kFU * kND * 4;            // fp32 master tile: 128 rows x 32 columns
   static constexpr int kBufD = kXtBytes + kMsBytes;
+  static constexpr int kZs = B + 4;                         // row stride of the partial z exchange (floats)
   static constexpr int kPipe = kStagesF * (kABytes + kBBytes);
   static constexpr int kPipeD = kNBD * kBufD;
-  static constexpr int kRegion = kPipe > kPipeD ? kPipe : kPipeD;   // TMA area, reused by both steps
-  static constexpr int kDzT = kFU * 128 * kKB;              // dz0^T tile: 128 rows x (64 k per block)
-  static constexpr int kTpr = 256 / B;                      // threads per row, partial logits (256 threads)
-  static constexpr int kHsd = kFU + 4 * kTpr;               // padded row stride of the float h tile
+  static constexpr int kZBytes = S > 1 ? kFU * kZs * 4 : 0;
+  static constexpr int kRegion0 = kPipe > kPipeD ? kPipe : kPipeD;
+  static constexpr int kRegion = kRegion0 > kZBytes ? kRegion0 : kZBytes;   // TMA area / z exchange
+  static constexpr int kDzT = kFU * 128;                    // dz0^T tile: 128 rows x 64 k (batch padded)
+  static constexpr int kTpr = 256 / B;                      // threads per row, partial logits
+  static constexpr int kHsd = kUPC + 4 * kTpr;              // padded row stride of the float h tile
+  static constexpr int kGrpRows = 256 / (kUPC / 4);         // rows per pass of the input-gradient items
   // shared memory carve-up (bytes, from a 1024-aligned base)
   static constexpr int oRegion = 0;
   static constexpr int oDzT = oRegion + kRegion;
   static constexpr int oHs = oDzT + kDzT;                    // [B][kHsd] float
-  static constexpr int oWc = oHs + B * kHsd * 4;             // [C][128] float
-  static constexpr int oPl = oWc + kFC * kFU * 4;            // [B][C] float
-  static constexpr int oDz = oPl + B * kFC * 4;              // [B][C] float
-  static constexpr int oDzb = oDz + B * kFC * 4;             // [B][C] float
-  static constexpr int oGbp = oDzb + B * kFC * 4;            // [8][128] float
-  static constexpr int oRowLoss = oGbp + 8 * kFU * 4;        // [B] float
-  static constexpr int oPre = (oRowLoss + B * 4 + 15) / 16 * 16;   // H inputs prefetched during F:
-  static constexpr int kPreFloats = kFC * kFU + kFU + 16 + B;       //   W1 master cols, b0, b1, labels
-  static constexpr int oEpi = (oPre + kPreFloats * 4 + 15) / 16 * 16;   // 8 x [32][36] float staging tiles
+  static constexpr int oWc = oHs + B * kHsd * 4;             // [C][kUPC] float (bf16 operand)
+  static constexpr int oW1m = oWc + kFC * kUPC * 4;          // [C][kUPC] fp32 master head columns
+  static constexpr int oPl = oW1m + kFC * kUPC * 4;          // [B][C]
+  static constexpr int oDz = oPl + B * kFC * 4;              // [B][C]
+  static constexpr int oDzb = oDz + B * kFC * 4;             // [B][C]
+  static constexpr int oGbp = oDzb + B * kFC * 4;            // [kGrpRows][kUPC]
+  static constexpr int oRowLoss = oGbp + kGrpRows * kUPC * 4;   // [B]
+  static constexpr int oB0 = oRowLoss + B * 4;               // [kFU] b0 of the group's units
+  static constexpr int oB1 = oB0 + kFU * 4;                  // [16]
+  static constexpr int oLab = oB1 + 16 * 4;                  // [B] int
+  static constexpr int oEpi = (oLab + B * 4 + 15) / 16 * 16; // 8 x [32][36] float staging tiles
   static constexpr int oBar = oEpi + 8 * 32 * 36 * 4;
   static constexpr int kBarBytes = 256;
   static constexpr int kSmem = oBar + kBarBytes + 1024;      // + alignment slack
@@ -114,38 +152,37 @@ struct FusedArgs {
   unsigned long long* phase_ts;   // [max_tau][4] phase start stamps of worker 0 (or null)
 };
 
-__device__ __forceinline__ unsigned long long global_ns() {
-  unsigned long long v;
-  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(v));
-  return v;
+// byte offset of element (row, k) in a K-major 128-byte-swizzled tile of one
+// 64-wide K-block (the layout TMA writes and UMMA reads)
+__device__ __forceinline__ uint32_t sw128_offset(int row, int k) {
+  return static_cast<uint32_t>((row >> 3) * 1024 + (row & 7) * 128 + ((((k >> 3) ^ (row & 7)) & 7) << 4) +
+                               (k & 7) * 2);
 }
 
-// byte offset of element (row, k) in a K-major 128-byte-swizzled tile of
-// `rows` rows per 64-wide K-block (the layout TMA writes and UMMA reads)
-__device__ __forceinline__ uint32_t sw128_offset(int row, int k, int rows) {
-  const int kb = k >> 6, kk = k & 63;
-  return static_cast<uint32_t>(kb * rows * 128 + (row >> 3) * 1024 + (row & 7) * 128 +
-                               ((((kk >> 3) ^ (row & 7)) & 7) << 4) + (kk & 7) * 2);
-}
-
-template <int B>
+template <int B, int S>
 __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_constant__ CUtensorMap mW0,
                                                                  const __grid_constant__ CUtensorMap mX,
                                                                  const __grid_constant__ CUtensorMap mXT,
                                                                  const __grid_constant__ CUtensorMap mWm,
                                                                  const __grid_constant__ FusedArgs a) {
-  using Cfg = FCfg<B>;
+  using Cfg = FCfg<B, S>;
+  constexpr int UPC = Cfg::kUPC;
   extern __shared__ uint8_t fs_raw[];
   uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(fs_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* region = sm + Cfg::oRegion;
+  float* zx = reinterpret_cast<float*>(region);   // [128][kZs] partial z (S = 2), after F
   uint8_t* dzT = sm + Cfg::oDzT;
   float* hs = reinterpret_cast<float*>(sm + Cfg::oHs);
   float* wcs = reinterpret_cast<float*>(sm + Cfg::oWc);
+  float* w1m = reinterpret_cast<float*>(sm + Cfg::oW1m);
   float* pl = reinterpret_cast<float*>(sm + Cfg::oPl);
   float* dz = reinterpret_cast<float*>(sm + Cfg::oDz);
   float* dzb = reinterpret_cast<float*>(sm + Cfg::oDzb);
   float* gbp = reinterpret_cast<float*>(sm + Cfg::oGbp);
   float* rowloss = reinterpret_cast<float*>(sm + Cfg::oRowLoss);
+  float* b0m = reinterpret_cast<float*>(sm + Cfg::oB0);
+  float* b1m = reinterpret_cast<float*>(sm + Cfg::oB1);
+  int* labs = reinterpret_cast<int*>(sm + Cfg::oLab);
   float* epi = reinterpret_cast<float*>(sm + Cfg::oEpi);
   uint64_t* bars = reinterpret_cast<uint64_t*>(sm + Cfg::oBar);
   uint64_t* fullF = bars;                      // [kStagesF]
@@ -155,21 +192,23 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
   uint64_t* accD = fullD + Cfg::kNBD;          // [kNBD] TMEM buffer full
   uint64_t* tfreeD = accD + Cfg::kNBD;         // [kNBD] TMEM + shared buffer drained (128 arrivals)
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(tfreeD + Cfg::kNBD);
-  float* pre = reinterpret_cast<float*>(sm + Cfg::oPre);
-  float* w1m = pre;                            // [C][128] fp32 master W1 columns (src)
-  float* b0m = w1m + kFC * kFU;                // [128] fp32 b0 of own units (src)
-  float* b1m = b0m + kFU;                      // [16] fp32 b1 (src)
-  int* labs = reinterpret_cast<int*>(b1m + 16);   // [B] labels of this step
 
   const int w = blockIdx.x;
   const int rank = static_cast<int>(cluster_ctarank());
   const int ncl = static_cast<int>(gridDim.y);
-  const int u0 = rank * kFU;                    // first hidden unit of this CTA
+  const int grp = rank / S, half = rank % S;    // unit group, column half
+  const int g0 = grp * kFU;                     // first unit of the group
+  const int ku0 = half * UPC;                   // first kept unit within the group
   const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
   const int D = a.D, H = a.H;
   const int tau = a.tau[w];
   const int nkF = (D + kFBK - 1) / kFBK;
-  const int nD = (D + Cfg::kND - 1) / Cfg::kND;
+  const int kb_split = S > 1 ? nkF / 2 : nkF;
+  const int kb_begin = half == 0 ? 0 : kb_split, kb_end = half == 0 ? kb_split : nkF;
+  const int col_begin = kb_begin * kFBK;
+  const int col_end = half == S - 1 ? D : kb_end * kFBK;
+  const int nkf = kb_end - kb_begin;
+  const int nD = (col_end - col_begin + Cfg::kND - 1) / Cfg::kND;
 
   if (t == 0) {
     prefetch_tmap(&mW0);
@@ -202,29 +241,29 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
   const uint32_t tmem = *tmem_slot;
 
   int kcount = 0;   // F K-blocks issued so far (ring position)
-  int dcount = 0;   // D tiles so far (TMEM / X^T double buffer position)
-
+  int dcount = 0;   // D tiles so far (buffer ring position)
   const bool stamp = a.phase_ts && w == 0 && rank == 0 && t == 0;
+
   for (int s = 0; s < tau; ++s) {
     if (stamp) a.phase_ts[s * 4 + 0] = global_ns();
     const int src = s == 0 ? a.global_slot : w;
     const int64_t so = static_cast<int64_t>(src) * a.slot_stride;
     const int64_t dof = static_cast<int64_t>(w) * a.slot_stride;
 
-    // ------------------------------------------------------------ F: forward of the hidden layer
+    // ------------------------------------------------------------ F: partial forward of the group's units
     if (warp == 0 && lane == 0) {
-      fence_proxy_async_global();     // this CTA's generic writes of W0 rows precede these TMA reads
-      for (int kb = 0; kb < nkF; ++kb) {
+      fence_proxy_async_global();     // this CTA's generic writes of W0 precede these TMA reads
+      for (int kb = 0; kb < nkf; ++kb) {
         const int c = kcount + kb, st = c % Cfg::kStagesF;
         if (c >= Cfg::kStagesF && !mbar_wait(&emptyF[st], ((c / Cfg::kStagesF) + 1) & 1, a.err, kDevTimeoutEmpty)) break;
         mbar_arrive_expect_tx(&fullF[st], Cfg::kABytes + Cfg::kBBytes);
         uint8_t* sa = region + st * (Cfg::kABytes + Cfg::kBBytes);
-        tma_load_3d(sa, &mW0, kb * kFBK, u0, src, &fullF[st]);
-        tma_load_4d(sa + Cfg::kABytes, &mX, kb * kFBK, 0, w, s, &fullF[st]);
+        tma_load_3d(sa, &mW0, (kb_begin + kb) * kFBK, g0, src, &fullF[st]);
+        tma_load_4d(sa + Cfg::kABytes, &mX, (kb_begin + kb) * kFBK, 0, w, s, &fullF[st]);
       }
     } else if (warp == 1 && lane == 0) {
       constexpr uint32_t idesc = idesc_bf16_f32(128, B);
-      for (int kb = 0; kb < nkF; ++kb) {
+      for (int kb = 0; kb < nkf; ++kb) {
         const int c = kcount + kb, st = c % Cfg::kStagesF;
         if (!mbar_wait(&fullF[st], (c / Cfg::kStagesF) & 1, a.err, kDevTimeoutFull)) break;
         tc_fence_after();
@@ -237,60 +276,89 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
       }
       umma_commit(accF);
     }
-    kcount += nkF;
-    // every global input of step H, fetched while the tensor core runs F:
-    // head weights of this CTA's columns (bf16 operand and fp32 master), b0 of
-    // its units, the head bias and this step's labels
-    for (int q = t; q < kFC * (kFU / 8); q += kFT) {
-      const int c = q / (kFU / 8), c8 = (q % (kFU / 8)) * 8;
-      const int64_t e = a.offW1 + static_cast<int64_t>(c) * H + u0 + c8;
+    kcount += nkf;
+    // every global input of the F epilogue and of step H, fetched while the tensor core works
+    for (int q = t; q < kFC * (UPC / 8); q += kFT) {
+      const int c = q / (UPC / 8), c8 = (q % (UPC / 8)) * 8;
+      const int64_t e = a.offW1 + static_cast<int64_t>(c) * H + g0 + ku0 + c8;
       const uint4 v = *reinterpret_cast<const uint4*>(a.shadow + so + e);
       const __nv_bfloat162* p2 = reinterpret_cast<const __nv_bfloat162*>(&v);
 #pragma unroll
       for (int j = 0; j < 4; ++j) {
         const float2 f = __bfloat1622float2(p2[j]);
-        wcs[c * kFU + c8 + 2 * j] = f.x;
-        wcs[c * kFU + c8 + 2 * j + 1] = f.y;
+        wcs[c * UPC + c8 + 2 * j] = f.x;
+        wcs[c * UPC + c8 + 2 * j + 1] = f.y;
       }
-      *reinterpret_cast<float4*>(w1m + c * kFU + c8) = *reinterpret_cast<const float4*>(a.master + so + e);
-      *reinterpret_cast<float4*>(w1m + c * kFU + c8 + 4) = *reinterpret_cast<const float4*>(a.master + so + e + 4);
+      *reinterpret_cast<float4*>(w1m + c * UPC + c8) = *reinterpret_cast<const float4*>(a.master + so + e);
+      *reinterpret_cast<float4*>(w1m + c * UPC + c8 + 4) = *reinterpret_cast<const float4*>(a.master + so + e + 4);
     }
-    if (t < kFU) b0m[t] = a.master[so + a.offB0 + u0 + t];
+    if (t < kFU) b0m[t] = a.master[so + a.offB0 + g0 + t];
     if (t < kFC) b1m[t] = a.master[so + a.offB1 + t];
     for (int b = t; b < B; b += kFT) labs[b] = a.labels[(static_cast<int64_t>(s) * a.W + w) * B + b];
     __syncthreads();   // the prefetched b0 is read by the F epilogue below
-    if (warp >= 4) {   // epilogue F: thread = hidden unit, columns = samples
+    if (warp >= 4) {   // epilogue F: thread = unit of the group, columns = samples
       int ok = mbar_wait(accF, s & 1, a.err, kDevTimeoutAccum) ? 1 : 0;
       ok = __all_sync(0xffffffffu, ok);
       tc_fence_after();
       if (ok) {
-        const int quarter = warp & 3, grp = (warp - 4) >> 2;
-        const int ul = quarter * 32 + lane;              // local unit
-        const float bias = b0m[ul];
+        const int quarter = warp & 3, eg = (warp - 4) >> 2;
+        const int u = quarter * 32 + lane;
         const uint32_t trow = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
-        for (int c0 = grp * 32; c0 < B; c0 += 64) {
+        for (int c0 = eg * 32; c0 < B; c0 += 64) {
           float v[32];
           tmem_ld_32x32b_x32(trow + c0, v);
+          if (S == 1) {
+            const float bias = b0m[u];
 #pragma unroll
-          for (int j = 0; j < 32; ++j) hs[(c0 + j) * Cfg::kHsd + ul] = bf16_round(fmaxf(v[j] + bias, 0.f));
+            for (int j = 0; j < 32; ++j) hs[(c0 + j) * Cfg::kHsd + u] = bf16_round(fmaxf(v[j] + bias, 0.f));
+          } else {
+#pragma unroll
+            for (int q = 0; q < 8; ++q)
+              *reinterpret_cast<float4*>(zx + u * Cfg::kZs + c0 + 4 * q) =
+                  make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+          }
         }
       }
     }
     tc_fence_before();
     __syncthreads();
+    if (S > 1) {
+      // pair exchange: z of this CTA's units = part(half 0) + part(half 1) + b0
+      cluster_sync();
+      for (int q = t; q < UPC * (B / 4); q += kFT) {
+        const int ul = q / (B / 4), b4 = (q % (B / 4)) * 4;
+        const int ug = ku0 + ul;                   // unit within the group
+        float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+        for (int j = 0; j < S; ++j) {
+          const float* p = zx + ug * Cfg::kZs + b4;
+          const float4 v = j == half ? *reinterpret_cast<const float4*>(p) : ld_dsmem_f32x4(p, grp * S + j);
+          z.x += v.x;
+          z.y += v.y;
+          z.z += v.z;
+          z.w += v.w;
+        }
+        const float bias = b0m[ug];
+        hs[(b4 + 0) * Cfg::kHsd + ul] = bf16_round(fmaxf(z.x + bias, 0.f));
+        hs[(b4 + 1) * Cfg::kHsd + ul] = bf16_round(fmaxf(z.y + bias, 0.f));
+        hs[(b4 + 2) * Cfg::kHsd + ul] = bf16_round(fmaxf(z.z + bias, 0.f));
+        hs[(b4 + 3) * Cfg::kHsd + ul] = bf16_round(fmaxf(z.w + bias, 0.f));
+      }
+      __syncthreads();
+    }
     if (stamp) a.phase_ts[s * 4 + 1] = global_ns();
 
-    // ------------------------------------------------------------ H: last layer
+    // ------------------------------------------------------------ H: last layer for this CTA's units
     if (t < 256) {   // partial logits: kTpr threads per row, all classes in registers
       const int rb = t / Cfg::kTpr, q = t % Cfg::kTpr;
       float acc[kFC];
 #pragma unroll
       for (int c = 0; c < kFC; ++c) acc[c] = 0.f;
-      for (int k = 4 * q; k < kFU; k += 4 * Cfg::kTpr) {
+      for (int k = 4 * q; k < UPC; k += 4 * Cfg::kTpr) {
         const float4 hv = *reinterpret_cast<const float4*>(hs + rb * Cfg::kHsd + k);
 #pragma unroll
         for (int c = 0; c < kFC; ++c) {
-          const float4 wv = *reinterpret_cast<const float4*>(wcs + c * kFU + k);
+          const float4 wv = *reinterpret_cast<const float4*>(wcs + c * UPC + k);
           acc[c] = fmaf(hv.x, wv.x, acc[c]);
           acc[c] = fmaf(hv.y, wv.y, acc[c]);
           acc[c] = fmaf(hv.z, wv.z, acc[c]);
@@ -314,7 +382,7 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
         if (r < ncl) acc += part[r];
       dz[q] = acc + b1m[q % kFC];
     }
-    cluster_sync();   // all remote reads of pl and all reads of the head bias are done
+    cluster_sync();   // all remote reads of pl (and of the partial z) are done
     for (int b = t; b < B; b += kFT) {
       float z[kFC], e[kFC];
 #pragma unroll
@@ -357,14 +425,15 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
       }
     }
     // masked input gradient dz0[b][u] of this CTA's units: item = (row, 4 units);
-    // 8 warps x 32 lanes x 4 units (warps 8..11 help with the head weight gradient)
+    // written into the dz0^T tile of every CTA of the group
     if (t < 256) {
-      const int u4 = (t & 31) * 4, wg = t >> 5;
+      constexpr int kLanesPerRow = UPC / 4;
+      const int u4 = (t % kLanesPerRow) * 4, rg = t / kLanesPerRow;
       float4 wc[kFC];
 #pragma unroll
-      for (int c = 0; c < kFC; ++c) wc[c] = *reinterpret_cast<const float4*>(wcs + c * kFU + u4);
+      for (int c = 0; c < kFC; ++c) wc[c] = *reinterpret_cast<const float4*>(wcs + c * UPC + u4);
       float4 gs = make_float4(0.f, 0.f, 0.f, 0.f);
-      for (int b = wg; b < B; b += 8) {
+      for (int b = rg; b < B; b += Cfg::kGrpRows) {
         const float4 hv = *reinterpret_cast<const float4*>(hs + b * Cfg::kHsd + u4);
         float4 dh = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
@@ -385,22 +454,28 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
         gs.w += dh.w;
         const float dv[4] = {dh.x, dh.y, dh.z, dh.w};
 #pragma unroll
-        for (int j = 0; j < 4; ++j)
-          *reinterpret_cast<__nv_bfloat16*>(dzT + sw128_offset(u4 + j, b, kFU)) = __float2bfloat16_rn(dv[j]);
+        for (int j = 0; j < 4; ++j) {
+          const __nv_bfloat16 g16 = __float2bfloat16_rn(dv[j]);
+          uint8_t* dst = dzT + sw128_offset(ku0 + u4 + j, b);
+          *reinterpret_cast<__nv_bfloat16*>(dst) = g16;
+#pragma unroll
+          for (int o = 0; o < S; ++o)
+            if (o != half) st_dsmem_b16(dst, grp * S + o, g16);
+        }
       }
-      *reinterpret_cast<float4*>(gbp + wg * kFU + u4) = gs;
+      *reinterpret_cast<float4*>(gbp + rg * UPC + u4) = gs;
     }
     fence_proxy_async_smem();   // dz0^T is read by the tensor core next
     __syncthreads();
-    if (t < kFU) {   // b0 of this CTA's units
+    if (t < UPC) {   // b0 of this CTA's units
       float g = 0.f;
 #pragma unroll
-      for (int r = 0; r < 8; ++r) g += gbp[r * kFU + t];
-      a.master_w[dof + a.offB0 + u0 + t] = fmaf(-a.lr, g, b0m[t]);
+      for (int r = 0; r < Cfg::kGrpRows; ++r) g += gbp[r * UPC + t];
+      a.master_w[dof + a.offB0 + g0 + ku0 + t] = fmaf(-a.lr, g, b0m[ku0 + t]);
     }
     // head weight gradient + SGD of this CTA's columns: item = (class, 4 units)
-    for (int q = t; q < kFC * (kFU / 4); q += kFT) {
-      const int c = q / (kFU / 4), u4 = (q % (kFU / 4)) * 4;
+    for (int q = t; q < kFC * (UPC / 4); q += kFT) {
+      const int c = q / (UPC / 4), u4 = (q % (UPC / 4)) * 4;
       float4 dw = make_float4(0.f, 0.f, 0.f, 0.f);
       for (int b = 0; b < B; ++b) {
         const float g = dzb[b * kFC + c];
@@ -410,8 +485,8 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
         dw.z = fmaf(g, hv.z, dw.z);
         dw.w = fmaf(g, hv.w, dw.w);
       }
-      const int64_t e = a.offW1 + static_cast<int64_t>(c) * H + u0 + u4;
-      const float4 o = *reinterpret_cast<const float4*>(w1m + c * kFU + u4);
+      const int64_t e = a.offW1 + static_cast<int64_t>(c) * H + g0 + ku0 + u4;
+      const float4 o = *reinterpret_cast<const float4*>(w1m + c * UPC + u4);
       float4 nw;
       nw.x = fmaf(-a.lr, dw.x, o.x);
       nw.y = fmaf(-a.lr, dw.y, o.y);
@@ -420,9 +495,13 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
       *reinterpret_cast<float4*>(a.master_w + dof + e) = nw;
       *reinterpret_cast<uint2*>(a.shadow + dof + e) = make_uint2(pack_bf16x2(nw.x, nw.y), pack_bf16x2(nw.z, nw.w));
     }
-
+    if (S > 1) {
+      cluster_sync();             // the partner's dz0^T rows have landed
+      fence_proxy_async_smem();
+    }
     if (stamp) a.phase_ts[s * 4 + 2] = global_ns();
-    // ------------------------------------------------------------ D: weight gradient + SGD of W0 rows
+
+    // ------------------------------------------------------------ D: weight gradient + SGD of own W0 block
     if (warp == 0 && lane == 0) {
       for (int tt = 0; tt < nD; ++tt) {
         const int c = dcount + tt, buf = c % Cfg::kNBD, use = c / Cfg::kNBD;
@@ -430,10 +509,9 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
         if (use >= 1 && !mbar_wait(&tfreeD[buf], (use - 1) & 1, a.err, kDevTimeoutEmpty)) break;
         mbar_arrive_expect_tx(&fullD[buf], Cfg::kBufD);
         uint8_t* dst = region + buf * Cfg::kBufD;
-#pragma unroll
-        for (int kb = 0; kb < Cfg::kKB; ++kb)
-          tma_load_4d(dst + kb * Cfg::kND * 128, &mXT, kb * kFBK, tt * Cfg::kND, w, s, &fullD[buf]);
-        tma_load_3d(dst + Cfg::kXtBytes, &mWm, tt * Cfg::kND, u0, src, &fullD[buf]);   // old W0 rows
+        const int n0 = col_begin + tt * Cfg::kND;
+        tma_load_4d(dst, &mXT, 0, n0, w, s, &fullD[buf]);
+        tma_load_3d(dst + Cfg::kXtBytes, &mWm, n0, g0, src, &fullD[buf]);   // old W0 block
       }
     } else if (warp == 1 && lane == 0) {
       constexpr uint32_t idesc = idesc_bf16_f32(128, Cfg::kND);
@@ -446,26 +524,23 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
         const uint32_t da = smem_u32(dzT);
         const uint32_t dcol = tmem + static_cast<uint32_t>(buf * Cfg::kND);
 #pragma unroll
-        for (int kb = 0; kb < Cfg::kKB; ++kb)
-#pragma unroll
-          for (int j = 0; j < kFBK / 16; ++j)
-            umma_bf16(dcol, smem_desc_k128(da + kb * kFU * 128 + j * 32),
-                      smem_desc_k128(xa + kb * Cfg::kND * 128 + j * 32), idesc, (kb | j) != 0 ? 1u : 0u);
+        for (int j = 0; j < kFBK / 16; ++j)
+          umma_bf16(dcol, smem_desc_k128(da + j * 32), smem_desc_k128(xa + j * 32), idesc, j != 0 ? 1u : 0u);
         umma_commit(&accD[buf]);
       }
     } else if (warp >= 4) {
       // the two warpgroups take alternate tiles; a warp covers 32 rows x 32 columns
-      const int quarter = warp & 3, grp = (warp - 4) >> 2;
-      const int mb = quarter * 32;                       // local rows of this warp
+      const int quarter = warp & 3, eg = (warp - 4) >> 2;
+      const int mb = quarter * 32;                       // rows of this warp within the group
       float* T = epi + (warp - 4) * 32 * 36;   // row stride 36: 16-byte accesses of 8 lanes hit distinct banks
-      for (int tt = grp; tt < nD; tt += 2) {
+      for (int tt = eg; tt < nD; tt += 2) {
         const int c = dcount + tt, buf = c % Cfg::kNBD, use = c / Cfg::kNBD;
         int ok = mbar_wait(&accD[buf], use & 1, a.err, kDevTimeoutAccum) ? 1 : 0;
         ok = __all_sync(0xffffffffu, ok);
         tc_fence_after();
         if (ok) {
           const float* Ms = reinterpret_cast<const float*>(region + buf * Cfg::kBufD + Cfg::kXtBytes);
-          const int n_base = tt * Cfg::kND;              // first input feature of the tile
+          const int n_base = col_begin + tt * Cfg::kND;  // first input column of the tile
           float v[32];
           tmem_ld_32x32b_x32(tmem + (static_cast<uint32_t>(quarter * 32) << 16) + buf * Cfg::kND, v);
 #pragma unroll
@@ -474,7 +549,7 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
           __syncwarp();
           // lane -> (row 4 i + lane / 8, columns 4 (lane % 8) .. + 3): 4 rows per instruction
           const int cq = (lane & 7) * 4;
-          const bool nok = n_base + cq < D;   // D % 8 == 0: a 4-column group is all in or all out
+          const bool nok = n_base + cq < col_end;   // column ends are multiples of 8
 #pragma unroll
           for (int i = 0; i < 8; ++i) {
             const int r = 4 * i + (lane >> 3);
@@ -486,7 +561,7 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
             nw.z = fmaf(-a.lr, g.z, o.z);
             nw.w = fmaf(-a.lr, g.w, o.w);
             if (nok) {
-              const int64_t e = dof + a.offW0 + static_cast<int64_t>(u0 + mb + r) * D + n_base + cq;
+              const int64_t e = dof + a.offW0 + static_cast<int64_t>(g0 + mb + r) * D + n_base + cq;
               *reinterpret_cast<float4*>(a.master_w + e) = nw;
               *reinterpret_cast<uint2*>(a.shadow + e) = make_uint2(pack_bf16x2(nw.x, nw.y), pack_bf16x2(nw.z, nw.w));
             }
@@ -498,11 +573,11 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
       }
     }
     dcount += nD;
-    fence_proxy_async_global();   // W0 rows written here are read by TMA next step
+    fence_proxy_async_global();   // W0 written here is read by TMA next step
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    cluster_sync();               // head bias (rank 0) visible; pl / dz0^T reusable
+    cluster_sync();               // head bias (rank 0) visible; exchange buffers reusable
     if (stamp) a.phase_ts[s * 4 + 3] = global_ns();
   }
   tc_fence_before();
@@ -513,38 +588,45 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
   }
 }
 
-template <int B>
-cudaError_t launch_b(const CUtensorMap& mW0, const CUtensorMap& mX, const CUtensorMap& mXT, const CUtensorMap& mWm,
-                     const FusedArgs& a, cudaStream_t s) {
-  using Cfg = FCfg<B>;
-  cudaError_t e = cudaFuncSetAttribute(fused_mlp2_round_kernel<B>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+template <int B, int S>
+cudaError_t launch_bs(const CUtensorMap& mW0, const CUtensorMap& mX, const CUtensorMap& mXT, const CUtensorMap& mWm,
+                      const FusedArgs& a, cudaStream_t s) {
+  using Cfg = FCfg<B, S>;
+  cudaError_t e = cudaFuncSetAttribute(fused_mlp2_round_kernel<B, S>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        Cfg::kSmem);
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(a.W, a.H / kFU, 1);
+  cfg.gridDim = dim3(a.W, S * (a.H / kFU), 1);
   cfg.blockDim = dim3(kFT, 1, 1);
   cfg.dynamicSmemBytes = Cfg::kSmem;
   cfg.stream = s;
   cudaLaunchAttribute attr[1];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = 1;
-  attr[0].val.clusterDim.y = a.H / kFU;
+  attr[0].val.clusterDim.y = S * (a.H / kFU);
   attr[0].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, fused_mlp2_round_kernel<B>, mW0, mX, mXT, mWm, a);
+  return cudaLaunchKernelEx(&cfg, fused_mlp2_round_kernel<B, S>, mW0, mX, mXT, mWm, a);
 }
+
+// two CTAs per unit group when the cluster stays within 8 CTAs and the input
+// has at least two K-blocks
+int split_for(int D, int H) { return (2 * (H / kFU) <= kFMaxCluster && (D + kFBK - 1) / kFBK >= 2) ? 2 : 1; }
 
 }  // namespace
 
 bool fused_round_supported(int L, int D, int H, int C, int B) {
   if (L != 2 || C != kFC || H % kFU != 0 || H / kFU > kFMaxCluster || D % 8 != 0) return false;
-  if (B != 32 && B != 64) return false;   // a batch of 128 does not fit the shared-memory budget
-  const int smem = B == 32 ? FCfg<32>::kSmem : FCfg<64>::kSmem;
+  if (B != 32 && B != 64) return false;
+  int smem = 0;
+  const int S = split_for(D, H);
+  if (B == 32) smem = S == 2 ? FCfg<32, 2>::kSmem : FCfg<32, 1>::kSmem;
+  else smem = S == 2 ? FCfg<64, 2>::kSmem : FCfg<64, 1>::kSmem;
   return smem <= 227 * 1024;
 }
 
-int fused_round_xt_rows(int B) { return FCfg<64>::kND; }
+int fused_round_xt_rows(int) { return 32; }
 
 cudaError_t launch_fused_round(const CUtensorMap& mW0, const CUtensorMap& mX, const CUtensorMap& mXT,
                                const CUtensorMap& mWm, const FusedRoundArgs& r, cudaStream_t s) {
@@ -568,11 +650,10 @@ cudaError_t launch_fused_round(const CUtensorMap& mW0, const CUtensorMap& mX, co
   a.max_tau = r.max_tau;
   a.err = r.err;
   a.phase_ts = r.phase_ts;
-  switch (r.B) {
-    case 32: return launch_b<32>(mW0, mX, mXT, mWm, a, s);
-    case 64: return launch_b<64>(mW0, mX, mXT, mWm, a, s);
-    default: return cudaErrorInvalidValue;
-  }
+  const int S = split_for(r.D, r.H);
+  if (r.B == 32) return S == 2 ? launch_bs<32, 2>(mW0, mX, mXT, mWm, a, s) : launch_bs<32, 1>(mW0, mX, mXT, mWm, a, s);
+  if (r.B == 64) return S == 2 ? launch_bs<64, 2>(mW0, mX, mXT, mWm, a, s) : launch_bs<64, 1>(mW0, mX, mXT, mWm, a, s);
+  return cudaErrorInvalidValue;
 }
 
 }  // namespace oscars
