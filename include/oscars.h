@@ -90,6 +90,7 @@ typedef struct {
   int32_t search_mode;     /* oscars_search_mode                                */
   const float* const* shard_x;   /* host array of W device pointers, worker i's  */
                                  /* samples [shard_n[i]][dims[0]] fp32 row-major  */
+                                 /* (bf16 MLP: 16-byte aligned)                   */
   const int32_t* const* shard_y; /* host array of W device pointers, labels      */
                                  /* [shard_n[i]] in [0, classes)                  */
   const int64_t* shard_n;        /* host, W shard sizes >= 1                      */

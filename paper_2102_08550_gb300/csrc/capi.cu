@@ -434,10 +434,12 @@ oscars_status build_tables(oscars_ctx* c) {
   return ensure_stage_buffers(c);
 }
 
-cudaError_t refresh_global_shadows(oscars_ctx* c, cudaStream_t s) {
+// bf16 copies of the global slot after it changed; `plain_done`: the merge
+// already wrote the (non-transposed) shadow
+cudaError_t refresh_global_shadows(oscars_ctx* c, cudaStream_t s, bool plain_done = false) {
   if (!c->shadow) return cudaSuccess;
   const int64_t g = static_cast<int64_t>(c->W) * c->P_pad;
-  cudaError_t e = launch_shadow_refresh(c->slab + g, c->shadow + g, c->P_pad, s);
+  cudaError_t e = plain_done ? cudaSuccess : launch_shadow_refresh(c->slab + g, c->shadow + g, c->P_pad, s);
   if (e != cudaSuccess) return e;
   for (const Layer& ly : c->layers) {
     if (ly.offT < 0) continue;
@@ -606,6 +608,9 @@ cudaError_t enqueue_round_mlp(oscars_ctx* c, cudaStream_t st) {
     f.max_tau = c->max_tau;
     f.err = c->err;
     f.phase_ts = (c->flags & 16) ? c->phase_ts : nullptr;
+    f.loss_out = c->loss_dev;
+    f.cursor = c->cursor;
+    f.shard_n = c->dn_tab;
     ProfScope ps(c, "fused_round", st);
     if ((e = launch_fused_round(c->mShadow[0], c->mX4, c->mXT4, c->mWm0, f, st)) != cudaSuccess) return e;
   } else {
@@ -627,6 +632,7 @@ cudaError_t enqueue_round_mlp(oscars_ctx* c, cudaStream_t st) {
       }
     }
   }
+  if (c->fused) return cudaSuccess;   // the round kernel did its own bookkeeping
   const int nc = c->B / kRowsPerLossChunk;
   ProfScope ps(c, "round_bookkeeping", st);
   if ((e = launch_loss_finalize(c->loss_part, c->tau_dev, c->W, c->max_tau, nc, c->B, c->loss_dev, st)) != cudaSuccess)
@@ -896,6 +902,8 @@ oscars_status oscars_create(const oscars_config* cfg, oscars_ctx** out) {
         for (int i = 0; st == OSCARS_OK && i < c->W; ++i) {
           if (!cfg->shard_x[i] || !cfg->shard_y[i] || cfg->shard_n[i] < 1)
             st = fail(c, OSCARS_EINVAL, "MLP: shard " + std::to_string(i) + " is NULL or empty");
+          else if (c->bf16 && (reinterpret_cast<uintptr_t>(cfg->shard_x[i]) & 15))
+            st = fail(c, OSCARS_EINVAL, "bf16 MLP: shard " + std::to_string(i) + " samples must be 16-byte aligned");
           else {
             c->shard_x.push_back(cfg->shard_x[i]);
             c->shard_y.push_back(cfg->shard_y[i]);
@@ -1046,11 +1054,12 @@ oscars_status oscars_push_merge(oscars_ctx* c, const float* const* deltas, const
       cudaError_t r;
       {
         ProfScope ps(c, "merge", st);
-        r = launch_merge(a, xg, c->P_pad, eta, true, st);
+        r = launch_merge(a, xg, c->P_pad, eta, true, st, c->shadow ? c->shadow + static_cast<int64_t>(c->W) * c->P_pad : nullptr);
       }
       if (r != cudaSuccess) return r;
+      if (c->PT_pad == 0) return cudaSuccess;   // no transposed copies to refresh
       ProfScope ps(c, "shadow_refresh", st);
-      return refresh_global_shadows(c, st);
+      return refresh_global_shadows(c, st, true);
     };
     if (c->flags & 1) {
       e = enqueue(c->stream);

@@ -150,6 +150,9 @@ struct FusedArgs {
   int max_tau;
   int* err;
   unsigned long long* phase_ts;   // [max_tau][4] phase start stamps of worker 0 (or null)
+  float* loss_out;                // [W]
+  int64_t* cursor;                // [W]
+  const int64_t* shard_n;         // [W]
 };
 
 // byte offset of element (row, k) in a K-major 128-byte-swizzled tile of one
@@ -580,6 +583,16 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
     cluster_sync();               // head bias (rank 0) visible; exchange buffers reusable
     if (stamp) a.phase_ts[s * 4 + 3] = global_ns();
   }
+  // round bookkeeping of this worker: mean loss over its steps (sum in step
+  // order, fp64) and the data cursor
+  if (rank == 0 && t == 0) {
+    constexpr int nc = B / kRowsPerLossChunk;
+    double sum = 0.0;
+    for (int st = 0; st < tau; ++st)
+      for (int c = 0; c < nc; ++c) sum += a.loss_part[(static_cast<int64_t>(w) * a.max_tau + st) * nc + c];
+    a.loss_out[w] = static_cast<float>(sum / (static_cast<double>(B) * tau));
+    a.cursor[w] = (a.cursor[w] + static_cast<int64_t>(tau) * B) % a.shard_n[w];
+  }
   tc_fence_before();
   __syncthreads();
   if (warp == 2) {
@@ -650,6 +663,9 @@ cudaError_t launch_fused_round(const CUtensorMap& mW0, const CUtensorMap& mX, co
   a.max_tau = r.max_tau;
   a.err = r.err;
   a.phase_ts = r.phase_ts;
+  a.loss_out = r.loss_out;
+  a.cursor = r.cursor;
+  a.shard_n = r.shard_n;
   const int S = split_for(r.D, r.H);
   if (r.B == 32) return S == 2 ? launch_bs<32, 2>(mW0, mX, mXT, mWm, a, s) : launch_bs<32, 1>(mW0, mX, mXT, mWm, a, s);
   if (r.B == 64) return S == 2 ? launch_bs<64, 2>(mW0, mX, mXT, mWm, a, s) : launch_bs<64, 1>(mW0, mX, mXT, mWm, a, s);

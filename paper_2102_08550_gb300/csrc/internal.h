@@ -20,9 +20,10 @@ struct MergeArgs {
   int W;
 };
 
-// x_g <- x_g + eta * sum_k w_k * (replica ? src_k - x_g : src_k), p < P.
+// x_g <- x_g + eta * sum_k w_k * (replica ? src_k - x_g : src_k), p < P;
+// shadow (optional): shadow[p] = bf16(new x_g[p]) in the same pass.
 cudaError_t launch_merge(const MergeArgs& a, float* x_g, int64_t P, float eta, bool replica,
-                         cudaStream_t s);
+                         cudaStream_t s, __nv_bfloat16* shadow = nullptr);
 
 // ---------------------------------------------------------------- scheduler (host)
 int iteration_ticks(const double* speed, int n, int64_t Q, int64_t* t, const char** why);
@@ -154,6 +155,9 @@ struct FusedRoundArgs {
   int max_tau;
   int* err;
   unsigned long long* phase_ts;   // [max_tau][4] phase stamps of worker 0, or null
+  float* loss_out;                // [W] mean mini-batch loss of the round (written at the end)
+  int64_t* cursor;                // [W] advanced by tau * B modulo n at the end
+  const int64_t* shard_n;         // [W]
 };
 // whole-round kernel for input -> H ReLU -> 10 classes (one cluster per worker)
 bool fused_round_supported(int L, int D, int H, int C, int B);

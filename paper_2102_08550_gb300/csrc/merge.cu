@@ -11,6 +11,8 @@
 // (W + 2) * P * 4 bytes.  The pointer table and weights travel in a
 // __grid_constant__ parameter block, so each thread only loads data.
 //
+// In MLP mode the same pass also writes the bf16 operand copy of x_g.
+//
 // Grid: persistent, (SM count) x (resident CTAs per SM) blocks of 256
 // threads striding over 16-byte chunks; each thread keeps 8 independent
 // 16-byte loads in flight per group of 8 workers.
@@ -26,10 +28,10 @@ constexpr int kGroup = 8;
 
 __device__ __forceinline__ float4 ld_stream4(const float4* p) { return __ldcs(p); }
 
-template <bool kReplica>
+template <bool kReplica, bool kShadow>
 __global__ void __launch_bounds__(kThreads) merge_vec4_kernel(const __grid_constant__ MergeArgs a,
                                                               float* __restrict__ x_g, int64_t n4,
-                                                              float eta) {
+                                                              float eta, __nv_bfloat16* __restrict__ shadow) {
   float4* xg4 = reinterpret_cast<float4*>(x_g);
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
   for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n4; i += stride) {
@@ -77,6 +79,8 @@ __global__ void __launch_bounds__(kThreads) merge_vec4_kernel(const __grid_const
     out.z = fmaf(eta, acc.z, x.z);
     out.w = fmaf(eta, acc.w, x.w);
     __stcs(xg4 + i, out);
+    if (kShadow)   // the bf16 operand copy of the new global model, same pass
+      reinterpret_cast<uint2*>(shadow)[i] = make_uint2(pack_bf16x2(out.x, out.y), pack_bf16x2(out.z, out.w));
   }
 }
 
@@ -84,7 +88,8 @@ __global__ void __launch_bounds__(kThreads) merge_vec4_kernel(const __grid_const
 template <bool kReplica>
 __global__ void __launch_bounds__(kThreads) merge_scalar_kernel(const __grid_constant__ MergeArgs a,
                                                                 float* __restrict__ x_g,
-                                                                int64_t begin, int64_t P, float eta) {
+                                                                int64_t begin, int64_t P, float eta,
+                                                                __nv_bfloat16* __restrict__ shadow) {
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
   for (int64_t p = begin + static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; p < P; p += stride) {
     const float x = x_g[p];
@@ -93,7 +98,9 @@ __global__ void __launch_bounds__(kThreads) merge_scalar_kernel(const __grid_con
       const float v = __ldcs(a.src[k] + p);
       acc = fmaf(a.w[k], kReplica ? v - x : v, acc);
     }
-    x_g[p] = fmaf(eta, acc, x);
+    const float out = fmaf(eta, acc, x);
+    x_g[p] = out;
+    if (shadow) shadow[p] = __float2bfloat16_rn(out);
   }
 }
 
@@ -112,9 +119,9 @@ int sm_count() {
 }  // namespace
 
 cudaError_t launch_merge(const MergeArgs& a, float* x_g, int64_t P, float eta, bool replica,
-                         cudaStream_t s) {
+                         cudaStream_t s, __nv_bfloat16* shadow) {
   if (P <= 0) return cudaSuccess;
-  bool aligned = (reinterpret_cast<uintptr_t>(x_g) & 15) == 0;
+  bool aligned = (reinterpret_cast<uintptr_t>(x_g) & 15) == 0 && (reinterpret_cast<uintptr_t>(shadow) & 7) == 0;
   for (int k = 0; k < a.W && aligned; ++k) aligned = (reinterpret_cast<uintptr_t>(a.src[k]) & 15) == 0;
   const int ctas_per_sm = 2048 / kThreads;
   const int64_t n4 = aligned ? P / 4 : 0;
@@ -122,10 +129,15 @@ cudaError_t launch_merge(const MergeArgs& a, float* x_g, int64_t P, float eta, b
     int64_t blocks = static_cast<int64_t>(sm_count()) * ctas_per_sm;
     const int64_t need = (n4 + kThreads - 1) / kThreads;
     if (need < blocks) blocks = need;
-    if (replica)
-      merge_vec4_kernel<true><<<static_cast<unsigned>(blocks), kThreads, 0, s>>>(a, x_g, n4, eta);
+    const unsigned nb = static_cast<unsigned>(blocks);
+    if (replica && shadow)
+      merge_vec4_kernel<true, true><<<nb, kThreads, 0, s>>>(a, x_g, n4, eta, shadow);
+    else if (replica)
+      merge_vec4_kernel<true, false><<<nb, kThreads, 0, s>>>(a, x_g, n4, eta, nullptr);
+    else if (shadow)
+      merge_vec4_kernel<false, true><<<nb, kThreads, 0, s>>>(a, x_g, n4, eta, shadow);
     else
-      merge_vec4_kernel<false><<<static_cast<unsigned>(blocks), kThreads, 0, s>>>(a, x_g, n4, eta);
+      merge_vec4_kernel<false, false><<<nb, kThreads, 0, s>>>(a, x_g, n4, eta, nullptr);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
   }
@@ -135,9 +147,9 @@ cudaError_t launch_merge(const MergeArgs& a, float* x_g, int64_t P, float eta, b
     const int64_t need = (P - begin + kThreads - 1) / kThreads;
     if (need < blocks) blocks = need;
     if (replica)
-      merge_scalar_kernel<true><<<static_cast<unsigned>(blocks), kThreads, 0, s>>>(a, x_g, begin, P, eta);
+      merge_scalar_kernel<true><<<static_cast<unsigned>(blocks), kThreads, 0, s>>>(a, x_g, begin, P, eta, shadow);
     else
-      merge_scalar_kernel<false><<<static_cast<unsigned>(blocks), kThreads, 0, s>>>(a, x_g, begin, P, eta);
+      merge_scalar_kernel<false><<<static_cast<unsigned>(blocks), kThreads, 0, s>>>(a, x_g, begin, P, eta, shadow);
     return cudaGetLastError();
   }
   return cudaSuccess;

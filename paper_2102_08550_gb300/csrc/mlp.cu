@@ -65,15 +65,60 @@ __global__ void __launch_bounds__(256) stage_kernel(const __grid_constant__ Stag
 
 // Every mini-batch of a round at once: grid z = step * W + worker; a CTA
 // whose worker has fewer local steps returns at once.  Step s of worker w
-// lands at offset (s * W + w) of the per-step buffers.
+// lands at offset (s * W + w) of the per-step buffers.  A CTA converts 32
+// rows x 128 features: 16-byte loads of fp32 (D % 4 == 0), 8-byte bf16
+// stores of the row-major copy, and the transposed copy assembled in shared
+// memory and written as 32-byte row pieces.
+constexpr int kStageRows = 32, kStageCols = 128;
+
 __global__ void __launch_bounds__(256) stage_round_kernel(const __grid_constant__ StageArgs a, const int32_t* tau,
                                                           int W) {
+  __shared__ __align__(16) __nv_bfloat16 tile[kStageCols][kStageRows + 8];
   const int z = blockIdx.z;
   const int s = z / W, w = z - s * W;
   if (s >= tau[w]) return;
   const int64_t slot = static_cast<int64_t>(s) * W + w;
   const int64_t off = slot * a.B * a.D;
-  stage_tile(a, w, a.start[w] + static_cast<int64_t>(s) * a.B, a.A0 + off, a.A0T + off, a.labels + slot * a.B);
+  __nv_bfloat16* A0 = a.A0 + off;
+  __nv_bfloat16* A0T = a.A0T + off;
+  const float* X = a.x[w];
+  const int64_t n = a.n[w];
+  const int64_t base = a.start[w] + static_cast<int64_t>(s) * a.B;
+  const int k0 = blockIdx.x * kStageCols, b0 = blockIdx.y * kStageRows;
+  const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;   // 32 x 8
+  const int k = k0 + tx * 4;
+  const bool kok = k < a.D;
+#pragma unroll
+  for (int i = 0; i < kStageRows / 8; ++i) {
+    const int r = ty + 8 * i, b = b0 + r;
+    float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (b < a.B && kok) {
+      const int64_t row = (base + b) % n;
+      v = *reinterpret_cast<const float4*>(X + row * a.D + k);
+      *reinterpret_cast<uint2*>(A0 + static_cast<int64_t>(b) * a.D + k) =
+          make_uint2(pack_bf16x2(v.x, v.y), pack_bf16x2(v.z, v.w));
+    }
+    tile[tx * 4 + 0][r] = __float2bfloat16_rn(v.x);
+    tile[tx * 4 + 1][r] = __float2bfloat16_rn(v.y);
+    tile[tx * 4 + 2][r] = __float2bfloat16_rn(v.z);
+    tile[tx * 4 + 3][r] = __float2bfloat16_rn(v.w);
+  }
+  __syncthreads();
+  {   // 128 feature rows x 32 samples: two 16-sample pieces per row
+    const int kr = threadIdx.x >> 1, piece = threadIdx.x & 1;
+    const int kk = k0 + kr;
+    const int bb = b0 + piece * 16;
+    if (kk < a.D && bb < a.B) {
+      const uint4* src = reinterpret_cast<const uint4*>(&tile[kr][piece * 16]);
+      uint4* dst = reinterpret_cast<uint4*>(A0T + static_cast<int64_t>(kk) * a.B + bb);
+      dst[0] = src[0];
+      dst[1] = src[1];
+    }
+  }
+  if (blockIdx.x == 0 && threadIdx.x < kStageRows) {
+    const int b = b0 + threadIdx.x;
+    if (b < a.B) a.labels[slot * a.B + b] = a.y[w][(base + b) % n];
+  }
 }
 
 // ---------------------------------------------------------------- head forward
@@ -608,7 +653,8 @@ cudaError_t launch_stage(const StageArgs& a, int n_active, cudaStream_t s) {
 }
 
 cudaError_t launch_stage_round(const StageArgs& a, const int32_t* tau, int W, int max_tau, cudaStream_t s) {
-  dim3 grid((a.D + 31) / 32, (a.B + 31) / 32, W * max_tau);
+  if (a.D % 4 != 0 || a.B % 16 != 0) return cudaErrorInvalidValue;
+  dim3 grid((a.D + kStageCols - 1) / kStageCols, (a.B + kStageRows - 1) / kStageRows, W * max_tau);
   stage_round_kernel<<<grid, 256, 0, s>>>(a, tau, W);
   return cudaGetLastError();
 }
