@@ -88,10 +88,12 @@ typedef struct {
   int64_t ticks_per_unit;  /* Q: t_i = max(1, floor(Q / s_i + 0.5)); 0 = 1000   */
   int64_t M;               /* local-step spread bound of Eq. 3, >= 1            */
   int32_t search_mode;     /* oscars_search_mode                                */
-  const float* const* shard_x;   /* host array of W device pointers, worker i's  */
-                                 /* samples [shard_n[i]][dims[0]] fp32 row-major  */
-                                 /* (bf16 MLP: 16-byte aligned)                   */
-  const int32_t* const* shard_y; /* host array of W device pointers, labels      */
+  const float* const* shard_x;   /* host array of W device-accessible pointers,  */
+                                 /* worker i's samples [shard_n[i]][dims[0]] fp32 */
+                                 /* row-major (bf16 MLP: 16-byte aligned).  Pinned */
+                                 /* host memory is accepted: each round's rows are */
+                                 /* then read over the host link by the kernels.   */
+  const int32_t* const* shard_y; /* host array of W device-accessible pointers,  */
                                  /* [shard_n[i]] in [0, classes)                  */
   const int64_t* shard_n;        /* host, W shard sizes >= 1                      */
   const float* init_params;      /* host or device, P fp32 canonical layout,     */

@@ -198,3 +198,22 @@ def test_protocol_errors(cuda_device):
     for k in range(2):
         np.testing.assert_array_equal(replica_flat(ctx, k, cuda_device), x)
     ctx.close()
+
+
+@pytest.mark.parametrize("dims", [[784, 512, 10], [256, 128, 128, 10]], ids=["fused", "per-layer"])
+def test_pinned_host_shards_match_device_shards(cuda_device, dims):
+    """Shards in pinned host memory (read over the host link by the staging
+    kernel) give bit-identical rounds to the same shards in device memory."""
+    w = synth.TrainWorkload("host-shards", 3, dims, 64, 0.05, 256, 6, 2)
+    dev_shards = device_shards(w, cuda_device, n=256)
+    host_shards = [(x.cpu().pin_memory(), y.cpu().pin_memory()) for x, y in dev_shards]
+    outs = []
+    for shards in (dev_shards, host_shards):
+        ctx, _ = make_context(w, shards, cuda_device)
+        for _ in range(2):
+            _, loss = ctx.local_steps()
+            ctx.push_merge()
+        outs.append((pull_flat(ctx, cuda_device), np.array(loss)))
+        ctx.close()
+    np.testing.assert_array_equal(outs[0][0], outs[1][0])
+    np.testing.assert_array_equal(outs[0][1], outs[1][1])
