@@ -9,9 +9,16 @@ round).  The same JSON line carries the server-merge microbenchmarks (P=25.6M,
 W=64 and P=340M, W=8) as GB/s and fraction of HBM bandwidth.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl oscars|reference]
+  python bench.py --compare [--compare-configs cfg1,cfg2,cfg3]
 
 --impl reference times the CPU oracle (the plain numpy restatement of the
 method) on the same workload and metric.
+
+--compare runs the paper's convergence comparison in simulated time instead:
+Oscars rounds against BSP (one step per barrier) and local SGD with a fixed
+period I (the median Oscars tau), each for the same simulated time, and
+prints one JSON line per workload with the eval-loss curves and the ticks each
+scheme needs to reach the loss BSP ends at.
 """
 from __future__ import annotations
 
@@ -46,6 +53,9 @@ def parse():
     ap.add_argument("--merge-reps", type=int, default=20)
     ap.add_argument("--only", choices=["all", "round", "merge"], default="all",
                     help="round: only the Oscars-round benchmark; merge: only the merge microbenchmarks")
+    ap.add_argument("--compare", action="store_true",
+                    help="simulated time-to-loss comparison of Oscars, BSP and fixed-period local SGD")
+    ap.add_argument("--compare-configs", default="cfg1,cfg2,cfg3")
     ap.add_argument("--merge-sizes", default="",
                     help="comma list of P:W merge cases replacing the two default workloads (profiling)")
     return ap.parse_args()
@@ -188,6 +198,22 @@ def roofline_of(name, ms_per_launch, launches_per_round, flops, bytes_, hbm, tfl
             "ms_per_launch": ms_per_launch, "traffic": None}
 
 
+def max_over_ranks(ms: float, world: int, device) -> float:
+    """The slowest rank's time (every rank gets it); identity for one rank."""
+    if world <= 1:
+        return ms
+    import torch
+    t = torch.tensor([ms], dtype=torch.float64, device=device)
+    torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_rate(units_per_rank: float, world: int, max_ms: float) -> float:
+    """Units processed by all ranks divided by the slowest rank's time (weak
+    scaling: every rank runs its own replica of the workload)."""
+    return units_per_rank * world / (max_ms / 1e3)
+
+
 def run_gpu(args, rank, world, local_rank):
     import torch
     import paper_2102_08550_gb300 as P
@@ -232,13 +258,9 @@ def run_gpu(args, rank, world, local_rank):
             one_round()
             evs[i][1].record(stream)
         torch.cuda.synchronize()
-    total_ms = sum(a.elapsed_time(b) for a, b in evs)
-    if world > 1:
-        t = torch.tensor([total_ms], device=dev)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        total_ms = float(t.item())
+    total_ms = max_over_ranks(sum(a.elapsed_time(b) for a, b in evs), world, dev)
     torch.cuda.synchronize()
-    value = samples_per_round * args.steps * world / (total_ms / 1e3)
+    value = whole_job_rate(samples_per_round * args.steps, world, total_ms)
 
     # ---- per-kernel device time: the same round graph with an event node
     # around every kernel (device timeline, no host launch gaps)
@@ -271,7 +293,7 @@ def run_gpu(args, rank, world, local_rank):
     # ---- end to end through the C ABI with host-resident inputs
     e2e = None
     if not args.no_e2e:
-        e2e = run_e2e(args, shards, w, tau, dev, stream)
+        e2e = run_e2e(args, shards, w, tau, dev, stream, world)
 
     merge = None if args.no_merge else run_merge(args, dev, stream, hbm, peak_kind)
     ctx.close()
@@ -282,7 +304,7 @@ def run_gpu(args, rank, world, local_rank):
     return out
 
 
-def run_e2e(args, shards, w, tau, dev, stream):
+def run_e2e(args, shards, w, tau, dev, stream, world=1):
     """End to end through the C ABI with the inputs in HOST memory: the
     shards live in pinned host memory and the library's staging kernel reads
     each round's mini-batches straight from there (over the host link), then
@@ -305,11 +327,11 @@ def run_e2e(args, shards, w, tau, dev, stream):
         _, loss = P.oscars_local_steps(ctx.handle, want_tau=False, want_loss=True)   # D2H of W losses
         P.oscars_push_merge(ctx.handle)
     torch.cuda.synchronize()
-    dt = time.perf_counter() - t0
+    dt = max_over_ranks(time.perf_counter() - t0, world, dev)
     ctx.close()
     samples = int(np.sum(tau)) * w.batch
     h2d = samples * (w.dims[0] * 4 + 4)
-    return {"value": samples * steps / dt, "unit": UNIT, "h2d_bytes_per_step": h2d,
+    return {"value": whole_job_rate(samples * steps, world, dt * 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": 4 * w.num_workers, "steps": steps,
             "note": "host wall clock; shards in pinned host memory read by the staging kernel each round "
                     "(host->device), local steps + merge, per-worker losses read back (device->host)"}
@@ -394,6 +416,57 @@ def cores_used():
         return os.cpu_count()
 
 
+COMPARE = {"cfg1": (synth.CFG1, 20), "cfg2": (synth.CFG2, 30), "cfg3": (synth.CFG3, 10)}
+
+
+def run_compare(args, dev):
+    """Eval loss against simulated time for three schemes on one workload,
+    all through oscars_train with the same data, init and eval set."""
+    import torch
+    import paper_2102_08550_gb300 as P
+    for key in [k for k in args.compare_configs.split(",") if k]:
+        w, oscars_rounds = COMPARE[key]
+        speeds = synth.speeds(w).tolist()
+        t = P.oscars_iteration_ticks(speeds, w.ticks_per_unit)
+        tau_o, B_o = P.oscars_policy_local_steps(P.POLICY_OSCARS, t, w.M)
+        I = max(1, int(round(float(np.median(tau_o)))))
+        horizon = oscars_rounds * B_o
+        shards = [synth.shard_t(w, k, dev) for k in range(w.num_workers)]
+        Xe, ye = synth.eval_t(w, dev)
+        init = torch.from_numpy(synth.flatten_layers(synth.init_layers_np(w))).to(dev)
+        res = {}
+        for name, pol, per in (("oscars", P.POLICY_OSCARS, 1), ("bsp", P.POLICY_BSP, 1),
+                               (f"local_sgd_I{I}", P.POLICY_LOCAL_SGD, I)):
+            tau, B = P.oscars_policy_local_steps(pol, t, w.M, P.SEARCH_CAPPED, per)
+            rounds = max(1, horizon // B)
+            ctx = P.OscarsContext(num_workers=w.num_workers, dims=w.dims, batch=w.batch, lr=w.lr,
+                                  bf16=w.bf16, speed=speeds, ticks_per_unit=w.ticks_per_unit, M=w.M,
+                                  shards=shards, init_params=init,
+                                  stream=torch.cuda.current_stream(dev).cuda_stream)
+            ctx.set_local_steps(tau)
+            torch.cuda.synchronize()
+            t0 = time.perf_counter()
+            log = ctx.train(rounds, Xe, ye)
+            wall = time.perf_counter() - t0
+            ctx.close()
+            step = max(1, len(log) // 20)
+            res[name] = {"tau": tau, "barrier_ticks": B, "rounds": len(log),
+                         "idle_frac": float(1.0 - sum(a * b for a, b in zip(tau, t)) / (B * len(t))),
+                         "samples": len(log) * int(sum(tau)) * w.batch, "final_eval_loss": log[-1]["eval_loss"],
+                         "curve": [[e["ticks"], round(e["eval_loss"], 6)] for e in log[step - 1::step]],
+                         "wall_s": wall, "_log": log}
+        target = res["bsp"]["final_eval_loss"]
+        for r in res.values():
+            log = r.pop("_log")
+            r["ticks_to_target"] = next((e["ticks"] for e in log if e["eval_loss"] <= target), None)
+        base = res["bsp"]["ticks_to_target"]
+        for r in res.values():
+            r["speedup_vs_bsp"] = base / r["ticks_to_target"] if r["ticks_to_target"] else None
+        print(json.dumps({"mode": "compare", "workload": workload_config(w, "n/a")["workload"],
+                          "dtype": "bf16" if w.bf16 else "fp32", "horizon_ticks": horizon,
+                          "target_loss": target, "policies": res}))
+
+
 def run_reference(args):
     w = WORKLOAD
     oracle_rounds(w, max(1, min(args.warmup, 2)), 30.0)          # warm-up (imports, caches)
@@ -422,6 +495,15 @@ def main():
         import torch
         torch.cuda.set_device(local_rank)
         torch.distributed.init_process_group("nccl")
+    if args.compare:
+        import torch
+        from paper_2102_08550_gb300 import _build
+        _build.build()
+        dev = torch.device(f"cuda:{local_rank}")
+        torch.cuda.set_device(dev)
+        if rank == 0:
+            run_compare(args, dev)
+        return
     if args.only == "merge":
         import torch
         from paper_2102_08550_gb300 import _build

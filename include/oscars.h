@@ -69,6 +69,12 @@ typedef enum {
   OSCARS_SEARCH_LITERAL = 1 /* Algorithm 1 as printed; needs min(t) < max(t)   */
 } oscars_search_mode;
 
+typedef enum {
+  OSCARS_POLICY_OSCARS = 0,    /* tau_i from Algorithm 1 (load-balanced rounds)      */
+  OSCARS_POLICY_BSP = 1,       /* tau_i = 1: a barrier after every iteration         */
+  OSCARS_POLICY_LOCAL_SGD = 2  /* tau_i = I: average every I iterations (Motivation)  */
+} oscars_policy;
+
 typedef struct {
   int32_t num_workers;  /* N = W >= 1 (notation table); <= 256, MLP <= 64       */
   int32_t model;        /* oscars_model                                          */
@@ -200,6 +206,30 @@ oscars_status oscars_set_local_steps(oscars_ctx* ctx, const int32_t* tau);
 oscars_status oscars_eval_loss(oscars_ctx* ctx, const float* x, const int32_t* y, int64_t n,
                                float* loss);
 
+/* One round of oscars_train. */
+typedef struct {
+  int64_t ticks;       /* simulated time at the end of the round: max_i clock_i   */
+  int64_t barrier;     /* length of this round in ticks                          */
+  float eval_loss;     /* eval loss of the merged global model (NaN without eval) */
+  float worker_loss;   /* mean over workers of their mean mini-batch loss         */
+} oscars_round_log;
+
+/*
+ * oscars_train - run up to `rounds` rounds natively: oscars_local_steps,
+ * oscars_push_merge from the replicas (weights of the context's rule; the
+ * explicit rule is refused), and, with eval_x != NULL, oscars_eval_loss of
+ * the merged model on eval_x [eval_n][dims[0]] / eval_y [eval_n] (device).
+ * With eval and target_loss > 0 it stops after the first round whose eval
+ * loss is <= target_loss (the time-to-loss of the paper's convergence
+ * comparison).  log: host array of `rounds` entries or NULL; rounds_done
+ * (host, may be NULL) receives the number of rounds run.  Synchronises every
+ * round (it reads the losses).  Errors: those of the calls it makes; EINVAL
+ * for rounds < 1 or eval_n < 1 with eval_x set.
+ */
+oscars_status oscars_train(oscars_ctx* ctx, int32_t rounds, const float* eval_x, const int32_t* eval_y,
+                           int64_t eval_n, float target_loss, oscars_round_log* log,
+                           int32_t* rounds_done);
+
 /*
  * oscars_read_replica - copy worker k's current model (the model it pushes at
  * the barrier; Section "Introduction": each worker holds a model copy) in
@@ -256,6 +286,20 @@ oscars_status oscars_schedule_solve(const int64_t* t_iter, int32_t n, int64_t M,
                                     int32_t search_mode, int64_t* T_star, int64_t* max_wait,
                                     int32_t* tau);
 oscars_status oscars_merge_weights(int32_t rule, const int32_t* tau, int32_t n, float* w);
+
+/*
+ * oscars_policy_local_steps - the local-step counts of one round under a
+ * synchronisation scheme (oscars_policy): Algorithm 1 (with M and the search
+ * mode), BSP (tau_i = 1) or local SGD with period I (tau_i = I, I >= 1; the
+ * scheme of the paper's Motivation, where the fast workers wait for the
+ * slowest).  tau[n] (host) receives the counts and *barrier (host, may be
+ * NULL) the round length max_i tau_i * t_i, which equals T* for Algorithm 1.
+ * Feed tau to oscars_set_local_steps to run a context under the scheme.
+ * Errors: EINVAL (unknown policy, I < 1, or the errors of
+ * oscars_schedule_solve).
+ */
+oscars_status oscars_policy_local_steps(int32_t policy, const int64_t* t_iter, int32_t n, int64_t M,
+                                        int32_t search_mode, int32_t I, int32_t* tau, int64_t* barrier);
 
 /*
  * oscars_merge - the server update of Eq. 4 (first branch) on caller buffers,

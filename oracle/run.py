@@ -8,7 +8,9 @@ the server replaces the global model with the merge of the pushed models
 (first branch).  Speeds are steady (Section "Problem Formulation"), so T* and
 tau are computed once; synchronisation time is ignored, so the simulated
 clock of worker i advances by tau_i * t_i of compute and mod(T*, t_i) of idle
-time (Eq. 1) per round.
+time (Eq. 1) per round.  Under the comparison schemes (BSP, local SGD with a
+fixed period, or any tau given by the caller) the round ends at the last
+push, max_i tau_i * t_i, which for Algorithm 1's tau is T* itself.
 
 Mini-batches (a reading; the data-partition section of the paper is empty):
 worker i reads its shard sequentially from a cursor that persists across
@@ -63,7 +65,7 @@ class OscarsState:
     clock: np.ndarray
     idle: np.ndarray
     t_iter: np.ndarray
-    T_star: int
+    T_star: int          # the round's barrier: T* of Algorithm 1, else max_i tau_i t_i
     max_wait: int
     tau: np.ndarray
 
@@ -72,6 +74,8 @@ def init_state(dims, layers0, t_iter, M: int, mode: int = _sched.CAPPED, tau_ove
     T_star, mw, tau = _sched.schedule(t_iter, M, mode)
     if tau_override is not None:
         tau = np.asarray(tau_override, dtype=np.int32)
+        T_star = _sched.round_barrier(t_iter, tau)
+        mw = int(np.max(T_star - tau.astype(np.int64) * np.asarray(t_iter, np.int64)))
     W = len(t_iter)
     return OscarsState(list(dims), [(W_.copy(), b.copy()) for W_, b in layers0],
                        np.zeros(W, np.int64), np.zeros(W, np.int64), np.zeros(W, np.int64),
@@ -101,7 +105,7 @@ def run_round(state: OscarsState, shards, batch: int, lr: float, rnd: Callable,
     w = _sched.merge_weights(weight_rule, state.tau, weights)
     x_new = _merge.merge_models(flatten(state.x_g), models, w, server_lr)
     state.x_g = unflatten(x_new, state.dims)
-    idle = state.T_star - state.tau.astype(np.int64) * state.t_iter     # = mod(T*, t_i)
+    idle = state.T_star - state.tau.astype(np.int64) * state.t_iter     # = mod(T*, t_i) under Algorithm 1
     state.clock += state.tau.astype(np.int64) * state.t_iter + idle
     state.idle += idle
     return RoundRecord(state.tau.copy(), state.T_star, wl, idle, x_new)
@@ -110,8 +114,10 @@ def run_round(state: OscarsState, shards, batch: int, lr: float, rnd: Callable,
 def run(dims, layers0, shards, speeds=None, t_iter=None, M: int = 8, rounds: int = 1,
         batch: int = 32, lr: float = 0.05, bf16: bool = True, weight_rule: str = "uniform",
         server_lr: float = 1.0, mode: int = _sched.CAPPED, tau_override=None,
-        eval_set=None, ticks_per_unit: int = 1000):
-    """Run ``rounds`` Oscars rounds; returns (final state, [RoundRecord])."""
+        eval_set=None, ticks_per_unit: int = 1000, target_loss=None):
+    """Run ``rounds`` rounds; returns (final state, [RoundRecord]).  With an
+    eval set and a target loss, stop after the first round whose eval loss
+    is at or below the target."""
     if t_iter is None:
         t_iter = _sched.iteration_ticks(speeds, ticks_per_unit)
     rnd = _bf16.round_bf16 if bf16 else _bf16.identity
@@ -122,4 +128,17 @@ def run(dims, layers0, shards, speeds=None, t_iter=None, M: int = 8, rounds: int
         if eval_set is not None:
             rec.eval_loss = _model.loss_of(state.x_g, eval_set[0], eval_set[1], rnd)
         records.append(rec)
+        if target_loss is not None and rec.eval_loss is not None and rec.eval_loss <= target_loss:
+            break
     return state, records
+
+
+def time_to_loss(records, target: float):
+    """Simulated ticks until the global model's eval loss first reaches
+    ``target`` (None if it never does): every round lasts its barrier."""
+    ticks = 0
+    for rec in records:
+        ticks += int(rec.T_star)
+        if rec.eval_loss is not None and rec.eval_loss <= target:
+            return ticks
+    return None

@@ -24,6 +24,19 @@ Readings where the paper is silent or ambiguous:
 * Termination: with all t_i equal the constraint never fails, so the default
   ("capped") search also stops once T > M * max(t).  The "literal" search has
   no cap and is only defined when min(t) < max(t).
+
+The comparison schemes of the paper's Introduction and Motivation share the
+round structure and differ only in the local-step counts:
+
+* BSP: a barrier after every iteration, tau_i = 1;
+* Local SGD with a fixed period I: every worker runs I iterations between
+  averages, tau_i = I, and the fast workers wait for the slowest;
+* Oscars: tau_i from Algorithm 1.
+
+A round ends when the last worker has pushed, at B = max_i tau_i * t_i, and
+worker i idles for B - tau_i * t_i.  For Algorithm 1's counts B equals T*:
+with all waits mod(T*, t_i) > 0 the barrier max_i tau_i t_i would be an
+earlier candidate with strictly smaller waits, so some worker has no wait.
 """
 from __future__ import annotations
 
@@ -95,6 +108,36 @@ def schedule(t_iter, M: int, mode: int = CAPPED):
     """(T*, max wait, tau) of the load-balanced semi-synchronous round."""
     T_star, mw, _ = load_balance_search(t_iter, M, mode)
     return T_star, mw, local_steps(t_iter, T_star)
+
+
+OSCARS = "oscars"
+BSP = "bsp"
+LOCAL_SGD = "local_sgd"
+
+
+def round_barrier(t_iter, tau) -> int:
+    """Length of a round in ticks: the time of the last push, max_i tau_i t_i."""
+    return int(np.max(np.asarray(tau, dtype=np.int64) * np.asarray(t_iter, dtype=np.int64)))
+
+
+def policy_local_steps(policy: str, t_iter, M: int = 1, period: int = 1, mode: int = CAPPED):
+    """(tau, barrier) of one round under a synchronisation scheme: "oscars"
+    (Algorithm 1), "bsp" (tau_i = 1) or "local_sgd" (tau_i = period)."""
+    t = np.asarray(t_iter, dtype=np.int64)
+    if t.size == 0 or np.any(t < 1):
+        raise ValueError("iteration times must be >= 1")
+    if policy == OSCARS:
+        T_star, _, tau = schedule(t, M, mode)
+        return tau, int(T_star)
+    if policy == BSP:
+        tau = np.ones(t.size, dtype=np.int32)
+    elif policy == LOCAL_SGD:
+        if period < 1:
+            raise ValueError("the local-SGD period must be >= 1")
+        tau = np.full(t.size, period, dtype=np.int32)
+    else:
+        raise ValueError(policy)
+    return tau, round_barrier(t, tau)
 
 
 def merge_weights(rule: str, tau, explicit=None) -> np.ndarray:

@@ -19,6 +19,7 @@ OSCARS_OK, OSCARS_EINVAL, OSCARS_ENOMEM, OSCARS_ECUDA, OSCARS_ESTATE, OSCARS_ETI
 MODEL_FLAT, MODEL_MLP = 0, 1
 W_UNIFORM, W_LOCALSTEPS, W_EXPLICIT = 0, 1, 2
 SEARCH_CAPPED, SEARCH_LITERAL = 0, 1
+POLICY_OSCARS, POLICY_BSP, POLICY_LOCAL_SGD = 0, 1, 2
 FLAG_NO_GRAPH = 1
 FLAG_PROFILE = 2
 FLAG_BRANCHES = 4
@@ -41,6 +42,10 @@ class OscarsConfig(ctypes.Structure):
         ("shard_x", POINTER(c_void_p)), ("shard_y", POINTER(c_void_p)), ("shard_n", POINTER(c_int64)),
         ("init_params", c_void_p), ("cuda_stream", c_void_p), ("flags", c_int32),
     ]
+
+
+class OscarsRoundLog(ctypes.Structure):
+    _fields_ = [("ticks", c_int64), ("barrier", c_int64), ("eval_loss", c_float), ("worker_loss", c_float)]
 
 
 _lib = None
@@ -70,6 +75,10 @@ _SIGS = {
     "oscars_phase_times": (c_int32, [c_void_p, c_int32, POINTER(c_double)]),
     "oscars_softreg_steps_noalloc": (c_int32, [c_void_p, c_void_p, c_void_p, c_void_p, c_int64, c_int64, c_int32,
                                                c_int32, c_int32, c_int32, c_float, c_void_p, c_void_p]),
+    "oscars_policy_local_steps": (c_int32, [c_int32, POINTER(c_int64), c_int32, c_int64, c_int32, c_int32,
+                                            POINTER(c_int32), POINTER(c_int64)]),
+    "oscars_train": (c_int32, [c_void_p, c_int32, c_void_p, c_void_p, c_int64, c_float, POINTER(OscarsRoundLog),
+                               POINTER(c_int32)]),
     "oscars_merge": (c_int32, [c_void_p, POINTER(c_void_p), POINTER(c_float), c_int32, c_int64, c_float, c_void_p]),
 }
 
@@ -121,6 +130,27 @@ def oscars_schedule_solve(t_iter: Sequence[int], M: int, search_mode: int = SEAR
     _check(lib().oscars_schedule_solve(_arr(c_int64, t_iter), n, M, search_mode, ctypes.byref(T),
                                        ctypes.byref(mw), tau))
     return T.value, mw.value, list(tau)
+
+
+def oscars_policy_local_steps(policy: int, t_iter: Sequence[int], M: int = 1, search_mode: int = SEARCH_CAPPED,
+                              I: int = 1):
+    """(tau, barrier) of one round under a synchronisation scheme."""
+    n = len(t_iter)
+    tau, B = (c_int32 * n)(), c_int64()
+    _check(lib().oscars_policy_local_steps(policy, _arr(c_int64, t_iter), n, M, search_mode, I, tau,
+                                           ctypes.byref(B)))
+    return list(tau), B.value
+
+
+def oscars_train(ctx: int, rounds: int, eval_x_ptr: Optional[int] = None, eval_y_ptr: Optional[int] = None,
+                 eval_n: int = 0, target_loss: float = 0.0):
+    """Rounds run natively; returns one dict per round run."""
+    log, done = (OscarsRoundLog * rounds)(), c_int32()
+    _check(lib().oscars_train(c_void_p(ctx), rounds, c_void_p(eval_x_ptr) if eval_x_ptr else None,
+                              c_void_p(eval_y_ptr) if eval_y_ptr else None, eval_n, target_loss, log,
+                              ctypes.byref(done)), c_void_p(ctx))
+    return [{"ticks": log[r].ticks, "barrier": log[r].barrier, "eval_loss": log[r].eval_loss,
+             "worker_loss": log[r].worker_loss} for r in range(done.value)]
 
 
 def oscars_merge_weights(rule: int, tau: Sequence[int]):
@@ -322,6 +352,11 @@ class OscarsContext:
 
     def eval_loss(self, x, y) -> float:
         return oscars_eval_loss(self.handle, x.data_ptr(), y.data_ptr(), x.shape[0])
+
+    def train(self, rounds: int, eval_x=None, eval_y=None, target_loss: float = 0.0):
+        if eval_x is None:
+            return oscars_train(self.handle, rounds)
+        return oscars_train(self.handle, rounds, eval_x.data_ptr(), eval_y.data_ptr(), eval_x.shape[0], target_loss)
 
     def close(self):
         if getattr(self, "handle", None):

@@ -14,6 +14,7 @@
 // Inside a slot every W_l and b_l starts on a 64-element boundary; the
 // padding stays zero.
 #include <algorithm>
+#include <limits>
 #include <cstdio>
 #include <cstring>
 #include <new>
@@ -1311,6 +1312,41 @@ oscars_status oscars_profile_reset(oscars_ctx* c) {
   c->prof_ms.clear();
   c->prof_count.clear();
   return OSCARS_OK;
+}
+
+oscars_status oscars_train(oscars_ctx* c, int32_t rounds, const float* eval_x, const int32_t* eval_y,
+                           int64_t eval_n, float target_loss, oscars_round_log* log, int32_t* rounds_done) {
+  if (rounds_done) *rounds_done = 0;
+  if (!c || rounds < 1) return OSCARS_EINVAL;
+  if (eval_x && (!eval_y || eval_n < 1)) return OSCARS_EINVAL;
+  if (c->rule == OSCARS_W_EXPLICIT) return fail(c, OSCARS_EINVAL, "train merges with the context's rule; explicit weights need push_merge");
+  try {
+    std::vector<float> wl(c->W);
+    for (int32_t r = 0; r < rounds; ++r) {
+      oscars_status st = oscars_local_steps(c, nullptr, wl.data());
+      if (st != OSCARS_OK) return st;
+      st = oscars_push_merge(c, nullptr, nullptr);
+      if (st != OSCARS_OK) return st;
+      float ev = std::numeric_limits<float>::quiet_NaN();
+      if (eval_x) {
+        st = oscars_eval_loss(c, eval_x, eval_y, eval_n, &ev);
+        if (st != OSCARS_OK) return st;
+      }
+      if (log) {
+        double m = 0.0;
+        for (int i = 0; i < c->W; ++i) m += wl[i];
+        log[r].ticks = *std::max_element(c->clock.begin(), c->clock.end());
+        log[r].barrier = c->barrier;
+        log[r].eval_loss = ev;
+        log[r].worker_loss = static_cast<float>(m / c->W);
+      }
+      if (rounds_done) *rounds_done = r + 1;
+      if (eval_x && target_loss > 0.f && ev <= target_loss) break;
+    }
+    return OSCARS_OK;
+  } catch (const std::bad_alloc&) {
+    return fail(c, OSCARS_ENOMEM, "host allocation failed");
+  }
 }
 
 oscars_status oscars_num_params(const oscars_ctx* c, int64_t* P) {

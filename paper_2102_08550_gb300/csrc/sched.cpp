@@ -12,6 +12,7 @@
 // candidate; the constraint is strict; ties keep the smallest T; the capped
 // search also stops once T > M * max(t) (with equal t_i the constraint never
 // fails); the literal search has no cap and needs min(t) < max(t).
+#include <algorithm>
 #include <climits>
 #include <cmath>
 #include <cstdint>
@@ -130,6 +131,34 @@ oscars_status oscars_merge_weights(int32_t rule, const int32_t* tau, int32_t n, 
     return OSCARS_EINVAL;
   }
   oscars::merge_weights(rule, tau, n, w);
+  return OSCARS_OK;
+}
+
+oscars_status oscars_policy_local_steps(int32_t policy, const int64_t* t_iter, int32_t n, int64_t M,
+                                        int32_t search_mode, int32_t I, int32_t* tau, int64_t* barrier) {
+  if (!t_iter || !tau || n < 1) return OSCARS_EINVAL;
+  for (int i = 0; i < n; ++i)
+    if (t_iter[i] < 1) return OSCARS_EINVAL;
+  if (policy == OSCARS_POLICY_OSCARS) {
+    const char* why = "";
+    int64_t T = 0;
+    const int st = oscars::schedule_solve(t_iter, n, M, search_mode, &T, nullptr, tau, &why);
+    if (st != OSCARS_OK) return static_cast<oscars_status>(st);
+    if (barrier) *barrier = T;
+    return OSCARS_OK;
+  }
+  int32_t k = 0;
+  if (policy == OSCARS_POLICY_BSP) k = 1;
+  else if (policy == OSCARS_POLICY_LOCAL_SGD) k = I;
+  else return OSCARS_EINVAL;
+  if (k < 1) return OSCARS_EINVAL;
+  int64_t b = 0;   // last push: max_i k * t_i
+  for (int i = 0; i < n; ++i) {
+    if (t_iter[i] > INT64_MAX / k) return OSCARS_EINVAL;
+    tau[i] = k;
+    b = std::max(b, static_cast<int64_t>(k) * t_iter[i]);
+  }
+  if (barrier) *barrier = b;
   return OSCARS_OK;
 }
 

@@ -132,3 +132,29 @@ def test_create_rejects_before_device_work(oscars_lib, change, status):
 
 def test_destroy_null_is_ok(oscars_lib):
     assert oscars_lib.oscars_destroy(None) == 0
+
+
+def test_policy_local_steps_match_oracle(oscars_lib):
+    rng = np.random.default_rng(17)
+    names = {P.POLICY_OSCARS: S.OSCARS, P.POLICY_BSP: S.BSP, P.POLICY_LOCAL_SGD: S.LOCAL_SGD}
+    for trial in range(200):
+        t = [int(v) for v in rng.integers(1, 2000, int(rng.integers(1, 20)))]
+        M = int(rng.integers(1, 12))
+        I = int(rng.integers(1, 9))
+        for pol, name in names.items():
+            tau, B = S.policy_local_steps(name, t, M=M, period=I)
+            assert P.oscars_policy_local_steps(pol, t, M, P.SEARCH_CAPPED, I) == (tau.tolist(), B), (pol, t, M, I)
+
+
+def test_policy_errors(oscars_lib):
+    for pol, I in ((3, 1), (P.POLICY_LOCAL_SGD, 0), (-1, 1)):
+        with pytest.raises(P.OscarsError):
+            P.oscars_policy_local_steps(pol, [3, 5], 4, P.SEARCH_CAPPED, I)
+    with pytest.raises(P.OscarsError):
+        P.oscars_policy_local_steps(P.POLICY_BSP, [0, 5])
+
+
+def test_train_rejects_null_context(oscars_lib):
+    done = ctypes.c_int32(7)
+    assert oscars_lib.oscars_train(None, 1, None, None, 0, 0.0, None, ctypes.byref(done)) == P.OSCARS_EINVAL
+    assert done.value == 0

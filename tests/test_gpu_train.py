@@ -217,3 +217,50 @@ def test_pinned_host_shards_match_device_shards(cuda_device, dims):
         ctx.close()
     np.testing.assert_array_equal(outs[0][0], outs[1][0])
     np.testing.assert_array_equal(outs[0][1], outs[1][1])
+
+
+POLICIES = [("oscars", P.POLICY_OSCARS, 1), ("bsp", P.POLICY_BSP, 1), ("local_sgd_3", P.POLICY_LOCAL_SGD, 3)]
+
+
+@pytest.mark.parametrize("name,policy,period", POLICIES, ids=[p[0] for p in POLICIES])
+def test_policies_train_to_loss(cuda_device, name, policy, period):
+    """The comparison schemes through the native round runner (oscars_train)
+    on the fp32 softmax-regression workload: per-round barriers and clocks
+    exact, eval losses within 1e-3, the merged model within 1e-5, and the
+    early stop at the first round whose eval loss reaches the target."""
+    w = dataclasses.replace(synth.CFG1, samples_per_worker=1024)
+    rounds = 8
+    t, _, _, _ = oracle_schedule(w)
+    tau, barrier = P.oscars_policy_local_steps(policy, t.tolist(), w.M, P.SEARCH_CAPPED, period)
+    ora_name = {P.POLICY_OSCARS: "oscars", P.POLICY_BSP: "bsp", P.POLICY_LOCAL_SGD: "local_sgd"}[policy]
+    tau_o, barrier_o = orun._sched.policy_local_steps(ora_name, t, M=w.M, period=period)
+    assert (tau, barrier) == (tau_o.tolist(), barrier_o)
+    Xe, ye = synth.eval_np(w, n=2048)
+    shards_h = oracle_inputs(w, w.samples_per_worker)
+    layers0 = synth.init_layers_np(w)
+    _, full = orun.run(w.dims, layers0, shards_h, t_iter=t, M=w.M, rounds=rounds, batch=w.batch, lr=w.lr,
+                       bf16=False, tau_override=tau_o, eval_set=(Xe, ye))
+    losses = np.array([r.eval_loss for r in full])
+    # a target crossed at a round whose neighbours are far from it
+    k = 4
+    target = float(0.5 * (losses[k] + losses[k - 1]))
+    assert np.all(np.abs(losses - target) > 1e-3 * target)
+    k_exp = int(np.argmax(losses <= target))
+    ex, ey = torch.from_numpy(Xe).to(cuda_device), torch.from_numpy(ye).to(cuda_device)
+    for tgt in (0.0, target):
+        ctx, _ = make_context(w, device_shards(w, cuda_device, n=w.samples_per_worker), cuda_device)
+        ctx.set_local_steps(tau)
+        log = ctx.train(rounds, ex, ey, target_loss=tgt)
+        n = rounds if tgt == 0.0 else k_exp + 1
+        assert len(log) == n
+        for r in range(n):
+            assert log[r]["barrier"] == barrier and log[r]["ticks"] == (r + 1) * barrier
+            assert abs(log[r]["eval_loss"] - losses[r]) <= LOSS_RTOL * losses[r], (r, log[r], losses[r])
+            assert abs(log[r]["worker_loss"] - full[r].worker_loss.mean()) <= LOSS_RTOL * full[r].worker_loss.mean()
+        assert_within(per_tensor_errors(pull_flat(ctx, cuda_device), full[n - 1].x_g, w.dims),
+                      np.zeros(2), f"{name} after {n} rounds")
+        sch = ctx.schedule()
+        idle = [barrier - a * b for a, b in zip(tau, t.tolist())]
+        assert sch["clock"] == [n * barrier] * w.num_workers and sch["idle"] == [n * i for i in idle]
+        ctx.close()
+    assert orun.time_to_loss(full, target) == (k_exp + 1) * barrier

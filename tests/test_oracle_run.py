@@ -77,3 +77,81 @@ def test_flatten_roundtrip():
     for (a, b), (c, d) in zip(layers, back):
         np.testing.assert_array_equal(a, c)
         np.testing.assert_array_equal(b, d)
+
+
+def test_policy_counts_and_barriers():
+    t = np.array([1000, 1000, 500, 250])
+    tau, B = schedule.policy_local_steps("bsp", t)
+    assert tau.tolist() == [1, 1, 1, 1] and B == 1000
+    tau, B = schedule.policy_local_steps("local_sgd", t, period=3)
+    assert tau.tolist() == [3, 3, 3, 3] and B == 3000
+    tau, B = schedule.policy_local_steps("oscars", t, M=8)
+    assert tau.tolist() == [1, 1, 2, 4] and B == 1000
+
+
+def test_alg1_barrier_is_last_push_brute_force():
+    """T* of Algorithm 1 equals max_i tau_i t_i: some worker never waits."""
+    rng = np.random.default_rng(5)
+    for _ in range(300):
+        t = rng.integers(1, 40, size=rng.integers(1, 6))
+        M = int(rng.integers(1, 6))
+        T, mw, tau = schedule.schedule(t, M)
+        assert schedule.round_barrier(t, tau) == T
+        assert (T % t).min() == 0
+
+
+def test_override_clock_is_last_push():
+    dims = [6, 10]
+    layers, shards = make(dims, 3, 64)
+    t = [700, 300, 200]
+    for tau in ([1, 1, 1], [2, 2, 2], [1, 3, 4]):
+        state, recs = run.run(dims, layers, shards, t_iter=t, M=8, rounds=2, batch=4, lr=0.05,
+                              bf16=False, tau_override=tau)
+        B = max(a * b for a, b in zip(tau, t))
+        assert all(r.T_star == B for r in recs)
+        assert state.clock.tolist() == [2 * B] * 3
+        idle = [B - a * b for a, b in zip(tau, t)]
+        assert state.idle.tolist() == [2 * i for i in idle] and min(idle) == 0
+
+
+def test_local_sgd_period_one_is_bsp():
+    dims = [8, 12, 10]
+    layers, shards = make(dims, 3, 32, seed=7)
+    t = [900, 400, 250]
+    a, ra = run.run(dims, layers, shards, t_iter=t, M=8, rounds=3, batch=4, lr=0.1, bf16=True,
+                    tau_override=schedule.policy_local_steps("local_sgd", t, period=1)[0])
+    b, rb = run.run(dims, layers, shards, t_iter=t, M=8, rounds=3, batch=4, lr=0.1, bf16=True,
+                    tau_override=schedule.policy_local_steps("bsp", t)[0])
+    np.testing.assert_array_equal(run.flatten(a.x_g), run.flatten(b.x_g))
+    assert [r.T_star for r in ra] == [900] * 3
+
+
+def test_oscars_uses_idle_time_of_bsp():
+    """Under Algorithm 1 the workers of the 4-worker example are never idle;
+    under BSP the fast ones idle, so per simulated tick Oscars runs twice as
+    many mini-batches (8 vs 4 per 1000 ticks)."""
+    t = np.array([1000, 1000, 500, 250])
+    tau_o, B_o = schedule.policy_local_steps("oscars", t, M=8)
+    tau_b, B_b = schedule.policy_local_steps("bsp", t)
+    assert (B_o - tau_o * t).sum() == 0
+    assert (B_b - tau_b * t).tolist() == [0, 0, 500, 750]
+    assert tau_o.sum() / B_o == 2 * tau_b.sum() / B_b
+
+
+def test_time_to_loss_and_early_stop():
+    recs = [run.RoundRecord(np.ones(2, np.int32), 100, np.zeros(2), np.zeros(2), eval_loss=v)
+            for v in (2.0, 1.5, 1.2, 0.9)]
+    assert run.time_to_loss(recs, 1.5) == 200
+    assert run.time_to_loss(recs, 0.95) == 400
+    assert run.time_to_loss(recs, 0.5) is None
+    dims = [6, 10]
+    layers, shards = make(dims, 2, 64, seed=9)
+    ev = (shards[0][0][:32], shards[0][1][:32])
+    _, full = run.run(dims, layers, shards, t_iter=[300, 100], M=8, rounds=6, batch=8, lr=0.2,
+                      bf16=False, eval_set=ev)
+    target = full[2].eval_loss
+    _, part = run.run(dims, layers, shards, t_iter=[300, 100], M=8, rounds=6, batch=8, lr=0.2,
+                      bf16=False, eval_set=ev, target_loss=target)
+    k = next(i for i, r in enumerate(full) if r.eval_loss <= target)
+    assert len(part) == k + 1
+    assert run.time_to_loss(part, target) == (k + 1) * 300
