@@ -56,6 +56,8 @@ def parse():
     ap.add_argument("--compare", action="store_true",
                     help="simulated time-to-loss comparison of Oscars, BSP and fixed-period local SGD")
     ap.add_argument("--compare-configs", default="cfg1,cfg2,cfg3")
+    ap.add_argument("--drift-sigma", type=float, default=0.25,
+                    help="--compare: sd of the per-window log-speed step of the drifting-speed scenario")
     ap.add_argument("--merge-sizes", default="",
                     help="comma list of P:W merge cases replacing the two default workloads (profiling)")
     return ap.parse_args()
@@ -467,6 +469,57 @@ def run_compare(args, dev):
                           "target_loss": target, "policies": res}))
 
 
+def run_compare_drift(args, dev, key):
+    """Drifting speeds: each worker's speed is constant over windows of T*_0
+    ticks (the first Oscars barrier) and takes a log-normal step between
+    windows.  Each scheme starts every round with the speeds in force at its
+    simulated time: Oscars re-solves Algorithm 1 (oscars_set_iteration_ticks),
+    "static" keeps the first round's tau while the round lengths follow the
+    true times, BSP runs one step per barrier."""
+    import torch
+    import paper_2102_08550_gb300 as P
+    w, oscars_rounds = COMPARE[key]
+    sp = synth.drifting_speeds(w, 4 * oscars_rounds + 1, sigma=args.drift_sigma)
+    ts = [P.oscars_iteration_ticks(sp[r].tolist(), w.ticks_per_unit) for r in range(sp.shape[0])]
+    tau0, window = P.oscars_policy_local_steps(P.POLICY_OSCARS, ts[0], w.M)
+    horizon = oscars_rounds * window
+    shards = [synth.shard_t(w, k, dev) for k in range(w.num_workers)]
+    Xe, ye = synth.eval_t(w, dev)
+    init = torch.from_numpy(synth.flatten_layers(synth.init_layers_np(w))).to(dev)
+    res = {}
+    for name in ("oscars_adaptive", "oscars_static", "bsp"):
+        ctx = P.OscarsContext(num_workers=w.num_workers, dims=w.dims, batch=w.batch, lr=w.lr, bf16=w.bf16,
+                              speed=sp[0].tolist(), ticks_per_unit=w.ticks_per_unit, M=w.M, shards=shards,
+                              init_params=init, stream=torch.cuda.current_stream(dev).cuda_stream)
+        now, log, samples, busy, span = 0, [], 0, 0, 0
+        while now < horizon:
+            t = ts[min(now // window, len(ts) - 1)]
+            ctx.set_iteration_ticks(t)                     # Algorithm 1 on the times in force
+            if name == "oscars_static":
+                ctx.set_local_steps(tau0)
+            elif name == "bsp":
+                ctx.set_local_steps([1] * w.num_workers)
+            e = ctx.train(1, Xe, ye)[0]
+            sch = ctx.schedule()
+            now += e["barrier"]
+            samples += int(sum(sch["tau"])) * w.batch
+            busy += sum(a * b for a, b in zip(sch["tau"], t))
+            span += e["barrier"] * w.num_workers
+            log.append([now, e["eval_loss"]])
+        ctx.close()
+        res[name] = {"rounds": len(log), "samples": samples, "idle_frac": 1.0 - busy / span,
+                     "final_eval_loss": log[-1][1], "_log": log}
+    target = max(r["final_eval_loss"] for r in res.values())
+    for r in res.values():
+        log = r.pop("_log")
+        r["ticks_to_target"] = next((tk for tk, ev in log if ev <= target), None)
+        step = max(1, len(log) // 20)
+        r["curve"] = [[tk, round(ev, 6)] for tk, ev in log[step - 1::step]]
+    print(json.dumps({"mode": "compare-drift", "workload": workload_config(w, "n/a")["workload"],
+                      "sigma": args.drift_sigma, "window_ticks": window, "horizon_ticks": horizon,
+                      "target_loss": target, "policies": res}))
+
+
 def run_reference(args):
     w = WORKLOAD
     oracle_rounds(w, max(1, min(args.warmup, 2)), 30.0)          # warm-up (imports, caches)
@@ -503,6 +556,8 @@ def main():
         torch.cuda.set_device(dev)
         if rank == 0:
             run_compare(args, dev)
+            for key in [k for k in args.compare_configs.split(",") if k in ("cfg1", "cfg2")]:
+                run_compare_drift(args, dev, key)
         return
     if args.only == "merge":
         import torch

@@ -199,6 +199,18 @@ oscars_status oscars_get_schedule(const oscars_ctx* ctx, int64_t* T_star, int64_
 oscars_status oscars_set_local_steps(oscars_ctx* ctx, const int32_t* tau);
 
 /*
+ * oscars_set_iteration_ticks - new iteration times t_iter[W] (host, ticks
+ * >= 1), e.g. measured ones when worker speeds drift (the volatile cloud of
+ * the paper's Introduction; the method itself assumes steady speeds, Section
+ * "Problem Formulation").  Re-runs Algorithm 1 with the context's M and
+ * search mode and replaces tau and the barrier T* for the following rounds;
+ * the simulated clocks keep what they have accumulated.  Errors: EINVAL
+ * (those of oscars_schedule_solve; the context is unchanged), ESTATE while a
+ * round is pending.
+ */
+oscars_status oscars_set_iteration_ticks(oscars_ctx* ctx, const int64_t* t_iter);
+
+/*
  * oscars_eval_loss - mean softmax cross-entropy of the global model on n
  * samples x [n][dims[0]] fp32 and labels y [n] (both device pointers), with
  * the same operand precision as training.  MLP mode; n >= 1; *loss is host.
@@ -300,6 +312,24 @@ oscars_status oscars_merge_weights(int32_t rule, const int32_t* tau, int32_t n, 
  */
 oscars_status oscars_policy_local_steps(int32_t policy, const int64_t* t_iter, int32_t n, int64_t M,
                                         int32_t search_mode, int32_t I, int32_t* tau, int64_t* barrier);
+
+/*
+ * oscars_partition_sizes - data-partition load balancing (the paper names the
+ * subsection and leaves it empty; this is the library's reading): split a
+ * data set of `total` samples into n contiguous shards whose sizes follow the
+ * per-round consumption of the workers, so that every worker sweeps its shard
+ * in the same number of rounds and every sample is visited equally often.
+ * weight[n] (host, >= 1) are the proportions, normally tau (samples per round
+ * = tau_i * B).  The data set is handed out in whole units of `unit` samples
+ * (normally B): Q = floor(total / unit) units in proportion to the weights
+ * by largest remainder (Hamilton's apportionment; exact integer arithmetic,
+ * ties to the lower index); sizes[n] (host) receive samples, a multiple of
+ * unit each, summing to Q * unit.  sizes is written only on success.
+ * Errors: EINVAL (NULL, n < 1, unit < 1, a weight < 1, or a worker that
+ * would get no unit).
+ */
+oscars_status oscars_partition_sizes(const int64_t* weight, int32_t n, int64_t total, int64_t unit,
+                                     int64_t* sizes);
 
 /*
  * oscars_merge - the server update of Eq. 4 (first branch) on caller buffers,

@@ -82,6 +82,14 @@ def init_state(dims, layers0, t_iter, M: int, mode: int = _sched.CAPPED, tau_ove
                        np.asarray(t_iter, np.int64), T_star, mw, tau)
 
 
+def reschedule(state: OscarsState, t_iter, M: int, mode: int = _sched.CAPPED) -> None:
+    """New iteration times (drifting speeds): Algorithm 1 again for the
+    following rounds; the clocks keep what they have accumulated."""
+    T_star, mw, tau = _sched.schedule(t_iter, M, mode)
+    state.t_iter = np.asarray(t_iter, np.int64)
+    state.T_star, state.max_wait, state.tau = T_star, mw, tau
+
+
 def local_steps(state: OscarsState, worker: int, shard, batch: int, lr: float, rnd: Callable):
     """Worker ``worker`` pulls the global model and runs tau_i local SGD steps."""
     X, y = shard
@@ -114,16 +122,20 @@ def run_round(state: OscarsState, shards, batch: int, lr: float, rnd: Callable,
 def run(dims, layers0, shards, speeds=None, t_iter=None, M: int = 8, rounds: int = 1,
         batch: int = 32, lr: float = 0.05, bf16: bool = True, weight_rule: str = "uniform",
         server_lr: float = 1.0, mode: int = _sched.CAPPED, tau_override=None,
-        eval_set=None, ticks_per_unit: int = 1000, target_loss=None):
+        eval_set=None, ticks_per_unit: int = 1000, target_loss=None, t_per_round=None):
     """Run ``rounds`` rounds; returns (final state, [RoundRecord]).  With an
     eval set and a target loss, stop after the first round whose eval loss
-    is at or below the target."""
+    is at or below the target.  ``t_per_round[r]`` (optional): iteration
+    times in force from round r on (drifting speeds), re-solved with
+    Algorithm 1 before that round."""
     if t_iter is None:
-        t_iter = _sched.iteration_ticks(speeds, ticks_per_unit)
+        t_iter = t_per_round[0] if t_per_round is not None else _sched.iteration_ticks(speeds, ticks_per_unit)
     rnd = _bf16.round_bf16 if bf16 else _bf16.identity
     state = init_state(dims, layers0, t_iter, M, mode, tau_override)
     records = []
-    for _ in range(rounds):
+    for r in range(rounds):
+        if t_per_round is not None and r > 0:
+            reschedule(state, t_per_round[r], M, mode)
         rec = run_round(state, shards, batch, lr, rnd, weight_rule, server_lr)
         if eval_set is not None:
             rec.eval_loss = _model.loss_of(state.x_g, eval_set[0], eval_set[1], rnd)

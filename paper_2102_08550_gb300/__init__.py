@@ -59,6 +59,7 @@ _SIGS = {
     "oscars_get_schedule": (c_int32, [c_void_p, POINTER(c_int64), POINTER(c_int64), POINTER(c_int64),
                                       POINTER(c_int32), POINTER(c_int64), POINTER(c_int64), POINTER(c_int64)]),
     "oscars_set_local_steps": (c_int32, [c_void_p, POINTER(c_int32)]),
+    "oscars_set_iteration_ticks": (c_int32, [c_void_p, POINTER(c_int64)]),
     "oscars_eval_loss": (c_int32, [c_void_p, c_void_p, c_void_p, c_int64, POINTER(c_float)]),
     "oscars_num_params": (c_int32, [c_void_p, POINTER(c_int64)]),
     "oscars_last_error": (ctypes.c_char_p, [c_void_p]),
@@ -77,6 +78,7 @@ _SIGS = {
                                                c_int32, c_int32, c_int32, c_float, c_void_p, c_void_p]),
     "oscars_policy_local_steps": (c_int32, [c_int32, POINTER(c_int64), c_int32, c_int64, c_int32, c_int32,
                                             POINTER(c_int32), POINTER(c_int64)]),
+    "oscars_partition_sizes": (c_int32, [POINTER(c_int64), c_int32, c_int64, c_int64, POINTER(c_int64)]),
     "oscars_train": (c_int32, [c_void_p, c_int32, c_void_p, c_void_p, c_int64, c_float, POINTER(OscarsRoundLog),
                                POINTER(c_int32)]),
     "oscars_merge": (c_int32, [c_void_p, POINTER(c_void_p), POINTER(c_float), c_int32, c_int64, c_float, c_void_p]),
@@ -140,6 +142,13 @@ def oscars_policy_local_steps(policy: int, t_iter: Sequence[int], M: int = 1, se
     _check(lib().oscars_policy_local_steps(policy, _arr(c_int64, t_iter), n, M, search_mode, I, tau,
                                            ctypes.byref(B)))
     return list(tau), B.value
+
+
+def oscars_partition_sizes(weight: Sequence[int], total: int, unit: int = 1):
+    n = len(weight)
+    out = (c_int64 * n)()
+    _check(lib().oscars_partition_sizes(_arr(c_int64, weight), n, total, unit, out))
+    return list(out)
 
 
 def oscars_train(ctx: int, rounds: int, eval_x_ptr: Optional[int] = None, eval_y_ptr: Optional[int] = None,
@@ -222,6 +231,10 @@ def oscars_get_schedule(ctx: int):
 
 def oscars_set_local_steps(ctx: int, tau: Sequence[int]):
     _check(lib().oscars_set_local_steps(c_void_p(ctx), _arr(c_int32, tau)), c_void_p(ctx))
+
+
+def oscars_set_iteration_ticks(ctx: int, t_iter: Sequence[int]):
+    _check(lib().oscars_set_iteration_ticks(c_void_p(ctx), _arr(c_int64, t_iter)), c_void_p(ctx))
 
 
 def oscars_eval_loss(ctx: int, x_ptr: int, y_ptr: int, n: int) -> float:
@@ -349,6 +362,9 @@ class OscarsContext:
 
     def set_local_steps(self, tau):
         oscars_set_local_steps(self.handle, tau)
+
+    def set_iteration_ticks(self, t_iter):
+        oscars_set_iteration_ticks(self.handle, t_iter)
 
     def eval_loss(self, x, y) -> float:
         return oscars_eval_loss(self.handle, x.data_ptr(), y.data_ptr(), x.shape[0])

@@ -383,9 +383,6 @@ oscars_status build_tables(oscars_ctx* c) {
       }
     c->n_active[s] = n;
   }
-  if (c->act_wid) {
-    // tables are reallocated when tau changes
-  }
   // branches: workers sorted by tau (descending), dealt round-robin
   std::vector<int> order(c->W);
   for (int i = 0; i < c->W; ++i) order[i] = i;
@@ -1165,6 +1162,27 @@ oscars_status oscars_set_local_steps(oscars_ctx* c, const int32_t* tau) {
     if (tau[i] < 1) return fail(c, OSCARS_EINVAL, "tau must be >= 1");
   for (int i = 0; i < c->W; ++i) c->tau[i] = tau[i];
   update_barrier(c, false);
+  if (c->model == OSCARS_MODEL_MLP) {
+    cudaStreamSynchronize(c->stream);
+    return build_tables(c);
+  }
+  return OSCARS_OK;
+}
+
+oscars_status oscars_set_iteration_ticks(oscars_ctx* c, const int64_t* t_iter) {
+  if (!c || !t_iter) return OSCARS_EINVAL;
+  if (c->pending) return fail(c, OSCARS_ESTATE, "cannot re-schedule while a round is pending");
+  std::vector<int64_t> t(t_iter, t_iter + c->W);
+  std::vector<int32_t> tau(c->W, 1);
+  int64_t T = 0, mw = 0;
+  const char* why = "";
+  const int r = schedule_solve(t.data(), c->W, c->M, c->search_mode, &T, &mw, tau.data(), &why);
+  if (r != OSCARS_OK) return fail(c, static_cast<oscars_status>(r), why);
+  c->t_iter = t;
+  c->tau = tau;
+  c->T_star = T;
+  c->max_wait = mw;
+  update_barrier(c, true);
   if (c->model == OSCARS_MODEL_MLP) {
     cudaStreamSynchronize(c->stream);
     return build_tables(c);

@@ -16,6 +16,7 @@
 #include <climits>
 #include <cmath>
 #include <cstdint>
+#include <vector>
 
 #include "../../include/oscars.h"
 #include "internal.h"
@@ -159,6 +160,36 @@ oscars_status oscars_policy_local_steps(int32_t policy, const int64_t* t_iter, i
     b = std::max(b, static_cast<int64_t>(k) * t_iter[i]);
   }
   if (barrier) *barrier = b;
+  return OSCARS_OK;
+}
+
+oscars_status oscars_partition_sizes(const int64_t* weight, int32_t n, int64_t total, int64_t unit,
+                                     int64_t* sizes) {
+  if (!weight || !sizes || n < 1 || unit < 1 || total < 0) return OSCARS_EINVAL;
+  const int64_t Q = total / unit;   // whole units to hand out
+  unsigned __int128 wsum = 0;
+  for (int i = 0; i < n; ++i) {
+    if (weight[i] < 1) return OSCARS_EINVAL;
+    wsum += static_cast<unsigned __int128>(weight[i]);
+  }
+  // Hamilton's apportionment: floors of the exact shares, the spare units to
+  // the largest remainders (exact integer arithmetic; ties to the lower index)
+  std::vector<unsigned __int128> rem(n);
+  std::vector<int64_t> units(n);
+  int64_t given = 0;
+  for (int i = 0; i < n; ++i) {
+    const unsigned __int128 num = static_cast<unsigned __int128>(Q) * static_cast<unsigned __int128>(weight[i]);
+    units[i] = static_cast<int64_t>(num / wsum);
+    rem[i] = num % wsum;
+    given += units[i];
+  }
+  std::vector<int> order(n);
+  for (int i = 0; i < n; ++i) order[i] = i;
+  std::stable_sort(order.begin(), order.end(), [&](int a, int b) { return rem[a] > rem[b]; });
+  for (int64_t k = 0; k < Q - given; ++k) units[order[k]] += 1;
+  for (int i = 0; i < n; ++i)
+    if (units[i] < 1) return OSCARS_EINVAL;   // a worker would get no data
+  for (int i = 0; i < n; ++i) sizes[i] = units[i] * unit;
   return OSCARS_OK;
 }
 

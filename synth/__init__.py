@@ -45,6 +45,7 @@ S_MERGE_DELTA = 8
 SEED_SPEED = 1
 SEED_INIT = 2
 SEED_EVAL = 3
+SEED_DRIFT = 4
 
 
 # --------------------------------------------------------------------------
@@ -203,6 +204,16 @@ def speeds(w: TrainWorkload) -> np.ndarray:
         return np.asarray(w.speeds, dtype=np.float64)
     rng = np.random.default_rng(w.seed + SEED_SPEED)
     return rng.lognormal(0.0, 0.5, w.num_workers).astype(np.float64)
+
+
+def drifting_speeds(w: TrainWorkload, rounds: int, sigma: float = 0.3) -> np.ndarray:
+    """[rounds][W] speed factors of a volatile cluster: round 0 has the
+    workload's speeds, then each worker's log-speed takes a Gaussian step of
+    sd ``sigma`` per round (seeded)."""
+    rng = np.random.default_rng(w.seed + SEED_DRIFT)
+    steps = rng.standard_normal((rounds, w.num_workers)) * sigma
+    steps[0] = 0.0
+    return speeds(w)[None, :] * np.exp(np.cumsum(steps, axis=0))
 
 
 def class_means_np(seed: int, d: int) -> np.ndarray:

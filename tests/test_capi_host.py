@@ -158,3 +158,8 @@ def test_train_rejects_null_context(oscars_lib):
     done = ctypes.c_int32(7)
     assert oscars_lib.oscars_train(None, 1, None, None, 0, 0.0, None, ctypes.byref(done)) == P.OSCARS_EINVAL
     assert done.value == 0
+
+
+def test_set_iteration_ticks_null_context(oscars_lib):
+    t = (ctypes.c_int64 * 2)(3, 5)
+    assert oscars_lib.oscars_set_iteration_ticks(None, t) == P.OSCARS_EINVAL

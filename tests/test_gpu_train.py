@@ -264,3 +264,70 @@ def test_policies_train_to_loss(cuda_device, name, policy, period):
         assert sch["clock"] == [n * barrier] * w.num_workers and sch["idle"] == [n * i for i in idle]
         ctx.close()
     assert orun.time_to_loss(full, target) == (k_exp + 1) * barrier
+
+
+def test_drifting_speeds_rescheduled_each_round(cuda_device):
+    """Speeds drift every round; oscars_set_iteration_ticks re-runs
+    Algorithm 1 before each round.  Per-round tau and barrier exact, clocks
+    and idle times exact, merged model within 1e-5 and losses within 1e-3
+    (fp32 softmax regression)."""
+    w = dataclasses.replace(synth.CFG1, samples_per_worker=1024)
+    rounds = 6
+    sp = synth.drifting_speeds(w, rounds, sigma=0.4)
+    ts = [P.oscars_iteration_ticks(sp[r].tolist(), w.ticks_per_unit) for r in range(rounds)]
+    assert len({tuple(t) for t in ts}) > 1
+    ctx, layers0 = make_context(w, device_shards(w, cuda_device, n=w.samples_per_worker), cuda_device)
+    ctx.set_iteration_ticks(ts[0])
+    losses, flats, taus = [], [], []
+    for r in range(rounds):
+        if r > 0:
+            ctx.set_iteration_ticks(ts[r])
+        tau, loss = ctx.local_steps()
+        ctx.push_merge()
+        taus.append(list(tau))
+        losses.append(np.array(loss))
+        flats.append(pull_flat(ctx, cuda_device))
+    sch = ctx.schedule()
+    ctx.close()
+    state, recs = orun.run(w.dims, layers0, oracle_inputs(w, w.samples_per_worker), M=w.M, rounds=rounds,
+                           batch=w.batch, lr=w.lr, bf16=False, t_per_round=[np.asarray(t) for t in ts])
+    for r in range(rounds):
+        assert taus[r] == recs[r].tau.tolist(), r
+        np.testing.assert_allclose(losses[r], recs[r].worker_loss, rtol=LOSS_RTOL)
+        assert_within(per_tensor_errors(flats[r], recs[r].x_g, w.dims), np.zeros(2), f"round {r}")
+    assert sch["clock"] == state.clock.tolist() and sch["idle"] == state.idle.tolist()
+    assert sch["T_star"] == recs[-1].T_star
+
+
+def test_shards_partitioned_by_tau(cuda_device):
+    """Data-partition load balancing: one data set cut into contiguous shards
+    sized by tau (oscars_partition_sizes), so the shards differ in size and
+    every cursor wraps in the same round.  fp32 softmax regression, 4 rounds
+    (the wrap falls inside), against the oracle on the same slices."""
+    from oracle import partition as opart
+    w = synth.CFG1
+    _, _, _, tau = oracle_schedule(w)
+    total = 3 * int(tau.sum()) * w.batch
+    sizes = P.oscars_partition_sizes([int(v) for v in tau], total, w.batch)
+    assert sizes == opart.partition_sizes(tau.tolist(), total, w.batch)
+    assert len(set(sizes)) > 1
+    X, y = synth.shard_np(w, 0, n=total)
+    offs = np.concatenate([[0], np.cumsum(sizes)])
+    Xd, yd = torch.from_numpy(X).to(cuda_device), torch.from_numpy(y).to(cuda_device)
+    shards_d = [(Xd[a:b], yd[a:b]) for a, b in zip(offs[:-1], offs[1:])]
+    shards_h = [(X[a:b], y[a:b]) for a, b in zip(offs[:-1], offs[1:])]
+    ctx, layers0 = make_context(w, shards_d, cuda_device)
+    flats, losses = [], []
+    for _ in range(4):
+        _, loss = ctx.local_steps()
+        ctx.push_merge()
+        losses.append(np.array(loss))
+        flats.append(pull_flat(ctx, cuda_device))
+    ctx.close()
+    t, _, _, _ = oracle_schedule(w)
+    state, recs = orun.run(w.dims, layers0, shards_h, t_iter=t, M=w.M, rounds=4, batch=w.batch, lr=w.lr,
+                           bf16=False)
+    for r in range(4):
+        np.testing.assert_allclose(losses[r], recs[r].worker_loss, rtol=LOSS_RTOL)
+        assert_within(per_tensor_errors(flats[r], recs[r].x_g, w.dims), np.zeros(2), f"round {r}")
+    assert state.cursor.tolist() == (tau.astype(np.int64) * w.batch).tolist()   # wrapped after round 3

@@ -155,3 +155,24 @@ def test_time_to_loss_and_early_stop():
     k = next(i for i, r in enumerate(full) if r.eval_loss <= target)
     assert len(part) == k + 1
     assert run.time_to_loss(part, target) == (k + 1) * 300
+
+
+def test_reschedule_follows_each_rounds_times():
+    """Drifting speeds: every round runs Algorithm 1's counts for the times
+    in force, and the clocks add up the rounds' barriers."""
+    dims = [6, 10]
+    layers, shards = make(dims, 3, 64, seed=11)
+    ts = [[700, 300, 200], [700, 300, 200], [300, 600, 250], [410, 410, 990]]
+    state, recs = run.run(dims, layers, shards, M=6, rounds=4, batch=4, lr=0.05, bf16=False, t_per_round=ts)
+    total = 0
+    for r, rec in enumerate(recs):
+        T, mw, tau = schedule.schedule(ts[r], 6)
+        assert rec.T_star == T and rec.tau.tolist() == tau.tolist()
+        assert rec.idle.tolist() == (T - tau * np.asarray(ts[r])).tolist()
+        total += T
+    assert state.clock.tolist() == [total] * 3
+    # constant times: the same run as without rescheduling
+    a, _ = run.run(dims, layers, shards, M=6, rounds=3, batch=4, lr=0.05, bf16=False, t_per_round=[ts[0]] * 3)
+    b, _ = run.run(dims, layers, shards, t_iter=ts[0], M=6, rounds=3, batch=4, lr=0.05, bf16=False)
+    np.testing.assert_array_equal(run.flatten(a.x_g), run.flatten(b.x_g))
+    assert a.clock.tolist() == b.clock.tolist()

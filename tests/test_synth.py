@@ -57,3 +57,15 @@ def test_workload_sizes():
     assert np.abs(layers[0][0]).max() <= 1 / np.sqrt(784)
     s = synth.speeds(synth.CFG2)
     assert s.shape == (16,) and np.all(s > 0)
+
+
+def test_drifting_speeds():
+    import synth
+    w = synth.CFG2
+    s = synth.drifting_speeds(w, 6, sigma=0.3)
+    assert s.shape == (6, w.num_workers)
+    np.testing.assert_array_equal(s[0], synth.speeds(w))
+    assert np.all(s > 0)
+    np.testing.assert_array_equal(s, synth.drifting_speeds(w, 6, sigma=0.3))   # seeded
+    r = np.log(s[1:] / s[:-1])
+    assert 0.15 < r.std() < 0.45
