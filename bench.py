@@ -167,13 +167,15 @@ def algorithmic_work(w, tau):
         n * (B * H * 2 + C * H * (2 + 4 + 4 + 2) + 2 * B * H * 2 + H * 4 + B * C * 4 + C * 8))
     add("stage", 0.0, n * B * (d[0] * 4 + 2 * d[0] * 2 + 8))
     # the one-launch round of a 2-layer model does all of the above per step
-    # without the intermediate round trips: its work is the sum of the parts,
-    # its bytes the parameters and inputs it must touch (weights read as bf16
-    # and fp32, written as fp32 and bf16, each input read twice as bf16)
+    # and keeps each worker's model on chip for the round: its work is the sum
+    # of the parts, its compulsory bytes the global model read once (the
+    # workers share it through L2), every worker's replica written once, and
+    # each step's staged inputs (X and X^T bf16, labels)
     if L == 2:
-        i, o = d[0], d[1]
+        i = d[0]
+        P_model = sum(a * b + b for a, b in zip(d[:-1], d[1:]))
         fl["fused_round"] = fl["gemm_fwd"] + fl["gemm_dw_sgd"] + fl["head_fwd"] + fl["head_bwd"]
-        by["fused_round"] = n * (o * i * (2 + 4 + 4 + 2) + 2 * B * i * 2 + C * H * (2 + 4 + 4 + 2) + o * 8 + B * 4)
+        by["fused_round"] = P_model * 4.0 * (1 + W) + n * (2 * B * i * 2 + B * 4)
     P_pad = w.num_params   # padding is < 0.1%
     add("merge", 2.0 * W * P_pad, (W + 2) * P_pad * 4.0)
     add("shadow_refresh", 0.0, P_pad * 6.0)

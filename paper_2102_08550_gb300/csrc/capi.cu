@@ -80,20 +80,6 @@ bool make_map4(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, uint6
            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-// 3-D fp32 tensor map without swizzle: boxes of box_x x box_y x 1
-bool make_map_f32(CUtensorMap* m, const void* base, uint64_t dx, uint64_t dy, uint64_t dz, uint64_t stride_y,
-                  uint64_t stride_z, uint32_t box_x, uint32_t box_y) {
-  EncodeTiledFn f = encode_fn();
-  if (!f) return false;
-  cuuint64_t dims[3] = {dx, dy, dz};
-  cuuint64_t strides[2] = {stride_y, stride_z};
-  cuuint32_t box[3] = {box_x, box_y, 1};
-  cuuint32_t es[3] = {1, 1, 1};
-  return f(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, const_cast<void*>(base), dims, strides, box, es,
-           CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-           CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
-}
-
 struct Layer {
   int in, out;
   int64_t offW, offB, offT;  // offT < 0: no transposed copy
@@ -132,6 +118,7 @@ struct oscars_ctx {
   float* loss_dev = nullptr;
   int64_t* cursor = nullptr;
   int32_t* tau_dev = nullptr;
+  int32_t* order_dev = nullptr;         // workers by decreasing tau (launch order of the round kernel)
   int* act_wid = nullptr;  // [max_tau][W]
   int* act_src = nullptr;
   int* lane_ids = nullptr;   // [W] 0..W-1
@@ -158,7 +145,6 @@ struct oscars_ctx {
   std::vector<CUtensorMap> mA0s, mAT0s;
   bool fused = false;                   // whole-round kernel (2-layer MLP)
   CUtensorMap mX4, mXT4;                // staged inputs of every step (fused kernel)
-  CUtensorMap mWm0;                     // fp32 master W0 of every slot (fused kernel)
   unsigned long long* phase_ts = nullptr;   // flag bit 4: phase stamps of the fused round
   // streams / graph
   cudaStream_t stream = nullptr;
@@ -353,9 +339,7 @@ oscars_status ensure_stage_buffers(oscars_ctx* c) {
     const uint64_t per_b = static_cast<uint64_t>(per) * 2;
     if (!make_map4(&c->mX4, c->A0all, D, B, W, cap, D * 2ull, static_cast<uint64_t>(B) * D * 2ull, per_b, B) ||
         !make_map4(&c->mXT4, c->A0Tall, B, D, W, cap, B * 2ull, static_cast<uint64_t>(B) * D * 2ull, per_b,
-                   fused_round_xt_rows(B)) ||
-        !make_map_f32(&c->mWm0, c->slab + c->layers[0].offW, D, c->dims[1], static_cast<uint64_t>(W) + 1, D * 4ull,
-                      c->P_pad * 4ull, fused_round_xt_rows(B), 128))
+                   fused_round_xt_rows(B)))
       return fail(c, OSCARS_ECUDA, "cuTensorMapEncodeTiled failed (fused round inputs)");
   }
   // step 0 doubles as the single-step buffers (evaluation)
@@ -420,6 +404,14 @@ oscars_status build_tables(oscars_ctx* c) {
   cudaError_t e = cudaMemcpy(c->act_wid, wid.data(), wid.size() * sizeof(int), cudaMemcpyHostToDevice);
   if (e == cudaSuccess) e = cudaMemcpy(c->act_src, src.data(), src.size() * sizeof(int), cudaMemcpyHostToDevice);
   if (e == cudaSuccess) e = cudaMemcpy(c->tau_dev, c->tau.data(), c->W * sizeof(int32_t), cudaMemcpyHostToDevice);
+  if (e == cudaSuccess) {   // longest first: workers by decreasing tau, ties by index
+    std::vector<int32_t> ord(c->W);
+    for (int i = 0; i < c->W; ++i) ord[i] = i;
+    std::stable_sort(ord.begin(), ord.end(), [&](int32_t x, int32_t y) { return c->tau[x] > c->tau[y]; });
+    if (!c->order_dev && !dev_alloc(c, &c->order_dev, c->W))
+      return fail(c, OSCARS_ENOMEM, "device allocation failed (worker order)");
+    e = cudaMemcpy(c->order_dev, ord.data(), c->W * sizeof(int32_t), cudaMemcpyHostToDevice);
+  }
   if (e != cudaSuccess) return cuda_fail(c, e, "schedule upload");
   if (c->round_exec) {
     cudaGraphExecDestroy(c->round_exec);
@@ -587,6 +579,7 @@ cudaError_t enqueue_round_mlp(oscars_ctx* c, cudaStream_t st) {
   if (c->fused) {
     FusedRoundArgs f;
     f.tau = c->tau_dev;
+    f.order = c->order_dev;
     f.W = c->W;
     f.D = c->dims[0];
     f.H = c->dims[1];
@@ -595,7 +588,6 @@ cudaError_t enqueue_round_mlp(oscars_ctx* c, cudaStream_t st) {
     f.lr = c->lr;
     f.master = c->slab;
     f.master_w = c->slab;
-    f.shadow = c->shadow;
     f.slot_stride = c->P_pad;
     f.offW0 = c->layers[0].offW;
     f.offB0 = c->layers[0].offB;
@@ -610,7 +602,7 @@ cudaError_t enqueue_round_mlp(oscars_ctx* c, cudaStream_t st) {
     f.cursor = c->cursor;
     f.shard_n = c->dn_tab;
     ProfScope ps(c, "fused_round", st);
-    if ((e = launch_fused_round(c->mShadow[0], c->mX4, c->mXT4, c->mWm0, f, st)) != cudaSuccess) return e;
+    if ((e = launch_fused_round(c->mX4, c->mXT4, f, st)) != cudaSuccess) return e;
   } else {
     if (c->n_br > 1) {
       cudaError_t e2 = cudaEventRecord(c->br_fork, st);

@@ -6,38 +6,63 @@
 // groups of 128 (one tensor-core tile of rows); each group is served by S
 // CTAs (S = 1 or 2) that split the INPUT dimension: CTA h of the group owns
 // input columns [c_h, c_{h+1}) of the group's 128 rows of W0 (a split on a
-// 64-column K-block boundary).  Cluster rank = group * S + h.  Every step of
-// the worker runs inside the cluster:
+// 64-column K-block boundary).  Cluster rank = group * S + h.
+//
+// The worker's model stays on chip for the whole round.  A CTA keeps its
+// block of W0 twice: the fp32 master values in tensor memory (TMEM lane =
+// hidden unit, column = input column) and their bf16 copy, the A operand of
+// the forward GEMM, in shared memory (K-major, 128-byte swizzled K-blocks).
+// Its head-weight columns, its b0 entries and a private copy of the head
+// bias (updated identically by every CTA) live in shared memory.  The model
+// is read from the global slot once, before the first step, and the worker's
+// replica is written once, during the last step.  Per step only the
+// mini-batch (staged bf16 X and X^T tiles, by TMA) and the labels come from
+// global memory.
+//
+// Every step of the worker runs inside the cluster:
 //
 //  F  forward: each CTA computes the partial pre-activation of the group's
-//     128 units over its own input columns on tcgen05 (TMA-fed, TMEM
-//     accumulator).  With S = 2 the pair exchanges partials through
-//     distributed shared memory and each CTA keeps 128/S of the units:
-//     z = (part_0 + part_1) + b0, h = relu(z), bf16, in shared memory;
+//     128 units over its own input columns on tcgen05 (resident W0; the
+//     first X tiles are prefetched during the previous step).  With S = 2
+//     the pair exchanges partials through distributed shared memory and each
+//     CTA keeps 128/S of the units: z = (part_0 + part_1) + b0, h = relu(z),
+//     bf16;
 //  H  last layer for the CTA's units: partial logits, summed over the whole
 //     cluster in rank order through distributed shared memory, softmax
 //     cross-entropy; the masked input gradient dz0[b][u] of its units is
 //     written (as bf16) into the 128-byte-swizzled K-major dz0^T tile of
 //     every CTA of its group (the A operand of step D); bias gradient and SGD
-//     of b0 (own units), of the head weights (own columns) and, on rank 0,
-//     of the head bias;
+//     of b0 (own units), of the head weights (own columns) and of the head
+//     bias;
 //  D  weight gradient of the group's 128 rows over the CTA's own input
-//     columns, dW0[o][k] = sum_b dz0[b][o] X[b][k] on tcgen05 (X^T tiles and
-//     the fp32 master tiles by TMA, four buffers), with the SGD update fused
-//     in the epilogue (16-byte staged accesses, full lines).
+//     columns, dW0[o][k] = sum_b dz0[b][o] X[b][k], on tcgen05 in 32-column
+//     tiles (X^T tiles by TMA into a six-deep ring, the first ones during
+//     step F; three TMEM buffers); the epilogue reads the
+//     gradient and the fp32 master from TMEM, applies W0 <- W0 - lr dW0,
+//     stores the master back to TMEM and its bf16 copy into the resident A
+//     operand.
 //
-// Ownership: a CTA rewrites only its own (rows x columns) block of W0, its
-// own b0 entries and head-weight columns, so its next step reads its own
-// writes; everything it reads from other CTAs (partials, dz0 rows, logits,
-// the head bias written by rank 0) is ordered by cluster barriers.
-// Generic-proxy writes that TMA or the tensor core read afterwards are
-// fenced with fence.proxy.async.  Arithmetic and rounding points are those of
-// the per-layer path (the pair's two partial sums are added in rank order).
+// Ownership: a CTA rewrites only its own block of W0, its own b0 entries and
+// head-weight columns, and its private head bias, so its next step reads its
+// own writes; what it reads from other CTAs (partials, dz0 rows, logits) is
+// ordered by cluster barriers, and a buffer that other CTAs read is not
+// rewritten before a later barrier has proved those reads done.
+// Generic-proxy writes that the tensor core reads are fenced with
+// fence.proxy.async.  Arithmetic and rounding points are those of the
+// per-layer path (the pair's two partial sums are added in rank order).
+//
+// Clusters are launched in order of decreasing tau (a table maps cluster to
+// worker): when fewer clusters fit on the GPU than there are workers, the
+// late ones start as the short workers finish (longest first).
 //
 // Warp roles (384 threads): warp 0 lane 0 issues TMA, warp 1 lane 0 issues
 // tcgen05.mma, warp 2 owns the TMEM allocation (all 512 columns: one CTA per
-// SM), warps 4..11 read TMEM in the epilogues (two warpgroups, each covering
-// the 128 accumulator lanes), all warps share the CUDA-core work of step H.
+// SM), warps 4..11 are the two epilogue warpgroups (each covering the 128
+// TMEM lanes), all warps share the CUDA-core work of step H.
+//
+// TMEM columns: [0, kTAcc) fp32 master of the W0 block; [kTAcc, 512) the
+// forward accumulator (B columns) and, in step D, the three 32-column
+// weight-gradient buffers (the two uses never overlap in time).
 #include "common.cuh"
 #include "internal.h"
 
@@ -49,6 +74,12 @@ constexpr int kFU = 128;               // hidden units per group (tensor-core ro
 constexpr int kFC = 10;                // classes
 constexpr int kFMaxCluster = 8;
 constexpr int kFBK = 64;               // K-block (bf16 elements, 128 bytes)
+constexpr int kND = 32;                // columns per weight-gradient tile
+constexpr int kNBD = 3;                // weight-gradient TMEM buffers
+constexpr int kNXD = 6;                // X^T tile buffers in shared memory
+constexpr int kTAcc = 512 - kNBD * kND;   // first TMEM column of the accumulators = master columns
+constexpr int kMaxKb = (kTAcc + kFBK - 1) / kFBK;   // resident K-blocks of W0
+constexpr int kW0Blk = kFU * kFBK * 2; // one resident K-block: 128 rows x 64 columns bf16
 
 __device__ __forceinline__ void tma_load_4d(void* smem_dst, const CUtensorMap* map, int c0, int c1, int c2, int c3,
                                             uint64_t* bar) {
@@ -57,10 +88,6 @@ __device__ __forceinline__ void tma_load_4d(void* smem_dst, const CUtensorMap* m
       " [%0], [%1, {%2, %3, %4, %5}], [%6];" ::"r"(smem_u32(smem_dst)),
       "l"(reinterpret_cast<uint64_t>(map)), "r"(c0), "r"(c1), "r"(c2), "r"(c3), "r"(smem_u32(bar))
       : "memory");
-}
-
-__device__ __forceinline__ void fence_proxy_async_global() {
-  asm volatile("fence.proxy.async.global;" ::: "memory");
 }
 
 __device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
@@ -91,33 +118,48 @@ __device__ __forceinline__ unsigned long long global_ns() {
   return v;
 }
 
+// byte offset of element (row, k) in a K-major 128-byte-swizzled tile of one
+// 64-wide K-block (the layout TMA writes and UMMA reads)
+__device__ __forceinline__ uint32_t sw128_offset(int row, int k) {
+  return static_cast<uint32_t>((row >> 3) * 1024 + (row & 7) * 128 + ((((k >> 3) ^ (row & 7)) & 7) << 4) +
+                               (k & 7) * 2);
+}
+
+// bf16 copy of columns [c0, c0 + 32) of row r (c0 a multiple of 32) into the
+// resident W0 operand: four 16-byte chunks of one swizzled 128-byte row
+__device__ __forceinline__ void put_w0_row32(uint8_t* w0s, int r, int c0, const float (&v)[32]) {
+  uint8_t* blk = w0s + (c0 / kFBK) * kW0Blk;
+  const int k0 = c0 % kFBK;
+#pragma unroll
+  for (int i = 0; i < 4; ++i)
+    *reinterpret_cast<uint4*>(blk + sw128_offset(r, k0 + 8 * i)) =
+        make_uint4(pack_bf16x2(v[8 * i], v[8 * i + 1]), pack_bf16x2(v[8 * i + 2], v[8 * i + 3]),
+                   pack_bf16x2(v[8 * i + 4], v[8 * i + 5]), pack_bf16x2(v[8 * i + 6], v[8 * i + 7]));
+}
+
 // Per-shape configuration (all sizes known at compile time).
 template <int B, int S>
 struct FCfg {
   static_assert(B == 32 || B == 64, "batch of 32 or 64");
   static_assert(S == 1 || S == 2, "one or two CTAs per group");
+  static_assert(kTAcc + B <= 512, "the forward accumulator must fit the accumulator columns");
   static constexpr int kUPC = kFU / S;                      // units per CTA in steps F (kept) and H
   static constexpr int kStagesF = 4;
-  static constexpr int kABytes = kFU * kFBK * 2;            // W0 tile: 128 rows x 64 k
   static constexpr int kBBytes = B * kFBK * 2;              // X tile: B rows x 64 k
-  static constexpr int kND = 32;                            // columns per weight-gradient tile
-  static constexpr int kNBD = 4;                            // weight-gradient buffers in flight
   static constexpr int kXtBytes = kND * kFBK * 2;           // X^T tile: 32 rows x 64 k (K padded)
-  static constexpr int kMsBytes = kFU * kND * 4;            // fp32 master tile: 128 rows x 32 columns
-  static constexpr int kBufD = kXtBytes + kMsBytes;
+  static constexpr int kDRing = kNXD * kXtBytes;
+  static constexpr int kFRing = kStagesF * kBBytes;
   static constexpr int kZs = B + 4;                         // row stride of the partial z exchange (floats)
-  static constexpr int kPipe = kStagesF * (kABytes + kBBytes);
-  static constexpr int kPipeD = kNBD * kBufD;
   static constexpr int kZBytes = S > 1 ? kFU * kZs * 4 : 0;
-  static constexpr int kRegion0 = kPipe > kPipeD ? kPipe : kPipeD;
-  static constexpr int kRegion = kRegion0 > kZBytes ? kRegion0 : kZBytes;   // TMA area / z exchange
+  static constexpr int kRegion = kDRing + (kFRing > kZBytes ? kFRing : kZBytes);   // D ring | F ring or z
   static constexpr int kDzT = kFU * 128;                    // dz0^T tile: 128 rows x 64 k (batch padded)
   static constexpr int kTpr = 256 / B;                      // threads per row, partial logits
   static constexpr int kHsd = kUPC + 4 * kTpr;              // padded row stride of the float h tile
   static constexpr int kGrpRows = 256 / (kUPC / 4);         // rows per pass of the input-gradient items
   // shared memory carve-up (bytes, from a 1024-aligned base)
   static constexpr int oRegion = 0;
-  static constexpr int oDzT = oRegion + kRegion;
+  static constexpr int oW0 = (oRegion + kRegion + 1023) / 1024 * 1024;
+  static constexpr int oDzT = oW0 + kMaxKb * kW0Blk;
   static constexpr int oHs = oDzT + kDzT;                    // [B][kHsd] float
   static constexpr int oWc = oHs + B * kHsd * 4;             // [C][kUPC] float (bf16 operand)
   static constexpr int oW1m = oWc + kFC * kUPC * 4;          // [C][kUPC] fp32 master head columns
@@ -127,22 +169,21 @@ struct FCfg {
   static constexpr int oGbp = oDzb + B * kFC * 4;            // [kGrpRows][kUPC]
   static constexpr int oRowLoss = oGbp + kGrpRows * kUPC * 4;   // [B]
   static constexpr int oB0 = oRowLoss + B * 4;               // [kFU] b0 of the group's units
-  static constexpr int oB1 = oB0 + kFU * 4;                  // [16]
+  static constexpr int oB1 = oB0 + kFU * 4;                  // [16] head bias (private copy)
   static constexpr int oLab = oB1 + 16 * 4;                  // [B] int
-  static constexpr int oEpi = (oLab + B * 4 + 15) / 16 * 16; // 8 x [32][36] float staging tiles
-  static constexpr int oBar = oEpi + 8 * 32 * 36 * 4;
+  static constexpr int oBar = (oLab + B * 4 + 15) / 16 * 16;
   static constexpr int kBarBytes = 256;
   static constexpr int kSmem = oBar + kBarBytes + 1024;      // + alignment slack
 };
 
 struct FusedArgs {
   const int32_t* tau;       // [W]
+  const int32_t* order;     // [W] worker of each cluster (decreasing tau)
   int W, D, H;
   int global_slot;
   float lr;
-  const float* master;
-  float* master_w;
-  __nv_bfloat16* shadow;
+  const float* master;      // slab read before the first step (the global slot)
+  float* master_w;          // slab written during the last step (slot w)
   int64_t slot_stride;
   int64_t offW0, offB0, offW1, offB1;
   const int32_t* labels;    // [max_tau][W][B]
@@ -155,25 +196,18 @@ struct FusedArgs {
   const int64_t* shard_n;         // [W]
 };
 
-// byte offset of element (row, k) in a K-major 128-byte-swizzled tile of one
-// 64-wide K-block (the layout TMA writes and UMMA reads)
-__device__ __forceinline__ uint32_t sw128_offset(int row, int k) {
-  return static_cast<uint32_t>((row >> 3) * 1024 + (row & 7) * 128 + ((((k >> 3) ^ (row & 7)) & 7) << 4) +
-                               (k & 7) * 2);
-}
-
 template <int B, int S>
-__global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_constant__ CUtensorMap mW0,
-                                                                 const __grid_constant__ CUtensorMap mX,
+__global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_constant__ CUtensorMap mX,
                                                                  const __grid_constant__ CUtensorMap mXT,
-                                                                 const __grid_constant__ CUtensorMap mWm,
                                                                  const __grid_constant__ FusedArgs a) {
   using Cfg = FCfg<B, S>;
   constexpr int UPC = Cfg::kUPC;
   extern __shared__ uint8_t fs_raw[];
   uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(fs_raw) + 1023) & ~uintptr_t(1023));
-  uint8_t* region = sm + Cfg::oRegion;
-  float* zx = reinterpret_cast<float*>(region);   // [128][kZs] partial z (S = 2), after F
+  uint8_t* dring = sm + Cfg::oRegion;                // X^T tiles of step D
+  uint8_t* fring = dring + Cfg::kDRing;              // X tiles of step F
+  float* zx = reinterpret_cast<float*>(fring);       // [128][kZs] partial z (S = 2), after the F MMAs
+  uint8_t* w0s = sm + Cfg::oW0;                      // resident bf16 W0 block
   uint8_t* dzT = sm + Cfg::oDzT;
   float* hs = reinterpret_cast<float*>(sm + Cfg::oHs);
   float* wcs = reinterpret_cast<float*>(sm + Cfg::oWc);
@@ -186,17 +220,17 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
   float* b0m = reinterpret_cast<float*>(sm + Cfg::oB0);
   float* b1m = reinterpret_cast<float*>(sm + Cfg::oB1);
   int* labs = reinterpret_cast<int*>(sm + Cfg::oLab);
-  float* epi = reinterpret_cast<float*>(sm + Cfg::oEpi);
   uint64_t* bars = reinterpret_cast<uint64_t*>(sm + Cfg::oBar);
   uint64_t* fullF = bars;                      // [kStagesF]
   uint64_t* emptyF = fullF + Cfg::kStagesF;    // [kStagesF]
   uint64_t* accF = emptyF + Cfg::kStagesF;     // [1]
-  uint64_t* fullD = accF + 1;                  // [kNBD] X^T + master tile landed
-  uint64_t* accD = fullD + Cfg::kNBD;          // [kNBD] TMEM buffer full
-  uint64_t* tfreeD = accD + Cfg::kNBD;         // [kNBD] TMEM + shared buffer drained (128 arrivals)
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(tfreeD + Cfg::kNBD);
+  uint64_t* fullD = accF + 1;                  // [kNXD] X^T tile landed
+  uint64_t* xfreeD = fullD + kNXD;             // [kNXD] X^T tile consumed by its MMA
+  uint64_t* accD = xfreeD + kNXD;              // [kNBD] TMEM buffer full
+  uint64_t* tfreeD = accD + kNBD;              // [kNBD] TMEM buffer drained (128 arrivals)
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(tfreeD + kNBD);
 
-  const int w = blockIdx.x;
+  const int w = a.order[blockIdx.x];
   const int rank = static_cast<int>(cluster_ctarank());
   const int ncl = static_cast<int>(gridDim.y);
   const int grp = rank / S, half = rank % S;    // unit group, column half
@@ -210,21 +244,27 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
   const int kb_begin = half == 0 ? 0 : kb_split, kb_end = half == 0 ? kb_split : nkF;
   const int col_begin = kb_begin * kFBK;
   const int col_end = half == S - 1 ? D : kb_end * kFBK;
+  const int ncols = col_end - col_begin;        // a multiple of 8
   const int nkf = kb_end - kb_begin;
-  const int nD = (col_end - col_begin + Cfg::kND - 1) / Cfg::kND;
+  const int nD = (ncols + kND - 1) / kND;
+  const int pre_f = nkf < Cfg::kStagesF ? nkf : Cfg::kStagesF;   // X tiles loaded ahead of a step
+  const int pre_d = nD < kNXD ? nD : kNXD;                       // X^T tiles loaded before step D
+  const int64_t gso = static_cast<int64_t>(a.global_slot) * a.slot_stride;
+  const int64_t dof = static_cast<int64_t>(w) * a.slot_stride;
 
   if (t == 0) {
-    prefetch_tmap(&mW0);
     prefetch_tmap(&mX);
     prefetch_tmap(&mXT);
-    prefetch_tmap(&mWm);
     for (int i = 0; i < Cfg::kStagesF; ++i) {
       mbar_init(&fullF[i], 1);
       mbar_init(&emptyF[i], 1);
     }
     mbar_init(accF, 1);
-    for (int i = 0; i < Cfg::kNBD; ++i) {
+    for (int i = 0; i < kNXD; ++i) {
       mbar_init(&fullD[i], 1);
+      mbar_init(&xfreeD[i], 1);
+    }
+    for (int i = 0; i < kNBD; ++i) {
       mbar_init(&accD[i], 1);
       mbar_init(&tfreeD[i], 128);
     }
@@ -235,70 +275,107 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
     tmem_alloc(tmem_slot, 512);
     tmem_relinquish();
   }
-  // zero the dz0^T tile once: for B < 64 its K padding must stay zero
+  // zero the dz0^T tile (its K padding must stay zero for B < 64) and the
+  // resident W0 (columns past the CTA's own stay zero)
   for (int i = t; i < Cfg::kDzT / 16; i += kFT) reinterpret_cast<uint4*>(dzT)[i] = make_uint4(0, 0, 0, 0);
-  fence_proxy_async_smem();
+  for (int i = t; i < kMaxKb * kW0Blk / 16; i += kFT) reinterpret_cast<uint4*>(w0s)[i] = make_uint4(0, 0, 0, 0);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
-
-  int kcount = 0;   // F K-blocks issued so far (ring position)
-  int dcount = 0;   // D tiles so far (buffer ring position)
   const bool stamp = a.phase_ts && w == 0 && rank == 0 && t == 0;
+
+  // producer (warp 0 lane 0): X tiles [from, to) of step s's forward; the
+  // ring position of K-block kb of step s is s * nkf + kb
+  auto issue_f = [&](int s, int from, int to) -> bool {
+    for (int kb = from; kb < to; ++kb) {
+      const int c = s * nkf + kb, st = c % Cfg::kStagesF;
+      if (c >= Cfg::kStagesF && !mbar_wait(&emptyF[st], ((c / Cfg::kStagesF) + 1) & 1, a.err, kDevTimeoutEmpty))
+        return false;
+      mbar_arrive_expect_tx(&fullF[st], Cfg::kBBytes);
+      tma_load_4d(fring + st * Cfg::kBBytes, &mX, (kb_begin + kb) * kFBK, 0, w, s, &fullF[st]);
+    }
+    return true;
+  };
+  // X^T tiles [from, to) of step s's weight gradient (ring position s * nD + tile)
+  auto issue_d = [&](int s, int from, int to) -> bool {
+    for (int tt = from; tt < to; ++tt) {
+      const int c = s * nD + tt, xb = c % kNXD, use = c / kNXD;
+      // the buffer's previous tile must have been read by its MMA
+      if (use >= 1 && !mbar_wait(&xfreeD[xb], (use - 1) & 1, a.err, kDevTimeoutEmpty)) return false;
+      mbar_arrive_expect_tx(&fullD[xb], Cfg::kXtBytes);
+      tma_load_4d(dring + xb * Cfg::kXtBytes, &mXT, 0, col_begin + tt * kND, w, s, &fullD[xb]);
+    }
+    return true;
+  };
+  bool producer_ok = true;
+  if (warp == 0 && lane == 0) producer_ok = issue_f(0, 0, pre_f);
+
+  // the global model, once: fp32 master block into TMEM and its bf16 copy
+  // into the resident operand (epilogue warps); head columns and biases
+  if (warp >= 4) {
+    const int quarter = warp & 3, eg = (warp - 4) >> 2;
+    const int r = quarter * 32 + lane;
+    const uint32_t trow = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
+    const float* src = a.master + gso + a.offW0 + static_cast<int64_t>(g0 + r) * D + col_begin;
+    for (int tt = eg; tt < nD; tt += 2) {
+      const int c0 = tt * kND;
+      float v[32];
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        const float4 x = c0 + 4 * q < ncols ? *reinterpret_cast<const float4*>(src + c0 + 4 * q)
+                                            : make_float4(0.f, 0.f, 0.f, 0.f);
+        v[4 * q] = x.x;
+        v[4 * q + 1] = x.y;
+        v[4 * q + 2] = x.z;
+        v[4 * q + 3] = x.w;
+      }
+      tmem_st_32x32b_x32(trow + c0, v);
+      put_w0_row32(w0s, r, c0, v);
+    }
+    tmem_wait_st();
+  } else {
+    for (int q = t; q < kFC * (UPC / 4); q += 128) {
+      const int c = q / (UPC / 4), u4 = (q % (UPC / 4)) * 4;
+      const float4 m = *reinterpret_cast<const float4*>(a.master + gso + a.offW1 + static_cast<int64_t>(c) * H + g0 +
+                                                       ku0 + u4);
+      *reinterpret_cast<float4*>(w1m + c * UPC + u4) = m;
+      *reinterpret_cast<float4*>(wcs + c * UPC + u4) =
+          make_float4(bf16_round(m.x), bf16_round(m.y), bf16_round(m.z), bf16_round(m.w));
+    }
+    for (int u = t; u < kFU; u += 128) b0m[u] = a.master[gso + a.offB0 + g0 + u];
+    if (t < kFC) b1m[t] = a.master[gso + a.offB1 + t];
+  }
+  fence_proxy_async_smem();   // the resident W0 is read by the tensor core
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
 
   for (int s = 0; s < tau; ++s) {
     if (stamp) a.phase_ts[s * 4 + 0] = global_ns();
-    const int src = s == 0 ? a.global_slot : w;
-    const int64_t so = static_cast<int64_t>(src) * a.slot_stride;
-    const int64_t dof = static_cast<int64_t>(w) * a.slot_stride;
+    const bool last = s == tau - 1;
 
     // ------------------------------------------------------------ F: partial forward of the group's units
     if (warp == 0 && lane == 0) {
-      fence_proxy_async_global();     // this CTA's generic writes of W0 precede these TMA reads
-      for (int kb = 0; kb < nkf; ++kb) {
-        const int c = kcount + kb, st = c % Cfg::kStagesF;
-        if (c >= Cfg::kStagesF && !mbar_wait(&emptyF[st], ((c / Cfg::kStagesF) + 1) & 1, a.err, kDevTimeoutEmpty)) break;
-        mbar_arrive_expect_tx(&fullF[st], Cfg::kABytes + Cfg::kBBytes);
-        uint8_t* sa = region + st * (Cfg::kABytes + Cfg::kBBytes);
-        tma_load_3d(sa, &mW0, (kb_begin + kb) * kFBK, g0, src, &fullF[st]);
-        tma_load_4d(sa + Cfg::kABytes, &mX, (kb_begin + kb) * kFBK, 0, w, s, &fullF[st]);
-      }
+      if (producer_ok) producer_ok = issue_f(s, pre_f, nkf);   // the rest of this step's X tiles
+      if (producer_ok) producer_ok = issue_d(s, 0, pre_d);     // the first X^T tiles of step D
     } else if (warp == 1 && lane == 0) {
       constexpr uint32_t idesc = idesc_bf16_f32(128, B);
       for (int kb = 0; kb < nkf; ++kb) {
-        const int c = kcount + kb, st = c % Cfg::kStagesF;
+        const int c = s * nkf + kb, st = c % Cfg::kStagesF;
         if (!mbar_wait(&fullF[st], (c / Cfg::kStagesF) & 1, a.err, kDevTimeoutFull)) break;
         tc_fence_after();
-        const uint32_t sa = smem_u32(region + st * (Cfg::kABytes + Cfg::kBBytes));
+        const uint32_t wa = smem_u32(w0s + kb * kW0Blk);
+        const uint32_t xb = smem_u32(fring + st * Cfg::kBBytes);
 #pragma unroll
         for (int j = 0; j < kFBK / 16; ++j)
-          umma_bf16(tmem, smem_desc_k128(sa + j * 32), smem_desc_k128(sa + Cfg::kABytes + j * 32), idesc,
+          umma_bf16(tmem + kTAcc, smem_desc_k128(wa + j * 32), smem_desc_k128(xb + j * 32), idesc,
                     (kb | j) != 0 ? 1u : 0u);
         umma_commit(&emptyF[st]);
       }
       umma_commit(accF);
     }
-    kcount += nkf;
-    // every global input of the F epilogue and of step H, fetched while the tensor core works
-    for (int q = t; q < kFC * (UPC / 8); q += kFT) {
-      const int c = q / (UPC / 8), c8 = (q % (UPC / 8)) * 8;
-      const int64_t e = a.offW1 + static_cast<int64_t>(c) * H + g0 + ku0 + c8;
-      const uint4 v = *reinterpret_cast<const uint4*>(a.shadow + so + e);
-      const __nv_bfloat162* p2 = reinterpret_cast<const __nv_bfloat162*>(&v);
-#pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        const float2 f = __bfloat1622float2(p2[j]);
-        wcs[c * UPC + c8 + 2 * j] = f.x;
-        wcs[c * UPC + c8 + 2 * j + 1] = f.y;
-      }
-      *reinterpret_cast<float4*>(w1m + c * UPC + c8) = *reinterpret_cast<const float4*>(a.master + so + e);
-      *reinterpret_cast<float4*>(w1m + c * UPC + c8 + 4) = *reinterpret_cast<const float4*>(a.master + so + e + 4);
-    }
-    if (t < kFU) b0m[t] = a.master[so + a.offB0 + g0 + t];
-    if (t < kFC) b1m[t] = a.master[so + a.offB1 + t];
     for (int b = t; b < B; b += kFT) labs[b] = a.labels[(static_cast<int64_t>(s) * a.W + w) * B + b];
-    __syncthreads();   // the prefetched b0 is read by the F epilogue below
     if (warp >= 4) {   // epilogue F: thread = unit of the group, columns = samples
       int ok = mbar_wait(accF, s & 1, a.err, kDevTimeoutAccum) ? 1 : 0;
       ok = __all_sync(0xffffffffu, ok);
@@ -306,7 +383,7 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
       if (ok) {
         const int quarter = warp & 3, eg = (warp - 4) >> 2;
         const int u = quarter * 32 + lane;
-        const uint32_t trow = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
+        const uint32_t trow = tmem + (static_cast<uint32_t>(quarter * 32) << 16) + kTAcc;
         for (int c0 = eg * 32; c0 < B; c0 += 64) {
           float v[32];
           tmem_ld_32x32b_x32(trow + c0, v);
@@ -385,7 +462,11 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
         if (r < ncl) acc += part[r];
       dz[q] = acc + b1m[q % kFC];
     }
-    cluster_sync();   // all remote reads of pl (and of the partial z) are done
+    // the softmax rows below read logits summed by other threads; with S = 1
+    // this barrier also separates the remote reads of pl from the next step's
+    // writes (with S = 2 the barrier after the dz0^T exchange does that)
+    if (S == 1) cluster_sync();
+    else __syncthreads();
     for (int b = t; b < B; b += kFT) {
       float z[kFC], e[kFC];
 #pragma unroll
@@ -412,19 +493,22 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
       }
     }
     __syncthreads();
-    if (rank == 0) {
-      if (t < B / kRowsPerLossChunk) {
-        float l = 0.f;
-        for (int r = 0; r < kRowsPerLossChunk; ++r) l += rowloss[t * kRowsPerLossChunk + r];
-        a.loss_part[(static_cast<int64_t>(w) * a.max_tau + s) * (B / kRowsPerLossChunk) + t] = l;
-      }
-      if (t < kFC * 16) {   // head bias
-        const int c = t >> 4, j = t & 15;
-        float g = 0.f;
-        for (int b = j; b < B; b += 16) g += dz[b * kFC + c];
+    if (rank == 0 && t < B / kRowsPerLossChunk) {
+      float l = 0.f;
+      for (int r = 0; r < kRowsPerLossChunk; ++r) l += rowloss[t * kRowsPerLossChunk + r];
+      a.loss_part[(static_cast<int64_t>(w) * a.max_tau + s) * (B / kRowsPerLossChunk) + t] = l;
+    }
+    if (warp >= 8 && warp < 11) {   // head bias, 8 lanes per class: the same arithmetic in every CTA
+      const int idx = t - 256, c = idx >> 3, j = idx & 7;
+      float g = 0.f;
+      if (c < kFC)
+        for (int b = j; b < B; b += 8) g += dz[b * kFC + c];
 #pragma unroll
-        for (int o = 8; o > 0; o >>= 1) g += __shfl_xor_sync(0xffffffffu, g, o, 16);
-        if (j == 0) a.master_w[dof + a.offB1 + c] = fmaf(-a.lr, g, b1m[c]);
+      for (int o = 4; o > 0; o >>= 1) g += __shfl_xor_sync(0xffffffffu, g, o, 8);
+      if (j == 0 && c < kFC) {
+        const float nb = fmaf(-a.lr, g, b1m[c]);
+        b1m[c] = nb;
+        if (last && rank == 0) a.master_w[dof + a.offB1 + c] = nb;
       }
     }
     // masked input gradient dz0[b][u] of this CTA's units: item = (row, 4 units);
@@ -474,7 +558,9 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
       float g = 0.f;
 #pragma unroll
       for (int r = 0; r < Cfg::kGrpRows; ++r) g += gbp[r * UPC + t];
-      a.master_w[dof + a.offB0 + g0 + ku0 + t] = fmaf(-a.lr, g, b0m[ku0 + t]);
+      const float nb = fmaf(-a.lr, g, b0m[ku0 + t]);
+      b0m[ku0 + t] = nb;
+      if (last) a.master_w[dof + a.offB0 + g0 + ku0 + t] = nb;
     }
     // head weight gradient + SGD of this CTA's columns: item = (class, 4 units)
     for (int q = t; q < kFC * (UPC / 4); q += kFT) {
@@ -488,15 +574,17 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
         dw.z = fmaf(g, hv.z, dw.z);
         dw.w = fmaf(g, hv.w, dw.w);
       }
-      const int64_t e = a.offW1 + static_cast<int64_t>(c) * H + g0 + ku0 + u4;
       const float4 o = *reinterpret_cast<const float4*>(w1m + c * UPC + u4);
       float4 nw;
       nw.x = fmaf(-a.lr, dw.x, o.x);
       nw.y = fmaf(-a.lr, dw.y, o.y);
       nw.z = fmaf(-a.lr, dw.z, o.z);
       nw.w = fmaf(-a.lr, dw.w, o.w);
-      *reinterpret_cast<float4*>(a.master_w + dof + e) = nw;
-      *reinterpret_cast<uint2*>(a.shadow + dof + e) = make_uint2(pack_bf16x2(nw.x, nw.y), pack_bf16x2(nw.z, nw.w));
+      *reinterpret_cast<float4*>(w1m + c * UPC + u4) = nw;
+      *reinterpret_cast<float4*>(wcs + c * UPC + u4) =
+          make_float4(bf16_round(nw.x), bf16_round(nw.y), bf16_round(nw.z), bf16_round(nw.w));
+      if (last)
+        *reinterpret_cast<float4*>(a.master_w + dof + a.offW1 + static_cast<int64_t>(c) * H + g0 + ku0 + u4) = nw;
     }
     if (S > 1) {
       cluster_sync();             // the partner's dz0^T rows have landed
@@ -506,81 +594,62 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
 
     // ------------------------------------------------------------ D: weight gradient + SGD of own W0 block
     if (warp == 0 && lane == 0) {
-      for (int tt = 0; tt < nD; ++tt) {
-        const int c = dcount + tt, buf = c % Cfg::kNBD, use = c / Cfg::kNBD;
-        // the buffer's previous tile must be fully consumed (MMA and epilogue)
-        if (use >= 1 && !mbar_wait(&tfreeD[buf], (use - 1) & 1, a.err, kDevTimeoutEmpty)) break;
-        mbar_arrive_expect_tx(&fullD[buf], Cfg::kBufD);
-        uint8_t* dst = region + buf * Cfg::kBufD;
-        const int n0 = col_begin + tt * Cfg::kND;
-        tma_load_4d(dst, &mXT, 0, n0, w, s, &fullD[buf]);
-        tma_load_3d(dst + Cfg::kXtBytes, &mWm, n0, g0, src, &fullD[buf]);   // old W0 block
-      }
+      if (producer_ok) producer_ok = issue_d(s, pre_d, nD);
+      // the first X tiles of the next step's forward, while this step's epilogue runs
+      if (producer_ok && s + 1 < tau) producer_ok = issue_f(s + 1, 0, pre_f);
     } else if (warp == 1 && lane == 0) {
-      constexpr uint32_t idesc = idesc_bf16_f32(128, Cfg::kND);
+      constexpr uint32_t idesc = idesc_bf16_f32(128, kND);
       for (int tt = 0; tt < nD; ++tt) {
-        const int c = dcount + tt, buf = c % Cfg::kNBD, use = c / Cfg::kNBD;
-        if (!mbar_wait(&fullD[buf], use & 1, a.err, kDevTimeoutFull)) break;
+        const int c = s * nD + tt, buf = c % kNBD, use = c / kNBD, xb = c % kNXD;
+        if (!mbar_wait(&fullD[xb], (c / kNXD) & 1, a.err, kDevTimeoutFull)) break;
         if (use >= 1 && !mbar_wait(&tfreeD[buf], (use - 1) & 1, a.err, kDevTimeoutAccum)) break;
         tc_fence_after();
-        const uint32_t xa = smem_u32(region + buf * Cfg::kBufD);
+        const uint32_t xa = smem_u32(dring + xb * Cfg::kXtBytes);
         const uint32_t da = smem_u32(dzT);
-        const uint32_t dcol = tmem + static_cast<uint32_t>(buf * Cfg::kND);
+        const uint32_t dcol = tmem + static_cast<uint32_t>(kTAcc + buf * kND);
 #pragma unroll
         for (int j = 0; j < kFBK / 16; ++j)
           umma_bf16(dcol, smem_desc_k128(da + j * 32), smem_desc_k128(xa + j * 32), idesc, j != 0 ? 1u : 0u);
         umma_commit(&accD[buf]);
+        umma_commit(&xfreeD[xb]);
       }
     } else if (warp >= 4) {
-      // the two warpgroups take alternate tiles; a warp covers 32 rows x 32 columns
+      // the two warpgroups take alternate tiles (a fixed split: a master tile
+      // always belongs to the same warpgroup); a warp covers 32 rows
       const int quarter = warp & 3, eg = (warp - 4) >> 2;
-      const int mb = quarter * 32;                       // rows of this warp within the group
-      float* T = epi + (warp - 4) * 32 * 36;   // row stride 36: 16-byte accesses of 8 lanes hit distinct banks
+      const int r = quarter * 32 + lane;
+      const uint32_t trow = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
+      float* dst_row = a.master_w + dof + a.offW0 + static_cast<int64_t>(g0 + r) * D + col_begin;
       for (int tt = eg; tt < nD; tt += 2) {
-        const int c = dcount + tt, buf = c % Cfg::kNBD, use = c / Cfg::kNBD;
+        const int c = s * nD + tt, buf = c % kNBD, use = c / kNBD;
         int ok = mbar_wait(&accD[buf], use & 1, a.err, kDevTimeoutAccum) ? 1 : 0;
         ok = __all_sync(0xffffffffu, ok);
         tc_fence_after();
         if (ok) {
-          const float* Ms = reinterpret_cast<const float*>(region + buf * Cfg::kBufD + Cfg::kXtBytes);
-          const int n_base = col_begin + tt * Cfg::kND;  // first input column of the tile
-          float v[32];
-          tmem_ld_32x32b_x32(tmem + (static_cast<uint32_t>(quarter * 32) << 16) + buf * Cfg::kND, v);
+          const int c0 = tt * kND;
+          float g[32], m[32];
+          tmem_ld_32x32b_x32_pair(trow + kTAcc + buf * kND, g, trow + c0, m);
 #pragma unroll
-          for (int q = 0; q < 8; ++q)
-            *reinterpret_cast<float4*>(T + lane * 36 + 4 * q) = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
-          __syncwarp();
-          // lane -> (row 4 i + lane / 8, columns 4 (lane % 8) .. + 3): 4 rows per instruction
-          const int cq = (lane & 7) * 4;
-          const bool nok = n_base + cq < col_end;   // column ends are multiples of 8
+          for (int j = 0; j < 32; ++j) m[j] = fmaf(-a.lr, g[j], m[j]);
+          tmem_st_32x32b_x32(trow + c0, m);
+          put_w0_row32(w0s, r, c0, m);
+          if (last) {
 #pragma unroll
-          for (int i = 0; i < 8; ++i) {
-            const int r = 4 * i + (lane >> 3);
-            const float4 g = *reinterpret_cast<const float4*>(T + r * 36 + cq);
-            const float4 o = *reinterpret_cast<const float4*>(Ms + (mb + r) * Cfg::kND + cq);
-            float4 nw;
-            nw.x = fmaf(-a.lr, g.x, o.x);
-            nw.y = fmaf(-a.lr, g.y, o.y);
-            nw.z = fmaf(-a.lr, g.z, o.z);
-            nw.w = fmaf(-a.lr, g.w, o.w);
-            if (nok) {
-              const int64_t e = dof + a.offW0 + static_cast<int64_t>(g0 + mb + r) * D + n_base + cq;
-              *reinterpret_cast<float4*>(a.master_w + e) = nw;
-              *reinterpret_cast<uint2*>(a.shadow + e) = make_uint2(pack_bf16x2(nw.x, nw.y), pack_bf16x2(nw.z, nw.w));
-            }
+            for (int q = 0; q < 8; ++q)
+              if (c0 + 4 * q < ncols)
+                *reinterpret_cast<float4*>(dst_row + c0 + 4 * q) =
+                    make_float4(m[4 * q], m[4 * q + 1], m[4 * q + 2], m[4 * q + 3]);
           }
-          __syncwarp();
+          tmem_wait_st();
         }
         tc_fence_before();
         mbar_arrive(&tfreeD[buf]);
       }
     }
-    dcount += nD;
-    fence_proxy_async_global();   // W0 written here is read by TMA next step
+    fence_proxy_async_smem();   // the resident W0 written here is read by the tensor core next step
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    cluster_sync();               // head bias (rank 0) visible; exchange buffers reusable
     if (stamp) a.phase_ts[s * 4 + 3] = global_ns();
   }
   // round bookkeeping of this worker: mean loss over its steps (sum in step
@@ -602,8 +671,7 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
 }
 
 template <int B, int S>
-cudaError_t launch_bs(const CUtensorMap& mW0, const CUtensorMap& mX, const CUtensorMap& mXT, const CUtensorMap& mWm,
-                      const FusedArgs& a, cudaStream_t s) {
+cudaError_t launch_bs(const CUtensorMap& mX, const CUtensorMap& mXT, const FusedArgs& a, cudaStream_t s) {
   using Cfg = FCfg<B, S>;
   cudaError_t e = cudaFuncSetAttribute(fused_mlp2_round_kernel<B, S>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        Cfg::kSmem);
@@ -620,31 +688,40 @@ cudaError_t launch_bs(const CUtensorMap& mW0, const CUtensorMap& mX, const CUten
   attr[0].val.clusterDim.z = 1;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
-  return cudaLaunchKernelEx(&cfg, fused_mlp2_round_kernel<B, S>, mW0, mX, mXT, mWm, a);
+  return cudaLaunchKernelEx(&cfg, fused_mlp2_round_kernel<B, S>, mX, mXT, a);
 }
 
 // two CTAs per unit group when the cluster stays within 8 CTAs and the input
 // has at least two K-blocks
 int split_for(int D, int H) { return (2 * (H / kFU) <= kFMaxCluster && (D + kFBK - 1) / kFBK >= 2) ? 2 : 1; }
 
+// input columns of the widest CTA of a group (the last one)
+int widest_cols(int D, int S) {
+  const int nkF = (D + kFBK - 1) / kFBK;
+  return S > 1 ? D - (nkF / 2) * kFBK : D;
+}
+
 }  // namespace
 
 bool fused_round_supported(int L, int D, int H, int C, int B) {
   if (L != 2 || C != kFC || H % kFU != 0 || H / kFU > kFMaxCluster || D % 8 != 0) return false;
   if (B != 32 && B != 64) return false;
-  int smem = 0;
   const int S = split_for(D, H);
+  // the CTA's master block must fit the TMEM columns below the accumulators
+  if ((widest_cols(D, S) + kND - 1) / kND * kND > kTAcc) return false;
+  int smem = 0;
   if (B == 32) smem = S == 2 ? FCfg<32, 2>::kSmem : FCfg<32, 1>::kSmem;
   else smem = S == 2 ? FCfg<64, 2>::kSmem : FCfg<64, 1>::kSmem;
   return smem <= 227 * 1024;
 }
 
-int fused_round_xt_rows(int) { return 32; }
+int fused_round_xt_rows(int) { return kND; }
 
-cudaError_t launch_fused_round(const CUtensorMap& mW0, const CUtensorMap& mX, const CUtensorMap& mXT,
-                               const CUtensorMap& mWm, const FusedRoundArgs& r, cudaStream_t s) {
+cudaError_t launch_fused_round(const CUtensorMap& mX, const CUtensorMap& mXT, const FusedRoundArgs& r,
+                               cudaStream_t s) {
   FusedArgs a;
   a.tau = r.tau;
+  a.order = r.order;
   a.W = r.W;
   a.D = r.D;
   a.H = r.H;
@@ -652,7 +729,6 @@ cudaError_t launch_fused_round(const CUtensorMap& mW0, const CUtensorMap& mX, co
   a.lr = r.lr;
   a.master = r.master;
   a.master_w = r.master_w;
-  a.shadow = r.shadow;
   a.slot_stride = r.slot_stride;
   a.offW0 = r.offW0;
   a.offB0 = r.offB0;
@@ -667,8 +743,8 @@ cudaError_t launch_fused_round(const CUtensorMap& mW0, const CUtensorMap& mX, co
   a.cursor = r.cursor;
   a.shard_n = r.shard_n;
   const int S = split_for(r.D, r.H);
-  if (r.B == 32) return S == 2 ? launch_bs<32, 2>(mW0, mX, mXT, mWm, a, s) : launch_bs<32, 1>(mW0, mX, mXT, mWm, a, s);
-  if (r.B == 64) return S == 2 ? launch_bs<64, 2>(mW0, mX, mXT, mWm, a, s) : launch_bs<64, 1>(mW0, mX, mXT, mWm, a, s);
+  if (r.B == 32) return S == 2 ? launch_bs<32, 2>(mX, mXT, a, s) : launch_bs<32, 1>(mX, mXT, a, s);
+  if (r.B == 64) return S == 2 ? launch_bs<64, 2>(mX, mXT, a, s) : launch_bs<64, 1>(mX, mXT, a, s);
   return cudaErrorInvalidValue;
 }
 

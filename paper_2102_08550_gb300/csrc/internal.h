@@ -142,12 +142,12 @@ cudaError_t launch_head_bwd(const HeadArgs& a, int n_active, cudaStream_t s);
 // ---------------------------------------------------------------- fused round (2-layer MLP)
 struct FusedRoundArgs {
   const int32_t* tau;
+  const int32_t* order;           // [W] workers by decreasing tau (cluster launch order)
   int W, D, H, B;
   int global_slot;
   float lr;
   const float* master;
   float* master_w;
-  __nv_bfloat16* shadow;
   int64_t slot_stride;
   int64_t offW0, offB0, offW1, offB1;
   const int32_t* labels;
@@ -159,15 +159,15 @@ struct FusedRoundArgs {
   int64_t* cursor;                // [W] advanced by tau * B modulo n at the end
   const int64_t* shard_n;         // [W]
 };
-// whole-round kernel for input -> H ReLU -> 10 classes (one cluster per worker)
+// whole-round kernel for input -> H ReLU -> 10 classes (one cluster per
+// worker, the worker's model resident on chip for the round)
 bool fused_round_supported(int L, int D, int H, int C, int B);
 int fused_round_xt_rows(int B);   // rows of the X^T box the kernel loads
-// mW0: shadow W0 of every slot {D, H, slots} box {64, 128}; mX: staged inputs
-// {D, B, W, steps} box {64, B}; mXT: staged transposed inputs {B, D, W, steps}
-// box {64, fused_round_xt_rows(B)}; mWm: fp32 master W0 of every slot
-// {D, H, slots} box {fused_round_xt_rows(B), 128}, no swizzle
-cudaError_t launch_fused_round(const CUtensorMap& mW0, const CUtensorMap& mX, const CUtensorMap& mXT,
-                               const CUtensorMap& mWm, const FusedRoundArgs& a, cudaStream_t s);
+// mX: staged inputs {D, B, W, steps} box {64, B}; mXT: staged transposed
+// inputs {B, D, W, steps} box {64, fused_round_xt_rows(B)}; both bf16,
+// 128-byte swizzle
+cudaError_t launch_fused_round(const CUtensorMap& mX, const CUtensorMap& mXT, const FusedRoundArgs& a,
+                               cudaStream_t s);
 
 // loss[w] = sum_{s < tau[w]} sum_c part[(w*max_tau + s)*nc + c] / (B * tau[w])
 cudaError_t launch_loss_finalize(const float* part, const int32_t* tau, int W, int max_tau,
