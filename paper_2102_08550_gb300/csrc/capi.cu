@@ -594,7 +594,6 @@ cudaError_t enqueue_round_mlp(oscars_ctx* c, cudaStream_t st) {
     f.offW1 = c->layers[1].offW;
     f.offB1 = c->layers[1].offB;
     f.labels = c->labels_all;
-    f.loss_part = c->loss_part;
     f.max_tau = c->max_tau;
     f.err = c->err;
     f.phase_ts = (c->flags & 16) ? c->phase_ts : nullptr;

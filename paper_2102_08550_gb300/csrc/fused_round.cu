@@ -15,9 +15,10 @@
 // Its head-weight columns, its b0 entries and a private copy of the head
 // bias (updated identically by every CTA) live in shared memory.  The model
 // is read from the global slot once, before the first step, and the worker's
-// replica is written once, during the last step.  Per step only the
-// mini-batch (staged bf16 X and X^T tiles, by TMA) and the labels come from
-// global memory.
+// replica is written once, after the last step (the W0 block through a
+// per-warp shared-memory transpose, so that every store instruction writes
+// whole 128-byte lines).  Per step only the mini-batch (staged bf16 X and X^T
+// tiles, by TMA) and the labels come from global memory.
 //
 // Every step of the worker runs inside the cluster:
 //
@@ -187,7 +188,6 @@ struct FusedArgs {
   int64_t slot_stride;
   int64_t offW0, offB0, offW1, offB1;
   const int32_t* labels;    // [max_tau][W][B]
-  float* loss_part;         // [(w * max_tau + s) * (B / 16) + chunk]
   int max_tau;
   int* err;
   unsigned long long* phase_ts;   // [max_tau][4] phase start stamps of worker 0 (or null)
@@ -310,6 +310,7 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
   };
   bool producer_ok = true;
   if (warp == 0 && lane == 0) producer_ok = issue_f(0, 0, pre_f);
+  double loss_sum = 0.0;   // rank 0, thread 0: sum of the 16-row loss chunks, in step and chunk order
 
   // the global model, once: fp32 master block into TMEM and its bf16 copy
   // into the resident operand (epilogue warps); head columns and biases
@@ -318,20 +319,30 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
     const int r = quarter * 32 + lane;
     const uint32_t trow = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
     const float* src = a.master + gso + a.offW0 + static_cast<int64_t>(g0 + r) * D + col_begin;
-    for (int tt = eg; tt < nD; tt += 2) {
-      const int c0 = tt * kND;
-      float v[32];
+    // two of the warpgroup's tiles per pass: both tiles' loads are in flight together
+    for (int tt = eg; tt < nD; tt += 4) {
+      float v[2][32];
 #pragma unroll
-      for (int q = 0; q < 8; ++q) {
-        const float4 x = c0 + 4 * q < ncols ? *reinterpret_cast<const float4*>(src + c0 + 4 * q)
-                                            : make_float4(0.f, 0.f, 0.f, 0.f);
-        v[4 * q] = x.x;
-        v[4 * q + 1] = x.y;
-        v[4 * q + 2] = x.z;
-        v[4 * q + 3] = x.w;
+      for (int h = 0; h < 2; ++h) {
+        const int c0 = (tt + 2 * h) * kND;
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+          const float4 x = c0 + 4 * q < ncols ? *reinterpret_cast<const float4*>(src + c0 + 4 * q)
+                                              : make_float4(0.f, 0.f, 0.f, 0.f);
+          v[h][4 * q] = x.x;
+          v[h][4 * q + 1] = x.y;
+          v[h][4 * q + 2] = x.z;
+          v[h][4 * q + 3] = x.w;
+        }
       }
-      tmem_st_32x32b_x32(trow + c0, v);
-      put_w0_row32(w0s, r, c0, v);
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        const int c0 = (tt + 2 * h) * kND;
+        if (tt + 2 * h < nD) {
+          tmem_st_32x32b_x32(trow + c0, v[h]);
+          put_w0_row32(w0s, r, c0, v[h]);
+        }
+      }
     }
     tmem_wait_st();
   } else {
@@ -493,10 +504,12 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
       }
     }
     __syncthreads();
-    if (rank == 0 && t < B / kRowsPerLossChunk) {
-      float l = 0.f;
-      for (int r = 0; r < kRowsPerLossChunk; ++r) l += rowloss[t * kRowsPerLossChunk + r];
-      a.loss_part[(static_cast<int64_t>(w) * a.max_tau + s) * (B / kRowsPerLossChunk) + t] = l;
+    if (rank == 0 && t == 0) {
+      for (int c = 0; c < B / kRowsPerLossChunk; ++c) {
+        float l = 0.f;
+        for (int r = 0; r < kRowsPerLossChunk; ++r) l += rowloss[c * kRowsPerLossChunk + r];
+        loss_sum += static_cast<double>(l);
+      }
     }
     if (warp >= 8 && warp < 11) {   // head bias, 8 lanes per class: the same arithmetic in every CTA
       const int idx = t - 256, c = idx >> 3, j = idx & 7;
@@ -619,7 +632,6 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
       const int quarter = warp & 3, eg = (warp - 4) >> 2;
       const int r = quarter * 32 + lane;
       const uint32_t trow = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
-      float* dst_row = a.master_w + dof + a.offW0 + static_cast<int64_t>(g0 + r) * D + col_begin;
       for (int tt = eg; tt < nD; tt += 2) {
         const int c = s * nD + tt, buf = c % kNBD, use = c / kNBD;
         int ok = mbar_wait(&accD[buf], use & 1, a.err, kDevTimeoutAccum) ? 1 : 0;
@@ -629,22 +641,18 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
           const int c0 = tt * kND;
           float g[32], m[32];
           tmem_ld_32x32b_x32_pair(trow + kTAcc + buf * kND, g, trow + c0, m);
+          tc_fence_before();
+          mbar_arrive(&tfreeD[buf]);   // the gradient buffer has been read: the next MMA may reuse it
 #pragma unroll
           for (int j = 0; j < 32; ++j) m[j] = fmaf(-a.lr, g[j], m[j]);
           tmem_st_32x32b_x32(trow + c0, m);
           put_w0_row32(w0s, r, c0, m);
-          if (last) {
-#pragma unroll
-            for (int q = 0; q < 8; ++q)
-              if (c0 + 4 * q < ncols)
-                *reinterpret_cast<float4*>(dst_row + c0 + 4 * q) =
-                    make_float4(m[4 * q], m[4 * q + 1], m[4 * q + 2], m[4 * q + 3]);
-          }
-          tmem_wait_st();
+        } else {
+          tc_fence_before();
+          mbar_arrive(&tfreeD[buf]);
         }
-        tc_fence_before();
-        mbar_arrive(&tfreeD[buf]);
       }
+      tmem_wait_st();   // the master columns stored above are read again next step
     }
     fence_proxy_async_smem();   // the resident W0 written here is read by the tensor core next step
     tc_fence_before();
@@ -652,14 +660,37 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
     tc_fence_after();
     if (stamp) a.phase_ts[s * 4 + 3] = global_ns();
   }
-  // round bookkeeping of this worker: mean loss over its steps (sum in step
-  // order, fp64) and the data cursor
+  // the worker's W0 block into its replica slot: each warp moves 32 rows x
+  // 32 columns at a time from TMEM through a padded shared tile (the TMA
+  // rings are idle now), 4 full 128-byte rows per store instruction
+  if (warp >= 4) {
+    const int quarter = warp & 3, eg = (warp - 4) >> 2;
+    const uint32_t trow = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
+    float* T = reinterpret_cast<float*>(sm + Cfg::oRegion) + (warp - 4) * 32 * 36;
+    float* dst = a.master_w + dof + a.offW0 + static_cast<int64_t>(g0 + quarter * 32) * D + col_begin;
+    const int cq = (lane & 7) * 4;
+    for (int tt = eg; tt < nD; tt += 2) {
+      const int c0 = tt * kND;
+      float m[32];
+      tmem_ld_32x32b_x32(trow + c0, m);
+#pragma unroll
+      for (int q = 0; q < 8; ++q)
+        *reinterpret_cast<float4*>(T + lane * 36 + 4 * q) = make_float4(m[4 * q], m[4 * q + 1], m[4 * q + 2], m[4 * q + 3]);
+      __syncwarp();
+      if (c0 + cq < ncols) {
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          const int rr = 4 * i + (lane >> 3);
+          *reinterpret_cast<float4*>(dst + static_cast<int64_t>(rr) * D + c0 + cq) =
+              *reinterpret_cast<const float4*>(T + rr * 36 + cq);
+        }
+      }
+      __syncwarp();
+    }
+  }
+  // round bookkeeping of this worker: mean loss over its steps and the data cursor
   if (rank == 0 && t == 0) {
-    constexpr int nc = B / kRowsPerLossChunk;
-    double sum = 0.0;
-    for (int st = 0; st < tau; ++st)
-      for (int c = 0; c < nc; ++c) sum += a.loss_part[(static_cast<int64_t>(w) * a.max_tau + st) * nc + c];
-    a.loss_out[w] = static_cast<float>(sum / (static_cast<double>(B) * tau));
+    a.loss_out[w] = static_cast<float>(loss_sum / (static_cast<double>(B) * tau));
     a.cursor[w] = (a.cursor[w] + static_cast<int64_t>(tau) * B) % a.shard_n[w];
   }
   tc_fence_before();
@@ -735,7 +766,6 @@ cudaError_t launch_fused_round(const CUtensorMap& mX, const CUtensorMap& mXT, co
   a.offW1 = r.offW1;
   a.offB1 = r.offB1;
   a.labels = r.labels;
-  a.loss_part = r.loss_part;
   a.max_tau = r.max_tau;
   a.err = r.err;
   a.phase_ts = r.phase_ts;

@@ -151,7 +151,6 @@ struct FusedRoundArgs {
   int64_t slot_stride;
   int64_t offW0, offB0, offW1, offB1;
   const int32_t* labels;
-  float* loss_part;
   int max_tau;
   int* err;
   unsigned long long* phase_ts;   // [max_tau][4] phase stamps of worker 0, or null
