@@ -25,14 +25,16 @@
 //  F  forward: each CTA computes the partial pre-activation of the group's
 //     128 units over its own input columns on tcgen05 (resident W0; the
 //     first X tiles are prefetched during the previous step).  With S = 2
-//     the pair exchanges partials through distributed shared memory and each
-//     CTA keeps 128/S of the units: z = (part_0 + part_1) + b0, h = relu(z),
-//     bf16;
+//     each CTA keeps 128/S of the units: the epilogue stores each partial
+//     into the shared memory of the CTA that keeps its unit (its own or,
+//     through distributed shared memory, its partner's), and after one
+//     barrier z = (part_0 + part_1) + b0, h = relu(z), bf16;
 //  H  last layer for the CTA's units: partial logits, summed over the whole
 //     cluster in rank order through distributed shared memory, softmax
 //     cross-entropy; the masked input gradient dz0[b][u] of its units is
-//     written (as bf16) into the 128-byte-swizzled K-major dz0^T tile of
-//     every CTA of its group (the A operand of step D); bias gradient and SGD
+//     written (as bf16, 16-byte chunks of 8 samples) into the
+//     128-byte-swizzled K-major dz0^T tile of every CTA of its group (the A
+//     operand of step D); bias gradient and SGD
 //     of b0 (own units), of the head weights (own columns) and of the head
 //     bias;
 //  D  weight gradient of the group's 128 rows over the CTA's own input
@@ -95,22 +97,17 @@ __device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
 }
 
-__device__ __forceinline__ float4 ld_dsmem_f32x4(const float* local, uint32_t rank) {
+__device__ __forceinline__ void st_dsmem_u32x4(void* local, uint32_t rank, uint4 v) {
   uint32_t remote;
   asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(smem_u32(local)), "r"(rank));
-  float4 v;
-  asm volatile("ld.shared::cluster.v4.f32 {%0, %1, %2, %3}, [%4];"
-               : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
-               : "r"(remote)
+  asm volatile("st.shared::cluster.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(remote), "r"(v.x), "r"(v.y), "r"(v.z),
+               "r"(v.w)
                : "memory");
-  return v;
 }
 
-__device__ __forceinline__ void st_dsmem_b16(void* local, uint32_t rank, __nv_bfloat16 v) {
-  uint32_t remote;
-  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(smem_u32(local)), "r"(rank));
-  const unsigned short bits = *reinterpret_cast<const unsigned short*>(&v);
-  asm volatile("st.shared::cluster.b16 [%0], %1;" ::"r"(remote), "h"(bits) : "memory");
+__device__ __forceinline__ void st_dsmem_f32x4(float* local, uint32_t rank, float4 v) {
+  st_dsmem_u32x4(local, rank, make_uint4(__float_as_uint(v.x), __float_as_uint(v.y), __float_as_uint(v.z),
+                                         __float_as_uint(v.w)));
 }
 
 __device__ __forceinline__ unsigned long long global_ns() {
@@ -151,12 +148,14 @@ struct FCfg {
   static constexpr int kDRing = kNXD * kXtBytes;
   static constexpr int kFRing = kStagesF * kBBytes;
   static constexpr int kZs = B + 4;                         // row stride of the partial z exchange (floats)
-  static constexpr int kZBytes = S > 1 ? kFU * kZs * 4 : 0;
+  static constexpr int kZBytes = S > 1 ? kUPC * kZs * 4 : 0;  // own partials (the incoming ones alias hs)
   static constexpr int kRegion = kDRing + (kFRing > kZBytes ? kFRing : kZBytes);   // D ring | F ring or z
   static constexpr int kDzT = kFU * 128;                    // dz0^T tile: 128 rows x 64 k (batch padded)
   static constexpr int kTpr = 256 / B;                      // threads per row, partial logits
   static constexpr int kHsd = kUPC + 4 * kTpr;              // padded row stride of the float h tile
-  static constexpr int kGrpRows = 256 / (kUPC / 4);         // rows per pass of the input-gradient items
+  static constexpr int kChunks = B / 8;                     // 8-sample chunks of a dz0^T row
+  static constexpr int kW1Items = kFC * (kUPC / 4);         // (class, 4 units) items of the head update
+  static_assert(2 * kW1Items * 16 <= kStagesF * B * kFBK * 2, "head-update partials must fit the F ring");
   // shared memory carve-up (bytes, from a 1024-aligned base)
   static constexpr int oRegion = 0;
   static constexpr int oW0 = (oRegion + kRegion + 1023) / 1024 * 1024;
@@ -167,14 +166,15 @@ struct FCfg {
   static constexpr int oPl = oW1m + kFC * kUPC * 4;          // [B][C]
   static constexpr int oDz = oPl + B * kFC * 4;              // [B][C]
   static constexpr int oDzb = oDz + B * kFC * 4;             // [B][C]
-  static constexpr int oGbp = oDzb + B * kFC * 4;            // [kGrpRows][kUPC]
-  static constexpr int oRowLoss = oGbp + kGrpRows * kUPC * 4;   // [B]
+  static constexpr int oGbp = oDzb + B * kFC * 4;            // [kChunks][kUPC]
+  static constexpr int oRowLoss = oGbp + kChunks * kUPC * 4;   // [B]
   static constexpr int oB0 = oRowLoss + B * 4;               // [kFU] b0 of the group's units
   static constexpr int oB1 = oB0 + kFU * 4;                  // [16] head bias (private copy)
   static constexpr int oLab = oB1 + 16 * 4;                  // [B] int
   static constexpr int oBar = (oLab + B * 4 + 15) / 16 * 16;
   static constexpr int kBarBytes = 256;
   static constexpr int kSmem = oBar + kBarBytes + 1024;      // + alignment slack
+  static_assert(S == 1 || kUPC * kZs <= B * kHsd, "the incoming partials must fit the h tile they alias");
 };
 
 struct FusedArgs {
@@ -206,10 +206,16 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
   uint8_t* sm = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(fs_raw) + 1023) & ~uintptr_t(1023));
   uint8_t* dring = sm + Cfg::oRegion;                // X^T tiles of step D
   uint8_t* fring = dring + Cfg::kDRing;              // X tiles of step F
-  float* zx = reinterpret_cast<float*>(fring);       // [128][kZs] partial z (S = 2), after the F MMAs
+  float* zx = reinterpret_cast<float*>(fring);       // [kUPC][kZs] own partials (S = 2), after the F MMAs
   uint8_t* w0s = sm + Cfg::oW0;                      // resident bf16 W0 block
   uint8_t* dzT = sm + Cfg::oDzT;
   float* hs = reinterpret_cast<float*>(sm + Cfg::oHs);
+  // [kUPC][kZs] partials that the partner computed for this CTA's units
+  // (S = 2).  They alias hs: the partner stores them in its forward epilogue,
+  // after this CTA has passed the last barrier of its previous step (hs is
+  // read only before it), and they are read into registers before hs is
+  // rewritten.
+  float* zin = hs;
   float* wcs = reinterpret_cast<float*>(sm + Cfg::oWc);
   float* w1m = reinterpret_cast<float*>(sm + Cfg::oW1m);
   float* pl = reinterpret_cast<float*>(sm + Cfg::oPl);
@@ -403,10 +409,16 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
 #pragma unroll
             for (int j = 0; j < 32; ++j) hs[(c0 + j) * Cfg::kHsd + u] = bf16_round(fmaxf(v[j] + bias, 0.f));
           } else {
+            // the partial goes to the CTA that keeps unit u: this one
+            // (own rows) or the partner (its incoming rows)
+            const int owner = u / UPC;
+            float* row = (owner == half ? zx : zin) + (u - owner * UPC) * Cfg::kZs + c0;
 #pragma unroll
-            for (int q = 0; q < 8; ++q)
-              *reinterpret_cast<float4*>(zx + u * Cfg::kZs + c0 + 4 * q) =
-                  make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+            for (int q = 0; q < 8; ++q) {
+              const float4 p4 = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+              if (owner == half) *reinterpret_cast<float4*>(row + 4 * q) = p4;
+              else st_dsmem_f32x4(row + 4 * q, grp * S + owner, p4);
+            }
           }
         }
       }
@@ -414,21 +426,39 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
     tc_fence_before();
     __syncthreads();
     if (S > 1) {
-      // pair exchange: z of this CTA's units = part(half 0) + part(half 1) + b0
+      // both partials of this CTA's units are local now:
+      // z = part(half 0) + part(half 1) + b0
       cluster_sync();
-      for (int q = t; q < UPC * (B / 4); q += kFT) {
+      constexpr int kZItems = UPC * (B / 4), kZPer = (kZItems + kFT - 1) / kFT;
+      float4 zr[kZPer];
+#pragma unroll
+      for (int k = 0; k < kZPer; ++k) {
+        const int q = t + k * kFT;
+        if (q < kZItems) {
+          const int ul = q / (B / 4), b4 = (q % (B / 4)) * 4;
+          const float4 own = *reinterpret_cast<const float4*>(zx + ul * Cfg::kZs + b4);
+          const float4 inc = *reinterpret_cast<const float4*>(zin + ul * Cfg::kZs + b4);
+          const float4 p0 = half == 0 ? own : inc, p1 = half == 0 ? inc : own;
+          float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
+          z.x += p0.x;
+          z.y += p0.y;
+          z.z += p0.z;
+          z.w += p0.w;
+          z.x += p1.x;
+          z.y += p1.y;
+          z.z += p1.z;
+          z.w += p1.w;
+          zr[k] = z;
+        }
+      }
+      __syncthreads();   // the incoming partials (aliasing hs) have been read
+#pragma unroll
+      for (int k = 0; k < kZPer; ++k) {
+        const int q = t + k * kFT;
+        if (q >= kZItems) break;
         const int ul = q / (B / 4), b4 = (q % (B / 4)) * 4;
         const int ug = ku0 + ul;                   // unit within the group
-        float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll
-        for (int j = 0; j < S; ++j) {
-          const float* p = zx + ug * Cfg::kZs + b4;
-          const float4 v = j == half ? *reinterpret_cast<const float4*>(p) : ld_dsmem_f32x4(p, grp * S + j);
-          z.x += v.x;
-          z.y += v.y;
-          z.z += v.z;
-          z.w += v.w;
-        }
+        const float4 z = zr[k];
         const float bias = b0m[ug];
         hs[(b4 + 0) * Cfg::kHsd + ul] = bf16_round(fmaxf(z.x + bias, 0.f));
         hs[(b4 + 1) * Cfg::kHsd + ul] = bf16_round(fmaxf(z.y + bias, 0.f));
@@ -524,62 +554,46 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
         if (last && rank == 0) a.master_w[dof + a.offB1 + c] = nb;
       }
     }
-    // masked input gradient dz0[b][u] of this CTA's units: item = (row, 4 units);
-    // written into the dz0^T tile of every CTA of the group
-    if (t < 256) {
-      constexpr int kLanesPerRow = UPC / 4;
-      const int u4 = (t % kLanesPerRow) * 4, rg = t / kLanesPerRow;
-      float4 wc[kFC];
+    // masked input gradient dz0[b][u] of this CTA's units: item = (unit, 8
+    // consecutive samples), one 16-byte chunk of the unit's K-major dz0^T
+    // row, stored here and into the other CTAs of the group
+    for (int it = t; it < UPC * Cfg::kChunks; it += kFT) {
+      const int u = it % UPC, j = it / UPC;
+      float wc[kFC];
 #pragma unroll
-      for (int c = 0; c < kFC; ++c) wc[c] = *reinterpret_cast<const float4*>(wcs + c * UPC + u4);
-      float4 gs = make_float4(0.f, 0.f, 0.f, 0.f);
-      for (int b = rg; b < B; b += Cfg::kGrpRows) {
-        const float4 hv = *reinterpret_cast<const float4*>(hs + b * Cfg::kHsd + u4);
-        float4 dh = make_float4(0.f, 0.f, 0.f, 0.f);
+      for (int c = 0; c < kFC; ++c) wc[c] = wcs[c * UPC + u];
+      float dv[8];
+      float gsum = 0.f;
 #pragma unroll
-        for (int c = 0; c < kFC; ++c) {
-          const float g = dzb[b * kFC + c];
-          dh.x = fmaf(g, wc[c].x, dh.x);
-          dh.y = fmaf(g, wc[c].y, dh.y);
-          dh.z = fmaf(g, wc[c].z, dh.z);
-          dh.w = fmaf(g, wc[c].w, dh.w);
-        }
-        dh.x = hv.x > 0.f ? dh.x : 0.f;
-        dh.y = hv.y > 0.f ? dh.y : 0.f;
-        dh.z = hv.z > 0.f ? dh.z : 0.f;
-        dh.w = hv.w > 0.f ? dh.w : 0.f;
-        gs.x += dh.x;
-        gs.y += dh.y;
-        gs.z += dh.z;
-        gs.w += dh.w;
-        const float dv[4] = {dh.x, dh.y, dh.z, dh.w};
+      for (int i = 0; i < 8; ++i) {
+        const int b = 8 * j + i;
+        float dh = 0.f;
 #pragma unroll
-        for (int j = 0; j < 4; ++j) {
-          const __nv_bfloat16 g16 = __float2bfloat16_rn(dv[j]);
-          uint8_t* dst = dzT + sw128_offset(ku0 + u4 + j, b);
-          *reinterpret_cast<__nv_bfloat16*>(dst) = g16;
-#pragma unroll
-          for (int o = 0; o < S; ++o)
-            if (o != half) st_dsmem_b16(dst, grp * S + o, g16);
-        }
+        for (int c = 0; c < kFC; ++c) dh = fmaf(dzb[b * kFC + c], wc[c], dh);
+        dh = hs[b * Cfg::kHsd + u] > 0.f ? dh : 0.f;
+        dv[i] = dh;
+        gsum += dh;
       }
-      *reinterpret_cast<float4*>(gbp + rg * UPC + u4) = gs;
+      const uint4 p = make_uint4(pack_bf16x2(dv[0], dv[1]), pack_bf16x2(dv[2], dv[3]), pack_bf16x2(dv[4], dv[5]),
+                                 pack_bf16x2(dv[6], dv[7]));
+      uint8_t* dst = dzT + sw128_offset(ku0 + u, 8 * j);
+      *reinterpret_cast<uint4*>(dst) = p;
+#pragma unroll
+      for (int o = 0; o < S; ++o)
+        if (o != half) st_dsmem_u32x4(dst, grp * S + o, p);
+      gbp[j * UPC + u] = gsum;
     }
     fence_proxy_async_smem();   // dz0^T is read by the tensor core next
     __syncthreads();
-    if (t < UPC) {   // b0 of this CTA's units
-      float g = 0.f;
-#pragma unroll
-      for (int r = 0; r < Cfg::kGrpRows; ++r) g += gbp[r * UPC + t];
-      const float nb = fmaf(-a.lr, g, b0m[ku0 + t]);
-      b0m[ku0 + t] = nb;
-      if (last) a.master_w[dof + a.offB0 + g0 + ku0 + t] = nb;
-    }
-    // head weight gradient + SGD of this CTA's columns: item = (class, 4 units)
-    for (int q = t; q < kFC * (UPC / 4); q += kFT) {
-      const int c = q / (UPC / 4), u4 = (q % (UPC / 4)) * 4;
+    // head weight gradient of this CTA's columns, item = (class, 4 units),
+    // split over the two halves of the batch (partials in the idle F ring)
+    float4* w1p = reinterpret_cast<float4*>(fring);   // [2][kW1Items]
+    for (int q = t; q < 2 * Cfg::kW1Items; q += kFT) {
+      const int item = q % Cfg::kW1Items, hb = q / Cfg::kW1Items;
+      const int c = item / (UPC / 4), u4 = (item % (UPC / 4)) * 4;
       float4 dw = make_float4(0.f, 0.f, 0.f, 0.f);
-      for (int b = 0; b < B; ++b) {
+#pragma unroll 8
+      for (int b = hb * (B / 2); b < (hb + 1) * (B / 2); ++b) {
         const float g = dzb[b * kFC + c];
         const float4 hv = *reinterpret_cast<const float4*>(hs + b * Cfg::kHsd + u4);
         dw.x = fmaf(g, hv.x, dw.x);
@@ -587,6 +601,22 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
         dw.z = fmaf(g, hv.z, dw.z);
         dw.w = fmaf(g, hv.w, dw.w);
       }
+      w1p[hb * Cfg::kW1Items + item] = dw;
+    }
+    if (t < UPC) {   // b0 of this CTA's units (chunk sums in chunk order)
+      float g = 0.f;
+#pragma unroll
+      for (int r = 0; r < Cfg::kChunks; ++r) g += gbp[r * UPC + t];
+      const float nb = fmaf(-a.lr, g, b0m[ku0 + t]);
+      b0m[ku0 + t] = nb;
+      if (last) a.master_w[dof + a.offB0 + g0 + ku0 + t] = nb;
+    }
+    __syncthreads();
+    // SGD of the head-weight columns: first half + second half of the batch
+    for (int item = t; item < Cfg::kW1Items; item += kFT) {
+      const int c = item / (UPC / 4), u4 = (item % (UPC / 4)) * 4;
+      const float4 d0 = w1p[item], d1 = w1p[Cfg::kW1Items + item];
+      const float4 dw = make_float4(d0.x + d1.x, d0.y + d1.y, d0.z + d1.z, d0.w + d1.w);
       const float4 o = *reinterpret_cast<const float4*>(w1m + c * UPC + u4);
       float4 nw;
       nw.x = fmaf(-a.lr, dw.x, o.x);
