@@ -54,6 +54,10 @@
 // fence.proxy.async.  Arithmetic and rounding points are those of the
 // per-layer path (the pair's two partial sums are added in rank order).
 //
+// The kernel is launched as a programmatic dependent of the staging grid:
+// TMEM allocation and the model load overlap the staging, and it waits for
+// the staging grid (griddepcontrol.wait) before touching a staged tile.
+//
 // Clusters are launched in order of decreasing tau (a table maps cluster to
 // worker): when fewer clusters fit on the GPU than there are workers, the
 // late ones start as the short workers finish (longest first).
@@ -315,7 +319,6 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
     return true;
   };
   bool producer_ok = true;
-  if (warp == 0 && lane == 0) producer_ok = issue_f(0, 0, pre_f);
   double loss_sum = 0.0;   // rank 0, thread 0: sum of the 16-row loss chunks, in step and chunk order
 
   // the global model, once: fp32 master block into TMEM and its bf16 copy
@@ -367,6 +370,10 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  // the staged mini-batches, labels and cursors are the staging grid's: wait
+  // for it (a no-op without programmatic dependent launch)
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  if (warp == 0 && lane == 0) producer_ok = issue_f(0, 0, pre_f);
 
   for (int s = 0; s < tau; ++s) {
     if (stamp) a.phase_ts[s * 4 + 0] = global_ns();
@@ -742,13 +749,16 @@ cudaError_t launch_bs(const CUtensorMap& mX, const CUtensorMap& mXT, const Fused
   cfg.blockDim = dim3(kFT, 1, 1);
   cfg.dynamicSmemBytes = Cfg::kSmem;
   cfg.stream = s;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = 1;
   attr[0].val.clusterDim.y = S * (a.H / kFU);
   attr[0].val.clusterDim.z = 1;
+  // may start before the staging grid ends (it waits for it after loading the model)
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = 2;
   return cudaLaunchKernelEx(&cfg, fused_mlp2_round_kernel<B, S>, mX, mXT, a);
 }
 

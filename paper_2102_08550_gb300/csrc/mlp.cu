@@ -74,6 +74,10 @@ constexpr int kStageRows = 32, kStageCols = 128;
 __global__ void __launch_bounds__(256) stage_round_kernel(const __grid_constant__ StageArgs a, const int32_t* tau,
                                                           int W) {
   __shared__ __align__(16) __nv_bfloat16 tile[kStageCols][kStageRows + 8];
+  // the round kernel that consumes these tiles may launch now (programmatic
+  // dependent launch: it loads the model first and waits for this grid
+  // before reading any staged tile)
+  asm volatile("griddepcontrol.launch_dependents;");
   const int z = blockIdx.z;
   const int s = z / W, w = z - s * W;
   if (s >= tau[w]) return;
