@@ -331,3 +331,36 @@ def test_shards_partitioned_by_tau(cuda_device):
         np.testing.assert_allclose(losses[r], recs[r].worker_loss, rtol=LOSS_RTOL)
         assert_within(per_tensor_errors(flats[r], recs[r].x_g, w.dims), np.zeros(2), f"round {r}")
     assert state.cursor.tolist() == (tau.astype(np.int64) * w.batch).tolist()   # wrapped after round 3
+
+
+def kernel_classes(w, device, rows):
+    """Kernel classes one round of a context runs (profiling context)."""
+    ctx, _ = make_context(w, device_shards(w, device, n=rows), device, flags=P.FLAG_PROFILE)
+    ctx.local_steps()
+    ctx.push_merge()
+    names = set(ctx.profile())
+    ctx.close()
+    return names
+
+
+FUSED_VARIANTS = [
+    # name, dims, W, B, one-launch round expected
+    ("b32-pair", [784, 512, 10], 3, 32, True),       # two CTAs per unit group, batch 32
+    ("b32-single", [384, 768, 10], 2, 32, True),     # one CTA per group (cluster of 6)
+    ("ragged-d", [200, 256, 10], 3, 64, True),       # 200 inputs: partial K-block and weight-gradient tile
+    ("b64-single", [384, 768, 10], 2, 64, False),    # too large for one CTA per group: per-layer path
+]
+
+
+@pytest.mark.parametrize("name,dims,W,B,fused", FUSED_VARIANTS, ids=[v[0] for v in FUSED_VARIANTS])
+def test_round_kernel_variants(cuda_device, name, dims, W, B, fused):
+    """Shapes of the one-launch round kernel beyond the headline one, and a
+    shape it refuses: the path taken is checked, then one exact step on
+    integer inputs (1e-5 per tensor) and three rounds on Gaussian inputs
+    (conditioning envelope) against the oracle."""
+    rows = 4 * B
+    w = synth.TrainWorkload(f"variant-{name}", W, dims, B, 0.05, rows, 6, 3)
+    names = kernel_classes(w, cuda_device, rows)
+    assert ("fused_round" in names) == fused, names
+    run_both(w, 1, cuda_device, rows=rows, tau_override=[1] * W, exact_inputs=True, eval_n=2 * B)
+    run_both(w, 3, cuda_device, rows=rows, eval_n=2 * B)
