@@ -158,6 +158,17 @@ oscars_status oscars_destroy(oscars_ctx* ctx);
 oscars_status oscars_local_steps(oscars_ctx* ctx, int32_t* tau_out, float* loss_out);
 
 /*
+ * oscars_losses_async - enqueue a copy of the per-worker mean mini-batch
+ * losses of the last oscars_local_steps (W floats) into dst (host or device)
+ * on the context's stream, without synchronising: the values are in dst once
+ * the stream has reached this point (use pinned host memory for an
+ * asynchronous copy).  Lets a training loop read each round's losses while
+ * the next round runs.  Errors: EINVAL (NULL), ESTATE (no local steps yet, or
+ * FLAT mode), ECUDA.
+ */
+oscars_status oscars_losses_async(oscars_ctx* ctx, float* dst);
+
+/*
  * oscars_push_merge - server merge and global update (Eq. 4, first branch).
  *
  * x_g <- x_g + server_lr * sum_k w_k * delta_k, accumulated in fp32 registers

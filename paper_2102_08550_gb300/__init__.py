@@ -54,6 +54,7 @@ _SIGS = {
     "oscars_create": (c_int32, [POINTER(OscarsConfig), POINTER(c_void_p)]),
     "oscars_destroy": (c_int32, [c_void_p]),
     "oscars_local_steps": (c_int32, [c_void_p, POINTER(c_int32), POINTER(c_float)]),
+    "oscars_losses_async": (c_int32, [c_void_p, c_void_p]),
     "oscars_push_merge": (c_int32, [c_void_p, POINTER(c_void_p), POINTER(c_float)]),
     "oscars_pull": (c_int32, [c_void_p, c_void_p]),
     "oscars_get_schedule": (c_int32, [c_void_p, POINTER(c_int64), POINTER(c_int64), POINTER(c_int64),
@@ -204,6 +205,11 @@ def oscars_local_steps(ctx: int, want_tau: bool = True, want_loss: bool = True):
     return (list(tau) if tau is not None else None), (list(loss) if loss is not None else None)
 
 
+def oscars_losses_async(ctx: int, dst_ptr: int):
+    """Enqueue the copy of the last round's W losses into dst (no synchronisation)."""
+    _check(lib().oscars_losses_async(c_void_p(ctx), c_void_p(dst_ptr)), c_void_p(ctx))
+
+
 def oscars_push_merge(ctx: int, delta_ptrs: Optional[Sequence[int]] = None, weights: Optional[Sequence[float]] = None):
     d = _arr(c_void_p, delta_ptrs) if delta_ptrs is not None else None
     w = _arr(c_float, weights) if weights is not None else None
@@ -340,6 +346,9 @@ class OscarsContext:
 
     def local_steps(self, want_loss: bool = True):
         return oscars_local_steps(self.handle, want_tau=True, want_loss=want_loss)
+
+    def losses_async(self, dst):
+        oscars_losses_async(self.handle, dst.data_ptr())
 
     def push_merge(self, deltas=None, weights=None):
         ptrs = [d.data_ptr() for d in deltas] if deltas is not None else None

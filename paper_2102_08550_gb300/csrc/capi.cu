@@ -161,6 +161,7 @@ struct oscars_ctx {
   int* br_src = nullptr;
   cudaGraphExec_t round_exec = nullptr;
   bool pending = false;
+  int64_t rounds_run = 0;               // oscars_local_steps calls that launched a round
   std::string last_error;
   // per-kernel-class CUDA-event profile (flag bit 1, direct launches only)
   struct ProfEntry {
@@ -1003,6 +1004,7 @@ oscars_status oscars_local_steps(oscars_ctx* c, int32_t* tau_out, float* loss_ou
       c->idle[i] += c->barrier - busy;
     }
     c->pending = true;
+    ++c->rounds_run;
     if (tau_out) std::memcpy(tau_out, c->tau.data(), c->W * sizeof(int32_t));
     if (loss_out) {
       e = cudaStreamSynchronize(c->stream);
@@ -1014,6 +1016,13 @@ oscars_status oscars_local_steps(oscars_ctx* c, int32_t* tau_out, float* loss_ou
   } catch (const std::bad_alloc&) {
     return fail(c, OSCARS_ENOMEM, "host allocation failed");
   }
+}
+
+oscars_status oscars_losses_async(oscars_ctx* c, float* dst) {
+  if (!c || !dst) return OSCARS_EINVAL;
+  if (c->model != OSCARS_MODEL_MLP || c->rounds_run == 0) return fail(c, OSCARS_ESTATE, "no local steps to report");
+  const cudaError_t e = cudaMemcpyAsync(dst, c->loss_dev, c->W * sizeof(float), cudaMemcpyDefault, c->stream);
+  return e == cudaSuccess ? OSCARS_OK : cuda_fail(c, e, "loss copy");
 }
 
 oscars_status oscars_push_merge(oscars_ctx* c, const float* const* deltas, const float* weights) {

@@ -364,3 +364,20 @@ def test_round_kernel_variants(cuda_device, name, dims, W, B, fused):
     assert ("fused_round" in names) == fused, names
     run_both(w, 1, cuda_device, rows=rows, tau_override=[1] * W, exact_inputs=True, eval_n=2 * B)
     run_both(w, 3, cuda_device, rows=rows, eval_n=2 * B)
+
+
+def test_losses_async_matches_synchronous_read(cuda_device):
+    w = synth.TrainWorkload("small-async", 3, [256, 128, 10], 32, 0.05, 128, 4, 2)
+    ctx, _ = make_context(w, device_shards(w, cuda_device, n=128), cuda_device)
+    buf = torch.empty(3, dtype=torch.float32).pin_memory()
+    with pytest.raises(P.OscarsError) as e:
+        ctx.losses_async(buf)                    # no round yet
+    assert e.value.status == P.OSCARS_ESTATE
+    for _ in range(2):
+        _, loss = ctx.local_steps()
+        buf.fill_(-1.0)
+        ctx.losses_async(buf)
+        torch.cuda.synchronize()
+        np.testing.assert_array_equal(buf.numpy(), np.asarray(loss, np.float32))
+        ctx.push_merge()
+    ctx.close()
