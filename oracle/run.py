@@ -43,6 +43,31 @@ def unflatten(flat: np.ndarray, dims: Sequence[int]):
     return out
 
 
+class MLPModel:
+    """The MLP of ``oracle.model`` behind the interface the round loop uses
+    (flatten, unflatten, sgd_step, loss_of); ``oracle.conv.CNN`` offers the
+    same interface for the convolutional worker."""
+
+    def __init__(self, dims: Sequence[int]):
+        self.dims = list(dims)
+
+    def flatten(self, layers):
+        return flatten(layers)
+
+    def unflatten(self, flat):
+        return unflatten(flat, self.dims)
+
+    def sgd_step(self, layers, X, y, lr, rnd):
+        return _model.sgd_step(layers, X, y, lr, rnd)
+
+    def loss_of(self, layers, X, y, rnd):
+        return _model.loss_of(layers, X, y, rnd)
+
+
+def _copy(params):
+    return [tuple(a.copy() for a in p) if isinstance(p, tuple) else p.copy() for p in params]
+
+
 def batch_indices(cursor: int, batch: int, n: int) -> np.ndarray:
     return (cursor + np.arange(batch, dtype=np.int64)) % n
 
@@ -60,7 +85,7 @@ class RoundRecord:
 @dataclass
 class OscarsState:
     dims: List[int]
-    x_g: List[Tuple[np.ndarray, np.ndarray]]
+    x_g: list                # the global model's parameters (the model's own structure)
     cursor: np.ndarray
     clock: np.ndarray
     idle: np.ndarray
@@ -68,18 +93,21 @@ class OscarsState:
     T_star: int          # the round's barrier: T* of Algorithm 1, else max_i tau_i t_i
     max_wait: int
     tau: np.ndarray
+    model: object = None
 
 
-def init_state(dims, layers0, t_iter, M: int, mode: int = _sched.CAPPED, tau_override=None) -> OscarsState:
+def init_state(dims, layers0, t_iter, M: int, mode: int = _sched.CAPPED, tau_override=None,
+               model=None) -> OscarsState:
     T_star, mw, tau = _sched.schedule(t_iter, M, mode)
     if tau_override is not None:
         tau = np.asarray(tau_override, dtype=np.int32)
         T_star = _sched.round_barrier(t_iter, tau)
         mw = int(np.max(T_star - tau.astype(np.int64) * np.asarray(t_iter, np.int64)))
     W = len(t_iter)
-    return OscarsState(list(dims), [(W_.copy(), b.copy()) for W_, b in layers0],
+    return OscarsState(list(dims), _copy(layers0),
                        np.zeros(W, np.int64), np.zeros(W, np.int64), np.zeros(W, np.int64),
-                       np.asarray(t_iter, np.int64), T_star, mw, tau)
+                       np.asarray(t_iter, np.int64), T_star, mw, tau,
+                       model if model is not None else MLPModel(dims))
 
 
 def reschedule(state: OscarsState, t_iter, M: int, mode: int = _sched.CAPPED) -> None:
@@ -93,12 +121,12 @@ def reschedule(state: OscarsState, t_iter, M: int, mode: int = _sched.CAPPED) ->
 def local_steps(state: OscarsState, worker: int, shard, batch: int, lr: float, rnd: Callable):
     """Worker ``worker`` pulls the global model and runs tau_i local SGD steps."""
     X, y = shard
-    layers = [(W.copy(), b.copy()) for W, b in state.x_g]          # pull
+    layers = _copy(state.x_g)                                      # pull
     losses = []
     for _ in range(int(state.tau[worker])):
         idx = batch_indices(int(state.cursor[worker]), batch, X.shape[0])
         state.cursor[worker] = (state.cursor[worker] + batch) % X.shape[0]
-        layers, loss = _model.sgd_step(layers, X[idx], y[idx], lr, rnd)
+        layers, loss = state.model.sgd_step(layers, X[idx], y[idx], lr, rnd)
         losses.append(loss)
     return layers, float(np.mean(losses))
 
@@ -109,10 +137,10 @@ def run_round(state: OscarsState, shards, batch: int, lr: float, rnd: Callable,
     models, wl = [], np.zeros(W)
     for i in range(W):
         layers, wl[i] = local_steps(state, i, shards[i], batch, lr, rnd)
-        models.append(flatten(layers))                             # push
+        models.append(state.model.flatten(layers))                 # push
     w = _sched.merge_weights(weight_rule, state.tau, weights)
-    x_new = _merge.merge_models(flatten(state.x_g), models, w, server_lr)
-    state.x_g = unflatten(x_new, state.dims)
+    x_new = _merge.merge_models(state.model.flatten(state.x_g), models, w, server_lr)
+    state.x_g = state.model.unflatten(x_new)
     idle = state.T_star - state.tau.astype(np.int64) * state.t_iter     # = mod(T*, t_i) under Algorithm 1
     state.clock += state.tau.astype(np.int64) * state.t_iter + idle
     state.idle += idle
@@ -122,7 +150,7 @@ def run_round(state: OscarsState, shards, batch: int, lr: float, rnd: Callable,
 def run(dims, layers0, shards, speeds=None, t_iter=None, M: int = 8, rounds: int = 1,
         batch: int = 32, lr: float = 0.05, bf16: bool = True, weight_rule: str = "uniform",
         server_lr: float = 1.0, mode: int = _sched.CAPPED, tau_override=None,
-        eval_set=None, ticks_per_unit: int = 1000, target_loss=None, t_per_round=None):
+        eval_set=None, ticks_per_unit: int = 1000, target_loss=None, t_per_round=None, model=None):
     """Run ``rounds`` rounds; returns (final state, [RoundRecord]).  With an
     eval set and a target loss, stop after the first round whose eval loss
     is at or below the target.  ``t_per_round[r]`` (optional): iteration
@@ -131,14 +159,14 @@ def run(dims, layers0, shards, speeds=None, t_iter=None, M: int = 8, rounds: int
     if t_iter is None:
         t_iter = t_per_round[0] if t_per_round is not None else _sched.iteration_ticks(speeds, ticks_per_unit)
     rnd = _bf16.round_bf16 if bf16 else _bf16.identity
-    state = init_state(dims, layers0, t_iter, M, mode, tau_override)
+    state = init_state(dims, layers0, t_iter, M, mode, tau_override, model)
     records = []
     for r in range(rounds):
         if t_per_round is not None and r > 0:
             reschedule(state, t_per_round[r], M, mode)
         rec = run_round(state, shards, batch, lr, rnd, weight_rule, server_lr)
         if eval_set is not None:
-            rec.eval_loss = _model.loss_of(state.x_g, eval_set[0], eval_set[1], rnd)
+            rec.eval_loss = state.model.loss_of(state.x_g, eval_set[0], eval_set[1], rnd)
         records.append(rec)
         if target_loss is not None and rec.eval_loss is not None and rec.eval_loss <= target_loss:
             break
