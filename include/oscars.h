@@ -55,8 +55,25 @@ typedef enum {
 
 typedef enum {
   OSCARS_MODEL_FLAT = 0, /* merge only: dims[0] = P parameters, no local steps */
-  OSCARS_MODEL_MLP = 1   /* ReLU MLP / softmax regression with softmax CE      */
+  OSCARS_MODEL_MLP = 1,  /* ReLU MLP / softmax regression with softmax CE      */
+  OSCARS_MODEL_CNN = 2   /* residual CNN on images (see below)                  */
 } oscars_model;
+
+/*
+ * OSCARS_MODEL_CNN: the convolutional worker, a residual network of the kind
+ * the paper trains (ResNet on CIFAR-10, Section "Dataset and DL Models") on
+ * H x W x Cin NHWC images:
+ *   s = relu(conv(x) + b0); per block u = relu(conv(h) + b_a),
+ *   v = relu(conv(u) + b_b + h); g = mean over positions of v;
+ *   logits = g W_f^T + b_f, softmax cross-entropy.
+ * Convolutions are 3x3, stride 1, zero padding 1.  dims = {H, W, Cin, C, K}
+ * (C channels, K classes), num_layers = number of residual blocks.  This
+ * build supports H = W = 32, C = 64, 1 <= Cin <= 64, 2 <= K <= 32, 1 to 4
+ * blocks, bf16 GEMMs, and a batch that is a multiple of 16 up to 256.
+ * Canonical parameter layout: W_0 [C][3][3][Cin], b_0 [C], then per block
+ * W_a [C][3][3][C], b_a, W_b, b_b, then W_f [K][C], b_f [K].  A shard holds
+ * n images of H*W*Cin fp32 values (NHWC) and n labels.
+ */
 
 typedef enum {
   OSCARS_W_UNIFORM = 0,    /* w_k = 1/N: the average of Eq. 4 (first branch)        */

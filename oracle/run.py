@@ -104,7 +104,7 @@ def init_state(dims, layers0, t_iter, M: int, mode: int = _sched.CAPPED, tau_ove
         T_star = _sched.round_barrier(t_iter, tau)
         mw = int(np.max(T_star - tau.astype(np.int64) * np.asarray(t_iter, np.int64)))
     W = len(t_iter)
-    return OscarsState(list(dims), _copy(layers0),
+    return OscarsState(list(dims) if dims is not None else [], _copy(layers0),
                        np.zeros(W, np.int64), np.zeros(W, np.int64), np.zeros(W, np.int64),
                        np.asarray(t_iter, np.int64), T_star, mw, tau,
                        model if model is not None else MLPModel(dims))

@@ -16,7 +16,7 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(HERE, "_lib", "liboscars.so")
 
 OSCARS_OK, OSCARS_EINVAL, OSCARS_ENOMEM, OSCARS_ECUDA, OSCARS_ESTATE, OSCARS_ETIMEOUT, OSCARS_ENOTSUP = range(7)
-MODEL_FLAT, MODEL_MLP = 0, 1
+MODEL_FLAT, MODEL_MLP, MODEL_CNN = 0, 1, 2
 W_UNIFORM, W_LOCALSTEPS, W_EXPLICIT = 0, 1, 2
 SEARCH_CAPPED, SEARCH_LITERAL = 0, 1
 POLICY_OSCARS, POLICY_BSP, POLICY_LOCAL_SGD = 0, 1, 2
@@ -301,13 +301,15 @@ class OscarsContext:
                  lr: float = 0.05, server_lr: float = 1.0, weight_rule: int = W_UNIFORM, bf16: bool = True,
                  speed: Optional[Sequence[float]] = None, t_ticks: Optional[Sequence[int]] = None,
                  ticks_per_unit: int = 1000, M: int = 8, search_mode: int = SEARCH_CAPPED, shards=None,
-                 init_params=None, stream: Optional[int] = None, flags: int = 0):
+                 init_params=None, stream: Optional[int] = None, flags: int = 0, blocks: int = 1):
+        """dims: MLP [input, hidden..., classes]; CNN [H, W, Cin, C, classes]
+        with ``blocks`` residual blocks; FLAT [P]."""
         W = num_workers
         self._keep = []
         cfg = OscarsConfig()
         cfg.num_workers = W
         cfg.model = model
-        L = len(dims) - 1 if model == MODEL_MLP else 1
+        L = len(dims) - 1 if model == MODEL_MLP else (blocks if model == MODEL_CNN else 1)
         cfg.num_layers = L
         dims_arr = _arr(c_int32, dims)
         self._keep.append(dims_arr)

@@ -80,6 +80,20 @@ bool make_map4(CUtensorMap* m, const void* base, uint64_t d0, uint64_t d1, uint6
            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// 4-D bf16 tensor map with an explicit box, 128-byte swizzle, zero fill
+bool make_map_box4(CUtensorMap* m, const void* base, const uint64_t (&d)[4], const uint64_t (&st)[3],
+                   const uint32_t (&box)[4]) {
+  EncodeTiledFn f = encode_fn();
+  if (!f) return false;
+  cuuint64_t dims[4] = {d[0], d[1], d[2], d[3]};
+  cuuint64_t strides[3] = {st[0], st[1], st[2]};
+  cuuint32_t bx[4] = {box[0], box[1], box[2], box[3]};
+  cuuint32_t es[4] = {1, 1, 1, 1};
+  return f(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 4, const_cast<void*>(base), dims, strides, bx, es,
+           CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+           CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 struct Layer {
   int in, out;
   int64_t offW, offB, offT;  // offT < 0: no transposed copy
@@ -146,6 +160,19 @@ struct oscars_ctx {
   bool fused = false;                   // whole-round kernel (2-layer MLP)
   CUtensorMap mX4, mXT4;                // staged inputs of every step (fused kernel)
   unsigned long long* phase_ts = nullptr;   // flag bit 4: phase stamps of the fused round
+  // convolutional worker (OSCARS_MODEL_CNN)
+  int cnn_blocks = 0, cnn_chunks = 0;
+  std::vector<int64_t> cnn_offW, cnn_offB;   // conv layers: stem, then (a, b) of every block
+  int64_t cnn_offWf = 0, cnn_offBf = 0;
+  int64_t cnn_wt_slot = 0;                   // elements per slot of the transposed copies
+  __nv_bfloat16* cnn_wt = nullptr;           // [slot][2 * blocks][9][64 in][64 out]
+  std::vector<__nv_bfloat16*> cnn_buf;       // x, s, (u_k, v_k) per block, dz0, dz1, dz2: [W][B][1024][64]
+  std::vector<CUtensorMap> cnn_m4, cnn_m2;   // per buffer: boxes of 4 and of 2 image rows
+  std::vector<CUtensorMap> cnn_mw, cnn_mwt;  // weights per conv layer: forward layout, transposed (blocks)
+  float* cnn_g = nullptr;                    // [W][B][64] pooled features
+  float* cnn_dg = nullptr;                   // [W][B][64] their gradient
+  float* cnn_wpart = nullptr;                // [layer][W][chunks][9][64][64]
+  float* cnn_bpart = nullptr;                // [layer][W][B * 8][64]
   // streams / graph
   cudaStream_t stream = nullptr;
   cudaStream_t cap = nullptr;
@@ -432,6 +459,12 @@ cudaError_t refresh_global_shadows(oscars_ctx* c, cudaStream_t s, bool plain_don
   const int64_t g = static_cast<int64_t>(c->W) * c->P_pad;
   cudaError_t e = plain_done ? cudaSuccess : launch_shadow_refresh(c->slab + g, c->shadow + g, c->P_pad, s);
   if (e != cudaSuccess) return e;
+  for (size_t l = 1; l < c->cnn_offW.size(); ++l) {   // CNN: transposed copies of the block convolutions
+    e = launch_conv_refresh_wt(c->slab + g, c->cnn_wt + static_cast<int64_t>(c->W) * c->cnn_wt_slot +
+                                                static_cast<int64_t>(l - 1) * 9 * 64 * 64,
+                               c->cnn_offW[l], s);
+    if (e != cudaSuccess) return e;
+  }
   for (const Layer& ly : c->layers) {
     if (ly.offT < 0) continue;
     e = launch_transpose_bf16(c->shadow + g + ly.offW,
@@ -661,7 +694,153 @@ cudaError_t enqueue_round_softreg(oscars_ctx* c, cudaStream_t st) {
   return launch_cursor_advance(c->cursor, c->tau_dev, c->dn_tab, c->B, c->W, st);
 }
 
+// one local step of the convolutional worker for the `na` active workers
+cudaError_t enqueue_step_cnn(oscars_ctx* c, int s, int na, const int* wid, const int* src, cudaStream_t st) {
+  cudaError_t e;
+  const int B = c->B, nb = c->cnn_blocks, layers = 1 + 2 * nb;
+  const int tiles = B * cnn_tiles_per_image();
+  const int X = 0, S = 1, dzbase = 2 + 2 * nb;
+  auto U = [&](int k) { return 2 + 2 * k; };
+  auto V = [&](int k) { return 3 + 2 * k; };
+  const size_t wpl = static_cast<size_t>(c->W) * c->cnn_chunks * 9 * 64 * 64;   // weight partials per layer
+  const size_t bpl = static_cast<size_t>(c->W) * tiles * 64;                    // bias partials per layer
+  {
+    CnnStageArgs a;
+    a.x = c->dx_tab;
+    a.y = c->dy_tab;
+    a.n = c->dn_tab;
+    a.start = c->cursor;
+    a.wid = wid;
+    a.step = s;
+    a.B = B;
+    a.Cin = c->dims[2];
+    a.out = c->cnn_buf[X];
+    a.labels = c->labels;
+    ProfScope ps(c, "cnn_stage", st);
+    if ((e = launch_cnn_stage(a, na, st)) != cudaSuccess) return e;
+  }
+  auto conv = [&](int mode, int layer, int in, int add, int mask, int out, float* bpart) -> cudaError_t {
+    ConvArgs a;
+    std::memset(&a, 0, sizeof(a));
+    a.wid = wid;
+    a.src = src;
+    a.B = B;
+    a.bias = c->slab;
+    a.slot_stride = c->P_pad;
+    a.off_bias = c->cnn_offB[layer];
+    a.add = add >= 0 ? c->cnn_buf[add] : nullptr;
+    a.mask = mask >= 0 ? c->cnn_buf[mask] : nullptr;
+    a.out = c->cnn_buf[out];
+    a.bias_part = bpart;
+    a.err = c->err;
+    ProfScope ps(c, mode == 0 ? "conv_fwd" : "conv_dgrad", st);
+    return launch_conv_igemm(mode, c->cnn_m4[in], mode == 0 ? c->cnn_mw[layer] : c->cnn_mwt[layer - 1], a, na, st);
+  };
+  auto wgrad = [&](int layer, int in, int dz) -> cudaError_t {
+    WgradArgs a;
+    a.wid = wid;
+    a.B = B;
+    a.n_chunks = c->cnn_chunks;
+    a.img_per_chunk = kWgradImagesPerChunk;
+    a.part = c->cnn_wpart + layer * wpl;
+    a.err = c->err;
+    ProfScope ps(c, "conv_wgrad", st);
+    return launch_conv_wgrad(c->cnn_m2[in], c->cnn_m2[dz], a, na, st);
+  };
+  // forward
+  if ((e = conv(0, 0, X, -1, -1, S, nullptr)) != cudaSuccess) return e;
+  for (int k = 0; k < nb; ++k) {
+    const int h = k == 0 ? S : V(k - 1);
+    if ((e = conv(0, 1 + 2 * k, h, -1, -1, U(k), nullptr)) != cudaSuccess) return e;
+    if ((e = conv(0, 2 + 2 * k, U(k), h, -1, V(k), nullptr)) != cudaSuccess) return e;
+  }
+  // head: pooling, FC, softmax cross-entropy, its backward and SGD
+  {
+    ProfScope ps(c, "cnn_head", st);
+    if ((e = launch_cnn_pool(c->cnn_buf[V(nb - 1)], wid, B, c->cnn_g, na, st)) != cudaSuccess) return e;
+    CnnHeadArgs h;
+    h.wid = wid;
+    h.src = src;
+    h.B = B;
+    h.K = c->C;
+    h.step = s;
+    h.max_tau = c->max_tau;
+    h.n_loss_chunks = B / kRowsPerLossChunk;
+    h.g = c->cnn_g;
+    h.labels = c->labels;
+    h.dg = c->cnn_dg;
+    h.loss_part = c->loss_part;
+    h.master = c->slab;
+    h.master_w = c->slab;
+    h.shadow = c->shadow;
+    h.slot_stride = c->P_pad;
+    h.offWf = c->cnn_offWf;
+    h.offBf = c->cnn_offBf;
+    h.lr = c->lr;
+    if ((e = launch_cnn_head(h, na, st)) != cudaSuccess) return e;
+  }
+  // backward through the blocks; dz buffers rotate: cur = output gradient of block k
+  int cur = dzbase, nxt = dzbase + 1, nx2 = dzbase + 2;
+  {
+    ProfScope ps(c, "cnn_dzb", st);
+    if ((e = launch_cnn_dzb(c->cnn_buf[V(nb - 1)], c->cnn_dg, wid, B, c->cnn_buf[cur],
+                            c->cnn_bpart + (2 + 2 * (nb - 1)) * bpl, na, st)) != cudaSuccess)
+      return e;
+  }
+  for (int k = nb - 1; k >= 0; --k) {
+    const int la = 1 + 2 * k, lb = 2 + 2 * k;
+    const int h = k == 0 ? S : V(k - 1);
+    const int lprev = k == 0 ? 0 : 2 + 2 * (k - 1);   // the layer whose output h is
+    if ((e = wgrad(lb, U(k), cur)) != cudaSuccess) return e;
+    if ((e = conv(1, lb, cur, -1, U(k), nxt, c->cnn_bpart + la * bpl)) != cudaSuccess) return e;
+    if ((e = wgrad(la, h, nxt)) != cudaSuccess) return e;
+    if ((e = conv(1, la, nxt, cur, h, nx2, c->cnn_bpart + lprev * bpl)) != cudaSuccess) return e;
+    const int t0 = cur;
+    cur = nx2;
+    nx2 = t0;
+  }
+  if ((e = wgrad(0, X, cur)) != cudaSuccess) return e;
+  // SGD of every convolution layer (after all input gradients used the old weights)
+  ProfScope ps(c, "conv_sgd", st);
+  for (int l = 0; l < layers; ++l) {
+    ConvSgdArgs a;
+    a.wid = wid;
+    a.src = src;
+    a.n_chunks = c->cnn_chunks;
+    a.n_tiles = tiles;
+    a.part = c->cnn_wpart + l * wpl;
+    a.bias_part = c->cnn_bpart + l * bpl;
+    a.master = c->slab;
+    a.master_w = c->slab;
+    a.shadow = c->shadow;
+    a.wt = l >= 1 ? c->cnn_wt + static_cast<int64_t>(l - 1) * 9 * 64 * 64 : nullptr;
+    a.slot_stride = c->P_pad;
+    a.offW = c->cnn_offW[l];
+    a.offB = c->cnn_offB[l];
+    a.wt_slot_stride = c->cnn_wt_slot;
+    a.lr = c->lr;
+    if ((e = launch_conv_sgd(a, na, st)) != cudaSuccess) return e;
+  }
+  return cudaSuccess;
+}
+
+cudaError_t enqueue_round_cnn(oscars_ctx* c, cudaStream_t st) {
+  cudaError_t e;
+  for (int s = 0; s < c->max_tau; ++s) {
+    const int na = c->n_active[s];
+    if ((e = enqueue_step_cnn(c, s, na, c->act_wid + static_cast<size_t>(s) * c->W,
+                              c->act_src + static_cast<size_t>(s) * c->W, st)) != cudaSuccess)
+      return e;
+  }
+  const int nc = c->B / kRowsPerLossChunk;
+  ProfScope ps(c, "round_bookkeeping", st);
+  if ((e = launch_loss_finalize(c->loss_part, c->tau_dev, c->W, c->max_tau, nc, c->B, c->loss_dev, st)) != cudaSuccess)
+    return e;
+  return launch_cursor_advance(c->cursor, c->tau_dev, c->dn_tab, c->B, c->W, st);
+}
+
 cudaError_t enqueue_round(oscars_ctx* c, cudaStream_t st) {
+  if (c->model == OSCARS_MODEL_CNN) return enqueue_round_cnn(c, st);
   return c->L == 1 && !c->bf16 ? enqueue_round_softreg(c, st) : enqueue_round_mlp(c, st);
 }
 
@@ -674,6 +853,46 @@ oscars_status check_err_word(oscars_ctx* c) {
     cudaMemset(c->err, 0, sizeof(int));
     return fail(c, OSCARS_ETIMEOUT, "a kernel's bounded wait ran out (code " + std::to_string(h) + ")");
   }
+  return OSCARS_OK;
+}
+
+bool slotted(const oscars_ctx* c) { return c->model == OSCARS_MODEL_MLP || c->model == OSCARS_MODEL_CNN; }
+
+// convolutional worker: checks and the slot layout (every tensor on a
+// 64-element boundary; the stem's input channels padded to 64)
+oscars_status layout_cnn(oscars_ctx* c, const oscars_config* cfg) {
+  c->cnn_blocks = cfg->num_layers;
+  c->dims.assign(cfg->dims, cfg->dims + 5);
+  const int H = c->dims[0], Wd = c->dims[1], Cin = c->dims[2], C = c->dims[3], K = c->dims[4];
+  c->B = cfg->batch;
+  c->C = K;
+  c->L = 0;
+  if (H < 1 || Wd < 1 || Cin < 1 || C < 1 || K < 1 || c->B < 1) return fail(c, OSCARS_EINVAL, "CNN: dims and batch must be >= 1");
+  if (!(c->lr == c->lr)) return fail(c, OSCARS_EINVAL, "lr is NaN");
+  if (c->cnn_blocks < 1 || c->cnn_blocks > 4) return fail(c, OSCARS_ENOTSUP, "CNN: 1 to 4 residual blocks");
+  if (H != 32 || Wd != 32 || C != 64) return fail(c, OSCARS_ENOTSUP, "CNN: 32 x 32 images and 64 channels");
+  if (Cin > 64) return fail(c, OSCARS_ENOTSUP, "CNN: at most 64 input channels");
+  if (K < 2 || K > kMaxClasses) return fail(c, OSCARS_ENOTSUP, "classes must be in [2, 32]");
+  if (!c->bf16) return fail(c, OSCARS_ENOTSUP, "CNN: bf16 GEMMs only");
+  if (c->B % kRowsPerLossChunk != 0 || c->B > 256) return fail(c, OSCARS_ENOTSUP, "CNN: batch must be a multiple of 16, <= 256");
+  if (c->W > kMaxWorkersMLP) return fail(c, OSCARS_ENOTSUP, "CNN mode supports at most 64 workers");
+  const int layers = 1 + 2 * c->cnn_blocks;
+  int64_t off = 0;
+  for (int l = 0; l < layers; ++l) {
+    c->cnn_offW.push_back(off);
+    off += 64 * 9 * 64;
+    c->cnn_offB.push_back(off);
+    off += 64;
+  }
+  c->cnn_offWf = off;
+  off += round_up(static_cast<int64_t>(K) * C, 64);
+  c->cnn_offBf = off;
+  off += round_up(K, 64);
+  c->P_pad = round_up(off, 64);
+  c->P = static_cast<int64_t>(C) * 9 * Cin + C + static_cast<int64_t>(c->cnn_blocks) * 2 * (C * 9 * C + C) +
+         static_cast<int64_t>(K) * C + K;
+  c->cnn_wt_slot = static_cast<int64_t>(2 * c->cnn_blocks) * 9 * 64 * 64;
+  c->cnn_chunks = cnn_wgrad_chunks(c->B);
   return OSCARS_OK;
 }
 
@@ -695,6 +914,7 @@ oscars_status validate_and_layout(oscars_ctx* c, const oscars_config* cfg) {
     c->P_pad = round_up(c->P, 64);
     return OSCARS_OK;
   }
+  if (c->model == OSCARS_MODEL_CNN) return layout_cnn(c, cfg);
   if (c->model != OSCARS_MODEL_MLP) return fail(c, OSCARS_EINVAL, "unknown model");
   c->L = cfg->num_layers;
   if (c->L < 1 || c->L > 16) return fail(c, OSCARS_EINVAL, "num_layers must be in [1, 16]");
@@ -742,8 +962,9 @@ oscars_status validate_and_layout(oscars_ctx* c, const oscars_config* cfg) {
   return OSCARS_OK;
 }
 
-oscars_status allocate_mlp(oscars_ctx* c) {
-  const int W = c->W, B = c->B, L = c->L;
+// the slab of W + 1 slots and the per-worker tables (MLP and CNN)
+oscars_status allocate_common(oscars_ctx* c) {
+  const int W = c->W;
   const size_t slots = static_cast<size_t>(W) + 1;
   if (!dev_alloc(c, &c->slab, slots * c->P_pad)) return fail(c, OSCARS_ENOMEM, "device allocation failed (model slab)");
   cudaMemset(c->slab, 0, slots * c->P_pad * sizeof(float));
@@ -762,6 +983,66 @@ oscars_status allocate_mlp(oscars_ctx* c) {
   cudaMemcpy(c->dy_tab, c->shard_y.data(), W * sizeof(int32_t*), cudaMemcpyHostToDevice);
   cudaError_t e = cudaMemcpy(c->dn_tab, c->shard_n.data(), W * sizeof(int64_t), cudaMemcpyHostToDevice);
   if (e != cudaSuccess) return cuda_fail(c, e, "table upload");
+  return OSCARS_OK;
+}
+
+oscars_status allocate_cnn(oscars_ctx* c) {
+  oscars_status st = allocate_common(c);
+  if (st != OSCARS_OK) return st;
+  const int W = c->W, B = c->B;
+  const size_t slots = static_cast<size_t>(W) + 1;
+  const int layers = 1 + 2 * c->cnn_blocks;
+  if (!dev_alloc(c, &c->shadow, slots * c->P_pad) || !dev_alloc(c, &c->cnn_wt, slots * c->cnn_wt_slot))
+    return fail(c, OSCARS_ENOMEM, "device allocation failed (bf16 weights)");
+  cudaMemset(c->shadow, 0, slots * c->P_pad * sizeof(__nv_bfloat16));
+  cudaMemset(c->cnn_wt, 0, slots * c->cnn_wt_slot * sizeof(__nv_bfloat16));
+  const size_t act = static_cast<size_t>(W) * B * 1024 * 64;
+  const int nbuf = 2 + 2 * c->cnn_blocks + 3;
+  c->cnn_buf.assign(nbuf, nullptr);
+  for (int i = 0; i < nbuf; ++i)
+    if (!dev_alloc(c, &c->cnn_buf[i], act)) return fail(c, OSCARS_ENOMEM, "device allocation failed (activations)");
+  const size_t tiles = static_cast<size_t>(B) * cnn_tiles_per_image();
+  if (!dev_alloc(c, &c->cnn_g, static_cast<size_t>(W) * B * 64) ||
+      !dev_alloc(c, &c->cnn_dg, static_cast<size_t>(W) * B * 64) ||
+      !dev_alloc(c, &c->labels, static_cast<size_t>(W) * B) ||
+      !dev_alloc(c, &c->cnn_wpart, static_cast<size_t>(layers) * W * c->cnn_chunks * 9 * 64 * 64) ||
+      !dev_alloc(c, &c->cnn_bpart, static_cast<size_t>(layers) * W * tiles * 64))
+    return fail(c, OSCARS_ENOMEM, "device allocation failed (gradients)");
+  // tensor maps: activations {64 ch, 32 x, 32 y, images}; weights per slot
+  c->cnn_m4.resize(nbuf);
+  c->cnn_m2.resize(nbuf);
+  const uint64_t imgs = static_cast<uint64_t>(W) * B;
+  bool ok = true;
+  for (int i = 0; i < nbuf; ++i) {
+    const uint64_t d[4] = {64, 32, 32, imgs};
+    const uint64_t stv[3] = {64 * 2, 32 * 64 * 2, 1024 * 64 * 2};
+    ok &= make_map_box4(&c->cnn_m4[i], c->cnn_buf[i], d, stv, {64, 32, 4, 1});
+    ok &= make_map_box4(&c->cnn_m2[i], c->cnn_buf[i], d, stv, {64, 32, 2, 1});
+  }
+  c->cnn_mw.resize(layers);
+  c->cnn_mwt.resize(layers > 1 ? layers - 1 : 1);
+  for (int l = 0; l < layers; ++l) {
+    // forward layout [out][tap][in] of every slot: dims {in, tap, out, slot}
+    const uint64_t d[4] = {64, 9, 64, slots};
+    const uint64_t stv[3] = {64 * 2, 9 * 64 * 2, static_cast<uint64_t>(c->P_pad) * 2};
+    ok &= make_map_box4(&c->cnn_mw[l], c->shadow + c->cnn_offW[l], d, stv, {64, 1, 64, 1});
+    if (l >= 1) {
+      // transposed [tap][in][out]: dims {out, in, tap, slot}
+      const uint64_t dt[4] = {64, 64, 9, slots};
+      const uint64_t stt[3] = {64 * 2, 64 * 64 * 2, static_cast<uint64_t>(c->cnn_wt_slot) * 2};
+      ok &= make_map_box4(&c->cnn_mwt[l - 1], c->cnn_wt + static_cast<int64_t>(l - 1) * 9 * 64 * 64, dt, stt,
+                          {64, 64, 1, 1});
+    }
+  }
+  if (!ok) return fail(c, OSCARS_ECUDA, "cuTensorMapEncodeTiled failed (CNN)");
+  return OSCARS_OK;
+}
+
+oscars_status allocate_mlp(oscars_ctx* c) {
+  oscars_status st0 = allocate_common(c);
+  if (st0 != OSCARS_OK) return st0;
+  const int W = c->W, B = c->B, L = c->L;
+  const size_t slots = static_cast<size_t>(W) + 1;
   if (L == 1 && !c->bf16) return OSCARS_OK;
 
   if (!dev_alloc(c, &c->shadow, slots * c->P_pad)) return fail(c, OSCARS_ENOMEM, "device allocation failed (bf16 shadow)");
@@ -821,6 +1102,31 @@ oscars_status allocate_mlp(oscars_ctx* c) {
 
 // copy a canonical-layout vector into the padded slot layout (or back)
 cudaError_t copy_canonical(oscars_ctx* c, float* padded, const float* canon, bool to_padded, cudaStream_t s) {
+  if (c->model == OSCARS_MODEL_CNN) {
+    const int Cin = c->dims[2], K = c->dims[4];
+    float* dst = const_cast<float*>(canon);
+    int64_t co = 0;
+    // stem [64][9][Cin] <-> [64][9][64] (the padded channels stay zero)
+    cudaError_t e = to_padded ? cudaMemcpy2DAsync(padded + c->cnn_offW[0], 64 * sizeof(float), canon, Cin * sizeof(float),
+                                                  Cin * sizeof(float), 64 * 9, cudaMemcpyDefault, s)
+                              : cudaMemcpy2DAsync(dst, Cin * sizeof(float), padded + c->cnn_offW[0], 64 * sizeof(float),
+                                                  Cin * sizeof(float), 64 * 9, cudaMemcpyDefault, s);
+    co = static_cast<int64_t>(64) * 9 * Cin;
+    auto seg = [&](int64_t off, int64_t n) -> cudaError_t {
+      cudaError_t r = to_padded ? cudaMemcpyAsync(padded + off, canon + co, n * sizeof(float), cudaMemcpyDefault, s)
+                                : cudaMemcpyAsync(dst + co, padded + off, n * sizeof(float), cudaMemcpyDefault, s);
+      co += n;
+      return r;
+    };
+    if (e == cudaSuccess) e = seg(c->cnn_offB[0], 64);
+    for (size_t l = 1; e == cudaSuccess && l < c->cnn_offW.size(); ++l) {
+      e = seg(c->cnn_offW[l], 64 * 9 * 64);
+      if (e == cudaSuccess) e = seg(c->cnn_offB[l], 64);
+    }
+    if (e == cudaSuccess) e = seg(c->cnn_offWf, static_cast<int64_t>(K) * 64);
+    if (e == cudaSuccess) e = seg(c->cnn_offBf, K);
+    return e;
+  }
   if (c->model == OSCARS_MODEL_FLAT) {
     return to_padded ? cudaMemcpyAsync(padded, canon, c->P * sizeof(float), cudaMemcpyDefault, s)
                      : cudaMemcpyAsync(const_cast<float*>(canon), padded, c->P * sizeof(float), cudaMemcpyDefault, s);
@@ -887,12 +1193,12 @@ oscars_status oscars_create(const oscars_config* cfg, oscars_ctx** out) {
       update_barrier(c, true);
       c->clock.assign(c->W, 0);
       c->idle.assign(c->W, 0);
-      if (c->model == OSCARS_MODEL_MLP) {
+      if (slotted(c)) {
         if (!cfg->shard_x || !cfg->shard_y || !cfg->shard_n) st = fail(c, OSCARS_EINVAL, "MLP: shard pointers are NULL");
         for (int i = 0; st == OSCARS_OK && i < c->W; ++i) {
           if (!cfg->shard_x[i] || !cfg->shard_y[i] || cfg->shard_n[i] < 1)
             st = fail(c, OSCARS_EINVAL, "MLP: shard " + std::to_string(i) + " is NULL or empty");
-          else if (c->bf16 && (reinterpret_cast<uintptr_t>(cfg->shard_x[i]) & 15))
+          else if (c->model == OSCARS_MODEL_MLP && c->bf16 && (reinterpret_cast<uintptr_t>(cfg->shard_x[i]) & 15))
             st = fail(c, OSCARS_EINVAL, "bf16 MLP: shard " + std::to_string(i) + " samples must be 16-byte aligned");
           else {
             c->shard_x.push_back(cfg->shard_x[i]);
@@ -902,11 +1208,11 @@ oscars_status oscars_create(const oscars_config* cfg, oscars_ctx** out) {
         }
         if (st == OSCARS_OK && !cfg->init_params) st = fail(c, OSCARS_EINVAL, "MLP: init_params is NULL");
         // a 2-layer bf16 MLP runs each round as one fused launch (flag bit 3: per-layer kernels)
-        c->fused = c->bf16 && !(cfg->flags & 8) && !(cfg->flags & 4) &&
+        c->fused = c->model == OSCARS_MODEL_MLP && c->bf16 && !(cfg->flags & 8) && !(cfg->flags & 4) &&
                    fused_round_supported(c->L, c->dims[0], c->L >= 2 ? c->dims[1] : 0, c->C, c->B);
         // flag bit 2: bf16 MLP rounds fork into up to 16 concurrent worker branches
-        c->n_br = (c->bf16 && c->L >= 2 && (cfg->flags & 4)) ? std::min(c->W, kMaxBranches) : 1;
-        if (st == OSCARS_OK) st = allocate_mlp(c);
+        c->n_br = (c->model == OSCARS_MODEL_MLP && c->bf16 && c->L >= 2 && (cfg->flags & 4)) ? std::min(c->W, kMaxBranches) : 1;
+        if (st == OSCARS_OK) st = c->model == OSCARS_MODEL_CNN ? allocate_cnn(c) : allocate_mlp(c);
         if (st == OSCARS_OK) st = build_tables(c);
         if (st == OSCARS_OK) {
           cudaError_t e = copy_canonical(c, c->slab + static_cast<int64_t>(c->W) * c->P_pad, cfg->init_params, true, c->stream);
@@ -965,7 +1271,7 @@ oscars_status oscars_destroy(oscars_ctx* c) {
 
 oscars_status oscars_local_steps(oscars_ctx* c, int32_t* tau_out, float* loss_out) {
   if (!c) return OSCARS_EINVAL;
-  if (c->model != OSCARS_MODEL_MLP) return fail(c, OSCARS_ESTATE, "local steps need an MLP context");
+  if (!slotted(c)) return fail(c, OSCARS_ESTATE, "local steps need an MLP or CNN context");
   if (c->pending) return fail(c, OSCARS_ESTATE, "the previous round has not been merged");
   try {
     cudaError_t e = cudaSuccess;
@@ -1020,7 +1326,7 @@ oscars_status oscars_local_steps(oscars_ctx* c, int32_t* tau_out, float* loss_ou
 
 oscars_status oscars_losses_async(oscars_ctx* c, float* dst) {
   if (!c || !dst) return OSCARS_EINVAL;
-  if (c->model != OSCARS_MODEL_MLP || c->rounds_run == 0) return fail(c, OSCARS_ESTATE, "no local steps to report");
+  if (!slotted(c) || c->rounds_run == 0) return fail(c, OSCARS_ESTATE, "no local steps to report");
   const cudaError_t e = cudaMemcpyAsync(dst, c->loss_dev, c->W * sizeof(float), cudaMemcpyDefault, c->stream);
   return e == cudaSuccess ? OSCARS_OK : cuda_fail(c, e, "loss copy");
 }
@@ -1042,10 +1348,10 @@ oscars_status oscars_push_merge(oscars_ctx* c, const float* const* deltas, const
     oscars_ctx* c;
     ~ProfOff() { c->profiling = false; }
   } prof_off{c};
-  float* xg = c->slab + (c->model == OSCARS_MODEL_MLP ? static_cast<int64_t>(c->W) * c->P_pad : 0);
+  float* xg = c->slab + (slotted(c) ? static_cast<int64_t>(c->W) * c->P_pad : 0);
   cudaError_t e = cudaSuccess;
   if (!deltas) {
-    if (c->model != OSCARS_MODEL_MLP || !c->pending)
+    if (!slotted(c) || !c->pending)
       return fail(c, OSCARS_ESTATE, "push_merge without deltas needs pending local steps");
     for (int k = 0; k < c->W; ++k) a.src[k] = c->slab + static_cast<int64_t>(k) * c->P_pad;
     auto enqueue = [&](cudaStream_t st) -> cudaError_t {
@@ -1055,7 +1361,7 @@ oscars_status oscars_push_merge(oscars_ctx* c, const float* const* deltas, const
         r = launch_merge(a, xg, c->P_pad, eta, true, st, c->shadow ? c->shadow + static_cast<int64_t>(c->W) * c->P_pad : nullptr);
       }
       if (r != cudaSuccess) return r;
-      if (c->PT_pad == 0) return cudaSuccess;   // no transposed copies to refresh
+      if (c->PT_pad == 0 && c->model != OSCARS_MODEL_CNN) return cudaSuccess;   // no transposed copies to refresh
       ProfScope ps(c, "shadow_refresh", st);
       return refresh_global_shadows(c, st, true);
     };
@@ -1092,6 +1398,7 @@ oscars_status oscars_push_merge(oscars_ctx* c, const float* const* deltas, const
   } else {
     for (int k = 0; k < c->W; ++k)
       if (!deltas[k]) return fail(c, OSCARS_EINVAL, "NULL delta pointer");
+    if (c->model == OSCARS_MODEL_CNN) return fail(c, OSCARS_ENOTSUP, "CNN: merge the workers' replicas (deltas == NULL)");
     if (c->model == OSCARS_MODEL_FLAT) {
       for (int k = 0; k < c->W; ++k) a.src[k] = deltas[k];
       ProfScope ps(c, "merge", c->stream);
@@ -1122,11 +1429,11 @@ oscars_status oscars_push_merge(oscars_ctx* c, const float* const* deltas, const
 oscars_status oscars_pull(oscars_ctx* c, float* dst) {
   if (!c) return OSCARS_EINVAL;
   cudaError_t e = cudaSuccess;
-  const int64_t g = c->model == OSCARS_MODEL_MLP ? static_cast<int64_t>(c->W) * c->P_pad : 0;
+  const int64_t g = slotted(c) ? static_cast<int64_t>(c->W) * c->P_pad : 0;
   if (dst) {
     e = copy_canonical(c, c->slab + g, dst, false, c->stream);
     if (e == cudaSuccess && is_host_ptr(dst)) e = cudaStreamSynchronize(c->stream);
-  } else if (c->model == OSCARS_MODEL_MLP) {
+  } else if (slotted(c)) {
     e = launch_broadcast(c->slab + g, c->slab, c->P_pad, c->W, c->P_pad, c->stream);
     for (int k = 0; e == cudaSuccess && k < c->W && c->shadow; ++k)
       e = cudaMemcpyAsync(c->shadow + static_cast<int64_t>(k) * c->P_pad, c->shadow + g,
@@ -1162,7 +1469,7 @@ oscars_status oscars_set_local_steps(oscars_ctx* c, const int32_t* tau) {
     if (tau[i] < 1) return fail(c, OSCARS_EINVAL, "tau must be >= 1");
   for (int i = 0; i < c->W; ++i) c->tau[i] = tau[i];
   update_barrier(c, false);
-  if (c->model == OSCARS_MODEL_MLP) {
+  if (slotted(c)) {
     cudaStreamSynchronize(c->stream);
     return build_tables(c);
   }
@@ -1183,7 +1490,7 @@ oscars_status oscars_set_iteration_ticks(oscars_ctx* c, const int64_t* t_iter) {
   c->T_star = T;
   c->max_wait = mw;
   update_barrier(c, true);
-  if (c->model == OSCARS_MODEL_MLP) {
+  if (slotted(c)) {
     cudaStreamSynchronize(c->stream);
     return build_tables(c);
   }
@@ -1192,10 +1499,73 @@ oscars_status oscars_set_iteration_ticks(oscars_ctx* c, const int64_t* t_iter) {
 
 oscars_status oscars_eval_loss(oscars_ctx* c, const float* x, const int32_t* y, int64_t n, float* loss) {
   if (!c || !x || !y || !loss || n < 1) return OSCARS_EINVAL;
-  if (c->model != OSCARS_MODEL_MLP) return fail(c, OSCARS_ESTATE, "eval needs an MLP context");
+  if (!slotted(c)) return fail(c, OSCARS_ESTATE, "eval needs an MLP or CNN context");
   cudaError_t e = cudaSuccess;
   const int64_t g = static_cast<int64_t>(c->W) * c->P_pad;
-  if (c->L == 1 && !c->bf16) {
+  if (c->model == OSCARS_MODEL_CNN) {
+    // chunks of up to B images through lane 0 with the global model's weights
+    const int64_t chunks = (n + c->B - 1) / c->B;
+    if (c->eval_part_cap < chunks) {
+      if (!dev_alloc(c, &c->eval_part, chunks)) return fail(c, OSCARS_ENOMEM, "eval scratch");
+      c->eval_part_cap = chunks;
+    }
+    if (c->estart_cap < 1) {
+      if (!dev_alloc(c, &c->estart, 1)) return fail(c, OSCARS_ENOMEM, "eval scratch");
+      c->estart_cap = 1;
+    }
+    const int64_t zero = 0;
+    const int64_t img = static_cast<int64_t>(c->dims[0]) * c->dims[1] * c->dims[2];
+    e = cudaMemcpyAsync(c->estart, &zero, sizeof(int64_t), cudaMemcpyHostToDevice, c->stream);
+    for (int64_t ch = 0; e == cudaSuccess && ch < chunks; ++ch) {
+      const int Bc = static_cast<int>(std::min<int64_t>(c->B, n - ch * c->B));
+      const float* xc = x + ch * c->B * img;
+      const int32_t* yc = y + ch * c->B;
+      const int64_t nc = Bc;
+      e = cudaMemcpyAsync(c->ex_tab, &xc, sizeof(float*), cudaMemcpyHostToDevice, c->stream);
+      if (e == cudaSuccess) e = cudaMemcpyAsync(c->ey_tab, &yc, sizeof(int32_t*), cudaMemcpyHostToDevice, c->stream);
+      if (e == cudaSuccess) e = cudaMemcpyAsync(c->en_tab, &nc, sizeof(int64_t), cudaMemcpyHostToDevice, c->stream);
+      if (e == cudaSuccess) e = cudaStreamSynchronize(c->stream);   // the host values above must not go out of scope early
+      if (e != cudaSuccess) break;
+      CnnStageArgs a;
+      a.x = c->ex_tab;
+      a.y = c->ey_tab;
+      a.n = c->en_tab;
+      a.start = c->estart;
+      a.wid = c->lane_ids;
+      a.step = 0;
+      a.B = Bc;
+      a.Cin = c->dims[2];
+      a.out = c->cnn_buf[0];
+      a.labels = c->labels;
+      e = launch_cnn_stage(a, 1, c->stream);
+      auto conv = [&](int layer, int in, int add, int out) -> cudaError_t {
+        ConvArgs ca;
+        std::memset(&ca, 0, sizeof(ca));
+        ca.wid = c->lane_ids;
+        ca.src = c->global_src;
+        ca.B = Bc;
+        ca.bias = c->slab;
+        ca.slot_stride = c->P_pad;
+        ca.off_bias = c->cnn_offB[layer];
+        ca.add = add >= 0 ? c->cnn_buf[add] : nullptr;
+        ca.out = c->cnn_buf[out];
+        ca.err = c->err;
+        return launch_conv_igemm(0, c->cnn_m4[in], c->cnn_mw[layer], ca, 1, c->stream);
+      };
+      if (e == cudaSuccess) e = conv(0, 0, -1, 1);
+      for (int k = 0; e == cudaSuccess && k < c->cnn_blocks; ++k) {
+        const int h = k == 0 ? 1 : 3 + 2 * (k - 1);
+        e = conv(1 + 2 * k, h, -1, 2 + 2 * k);
+        if (e == cudaSuccess) e = conv(2 + 2 * k, 2 + 2 * k, h, 3 + 2 * k);
+      }
+      if (e == cudaSuccess)
+        e = launch_cnn_pool(c->cnn_buf[3 + 2 * (c->cnn_blocks - 1)], c->lane_ids, Bc, c->cnn_g, 1, c->stream);
+      if (e == cudaSuccess)
+        e = launch_cnn_head_loss(c->cnn_g, c->labels, Bc, c->C, c->slab + g, c->cnn_offWf, c->cnn_offBf,
+                                 c->eval_part + ch, c->stream);
+    }
+    if (e == cudaSuccess) e = launch_sum_scaled(c->eval_part, chunks, 1.0 / static_cast<double>(n), c->loss_dev, c->stream);
+  } else if (c->L == 1 && !c->bf16) {
     const int blocks = static_cast<int>(std::min<int64_t>(1024, (n + 7) / 8));
     if (c->eval_part_cap < blocks) {
       if (!dev_alloc(c, &c->eval_part, blocks)) return fail(c, OSCARS_ENOMEM, "eval scratch");
@@ -1271,7 +1641,7 @@ oscars_status oscars_eval_loss(oscars_ctx* c, const float* x, const int32_t* y, 
 
 oscars_status oscars_read_replica(oscars_ctx* c, int32_t k, float* dst) {
   if (!c || !dst) return OSCARS_EINVAL;
-  if (c->model != OSCARS_MODEL_MLP) return fail(c, OSCARS_ESTATE, "replicas exist in MLP mode only");
+  if (!slotted(c)) return fail(c, OSCARS_ESTATE, "replicas exist in MLP and CNN mode only");
   if (k < 0 || k >= c->W) return fail(c, OSCARS_EINVAL, "worker index out of range");
   cudaError_t e = copy_canonical(c, c->slab + static_cast<int64_t>(k) * c->P_pad, dst, false, c->stream);
   if (e == cudaSuccess && is_host_ptr(dst)) e = cudaStreamSynchronize(c->stream);

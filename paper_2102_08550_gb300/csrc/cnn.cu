@@ -1,0 +1,613 @@
+// The convolutional worker: local SGD steps of a CIFAR-shaped residual
+// network (Eq. 4, "otherwise" branch, for the paper's kind of workload:
+// ResNet on CIFAR-10, Section "Dataset and DL Models").
+//
+//   s = relu(conv(x) + b0);  per block u = relu(conv(h) + b_a),
+//   v = relu(conv(u) + b_b + h);  g = mean_{y,x} v;  logits = g W_f^T + b_f
+//
+// Every convolution is 3x3, stride 1, zero padding 1, on 32 x 32 images with
+// 64 channels (the input's channels are zero-padded to 64).  Activations are
+// bf16 NHWC [lane][image][32][32][64]; a lane is one worker's batch.
+//
+// Kernels (all workers of a local step in one launch, grid y = active worker):
+//  * conv_igemm_kernel: implicit GEMM on tcgen05.  A CTA computes 128 output
+//    pixels (4 image rows) x 64 channels as the sum over the 9 taps of
+//    [128 pixels x 64 in-channels] x [64 x 64] products: per tap TMA loads
+//    the input box shifted by the tap offset (the zero padding is TMA's
+//    out-of-bounds fill) and the tap's weights.  Forward epilogue: bias,
+//    optional residual, ReLU, bf16.  Input-gradient mode: the box is shifted
+//    the other way and the weights are the transposed copy; epilogue: optional
+//    skip-path gradient, the ReLU mask of the layer input, bf16, and per-tile
+//    channel sums for the bias gradient.
+//  * conv_wgrad_kernel: dW[o][tap][i] = sum_p dz[p][o] x[p + off(tap)][i] on
+//    tcgen05 with both operands MN-major straight from the NHWC tensors: the
+//    K dimension is the pixels, taps are stacked in pairs to make M = 128
+//    (in-channels of two taps), N = 64 out-channels.  Split over chunks of
+//    images; partial sums go to global memory.
+//  * conv_sgd_kernel: sums the chunks in order, SGD of the fp32 master and
+//    its bf16 copies (the forward layout and the transposed one), bias from
+//    the per-tile sums.
+//  * pool, head, and output-gradient kernels on CUDA cores; input staging.
+#include "common.cuh"
+#include "internal.h"
+
+namespace oscars {
+namespace {
+
+constexpr int kCC = 64;                     // channels
+constexpr int kImg = 32;                    // image height and width
+constexpr int kPix = kImg * kImg;
+constexpr int kTileRows = 4;                // image rows per 128-pixel tile
+constexpr int kTilePix = kTileRows * kImg;  // 128
+constexpr int kTilesPerImg = kImg / kTileRows;
+constexpr int kTaps = 9;
+constexpr int kCT = 128;                    // threads of the implicit-GEMM and pixel kernels
+constexpr int kCStages = 4;
+constexpr int kCA = kTilePix * kCC * 2;     // 16 KB: 128 pixels x 64 channels
+constexpr int kCB = kCC * kCC * 2;          // 8 KB: one tap of the weights
+constexpr int kCSmem = kCStages * (kCA + kCB) + 256 + 1024;
+// weight gradient
+constexpr int kWT = 128;
+constexpr int kWStages = 2;
+constexpr int kWTile = 2 * kImg * kCC * 2;  // 8 KB: 64 pixels (2 rows) x 64 channels
+constexpr int kWPairs = 5;                  // tap pairs (0,1) (2,3) (4,5) (6,7) (8,8)
+constexpr int kWStage = (2 * kWPairs + 1) * kWTile;   // 10 input tiles + the output-gradient tile
+constexpr int kWSmem = kWStages * kWStage + 256 + 1024;
+
+__device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
+  return reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(p) + 1023) & ~uintptr_t(1023));
+}
+
+// ------------------------------------------------------------------ implicit GEMM (forward / input gradient)
+template <int MODE>   // 0 forward, 1 input gradient
+__global__ void __launch_bounds__(kCT) conv_igemm_kernel(const __grid_constant__ CUtensorMap mIn,
+                                                         const __grid_constant__ CUtensorMap mW,
+                                                         const __grid_constant__ ConvArgs a) {
+  extern __shared__ uint8_t cs_raw[];
+  uint8_t* sm = align1024(cs_raw);
+  uint64_t* full = reinterpret_cast<uint64_t*>(sm + kCStages * (kCA + kCB));
+  uint64_t* empty = full + kCStages;
+  uint64_t* accb = empty + kCStages;
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(accb + 1);
+  const int t = threadIdx.x, warp = t >> 5;
+  const int tile = blockIdx.x, e = blockIdx.y;
+  const int lane = a.wid[e], slot = a.src[e];
+  const int b = tile / kTilesPerImg, y0 = (tile % kTilesPerImg) * kTileRows;
+  const int img = lane * a.B + b;
+  if (t == 0) {
+    prefetch_tmap(&mIn);
+    prefetch_tmap(&mW);
+    for (int i = 0; i < kCStages; ++i) {
+      mbar_init(&full[i], 1);
+      mbar_init(&empty[i], 1);
+    }
+    mbar_init(accb, 1);
+    fence_barrier_init();
+  }
+  if (warp == 0) {
+    tmem_alloc(tslot, 64);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tslot;
+  const int sgn = MODE == 0 ? 1 : -1;   // the input gradient reads the output gradient at p - off(tap)
+  if (t == 0) {
+    for (int tap = 0; tap < kTaps; ++tap) {
+      const int st = tap % kCStages;
+      if (tap >= kCStages && !mbar_wait(&empty[st], ((tap / kCStages) + 1) & 1, a.err, kDevTimeoutEmpty)) break;
+      uint8_t* sa = sm + st * (kCA + kCB);
+      mbar_arrive_expect_tx(&full[st], kCA + kCB);
+      const int dy = tap / 3, dx = tap % 3;
+      tma_load_4d(sa, &mIn, 0, sgn * (dx - 1), y0 + sgn * (dy - 1), img, &full[st]);
+      if (MODE == 0) tma_load_4d(sa + kCA, &mW, 0, tap, 0, slot, &full[st]);   // {in, tap, out, slot}
+      else tma_load_4d(sa + kCA, &mW, 0, 0, tap, slot, &full[st]);             // {out, in, tap, slot}
+    }
+  } else if (t == 32) {
+    constexpr uint32_t idesc = idesc_bf16_f32(128, kCC);
+    for (int tap = 0; tap < kTaps; ++tap) {
+      const int st = tap % kCStages;
+      if (!mbar_wait(&full[st], (tap / kCStages) & 1, a.err, kDevTimeoutFull)) break;
+      tc_fence_after();
+      const uint32_t sa = smem_u32(sm + st * (kCA + kCB));
+#pragma unroll
+      for (int j = 0; j < kCC / 16; ++j)
+        umma_bf16(tmem, smem_desc_k128(sa + j * 32), smem_desc_k128(sa + kCA + j * 32), idesc,
+                  (tap | j) != 0 ? 1u : 0u);
+      umma_commit(&empty[st]);
+    }
+    umma_commit(accb);
+  }
+  // epilogue: thread = output pixel (TMEM lane), 64 channels
+  int ok = mbar_wait(accb, 0, a.err, kDevTimeoutAccum) ? 1 : 0;
+  ok = __all_sync(0xffffffffu, ok);
+  tc_fence_after();
+  const int p = t;
+  const int64_t base = (static_cast<int64_t>(img) * kPix + y0 * kImg + p) * kCC;
+  float v[kCC];
+  if (ok) {
+    float lo[32], hi[32];
+    tmem_ld_32x32b_x32_pair(tmem + (static_cast<uint32_t>(warp * 32) << 16), lo,
+                            tmem + (static_cast<uint32_t>(warp * 32) << 16) + 32, hi);
+#pragma unroll
+    for (int c = 0; c < 32; ++c) {
+      v[c] = lo[c];
+      v[32 + c] = hi[c];
+    }
+  } else {
+#pragma unroll
+    for (int c = 0; c < kCC; ++c) v[c] = 0.f;
+  }
+  if (MODE == 0) {
+    const float* bias = a.bias + static_cast<int64_t>(slot) * a.slot_stride + a.off_bias;
+#pragma unroll
+    for (int c = 0; c < kCC; ++c) v[c] += bias[c];
+  }
+  if (a.add) {
+#pragma unroll
+    for (int q = 0; q < kCC / 8; ++q) {
+      const uint4 r = *reinterpret_cast<const uint4*>(a.add + base + 8 * q);
+      const __nv_bfloat162* r2 = reinterpret_cast<const __nv_bfloat162*>(&r);
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const float2 f = __bfloat1622float2(r2[j]);
+        v[8 * q + 2 * j] += f.x;
+        v[8 * q + 2 * j + 1] += f.y;
+      }
+    }
+  }
+  if (MODE == 0) {
+#pragma unroll
+    for (int c = 0; c < kCC; ++c) v[c] = fmaxf(v[c], 0.f);
+  } else {
+#pragma unroll
+    for (int q = 0; q < kCC / 8; ++q) {
+      const uint4 r = *reinterpret_cast<const uint4*>(a.mask + base + 8 * q);
+      const __nv_bfloat162* r2 = reinterpret_cast<const __nv_bfloat162*>(&r);
+#pragma unroll
+      for (int j = 0; j < 4; ++j) {
+        const float2 f = __bfloat1622float2(r2[j]);
+        if (!(f.x > 0.f)) v[8 * q + 2 * j] = 0.f;
+        if (!(f.y > 0.f)) v[8 * q + 2 * j + 1] = 0.f;
+      }
+    }
+  }
+#pragma unroll
+  for (int q = 0; q < kCC / 8; ++q)
+    *reinterpret_cast<uint4*>(a.out + base + 8 * q) =
+        make_uint4(pack_bf16x2(v[8 * q], v[8 * q + 1]), pack_bf16x2(v[8 * q + 2], v[8 * q + 3]),
+                   pack_bf16x2(v[8 * q + 4], v[8 * q + 5]), pack_bf16x2(v[8 * q + 6], v[8 * q + 7]));
+  if (MODE == 1 && a.bias_part) {
+    // channel sums of the fp32 output over the tile's pixels (fixed order),
+    // through the idle stage buffers: [128 pixels][65]
+    float* T = reinterpret_cast<float*>(sm);
+    __syncthreads();
+#pragma unroll
+    for (int c = 0; c < kCC; ++c) T[p * 65 + c] = v[c];
+    __syncthreads();
+    if (t < kCC) {
+      float s = 0.f;
+      for (int q = 0; q < kTilePix; ++q) s += T[q * 65 + t];
+      a.bias_part[(static_cast<int64_t>(lane) * a.B * kTilesPerImg + tile) * kCC + t] = s;
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) {
+    tc_fence_after();
+    tmem_dealloc(tmem, 64);
+  }
+}
+
+// ------------------------------------------------------------------ weight gradient
+__global__ void __launch_bounds__(kWT, 1) conv_wgrad_kernel(const __grid_constant__ CUtensorMap mIn,
+                                                            const __grid_constant__ CUtensorMap mDz,
+                                                            const __grid_constant__ WgradArgs a) {
+  extern __shared__ uint8_t ws_raw[];
+  uint8_t* sm = align1024(ws_raw);
+  uint64_t* full = reinterpret_cast<uint64_t*>(sm + kWStages * kWStage);
+  uint64_t* empty = full + kWStages;
+  uint64_t* accb = empty + kWStages;
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(accb + 1);
+  const int t = threadIdx.x, warp = t >> 5;
+  const int chunk = blockIdx.x, e = blockIdx.y;
+  const int lane = a.wid[e];
+  const int i0 = chunk * a.img_per_chunk;
+  const int n_img = min(a.img_per_chunk, a.B - i0);
+  const int nk = n_img * (kImg / 2);             // K-blocks: 64 pixels = 2 image rows
+  if (t == 0) {
+    prefetch_tmap(&mIn);
+    prefetch_tmap(&mDz);
+    for (int i = 0; i < kWStages; ++i) {
+      mbar_init(&full[i], 1);
+      mbar_init(&empty[i], 1);
+    }
+    mbar_init(accb, 1);
+    fence_barrier_init();
+  }
+  if (warp == 0) {
+    tmem_alloc(tslot, 512);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *tslot;
+  if (t == 0) {
+    for (int kb = 0; kb < nk; ++kb) {
+      const int st = kb % kWStages;
+      if (kb >= kWStages && !mbar_wait(&empty[st], ((kb / kWStages) + 1) & 1, a.err, kDevTimeoutEmpty)) break;
+      uint8_t* sa = sm + st * kWStage;
+      const int img = lane * a.B + i0 + kb / (kImg / 2), yr = (kb % (kImg / 2)) * 2;
+      mbar_arrive_expect_tx(&full[st], kWStage);
+      tma_load_4d(sa + 2 * kWPairs * kWTile, &mDz, 0, 0, yr, img, &full[st]);
+      for (int q = 0; q < 2 * kWPairs; ++q) {
+        const int tap = q < kTaps ? q : kTaps - 1;
+        const int dy = tap / 3, dx = tap % 3;
+        tma_load_4d(sa + q * kWTile, &mIn, 0, dx - 1, yr + dy - 1, img, &full[st]);
+      }
+    }
+  } else if (t == 32) {
+    constexpr uint32_t idesc = idesc_bf16_f32_mn(128, kCC);
+    for (int kb = 0; kb < nk; ++kb) {
+      const int st = kb % kWStages;
+      if (!mbar_wait(&full[st], (kb / kWStages) & 1, a.err, kDevTimeoutFull)) break;
+      tc_fence_after();
+      const uint32_t sa = smem_u32(sm + st * kWStage);
+      const uint32_t sb = sa + 2 * kWPairs * kWTile;
+#pragma unroll
+      for (int pr = 0; pr < kWPairs; ++pr)
+#pragma unroll
+        for (int j = 0; j < 4; ++j)   // K = 16 pixels per MMA: two 8-row groups
+          umma_bf16(tmem + pr * kCC, smem_desc_mn128(sa + pr * 2 * kWTile + j * 2048, kWTile),
+                    smem_desc_mn128(sb + j * 2048, kWTile), idesc, (kb | j) != 0 ? 1u : 0u);
+      umma_commit(&empty[st]);
+    }
+    umma_commit(accb);
+  }
+  int ok = mbar_wait(accb, 0, a.err, kDevTimeoutAccum) ? 1 : 0;
+  ok = __all_sync(0xffffffffu, ok);
+  tc_fence_after();
+  // TMEM lane r: row r of each pair's accumulator = (tap 2 pr + r / 64, in-channel r % 64)
+  const int r = t;
+  const int ci = r & (kCC - 1);
+  for (int pr = 0; pr < kWPairs; ++pr) {
+    const int tap = 2 * pr + (r >> 6);
+    float lo[32], hi[32];
+    tmem_ld_32x32b_x32_pair(tmem + (static_cast<uint32_t>(warp * 32) << 16) + pr * kCC, lo,
+                            tmem + (static_cast<uint32_t>(warp * 32) << 16) + pr * kCC + 32, hi);
+    if (tap < kTaps && ok) {
+      float* dst = a.part + ((static_cast<int64_t>(lane) * a.n_chunks + chunk) * kTaps + tap) * kCC * kCC + ci * kCC;
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        reinterpret_cast<float4*>(dst)[q] = make_float4(lo[4 * q], lo[4 * q + 1], lo[4 * q + 2], lo[4 * q + 3]);
+        reinterpret_cast<float4*>(dst + 32)[q] = make_float4(hi[4 * q], hi[4 * q + 1], hi[4 * q + 2], hi[4 * q + 3]);
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == 0) {
+    tc_fence_after();
+    tmem_dealloc(tmem, 512);
+  }
+}
+
+// ------------------------------------------------------------------ reduce + SGD of a convolution layer
+// grid (taps, active workers), 256 threads: one tap's [64 in][64 out] tile
+__global__ void __launch_bounds__(256) conv_sgd_kernel(const __grid_constant__ ConvSgdArgs a) {
+  __shared__ float T[kCC][kCC + 1];   // [in][out]
+  const int tap = blockIdx.x, e = blockIdx.y;
+  const int lane = a.wid[e], src = a.src[e];
+  const int t = threadIdx.x;
+  // sum of the chunks in chunk order; thread -> (in = t / 4 + 64 k / ..., out) with out fastest
+  for (int q = t; q < kCC * kCC; q += 256) {
+    const int ci = q / kCC, co = q % kCC;
+    float s = 0.f;
+    for (int c = 0; c < a.n_chunks; ++c)
+      s += a.part[((static_cast<int64_t>(lane) * a.n_chunks + c) * kTaps + tap) * kCC * kCC + q];
+    T[ci][co] = s;
+  }
+  __syncthreads();
+  const int64_t so = static_cast<int64_t>(src) * a.slot_stride, dof = static_cast<int64_t>(lane) * a.slot_stride;
+  // master / forward copy: [out][tap][in], in fastest
+  for (int q = t; q < kCC * kCC; q += 256) {
+    const int co = q / kCC, ci = q % kCC;
+    const int64_t off = a.offW + (static_cast<int64_t>(co) * kTaps + tap) * kCC + ci;
+    const float nw = fmaf(-a.lr, T[ci][co], a.master[so + off]);
+    a.master_w[dof + off] = nw;
+    a.shadow[dof + off] = __float2bfloat16_rn(nw);
+    T[ci][co] = nw;   // in this loop every element is read and rewritten by one thread
+  }
+  if (a.wt) {
+    __syncthreads();
+    // transposed copy [tap][in][out], out fastest
+    __nv_bfloat16* wt = a.wt + static_cast<int64_t>(lane) * a.wt_slot_stride + static_cast<int64_t>(tap) * kCC * kCC;
+    for (int q = t; q < kCC * kCC; q += 256) wt[q] = __float2bfloat16_rn(T[q / kCC][q % kCC]);
+  }
+  if (tap == 0 && t < kCC) {   // bias: per-tile sums in tile order
+    float s = 0.f;
+    for (int i = 0; i < a.n_tiles; ++i) s += a.bias_part[(static_cast<int64_t>(lane) * a.n_tiles + i) * kCC + t];
+    a.master_w[dof + a.offB + t] = fmaf(-a.lr, s, a.master[so + a.offB + t]);
+  }
+}
+
+// bf16 transposed weight copies of one slot from its fp32 master (after a merge)
+__global__ void conv_refresh_wt_kernel(const float* master, __nv_bfloat16* wt, int64_t offW) {
+  const int tap = blockIdx.x;
+  for (int q = threadIdx.x; q < kCC * kCC; q += blockDim.x) {
+    const int ci = q / kCC, co = q % kCC;
+    wt[static_cast<int64_t>(tap) * kCC * kCC + q] =
+        __float2bfloat16_rn(master[offW + (static_cast<int64_t>(co) * kTaps + tap) * kCC + ci]);
+  }
+}
+
+// ------------------------------------------------------------------ input staging
+// grid (B * 8 tiles, active), 128 threads: one pixel each; the image row of
+// sample b is (start[lane] + s * B + b) mod n[lane] of the lane's shard
+// (fp32 NHWC, Cin channels); channels >= Cin are zero
+__global__ void __launch_bounds__(kCT) cnn_stage_kernel(const __grid_constant__ CnnStageArgs a) {
+  const int tile = blockIdx.x, e = blockIdx.y;
+  const int lane = a.wid[e];
+  const int b = tile / kTilesPerImg, pix = (tile % kTilesPerImg) * kTilePix + threadIdx.x;
+  const int64_t n = a.n[lane];
+  const int64_t row = (a.start[lane] + static_cast<int64_t>(a.step) * a.B + b) % n;
+  const float* src = a.x[lane] + row * static_cast<int64_t>(kPix) * a.Cin + static_cast<int64_t>(pix) * a.Cin;
+  float v[kCC];
+#pragma unroll
+  for (int c = 0; c < kCC; ++c) v[c] = c < a.Cin ? src[c] : 0.f;
+  __nv_bfloat16* dst = a.out + ((static_cast<int64_t>(lane) * a.B + b) * kPix + pix) * kCC;
+#pragma unroll
+  for (int q = 0; q < kCC / 8; ++q)
+    *reinterpret_cast<uint4*>(dst + 8 * q) =
+        make_uint4(pack_bf16x2(v[8 * q], v[8 * q + 1]), pack_bf16x2(v[8 * q + 2], v[8 * q + 3]),
+                   pack_bf16x2(v[8 * q + 4], v[8 * q + 5]), pack_bf16x2(v[8 * q + 6], v[8 * q + 7]));
+  if (a.labels && tile == 0 && threadIdx.x < 1) {
+    for (int bb = 0; bb < a.B; ++bb) {
+      const int64_t rr = (a.start[lane] + static_cast<int64_t>(a.step) * a.B + bb) % n;
+      a.labels[static_cast<int64_t>(lane) * a.B + bb] = a.y[lane][rr];
+    }
+  }
+}
+
+// ------------------------------------------------------------------ pooling
+// grid (B, active), 256 threads: g[lane][b][c] = sum over the 1024 pixels / 1024
+__global__ void __launch_bounds__(256) cnn_pool_kernel(const __nv_bfloat16* v, const int* wid, int B, float* g) {
+  __shared__ float part[4][kCC];
+  const int b = blockIdx.x, lane = wid[blockIdx.y];
+  const int c = threadIdx.x % kCC, grp = threadIdx.x / kCC;
+  const __nv_bfloat16* src = v + (static_cast<int64_t>(lane) * B + b) * kPix * kCC;
+  float s = 0.f;
+  for (int p = grp; p < kPix; p += 4) s += __bfloat162float(src[static_cast<int64_t>(p) * kCC + c]);
+  part[grp][c] = s;
+  __syncthreads();
+  if (threadIdx.x < kCC)
+    g[(static_cast<int64_t>(lane) * B + b) * kCC + threadIdx.x] =
+        (((part[0][threadIdx.x] + part[1][threadIdx.x]) + part[2][threadIdx.x]) + part[3][threadIdx.x]) /
+        static_cast<float>(kPix);
+}
+
+// ------------------------------------------------------------------ head: FC, softmax CE, backward, SGD of the FC
+// grid (active), 256 threads; B <= 256, K <= 32
+__global__ void __launch_bounds__(256) cnn_head_kernel(const __grid_constant__ CnnHeadArgs a) {
+  extern __shared__ float hsm[];
+  const int K = a.K, B = a.B;
+  float* gb = hsm;                    // [B][64] bf16-rounded pooled features
+  float* wf = gb + B * kCC;           // [K][64] bf16-rounded head weights
+  float* wm = wf + K * kCC;           // [K][64] fp32 master
+  float* dl = wm + K * kCC;           // [B][K] fp32 logit gradient
+  float* dlb = dl + B * K;            // [B][K] bf16-rounded
+  float* rl = dlb + B * K;            // [B] per-sample loss
+  float* bfm = rl + B;                // [32]
+  const int e = blockIdx.x, lane = a.wid[e], src = a.src[e];
+  const int t = threadIdx.x;
+  const int64_t so = static_cast<int64_t>(src) * a.slot_stride, dof = static_cast<int64_t>(lane) * a.slot_stride;
+  for (int q = t; q < B * kCC; q += 256) gb[q] = bf16_round(a.g[static_cast<int64_t>(lane) * B * kCC + q]);
+  for (int q = t; q < K * kCC; q += 256) {
+    const float m = a.master[so + a.offWf + q];
+    wm[q] = m;
+    wf[q] = bf16_round(m);
+  }
+  if (t < K) bfm[t] = a.master[so + a.offBf + t];
+  __syncthreads();
+  for (int b = t; b < B; b += 256) {
+    const int y = a.labels[static_cast<int64_t>(lane) * B + b];
+    float z[32];
+    float mx = -INFINITY, zy = 0.f;
+    for (int k = 0; k < K; ++k) {
+      float acc = 0.f;
+      for (int c = 0; c < kCC; ++c) acc = fmaf(gb[b * kCC + c], wf[k * kCC + c], acc);
+      z[k] = acc + bfm[k];
+      if (k == y) zy = z[k];
+      mx = fmaxf(mx, z[k]);
+    }
+    float se = 0.f, so_ = 0.f;
+    for (int k = 0; k < K; ++k) {
+      const float ev = expf(z[k] - mx);
+      z[k] = ev;
+      se += ev;
+      if (k != y) so_ += ev;
+    }
+    rl[b] = mx + logf(se) - zy;
+    const float inv = 1.0f / static_cast<float>(B);
+    for (int k = 0; k < K; ++k) {
+      const float gk = (k == y ? -(so_ / se) : z[k] / se) * inv;
+      dl[b * K + k] = gk;
+      dlb[b * K + k] = bf16_round(gk);
+    }
+  }
+  __syncthreads();
+  if (a.loss_part && t < (B + kRowsPerLossChunk - 1) / kRowsPerLossChunk) {
+    float l = 0.f;
+    for (int r = t * kRowsPerLossChunk; r < min(B, (t + 1) * kRowsPerLossChunk); ++r) l += rl[r];
+    a.loss_part[(static_cast<int64_t>(lane) * a.max_tau + a.step) * a.n_loss_chunks + t] = l;
+  }
+  // dg[b][c] = sum_k dlb[b][k] wf[k][c] (old weights)
+  for (int q = t; q < B * kCC; q += 256) {
+    const int b = q / kCC, c = q % kCC;
+    float acc = 0.f;
+    for (int k = 0; k < K; ++k) acc = fmaf(dlb[b * K + k], wf[k * kCC + c], acc);
+    a.dg[static_cast<int64_t>(lane) * B * kCC + q] = acc;
+  }
+  // head weights and bias
+  for (int q = t; q < K * kCC; q += 256) {
+    const int k = q / kCC, c = q % kCC;
+    float acc = 0.f;
+    for (int b = 0; b < B; ++b) acc = fmaf(dlb[b * K + k], gb[b * kCC + c], acc);
+    const float nw = fmaf(-a.lr, acc, wm[q]);
+    a.master_w[dof + a.offWf + q] = nw;
+    a.shadow[dof + a.offWf + q] = __float2bfloat16_rn(nw);
+  }
+  if (t < K) {
+    float acc = 0.f;
+    for (int b = 0; b < B; ++b) acc += dl[b * K + t];
+    const float nb = fmaf(-a.lr, acc, bfm[t]);
+    a.master_w[dof + a.offBf + t] = nb;
+    a.shadow[dof + a.offBf + t] = __float2bfloat16_rn(nb);
+  }
+}
+
+// loss of the global model on labelled pooled features (evaluation): grid 1, 256 threads
+__global__ void __launch_bounds__(256) cnn_head_loss_kernel(const float* g, const int32_t* labels, int B, int K,
+                                                            const float* master, int64_t offWf, int64_t offBf,
+                                                            float* out) {
+  __shared__ float wf[32 * kCC];
+  __shared__ float bfm[32];
+  __shared__ float rl[256];
+  const int t = threadIdx.x;
+  for (int q = t; q < K * kCC; q += 256) wf[q] = bf16_round(master[offWf + q]);
+  if (t < K) bfm[t] = master[offBf + t];
+  __syncthreads();
+  float l = 0.f;
+  for (int b = t; b < B; b += 256) {
+    float z[32], mx = -INFINITY;
+    for (int k = 0; k < K; ++k) {
+      float acc = 0.f;
+      for (int c = 0; c < kCC; ++c) acc = fmaf(bf16_round(g[static_cast<int64_t>(b) * kCC + c]), wf[k * kCC + c], acc);
+      z[k] = acc + bfm[k];
+      mx = fmaxf(mx, z[k]);
+    }
+    float se = 0.f;
+    for (int k = 0; k < K; ++k) se += expf(z[k] - mx);
+    l += mx + logf(se) - z[labels[b]];
+  }
+  rl[t] = l;
+  __syncthreads();
+  if (t == 0) {
+    float s = 0.f;
+    for (int i = 0; i < 256; ++i) s += rl[i];
+    out[0] = s;
+  }
+}
+
+// ------------------------------------------------------------------ output gradient of the last block
+// grid (B * 8 tiles, active), 128 threads (pixel): dz = v > 0 ? dg / 1024 : 0,
+// bf16, and per-tile channel sums of the fp32 values
+__global__ void __launch_bounds__(kCT) cnn_dzb_kernel(const __nv_bfloat16* v, const float* dg, const int* wid, int B,
+                                                      __nv_bfloat16* dz, float* bias_part) {
+  __shared__ float T[kTilePix][kCC + 1];
+  const int tile = blockIdx.x, lane = wid[blockIdx.y];
+  const int b = tile / kTilesPerImg, pix = (tile % kTilesPerImg) * kTilePix + threadIdx.x;
+  const int64_t base = ((static_cast<int64_t>(lane) * B + b) * kPix + pix) * kCC;
+  const float* d = dg + (static_cast<int64_t>(lane) * B + b) * kCC;
+  float o[kCC];
+#pragma unroll
+  for (int q = 0; q < kCC / 8; ++q) {
+    const uint4 r = *reinterpret_cast<const uint4*>(v + base + 8 * q);
+    const __nv_bfloat162* r2 = reinterpret_cast<const __nv_bfloat162*>(&r);
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const float2 f = __bfloat1622float2(r2[j]);
+      const int c = 8 * q + 2 * j;
+      o[c] = f.x > 0.f ? d[c] / static_cast<float>(kPix) : 0.f;
+      o[c + 1] = f.y > 0.f ? d[c + 1] / static_cast<float>(kPix) : 0.f;
+    }
+  }
+#pragma unroll
+  for (int q = 0; q < kCC / 8; ++q)
+    *reinterpret_cast<uint4*>(dz + base + 8 * q) =
+        make_uint4(pack_bf16x2(o[8 * q], o[8 * q + 1]), pack_bf16x2(o[8 * q + 2], o[8 * q + 3]),
+                   pack_bf16x2(o[8 * q + 4], o[8 * q + 5]), pack_bf16x2(o[8 * q + 6], o[8 * q + 7]));
+#pragma unroll
+  for (int c = 0; c < kCC; ++c) T[threadIdx.x][c] = o[c];
+  __syncthreads();
+  if (threadIdx.x < kCC) {
+    float s = 0.f;
+    for (int q = 0; q < kTilePix; ++q) s += T[q][threadIdx.x];
+    bias_part[(static_cast<int64_t>(lane) * B * kTilesPerImg + tile) * kCC + threadIdx.x] = s;
+  }
+}
+
+}  // namespace
+
+// ------------------------------------------------------------------ launchers
+int cnn_tiles_per_image() { return kTilesPerImg; }
+int cnn_wgrad_chunks(int B) { return (B + kWgradImagesPerChunk - 1) / kWgradImagesPerChunk; }
+
+cudaError_t launch_conv_igemm(int mode, const CUtensorMap& mIn, const CUtensorMap& mW, const ConvArgs& a, int n_active,
+                              cudaStream_t s) {
+  const dim3 grid(a.B * kTilesPerImg, n_active);
+  if (mode == 0) {
+    cudaError_t e = cudaFuncSetAttribute(conv_igemm_kernel<0>, cudaFuncAttributeMaxDynamicSharedMemorySize, kCSmem);
+    if (e != cudaSuccess) return e;
+    conv_igemm_kernel<0><<<grid, kCT, kCSmem, s>>>(mIn, mW, a);
+  } else {
+    cudaError_t e = cudaFuncSetAttribute(conv_igemm_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, kCSmem);
+    if (e != cudaSuccess) return e;
+    conv_igemm_kernel<1><<<grid, kCT, kCSmem, s>>>(mIn, mW, a);
+  }
+  return cudaGetLastError();
+}
+
+cudaError_t launch_conv_wgrad(const CUtensorMap& mIn, const CUtensorMap& mDz, const WgradArgs& a, int n_active,
+                              cudaStream_t s) {
+  cudaError_t e = cudaFuncSetAttribute(conv_wgrad_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kWSmem);
+  if (e != cudaSuccess) return e;
+  conv_wgrad_kernel<<<dim3(a.n_chunks, n_active), kWT, kWSmem, s>>>(mIn, mDz, a);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_conv_sgd(const ConvSgdArgs& a, int n_active, cudaStream_t s) {
+  conv_sgd_kernel<<<dim3(kTaps, n_active), 256, 0, s>>>(a);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_conv_refresh_wt(const float* master, __nv_bfloat16* wt, int64_t offW, cudaStream_t s) {
+  conv_refresh_wt_kernel<<<kTaps, 256, 0, s>>>(master, wt, offW);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_cnn_stage(const CnnStageArgs& a, int n_active, cudaStream_t s) {
+  cnn_stage_kernel<<<dim3(a.B * kTilesPerImg, n_active), kCT, 0, s>>>(a);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_cnn_pool(const __nv_bfloat16* v, const int* wid, int B, float* g, int n_active, cudaStream_t s) {
+  cnn_pool_kernel<<<dim3(B, n_active), 256, 0, s>>>(v, wid, B, g);
+  return cudaGetLastError();
+}
+
+size_t cnn_head_smem(int B, int K) { return sizeof(float) * (static_cast<size_t>(B) * kCC + 2 * K * kCC + 2 * B * K + B + 32); }
+
+cudaError_t launch_cnn_head(const CnnHeadArgs& a, int n_active, cudaStream_t s) {
+  const size_t smem = cnn_head_smem(a.B, a.K);
+  cudaError_t e = cudaFuncSetAttribute(cnn_head_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, static_cast<int>(smem));
+  if (e != cudaSuccess) return e;
+  cnn_head_kernel<<<n_active, 256, smem, s>>>(a);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_cnn_head_loss(const float* g, const int32_t* labels, int B, int K, const float* master,
+                                 int64_t offWf, int64_t offBf, float* out, cudaStream_t s) {
+  cnn_head_loss_kernel<<<1, 256, 0, s>>>(g, labels, B, K, master, offWf, offBf, out);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_cnn_dzb(const __nv_bfloat16* v, const float* dg, const int* wid, int B, __nv_bfloat16* dz,
+                           float* bias_part, int n_active, cudaStream_t s) {
+  cnn_dzb_kernel<<<dim3(B * kTilesPerImg, n_active), kCT, 0, s>>>(v, dg, wid, B, dz, bias_part);
+  return cudaGetLastError();
+}
+
+}  // namespace oscars

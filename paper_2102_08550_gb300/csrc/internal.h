@@ -186,4 +186,80 @@ cudaError_t launch_transpose_bf16(const __nv_bfloat16* src, __nv_bfloat16* dst, 
 cudaError_t launch_broadcast(const float* xg, float* slab, int64_t stride, int W, int64_t count,
                              cudaStream_t s);
 
+// ---------------------------------------------------------------- convolutional worker
+// 32 x 32 images, 64 channels, 3x3 convolutions (csrc/cnn.cu)
+constexpr int kWgradImagesPerChunk = 2;   // images per split-K chunk of the weight gradient
+
+struct ConvArgs {
+  const int* wid;              // [n_active] lane of each active entry
+  const int* src;              // [n_active] slot whose weights the step reads
+  int B;                       // images per lane
+  const float* bias;           // forward: fp32 slab; bias of slot s at bias + s * slot_stride + off_bias
+  int64_t slot_stride, off_bias;
+  const __nv_bfloat16* add;    // [lane][B][1024][64] added before the activation / mask, or null
+  const __nv_bfloat16* mask;   // input gradient: stored activation of the layer input (> 0 keeps)
+  __nv_bfloat16* out;          // [lane][B][1024][64]
+  float* bias_part;            // input gradient: [lane][B * 8][64] per-tile channel sums, or null
+  int* err;
+};
+struct WgradArgs {
+  const int* wid;
+  int B, n_chunks, img_per_chunk;
+  float* part;                 // [lane][n_chunks][9][64 in][64 out]
+  int* err;
+};
+struct ConvSgdArgs {
+  const int* wid;
+  const int* src;
+  int n_chunks, n_tiles;
+  const float* part;           // as WgradArgs::part
+  const float* bias_part;      // [lane][n_tiles][64]
+  const float* master;
+  float* master_w;
+  __nv_bfloat16* shadow;
+  __nv_bfloat16* wt;           // transposed bf16 copy of this layer in slot 0, or null
+  int64_t slot_stride, offW, offB, wt_slot_stride;
+  float lr;
+};
+struct CnnStageArgs {
+  const float* const* x;       // [W] fp32 NHWC shards
+  const int32_t* const* y;
+  const int64_t* n;
+  const int64_t* start;        // [W] cursors
+  const int* wid;
+  int step, B, Cin;
+  __nv_bfloat16* out;          // [lane][B][1024][64]
+  int32_t* labels;             // [lane][B] or null
+};
+struct CnnHeadArgs {
+  const int* wid;
+  const int* src;
+  int B, K, step, max_tau, n_loss_chunks;
+  const float* g;              // [lane][B][64]
+  const int32_t* labels;       // [lane][B]
+  float* dg;                   // [lane][B][64]
+  float* loss_part;            // [(lane * max_tau + step) * n_loss_chunks + chunk]
+  const float* master;
+  float* master_w;
+  __nv_bfloat16* shadow;
+  int64_t slot_stride, offWf, offBf;
+  float lr;
+};
+int cnn_tiles_per_image();
+int cnn_wgrad_chunks(int B);
+cudaError_t launch_conv_igemm(int mode, const CUtensorMap& mIn, const CUtensorMap& mW, const ConvArgs& a, int n_active,
+                              cudaStream_t s);
+cudaError_t launch_conv_wgrad(const CUtensorMap& mIn, const CUtensorMap& mDz, const WgradArgs& a, int n_active,
+                              cudaStream_t s);
+cudaError_t launch_conv_sgd(const ConvSgdArgs& a, int n_active, cudaStream_t s);
+cudaError_t launch_conv_refresh_wt(const float* master, __nv_bfloat16* wt, int64_t offW, cudaStream_t s);
+cudaError_t launch_cnn_stage(const CnnStageArgs& a, int n_active, cudaStream_t s);
+cudaError_t launch_cnn_pool(const __nv_bfloat16* v, const int* wid, int B, float* g, int n_active, cudaStream_t s);
+size_t cnn_head_smem(int B, int K);
+cudaError_t launch_cnn_head(const CnnHeadArgs& a, int n_active, cudaStream_t s);
+cudaError_t launch_cnn_head_loss(const float* g, const int32_t* labels, int B, int K, const float* master,
+                                 int64_t offWf, int64_t offBf, float* out, cudaStream_t s);
+cudaError_t launch_cnn_dzb(const __nv_bfloat16* v, const float* dg, const int* wid, int B, __nv_bfloat16* dz,
+                           float* bias_part, int n_active, cudaStream_t s);
+
 }  // namespace oscars

@@ -175,6 +175,37 @@ class TrainWorkload:
 
 
 @dataclass
+class ConvWorkload(TrainWorkload):
+    """A local-SGD workload with the convolutional worker: CIFAR-shaped
+    images (height x width x in_ch, NHWC, flattened as the data vector),
+    a stem, ``blocks`` residual blocks of ``ch`` channels, pooling and a
+    linear head.  ``dims`` is [height * width * in_ch, classes] (the data
+    generator's view)."""
+    height: int = 32
+    width: int = 32
+    in_ch: int = 3
+    ch: int = 64
+    blocks: int = 1
+
+    @property
+    def cnn_dims(self) -> List[int]:
+        return [self.height, self.width, self.in_ch, self.ch, self.dims[-1]]
+
+    @property
+    def num_params(self) -> int:
+        C, K = self.ch, self.dims[-1]
+        return C * 9 * self.in_ch + C + self.blocks * 2 * (C * 9 * C + C) + K * C + K
+
+    def flops_per_sample(self) -> float:
+        """Multiply-adds x2 of the convolutions (forward, weight gradient, and
+        the input gradient of the block convolutions) and the head."""
+        hw, C, K = self.height * self.width, self.ch, self.dims[-1]
+        stem = 2 * hw * C * 9 * self.in_ch
+        block = 2 * hw * C * 9 * C
+        return float(2 * stem + self.blocks * 2 * 3 * block + 3 * 2 * C * K)
+
+
+@dataclass
 class MergeWorkload:
     """A server-merge microbench: W pushed deltas of P fp32 parameters."""
     name: str
@@ -195,7 +226,9 @@ CFG3 = TrainWorkload("mlp-3072-1024-1024-10-W32", 32, [3072, 1024, 1024, 10], 12
 CFG4 = MergeWorkload("merge-P25.6M-W64", 64, 25_600_000, 1e-3, 8, "localsteps")
 CFG5 = MergeWorkload("merge-P340M-W8", 8, 340_000_000, 1e-3, 16, "uniform")
 
-WORKLOADS = {"cfg1": CFG1, "cfg2": CFG2, "cfg3": CFG3, "cfg4": CFG4, "cfg5": CFG5}
+CFG6 = ConvWorkload("resnet-mini-c64-W16", 16, [32 * 32 * 3, 10], 32, 0.05, 2048, 16, 20, clip=3.0)
+
+WORKLOADS = {"cfg1": CFG1, "cfg2": CFG2, "cfg3": CFG3, "cfg4": CFG4, "cfg5": CFG5, "cfg6": CFG6}
 
 
 def speeds(w: TrainWorkload) -> np.ndarray:
@@ -253,6 +286,27 @@ def init_layers_np(w: TrainWorkload) -> List[Tuple[np.ndarray, np.ndarray]]:
         a = np.float32(1.0 / math.sqrt(i))
         W = ((u * np.float32(2.0) - np.float32(1.0)) * a).astype(np.float32).reshape(o, i)
         out.append((W, np.zeros(o, dtype=np.float32)))
+    return out
+
+
+def init_cnn_np(w: "ConvWorkload") -> List[np.ndarray]:
+    """Initial convolutional model in canonical order: weights
+    U(-1/sqrt(fan_in), 1/sqrt(fan_in)) (fan_in = 9 Cin for a 3x3 convolution,
+    C for the head), biases 0."""
+    rng = np.random.default_rng(w.seed + SEED_INIT)
+    C, K = w.ch, w.dims[-1]
+    shapes = [(C, 3, 3, w.in_ch), (C,)]
+    for _ in range(w.blocks):
+        shapes += [(C, 3, 3, C), (C,), (C, 3, 3, C), (C,)]
+    shapes += [(K, C), (K,)]
+    out = []
+    for s in shapes:
+        if len(s) == 1:
+            out.append(np.zeros(s, np.float32))
+        else:
+            fan_in = int(np.prod(s[1:]))
+            lim = 1.0 / np.sqrt(fan_in)
+            out.append(rng.uniform(-lim, lim, size=s).astype(np.float32))
     return out
 
 

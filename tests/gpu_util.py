@@ -70,7 +70,7 @@ def oracle_schedule(w: synth.TrainWorkload):
 
 # ---------------------------------------------------------------- conditioning envelope
 class perturbed_gemms:
-    """Context manager: every GEMM output of the oracle is multiplied by
+    """Context manager: every GEMM (and convolution) output of the oracle is multiplied by
     (1 + rel * N(0, 1)), the size of the difference a different fp32
     summation order makes.  Used to measure how far the oracle moves from
     itself, i.e. how well conditioned a run is (test infrastructure only)."""
@@ -79,8 +79,10 @@ class perturbed_gemms:
         self.rel, self.rng = rel, np.random.default_rng(seed)
 
     def __enter__(self):
+        from oracle import conv as oc
         from oracle import model as om
         self.om, self.nt, self.nn = om, om.gemm_nt, om.gemm_nn
+        self.oc, self.convs = oc, (oc.conv3x3, oc.conv3x3_transposed, oc.conv3x3_weight_grad)
         rel, rng = self.rel, self.rng
 
         def wrap(f):
@@ -89,10 +91,12 @@ class perturbed_gemms:
                 return (out * (1.0 + rel * rng.standard_normal(out.shape))).astype(np.float32)
             return g
         om.gemm_nt, om.gemm_nn = wrap(self.nt), wrap(self.nn)
+        oc.conv3x3, oc.conv3x3_transposed, oc.conv3x3_weight_grad = (wrap(f) for f in self.convs)
         return self
 
     def __exit__(self, *a):
         self.om.gemm_nt, self.om.gemm_nn = self.nt, self.nn
+        self.oc.conv3x3, self.oc.conv3x3_transposed, self.oc.conv3x3_weight_grad = self.convs
 
 
 ENV_REL = 2e-6       # relative GEMM-output perturbation (about 30 fp32 ulps)
@@ -100,15 +104,19 @@ ENV_SEEDS = (11, 12)
 ENV_FACTOR = 4.0
 
 
-def envelope(run_fn, dims, ref_flats):
+def envelope(run_fn, dims, ref_flats, errors=None):
     """Per-round, per-tensor max divergence of perturbed oracle runs from the
-    unperturbed ones; ``run_fn()`` returns a list of flat parameter vectors."""
-    env = [np.zeros(2 * (len(dims) - 1)) for _ in ref_flats]
+    unperturbed ones; ``run_fn()`` returns a list of flat parameter vectors.
+    ``errors(flat, ref)`` gives the per-tensor errors (default: the MLP
+    layout of ``dims``)."""
+    errors = errors or (lambda f, ref: per_tensor_errors(f, ref, dims))
+    env = [None for _ in ref_flats]
     for s in ENV_SEEDS:
         with perturbed_gemms(ENV_REL, s):
             flats = run_fn()
         for r, (f, ref) in enumerate(zip(flats, ref_flats)):
-            env[r] = np.maximum(env[r], per_tensor_errors(f, ref, dims))
+            e = np.asarray(errors(f, ref))
+            env[r] = e if env[r] is None else np.maximum(env[r], e)
     return env
 
 

@@ -1,0 +1,114 @@
+"""The convolutional worker on the GPU against the oracle (oracle/conv.py):
+schedules exact, merged parameters per tensor within 1e-5 or the measured
+conditioning envelope of the oracle (bf16 rounding and ReLU masks amplify
+fp32 summation-order differences), worker losses and eval loss within 1e-3.
+
+Cases: small runs of one and two residual blocks through two rounds (the
+second round starts from the merged model), and the full-size workload
+(16 workers, batch 32) for one local step of two sampled workers."""
+import dataclasses
+
+import numpy as np
+import pytest
+import torch
+
+import paper_2102_08550_gb300 as P
+import synth
+from oracle import bf16 as obf16
+from oracle import conv as oconv
+from oracle import run as orun
+from tests.gpu_util import LOSS_RTOL, assert_within, envelope, oracle_schedule, per_tensor_errors
+
+pytestmark = pytest.mark.gpu
+
+
+def cnn_errors(m, got, ref):
+    """Per-tensor max-abs error / max-abs value (canonical order)."""
+    out = []
+    for g, r in zip(m.unflatten(got), m.unflatten(ref)):
+        den = np.abs(r).max()
+        out.append(float(np.abs(g.astype(np.float64) - r).max() / (den if den > 0 else 1.0)))
+    return out
+
+
+def make_cnn_context(w, device, rows, flags=0):
+    shards = [synth.shard_t(w, k, device, n=rows) for k in range(w.num_workers)]
+    params0 = synth.init_cnn_np(w)
+    m = oconv.CNN(w.height, w.width, w.in_ch, w.ch, w.blocks, w.dims[-1])
+    init = torch.from_numpy(m.flatten(params0)).to(device)
+    ctx = P.OscarsContext(num_workers=w.num_workers, dims=w.cnn_dims, model=P.MODEL_CNN, blocks=w.blocks,
+                          batch=w.batch, lr=w.lr, speed=synth.speeds(w).tolist(), M=w.M, shards=shards,
+                          init_params=init, stream=torch.cuda.current_stream().cuda_stream, flags=flags)
+    return ctx, m, params0
+
+
+def pull(ctx, device):
+    out = torch.empty(ctx.P, dtype=torch.float32, device=device)
+    ctx.pull(out)
+    torch.cuda.synchronize()
+    return out.cpu().numpy()
+
+
+SMALL = [("1block", 1, 3, 16), ("2blocks", 2, 2, 16)]
+
+
+@pytest.mark.parametrize("name,blocks,W,B", SMALL, ids=[s[0] for s in SMALL])
+def test_cnn_small_two_rounds(cuda_device, name, blocks, W, B):
+    rows = 4 * B
+    w = synth.ConvWorkload(f"cnn-{name}", W, [32 * 32 * 3, 10], B, 0.05, rows, 4, 2, clip=3.0, blocks=blocks)
+    ctx, m, params0 = make_cnn_context(w, cuda_device, rows)
+    rounds = 2
+    losses, flats = [], []
+    for _ in range(rounds):
+        tau, loss = ctx.local_steps()
+        ctx.push_merge()
+        losses.append(np.array(loss))
+        flats.append(pull(ctx, cuda_device))
+    Xe, ye = synth.eval_np(w, n=2 * B)
+    ge = ctx.eval_loss(torch.from_numpy(Xe).to(cuda_device), torch.from_numpy(ye).to(cuda_device))
+    sch = ctx.schedule()
+    ctx.close()
+    t, T, mw, tau_o = oracle_schedule(w)
+    assert sch["tau"] == tau_o.tolist() and sch["T_star"] == T
+    shards_h = [synth.shard_np(w, k, n=rows) for k in range(W)]
+
+    def oracle_run():
+        return orun.run(None, params0, shards_h, t_iter=t, M=w.M, rounds=rounds, batch=B, lr=w.lr,
+                        bf16=True, model=m)
+    state, recs = oracle_run()
+    env = envelope(lambda: [r.x_g for r in oracle_run()[1]], None, [r.x_g for r in recs],
+                   errors=lambda f, ref: cnn_errors(m, f, ref))
+    for r in range(rounds):
+        np.testing.assert_allclose(losses[r], recs[r].worker_loss, rtol=LOSS_RTOL)
+        errs = cnn_errors(m, flats[r], recs[r].x_g)
+        assert_within(errs, env[r], f"{name} round {r}")
+    oe = m.loss_of(state.x_g, Xe, ye, obf16.round_bf16)   # the model's own structure (state.x_g)
+    assert abs(ge - oe) <= LOSS_RTOL * abs(oe), (ge, oe)
+
+
+def test_cnn_full_size_one_step_sampled(cuda_device):
+    """The 16-worker, batch-32 workload: one local step per worker, the
+    replicas of the first and the last worker against the oracle."""
+    w = synth.CFG6
+    rows = 2 * w.batch
+    ctx, m, params0 = make_cnn_context(w, cuda_device, rows)
+    ctx.set_local_steps([1] * w.num_workers)
+    _, loss = ctx.local_steps()
+    t, _, _, _ = oracle_schedule(w)
+    for k in (0, w.num_workers - 1):
+        out = torch.empty(ctx.P, dtype=torch.float32, device=cuda_device)
+        ctx.read_replica(k, out)
+        torch.cuda.synchronize()
+        got = out.cpu().numpy()
+        Xk, yk = synth.shard_np(w, k, n=rows)
+
+        def worker_run():
+            state = orun.init_state(None, params0, t, w.M, tau_override=[1] * w.num_workers, model=m)
+            layers, l = orun.local_steps(state, k, (Xk, yk), w.batch, w.lr, obf16.round_bf16)
+            return m.flatten(layers), l
+        ref, lref = worker_run()
+        env = envelope(lambda: [worker_run()[0]], None, [ref], errors=lambda f, r: cnn_errors(m, f, r))[0]
+        assert_within(cnn_errors(m, got, ref), env, f"worker {k}")
+        assert abs(loss[k] - lref) <= LOSS_RTOL * abs(lref)
+    ctx.push_merge()
+    ctx.close()
