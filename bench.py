@@ -10,6 +10,7 @@ W=64 and P=340M, W=8) as GB/s and fraction of HBM bandwidth.
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl oscars|reference]
   python bench.py --compare [--compare-configs cfg1,cfg2,cfg3]
+  python bench.py --cnn [--steps K] [--warmup W]
 
 --impl reference times the CPU oracle (the plain numpy restatement of the
 method) on the same workload and metric.
@@ -53,6 +54,8 @@ def parse():
     ap.add_argument("--merge-reps", type=int, default=20)
     ap.add_argument("--only", choices=["all", "round", "merge"], default="all",
                     help="round: only the Oscars-round benchmark; merge: only the merge microbenchmarks")
+    ap.add_argument("--cnn", action="store_true",
+                    help="the convolutional worker workload (resnet-mini-c64-W16) instead of the MLP headline")
     ap.add_argument("--compare", action="store_true",
                     help="simulated time-to-loss comparison of Oscars, BSP and fixed-period local SGD")
     ap.add_argument("--compare-configs", default="cfg1,cfg2,cfg3")
@@ -546,6 +549,101 @@ def run_compare_drift(args, dev, key):
                       "target_loss": target, "policies": res}))
 
 
+def cnn_work(w, tau, tiles_per_image=8):
+    """Per-round algorithmic FLOPs of the convolutional worker by kernel class
+    (multiply-adds x2; the stem counts its real input channels)."""
+    n = float(np.sum(tau)) * w.batch            # samples per round
+    hw, C, K = w.height * w.width, w.ch, w.dims[-1]
+    block = 2.0 * hw * C * 9 * C
+    stem = 2.0 * hw * C * 9 * w.in_ch
+    return {"conv_fwd": n * (stem + 2 * w.blocks * block),
+            "conv_dgrad": n * 2 * w.blocks * block,
+            "conv_wgrad": n * (stem + 2 * w.blocks * block),
+            "cnn_head": n * 3 * 2 * C * K}
+
+
+def run_cnn(args, dev):
+    """Oscars rounds of the convolutional worker: samples/s with the tensor
+    roofline of its convolution kernels."""
+    import torch
+    import paper_2102_08550_gb300 as P
+    from oracle import schedule as S   # schedule inputs only; not timed
+    w = synth.CFG6
+    hbm, tf_burst, tf_sus, peak_kind = peaks()
+    t = S.iteration_ticks(synth.speeds(w), w.ticks_per_unit)
+    T_star, mw, tau = S.schedule(t, w.M)
+    samples_per_round = int(np.sum(tau)) * w.batch
+    shards = [synth.shard_t(w, k, dev) for k in range(w.num_workers)]
+    from oracle import conv as oconv
+    m = oconv.CNN(w.height, w.width, w.in_ch, w.ch, w.blocks, w.dims[-1])
+    init = torch.from_numpy(m.flatten(synth.init_cnn_np(w))).to(dev)
+    stream = torch.cuda.current_stream(dev)
+
+    def make(flags=0):
+        return P.OscarsContext(num_workers=w.num_workers, dims=w.cnn_dims, model=P.MODEL_CNN, blocks=w.blocks,
+                               batch=w.batch, lr=w.lr, speed=synth.speeds(w).tolist(), M=w.M, shards=shards,
+                               init_params=init, stream=stream.cuda_stream, flags=flags)
+    ctx = make()
+    flush = torch.empty(512 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)
+    for _ in range(args.warmup):
+        P.oscars_local_steps(ctx.handle, want_tau=False, want_loss=False)
+        P.oscars_push_merge(ctx.handle)
+    torch.cuda.synchronize()
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    with ClockSampler(0) as clk:
+        for i in range(args.steps):
+            flush.fill_(float(i))
+            evs[i][0].record(stream)
+            P.oscars_local_steps(ctx.handle, want_tau=False, want_loss=False)
+            P.oscars_push_merge(ctx.handle)
+            evs[i][1].record(stream)
+        torch.cuda.synchronize()
+    total_ms = sum(a.elapsed_time(b) for a, b in evs)
+    _, loss = P.oscars_local_steps(ctx.handle, want_tau=False, want_loss=True)
+    P.oscars_push_merge(ctx.handle)
+    ctx.close()
+    # per-kernel-class device time
+    pctx = make(flags=P.FLAG_PROFILE)
+    P.oscars_local_steps(pctx.handle, want_tau=False, want_loss=False)
+    P.oscars_push_merge(pctx.handle)
+    torch.cuda.synchronize()
+    pctx.profile_reset()
+    prof_rounds = 3
+    for i in range(prof_rounds):
+        flush.fill_(float(i))
+        P.oscars_local_steps(pctx.handle, want_tau=False, want_loss=False)
+        P.oscars_push_merge(pctx.handle)
+    prof = pctx.profile()
+    torch.cuda.synchronize()
+    pctx.close()
+    work = cnn_work(w, tau)
+    kernels = {}
+    for name, (ms, cnt) in prof.items():
+        per_round = ms / prof_rounds
+        k = {"ms_per_round": per_round, "launches_per_round": cnt / prof_rounds}
+        if name in work:
+            k["tflops"] = work[name] / (per_round / 1e3) / 1e12
+            k["frac"] = k["tflops"] / tf_sus
+        kernels[name] = k
+    conv_ms = sum(kernels[k]["ms_per_round"] for k in ("conv_fwd", "conv_dgrad", "conv_wgrad") if k in kernels)
+    conv_fl = sum(work[k] for k in ("conv_fwd", "conv_dgrad", "conv_wgrad"))
+    ach = conv_fl / (conv_ms / 1e3) / 1e12
+    line = {"metric": "simulated-worker samples/s (Oscars rounds, convolutional worker)",
+            "value": samples_per_round * args.steps / (total_ms / 1e3), "unit": "samples/s", "n_gpus": 1,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": total_ms / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "bf16 (fp32 master, fp32 accumulate)", "data": "synthetic (seeded CIFAR-shaped Gaussian mixture)",
+            "config": {"workload": f"{w.name} (W={w.num_workers}, 32x32x3 images, stem + {w.blocks} residual block(s) "
+                                   f"of 64 channels, batch={w.batch}, M={w.M})", "l2": "flushed between timed rounds"},
+            "roofline": {"kernel": "conv_fwd + conv_dgrad + conv_wgrad", "bound": "tensor", "achieved": ach,
+                         "peak": tf_sus, "unit": "TFLOP/s", "frac": ach / tf_sus,
+                         "peak_kind": f"{peak_kind} bf16 dense (sustained)", "flops_per_round": conv_fl,
+                         "traffic": None},
+            "kernels": kernels, "samples_per_round": samples_per_round, "T_star": int(T_star),
+            "tau": [int(v) for v in tau], "clocks": clk.summary(), "last_loss": [float(v) for v in loss]}
+    print(json.dumps(line))
+
+
 def run_reference(args):
     w = WORKLOAD
     oracle_rounds(w, max(1, min(args.warmup, 2)), 30.0)          # warm-up (imports, caches)
@@ -574,6 +672,15 @@ def main():
         import torch
         torch.cuda.set_device(local_rank)
         torch.distributed.init_process_group("nccl")
+    if args.cnn:
+        import torch
+        from paper_2102_08550_gb300 import _build
+        _build.build()
+        dev = torch.device(f"cuda:{local_rank}")
+        torch.cuda.set_device(dev)
+        if rank == 0:
+            run_cnn(args, dev)
+        return
     if args.compare:
         import torch
         from paper_2102_08550_gb300 import _build

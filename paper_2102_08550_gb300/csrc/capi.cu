@@ -802,26 +802,27 @@ cudaError_t enqueue_step_cnn(oscars_ctx* c, int s, int na, const int* wid, const
   if ((e = wgrad(0, X, cur)) != cudaSuccess) return e;
   // SGD of every convolution layer (after all input gradients used the old weights)
   ProfScope ps(c, "conv_sgd", st);
+  ConvSgdArgs a;
+  std::memset(&a, 0, sizeof(a));
+  a.wid = wid;
+  a.src = src;
+  a.n_chunks = c->cnn_chunks;
+  a.n_tiles = tiles;
+  a.layers = layers;
   for (int l = 0; l < layers; ++l) {
-    ConvSgdArgs a;
-    a.wid = wid;
-    a.src = src;
-    a.n_chunks = c->cnn_chunks;
-    a.n_tiles = tiles;
-    a.part = c->cnn_wpart + l * wpl;
-    a.bias_part = c->cnn_bpart + l * bpl;
-    a.master = c->slab;
-    a.master_w = c->slab;
-    a.shadow = c->shadow;
-    a.wt = l >= 1 ? c->cnn_wt + static_cast<int64_t>(l - 1) * 9 * 64 * 64 : nullptr;
-    a.slot_stride = c->P_pad;
-    a.offW = c->cnn_offW[l];
-    a.offB = c->cnn_offB[l];
-    a.wt_slot_stride = c->cnn_wt_slot;
-    a.lr = c->lr;
-    if ((e = launch_conv_sgd(a, na, st)) != cudaSuccess) return e;
+    a.part[l] = c->cnn_wpart + l * wpl;
+    a.bias_part[l] = c->cnn_bpart + l * bpl;
+    a.wt[l] = l >= 1 ? c->cnn_wt + static_cast<int64_t>(l - 1) * 9 * 64 * 64 : nullptr;
+    a.offW[l] = c->cnn_offW[l];
+    a.offB[l] = c->cnn_offB[l];
   }
-  return cudaSuccess;
+  a.master = c->slab;
+  a.master_w = c->slab;
+  a.shadow = c->shadow;
+  a.slot_stride = c->P_pad;
+  a.wt_slot_stride = c->cnn_wt_slot;
+  a.lr = c->lr;
+  return launch_conv_sgd(a, na, st);
 }
 
 cudaError_t enqueue_round_cnn(oscars_ctx* c, cudaStream_t st) {

@@ -294,42 +294,48 @@ __global__ void __launch_bounds__(kWT, 1) conv_wgrad_kernel(const __grid_constan
   }
 }
 
-// ------------------------------------------------------------------ reduce + SGD of a convolution layer
-// grid (taps, active workers), 256 threads: one tap's [64 in][64 out] tile
+// ------------------------------------------------------------------ reduce + SGD of the convolution layers
+// grid (taps * 4, active workers, layers), 256 threads: one tap's 16 in-channel
+// rows x 64 out-channels of one layer; the chunks are summed in chunk order
+constexpr int kSgdRows = 16;
 __global__ void __launch_bounds__(256) conv_sgd_kernel(const __grid_constant__ ConvSgdArgs a) {
-  __shared__ float T[kCC][kCC + 1];   // [in][out]
-  const int tap = blockIdx.x, e = blockIdx.y;
+  __shared__ float T[kSgdRows][kCC + 1];   // [in][out]
+  const int tap = blockIdx.x / (kCC / kSgdRows), r0 = (blockIdx.x % (kCC / kSgdRows)) * kSgdRows;
+  const int e = blockIdx.y, layer = blockIdx.z;
   const int lane = a.wid[e], src = a.src[e];
   const int t = threadIdx.x;
-  // sum of the chunks in chunk order; thread -> (in = t / 4 + 64 k / ..., out) with out fastest
-  for (int q = t; q < kCC * kCC; q += 256) {
-    const int ci = q / kCC, co = q % kCC;
+  const float* part = a.part[layer] + (static_cast<int64_t>(lane) * a.n_chunks * kTaps + tap) * kCC * kCC + r0 * kCC;
+  const int64_t chunk_stride = static_cast<int64_t>(kTaps) * kCC * kCC;
+  for (int q = t; q < kSgdRows * kCC; q += 256) {
     float s = 0.f;
-    for (int c = 0; c < a.n_chunks; ++c)
-      s += a.part[((static_cast<int64_t>(lane) * a.n_chunks + c) * kTaps + tap) * kCC * kCC + q];
-    T[ci][co] = s;
+#pragma unroll 4
+    for (int c = 0; c < a.n_chunks; ++c) s += part[c * chunk_stride + q];
+    T[q / kCC][q % kCC] = s;
   }
   __syncthreads();
   const int64_t so = static_cast<int64_t>(src) * a.slot_stride, dof = static_cast<int64_t>(lane) * a.slot_stride;
+  const int64_t offW = a.offW[layer];
   // master / forward copy: [out][tap][in], in fastest
-  for (int q = t; q < kCC * kCC; q += 256) {
-    const int co = q / kCC, ci = q % kCC;
-    const int64_t off = a.offW + (static_cast<int64_t>(co) * kTaps + tap) * kCC + ci;
+  for (int q = t; q < kSgdRows * kCC; q += 256) {
+    const int co = q / kSgdRows, ci = q % kSgdRows;
+    const int64_t off = offW + (static_cast<int64_t>(co) * kTaps + tap) * kCC + r0 + ci;
     const float nw = fmaf(-a.lr, T[ci][co], a.master[so + off]);
     a.master_w[dof + off] = nw;
     a.shadow[dof + off] = __float2bfloat16_rn(nw);
     T[ci][co] = nw;   // in this loop every element is read and rewritten by one thread
   }
-  if (a.wt) {
+  if (a.wt[layer]) {
     __syncthreads();
     // transposed copy [tap][in][out], out fastest
-    __nv_bfloat16* wt = a.wt + static_cast<int64_t>(lane) * a.wt_slot_stride + static_cast<int64_t>(tap) * kCC * kCC;
-    for (int q = t; q < kCC * kCC; q += 256) wt[q] = __float2bfloat16_rn(T[q / kCC][q % kCC]);
+    __nv_bfloat16* wt = a.wt[layer] + static_cast<int64_t>(lane) * a.wt_slot_stride +
+                        (static_cast<int64_t>(tap) * kCC + r0) * kCC;
+    for (int q = t; q < kSgdRows * kCC; q += 256) wt[q] = __float2bfloat16_rn(T[q / kCC][q % kCC]);
   }
-  if (tap == 0 && t < kCC) {   // bias: per-tile sums in tile order
+  if (blockIdx.x == 0 && t < kCC) {   // bias: per-tile sums in tile order
+    const float* bp = a.bias_part[layer] + static_cast<int64_t>(lane) * a.n_tiles * kCC;
     float s = 0.f;
-    for (int i = 0; i < a.n_tiles; ++i) s += a.bias_part[(static_cast<int64_t>(lane) * a.n_tiles + i) * kCC + t];
-    a.master_w[dof + a.offB + t] = fmaf(-a.lr, s, a.master[so + a.offB + t]);
+    for (int i = 0; i < a.n_tiles; ++i) s += bp[static_cast<int64_t>(i) * kCC + t];
+    a.master_w[dof + a.offB[layer] + t] = fmaf(-a.lr, s, a.master[so + a.offB[layer] + t]);
   }
 }
 
@@ -569,7 +575,8 @@ cudaError_t launch_conv_wgrad(const CUtensorMap& mIn, const CUtensorMap& mDz, co
 }
 
 cudaError_t launch_conv_sgd(const ConvSgdArgs& a, int n_active, cudaStream_t s) {
-  conv_sgd_kernel<<<dim3(kTaps, n_active), 256, 0, s>>>(a);
+  if (a.layers < 1 || a.layers > kMaxConvLayers) return cudaErrorInvalidValue;
+  conv_sgd_kernel<<<dim3(kTaps * (kCC / kSgdRows), n_active, a.layers), 256, 0, s>>>(a);
   return cudaGetLastError();
 }
 

@@ -208,17 +208,19 @@ struct WgradArgs {
   float* part;                 // [lane][n_chunks][9][64 in][64 out]
   int* err;
 };
+constexpr int kMaxConvLayers = 9;
 struct ConvSgdArgs {
   const int* wid;
   const int* src;
-  int n_chunks, n_tiles;
-  const float* part;           // as WgradArgs::part
-  const float* bias_part;      // [lane][n_tiles][64]
+  int n_chunks, n_tiles, layers;
+  const float* part[kMaxConvLayers];       // per layer, as WgradArgs::part
+  const float* bias_part[kMaxConvLayers];  // per layer: [lane][n_tiles][64]
+  __nv_bfloat16* wt[kMaxConvLayers];       // per layer: transposed bf16 copy in slot 0, or null
+  int64_t offW[kMaxConvLayers], offB[kMaxConvLayers];
   const float* master;
   float* master_w;
   __nv_bfloat16* shadow;
-  __nv_bfloat16* wt;           // transposed bf16 copy of this layer in slot 0, or null
-  int64_t slot_stride, offW, offB, wt_slot_stride;
+  int64_t slot_stride, wt_slot_stride;
   float lr;
 };
 struct CnnStageArgs {
