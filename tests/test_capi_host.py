@@ -163,3 +163,40 @@ def test_train_rejects_null_context(oscars_lib):
 def test_set_iteration_ticks_null_context(oscars_lib):
     t = (ctypes.c_int64 * 2)(3, 5)
     assert oscars_lib.oscars_set_iteration_ticks(None, t) == P.OSCARS_EINVAL
+
+
+def _cnn_cfg(**kw):
+    cfg = P.OscarsConfig()
+    dims = kw.pop("dims", [32, 32, 3, 64, 10])
+    arr = (ctypes.c_int32 * len(dims))(*dims)
+    cfg.dims = arr
+    cfg.num_workers = kw.pop("W", 2)
+    cfg.model = P.MODEL_CNN
+    cfg.num_layers = kw.pop("blocks", 1)
+    cfg.batch = kw.pop("batch", 16)
+    cfg.lr = 0.05
+    cfg.server_lr = 1.0
+    cfg.bf16_gemm = kw.pop("bf16", 1)
+    cfg.M = 4
+    t = (ctypes.c_int64 * 2)(3, 5)
+    cfg.t_ticks = t
+    return cfg, (arr, t)
+
+
+@pytest.mark.parametrize("change, status", [
+    (dict(dims=[28, 28, 1, 64, 10]), P.OSCARS_ENOTSUP),    # image size
+    (dict(dims=[32, 32, 3, 32, 10]), P.OSCARS_ENOTSUP),    # channels
+    (dict(dims=[32, 32, 65, 64, 10]), P.OSCARS_ENOTSUP),   # input channels
+    (dict(dims=[32, 32, 3, 64, 40]), P.OSCARS_ENOTSUP),    # classes
+    (dict(blocks=0), P.OSCARS_ENOTSUP),
+    (dict(blocks=5), P.OSCARS_ENOTSUP),
+    (dict(batch=24), P.OSCARS_ENOTSUP),                     # not a multiple of 16
+    (dict(bf16=0), P.OSCARS_ENOTSUP),
+    (dict(dims=[32, 32, 0, 64, 10]), P.OSCARS_EINVAL),
+    (dict(), P.OSCARS_EINVAL),                              # valid shape but NULL shards
+])
+def test_cnn_create_rejects_before_device_work(oscars_lib, change, status):
+    cfg, keep = _cnn_cfg(**change)
+    h = ctypes.c_void_p()
+    assert oscars_lib.oscars_create(ctypes.byref(cfg), ctypes.byref(h)) == status
+    assert h.value is None
