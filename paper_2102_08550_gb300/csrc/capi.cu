@@ -167,7 +167,8 @@ struct oscars_ctx {
   int64_t cnn_wt_slot = 0;                   // elements per slot of the transposed copies
   __nv_bfloat16* cnn_wt = nullptr;           // [slot][2 * blocks][9][64 in][64 out]
   std::vector<__nv_bfloat16*> cnn_buf;       // x, s, (u_k, v_k) per block, dz0, dz1, dz2: [W][B][1024][64]
-  std::vector<CUtensorMap> cnn_m4, cnn_m2;   // per buffer: boxes of 4 and of 2 image rows
+  std::vector<CUtensorMap> cnn_m6, cnn_m2;   // per buffer: boxes of 6 and of 2 image rows
+  int sms = 0;                               // multiprocessors of the device
   std::vector<CUtensorMap> cnn_mw, cnn_mwt;  // weights per conv layer: forward layout, transposed (blocks)
   float* cnn_g = nullptr;                    // [W][B][64] pooled features
   float* cnn_dg = nullptr;                   // [W][B][64] their gradient
@@ -734,7 +735,8 @@ cudaError_t enqueue_step_cnn(oscars_ctx* c, int s, int na, const int* wid, const
     a.bias_part = bpart;
     a.err = c->err;
     ProfScope ps(c, mode == 0 ? "conv_fwd" : "conv_dgrad", st);
-    return launch_conv_igemm(mode, c->cnn_m4[in], mode == 0 ? c->cnn_mw[layer] : c->cnn_mwt[layer - 1], a, na, st);
+    return launch_conv_igemm(mode, c->cnn_m6[in], mode == 0 ? c->cnn_mw[layer] : c->cnn_mwt[layer - 1], a, na,
+                             conv_ctas_per_worker(B, na, c->sms), st);
   };
   auto wgrad = [&](int layer, int in, int dz) -> cudaError_t {
     WgradArgs a;
@@ -807,9 +809,12 @@ cudaError_t enqueue_step_cnn(oscars_ctx* c, int s, int na, const int* wid, const
   a.wid = wid;
   a.src = src;
   a.n_chunks = c->cnn_chunks;
-  a.n_tiles = tiles;
   a.layers = layers;
+  const int cpw = conv_ctas_per_worker(B, na, c->sms);
   for (int l = 0; l < layers; ++l) {
+    // the last block's b_b sums come from the output-gradient kernel (one per
+    // tile), all others from an input-gradient launch (one per CTA)
+    a.n_tiles[l] = l == layers - 1 ? tiles : cpw;
     a.part[l] = c->cnn_wpart + l * wpl;
     a.bias_part[l] = c->cnn_bpart + l * bpl;
     a.wt[l] = l >= 1 ? c->cnn_wt + static_cast<int64_t>(l - 1) * 9 * 64 * 64 : nullptr;
@@ -1010,14 +1015,19 @@ oscars_status allocate_cnn(oscars_ctx* c) {
       !dev_alloc(c, &c->cnn_bpart, static_cast<size_t>(layers) * W * tiles * 64))
     return fail(c, OSCARS_ENOMEM, "device allocation failed (gradients)");
   // tensor maps: activations {64 ch, 32 x, 32 y, images}; weights per slot
-  c->cnn_m4.resize(nbuf);
+  c->cnn_m6.resize(nbuf);
+  {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (cudaDeviceGetAttribute(&c->sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || c->sms < 1) c->sms = 1;
+  }
   c->cnn_m2.resize(nbuf);
   const uint64_t imgs = static_cast<uint64_t>(W) * B;
   bool ok = true;
   for (int i = 0; i < nbuf; ++i) {
     const uint64_t d[4] = {64, 32, 32, imgs};
     const uint64_t stv[3] = {64 * 2, 32 * 64 * 2, 1024 * 64 * 2};
-    ok &= make_map_box4(&c->cnn_m4[i], c->cnn_buf[i], d, stv, {64, 32, 4, 1});
+    ok &= make_map_box4(&c->cnn_m6[i], c->cnn_buf[i], d, stv, {64, 32, 6, 1});
     ok &= make_map_box4(&c->cnn_m2[i], c->cnn_buf[i], d, stv, {64, 32, 2, 1});
   }
   c->cnn_mw.resize(layers);
@@ -1551,7 +1561,8 @@ oscars_status oscars_eval_loss(oscars_ctx* c, const float* x, const int32_t* y, 
         ca.add = add >= 0 ? c->cnn_buf[add] : nullptr;
         ca.out = c->cnn_buf[out];
         ca.err = c->err;
-        return launch_conv_igemm(0, c->cnn_m4[in], c->cnn_mw[layer], ca, 1, c->stream);
+        return launch_conv_igemm(0, c->cnn_m6[in], c->cnn_mw[layer], ca, 1, conv_ctas_per_worker(Bc, 1, c->sms),
+                                 c->stream);
       };
       if (e == cudaSuccess) e = conv(0, 0, -1, 1);
       for (int k = 0; e == cudaSuccess && k < c->cnn_blocks; ++k) {

@@ -10,15 +10,17 @@
 // bf16 NHWC [lane][image][32][32][64]; a lane is one worker's batch.
 //
 // Kernels (all workers of a local step in one launch, grid y = active worker):
-//  * conv_igemm_kernel: implicit GEMM on tcgen05.  A CTA computes 128 output
-//    pixels (4 image rows) x 64 channels as the sum over the 9 taps of
-//    [128 pixels x 64 in-channels] x [64 x 64] products: per tap TMA loads
-//    the input box shifted by the tap offset (the zero padding is TMA's
-//    out-of-bounds fill) and the tap's weights.  Forward epilogue: bias,
-//    optional residual, ReLU, bf16.  Input-gradient mode: the box is shifted
-//    the other way and the weights are the transposed copy; epilogue: optional
-//    skip-path gradient, the ReLU mask of the layer input, bf16, and per-tile
-//    channel sums for the bias gradient.
+//  * conv_igemm_kernel: implicit GEMM on tcgen05.  An output tile is 128
+//    pixels (4 image rows) x 64 channels, the sum over the 9 taps of
+//    [128 pixels x 64 in-channels] x [64 x 64] products; the input boxes are
+//    loaded by TMA shifted by the tap offsets (the zero padding is TMA's
+//    out-of-bounds fill), one 6-row box per x-offset serving the three
+//    y-offsets, and a CTA keeps its worker's weights resident across its
+//    tiles.  Forward epilogue: bias, optional residual, ReLU, bf16.
+//    Input-gradient mode: the boxes are shifted the other way and the weights
+//    are the transposed copy; epilogue: optional skip-path gradient, the ReLU
+//    mask of the layer input, bf16, and per-CTA channel sums for the bias
+//    gradient.
 //  * conv_wgrad_kernel: dW[o][tap][i] = sum_p dz[p][o] x[p + off(tap)][i] on
 //    tcgen05 with both operands MN-major straight from the NHWC tensors: the
 //    K dimension is the pixels, taps are stacked in pairs to make M = 128
@@ -42,10 +44,7 @@ constexpr int kTilePix = kTileRows * kImg;  // 128
 constexpr int kTilesPerImg = kImg / kTileRows;
 constexpr int kTaps = 9;
 constexpr int kCT = 128;                    // threads of the implicit-GEMM and pixel kernels
-constexpr int kCStages = 4;
-constexpr int kCA = kTilePix * kCC * 2;     // 16 KB: 128 pixels x 64 channels
 constexpr int kCB = kCC * kCC * 2;          // 8 KB: one tap of the weights
-constexpr int kCSmem = kCStages * (kCA + kCB) + 256 + 1024;
 // weight gradient
 constexpr int kWT = 128;
 constexpr int kWStages = 2;
@@ -59,144 +58,205 @@ __device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
 }
 
 // ------------------------------------------------------------------ implicit GEMM (forward / input gradient)
+// A CTA works through tiles c, c + cpw, c + 2 cpw, ... of one worker (grid x
+// = c < cpw, grid y = active worker) with that worker's 9 weight taps resident
+// in shared memory.  Per tile and x-offset dx one TMA box of 6 image rows
+// (rows y0 - 1 .. y0 + 4, shifted by the x-offset) is loaded; the three
+// y-offsets are its 4-row sub-tiles at row offsets 0, 1, 2 (multiples of 8
+// pixel rows of 128 bytes, so the 128-byte swizzle phase is unchanged).  Two
+// TMEM accumulators: the epilogue of one tile overlaps the MMAs of the next.
+constexpr int kGT = 192;                    // warp 0 TMA, warp 1 MMA, warps 2-5 epilogue
+constexpr int kGSlots = 6;                  // input boxes in flight (two tiles)
+constexpr int kGBox = 6 * kImg * kCC * 2;   // 24 KB: 6 rows x 32 pixels x 64 channels
+constexpr int kGW = kTaps * kCB;            // 72 KB of resident weights
+constexpr int kGSmem = kGW + kGSlots * kGBox + 256 + 1024;
+static_assert(kTilePix * (kCC + 1) * 4 <= kGSlots * kGBox, "the bias reduction reuses the input slots");
+
 template <int MODE>   // 0 forward, 1 input gradient
-__global__ void __launch_bounds__(kCT) conv_igemm_kernel(const __grid_constant__ CUtensorMap mIn,
-                                                         const __grid_constant__ CUtensorMap mW,
-                                                         const __grid_constant__ ConvArgs a) {
+__global__ void __launch_bounds__(kGT, 1) conv_igemm_kernel(const __grid_constant__ CUtensorMap mIn,
+                                                            const __grid_constant__ CUtensorMap mW,
+                                                            const __grid_constant__ ConvArgs a) {
   extern __shared__ uint8_t cs_raw[];
   uint8_t* sm = align1024(cs_raw);
-  uint64_t* full = reinterpret_cast<uint64_t*>(sm + kCStages * (kCA + kCB));
-  uint64_t* empty = full + kCStages;
-  uint64_t* accb = empty + kCStages;
-  uint32_t* tslot = reinterpret_cast<uint32_t*>(accb + 1);
-  const int t = threadIdx.x, warp = t >> 5;
-  const int tile = blockIdx.x, e = blockIdx.y;
+  uint8_t* wts = sm;                 // [9][64][64] bf16, 128-byte swizzled K-major
+  uint8_t* slots = sm + kGW;         // [kGSlots][6 rows][32][64]
+  uint64_t* wfull = reinterpret_cast<uint64_t*>(slots + kGSlots * kGBox);
+  uint64_t* full = wfull + 1;
+  uint64_t* empty = full + kGSlots;
+  uint64_t* accf = empty + kGSlots;  // [2]
+  uint64_t* acce = accf + 2;         // [2] 128 arrivals
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(acce + 2);
+  const int t = threadIdx.x, warp = t >> 5, lane_id = t & 31;
+  const int c0 = blockIdx.x, cpw = gridDim.x, e = blockIdx.y;
   const int lane = a.wid[e], slot = a.src[e];
-  const int b = tile / kTilesPerImg, y0 = (tile % kTilesPerImg) * kTileRows;
-  const int img = lane * a.B + b;
+  const int ntiles = a.B * kTilesPerImg;
+  const int my_tiles = (ntiles - c0 + cpw - 1) / cpw;
   if (t == 0) {
     prefetch_tmap(&mIn);
     prefetch_tmap(&mW);
-    for (int i = 0; i < kCStages; ++i) {
+    mbar_init(wfull, 1);
+    for (int i = 0; i < kGSlots; ++i) {
       mbar_init(&full[i], 1);
       mbar_init(&empty[i], 1);
     }
-    mbar_init(accb, 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(&accf[i], 1);
+      mbar_init(&acce[i], 128);
+    }
     fence_barrier_init();
   }
   if (warp == 0) {
-    tmem_alloc(tslot, 64);
+    tmem_alloc(tslot, 128);
     tmem_relinquish();
   }
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tslot;
-  const int sgn = MODE == 0 ? 1 : -1;   // the input gradient reads the output gradient at p - off(tap)
+  constexpr int sgn = MODE == 0 ? 1 : -1;   // the input gradient reads the output gradient at p - off(tap)
   if (t == 0) {
+    mbar_arrive_expect_tx(wfull, kGW);
     for (int tap = 0; tap < kTaps; ++tap) {
-      const int st = tap % kCStages;
-      if (tap >= kCStages && !mbar_wait(&empty[st], ((tap / kCStages) + 1) & 1, a.err, kDevTimeoutEmpty)) break;
-      uint8_t* sa = sm + st * (kCA + kCB);
-      mbar_arrive_expect_tx(&full[st], kCA + kCB);
-      const int dy = tap / 3, dx = tap % 3;
-      tma_load_4d(sa, &mIn, 0, sgn * (dx - 1), y0 + sgn * (dy - 1), img, &full[st]);
-      if (MODE == 0) tma_load_4d(sa + kCA, &mW, 0, tap, 0, slot, &full[st]);   // {in, tap, out, slot}
-      else tma_load_4d(sa + kCA, &mW, 0, 0, tap, slot, &full[st]);             // {out, in, tap, slot}
+      if (MODE == 0) tma_load_4d(wts + tap * kCB, &mW, 0, tap, 0, slot, wfull);   // {in, tap, out, slot}
+      else tma_load_4d(wts + tap * kCB, &mW, 0, 0, tap, slot, wfull);             // {out, in, tap, slot}
+    }
+    int it = 0;
+    for (int k = 0; k < my_tiles; ++k) {
+      const int tile = c0 + k * cpw;
+      const int img = lane * a.B + tile / kTilesPerImg, y0 = (tile % kTilesPerImg) * kTileRows;
+      for (int dx = 0; dx < 3; ++dx, ++it) {
+        const int sl = it % kGSlots;
+        if (it >= kGSlots && !mbar_wait(&empty[sl], ((it / kGSlots) + 1) & 1, a.err, kDevTimeoutEmpty)) {
+          k = my_tiles;
+          break;
+        }
+        mbar_arrive_expect_tx(&full[sl], kGBox);
+        tma_load_4d(slots + sl * kGBox, &mIn, 0, sgn * (dx - 1), y0 - 1, img, &full[sl]);
+      }
     }
   } else if (t == 32) {
     constexpr uint32_t idesc = idesc_bf16_f32(128, kCC);
-    for (int tap = 0; tap < kTaps; ++tap) {
-      const int st = tap % kCStages;
-      if (!mbar_wait(&full[st], (tap / kCStages) & 1, a.err, kDevTimeoutFull)) break;
+    bool ok = mbar_wait(wfull, 0, a.err, kDevTimeoutFull);
+    tc_fence_after();
+    int it = 0;
+    for (int k = 0; ok && k < my_tiles; ++k) {
+      const int buf = k & 1, use = k >> 1;
+      if (use >= 1 && !mbar_wait(&acce[buf], (use - 1) & 1, a.err, kDevTimeoutAccum)) break;
       tc_fence_after();
-      const uint32_t sa = smem_u32(sm + st * (kCA + kCB));
+      for (int dx = 0; dx < 3; ++dx, ++it) {
+        const int sl = it % kGSlots;
+        if (!mbar_wait(&full[sl], (it / kGSlots) & 1, a.err, kDevTimeoutFull)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t sa = smem_u32(slots + sl * kGBox);
 #pragma unroll
-      for (int j = 0; j < kCC / 16; ++j)
-        umma_bf16(tmem, smem_desc_k128(sa + j * 32), smem_desc_k128(sa + kCA + j * 32), idesc,
-                  (tap | j) != 0 ? 1u : 0u);
-      umma_commit(&empty[st]);
+        for (int dy = 0; dy < 3; ++dy) {
+          const int rowoff = MODE == 0 ? dy : 2 - dy;   // sub-tile of the 6-row box
+          const uint32_t aa = sa + rowoff * kImg * kCC * 2;
+          const uint32_t bb = smem_u32(wts + (dy * 3 + dx) * kCB);
+#pragma unroll
+          for (int j = 0; j < kCC / 16; ++j)
+            umma_bf16(tmem + buf * kCC, smem_desc_k128(aa + j * 32), smem_desc_k128(bb + j * 32), idesc,
+                      (dx | dy | j) != 0 ? 1u : 0u);
+        }
+        umma_commit(&empty[sl]);
+      }
+      if (ok) umma_commit(&accf[buf]);
     }
-    umma_commit(accb);
-  }
-  // epilogue: thread = output pixel (TMEM lane), 64 channels
-  int ok = mbar_wait(accb, 0, a.err, kDevTimeoutAccum) ? 1 : 0;
-  ok = __all_sync(0xffffffffu, ok);
-  tc_fence_after();
-  const int p = t;
-  const int64_t base = (static_cast<int64_t>(img) * kPix + y0 * kImg + p) * kCC;
-  float v[kCC];
-  if (ok) {
-    float lo[32], hi[32];
-    tmem_ld_32x32b_x32_pair(tmem + (static_cast<uint32_t>(warp * 32) << 16), lo,
-                            tmem + (static_cast<uint32_t>(warp * 32) << 16) + 32, hi);
+  } else if (warp >= 2) {
+    // epilogue: thread = output pixel (TMEM lane of its warp's quarter), 64 channels
+    const int quarter = warp & 3;
+    const int p = quarter * 32 + lane_id;
+    const uint32_t trow = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
+    float bsum[kCC];
 #pragma unroll
-    for (int c = 0; c < 32; ++c) {
-      v[c] = lo[c];
-      v[32 + c] = hi[c];
-    }
-  } else {
-#pragma unroll
-    for (int c = 0; c < kCC; ++c) v[c] = 0.f;
-  }
-  if (MODE == 0) {
+    for (int c = 0; c < kCC; ++c) bsum[c] = 0.f;
     const float* bias = a.bias + static_cast<int64_t>(slot) * a.slot_stride + a.off_bias;
+    for (int k = 0; k < my_tiles; ++k) {
+      const int tile = c0 + k * cpw;
+      const int img = lane * a.B + tile / kTilesPerImg, y0 = (tile % kTilesPerImg) * kTileRows;
+      const int buf = k & 1, use = k >> 1;
+      int ok = mbar_wait(&accf[buf], use & 1, a.err, kDevTimeoutAccum) ? 1 : 0;
+      ok = __all_sync(0xffffffffu, ok);
+      tc_fence_after();
+      float v[kCC];
+      {
+        float lo[32], hi[32];
+        tmem_ld_32x32b_x32_pair(trow + buf * kCC, lo, trow + buf * kCC + 32, hi);
 #pragma unroll
-    for (int c = 0; c < kCC; ++c) v[c] += bias[c];
-  }
-  if (a.add) {
-#pragma unroll
-    for (int q = 0; q < kCC / 8; ++q) {
-      const uint4 r = *reinterpret_cast<const uint4*>(a.add + base + 8 * q);
-      const __nv_bfloat162* r2 = reinterpret_cast<const __nv_bfloat162*>(&r);
-#pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        const float2 f = __bfloat1622float2(r2[j]);
-        v[8 * q + 2 * j] += f.x;
-        v[8 * q + 2 * j + 1] += f.y;
+        for (int c = 0; c < 32; ++c) {
+          v[c] = ok ? lo[c] : 0.f;
+          v[32 + c] = ok ? hi[c] : 0.f;
+        }
       }
+      tc_fence_before();
+      mbar_arrive(&acce[buf]);   // the accumulator has been read: the next tile may use it
+      const int64_t base = (static_cast<int64_t>(img) * kPix + y0 * kImg + p) * kCC;
+      if (MODE == 0) {
+#pragma unroll
+        for (int c = 0; c < kCC; ++c) v[c] += bias[c];
+      }
+      if (a.add) {
+#pragma unroll
+        for (int q = 0; q < kCC / 8; ++q) {
+          const uint4 r = *reinterpret_cast<const uint4*>(a.add + base + 8 * q);
+          const __nv_bfloat162* r2 = reinterpret_cast<const __nv_bfloat162*>(&r);
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            const float2 f = __bfloat1622float2(r2[j]);
+            v[8 * q + 2 * j] += f.x;
+            v[8 * q + 2 * j + 1] += f.y;
+          }
+        }
+      }
+      if (MODE == 0) {
+#pragma unroll
+        for (int c = 0; c < kCC; ++c) v[c] = fmaxf(v[c], 0.f);
+      } else {
+#pragma unroll
+        for (int q = 0; q < kCC / 8; ++q) {
+          const uint4 r = *reinterpret_cast<const uint4*>(a.mask + base + 8 * q);
+          const __nv_bfloat162* r2 = reinterpret_cast<const __nv_bfloat162*>(&r);
+#pragma unroll
+          for (int j = 0; j < 4; ++j) {
+            const float2 f = __bfloat1622float2(r2[j]);
+            if (!(f.x > 0.f)) v[8 * q + 2 * j] = 0.f;
+            if (!(f.y > 0.f)) v[8 * q + 2 * j + 1] = 0.f;
+          }
+        }
+#pragma unroll
+        for (int c = 0; c < kCC; ++c) bsum[c] += v[c];
+      }
+#pragma unroll
+      for (int q = 0; q < kCC / 8; ++q)
+        *reinterpret_cast<uint4*>(a.out + base + 8 * q) =
+            make_uint4(pack_bf16x2(v[8 * q], v[8 * q + 1]), pack_bf16x2(v[8 * q + 2], v[8 * q + 3]),
+                       pack_bf16x2(v[8 * q + 4], v[8 * q + 5]), pack_bf16x2(v[8 * q + 6], v[8 * q + 7]));
+    }
+    if (MODE == 1 && a.bias_part) {
+      // this CTA's channel sums: per thread over its tiles in order, then over
+      // the 128 pixels of the tile in pixel order (the input slots are idle now)
+      float* T = reinterpret_cast<float*>(slots);
+#pragma unroll
+      for (int c = 0; c < kCC; ++c) T[p * (kCC + 1) + c] = bsum[c];
     }
   }
-  if (MODE == 0) {
-#pragma unroll
-    for (int c = 0; c < kCC; ++c) v[c] = fmaxf(v[c], 0.f);
-  } else {
-#pragma unroll
-    for (int q = 0; q < kCC / 8; ++q) {
-      const uint4 r = *reinterpret_cast<const uint4*>(a.mask + base + 8 * q);
-      const __nv_bfloat162* r2 = reinterpret_cast<const __nv_bfloat162*>(&r);
-#pragma unroll
-      for (int j = 0; j < 4; ++j) {
-        const float2 f = __bfloat1622float2(r2[j]);
-        if (!(f.x > 0.f)) v[8 * q + 2 * j] = 0.f;
-        if (!(f.y > 0.f)) v[8 * q + 2 * j + 1] = 0.f;
-      }
-    }
-  }
-#pragma unroll
-  for (int q = 0; q < kCC / 8; ++q)
-    *reinterpret_cast<uint4*>(a.out + base + 8 * q) =
-        make_uint4(pack_bf16x2(v[8 * q], v[8 * q + 1]), pack_bf16x2(v[8 * q + 2], v[8 * q + 3]),
-                   pack_bf16x2(v[8 * q + 4], v[8 * q + 5]), pack_bf16x2(v[8 * q + 6], v[8 * q + 7]));
   if (MODE == 1 && a.bias_part) {
-    // channel sums of the fp32 output over the tile's pixels (fixed order),
-    // through the idle stage buffers: [128 pixels][65]
-    float* T = reinterpret_cast<float*>(sm);
-    __syncthreads();
-#pragma unroll
-    for (int c = 0; c < kCC; ++c) T[p * 65 + c] = v[c];
     __syncthreads();
     if (t < kCC) {
+      const float* T = reinterpret_cast<const float*>(slots);
       float s = 0.f;
-      for (int q = 0; q < kTilePix; ++q) s += T[q * 65 + t];
-      a.bias_part[(static_cast<int64_t>(lane) * a.B * kTilesPerImg + tile) * kCC + t] = s;
+      for (int q = 0; q < kTilePix; ++q) s += T[q * (kCC + 1) + t];
+      a.bias_part[(static_cast<int64_t>(lane) * cpw + c0) * kCC + t] = s;
     }
   }
   tc_fence_before();
   __syncthreads();
   if (warp == 0) {
     tc_fence_after();
-    tmem_dealloc(tmem, 64);
+    tmem_dealloc(tmem, 128);
   }
 }
 
@@ -332,9 +392,9 @@ __global__ void __launch_bounds__(256) conv_sgd_kernel(const __grid_constant__ C
     for (int q = t; q < kSgdRows * kCC; q += 256) wt[q] = __float2bfloat16_rn(T[q / kCC][q % kCC]);
   }
   if (blockIdx.x == 0 && t < kCC) {   // bias: per-tile sums in tile order
-    const float* bp = a.bias_part[layer] + static_cast<int64_t>(lane) * a.n_tiles * kCC;
+    const float* bp = a.bias_part[layer] + static_cast<int64_t>(lane) * a.n_tiles[layer] * kCC;
     float s = 0.f;
-    for (int i = 0; i < a.n_tiles; ++i) s += bp[static_cast<int64_t>(i) * kCC + t];
+    for (int i = 0; i < a.n_tiles[layer]; ++i) s += bp[static_cast<int64_t>(i) * kCC + t];
     a.master_w[dof + a.offB[layer] + t] = fmaf(-a.lr, s, a.master[so + a.offB[layer] + t]);
   }
 }
@@ -551,17 +611,25 @@ __global__ void __launch_bounds__(kCT) cnn_dzb_kernel(const __nv_bfloat16* v, co
 int cnn_tiles_per_image() { return kTilesPerImg; }
 int cnn_wgrad_chunks(int B) { return (B + kWgradImagesPerChunk - 1) / kWgradImagesPerChunk; }
 
+int conv_ctas_per_worker(int B, int n_active, int sms) {
+  const int tiles = B * kTilesPerImg;
+  int cpw = sms / (n_active > 0 ? n_active : 1);
+  if (cpw < 1) cpw = 1;
+  if (cpw > tiles) cpw = tiles;
+  return cpw;
+}
+
 cudaError_t launch_conv_igemm(int mode, const CUtensorMap& mIn, const CUtensorMap& mW, const ConvArgs& a, int n_active,
-                              cudaStream_t s) {
-  const dim3 grid(a.B * kTilesPerImg, n_active);
+                              int cpw, cudaStream_t s) {
+  const dim3 grid(cpw, n_active);
   if (mode == 0) {
-    cudaError_t e = cudaFuncSetAttribute(conv_igemm_kernel<0>, cudaFuncAttributeMaxDynamicSharedMemorySize, kCSmem);
+    cudaError_t e = cudaFuncSetAttribute(conv_igemm_kernel<0>, cudaFuncAttributeMaxDynamicSharedMemorySize, kGSmem);
     if (e != cudaSuccess) return e;
-    conv_igemm_kernel<0><<<grid, kCT, kCSmem, s>>>(mIn, mW, a);
+    conv_igemm_kernel<0><<<grid, kGT, kGSmem, s>>>(mIn, mW, a);
   } else {
-    cudaError_t e = cudaFuncSetAttribute(conv_igemm_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, kCSmem);
+    cudaError_t e = cudaFuncSetAttribute(conv_igemm_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, kGSmem);
     if (e != cudaSuccess) return e;
-    conv_igemm_kernel<1><<<grid, kCT, kCSmem, s>>>(mIn, mW, a);
+    conv_igemm_kernel<1><<<grid, kGT, kGSmem, s>>>(mIn, mW, a);
   }
   return cudaGetLastError();
 }

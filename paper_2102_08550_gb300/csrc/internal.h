@@ -199,7 +199,7 @@ struct ConvArgs {
   const __nv_bfloat16* add;    // [lane][B][1024][64] added before the activation / mask, or null
   const __nv_bfloat16* mask;   // input gradient: stored activation of the layer input (> 0 keeps)
   __nv_bfloat16* out;          // [lane][B][1024][64]
-  float* bias_part;            // input gradient: [lane][B * 8][64] per-tile channel sums, or null
+  float* bias_part;            // input gradient: [lane][cpw][64] per-CTA channel sums, or null
   int* err;
 };
 struct WgradArgs {
@@ -212,7 +212,8 @@ constexpr int kMaxConvLayers = 9;
 struct ConvSgdArgs {
   const int* wid;
   const int* src;
-  int n_chunks, n_tiles, layers;
+  int n_chunks, layers;
+  int n_tiles[kMaxConvLayers];             // per layer: bias partials per lane
   const float* part[kMaxConvLayers];       // per layer, as WgradArgs::part
   const float* bias_part[kMaxConvLayers];  // per layer: [lane][n_tiles][64]
   __nv_bfloat16* wt[kMaxConvLayers];       // per layer: transposed bf16 copy in slot 0, or null
@@ -249,8 +250,10 @@ struct CnnHeadArgs {
 };
 int cnn_tiles_per_image();
 int cnn_wgrad_chunks(int B);
+// CTAs per worker of the implicit-GEMM kernel (one per SM over the active workers)
+int conv_ctas_per_worker(int B, int n_active, int sms);
 cudaError_t launch_conv_igemm(int mode, const CUtensorMap& mIn, const CUtensorMap& mW, const ConvArgs& a, int n_active,
-                              cudaStream_t s);
+                              int cpw, cudaStream_t s);
 cudaError_t launch_conv_wgrad(const CUtensorMap& mIn, const CUtensorMap& mDz, const WgradArgs& a, int n_active,
                               cudaStream_t s);
 cudaError_t launch_conv_sgd(const ConvSgdArgs& a, int n_active, cudaStream_t s);
