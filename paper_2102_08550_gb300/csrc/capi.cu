@@ -167,7 +167,7 @@ struct oscars_ctx {
   int64_t cnn_wt_slot = 0;                   // elements per slot of the transposed copies
   __nv_bfloat16* cnn_wt = nullptr;           // [slot][2 * blocks][9][64 in][64 out]
   std::vector<__nv_bfloat16*> cnn_buf;       // x, s, (u_k, v_k) per block, dz0, dz1, dz2: [W][B][1024][64]
-  std::vector<CUtensorMap> cnn_m6, cnn_m2;   // per buffer: boxes of 6 and of 2 image rows
+  std::vector<CUtensorMap> cnn_m6, cnn_m4, cnn_m2;   // per buffer: boxes of 6, 4 and 2 image rows
   int sms = 0;                               // multiprocessors of the device
   std::vector<CUtensorMap> cnn_mw, cnn_mwt;  // weights per conv layer: forward layout, transposed (blocks)
   float* cnn_g = nullptr;                    // [W][B][64] pooled features
@@ -703,7 +703,9 @@ cudaError_t enqueue_step_cnn(oscars_ctx* c, int s, int na, const int* wid, const
   const int X = 0, S = 1, dzbase = 2 + 2 * nb;
   auto U = [&](int k) { return 2 + 2 * k; };
   auto V = [&](int k) { return 3 + 2 * k; };
-  const size_t wpl = static_cast<size_t>(c->W) * c->cnn_chunks * 9 * 64 * 64;   // weight partials per layer
+  const int ipc = conv_wgrad_images_per_chunk(B, na, c->sms);
+  const int chunks = (B + ipc - 1) / ipc;
+  const size_t wpl = static_cast<size_t>(c->W) * chunks * 9 * 64 * 64;          // weight partials per layer
   const size_t bpl = static_cast<size_t>(c->W) * tiles * 64;                    // bias partials per layer
   {
     CnnStageArgs a;
@@ -742,12 +744,12 @@ cudaError_t enqueue_step_cnn(oscars_ctx* c, int s, int na, const int* wid, const
     WgradArgs a;
     a.wid = wid;
     a.B = B;
-    a.n_chunks = c->cnn_chunks;
-    a.img_per_chunk = kWgradImagesPerChunk;
+    a.n_chunks = chunks;
+    a.img_per_chunk = ipc;
     a.part = c->cnn_wpart + layer * wpl;
     a.err = c->err;
     ProfScope ps(c, "conv_wgrad", st);
-    return launch_conv_wgrad(c->cnn_m2[in], c->cnn_m2[dz], a, na, st);
+    return launch_conv_wgrad(c->cnn_m4[in], c->cnn_m2[dz], a, na, st);
   };
   // forward
   if ((e = conv(0, 0, X, -1, -1, S, nullptr)) != cudaSuccess) return e;
@@ -808,7 +810,7 @@ cudaError_t enqueue_step_cnn(oscars_ctx* c, int s, int na, const int* wid, const
   std::memset(&a, 0, sizeof(a));
   a.wid = wid;
   a.src = src;
-  a.n_chunks = c->cnn_chunks;
+  a.n_chunks = chunks;
   a.layers = layers;
   const int cpw = conv_ctas_per_worker(B, na, c->sms);
   for (int l = 0; l < layers; ++l) {
@@ -898,7 +900,7 @@ oscars_status layout_cnn(oscars_ctx* c, const oscars_config* cfg) {
   c->P = static_cast<int64_t>(C) * 9 * Cin + C + static_cast<int64_t>(c->cnn_blocks) * 2 * (C * 9 * C + C) +
          static_cast<int64_t>(K) * C + K;
   c->cnn_wt_slot = static_cast<int64_t>(2 * c->cnn_blocks) * 9 * 64 * 64;
-  c->cnn_chunks = cnn_wgrad_chunks(c->B);
+  c->cnn_chunks = c->B;   // capacity: at most one image per chunk
   return OSCARS_OK;
 }
 
@@ -1016,6 +1018,7 @@ oscars_status allocate_cnn(oscars_ctx* c) {
     return fail(c, OSCARS_ENOMEM, "device allocation failed (gradients)");
   // tensor maps: activations {64 ch, 32 x, 32 y, images}; weights per slot
   c->cnn_m6.resize(nbuf);
+  c->cnn_m4.resize(nbuf);
   {
     int dev = 0;
     cudaGetDevice(&dev);
@@ -1028,6 +1031,7 @@ oscars_status allocate_cnn(oscars_ctx* c) {
     const uint64_t d[4] = {64, 32, 32, imgs};
     const uint64_t stv[3] = {64 * 2, 32 * 64 * 2, 1024 * 64 * 2};
     ok &= make_map_box4(&c->cnn_m6[i], c->cnn_buf[i], d, stv, {64, 32, 6, 1});
+    ok &= make_map_box4(&c->cnn_m4[i], c->cnn_buf[i], d, stv, {64, 32, 4, 1});
     ok &= make_map_box4(&c->cnn_m2[i], c->cnn_buf[i], d, stv, {64, 32, 2, 1});
   }
   c->cnn_mw.resize(layers);

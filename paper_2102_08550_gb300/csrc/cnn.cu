@@ -24,8 +24,9 @@
 //  * conv_wgrad_kernel: dW[o][tap][i] = sum_p dz[p][o] x[p + off(tap)][i] on
 //    tcgen05 with both operands MN-major straight from the NHWC tensors: the
 //    K dimension is the pixels, taps are stacked in pairs to make M = 128
-//    (in-channels of two taps), N = 64 out-channels.  Split over chunks of
-//    images; partial sums go to global memory.
+//    (in-channels of two taps), N = 64 out-channels; one 4-row input box per
+//    x-offset serves the three y-offsets.  Split over chunks of images (one
+//    wave of CTAs); partial sums go to global memory.
 //  * conv_sgd_kernel: sums the chunks in order, SGD of the fp32 master and
 //    its bf16 copies (the forward layout and the transposed one), bias from
 //    the per-tile sums.
@@ -47,11 +48,8 @@ constexpr int kCT = 128;                    // threads of the implicit-GEMM and 
 constexpr int kCB = kCC * kCC * 2;          // 8 KB: one tap of the weights
 // weight gradient
 constexpr int kWT = 128;
-constexpr int kWStages = 2;
 constexpr int kWTile = 2 * kImg * kCC * 2;  // 8 KB: 64 pixels (2 rows) x 64 channels
-constexpr int kWPairs = 5;                  // tap pairs (0,1) (2,3) (4,5) (6,7) (8,8)
-constexpr int kWStage = (2 * kWPairs + 1) * kWTile;   // 10 input tiles + the output-gradient tile
-constexpr int kWSmem = kWStages * kWStage + 256 + 1024;
+constexpr int kWPairs = 5;                  // accumulators of stacked tap pairs
 
 __device__ __forceinline__ uint8_t* align1024(uint8_t* p) {
   return reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(p) + 1023) & ~uintptr_t(1023));
@@ -261,14 +259,47 @@ __global__ void __launch_bounds__(kGT, 1) conv_igemm_kernel(const __grid_constan
 }
 
 // ------------------------------------------------------------------ weight gradient
+// K-block = 64 pixels (2 image rows yr, yr + 1).  Per K-block TMA loads the
+// output-gradient tile (2 rows) and, per x-offset dx, one 4-row box of the
+// input (rows yr - 1 .. yr + 2, shifted by dx - 1); tap (dy, dx)'s operand is
+// the box's 2-row sub-tile at row offset dy.  The A operand (M = 128) stacks
+// two taps as two 64-channel atoms `lbo` bytes apart:
+//   pair 0..2: (dy 0, dy 1) of box dx = pair      (atoms 4 KB apart)
+//   pair 3:    dy 2 of box 0 and of box 1         (atoms one box apart)
+//   pair 4:    dy 2 of box 2                      (upper half unused)
+constexpr int kWRow = kImg * kCC * 2;           // 4 KB: one image row, 64 channels
+constexpr int kWBox = 4 * kWRow;                // 16 KB
+constexpr int kWStage2 = 3 * kWBox + kWTile;    // 56 KB: three input boxes + the output-gradient tile
+constexpr int kWStages2 = 3;
+constexpr int kWSmem2 = kWStages2 * kWStage2 + 256 + 1024;
+
+__device__ __forceinline__ void wgrad_pair(int pr, int& start, int& lbo, int& tap0, int& tap1) {
+  if (pr < 3) {
+    start = pr * kWBox;
+    lbo = kWRow;
+    tap0 = pr;            // (dy 0, dx pr)
+    tap1 = 3 + pr;        // (dy 1, dx pr)
+  } else if (pr == 3) {
+    start = 2 * kWRow;
+    lbo = kWBox;
+    tap0 = 6;             // (dy 2, dx 0)
+    tap1 = 7;             // (dy 2, dx 1)
+  } else {
+    start = 2 * kWBox + 2 * kWRow;
+    lbo = kWRow;
+    tap0 = 8;             // (dy 2, dx 2)
+    tap1 = -1;
+  }
+}
+
 __global__ void __launch_bounds__(kWT, 1) conv_wgrad_kernel(const __grid_constant__ CUtensorMap mIn,
                                                             const __grid_constant__ CUtensorMap mDz,
                                                             const __grid_constant__ WgradArgs a) {
   extern __shared__ uint8_t ws_raw[];
   uint8_t* sm = align1024(ws_raw);
-  uint64_t* full = reinterpret_cast<uint64_t*>(sm + kWStages * kWStage);
-  uint64_t* empty = full + kWStages;
-  uint64_t* accb = empty + kWStages;
+  uint64_t* full = reinterpret_cast<uint64_t*>(sm + kWStages2 * kWStage2);
+  uint64_t* empty = full + kWStages2;
+  uint64_t* accb = empty + kWStages2;
   uint32_t* tslot = reinterpret_cast<uint32_t*>(accb + 1);
   const int t = threadIdx.x, warp = t >> 5;
   const int chunk = blockIdx.x, e = blockIdx.y;
@@ -279,7 +310,7 @@ __global__ void __launch_bounds__(kWT, 1) conv_wgrad_kernel(const __grid_constan
   if (t == 0) {
     prefetch_tmap(&mIn);
     prefetch_tmap(&mDz);
-    for (int i = 0; i < kWStages; ++i) {
+    for (int i = 0; i < kWStages2; ++i) {
       mbar_init(&full[i], 1);
       mbar_init(&empty[i], 1);
     }
@@ -296,32 +327,31 @@ __global__ void __launch_bounds__(kWT, 1) conv_wgrad_kernel(const __grid_constan
   const uint32_t tmem = *tslot;
   if (t == 0) {
     for (int kb = 0; kb < nk; ++kb) {
-      const int st = kb % kWStages;
-      if (kb >= kWStages && !mbar_wait(&empty[st], ((kb / kWStages) + 1) & 1, a.err, kDevTimeoutEmpty)) break;
-      uint8_t* sa = sm + st * kWStage;
+      const int st = kb % kWStages2;
+      if (kb >= kWStages2 && !mbar_wait(&empty[st], ((kb / kWStages2) + 1) & 1, a.err, kDevTimeoutEmpty)) break;
+      uint8_t* sa = sm + st * kWStage2;
       const int img = lane * a.B + i0 + kb / (kImg / 2), yr = (kb % (kImg / 2)) * 2;
-      mbar_arrive_expect_tx(&full[st], kWStage);
-      tma_load_4d(sa + 2 * kWPairs * kWTile, &mDz, 0, 0, yr, img, &full[st]);
-      for (int q = 0; q < 2 * kWPairs; ++q) {
-        const int tap = q < kTaps ? q : kTaps - 1;
-        const int dy = tap / 3, dx = tap % 3;
-        tma_load_4d(sa + q * kWTile, &mIn, 0, dx - 1, yr + dy - 1, img, &full[st]);
-      }
+      mbar_arrive_expect_tx(&full[st], kWStage2);
+      for (int dx = 0; dx < 3; ++dx) tma_load_4d(sa + dx * kWBox, &mIn, 0, dx - 1, yr - 1, img, &full[st]);
+      tma_load_4d(sa + 3 * kWBox, &mDz, 0, 0, yr, img, &full[st]);
     }
   } else if (t == 32) {
     constexpr uint32_t idesc = idesc_bf16_f32_mn(128, kCC);
     for (int kb = 0; kb < nk; ++kb) {
-      const int st = kb % kWStages;
-      if (!mbar_wait(&full[st], (kb / kWStages) & 1, a.err, kDevTimeoutFull)) break;
+      const int st = kb % kWStages2;
+      if (!mbar_wait(&full[st], (kb / kWStages2) & 1, a.err, kDevTimeoutFull)) break;
       tc_fence_after();
-      const uint32_t sa = smem_u32(sm + st * kWStage);
-      const uint32_t sb = sa + 2 * kWPairs * kWTile;
+      const uint32_t sa = smem_u32(sm + st * kWStage2);
+      const uint32_t sb = sa + 3 * kWBox;
 #pragma unroll
-      for (int pr = 0; pr < kWPairs; ++pr)
+      for (int pr = 0; pr < kWPairs; ++pr) {
+        int start, lbo, tap0, tap1;
+        wgrad_pair(pr, start, lbo, tap0, tap1);
 #pragma unroll
         for (int j = 0; j < 4; ++j)   // K = 16 pixels per MMA: two 8-row groups
-          umma_bf16(tmem + pr * kCC, smem_desc_mn128(sa + pr * 2 * kWTile + j * 2048, kWTile),
-                    smem_desc_mn128(sb + j * 2048, kWTile), idesc, (kb | j) != 0 ? 1u : 0u);
+          umma_bf16(tmem + pr * kCC, smem_desc_mn128(sa + start + j * 2048, lbo), smem_desc_mn128(sb + j * 2048, kWTile),
+                    idesc, (kb | j) != 0 ? 1u : 0u);
+      }
       umma_commit(&empty[st]);
     }
     umma_commit(accb);
@@ -329,15 +359,17 @@ __global__ void __launch_bounds__(kWT, 1) conv_wgrad_kernel(const __grid_constan
   int ok = mbar_wait(accb, 0, a.err, kDevTimeoutAccum) ? 1 : 0;
   ok = __all_sync(0xffffffffu, ok);
   tc_fence_after();
-  // TMEM lane r: row r of each pair's accumulator = (tap 2 pr + r / 64, in-channel r % 64)
+  // TMEM lane r: row r of each pair's accumulator = (tap of atom r / 64, in-channel r % 64)
   const int r = t;
   const int ci = r & (kCC - 1);
   for (int pr = 0; pr < kWPairs; ++pr) {
-    const int tap = 2 * pr + (r >> 6);
+    int start, lbo, tap0, tap1;
+    wgrad_pair(pr, start, lbo, tap0, tap1);
+    const int tap = r < 64 ? tap0 : tap1;
     float lo[32], hi[32];
     tmem_ld_32x32b_x32_pair(tmem + (static_cast<uint32_t>(warp * 32) << 16) + pr * kCC, lo,
                             tmem + (static_cast<uint32_t>(warp * 32) << 16) + pr * kCC + 32, hi);
-    if (tap < kTaps && ok) {
+    if (tap >= 0 && ok) {
       float* dst = a.part + ((static_cast<int64_t>(lane) * a.n_chunks + chunk) * kTaps + tap) * kCC * kCC + ci * kCC;
 #pragma unroll
       for (int q = 0; q < 8; ++q) {
@@ -609,7 +641,6 @@ __global__ void __launch_bounds__(kCT) cnn_dzb_kernel(const __nv_bfloat16* v, co
 
 // ------------------------------------------------------------------ launchers
 int cnn_tiles_per_image() { return kTilesPerImg; }
-int cnn_wgrad_chunks(int B) { return (B + kWgradImagesPerChunk - 1) / kWgradImagesPerChunk; }
 
 int conv_ctas_per_worker(int B, int n_active, int sms) {
   const int tiles = B * kTilesPerImg;
@@ -634,11 +665,17 @@ cudaError_t launch_conv_igemm(int mode, const CUtensorMap& mIn, const CUtensorMa
   return cudaGetLastError();
 }
 
+int conv_wgrad_images_per_chunk(int B, int n_active, int sms) {
+  int per_worker = sms / (n_active > 0 ? n_active : 1);   // CTAs per worker in one wave
+  if (per_worker < 1) per_worker = 1;
+  return (B + per_worker - 1) / per_worker;
+}
+
 cudaError_t launch_conv_wgrad(const CUtensorMap& mIn, const CUtensorMap& mDz, const WgradArgs& a, int n_active,
                               cudaStream_t s) {
-  cudaError_t e = cudaFuncSetAttribute(conv_wgrad_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kWSmem);
+  cudaError_t e = cudaFuncSetAttribute(conv_wgrad_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kWSmem2);
   if (e != cudaSuccess) return e;
-  conv_wgrad_kernel<<<dim3(a.n_chunks, n_active), kWT, kWSmem, s>>>(mIn, mDz, a);
+  conv_wgrad_kernel<<<dim3(a.n_chunks, n_active), kWT, kWSmem2, s>>>(mIn, mDz, a);
   return cudaGetLastError();
 }
 

@@ -188,7 +188,6 @@ cudaError_t launch_broadcast(const float* xg, float* slab, int64_t stride, int W
 
 // ---------------------------------------------------------------- convolutional worker
 // 32 x 32 images, 64 channels, 3x3 convolutions (csrc/cnn.cu)
-constexpr int kWgradImagesPerChunk = 2;   // images per split-K chunk of the weight gradient
 
 struct ConvArgs {
   const int* wid;              // [n_active] lane of each active entry
@@ -249,7 +248,8 @@ struct CnnHeadArgs {
   float lr;
 };
 int cnn_tiles_per_image();
-int cnn_wgrad_chunks(int B);
+// images per split-K chunk of the weight gradient (one wave of CTAs over the active workers)
+int conv_wgrad_images_per_chunk(int B, int n_active, int sms);
 // CTAs per worker of the implicit-GEMM kernel (one per SM over the active workers)
 int conv_ctas_per_worker(int B, int n_active, int sms);
 cudaError_t launch_conv_igemm(int mode, const CUtensorMap& mIn, const CUtensorMap& mW, const ConvArgs& a, int n_active,
