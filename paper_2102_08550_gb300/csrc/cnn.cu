@@ -67,7 +67,7 @@ constexpr int kGT = 192;                    // warp 0 TMA, warp 1 MMA, warps 2-5
 constexpr int kGSlots = 6;                  // input boxes in flight (two tiles)
 constexpr int kGBox = 6 * kImg * kCC * 2;   // 24 KB: 6 rows x 32 pixels x 64 channels
 constexpr int kGW = kTaps * kCB;            // 72 KB of resident weights
-constexpr int kGSmem = kGW + kGSlots * kGBox + 256 + 1024;
+constexpr int kGSmem = kGW + kGSlots * kGBox + 512 + 1024;   // + barriers, TMEM slot, bias
 static_assert(kTilePix * (kCC + 1) * 4 <= kGSlots * kGBox, "the bias reduction reuses the input slots");
 
 template <int MODE>   // 0 forward, 1 input gradient
@@ -84,6 +84,7 @@ __global__ void __launch_bounds__(kGT, 1) conv_igemm_kernel(const __grid_constan
   uint64_t* accf = empty + kGSlots;  // [2]
   uint64_t* acce = accf + 2;         // [2] 128 arrivals
   uint32_t* tslot = reinterpret_cast<uint32_t*>(acce + 2);
+  float* bias_s = reinterpret_cast<float*>(tslot + 4);   // [64] this worker's bias (forward)
   const int t = threadIdx.x, warp = t >> 5, lane_id = t & 31;
   const int c0 = blockIdx.x, cpw = gridDim.x, e = blockIdx.y;
   const int lane = a.wid[e], slot = a.src[e];
@@ -107,6 +108,8 @@ __global__ void __launch_bounds__(kGT, 1) conv_igemm_kernel(const __grid_constan
     tmem_alloc(tslot, 128);
     tmem_relinquish();
   }
+  if (MODE == 0 && t >= 64 && t < 64 + kCC)
+    bias_s[t - 64] = a.bias[static_cast<int64_t>(slot) * a.slot_stride + a.off_bias + (t - 64)];
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
@@ -171,7 +174,6 @@ __global__ void __launch_bounds__(kGT, 1) conv_igemm_kernel(const __grid_constan
     float bsum[kCC];
 #pragma unroll
     for (int c = 0; c < kCC; ++c) bsum[c] = 0.f;
-    const float* bias = a.bias + static_cast<int64_t>(slot) * a.slot_stride + a.off_bias;
     for (int k = 0; k < my_tiles; ++k) {
       const int tile = c0 + k * cpw;
       const int img = lane * a.B + tile / kTilesPerImg, y0 = (tile % kTilesPerImg) * kTileRows;
@@ -194,7 +196,7 @@ __global__ void __launch_bounds__(kGT, 1) conv_igemm_kernel(const __grid_constan
       const int64_t base = (static_cast<int64_t>(img) * kPix + y0 * kImg + p) * kCC;
       if (MODE == 0) {
 #pragma unroll
-        for (int c = 0; c < kCC; ++c) v[c] += bias[c];
+        for (int c = 0; c < kCC; ++c) v[c] += bias_s[c];
       }
       if (a.add) {
 #pragma unroll
