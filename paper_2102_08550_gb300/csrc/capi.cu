@@ -159,6 +159,15 @@ struct oscars_ctx {
   std::vector<CUtensorMap> mA0s, mAT0s;
   bool fused = false;                   // whole-round kernel (2-layer MLP)
   CUtensorMap mX4, mXT4;                // staged inputs of every step (fused kernel)
+  // the one-launch round stages the next round while the current one runs:
+  // two input buffers, used alternately (index `parity` holds the next round)
+  __nv_bfloat16* A0b[2] = {};
+  __nv_bfloat16* A0Tb[2] = {};
+  int32_t* labb[2] = {};
+  CUtensorMap mX4b[2], mXT4b[2];
+  int parity = 0;
+  bool staged = false;                  // A0b[parity] holds the mini-batches of the next round
+  cudaGraphExec_t ahead_exec[2] = {};   // round graphs, one per parity
   unsigned long long* phase_ts = nullptr;   // flag bit 4: phase stamps of the fused round
   // convolutional worker (OSCARS_MODEL_CNN)
   int cnn_blocks = 0, cnn_chunks = 0;
@@ -199,6 +208,7 @@ struct oscars_ctx {
   };
   std::vector<ProfEntry> prof_pending;
   std::vector<ProfEntry> prof_round_graph, prof_merge_graph;   // event nodes of the captured graphs
+  std::vector<ProfEntry> prof_ahead_graph[2];                   // event nodes of the two parity round graphs
   std::vector<ProfEntry>* prof_sink = nullptr;                  // where ProfScope files entries
   cudaGraphExec_t merge_exec = nullptr;                         // replica-mode merge + shadow refresh
   std::vector<cudaEvent_t> prof_pool;
@@ -239,16 +249,19 @@ struct ProfScope {
   const char* name;
   cudaStream_t s;
   cudaEvent_t a = nullptr;
+  // an event record is an event node of the graph while a round is captured
+  // (prof_sink set), a plain record otherwise
+  unsigned flags() const { return c->prof_sink ? cudaEventRecordExternal : cudaEventRecordDefault; }
   ProfScope(oscars_ctx* c_, const char* n, cudaStream_t s_) : c(c_), name(n), s(s_) {
     if (c->profiling) {
       a = prof_event(c);
-      cudaEventRecordWithFlags(a, s, cudaEventRecordExternal);
+      cudaEventRecordWithFlags(a, s, flags());
     }
   }
   ~ProfScope() {
     if (a) {
       cudaEvent_t b = prof_event(c);
-      cudaEventRecordWithFlags(b, s, cudaEventRecordExternal);
+      cudaEventRecordWithFlags(b, s, flags());
       if (c->prof_sink)
         c->prof_sink->push_back({name, a, b, true});
       else
@@ -308,7 +321,7 @@ void free_all(oscars_ctx* c) {
       cudaEventDestroy(p.b);
     }
   c->prof_pending.clear();
-  for (auto* v : {&c->prof_round_graph, &c->prof_merge_graph}) {
+  for (auto* v : {&c->prof_round_graph, &c->prof_merge_graph, &c->prof_ahead_graph[0], &c->prof_ahead_graph[1]}) {
     for (auto& p : *v) {
       cudaEventDestroy(p.a);
       cudaEventDestroy(p.b);
@@ -321,6 +334,10 @@ void free_all(oscars_ctx* c) {
   c->prof_pool.clear();
   if (c->round_exec) cudaGraphExecDestroy(c->round_exec);
   c->round_exec = nullptr;
+  for (auto& g : c->ahead_exec) {
+    if (g) cudaGraphExecDestroy(g);
+    g = nullptr;
+  }
   for (void* p : c->allocs) cudaFree(p);
   c->allocs.clear();
   if (c->cap) cudaStreamDestroy(c->cap);
@@ -366,10 +383,19 @@ oscars_status ensure_stage_buffers(oscars_ctx* c) {
     return fail(c, OSCARS_ENOMEM, "device allocation failed (phase stamps)");
   if (c->fused) {
     const uint64_t per_b = static_cast<uint64_t>(per) * 2;
-    if (!make_map4(&c->mX4, c->A0all, D, B, W, cap, D * 2ull, static_cast<uint64_t>(B) * D * 2ull, per_b, B) ||
-        !make_map4(&c->mXT4, c->A0Tall, B, D, W, cap, B * 2ull, static_cast<uint64_t>(B) * D * 2ull, per_b,
-                   fused_round_xt_rows(B)))
-      return fail(c, OSCARS_ECUDA, "cuTensorMapEncodeTiled failed (fused round inputs)");
+    c->A0b[0] = c->A0all;
+    c->A0Tb[0] = c->A0Tall;
+    c->labb[0] = c->labels_all;
+    if (!dev_alloc(c, &c->A0b[1], per * cap) || !dev_alloc(c, &c->A0Tb[1], per * cap) ||
+        !dev_alloc(c, &c->labb[1], static_cast<size_t>(W) * B * cap))
+      return fail(c, OSCARS_ENOMEM, "device allocation failed (second input buffer)");
+    for (int i = 0; i < 2; ++i)
+      if (!make_map4(&c->mX4b[i], c->A0b[i], D, B, W, cap, D * 2ull, static_cast<uint64_t>(B) * D * 2ull, per_b, B) ||
+          !make_map4(&c->mXT4b[i], c->A0Tb[i], B, D, W, cap, B * 2ull, static_cast<uint64_t>(B) * D * 2ull, per_b,
+                     fused_round_xt_rows(B)))
+        return fail(c, OSCARS_ECUDA, "cuTensorMapEncodeTiled failed (fused round inputs)");
+    c->mX4 = c->mX4b[0];
+    c->mXT4 = c->mXT4b[0];
   }
   // step 0 doubles as the single-step buffers (evaluation)
   c->A[0] = c->A0all;
@@ -446,6 +472,16 @@ oscars_status build_tables(oscars_ctx* c) {
     cudaGraphExecDestroy(c->round_exec);
     c->round_exec = nullptr;
   }
+  for (int i = 0; i < 2; ++i) {
+    if (c->ahead_exec[i]) cudaGraphExecDestroy(c->ahead_exec[i]);
+    c->ahead_exec[i] = nullptr;
+    for (auto& p : c->prof_ahead_graph[i]) {   // the graph's event nodes go with it
+      cudaEventDestroy(p.a);
+      cudaEventDestroy(p.b);
+    }
+    c->prof_ahead_graph[i].clear();
+  }
+  c->staged = false;   // the staged next round used the previous tau
   if (c->merge_exec) {
     cudaGraphExecDestroy(c->merge_exec);
     c->merge_exec = nullptr;
@@ -593,10 +629,83 @@ cudaError_t enqueue_step(oscars_ctx* c, int s, int na, const int* wid, const int
   return cudaSuccess;
 }
 
+FusedRoundArgs fused_args(oscars_ctx* c) {
+  FusedRoundArgs f{};
+  f.tau = c->tau_dev;
+  f.order = c->order_dev;
+  f.W = c->W;
+  f.D = c->dims[0];
+  f.H = c->dims[1];
+  f.B = c->B;
+  f.global_slot = c->W;
+  f.lr = c->lr;
+  f.master = c->slab;
+  f.master_w = c->slab;
+  f.slot_stride = c->P_pad;
+  f.offW0 = c->layers[0].offW;
+  f.offB0 = c->layers[0].offB;
+  f.offW1 = c->layers[1].offW;
+  f.offB1 = c->layers[1].offB;
+  f.labels = c->labels_all;
+  f.max_tau = c->max_tau;
+  f.err = c->err;
+  f.phase_ts = (c->flags & 16) ? c->phase_ts : nullptr;
+  f.loss_out = c->loss_dev;
+  f.cursor = c->cursor;
+  f.shard_n = c->dn_tab;
+  return f;
+}
+
+StageArgs stage_args(oscars_ctx* c, int buf, const int32_t* ahead) {
+  StageArgs sa{};
+  sa.x = c->dx_tab;
+  sa.y = c->dy_tab;
+  sa.n = c->dn_tab;
+  sa.start = c->cursor;
+  sa.row_add = 0;
+  sa.wid = nullptr;
+  sa.D = c->dims[0];
+  sa.B = c->B;
+  sa.A0 = c->A0b[buf];
+  sa.A0T = c->A0Tb[buf];
+  sa.labels = c->labb[buf];
+  sa.ahead = ahead;
+  return sa;
+}
+
+// one-launch round from input buffer `buf` (staged earlier), then the staging
+// of the next round into the other buffer as a programmatic dependent (it
+// starts once the round's clusters have all started, on the SMs they leave
+// free), then the cursor advance
+cudaError_t enqueue_round_fused_ahead(oscars_ctx* c, int buf, cudaStream_t st) {
+  cudaError_t e;
+  FusedRoundArgs f = fused_args(c);
+  f.labels = c->labb[buf];
+  f.cursor = nullptr;   // advanced below, after the next round's rows were read
+  // while profiling the staging is a plain launch, and the round kernel's
+  // event must bracket the whole kernel: no early trigger then
+  f.trigger_dependents = c->profiling ? 0 : 1;
+  {
+    ProfScope ps(c, "fused_round", st);
+    if ((e = launch_fused_round(c->mX4b[buf], c->mXT4b[buf], f, false, st)) != cudaSuccess) return e;
+  }
+  {
+    // while profiling, a plain launch: event nodes around a kernel that lets
+    // its dependent start early would not bracket the whole kernel
+    ProfScope ps(c, "stage", st);
+    const StageArgs sa = stage_args(c, buf ^ 1, c->tau_dev);
+    e = c->profiling ? launch_stage_round(sa, c->tau_dev, c->W, c->max_tau, st)
+                     : launch_stage_round_dependent(sa, c->tau_dev, c->W, c->max_tau, st);
+    if (e != cudaSuccess) return e;
+  }
+  ProfScope ps(c, "round_bookkeeping", st);
+  return launch_cursor_advance(c->cursor, c->tau_dev, c->dn_tab, c->B, c->W, st);
+}
+
 cudaError_t enqueue_round_mlp(oscars_ctx* c, cudaStream_t st) {
   cudaError_t e;
   {
-    StageArgs sa;
+    StageArgs sa{};
     sa.x = c->dx_tab;
     sa.y = c->dy_tab;
     sa.n = c->dn_tab;
@@ -612,31 +721,9 @@ cudaError_t enqueue_round_mlp(oscars_ctx* c, cudaStream_t st) {
     if ((e = launch_stage_round(sa, c->tau_dev, c->W, c->max_tau, st)) != cudaSuccess) return e;
   }
   if (c->fused) {
-    FusedRoundArgs f;
-    f.tau = c->tau_dev;
-    f.order = c->order_dev;
-    f.W = c->W;
-    f.D = c->dims[0];
-    f.H = c->dims[1];
-    f.B = c->B;
-    f.global_slot = c->W;
-    f.lr = c->lr;
-    f.master = c->slab;
-    f.master_w = c->slab;
-    f.slot_stride = c->P_pad;
-    f.offW0 = c->layers[0].offW;
-    f.offB0 = c->layers[0].offB;
-    f.offW1 = c->layers[1].offW;
-    f.offB1 = c->layers[1].offB;
-    f.labels = c->labels_all;
-    f.max_tau = c->max_tau;
-    f.err = c->err;
-    f.phase_ts = (c->flags & 16) ? c->phase_ts : nullptr;
-    f.loss_out = c->loss_dev;
-    f.cursor = c->cursor;
-    f.shard_n = c->dn_tab;
+    FusedRoundArgs f = fused_args(c);
     ProfScope ps(c, "fused_round", st);
-    if ((e = launch_fused_round(c->mX4, c->mXT4, f, st)) != cudaSuccess) return e;
+    if ((e = launch_fused_round(c->mX4, c->mXT4, f, true, st)) != cudaSuccess) return e;
   } else {
     if (c->n_br > 1) {
       cudaError_t e2 = cudaEventRecord(c->br_fork, st);
@@ -708,7 +795,7 @@ cudaError_t enqueue_step_cnn(oscars_ctx* c, int s, int na, const int* wid, const
   const size_t wpl = static_cast<size_t>(c->W) * chunks * 9 * 64 * 64;          // weight partials per layer
   const size_t bpl = static_cast<size_t>(c->W) * tiles * 64;                    // bias partials per layer
   {
-    CnnStageArgs a;
+    CnnStageArgs a{};
     a.x = c->dx_tab;
     a.y = c->dy_tab;
     a.n = c->dn_tab;
@@ -1290,7 +1377,47 @@ oscars_status oscars_local_steps(oscars_ctx* c, int32_t* tau_out, float* loss_ou
   if (c->pending) return fail(c, OSCARS_ESTATE, "the previous round has not been merged");
   try {
     cudaError_t e = cudaSuccess;
-    if (c->flags & 1) {
+    if (c->fused) {
+      // the one-launch round: the first round (or the first after tau changed)
+      // stages its own mini-batches; every round stages the next one
+      const int buf = c->parity;
+      if (!c->staged) {
+        c->profiling = (c->flags & 2) != 0;
+        {
+          ProfScope ps(c, "stage", c->stream);
+          e = launch_stage_round(stage_args(c, buf, nullptr), c->tau_dev, c->W, c->max_tau, c->stream);
+        }
+        c->profiling = false;
+        if (e != cudaSuccess) return cuda_fail(c, e, "local steps launch");
+      }
+      if (c->flags & 1) {
+        c->profiling = (c->flags & 2) != 0;
+        e = enqueue_round_fused_ahead(c, buf, c->stream);
+        c->profiling = false;
+      } else {
+        if (!c->ahead_exec[buf]) {
+          cudaGraph_t g = nullptr;
+          c->profiling = (c->flags & 2) != 0;
+          c->prof_sink = &c->prof_ahead_graph[buf];   // empty: this parity's graph does not exist yet
+          e = cudaStreamBeginCapture(c->cap, cudaStreamCaptureModeThreadLocal);
+          if (e == cudaSuccess) {
+            cudaError_t e2 = enqueue_round_fused_ahead(c, buf, c->cap);
+            e = cudaStreamEndCapture(c->cap, &g);
+            if (e2 != cudaSuccess) e = e2;
+          }
+          c->profiling = false;
+          c->prof_sink = nullptr;
+          if (e == cudaSuccess) e = cudaGraphInstantiateWithFlags(&c->ahead_exec[buf], g, 0);
+          if (g) cudaGraphDestroy(g);
+        }
+        if (e == cudaSuccess) e = cudaGraphLaunch(c->ahead_exec[buf], c->stream);
+        if (e == cudaSuccess) prof_after_replay(c, c->prof_ahead_graph[buf]);
+      }
+      if (e == cudaSuccess) {
+        c->staged = true;
+        c->parity = buf ^ 1;
+      }
+    } else if (c->flags & 1) {
       c->profiling = (c->flags & 2) != 0;
       e = enqueue_round(c, c->stream);
       c->profiling = false;
@@ -1541,7 +1668,7 @@ oscars_status oscars_eval_loss(oscars_ctx* c, const float* x, const int32_t* y, 
       if (e == cudaSuccess) e = cudaMemcpyAsync(c->en_tab, &nc, sizeof(int64_t), cudaMemcpyHostToDevice, c->stream);
       if (e == cudaSuccess) e = cudaStreamSynchronize(c->stream);   // the host values above must not go out of scope early
       if (e != cudaSuccess) break;
-      CnnStageArgs a;
+      CnnStageArgs a{};
       a.x = c->ex_tab;
       a.y = c->ey_tab;
       a.n = c->en_tab;
@@ -1622,7 +1749,7 @@ oscars_status oscars_eval_loss(oscars_ctx* c, const float* x, const int32_t* y, 
     if (e == cudaSuccess) e = cudaMemcpy(c->en_tab, ns.data(), c->W * sizeof(int64_t), cudaMemcpyHostToDevice);
     for (int64_t base = 0; e == cudaSuccess && base < chunks; base += c->W) {
       const int na = static_cast<int>(std::min<int64_t>(c->W, chunks - base));
-      StageArgs sa;
+      StageArgs sa{};
       sa.x = c->ex_tab;
       sa.y = c->ey_tab;
       sa.n = c->en_tab;
@@ -1649,6 +1776,7 @@ oscars_status oscars_eval_loss(oscars_ctx* c, const float* x, const int32_t* y, 
     if (e == cudaSuccess)
       e = launch_sum_scaled(c->eval_part, chunks * nc, 1.0 / static_cast<double>(n), c->loss_dev, c->stream);
   }
+  if (c->model == OSCARS_MODEL_MLP && c->L >= 2) c->staged = false;   // eval used the first input buffer
   if (e == cudaSuccess) e = cudaStreamSynchronize(c->stream);
   if (e == cudaSuccess) e = cudaMemcpy(loss, c->loss_dev, sizeof(float), cudaMemcpyDeviceToHost);
   if (e != cudaSuccess) return cuda_fail(c, e, "eval");

@@ -54,9 +54,11 @@
 // fence.proxy.async.  Arithmetic and rounding points are those of the
 // per-layer path (the pair's two partial sums are added in rank order).
 //
-// The kernel is launched as a programmatic dependent of the staging grid:
-// TMEM allocation and the model load overlap the staging, and it waits for
-// the staging grid (griddepcontrol.wait) before touching a staged tile.
+// The kernel may be launched as a programmatic dependent of the staging grid
+// (TMEM allocation and the model load overlap the staging; it waits for the
+// staging grid with griddepcontrol.wait before touching a staged tile), and it
+// lets its own programmatic dependent (the staging of the next round into the
+// other buffer) start once all its CTAs have started.
 //
 // Clusters are launched in order of decreasing tau (a table maps cluster to
 // worker): when fewer clusters fit on the GPU than there are workers, the
@@ -185,6 +187,7 @@ struct FusedArgs {
   float* loss_out;                // [W]
   int64_t* cursor;                // [W]
   const int64_t* shard_n;         // [W]
+  int trigger_dependents;         // let a programmatic dependent start once all CTAs started
 };
 
 template <int B, int S>
@@ -250,6 +253,9 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
   const int64_t dof = static_cast<int64_t>(w) * a.slot_stride;
 
   if (t == 0) {
+    // a grid launched as this kernel's programmatic dependent (the staging of
+    // the next round) may start once every CTA of this grid has started
+    if (a.trigger_dependents) asm volatile("griddepcontrol.launch_dependents;");
     prefetch_tmap(&mX);
     prefetch_tmap(&mXT);
     for (int i = 0; i < Cfg::kStagesF; ++i) {
@@ -715,7 +721,7 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
   // round bookkeeping of this worker: mean loss over its steps and the data cursor
   if (rank == 0 && t == 0) {
     a.loss_out[w] = static_cast<float>(loss_sum / (static_cast<double>(B) * tau));
-    a.cursor[w] = (a.cursor[w] + static_cast<int64_t>(tau) * B) % a.shard_n[w];
+    if (a.cursor) a.cursor[w] = (a.cursor[w] + static_cast<int64_t>(tau) * B) % a.shard_n[w];
   }
   tc_fence_before();
   __syncthreads();
@@ -726,7 +732,8 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
 }
 
 template <int B, int S>
-cudaError_t launch_bs(const CUtensorMap& mX, const CUtensorMap& mXT, const FusedArgs& a, cudaStream_t s) {
+cudaError_t launch_bs(const CUtensorMap& mX, const CUtensorMap& mXT, const FusedArgs& a, bool dependent,
+                      cudaStream_t s) {
   using Cfg = FCfg<B, S>;
   cudaError_t e = cudaFuncSetAttribute(fused_mlp2_round_kernel<B, S>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        Cfg::kSmem);
@@ -745,7 +752,7 @@ cudaError_t launch_bs(const CUtensorMap& mX, const CUtensorMap& mXT, const Fused
   attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 2;
+  cfg.numAttrs = dependent ? 2 : 1;
   return cudaLaunchKernelEx(&cfg, fused_mlp2_round_kernel<B, S>, mX, mXT, a);
 }
 
@@ -775,7 +782,7 @@ bool fused_round_supported(int L, int D, int H, int C, int B) {
 
 int fused_round_xt_rows(int) { return kND; }
 
-cudaError_t launch_fused_round(const CUtensorMap& mX, const CUtensorMap& mXT, const FusedRoundArgs& r,
+cudaError_t launch_fused_round(const CUtensorMap& mX, const CUtensorMap& mXT, const FusedRoundArgs& r, bool dependent,
                                cudaStream_t s) {
   FusedArgs a;
   a.tau = r.tau;
@@ -799,9 +806,12 @@ cudaError_t launch_fused_round(const CUtensorMap& mX, const CUtensorMap& mXT, co
   a.loss_out = r.loss_out;
   a.cursor = r.cursor;
   a.shard_n = r.shard_n;
+  a.trigger_dependents = r.trigger_dependents;
   const int S = split_for(r.D, r.H);
-  if (r.B == 32) return S == 2 ? launch_bs<32, 2>(mX, mXT, a, s) : launch_bs<32, 1>(mX, mXT, a, s);
-  if (r.B == 64) return S == 2 ? launch_bs<64, 2>(mX, mXT, a, s) : launch_bs<64, 1>(mX, mXT, a, s);
+  if (r.B == 32)
+    return S == 2 ? launch_bs<32, 2>(mX, mXT, a, dependent, s) : launch_bs<32, 1>(mX, mXT, a, dependent, s);
+  if (r.B == 64)
+    return S == 2 ? launch_bs<64, 2>(mX, mXT, a, dependent, s) : launch_bs<64, 1>(mX, mXT, a, dependent, s);
   return cudaErrorInvalidValue;
 }
 

@@ -87,7 +87,7 @@ __global__ void __launch_bounds__(256) stage_round_kernel(const __grid_constant_
   __nv_bfloat16* A0T = a.A0T + off;
   const float* X = a.x[w];
   const int64_t n = a.n[w];
-  const int64_t base = a.start[w] + static_cast<int64_t>(s) * a.B;
+  const int64_t base = a.start[w] + (static_cast<int64_t>(s) + (a.ahead ? a.ahead[w] : 0)) * a.B;
   const int k0 = blockIdx.x * kStageCols, b0 = blockIdx.y * kStageRows;
   const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;   // 32 x 8
   const int k = k0 + tx * 4;
@@ -654,6 +654,20 @@ cudaError_t launch_stage(const StageArgs& a, int n_active, cudaStream_t s) {
   dim3 grid((a.D + 31) / 32, (a.B + 31) / 32, n_active);
   stage_kernel<<<grid, 256, 0, s>>>(a);
   return cudaGetLastError();
+}
+
+cudaError_t launch_stage_round_dependent(const StageArgs& a, const int32_t* tau, int W, int max_tau, cudaStream_t s) {
+  if (a.D % 4 != 0 || a.B % 16 != 0) return cudaErrorInvalidValue;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3((a.D + kStageCols - 1) / kStageCols, (a.B + kStageRows - 1) / kStageRows, W * max_tau);
+  cfg.blockDim = dim3(256, 1, 1);
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, stage_round_kernel, a, tau, W);
 }
 
 cudaError_t launch_stage_round(const StageArgs& a, const int32_t* tau, int W, int max_tau, cudaStream_t s) {
