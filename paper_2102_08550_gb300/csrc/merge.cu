@@ -24,7 +24,7 @@ namespace oscars {
 namespace {
 
 constexpr int kThreads = 256;
-constexpr int kGroup = 8;
+constexpr int kGroup = 16;   // replica loads in flight per thread before the first is used
 
 __device__ __forceinline__ float4 ld_stream4(const float4* p) { return __ldcs(p); }
 
