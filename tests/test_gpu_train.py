@@ -381,3 +381,56 @@ def test_losses_async_matches_synchronous_read(cuda_device):
         np.testing.assert_array_equal(buf.numpy(), np.asarray(loss, np.float32))
         ctx.push_merge()
     ctx.close()
+
+
+def test_round_kernel_restaging_between_rounds(cuda_device):
+    """The one-launch round stages the next round's mini-batches while it
+    runs.  Between rounds: an evaluation (which reuses the first input
+    buffer), a tau override, new iteration times (Algorithm 1 again) and a
+    plain round; the staged data must follow every change.  Against the
+    oracle driven through the same changes."""
+    from oracle import schedule as osched
+    w = synth.TrainWorkload("restage", 4, [784, 512, 10], 64, 0.05, 1024, 8, 1)
+    ctx, layers0 = make_context(w, device_shards(w, cuda_device, n=w.samples_per_worker), cuda_device,
+                                flags=P.FLAG_PROFILE)
+    Xe, ye = synth.eval_np(w, n=128)
+    ex, ey = torch.from_numpy(Xe).to(cuda_device), torch.from_numpy(ye).to(cuda_device)
+    t0 = oracle_schedule(w)[0]
+    t_new = (t0[::-1]).copy()                      # the speeds swap
+    plan = ["round", "eval", "round", "tau", "round", "ticks", "round", "round"]
+    gpu_flats, gpu_losses = [], []
+    for op in plan:
+        if op == "round":
+            _, loss = ctx.local_steps()
+            ctx.push_merge()
+            gpu_losses.append(np.array(loss))
+            gpu_flats.append(pull_flat(ctx, cuda_device))
+        elif op == "eval":
+            ctx.eval_loss(ex, ey)
+        elif op == "tau":
+            ctx.set_local_steps([2, 1, 3, 1])
+        elif op == "ticks":
+            ctx.set_iteration_ticks(t_new.tolist())
+    assert "fused_round" in ctx.profile()
+    ctx.close()
+
+    def oracle_run():
+        state = orun.init_state(w.dims, layers0, t0, w.M)
+        shards_h = oracle_inputs(w, w.samples_per_worker)
+        flats, losses = [], []
+        for op in plan:
+            if op == "round":
+                rec = orun.run_round(state, shards_h, w.batch, w.lr, obf16.round_bf16)
+                flats.append(rec.x_g)
+                losses.append(rec.worker_loss)
+            elif op == "tau":
+                state.tau = np.array([2, 1, 3, 1], np.int32)
+                state.T_star = osched.round_barrier(state.t_iter, state.tau)
+            elif op == "ticks":
+                orun.reschedule(state, t_new, w.M)
+        return flats, losses
+    ref, ref_losses = oracle_run()
+    env = envelope(lambda: oracle_run()[0], w.dims, ref)
+    for r in range(len(ref)):
+        np.testing.assert_allclose(gpu_losses[r], ref_losses[r], rtol=LOSS_RTOL)
+        assert_within(per_tensor_errors(gpu_flats[r], ref[r], w.dims), env[r], f"round {r}")
