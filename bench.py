@@ -38,6 +38,7 @@ import numpy as np  # noqa: E402
 import synth  # noqa: E402
 
 WORKLOAD = synth.CFG2
+WORKLOADS = {w.name: w for w in (synth.CFG2, synth.CFG3)}
 METRIC = "simulated-worker samples/s (Oscars rounds; merge GB/s alongside)"
 UNIT = "samples/s"
 
@@ -48,6 +49,9 @@ def parse():
     ap.add_argument("--steps", type=int, default=30)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="oscars", choices=["oscars", "reference"])
+    ap.add_argument("--workload", default=WORKLOAD.name, choices=sorted(WORKLOADS),
+                    help="MLP workload of the round benchmark (default: the 784-512-10 headline); the "
+                         "server-merge microbenchmarks run with the headline only")
     ap.add_argument("--no-merge", action="store_true", help="skip the merge microbenchmarks")
     ap.add_argument("--no-cpu", action="store_true", help="skip the CPU oracle baseline")
     ap.add_argument("--no-e2e", action="store_true")
@@ -197,7 +201,7 @@ def roofline_of(name, ms_per_launch, launches_per_round, flops, bytes_, hbm, tfl
     if t_flop >= t_mem:
         ach = f / t / 1e12
         return {"kernel": name, "bound": "tensor", "achieved": ach, "peak": tflops, "unit": "TFLOP/s",
-                "frac": ach / tflops, "peak_kind": f"{peak_kind} bf16 dense (burst)", "flops_per_launch": f,
+                "frac": ach / tflops, "peak_kind": f"{peak_kind} bf16 dense (sustained)", "flops_per_launch": f,
                 "bytes_per_launch": b, "ms_per_launch": ms_per_launch, "traffic": None}
     ach = b / t / 1e9
     return {"kernel": name, "bound": "hbm", "achieved": ach, "peak": hbm, "unit": "GB/s", "frac": ach / hbm,
@@ -229,7 +233,7 @@ def run_gpu(args, rank, world, local_rank):
     _build.build()
     dev = torch.device(f"cuda:{local_rank}")
     torch.cuda.set_device(dev)
-    w = WORKLOAD
+    w = WORKLOADS[args.workload]
     hbm, tf_burst, tf_sus, peak_kind = peaks()
     T_star, mw, tau = schedule_of(w)
     samples_per_round = int(np.sum(tau)) * w.batch
@@ -291,10 +295,20 @@ def run_gpu(args, rank, world, local_rank):
     kernels = {}
     tot = sum(x[0] for x in prof.values())
     for k, (ms, cnt) in prof.items():
-        r = roofline_of(k, ms / cnt, cnt / prof_rounds, flops, bytes_, hbm, tf_burst, peak_kind)
+        r = roofline_of(k, ms / cnt, cnt / prof_rounds, flops, bytes_, hbm, tf_sus, peak_kind)
         kernels[k] = {"ms_per_round": ms / prof_rounds, "launches_per_round": cnt / prof_rounds,
                       "share": ms / tot, "bound": r["bound"], "frac": r["frac"]}
-    roof = roofline_of(dom, prof[dom][0] / prof[dom][1], prof[dom][1] / prof_rounds, flops, bytes_, hbm, tf_burst,
+        if flops.get(k, 0.0) > 0.0:     # every kernel that does tensor work: its fraction of the tensor peak
+            tf = flops[k] / (ms / prof_rounds / 1e3) / 1e12
+            kernels[k]["tflops"] = tf
+            kernels[k]["tensor_frac"] = tf / tf_sus
+    gemm = [k for k in kernels if k.startswith("gemm_")]
+    if gemm:                            # the grouped worker GEMMs together
+        g_ms = sum(prof[k][0] for k in gemm) / prof_rounds
+        g_tf = sum(flops[k] for k in gemm) / (g_ms / 1e3) / 1e12
+        kernels["all_gemms"] = {"ms_per_round": g_ms, "share": g_ms * prof_rounds / tot, "tflops": g_tf,
+                                "tensor_frac": g_tf / tf_sus}
+    roof = roofline_of(dom, prof[dom][0] / prof[dom][1], prof[dom][1] / prof_rounds, flops, bytes_, hbm, tf_sus,
                        peak_kind)
 
     # ---- end to end through the C ABI with host-resident inputs
@@ -324,48 +338,34 @@ def run_e2e(args, shards, w, tau, dev, stream, world=1):
     ctx = P.OscarsContext(num_workers=w.num_workers, dims=w.dims, batch=w.batch, lr=w.lr,
                           speed=synth.speeds(w).tolist(), M=w.M, shards=host, init_params=init,
                           stream=stream.cuda_stream)
-    # warm-up: one full pass over every shard (at least W rounds).  The first
-    # touch of each pinned host page costs extra once per process; the timed
-    # rounds measure the steady state and the first pass is reported beside it.
+    # warm-up: one full pass over every shard.  The first touch of each
+    # pinned host page costs extra once per process; the timed rounds measure
+    # the steady state and the first pass is reported beside it.
     samples = int(np.sum(tau)) * w.batch
-    epoch = max(int(np.ceil(w.samples_per_worker / (int(t) * w.batch))) for t in tau)
+    epoch = max(3, args.warmup, max(int(np.ceil(w.samples_per_worker / (int(t) * w.batch))) for t in tau))
     torch.cuda.synchronize()
     t0 = time.perf_counter()
-    for _ in range(max(3, args.warmup, epoch)):
-        P.oscars_local_steps(ctx.handle, want_tau=False, want_loss=True)
-        P.oscars_push_merge(ctx.handle)
-    torch.cuda.synchronize()
-    first_pass = samples * max(3, args.warmup, epoch) / (time.perf_counter() - t0)
-    # timed rounds, pipelined one deep: round r is enqueued (with the async
-    # copy of its W losses into pinned host memory) before the host waits for
-    # round r - 1 and reads that round's losses
+    ctx.train(epoch)
+    first_pass = samples * epoch / (time.perf_counter() - t0)
+    # timed: one oscars_train call, the API a user trains with.  Every round
+    # its W per-worker losses are copied to pinned host memory and read by the
+    # host (the library pipelines the rounds one deep).
     steps = max(200, args.steps)      # a wall-clock measurement: tens of milliseconds, not a few
-    lbuf = [torch.empty(w.num_workers, dtype=torch.float32).pin_memory() for _ in range(2)]
-    done = [torch.cuda.Event() for _ in range(2)]
-    seen = []
+    torch.cuda.synchronize()
     t0 = time.perf_counter()
-    for r in range(steps):
-        P.oscars_local_steps(ctx.handle, want_tau=False, want_loss=False)
-        P.oscars_losses_async(ctx.handle, lbuf[r % 2].data_ptr())      # D2H of the round's W losses
-        P.oscars_push_merge(ctx.handle)
-        done[r % 2].record(stream)
-        if r >= 1:
-            done[(r - 1) % 2].synchronize()
-            seen.append(float(lbuf[(r - 1) % 2].sum()))
-    done[(steps - 1) % 2].synchronize()
-    seen.append(float(lbuf[(steps - 1) % 2].sum()))
+    log = ctx.train(steps)
     dt = max_over_ranks(time.perf_counter() - t0, world, dev)
-    assert len(seen) == steps and all(np.isfinite(seen))
+    assert len(log) == steps and all(np.isfinite(r["worker_loss"]) for r in log)
     ctx.close()
     h2d = samples * (w.dims[0] * 4 + 4)
     return {"value": whole_job_rate(samples * steps, world, dt * 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
-            "d2h_bytes_per_step": 4 * w.num_workers, "steps": steps, "warmup_rounds": max(3, args.warmup, epoch),
+            "d2h_bytes_per_step": 4 * w.num_workers, "steps": steps, "warmup_rounds": epoch,
             "first_pass_value": first_pass,
-            "note": "host wall clock; shards in pinned host memory read by the staging kernel each round "
-                    "(host->device), local steps + merge, every round's per-worker losses copied to pinned host "
-                    "memory and read by the host one round later (rounds pipelined one deep); timed after one "
-                    "warm-up pass over every shard (first_pass_value: that pass, synchronous rounds, including "
-                    "the first touch of every pinned page)"}
+            "note": "host wall clock around one oscars_train call; shards in pinned host memory read by the "
+                    "staging kernel each round (host->device), local steps + merge, every round's per-worker "
+                    "losses copied to pinned host memory and read by the host (rounds pipelined one deep in the "
+                    "library); timed after one warm-up pass over every shard (first_pass_value: that pass, "
+                    "including the first touch of every pinned page)"}
 
 
 def merge_workloads(args):
@@ -645,7 +645,7 @@ def run_cnn(args, dev):
 
 
 def run_reference(args):
-    w = WORKLOAD
+    w = WORKLOADS[args.workload]
     oracle_rounds(w, max(1, min(args.warmup, 2)), 30.0)          # warm-up (imports, caches)
     samples, dt, done = oracle_rounds(w, args.steps, 120.0)
     value = samples / dt
@@ -701,16 +701,16 @@ def main():
         hbm, _, _, kind = peaks()
         print(json.dumps({"merge": run_merge(args, dev, torch.cuda.current_stream(dev), hbm, kind)}))
         return
-    if args.only == "round":
+    if args.only == "round" or args.workload != WORKLOAD.name:
         args.no_merge = True
     res = run_gpu(args, rank, world, local_rank)
+    w = WORKLOADS[args.workload]
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu:
-        samples, dt, done = oracle_rounds(WORKLOAD, 6, 15.0)
+        samples, dt, done = oracle_rounds(w, 6, 15.0)
         cpu = {"value": samples / dt, "unit": UNIT, "cores": cores_used(), "kind": "oracle",
-               "sample": f"{done} Oscars rounds of {WORKLOAD.name} (numpy fp64 with bf16 operand emulation)"}
+               "sample": f"{done} Oscars rounds of {w.name} (numpy fp64 with bf16 operand emulation)"}
     if rank == 0:
-        w = WORKLOAD
         line = {"metric": METRIC, "value": res["value"], "unit": UNIT, "n_gpus": world, "steps": args.steps,
                 "warmup": args.warmup, "ms_per_step": res["ms_per_step"], "higher_is_better": True,
                 "scaling": "weak", "vs_baseline": None, "dtype": "bf16 (fp32 master, fp32 accumulate)",

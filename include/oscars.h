@@ -262,9 +262,15 @@ typedef struct {
  * With eval and target_loss > 0 it stops after the first round whose eval
  * loss is <= target_loss (the time-to-loss of the paper's convergence
  * comparison).  log: host array of `rounds` entries or NULL; rounds_done
- * (host, may be NULL) receives the number of rounds run.  Synchronises every
- * round (it reads the losses).  Errors: those of the calls it makes; EINVAL
- * for rounds < 1 or eval_n < 1 with eval_x set.
+ * (host, may be NULL) receives the number of rounds run.  With eval_x it
+ * synchronises every round (it reads the losses and the eval loss).  Without
+ * eval_x the rounds are pipelined one deep: round r, with an asynchronous
+ * copy of its W losses into a pinned host slot, is enqueued before the host
+ * waits for round r - 1 and reads that round's losses; the call returns after
+ * the last round's losses were read.  Errors: those of the calls it makes;
+ * EINVAL for rounds < 1 or eval_n < 1 with eval_x set; ETIMEOUT when a
+ * kernel's bounded wait ran out in any round (without eval_x, reported after
+ * the last round).
  */
 oscars_status oscars_train(oscars_ctx* ctx, int32_t rounds, const float* eval_x, const int32_t* eval_y,
                            int64_t eval_n, float target_loss, oscars_round_log* log,

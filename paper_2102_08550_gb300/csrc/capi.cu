@@ -158,7 +158,6 @@ struct oscars_ctx {
   int32_t* labels_all = nullptr;
   std::vector<CUtensorMap> mA0s, mAT0s;
   bool fused = false;                   // whole-round kernel (2-layer MLP)
-  CUtensorMap mX4, mXT4;                // staged inputs of every step (fused kernel)
   // the one-launch round stages the next round while the current one runs:
   // two input buffers, used alternately (index `parity` holds the next round)
   __nv_bfloat16* A0b[2] = {};
@@ -192,6 +191,11 @@ struct oscars_ctx {
   std::vector<cudaStream_t> br_streams;
   std::vector<cudaEvent_t> br_join;
   cudaEvent_t br_fork = nullptr;
+  // one-launch rounds: the next round's staging runs beside the round on a
+  // side stream, at the lowest launch priority (the round at the highest)
+  cudaStream_t side = nullptr;
+  cudaEvent_t side_fork = nullptr, side_join = nullptr;
+  int prio_least = 0, prio_greatest = 0;
   std::vector<int> br_max_tau;          // [n_br]
   std::vector<int> br_na;               // [n_br][max_tau] active workers per step
   int* br_wid = nullptr;                // [n_br][max_tau][W]
@@ -216,6 +220,10 @@ struct oscars_ctx {
   std::vector<double> prof_ms;
   std::vector<int> prof_count;
   bool profiling = false;
+  // oscars_train without evaluation: two pinned host slots for the per-worker
+  // losses and one event per slot (rounds pipelined one deep)
+  float* train_loss_host = nullptr;
+  cudaEvent_t train_done[2] = {nullptr, nullptr};
 };
 
 namespace {
@@ -332,6 +340,12 @@ void free_all(oscars_ctx* c) {
   c->merge_exec = nullptr;
   for (cudaEvent_t e : c->prof_pool) cudaEventDestroy(e);
   c->prof_pool.clear();
+  for (auto& e : c->train_done) {
+    if (e) cudaEventDestroy(e);
+    e = nullptr;
+  }
+  if (c->train_loss_host) cudaFreeHost(c->train_loss_host);
+  c->train_loss_host = nullptr;
   if (c->round_exec) cudaGraphExecDestroy(c->round_exec);
   c->round_exec = nullptr;
   for (auto& g : c->ahead_exec) {
@@ -348,6 +362,12 @@ void free_all(oscars_ctx* c) {
   c->br_join.clear();
   if (c->br_fork) cudaEventDestroy(c->br_fork);
   c->br_fork = nullptr;
+  if (c->side) cudaStreamDestroy(c->side);
+  c->side = nullptr;
+  for (auto* e : {&c->side_fork, &c->side_join}) {
+    if (*e) cudaEventDestroy(*e);
+    *e = nullptr;
+  }
 }
 
 // Simulated barrier and idle time per worker for the current tau (Eq. 1).
@@ -394,8 +414,6 @@ oscars_status ensure_stage_buffers(oscars_ctx* c) {
           !make_map4(&c->mXT4b[i], c->A0Tb[i], B, D, W, cap, B * 2ull, static_cast<uint64_t>(B) * D * 2ull, per_b,
                      fused_round_xt_rows(B)))
         return fail(c, OSCARS_ECUDA, "cuTensorMapEncodeTiled failed (fused round inputs)");
-    c->mX4 = c->mX4b[0];
-    c->mXT4 = c->mXT4b[0];
   }
   // step 0 doubles as the single-step buffers (evaluation)
   c->A[0] = c->A0all;
@@ -673,33 +691,42 @@ StageArgs stage_args(oscars_ctx* c, int buf, const int32_t* ahead) {
   return sa;
 }
 
-// one-launch round from input buffer `buf` (staged earlier), then the staging
-// of the next round into the other buffer as a programmatic dependent (it
-// starts once the round's clusters have all started, on the SMs they leave
-// free), then the cursor advance
+// one-launch round from input buffer `buf` (staged earlier) and, beside it,
+// the staging of the next round into the other buffer followed by the cursor
+// advance.  The staging forks onto the side stream at the lowest launch
+// priority and the round kernel launches at the highest, so the staging
+// reads its rows (from host memory, for host-resident shards) on the SMs
+// the round's clusters leave free from the round's start, and a cluster
+// still waiting to start takes an SM before any staging block does.  While
+// profiling, everything runs in sequence on `st` so that the event pairs
+// bracket whole kernels.
 cudaError_t enqueue_round_fused_ahead(oscars_ctx* c, int buf, cudaStream_t st) {
   cudaError_t e;
   FusedRoundArgs f = fused_args(c);
   f.labels = c->labb[buf];
   f.cursor = nullptr;   // advanced below, after the next round's rows were read
-  // while profiling the staging is a plain launch, and the round kernel's
-  // event must bracket the whole kernel: no early trigger then
-  f.trigger_dependents = c->profiling ? 0 : 1;
-  {
-    ProfScope ps(c, "fused_round", st);
-    if ((e = launch_fused_round(c->mX4b[buf], c->mXT4b[buf], f, false, st)) != cudaSuccess) return e;
+  const StageArgs sa = stage_args(c, buf ^ 1, c->tau_dev);
+  if (c->profiling) {
+    {
+      ProfScope ps(c, "fused_round", st);
+      if ((e = launch_fused_round(c->mX4b[buf], c->mXT4b[buf], f, st)) != cudaSuccess) return e;
+    }
+    {
+      ProfScope ps(c, "stage", st);
+      if ((e = launch_stage_round(sa, c->tau_dev, c->W, c->max_tau, st)) != cudaSuccess) return e;
+    }
+    ProfScope ps(c, "round_bookkeeping", st);
+    return launch_cursor_advance(c->cursor, c->tau_dev, c->dn_tab, c->B, c->W, st);
   }
-  {
-    // while profiling, a plain launch: event nodes around a kernel that lets
-    // its dependent start early would not bracket the whole kernel
-    ProfScope ps(c, "stage", st);
-    const StageArgs sa = stage_args(c, buf ^ 1, c->tau_dev);
-    e = c->profiling ? launch_stage_round(sa, c->tau_dev, c->W, c->max_tau, st)
-                     : launch_stage_round_dependent(sa, c->tau_dev, c->W, c->max_tau, st);
-    if (e != cudaSuccess) return e;
-  }
-  ProfScope ps(c, "round_bookkeeping", st);
-  return launch_cursor_advance(c->cursor, c->tau_dev, c->dn_tab, c->B, c->W, st);
+  if ((e = cudaEventRecord(c->side_fork, st)) != cudaSuccess) return e;
+  if ((e = cudaStreamWaitEvent(c->side, c->side_fork, 0)) != cudaSuccess) return e;
+  f.priority = c->prio_greatest;
+  if ((e = launch_fused_round(c->mX4b[buf], c->mXT4b[buf], f, st)) != cudaSuccess) return e;
+  if ((e = launch_stage_round_priority(sa, c->tau_dev, c->W, c->max_tau, c->prio_least, c->side)) != cudaSuccess)
+    return e;
+  if ((e = launch_cursor_advance(c->cursor, c->tau_dev, c->dn_tab, c->B, c->W, c->side)) != cudaSuccess) return e;
+  if ((e = cudaEventRecord(c->side_join, c->side)) != cudaSuccess) return e;
+  return cudaStreamWaitEvent(st, c->side_join, 0);
 }
 
 cudaError_t enqueue_round_mlp(oscars_ctx* c, cudaStream_t st) {
@@ -720,11 +747,7 @@ cudaError_t enqueue_round_mlp(oscars_ctx* c, cudaStream_t st) {
     ProfScope ps(c, "stage", st);
     if ((e = launch_stage_round(sa, c->tau_dev, c->W, c->max_tau, st)) != cudaSuccess) return e;
   }
-  if (c->fused) {
-    FusedRoundArgs f = fused_args(c);
-    ProfScope ps(c, "fused_round", st);
-    if ((e = launch_fused_round(c->mX4, c->mXT4, f, true, st)) != cudaSuccess) return e;
-  } else {
+  {
     if (c->n_br > 1) {
       cudaError_t e2 = cudaEventRecord(c->br_fork, st);
       if (e2 != cudaSuccess) return e2;
@@ -743,7 +766,6 @@ cudaError_t enqueue_round_mlp(oscars_ctx* c, cudaStream_t st) {
       }
     }
   }
-  if (c->fused) return cudaSuccess;   // the round kernel did its own bookkeeping
   const int nc = c->B / kRowsPerLossChunk;
   ProfScope ps(c, "round_bookkeeping", st);
   if ((e = launch_loss_finalize(c->loss_part, c->tau_dev, c->W, c->max_tau, nc, c->B, c->loss_dev, st)) != cudaSuccess)
@@ -1338,6 +1360,12 @@ oscars_status oscars_create(const oscars_config* cfg, oscars_ctx** out) {
         }
         if (st == OSCARS_OK && c->n_br > 1 && cudaEventCreateWithFlags(&c->br_fork, cudaEventDisableTiming) != cudaSuccess)
           st = fail(c, OSCARS_ECUDA, "event creation failed");
+        if (st == OSCARS_OK && c->fused &&
+            (cudaDeviceGetStreamPriorityRange(&c->prio_least, &c->prio_greatest) != cudaSuccess ||
+             cudaStreamCreateWithFlags(&c->side, cudaStreamNonBlocking) != cudaSuccess ||
+             cudaEventCreateWithFlags(&c->side_fork, cudaEventDisableTiming) != cudaSuccess ||
+             cudaEventCreateWithFlags(&c->side_join, cudaEventDisableTiming) != cudaSuccess))
+          st = fail(c, OSCARS_ECUDA, "stream creation failed");
       } else {
         c->flags = cfg->flags;
         if (!dev_alloc(c, &c->slab, c->P_pad)) st = fail(c, OSCARS_ENOMEM, "device allocation failed (global model)");
@@ -1846,6 +1874,56 @@ oscars_status oscars_profile_reset(oscars_ctx* c) {
   return OSCARS_OK;
 }
 
+namespace {
+
+// oscars_train without evaluation: round r (local steps, the asynchronous copy
+// of its W losses into a pinned host slot, push + merge) is enqueued before
+// the host waits for round r - 1 and reads that round's losses, so the host
+// work of one round overlaps the device work of the next.
+oscars_status train_pipelined(oscars_ctx* c, int32_t rounds, oscars_round_log* log, int32_t* rounds_done) {
+  if (!c->train_loss_host) {
+    cudaError_t e = cudaHostAlloc(&c->train_loss_host, 2 * sizeof(float) * c->W, cudaHostAllocDefault);
+    if (e != cudaSuccess) {
+      c->train_loss_host = nullptr;
+      return cuda_fail(c, e, "train loss buffer");
+    }
+    for (auto& ev : c->train_done)
+      if ((e = cudaEventCreateWithFlags(&ev, cudaEventDisableTiming)) != cudaSuccess) return cuda_fail(c, e, "train event");
+  }
+  auto finish = [&](int32_t r) -> oscars_status {
+    const cudaError_t e = cudaEventSynchronize(c->train_done[r & 1]);
+    if (e != cudaSuccess) return cuda_fail(c, e, "train round");
+    if (log) {
+      const float* l = c->train_loss_host + (r & 1) * c->W;
+      double m = 0.0;
+      for (int i = 0; i < c->W; ++i) m += l[i];
+      log[r].worker_loss = static_cast<float>(m / c->W);
+    }
+    if (rounds_done) *rounds_done = r + 1;
+    return OSCARS_OK;
+  };
+  for (int32_t r = 0; r < rounds; ++r) {
+    oscars_status st = oscars_local_steps(c, nullptr, nullptr);
+    if (st == OSCARS_OK) st = oscars_losses_async(c, c->train_loss_host + (r & 1) * c->W);
+    if (st == OSCARS_OK) st = oscars_push_merge(c, nullptr, nullptr);
+    if (st != OSCARS_OK) return st;
+    if (log) {
+      log[r].ticks = *std::max_element(c->clock.begin(), c->clock.end());
+      log[r].barrier = c->barrier;
+      log[r].eval_loss = std::numeric_limits<float>::quiet_NaN();
+    }
+    const cudaError_t e = cudaEventRecord(c->train_done[r & 1], c->stream);
+    if (e != cudaSuccess) return cuda_fail(c, e, "train event");
+    if (r >= 1 && (st = finish(r - 1)) != OSCARS_OK) return st;
+  }
+  const oscars_status st = finish(rounds - 1);
+  // the kernels' error word is sticky: one read after the last round reports
+  // a bounded wait that ran out in any of them
+  return st == OSCARS_OK ? check_err_word(c) : st;
+}
+
+}  // namespace
+
 oscars_status oscars_train(oscars_ctx* c, int32_t rounds, const float* eval_x, const int32_t* eval_y,
                            int64_t eval_n, float target_loss, oscars_round_log* log, int32_t* rounds_done) {
   if (rounds_done) *rounds_done = 0;
@@ -1853,6 +1931,7 @@ oscars_status oscars_train(oscars_ctx* c, int32_t rounds, const float* eval_x, c
   if (eval_x && (!eval_y || eval_n < 1)) return OSCARS_EINVAL;
   if (c->rule == OSCARS_W_EXPLICIT) return fail(c, OSCARS_EINVAL, "train merges with the context's rule; explicit weights need push_merge");
   try {
+    if (!eval_x) return train_pipelined(c, rounds, log, rounds_done);
     std::vector<float> wl(c->W);
     for (int32_t r = 0; r < rounds; ++r) {
       oscars_status st = oscars_local_steps(c, nullptr, wl.data());

@@ -54,11 +54,8 @@
 // fence.proxy.async.  Arithmetic and rounding points are those of the
 // per-layer path (the pair's two partial sums are added in rank order).
 //
-// The kernel may be launched as a programmatic dependent of the staging grid
-// (TMEM allocation and the model load overlap the staging; it waits for the
-// staging grid with griddepcontrol.wait before touching a staged tile), and it
-// lets its own programmatic dependent (the staging of the next round into the
-// other buffer) start once all its CTAs have started.
+// The staging of the next round into the other input buffer runs beside
+// the kernel at a lower launch priority, on the SMs its clusters leave free.
 //
 // Clusters are launched in order of decreasing tau (a table maps cluster to
 // worker): when fewer clusters fit on the GPU than there are workers, the
@@ -187,7 +184,6 @@ struct FusedArgs {
   float* loss_out;                // [W]
   int64_t* cursor;                // [W]
   const int64_t* shard_n;         // [W]
-  int trigger_dependents;         // let a programmatic dependent start once all CTAs started
 };
 
 template <int B, int S>
@@ -253,9 +249,6 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
   const int64_t dof = static_cast<int64_t>(w) * a.slot_stride;
 
   if (t == 0) {
-    // a grid launched as this kernel's programmatic dependent (the staging of
-    // the next round) may start once every CTA of this grid has started
-    if (a.trigger_dependents) asm volatile("griddepcontrol.launch_dependents;");
     prefetch_tmap(&mX);
     prefetch_tmap(&mXT);
     for (int i = 0; i < Cfg::kStagesF; ++i) {
@@ -363,9 +356,6 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
-  // the staged mini-batches, labels and cursors are the staging grid's: wait
-  // for it (a no-op without programmatic dependent launch)
-  asm volatile("griddepcontrol.wait;" ::: "memory");
   if (warp == 0 && lane == 0) producer_ok = issue_f(0, 0, pre_f);
 
   for (int s = 0; s < tau; ++s) {
@@ -732,7 +722,7 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
 }
 
 template <int B, int S>
-cudaError_t launch_bs(const CUtensorMap& mX, const CUtensorMap& mXT, const FusedArgs& a, bool dependent,
+cudaError_t launch_bs(const CUtensorMap& mX, const CUtensorMap& mXT, const FusedArgs& a, int priority,
                       cudaStream_t s) {
   using Cfg = FCfg<B, S>;
   cudaError_t e = cudaFuncSetAttribute(fused_mlp2_round_kernel<B, S>, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -744,15 +734,19 @@ cudaError_t launch_bs(const CUtensorMap& mX, const CUtensorMap& mXT, const Fused
   cfg.dynamicSmemBytes = Cfg::kSmem;
   cfg.stream = s;
   cudaLaunchAttribute attr[2];
-  attr[0].id = cudaLaunchAttributeClusterDimension;
-  attr[0].val.clusterDim.x = 1;
-  attr[0].val.clusterDim.y = S * (a.H / kFU);
-  attr[0].val.clusterDim.z = 1;
-  // may start before the staging grid ends (it waits for it after loading the model)
-  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[1].val.programmaticStreamSerializationAllowed = 1;
+  int n = 0;
+  attr[n].id = cudaLaunchAttributeClusterDimension;
+  attr[n].val.clusterDim.x = 1;
+  attr[n].val.clusterDim.y = S * (a.H / kFU);
+  attr[n].val.clusterDim.z = 1;
+  ++n;
+  if (priority != 0) {   // ahead of concurrent work (the next round's staging) for free SMs
+    attr[n].id = cudaLaunchAttributePriority;
+    attr[n].val.priority = priority;
+    ++n;
+  }
   cfg.attrs = attr;
-  cfg.numAttrs = dependent ? 2 : 1;
+  cfg.numAttrs = n;
   return cudaLaunchKernelEx(&cfg, fused_mlp2_round_kernel<B, S>, mX, mXT, a);
 }
 
@@ -782,8 +776,7 @@ bool fused_round_supported(int L, int D, int H, int C, int B) {
 
 int fused_round_xt_rows(int) { return kND; }
 
-cudaError_t launch_fused_round(const CUtensorMap& mX, const CUtensorMap& mXT, const FusedRoundArgs& r, bool dependent,
-                               cudaStream_t s) {
+cudaError_t launch_fused_round(const CUtensorMap& mX, const CUtensorMap& mXT, const FusedRoundArgs& r, cudaStream_t s) {
   FusedArgs a;
   a.tau = r.tau;
   a.order = r.order;
@@ -806,12 +799,11 @@ cudaError_t launch_fused_round(const CUtensorMap& mX, const CUtensorMap& mXT, co
   a.loss_out = r.loss_out;
   a.cursor = r.cursor;
   a.shard_n = r.shard_n;
-  a.trigger_dependents = r.trigger_dependents;
   const int S = split_for(r.D, r.H);
   if (r.B == 32)
-    return S == 2 ? launch_bs<32, 2>(mX, mXT, a, dependent, s) : launch_bs<32, 1>(mX, mXT, a, dependent, s);
+    return S == 2 ? launch_bs<32, 2>(mX, mXT, a, r.priority, s) : launch_bs<32, 1>(mX, mXT, a, r.priority, s);
   if (r.B == 64)
-    return S == 2 ? launch_bs<64, 2>(mX, mXT, a, dependent, s) : launch_bs<64, 1>(mX, mXT, a, dependent, s);
+    return S == 2 ? launch_bs<64, 2>(mX, mXT, a, r.priority, s) : launch_bs<64, 1>(mX, mXT, a, r.priority, s);
   return cudaErrorInvalidValue;
 }
 

@@ -74,8 +74,20 @@ __device__ __forceinline__ void epi_fwd(const GemmArgs& a, int wid, int src, int
   for (int q = 0; q < 4; ++q) outT[q] = make_uint4(pk[4 * q], pk[4 * q + 1], pk[4 * q + 2], pk[4 * q + 3]);
 }
 
-__device__ __forceinline__ float epi_dh(const GemmArgs& a, int wid, int m, int n0, const float (&v)[32]) {
-  const __nv_bfloat16* hm = a.hmask + static_cast<int64_t>(wid) * a.N * a.M;
+// The input-gradient epilogue's ReLU mask for 32 columns: mk[c] = the raw
+// bf16 bits of Hmask[n0 + c][m].  All 32 loads are issued before any is
+// used, and the caller issues the next chunk's loads before it stores the
+// current one, so the mask reads of a thread overlap instead of waiting
+// one by one behind its stores.
+__device__ __forceinline__ void epi_dh_mask(const GemmArgs& a, int wid, int m, int n0, unsigned short (&mk)[32]) {
+  const unsigned short* hm = reinterpret_cast<const unsigned short*>(a.hmask) +
+                             static_cast<int64_t>(wid) * a.N * a.M + static_cast<int64_t>(n0) * a.M + m;
+#pragma unroll
+  for (int c = 0; c < 32; ++c) mk[c] = __ldg(hm + static_cast<int64_t>(c) * a.M);
+}
+
+__device__ __forceinline__ float epi_dh(const GemmArgs& a, int wid, int m, int n0, const float (&v)[32],
+                                        const unsigned short (&mk)[32]) {
   __nv_bfloat16* out = a.out + static_cast<int64_t>(wid) * a.N * a.M;
   uint32_t pk[16];
   float gsum = 0.f;
@@ -83,8 +95,8 @@ __device__ __forceinline__ float epi_dh(const GemmArgs& a, int wid, int m, int n
   for (int c = 0; c < 32; c += 2) {
     const int64_t e0 = static_cast<int64_t>(n0 + c) * a.M + m;
     const int64_t e1 = e0 + a.M;
-    const float g0 = __bfloat162float(hm[e0]) > 0.f ? v[c] : 0.f;
-    const float g1 = __bfloat162float(hm[e1]) > 0.f ? v[c + 1] : 0.f;
+    const float g0 = __bfloat162float(__ushort_as_bfloat16(mk[c])) > 0.f ? v[c] : 0.f;
+    const float g1 = __bfloat162float(__ushort_as_bfloat16(mk[c + 1])) > 0.f ? v[c + 1] : 0.f;
     gsum += g0;
     gsum += g1;
     const __nv_bfloat162 p = __floats2bfloat162_rn(g0, g1);
@@ -248,6 +260,15 @@ __global__ void __launch_bounds__(warps_for<EPI>() * 32) gemm_tc_kernel(const __
   __syncwarp();
 
   // epilogue: thread = one accumulator row
+  unsigned short mk[32];   // input-gradient mask of the next 32 columns, read while the MMAs run
+  if constexpr (EPI == kEpiDh) epi_dh_mask(a, wid, m0 + (warp & 3) * 32 + lane, n0, mk);
+  float4 old0[8], old1[8];  // weight-gradient epilogue: the fp32 master block, read while the MMAs run
+  if constexpr (EPI == kEpiDw) {
+    const int c_begin = (warp >> 2) * (BN / 2);
+    const int mb = m0 + (warp & 3) * 32;
+    epi_dw_load(a, src, mb, n0 + c_begin, lane, old0);
+    epi_dw_load(a, src, mb, n0 + c_begin + 32, lane, old1);
+  }
   int acc_ok = mbar_wait(accum, 0, a.err, kDevTimeoutAccum) ? 1 : 0;
   acc_ok = __all_sync(0xffffffffu, acc_ok);
   tc_fence_after();
@@ -260,9 +281,6 @@ __global__ void __launch_bounds__(warps_for<EPI>() * 32) gemm_tc_kernel(const __
       const int c_begin = (warp >> 2) * (BN / 2);
       const int mb = m0 + quarter * 32;
       float* T = epi_tiles + warp * kEpiTileFloats;
-      float4 old0[8], old1[8];
-      epi_dw_load(a, src, mb, n0 + c_begin, lane, old0);        // both chunks' loads in flight
-      epi_dw_load(a, src, mb, n0 + c_begin + 32, lane, old1);
       if (n0 + c_begin < a.N) {
         float v[32];
         tmem_ld_32x32b_x32(trow + c_begin, v);
@@ -278,21 +296,30 @@ __global__ void __launch_bounds__(warps_for<EPI>() * 32) gemm_tc_kernel(const __
         a.master_w[static_cast<int64_t>(wid) * a.slot_stride + bo] =
             fmaf(-a.lr, a.gb_in[static_cast<int64_t>(wid) * a.M + m], a.master[static_cast<int64_t>(src) * a.slot_stride + bo]);
       }
-    } else {
+    } else if constexpr (EPI == kEpiDh) {
       float gsum = 0.f;
+#pragma unroll
+      for (int c0 = 0; c0 < BN; c0 += 32) {
+        float v[32];
+        tmem_ld_32x32b_x32(trow + c0, v);
+        unsigned short cur[32];
+#pragma unroll
+        for (int c = 0; c < 32; ++c) cur[c] = mk[c];
+        if (c0 + 32 < BN) epi_dh_mask(a, wid, m, n0 + c0 + 32, mk);
+        gsum += epi_dh(a, wid, m, n0 + c0, v, cur);
+      }
+      a.gb_out[static_cast<int64_t>(wid) * a.M + m] = gsum;
+    } else {
 #pragma unroll 1
       for (int c0 = 0; c0 < BN; c0 += 32) {
         float v[32];
         tmem_ld_32x32b_x32(trow + c0, v);
         if (EPI == kEpiFwd) {
           epi_fwd<EPI>(a, wid, src, m, n0 + c0, v);
-        } else if (EPI == kEpiDh) {
-          gsum += epi_dh(a, wid, m, n0 + c0, v);
         } else if (EPI == kEpiStore) {
           if (n0 + c0 < a.N) epi_store(a, m, n0 + c0, v);
         }
       }
-      if (EPI == kEpiDh) a.gb_out[static_cast<int64_t>(wid) * a.M + m] = gsum;
     }
   }
   tc_fence_before();

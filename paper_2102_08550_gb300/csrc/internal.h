@@ -82,9 +82,9 @@ struct StageArgs {
 cudaError_t launch_stage(const StageArgs& a, int n_active, cudaStream_t s);
 // all mini-batches of a round: step s of worker w (s < tau[w]) at slot s * W + w
 cudaError_t launch_stage_round(const StageArgs& a, const int32_t* tau, int W, int max_tau, cudaStream_t s);
-// the same, launched as a programmatic dependent of the preceding kernel on `s`
-// (it may start once that kernel's CTAs have all started)
-cudaError_t launch_stage_round_dependent(const StageArgs& a, const int32_t* tau, int W, int max_tau, cudaStream_t s);
+// the same with a launch priority (cudaLaunchAttributePriority)
+cudaError_t launch_stage_round_priority(const StageArgs& a, const int32_t* tau, int W, int max_tau, int priority,
+                                        cudaStream_t s);
 
 enum GemmEpi { kEpiFwd = 0, kEpiDh = 1, kEpiDw = 2, kEpiStore = 3 };
 
@@ -161,7 +161,7 @@ struct FusedRoundArgs {
   float* loss_out;                // [W] mean mini-batch loss of the round (written at the end)
   int64_t* cursor;                // [W] advanced by tau * B modulo n at the end, or null
   const int64_t* shard_n;         // [W]
-  int trigger_dependents;         // 1: a programmatic dependent follows (the next round's staging)
+  int priority;                   // launch priority (cudaLaunchAttributePriority); 0: the stream's
 };
 // whole-round kernel for input -> H ReLU -> 10 classes (one cluster per
 // worker, the worker's model resident on chip for the round)
@@ -170,10 +170,7 @@ int fused_round_xt_rows(int B);   // rows of the X^T box the kernel loads
 // mX: staged inputs {D, B, W, steps} box {64, B}; mXT: staged transposed
 // inputs {B, D, W, steps} box {64, fused_round_xt_rows(B)}; both bf16,
 // 128-byte swizzle
-// dependent: launched as a programmatic dependent of the staging grid that
-// precedes it on `s` (it waits for that grid before reading a staged tile)
-cudaError_t launch_fused_round(const CUtensorMap& mX, const CUtensorMap& mXT, const FusedRoundArgs& a, bool dependent,
-                               cudaStream_t s);
+cudaError_t launch_fused_round(const CUtensorMap& mX, const CUtensorMap& mXT, const FusedRoundArgs& a, cudaStream_t s);
 
 // loss[w] = sum_{s < tau[w]} sum_c part[(w*max_tau + s)*nc + c] / (B * tau[w])
 cudaError_t launch_loss_finalize(const float* part, const int32_t* tau, int W, int max_tau,

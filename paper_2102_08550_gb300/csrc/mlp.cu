@@ -74,10 +74,6 @@ constexpr int kStageRows = 32, kStageCols = 128;
 __global__ void __launch_bounds__(256) stage_round_kernel(const __grid_constant__ StageArgs a, const int32_t* tau,
                                                           int W) {
   __shared__ __align__(16) __nv_bfloat16 tile[kStageCols][kStageRows + 8];
-  // the round kernel that consumes these tiles may launch now (programmatic
-  // dependent launch: it loads the model first and waits for this grid
-  // before reading any staged tile)
-  asm volatile("griddepcontrol.launch_dependents;");
   const int z = blockIdx.z;
   const int s = z / W, w = z - s * W;
   if (s >= tau[w]) return;
@@ -92,16 +88,22 @@ __global__ void __launch_bounds__(256) stage_round_kernel(const __grid_constant_
   const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;   // 32 x 8
   const int k = k0 + tx * 4;
   const bool kok = k < a.D;
+  // all of this thread's rows are loaded before any is stored: the shards may
+  // sit in host memory, where every load waits a round trip over the link
+  float4 xv[kStageRows / 8];
+#pragma unroll
+  for (int i = 0; i < kStageRows / 8; ++i) {
+    const int b = b0 + ty + 8 * i;
+    xv[i] = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (b < a.B && kok) xv[i] = *reinterpret_cast<const float4*>(X + ((base + b) % n) * a.D + k);
+  }
 #pragma unroll
   for (int i = 0; i < kStageRows / 8; ++i) {
     const int r = ty + 8 * i, b = b0 + r;
-    float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
-    if (b < a.B && kok) {
-      const int64_t row = (base + b) % n;
-      v = *reinterpret_cast<const float4*>(X + row * a.D + k);
+    const float4 v = xv[i];
+    if (b < a.B && kok)
       *reinterpret_cast<uint2*>(A0 + static_cast<int64_t>(b) * a.D + k) =
           make_uint2(pack_bf16x2(v.x, v.y), pack_bf16x2(v.z, v.w));
-    }
     tile[tx * 4 + 0][r] = __float2bfloat16_rn(v.x);
     tile[tx * 4 + 1][r] = __float2bfloat16_rn(v.y);
     tile[tx * 4 + 2][r] = __float2bfloat16_rn(v.z);
@@ -359,63 +361,65 @@ __global__ void __launch_bounds__(kHeadBwdThreads) head_bwd_kernel(const __grid_
 //     values), then the softmax cross-entropy without cancellation;
 //  3. a second cluster barrier (no CTA leaves while others read its partials);
 //  4. masked input gradient of the layer below for its features: item =
-//     (row, 4 features), the 4 x C old weights stay in registers -> bf16 G,
-//     G^T (through shared memory) and the fp32 bias gradient;
+//     (2 features, 8 rows), the 2 x C old weights in registers -> bf16 G
+//     (4 bytes per row), G^T (16 bytes per feature) and the fp32 bias
+//     gradient;
 //  5. head weight gradient + SGD: item = (class, 4 features).
 // Rank 0 also writes the loss partials and updates the head bias.
+// The h tile stays bf16 in shared memory (about 60 KB per CTA at B = 128),
+// so several clusters share an SM and all active lanes run in one wave.
 constexpr int kHF = 128;                 // hidden features per CTA
 constexpr int kHFThreads = 256;
 constexpr int kHFWarps = kHFThreads / 32;
 constexpr int kHFMaxCluster = 8;
 constexpr int kHFClasses = 10;           // the fused path's class count
+constexpr int kHFPairs = kHF / 2;        // phase 4: feature pairs ...
+constexpr int kHFRowGroups = kHFThreads / kHFPairs;   // ... x interleaved groups of 8-row blocks
 
-// threads per row in phase 1 and the padded row stride of the h tile (row
-// stride / 4 == threads per row (mod 8): the 16-byte reads of one 8-lane
-// phase hit distinct banks)
+// threads per row in phase 1 and the row stride of the bf16 h tile in
+// elements (stride / 2 = 4 (mod 32) words: the 8-byte reads of rows r and
+// r + 1 land 4 banks apart, so 8 rows x 2 threads cover the 32 banks once)
 __host__ __device__ constexpr int hf_tpr(int B) { return B >= 256 ? 1 : kHFThreads / B; }
-__host__ __device__ constexpr int hf_stride(int B) { return kHF + 4 * hf_tpr(B); }
+constexpr int kHFStride = kHF + 8;
 
 size_t head_fused_smem(int B, int C) {
-  return sizeof(float) * (static_cast<size_t>(B) * hf_stride(B) + static_cast<size_t>(C) * kHF +
-                          3 * static_cast<size_t>(B) * C + kHFWarps * kHF + B) +
-         sizeof(__nv_bfloat16) * static_cast<size_t>(kHF) * (B + 8);
+  return sizeof(__nv_bfloat16) * static_cast<size_t>(B) * kHFStride +
+         sizeof(float) * (static_cast<size_t>(C) * kHF + 3 * static_cast<size_t>(B) * C + kHFRowGroups * kHF + B);
+}
+
+// 4 bf16 of the h tile as floats
+__device__ __forceinline__ float4 hf_ld4(const __nv_bfloat16* p) {
+  const uint2 v = *reinterpret_cast<const uint2*>(p);
+  const float2 lo = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&v.x));
+  const float2 hi = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&v.y));
+  return make_float4(lo.x, lo.y, hi.x, hi.y);
 }
 
 template <int C>
 __global__ void __launch_bounds__(kHFThreads) head_fused_kernel(const __grid_constant__ HeadArgs a) {
-  extern __shared__ __align__(16) float fsm[];
+  extern __shared__ __align__(16) float hfsm[];
   const int H = a.H, B = a.B;
-  const int hsd = hf_stride(B);
-  float* hs = fsm;                         // [B][hsd] bf16 h as float
-  float* wcs = hs + B * hsd;               // [C][kHF] old bf16 head weights as float
+  __nv_bfloat16* hs = reinterpret_cast<__nv_bfloat16*>(hfsm);  // [B][kHFStride] bf16 h
+  float* wcs = reinterpret_cast<float*>(hs + B * kHFStride);   // [C][kHF] old bf16 head weights as float
   float* pl = wcs + C * kHF;               // [B][C] partial logits (read by the cluster)
   float* dz = pl + B * C;                  // [B][C] logits, then dlogits fp32
   float* dzb = dz + B * C;                 // [B][C] bf16-rounded dlogits
-  float* gbp = dzb + B * C;                // [kHFWarps][kHF] bias-gradient partials
-  float* rowloss = gbp + kHFWarps * kHF;   // [B]
-  __nv_bfloat16* gts = reinterpret_cast<__nv_bfloat16*>(rowloss + B);   // [kHF][B + 8]
-  const int gts_ld = B + 8;
+  float* gbp = dzb + B * C;                // [kHFRowGroups][kHF] bias-gradient partials
+  float* rowloss = gbp + kHFRowGroups * kHF;   // [B]
   const int i = blockIdx.x;
   const int w = a.wid[i], src = a.src[i];
   const uint32_t rank = cluster_ctarank();
   const int ncl = static_cast<int>(gridDim.y);
   const int k0 = blockIdx.y * kHF;
-  const int t = threadIdx.x, lane = t & 31, warp = t >> 5;
+  const int t = threadIdx.x;
   const int64_t so = static_cast<int64_t>(src) * a.slot_stride;
   const int64_t dof = static_cast<int64_t>(w) * a.slot_stride;
   const __nv_bfloat16* h = a.Ain + static_cast<int64_t>(w) * B * H;
 
   for (int q = t; q < B * (kHF / 8); q += kHFThreads) {
     const int b = q / (kHF / 8), c8 = (q % (kHF / 8)) * 8;
-    const uint4 v = *reinterpret_cast<const uint4*>(h + static_cast<int64_t>(b) * H + k0 + c8);
-    const __nv_bfloat162* p2 = reinterpret_cast<const __nv_bfloat162*>(&v);
-    float4 lo, hi;
-    float2 f = __bfloat1622float2(p2[0]); lo.x = f.x; lo.y = f.y;
-    f = __bfloat1622float2(p2[1]); lo.z = f.x; lo.w = f.y;
-    f = __bfloat1622float2(p2[2]); hi.x = f.x; hi.y = f.y;
-    f = __bfloat1622float2(p2[3]); hi.z = f.x; hi.w = f.y;
-    *reinterpret_cast<float4*>(hs + b * hsd + c8) = lo;
-    *reinterpret_cast<float4*>(hs + b * hsd + c8 + 4) = hi;
+    *reinterpret_cast<uint4*>(hs + b * kHFStride + c8) =
+        *reinterpret_cast<const uint4*>(h + static_cast<int64_t>(b) * H + k0 + c8);
   }
   for (int q = t; q < C * (kHF / 8); q += kHFThreads) {
     const int c = q / (kHF / 8), c8 = (q % (kHF / 8)) * 8;
@@ -439,7 +443,7 @@ __global__ void __launch_bounds__(kHFThreads) head_fused_kernel(const __grid_con
 #pragma unroll
       for (int c = 0; c < C; ++c) acc[c] = 0.f;
       for (int k = 4 * q; k < kHF; k += 4 * tpr) {
-        const float4 hv = *reinterpret_cast<const float4*>(hs + rb * hsd + k);
+        const float4 hv = hf_ld4(hs + rb * kHFStride + k);
 #pragma unroll
         for (int c = 0; c < C; ++c) {
           const float4 wv = *reinterpret_cast<const float4*>(wcs + c * kHF + k);
@@ -513,58 +517,55 @@ __global__ void __launch_bounds__(kHFThreads) head_fused_kernel(const __grid_con
       if (j == 0) a.master_w[dof + a.offB + c] = fmaf(-a.lr, g, a.master[so + a.offB + c]);
     }
   }
-  // 4. masked input gradient of the layer below: item = (row, 4 features)
+  // 4. masked input gradient of the layer below: item = (2 features, 8 rows)
   {
-    const int k4 = (t & 31) * 4;           // this thread's 4 features
-    float4 wc[C];
+    const int kk = (t % kHFPairs) * 2;     // this thread's 2 features
+    const int rg = t / kHFPairs;
+    float2 wc[C];
 #pragma unroll
-    for (int c = 0; c < C; ++c) wc[c] = *reinterpret_cast<const float4*>(wcs + c * kHF + k4);
-    float4 gs = make_float4(0.f, 0.f, 0.f, 0.f);
-    __nv_bfloat16* G = a.G + static_cast<int64_t>(w) * B * H + k0 + k4;
-    for (int b = warp; b < B; b += kHFWarps) {
-      const float4 hv = *reinterpret_cast<const float4*>(hs + b * hsd + k4);
-      float4 dh = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int c = 0; c < C; ++c) wc[c] = *reinterpret_cast<const float2*>(wcs + c * kHF + kk);
+    float2 gs = make_float2(0.f, 0.f);
+    __nv_bfloat16* G = a.G + static_cast<int64_t>(w) * B * H + k0 + kk;
+    __nv_bfloat16* GT = a.GT + (static_cast<int64_t>(w) * H + k0 + kk) * B;
+    for (int b8 = rg * 8; b8 < B; b8 += kHFRowGroups * 8) {
+      uint32_t p0[4], p1[4];               // G^T rows kk and kk + 1 over these 8 rows
 #pragma unroll
-      for (int c = 0; c < C; ++c) {
-        const float g = dzb[b * C + c];
-        dh.x = fmaf(g, wc[c].x, dh.x);
-        dh.y = fmaf(g, wc[c].y, dh.y);
-        dh.z = fmaf(g, wc[c].z, dh.z);
-        dh.w = fmaf(g, wc[c].w, dh.w);
+      for (int r = 0; r < 8; ++r) {
+        const int b = b8 + r;
+        const float2 hv = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(hs + b * kHFStride + kk));
+        float2 dh = make_float2(0.f, 0.f);
+#pragma unroll
+        for (int c = 0; c < C; ++c) {
+          const float g = dzb[b * C + c];
+          dh.x = fmaf(g, wc[c].x, dh.x);
+          dh.y = fmaf(g, wc[c].y, dh.y);
+        }
+        dh.x = hv.x > 0.f ? dh.x : 0.f;
+        dh.y = hv.y > 0.f ? dh.y : 0.f;
+        gs.x += dh.x;
+        gs.y += dh.y;
+        const __nv_bfloat162 pr = __floats2bfloat162_rn(dh.x, dh.y);
+        *reinterpret_cast<__nv_bfloat162*>(G + static_cast<int64_t>(b) * H) = pr;
+        const uint32_t lo = __bfloat16_as_ushort(pr.x), hi = __bfloat16_as_ushort(pr.y);
+        if (r & 1) {
+          p0[r >> 1] |= lo << 16;
+          p1[r >> 1] |= hi << 16;
+        } else {
+          p0[r >> 1] = lo;
+          p1[r >> 1] = hi;
+        }
       }
-      dh.x = hv.x > 0.f ? dh.x : 0.f;
-      dh.y = hv.y > 0.f ? dh.y : 0.f;
-      dh.z = hv.z > 0.f ? dh.z : 0.f;
-      dh.w = hv.w > 0.f ? dh.w : 0.f;
-      gs.x += dh.x;
-      gs.y += dh.y;
-      gs.z += dh.z;
-      gs.w += dh.w;
-      const __nv_bfloat162 p01 = __floats2bfloat162_rn(dh.x, dh.y);
-      const __nv_bfloat162 p23 = __floats2bfloat162_rn(dh.z, dh.w);
-      *reinterpret_cast<uint2*>(G + static_cast<int64_t>(b) * H) =
-          make_uint2(*reinterpret_cast<const uint32_t*>(&p01), *reinterpret_cast<const uint32_t*>(&p23));
-      gts[(k4 + 0) * gts_ld + b] = p01.x;
-      gts[(k4 + 1) * gts_ld + b] = p01.y;
-      gts[(k4 + 2) * gts_ld + b] = p23.x;
-      gts[(k4 + 3) * gts_ld + b] = p23.y;
+      *reinterpret_cast<uint4*>(GT + b8) = make_uint4(p0[0], p0[1], p0[2], p0[3]);
+      *reinterpret_cast<uint4*>(GT + B + b8) = make_uint4(p1[0], p1[1], p1[2], p1[3]);
     }
-    *reinterpret_cast<float4*>(gbp + warp * kHF + k4) = gs;
+    *reinterpret_cast<float2*>(gbp + rg * kHF + kk) = gs;
   }
   __syncthreads();
   if (t < kHF) {
     float g = 0.f;
 #pragma unroll
-    for (int r = 0; r < kHFWarps; ++r) g += gbp[r * kHF + t];
+    for (int r = 0; r < kHFRowGroups; ++r) g += gbp[r * kHF + t];
     a.gb[static_cast<int64_t>(w) * H + k0 + t] = g;
-  }
-  {
-    uint4* GT = reinterpret_cast<uint4*>(a.GT + (static_cast<int64_t>(w) * H + k0) * B);
-    const int per_row = B / 8;
-    for (int q = t; q < kHF * per_row; q += kHFThreads) {
-      const int k = q / per_row, j = q - k * per_row;
-      GT[static_cast<int64_t>(k) * per_row + j] = *reinterpret_cast<const uint4*>(gts + k * gts_ld + j * 8);
-    }
   }
   // 5. head weight gradient + SGD: item = (class, 4 features)
   for (int q = t; q < C * (kHF / 4); q += kHFThreads) {
@@ -572,7 +573,7 @@ __global__ void __launch_bounds__(kHFThreads) head_fused_kernel(const __grid_con
     float4 dw = make_float4(0.f, 0.f, 0.f, 0.f);
     for (int b = 0; b < B; ++b) {
       const float g = dzb[b * C + c];
-      const float4 hv = *reinterpret_cast<const float4*>(hs + b * hsd + k4);
+      const float4 hv = hf_ld4(hs + b * kHFStride + k4);
       dw.x = fmaf(g, hv.x, dw.x);
       dw.y = fmaf(g, hv.y, dw.y);
       dw.z = fmaf(g, hv.z, dw.z);
@@ -656,15 +657,16 @@ cudaError_t launch_stage(const StageArgs& a, int n_active, cudaStream_t s) {
   return cudaGetLastError();
 }
 
-cudaError_t launch_stage_round_dependent(const StageArgs& a, const int32_t* tau, int W, int max_tau, cudaStream_t s) {
+cudaError_t launch_stage_round_priority(const StageArgs& a, const int32_t* tau, int W, int max_tau, int priority,
+                                        cudaStream_t s) {
   if (a.D % 4 != 0 || a.B % 16 != 0) return cudaErrorInvalidValue;
   cudaLaunchConfig_t cfg = {};
   cfg.gridDim = dim3((a.D + kStageCols - 1) / kStageCols, (a.B + kStageRows - 1) / kStageRows, W * max_tau);
   cfg.blockDim = dim3(256, 1, 1);
   cfg.stream = s;
   cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  attr[0].id = cudaLaunchAttributePriority;
+  attr[0].val.priority = priority;
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   return cudaLaunchKernelEx(&cfg, stage_round_kernel, a, tau, W);

@@ -383,6 +383,28 @@ def test_losses_async_matches_synchronous_read(cuda_device):
     ctx.close()
 
 
+@pytest.mark.parametrize("dims", [[784, 512, 10], [256, 256, 128, 10]], ids=["one-launch", "per-layer"])
+def test_train_without_eval_matches_round_by_round(cuda_device, dims):
+    """oscars_train without evaluation pipelines its rounds one deep; the
+    models and per-round losses must be those of the same rounds run one
+    call at a time (bit for bit: the same kernels in the same order)."""
+    w = synth.TrainWorkload("train-pipe", 4, dims, 64, 0.05, 512, 8, 5)
+    shards = device_shards(w, cuda_device, n=512)
+    a, _ = make_context(w, shards, cuda_device)
+    log = a.train(5)
+    assert len(log) == 5
+    b, _ = make_context(w, shards, cuda_device)
+    for r in range(5):
+        _, loss = b.local_steps()
+        b.push_merge()
+        assert log[r]["worker_loss"] == pytest.approx(float(np.mean(np.asarray(loss, np.float64))), rel=1e-6)
+        assert np.isnan(log[r]["eval_loss"])
+        assert log[r]["ticks"] == b.schedule()["clock"][0]
+    np.testing.assert_array_equal(pull_flat(a, cuda_device), pull_flat(b, cuda_device))
+    a.close()
+    b.close()
+
+
 def test_round_kernel_restaging_between_rounds(cuda_device):
     """The one-launch round stages the next round's mini-batches while it
     runs.  Between rounds: an evaluation (which reuses the first input
