@@ -189,7 +189,15 @@ def algorithmic_work(w, tau):
     return fl, by
 
 
-def roofline_of(name, ms_per_launch, launches_per_round, flops, bytes_, hbm, tflops, peak_kind):
+# DRAM bytes (dram__bytes_read.sum + dram__bytes_write.sum) per launch from one
+# ncu capture of the kernel as it stands, with the profile summary that holds
+# it; a kernel missing here reports traffic null.
+NCU_TRAFFIC = {
+    ("fused_round", "mlp-784-512-10-W16"): (15.97568e6, "profiles/fused_round_mlp784-512-10_W16.md"),
+}
+
+
+def roofline_of(name, ms_per_launch, launches_per_round, flops, bytes_, hbm, tflops, peak_kind, workload=None):
     f = flops.get(name, 0.0) / launches_per_round
     b = bytes_.get(name, 0.0) / launches_per_round
     t = ms_per_launch / 1e3
@@ -198,15 +206,18 @@ def roofline_of(name, ms_per_launch, launches_per_round, flops, bytes_, hbm, tfl
                 "ms_per_launch": ms_per_launch, "traffic": None}
     t_flop = f / (tflops * 1e12)
     t_mem = b / (hbm * 1e9)
+    tr = NCU_TRAFFIC.get((name, workload))
+    traffic = tr[0] if tr else None
     if t_flop >= t_mem:
         ach = f / t / 1e12
         return {"kernel": name, "bound": "tensor", "achieved": ach, "peak": tflops, "unit": "TFLOP/s",
                 "frac": ach / tflops, "peak_kind": f"{peak_kind} bf16 dense (sustained)", "flops_per_launch": f,
-                "bytes_per_launch": b, "ms_per_launch": ms_per_launch, "traffic": None}
+                "bytes_per_launch": b, "ms_per_launch": ms_per_launch, "traffic": traffic}
     ach = b / t / 1e9
     return {"kernel": name, "bound": "hbm", "achieved": ach, "peak": hbm, "unit": "GB/s", "frac": ach / hbm,
             "peak_kind": f"{peak_kind} HBM copy", "flops_per_launch": f, "bytes_per_launch": b,
-            "ms_per_launch": ms_per_launch, "traffic": None}
+            "ms_per_launch": ms_per_launch, "traffic": traffic,
+            "traffic_source": tr[1] if tr else None}
 
 
 def max_over_ranks(ms: float, world: int, device) -> float:
@@ -309,7 +320,7 @@ def run_gpu(args, rank, world, local_rank):
         kernels["all_gemms"] = {"ms_per_round": g_ms, "share": g_ms * prof_rounds / tot, "tflops": g_tf,
                                 "tensor_frac": g_tf / tf_sus}
     roof = roofline_of(dom, prof[dom][0] / prof[dom][1], prof[dom][1] / prof_rounds, flops, bytes_, hbm, tf_sus,
-                       peak_kind)
+                       peak_kind, w.name)
 
     # ---- end to end through the C ABI with host-resident inputs
     e2e = None
