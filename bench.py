@@ -162,10 +162,9 @@ def algorithmic_work(w, tau):
         by[k] = by.get(k, 0.0) + b
     for l in range(L - 1):            # hidden layers on the tensor cores
         i, o = d[l], d[l + 1]
-        T = 2 if 1 <= l <= L - 2 else 0
         add("gemm_fwd", n * 2 * B * i * o, n * (o * i * 2 + B * i * 2 + 2 * B * o * 2 + o * 4))
         add("gemm_dw_sgd", n * 2 * B * i * o,
-            n * (o * i * (4 + 4 + 2 + T) + o * B * 2 + i * B * 2 + o * (4 + 4 + 4)))
+            n * (o * i * (4 + 4 + 2) + o * B * 2 + i * B * 2 + o * (4 + 4 + 4)))
         if l >= 1:
             add("gemm_dh", n * 2 * B * i * o, n * (o * i * 2 + B * o * 2 + B * i * 2 + 2 * B * i * 2 + i * 4))
     H, C = d[L - 1], d[L]

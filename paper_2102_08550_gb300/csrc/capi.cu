@@ -7,9 +7,8 @@
 // Device memory of a context (MLP mode):
 //   slab    (W+1) slots x P_pad fp32   slots 0..W-1 worker replicas (the
 //                                      pushed models), slot W the global model
-//   shadow  (W+1) x P_pad bf16         bf16 copy of every slot (GEMM operand)
-//   shadowT (W+1) x PT_pad bf16        transposed bf16 copy of the middle
-//                                      layers (K-major operand of dX GEMMs)
+//   shadow  (W+1) x P_pad bf16         bf16 copy of every slot (GEMM operand;
+//                                      read MN-major by the input-gradient GEMM)
 //   per-worker activations, gradients, labels, loss partials, cursors.
 // Inside a slot every W_l and b_l starts on a 64-element boundary; the
 // padding stays zero.
@@ -94,9 +93,23 @@ bool make_map_box4(CUtensorMap* m, const void* base, const uint64_t (&d)[4], con
            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// 3-D fp32 tensor map, boxes of 32 x box_y x 1 (128-byte rows), 128-byte swizzle
+bool make_map_f32(CUtensorMap* m, const void* base, uint64_t dx, uint64_t dy, uint64_t dz, uint64_t stride_y,
+                  uint64_t stride_z, uint32_t box_y) {
+  EncodeTiledFn f = encode_fn();
+  if (!f) return false;
+  cuuint64_t dims[3] = {dx, dy, dz};
+  cuuint64_t strides[2] = {stride_y, stride_z};
+  cuuint32_t box[3] = {32, box_y, 1};
+  cuuint32_t es[3] = {1, 1, 1};
+  return f(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, const_cast<void*>(base), dims, strides, box, es,
+           CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+           CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 struct Layer {
   int in, out;
-  int64_t offW, offB, offT;  // offT < 0: no transposed copy
+  int64_t offW, offB;
 };
 
 }  // namespace
@@ -107,7 +120,7 @@ struct oscars_ctx {
   std::vector<int> dims;
   float lr = 0.f, server_lr = 1.f;
   int rule = 0, bf16 = 0, flags = 0;
-  int64_t P = 0, P_pad = 0, PT_pad = 0;
+  int64_t P = 0, P_pad = 0;
   std::vector<Layer> layers;
   // schedule (Eq. 1-3, Algorithm 1)
   std::vector<int64_t> t_iter, clock, idle;
@@ -123,7 +136,6 @@ struct oscars_ctx {
   std::vector<void*> allocs;
   float* slab = nullptr;
   __nv_bfloat16* shadow = nullptr;
-  __nv_bfloat16* shadowT = nullptr;
   std::vector<__nv_bfloat16*> A, AT, G, GT;  // per layer
   std::vector<float*> gb;
   int32_t* labels = nullptr;
@@ -150,7 +162,10 @@ struct oscars_ctx {
   float* eval_part = nullptr;
   int64_t eval_part_cap = 0;
   // tensor maps per layer
-  std::vector<CUtensorMap> mShadow, mShadowT, mA, mG, mGT, mAT;
+  std::vector<CUtensorMap> mShadow, mShadowMN, mA, mG, mGT, mAT;
+  // fp32 W_l of every slot: boxes {32, 128} (loads) and {32, 32} (stores), and
+  // the bf16 copy with boxes {64, 32} (stores): the persistent weight gradient
+  std::vector<CUtensorMap> mMaster, mMasterSt, mShadowSt;
   // per-step input buffers of layer 0 (a round's mini-batches are staged at once)
   int stage_cap = 0;
   __nv_bfloat16* A0all = nullptr;
@@ -520,12 +535,6 @@ cudaError_t refresh_global_shadows(oscars_ctx* c, cudaStream_t s, bool plain_don
                                c->cnn_offW[l], s);
     if (e != cudaSuccess) return e;
   }
-  for (const Layer& ly : c->layers) {
-    if (ly.offT < 0) continue;
-    e = launch_transpose_bf16(c->shadow + g + ly.offW,
-                              c->shadowT + static_cast<int64_t>(c->W) * c->PT_pad + ly.offT, ly.out, ly.in, s);
-    if (e != cudaSuccess) return e;
-  }
   return cudaSuccess;
 }
 
@@ -539,7 +548,6 @@ GemmArgs gemm_base(oscars_ctx* c, const int* wid, const int* src) {
   g.master_w = c->slab;
   g.shadow = c->shadow;
   g.slot_stride = c->P_pad;
-  g.slotT_stride = c->PT_pad;
   g.lr = c->lr;
   return g;
 }
@@ -628,7 +636,29 @@ cudaError_t enqueue_step(oscars_ctx* c, int s, int na, const int* wid, const int
       g.outT = c->GT[l - 1];
       g.gb_out = c->gb[l - 1];
       ProfScope ps(c, "gemm_dh", st);
-      if ((e = launch_gemm(kEpiDh, c->mShadowT[l], c->mG[l], g, na, st)) != cudaSuccess) return e;
+      if ((e = launch_gemm(kEpiDh, c->mShadowMN[l], c->mG[l], g, na, st)) != cudaSuccess) return e;
+    }
+    const CUtensorMap& mX = l == 0 ? c->mAT0s[s] : c->mAT[l];
+    if (gemm_dw_supported(ly.out, ly.in, c->B)) {
+      DwArgs d{};
+      d.wid = wid;
+      d.src = src;
+      d.n_active = na;
+      d.M = ly.out;
+      d.N = ly.in;
+      d.K = c->B;
+      d.lr = c->lr;
+      d.master = c->slab;
+      d.master_w = c->slab;
+      d.slot_stride = c->P_pad;
+      d.offB = ly.offB;
+      d.gb = c->gb[l];
+      d.err = c->err;
+      ProfScope ps(c, "gemm_dw_sgd", st);
+      if ((e = launch_gemm_dw(c->mGT[l], mX, c->mMaster[l], c->mMasterSt[l], c->mShadowSt[l], d, c->sms, st)) !=
+          cudaSuccess)
+        return e;
+      continue;
     }
     GemmArgs g = gemm_base(c, wid, src);
     g.M = ly.out;
@@ -638,11 +668,9 @@ cudaError_t enqueue_step(oscars_ctx* c, int s, int na, const int* wid, const int
     g.b_z_src = 0;
     g.offW = ly.offW;
     g.offB = ly.offB;
-    g.offT = ly.offT;
-    g.shadowT = ly.offT >= 0 ? c->shadowT : nullptr;
     g.gb_in = c->gb[l];
     ProfScope ps(c, "gemm_dw_sgd", st);
-    if ((e = launch_gemm(kEpiDw, c->mGT[l], l == 0 ? c->mAT0s[s] : c->mAT[l], g, na, st)) != cudaSuccess) return e;
+    if ((e = launch_gemm(kEpiDw, c->mGT[l], mX, g, na, st)) != cudaSuccess) return e;
   }
   return cudaSuccess;
 }
@@ -1056,7 +1084,7 @@ oscars_status validate_and_layout(oscars_ctx* c, const oscars_config* cfg) {
   } else {
     return fail(c, OSCARS_ENOTSUP, "supported: fp32 softmax regression (L=1) or bf16 MLP (L>=2)");
   }
-  int64_t off = 0, offT = 0;
+  int64_t off = 0;
   c->P = 0;
   for (int l = 0; l < c->L; ++l) {
     Layer ly;
@@ -1066,21 +1094,20 @@ oscars_status validate_and_layout(oscars_ctx* c, const oscars_config* cfg) {
     off += round_up(static_cast<int64_t>(ly.in) * ly.out, 64);
     ly.offB = off;
     off += round_up(ly.out, 64);
-    ly.offT = -1;
-    if (c->bf16 && l >= 1 && l <= c->L - 2) {
-      ly.offT = offT;
-      offT += round_up(static_cast<int64_t>(ly.in) * ly.out, 64);
-    }
     c->P += static_cast<int64_t>(ly.in) * ly.out + ly.out;
     c->layers.push_back(ly);
   }
   c->P_pad = round_up(off, 64);
-  c->PT_pad = round_up(offT, 64);
   return OSCARS_OK;
 }
 
 // the slab of W + 1 slots and the per-worker tables (MLP and CNN)
 oscars_status allocate_common(oscars_ctx* c) {
+  {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (cudaDeviceGetAttribute(&c->sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || c->sms < 1) c->sms = 1;
+  }
   const int W = c->W;
   const size_t slots = static_cast<size_t>(W) + 1;
   if (!dev_alloc(c, &c->slab, slots * c->P_pad)) return fail(c, OSCARS_ENOMEM, "device allocation failed (model slab)");
@@ -1128,11 +1155,6 @@ oscars_status allocate_cnn(oscars_ctx* c) {
   // tensor maps: activations {64 ch, 32 x, 32 y, images}; weights per slot
   c->cnn_m6.resize(nbuf);
   c->cnn_m4.resize(nbuf);
-  {
-    int dev = 0;
-    cudaGetDevice(&dev);
-    if (cudaDeviceGetAttribute(&c->sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || c->sms < 1) c->sms = 1;
-  }
   c->cnn_m2.resize(nbuf);
   const uint64_t imgs = static_cast<uint64_t>(W) * B;
   bool ok = true;
@@ -1171,10 +1193,6 @@ oscars_status allocate_mlp(oscars_ctx* c) {
 
   if (!dev_alloc(c, &c->shadow, slots * c->P_pad)) return fail(c, OSCARS_ENOMEM, "device allocation failed (bf16 shadow)");
   cudaMemset(c->shadow, 0, slots * c->P_pad * sizeof(__nv_bfloat16));
-  if (c->PT_pad > 0) {
-    if (!dev_alloc(c, &c->shadowT, slots * c->PT_pad)) return fail(c, OSCARS_ENOMEM, "device allocation failed (bf16 shadow^T)");
-    cudaMemset(c->shadowT, 0, slots * c->PT_pad * sizeof(__nv_bfloat16));
-  }
   c->A.assign(L, nullptr);
   c->AT.assign(L, nullptr);
   c->G.assign(L, nullptr);
@@ -1196,7 +1214,10 @@ oscars_status allocate_mlp(oscars_ctx* c) {
 
   // tensor maps
   c->mShadow.resize(L);
-  c->mShadowT.resize(L);
+  c->mMaster.resize(L);
+  c->mMasterSt.resize(L);
+  c->mShadowSt.resize(L);
+  c->mShadowMN.resize(L);
   c->mA.resize(L);
   c->mG.resize(L);
   c->mGT.resize(L);
@@ -1207,6 +1228,10 @@ oscars_status allocate_mlp(oscars_ctx* c) {
     bool ok = true;
     // W_l [out][in] of every slot: A operand of the forward GEMM
     ok &= make_map(&c->mShadow[l], c->shadow + ly.offW, ly.in, ly.out, slots64, ly.in * 2ull, c->P_pad * 2ull, 128);
+    // the fp32 master of W_l in every slot: read and written by the weight-gradient kernel
+    ok &= make_map_f32(&c->mMaster[l], c->slab + ly.offW, ly.in, ly.out, slots64, ly.in * 4ull, c->P_pad * 4ull, 128);
+    ok &= make_map_f32(&c->mMasterSt[l], c->slab + ly.offW, ly.in, ly.out, slots64, ly.in * 4ull, c->P_pad * 4ull, 32);
+    ok &= make_map(&c->mShadowSt[l], c->shadow + ly.offW, ly.in, ly.out, slots64, ly.in * 2ull, c->P_pad * 2ull, 32);
     // layer input [lane][B][in]: B operand of the forward GEMM (layer 0: per step)
     if (l > 0) ok &= make_map(&c->mA[l], c->A[l], ly.in, B, W, ly.in * 2ull, static_cast<uint64_t>(B) * ly.in * 2ull, B);
     // output gradient^T [lane][out][B]: A operand of the weight-gradient GEMM
@@ -1214,8 +1239,9 @@ oscars_status allocate_mlp(oscars_ctx* c) {
     // layer input^T [lane][in][B]: B operand of the weight-gradient GEMM (layer 0: per step)
     if (l > 0) ok &= make_map(&c->mAT[l], c->AT[l], B, ly.in, W, B * 2ull, static_cast<uint64_t>(B) * ly.in * 2ull, 128);
     if (l >= 1) {
-      // W_l^T [in][out] of every slot: A operand of the input-gradient GEMM
-      ok &= make_map(&c->mShadowT[l], c->shadowT + ly.offT, ly.out, ly.in, slots64, ly.out * 2ull, c->PT_pad * 2ull, 128);
+      // W_l [out][in] of every slot, boxes of 64 inputs x 64 outputs: the
+      // MN-major A operand (M = in, K = out) of the input-gradient GEMM
+      ok &= make_map(&c->mShadowMN[l], c->shadow + ly.offW, ly.in, ly.out, slots64, ly.in * 2ull, c->P_pad * 2ull, 64);
       // output gradient [lane][B][out]: B operand of the input-gradient GEMM
       ok &= make_map(&c->mG[l], c->G[l], ly.out, B, W, ly.out * 2ull, static_cast<uint64_t>(B) * ly.out * 2ull, B);
     }
@@ -1531,7 +1557,7 @@ oscars_status oscars_push_merge(oscars_ctx* c, const float* const* deltas, const
         r = launch_merge(a, xg, c->P_pad, eta, true, st, c->shadow ? c->shadow + static_cast<int64_t>(c->W) * c->P_pad : nullptr);
       }
       if (r != cudaSuccess) return r;
-      if (c->PT_pad == 0 && c->model != OSCARS_MODEL_CNN) return cudaSuccess;   // no transposed copies to refresh
+      if (c->model != OSCARS_MODEL_CNN) return cudaSuccess;   // no transposed copies to refresh
       ProfScope ps(c, "shadow_refresh", st);
       return refresh_global_shadows(c, st, true);
     };

@@ -117,8 +117,9 @@ __device__ __forceinline__ float epi_dh(const GemmArgs& a, int wid, int m, int n
 // m_base + 4 i + lane / 8.  The accumulators go through a shared-memory tile
 // (row stride 36: 16-byte accesses of 8 lanes hit distinct banks both along
 // rows and along columns) so that the fp32 master and bf16 shadow writes move
-// full lines, 4 rows per instruction; the transposed shadow is written from
-// the row layout (lane = row, consecutive addresses).
+// full lines, 4 rows per instruction.  (The persistent kernel of gemm_dw.cu
+// serves every layer whose input count is a multiple of 8; this epilogue is
+// the general fallback.)
 __device__ __forceinline__ void epi_dw_block(const GemmArgs& a, int wid, int m_base, int n_base,
                                              const float (&v)[32], const float4 (&old)[8], float* T, int lane) {
 #pragma unroll
@@ -141,19 +142,6 @@ __device__ __forceinline__ void epi_dw_block(const GemmArgs& a, int wid, int m_b
       const int64_t e = dof + static_cast<int64_t>(m_base + r) * a.N;
       *reinterpret_cast<float4*>(a.master_w + e) = nw;
       *reinterpret_cast<uint2*>(a.shadow + e) = make_uint2(pack_bf16x2(nw.x, nw.y), pack_bf16x2(nw.z, nw.w));
-    }
-    *reinterpret_cast<float4*>(T + r * 36 + cq) = nw;
-  }
-  __syncwarp();
-  if (a.shadowT) {
-    __nv_bfloat16* t = a.shadowT + static_cast<int64_t>(wid) * a.slotT_stride + a.offT + m_base + lane;
-#pragma unroll
-    for (int q = 0; q < 8; ++q) {
-      const float4 nv = *reinterpret_cast<const float4*>(T + lane * 36 + 4 * q);
-      const float f[4] = {nv.x, nv.y, nv.z, nv.w};
-#pragma unroll
-      for (int j = 0; j < 4; ++j)
-        if (n_base + 4 * q + j < a.N) t[static_cast<int64_t>(n_base + 4 * q + j) * a.M] = __float2bfloat16_rn(f[j]);
     }
   }
   __syncwarp();
@@ -237,12 +225,20 @@ __global__ void __launch_bounds__(warps_for<EPI>() * 32) gemm_tc_kernel(const __
       const int s = kb % stages;
       if (kb >= stages && !mbar_wait(&empty[s], ((kb / stages) + 1) & 1, a.err, kDevTimeoutEmpty)) break;
       mbar_arrive_expect_tx(&full[s], kABytes + Cfg::kBBytes);
-      tma_load_3d(sA + s * kABytes, &mapA, kb * BK, m0, za, &full[s]);
+      if constexpr (EPI == kEpiDh) {
+        // A = W^T read MN-major from W [K = out][M = in]: two boxes of 64 M x
+        // 64 K, the second 64 M-elements further along (8 KB in shared memory)
+        tma_load_3d(sA + s * kABytes, &mapA, m0, kb * BK, za, &full[s]);
+        tma_load_3d(sA + s * kABytes + kABytes / 2, &mapA, m0 + 64, kb * BK, za, &full[s]);
+      } else {
+        tma_load_3d(sA + s * kABytes, &mapA, kb * BK, m0, za, &full[s]);
+      }
       tma_load_3d(sB + s * Cfg::kBBytes, &mapB, kb * BK, n0, zb, &full[s]);
     }
   } else if (warp == 1 && lane == 0) {
     // MMA issuer
-    constexpr uint32_t idesc = idesc_bf16_f32(BM, BN);
+    // A MN-major (transpose-A bit 15) for the input gradient, K-major otherwise
+    constexpr uint32_t idesc = idesc_bf16_f32(BM, BN) | (EPI == kEpiDh ? (1u << 15) : 0u);
     for (int kb = 0; kb < nk; ++kb) {
       const int s = kb % stages;
       if (!mbar_wait(&full[s], (kb / stages) & 1, a.err, kDevTimeoutFull)) break;
@@ -250,9 +246,12 @@ __global__ void __launch_bounds__(warps_for<EPI>() * 32) gemm_tc_kernel(const __
       const uint32_t a_base = smem_u32(sA + s * kABytes);
       const uint32_t b_base = smem_u32(sB + s * Cfg::kBBytes);
 #pragma unroll
-      for (int j = 0; j < BK / 16; ++j)
-        umma_bf16(tmem, smem_desc_k128(a_base + j * 32), smem_desc_k128(b_base + j * 32), idesc,
-                  (kb | j) != 0 ? 1u : 0u);
+      for (int j = 0; j < BK / 16; ++j) {
+        // K-major: 16 K-elements are 32 bytes along a row; MN-major: 16 rows of 128 bytes
+        const uint64_t adesc = EPI == kEpiDh ? smem_desc_mn128(a_base + j * 2048, kABytes / 2)
+                                             : smem_desc_k128(a_base + j * 32);
+        umma_bf16(tmem, adesc, smem_desc_k128(b_base + j * 32), idesc, (kb | j) != 0 ? 1u : 0u);
+      }
       umma_commit(&empty[s]);
     }
     umma_commit(accum);  // arrives once every issued MMA has completed

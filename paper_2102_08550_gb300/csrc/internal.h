@@ -100,10 +100,8 @@ struct GemmArgs {
   const float* master;      // fp32 slab base
   float* master_w;          // same slab (written)
   __nv_bfloat16* shadow;    // bf16 slab (same layout as master)
-  __nv_bfloat16* shadowT;   // bf16 transposed slab (or null)
   int64_t slot_stride;      // P_pad
-  int64_t slotT_stride;     // PT_pad
-  int64_t offW, offB, offT; // element offsets of W_l, b_l, W_l^T in a slot
+  int64_t offW, offB;       // element offsets of W_l, b_l in a slot
   float lr;
   const float* gb_in;       // [lanes][M] bias gradient (kEpiDw)
   const __nv_bfloat16* hmask;  // [lanes][N][M] (kEpiDh)
@@ -114,6 +112,32 @@ struct GemmArgs {
 };
 cudaError_t launch_gemm(int epi, const CUtensorMap& mapA, const CUtensorMap& mapB,
                         const GemmArgs& a, int n_active, cudaStream_t s);
+
+// Weight gradient + SGD of one layer, persistent (csrc/gemm_dw.cu):
+// W[wid] = W[src] - lr * G^T X over the batch, its bf16 copy, and the bias
+// b[wid] = b[src] - lr * gb[wid] (outputs m < M, inputs n < N, batch K).
+struct DwArgs {
+  const int* wid;           // [n_active] destination slots (device), or null = lane id
+  const int* src;           // [n_active] source slots (device), or null = lane id
+  int n_active;
+  int M, N, K;
+  float lr;
+  const float* master;      // fp32 slab (bias read)
+  float* master_w;          // fp32 slab (bias written)
+  int64_t slot_stride;      // P_pad
+  int64_t offB;             // element offset of b_l in a slot
+  const float* gb;          // [W][M] bias gradient
+  int* err;
+};
+bool gemm_dw_supported(int M, int N, int K);
+// mA: G^T [lane][M][K] bf16, box {64, 128}; mB: X^T [lane][N][K] bf16, box
+// {64, 128}; mMaster: W_l fp32 [slot][M][N], box {32, 128} (loads);
+// mMasterSt: the same with box {32, 32} (stores); mShadowSt: W_l bf16
+// [slot][M][N], box {64, 32} (stores); all with 128-byte swizzle.  `sms`:
+// the device's multiprocessors (one CTA each at most).
+cudaError_t launch_gemm_dw(const CUtensorMap& mA, const CUtensorMap& mB, const CUtensorMap& mMaster,
+                           const CUtensorMap& mMasterSt, const CUtensorMap& mShadowSt, const DwArgs& a, int sms,
+                           cudaStream_t s);
 int gemm_bn_for(int epi, int N);
 
 struct HeadArgs {
