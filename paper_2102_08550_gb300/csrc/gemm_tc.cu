@@ -342,10 +342,23 @@ cudaError_t launch_tile(const CUtensorMap& mA, const CUtensorMap& mB, const Gemm
                         cudaStream_t s) {
   using Cfg = TileCfg<BN>;
   const int nk = (a.K + BK - 1) / BK;
-  // as many stages as K-blocks, within ~200 KB of shared memory: the whole
-  // K extent of these skinny GEMMs is then in flight at once
-  const int max_stages = static_cast<int>((200 * 1024 - (EPI == kEpiDw ? 8 * 32 * 33 * 4 : 0)) / Cfg::kStageBytes);
-  const int stages = nk < max_stages ? nk : (max_stages < 8 ? max_stages : 8);
+  dim3 grid(a.M / BM, (a.N + BN - 1) / BN, n_active);
+  // A grid that fits one CTA per SM gets as many stages as K-blocks, within
+  // ~200 KB of shared memory: the whole K extent of these skinny GEMMs is
+  // then in flight at once.  A larger grid gets stages for ~100 KB, so two
+  // CTAs share each SM and the grid runs in one wave instead of two (the
+  // bytes in flight per SM stay the same).
+  static int sms = 0;
+  if (sms == 0) {
+    int dev = 0;
+    cudaGetDevice(&dev);
+    if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms < 1) sms = 1;
+  }
+  const long long ctas = static_cast<long long>(grid.x) * grid.y * grid.z;
+  const int budget = ctas > sms ? 100 * 1024 : 200 * 1024;
+  const int max_stages = static_cast<int>((budget - (EPI == kEpiDw ? 8 * 32 * 33 * 4 : 0)) / Cfg::kStageBytes);
+  int stages = nk < max_stages ? nk : (max_stages < 8 ? max_stages : 8);
+  if (stages < 2) stages = nk < 2 ? nk : 2;
   constexpr int kWarps = warps_for<EPI>();
   size_t smem = 1024 + static_cast<size_t>(stages) * Cfg::kStageBytes + kBarrierBytes +
                 (EPI == kEpiDw ? sizeof(float) * kWarps * kEpiTileFloats : 0);
@@ -354,7 +367,6 @@ cudaError_t launch_tile(const CUtensorMap& mA, const CUtensorMap& mB, const Gemm
   cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<BN, EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(smem));
   if (e != cudaSuccess) return e;
-  dim3 grid(a.M / BM, (a.N + BN - 1) / BN, n_active);
   gemm_tc_kernel<BN, EPI><<<grid, kWarps * 32, smem, s>>>(mA, mB, a, stages);
   return cudaGetLastError();
 }
