@@ -55,6 +55,8 @@ def parse():
     ap.add_argument("--no-merge", action="store_true", help="skip the merge microbenchmarks")
     ap.add_argument("--no-cpu", action="store_true", help="skip the CPU oracle baseline")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-side", action="store_true",
+                    help="skip the other training workloads (softmax regression, 3072-1024-1024-10 MLP)")
     ap.add_argument("--merge-reps", type=int, default=20)
     ap.add_argument("--only", choices=["all", "round", "merge"], default="all",
                     help="round: only the Oscars-round benchmark; merge: only the merge microbenchmarks")
@@ -99,6 +101,8 @@ class ClockSampler:
         self.path = os.path.join(ROOT, "gpurun_out", f"clocks_{os.getpid()}.csv")
 
     def __enter__(self):
+        if self.index < 0:                # sampling off
+            return self
         try:
             os.makedirs(os.path.dirname(self.path), exist_ok=True)
             self.f = open(self.path, "w")
@@ -168,6 +172,8 @@ def algorithmic_work(w, tau):
         if l >= 1:
             add("gemm_dh", n * 2 * B * i * o, n * (o * i * 2 + B * o * 2 + B * i * 2 + 2 * B * i * 2 + i * 4))
     H, C = d[L - 1], d[L]
+    if L == 1:                        # fp32 softmax regression on the CUDA cores: logits + weight gradient
+        add("softreg_round", n * 4 * B * H * C, n * (B * H * 4 + B * 4) + W * (C * H + C) * 4 * 2)
     add("head_fwd", n * 2 * B * H * C, n * (C * H * 2 + B * H * 2 + B * C * 4 + B * 4 + C * 4))
     add("head_bwd", n * 4 * B * H * C,
         n * (B * H * 2 + C * H * (2 + 4 + 4 + 2) + 2 * B * H * 2 + H * 4 + B * C * 4 + C * 8))
@@ -196,10 +202,37 @@ NCU_TRAFFIC = {
 }
 
 
+_ALU_PEAK = None
+
+
+def alu_peak_tflops():
+    """fp32 FFMA peak of the CUDA cores: SMs x 128 FFMA per clock x 2 FLOP x
+    the maximum SM clock (nvidia-smi; 2070 MHz if it cannot be read)."""
+    global _ALU_PEAK
+    if _ALU_PEAK is None:
+        import torch
+        sms = torch.cuda.get_device_properties(torch.cuda.current_device()).multi_processor_count
+        mhz = 2070.0
+        try:
+            out = subprocess.run(["nvidia-smi", "-i", str(torch.cuda.current_device()), "--query-gpu=clocks.max.sm",
+                                  "--format=csv,noheader,nounits"], capture_output=True, text=True, timeout=10)
+            mhz = float(out.stdout.strip().splitlines()[0])
+        except Exception:
+            pass
+        _ALU_PEAK = (sms * 128 * 2 * mhz * 1e6 / 1e12, f"{sms} SMs x 128 FFMA x 2 x {mhz:.0f} MHz")
+    return _ALU_PEAK
+
+
 def roofline_of(name, ms_per_launch, launches_per_round, flops, bytes_, hbm, tflops, peak_kind, workload=None):
     f = flops.get(name, 0.0) / launches_per_round
     b = bytes_.get(name, 0.0) / launches_per_round
     t = ms_per_launch / 1e3
+    if name == "softreg_round" and f > 0.0:     # fp32 CUDA-core arithmetic
+        peak, how = alu_peak_tflops()
+        ach = f / t / 1e12
+        return {"kernel": name, "bound": "alu", "achieved": ach, "peak": peak, "unit": "TFLOP/s", "frac": ach / peak,
+                "peak_kind": f"fp32 FFMA ({how})", "flops_per_launch": f, "bytes_per_launch": b,
+                "ms_per_launch": ms_per_launch, "traffic": None}
     if f == 0.0 and b == 0.0:
         return {"kernel": name, "bound": "alu", "achieved": None, "peak": None, "unit": None, "frac": None,
                 "ms_per_launch": ms_per_launch, "traffic": None}
@@ -235,45 +268,42 @@ def whole_job_rate(units_per_rank: float, world: int, max_ms: float) -> float:
     return units_per_rank * world / (max_ms / 1e3)
 
 
-def run_gpu(args, rank, world, local_rank):
+def measure_rounds(w, steps, warmup, dev, world=1, local_rank=0, flush=None, clock=True, prof_rounds=None):
+    """Oscars rounds of the MLP workload ``w`` on ``dev``: device time of
+    ``steps`` rounds (CUDA events, L2 flushed between rounds), then the
+    per-kernel split from an instrumented replay."""
     import torch
     import paper_2102_08550_gb300 as P
-    from paper_2102_08550_gb300 import _build
-
-    _build.build()
-    dev = torch.device(f"cuda:{local_rank}")
-    torch.cuda.set_device(dev)
-    w = WORKLOADS[args.workload]
     hbm, tf_burst, tf_sus, peak_kind = peaks()
     T_star, mw, tau = schedule_of(w)
     samples_per_round = int(np.sum(tau)) * w.batch
-
     shards = [synth.shard_t(w, k, dev) for k in range(w.num_workers)]
     layers0 = synth.init_layers_np(w)
     init = torch.from_numpy(synth.flatten_layers(layers0)).to(dev)
     stream = torch.cuda.current_stream(dev)
 
     def make(flags=0):
-        return P.OscarsContext(num_workers=w.num_workers, dims=w.dims, batch=w.batch, lr=w.lr,
+        return P.OscarsContext(num_workers=w.num_workers, dims=w.dims, batch=w.batch, lr=w.lr, bf16=w.bf16,
                                speed=synth.speeds(w).tolist(), M=w.M, shards=shards, init_params=init,
                                stream=stream.cuda_stream, flags=flags)
 
     ctx = make()
-    flush = torch.empty(512 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)   # > L2 (129 MB)
+    if flush is None:
+        flush = torch.empty(512 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)   # > L2 (129 MB)
 
     def one_round():
         P.oscars_local_steps(ctx.handle, want_tau=False, want_loss=False)
         P.oscars_push_merge(ctx.handle)
 
-    for _ in range(args.warmup):
+    for _ in range(warmup):
         one_round()
     torch.cuda.synchronize()
     if world > 1:
         torch.distributed.barrier()
     torch.cuda.synchronize()
-    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
-    with ClockSampler(local_rank) as clk:
-        for i in range(args.steps):
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
+    with ClockSampler(local_rank if clock else -1) as clk:
+        for i in range(steps):
             flush.fill_(float(i))            # evict the previous round's state from L2 (untimed)
             evs[i][0].record(stream)
             one_round()
@@ -281,7 +311,8 @@ def run_gpu(args, rank, world, local_rank):
         torch.cuda.synchronize()
     total_ms = max_over_ranks(sum(a.elapsed_time(b) for a, b in evs), world, dev)
     torch.cuda.synchronize()
-    value = whole_job_rate(samples_per_round * args.steps, world, total_ms)
+    ctx.close()
+    value = whole_job_rate(samples_per_round * steps, world, total_ms)
 
     # ---- per-kernel device time: the same round graph with an event node
     # around every kernel (device timeline, no host launch gaps)
@@ -291,7 +322,7 @@ def run_gpu(args, rank, world, local_rank):
         P.oscars_push_merge(pctx.handle)
     torch.cuda.synchronize()
     pctx.profile_reset()
-    prof_rounds = max(3, min(args.steps, 10))
+    prof_rounds = prof_rounds or max(3, min(steps, 10))
     for i in range(prof_rounds):
         flush.fill_(float(i))
         P.oscars_local_steps(pctx.handle, want_tau=False, want_loss=False)
@@ -299,6 +330,7 @@ def run_gpu(args, rank, world, local_rank):
     prof = pctx.profile()
     torch.cuda.synchronize()
     pctx.close()
+    del shards
     launches_per_round = sum(c for _, c in prof.values()) / prof_rounds
     flops, bytes_ = algorithmic_work(w, tau)
     dom = max(prof, key=lambda k: prof[k][0])
@@ -308,7 +340,7 @@ def run_gpu(args, rank, world, local_rank):
         r = roofline_of(k, ms / cnt, cnt / prof_rounds, flops, bytes_, hbm, tf_sus, peak_kind)
         kernels[k] = {"ms_per_round": ms / prof_rounds, "launches_per_round": cnt / prof_rounds,
                       "share": ms / tot, "bound": r["bound"], "frac": r["frac"]}
-        if flops.get(k, 0.0) > 0.0:     # every kernel that does tensor work: its fraction of the tensor peak
+        if k in TENSOR_KERNELS and flops.get(k, 0.0) > 0.0:   # tensor-core work: its fraction of the tensor peak
             tf = flops[k] / (ms / prof_rounds / 1e3) / 1e12
             kernels[k]["tflops"] = tf
             kernels[k]["tensor_frac"] = tf / tf_sus
@@ -320,19 +352,58 @@ def run_gpu(args, rank, world, local_rank):
                                 "tensor_frac": g_tf / tf_sus}
     roof = roofline_of(dom, prof[dom][0] / prof[dom][1], prof[dom][1] / prof_rounds, flops, bytes_, hbm, tf_sus,
                        peak_kind, w.name)
+    return {"value": value, "ms_per_step": total_ms / steps, "roofline": roof, "kernels": kernels,
+            "gpu_launches": int(round(launches_per_round * steps)), "clocks": clk.summary() if clock else None,
+            "samples_per_round": samples_per_round, "T_star": int(T_star), "tau": [int(v) for v in tau]}
+
+
+# kernel classes whose FLOPs run on the tensor cores (tcgen05)
+TENSOR_KERNELS = ("gemm_fwd", "gemm_dh", "gemm_dw_sgd", "fused_round")
+
+# the training workloads measured beside the headline (absolute samples/s and
+# the roofline of their dominant kernel)
+SIDE_WORKLOADS = (synth.CFG1, synth.CFG3)
+
+
+def run_side_workloads(args, dev):
+    import torch
+    out = {}
+    for w in SIDE_WORKLOADS:
+        r = measure_rounds(w, max(20, args.steps), max(3, args.warmup), dev, clock=False, prof_rounds=3)
+        out[w.name] = {"metric": "simulated-worker samples/s", "value": r["value"], "unit": UNIT,
+                       "ms_per_round": r["ms_per_step"], "config": workload_config(w, "flushed between timed rounds"),
+                       "dtype": "bf16 (fp32 master, fp32 accumulate)" if w.bf16 else "f32",
+                       "roofline": r["roofline"], "kernels": r["kernels"], "samples_per_round": r["samples_per_round"]}
+        torch.cuda.empty_cache()
+    return out
+
+
+def run_gpu(args, rank, world, local_rank):
+    import torch
+    from paper_2102_08550_gb300 import _build
+
+    _build.build()
+    dev = torch.device(f"cuda:{local_rank}")
+    torch.cuda.set_device(dev)
+    w = WORKLOADS[args.workload]
+    hbm, tf_burst, tf_sus, peak_kind = peaks()
+    T_star, mw, tau = schedule_of(w)
+    stream = torch.cuda.current_stream(dev)
+    res = measure_rounds(w, args.steps, args.warmup, dev, world, local_rank)
 
     # ---- end to end through the C ABI with host-resident inputs
     e2e = None
     if not args.no_e2e:
+        shards = [synth.shard_t(w, k, dev) for k in range(w.num_workers)]
         e2e = run_e2e(args, shards, w, tau, dev, stream, world)
+        del shards
+        torch.cuda.empty_cache()
 
-    merge = None if args.no_merge else run_merge(args, dev, stream, hbm, peak_kind)
-    ctx.close()
-    out = {"value": value, "ms_per_step": total_ms / args.steps, "roofline": roof, "kernels": kernels,
-           "gpu_launches": int(round(launches_per_round * args.steps)), "clocks": clk.summary(), "e2e": e2e,
-           "merge": merge, "samples_per_round": samples_per_round, "T_star": int(T_star),
-           "tau": [int(v) for v in tau]}
-    return out
+    res["e2e"] = e2e
+    res["merge"] = None if args.no_merge else run_merge(args, dev, stream, hbm, peak_kind)
+    res["workloads"] = (run_side_workloads(args, dev)
+                        if world == 1 and args.workload == WORKLOAD.name and not args.no_side else None)
+    return res
 
 
 def run_e2e(args, shards, w, tau, dev, stream, world=1):
@@ -729,7 +800,7 @@ def main():
                 "roofline": res["roofline"], "cpu_baseline": cpu, "e2e": res["e2e"],
                 "gpu_launches": res["gpu_launches"], "clocks": res["clocks"], "merge": res["merge"],
                 "kernels": res["kernels"], "samples_per_round": res["samples_per_round"],
-                "T_star": res["T_star"], "tau": res["tau"]}
+                "T_star": res["T_star"], "tau": res["tau"], "workloads": res["workloads"]}
         print(json.dumps(line))
     if world > 1:
         import torch

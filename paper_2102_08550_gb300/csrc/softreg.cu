@@ -29,6 +29,10 @@ __device__ __forceinline__ float warp_sum(float v) {
   return v;
 }
 
+// float4 items of one mini-batch a thread holds in registers while the
+// previous step computes (the next step's rows are loaded ahead)
+constexpr int kPrefetch = 16;
+
 __global__ void __launch_bounds__(kThreads) softreg_round_kernel(const __grid_constant__ SoftregArgs a) {
   extern __shared__ __align__(16) float sm[];
   const int D = a.D, C = a.C, B = a.B;
@@ -38,6 +42,7 @@ __global__ void __launch_bounds__(kThreads) softreg_round_kernel(const __grid_co
   float* Zsm = Xsm + B * D;        // [B][C] logits, then dz
   float* Lsm = Zsm + B * C;        // [B] per-sample loss
   int* Ysm = reinterpret_cast<int*>(Lsm + B);  // [B]
+  int64_t* Rsm = reinterpret_cast<int64_t*>((reinterpret_cast<uintptr_t>(Ysm + B) + 7) & ~uintptr_t(7));   // [B] row offsets
 
   const int w = blockIdx.x;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -54,35 +59,91 @@ __global__ void __launch_bounds__(kThreads) softreg_round_kernel(const __grid_co
   const int64_t n = a.shard_n[w];
   const int64_t cur = a.cursor[w];
   const float invB = 1.0f / static_cast<float>(B);
+  // with D % 4 == 0 and a mini-batch of at most kPrefetch float4 per thread,
+  // step s + 1's rows are loaded into registers while step s computes
+  const int D4 = D / 4;
+  const bool vec = (D & 3) == 0 && B * D4 <= kPrefetch * kThreads;
+  float4 pf[kPrefetch];
+  auto fetch = [&](int s) {   // rows of step s into registers (row offsets already in Rsm)
+#pragma unroll
+    for (int j = 0; j < kPrefetch; ++j) {
+      const int i = tid + j * kThreads;
+      if (i < B * D4) {
+        const int b = i / D4, k4 = i - b * D4;
+        pf[j] = *reinterpret_cast<const float4*>(X + Rsm[b] + 4 * k4);
+      }
+    }
+  };
+  auto row_offsets = [&](int s) {
+    if (tid < B) {
+      const int64_t r = (cur + static_cast<int64_t>(s) * B + tid) % n;
+      Rsm[tid] = r * D;
+      Ysm[tid] = Y[r];
+    }
+  };
+  if (vec && tau > 0) {
+    row_offsets(0);
+    __syncthreads();
+    fetch(0);
+  }
 
   for (int s = 0; s < tau; ++s) {
-    __syncthreads();
-    // mini-batch rows (cursor + s*B + b) mod n
-    for (int i = tid; i < B * D; i += kThreads) {
-      const int b = i / D, k = i - b * D;
-      const int64_t r = (cur + static_cast<int64_t>(s) * B + b) % n;
-      Xsm[i] = X[r * D + k];
+    __syncthreads();   // the previous step is done with Xsm and Zsm
+    int yl = 0;        // the label of row tid (tid < B) of this step
+    if (vec) {
+      // this step's rows, fetched during the previous step; then the next
+      // step's row offsets and labels (thread tid rewrites only entry tid,
+      // which it alone has read) and its rows, in flight during this step
+      if (tid < B) yl = Ysm[tid];
+#pragma unroll
+      for (int j = 0; j < kPrefetch; ++j) {
+        const int i = tid + j * kThreads;
+        if (i < B * D4) reinterpret_cast<float4*>(Xsm)[i] = pf[j];
+      }
+      if (s + 1 < tau) row_offsets(s + 1);
+      __syncthreads();
+      if (s + 1 < tau) fetch(s + 1);
+    } else {
+      // mini-batch rows (cursor + s*B + b) mod n
+      row_offsets(s);
+      __syncthreads();
+      for (int i = tid; i < B * D; i += kThreads) {
+        const int b = i / D, k = i - b * D;
+        Xsm[i] = X[Rsm[b] + k];
+      }
+      if (tid < B) yl = Ysm[tid];
+      __syncthreads();
     }
-    for (int b = tid; b < B; b += kThreads) Ysm[b] = Y[(cur + static_cast<int64_t>(s) * B + b) % n];
-    __syncthreads();
     // logits: one warp per (b, c) dot product
     for (int q = warp; q < B * C; q += kWarps) {
       const int b = q / C, c = q - b * C;
       const float* xr = Xsm + b * D;
       const float* wr = Wsm + c * D;
       float acc = 0.f;
-      for (int k = lane; k < D; k += 32) acc = fmaf(xr[k], wr[k], acc);
+      if ((D & 3) == 0) {
+        for (int k4 = lane; k4 < D4; k4 += 32) {
+          const float4 xv = reinterpret_cast<const float4*>(xr)[k4];
+          const float4 wv = reinterpret_cast<const float4*>(wr)[k4];
+          acc = fmaf(xv.x, wv.x, acc);
+          acc = fmaf(xv.y, wv.y, acc);
+          acc = fmaf(xv.z, wv.z, acc);
+          acc = fmaf(xv.w, wv.w, acc);
+        }
+      } else {
+        for (int k = lane; k < D; k += 32) acc = fmaf(xr[k], wr[k], acc);
+      }
       acc = warp_sum(acc);
       if (lane == 0) Zsm[q] = acc + bsm[c];
     }
     __syncthreads();
     // softmax cross-entropy, one thread per row
-    for (int b = tid; b < B; b += kThreads) {
+    if (tid < B) {
+      const int b = tid;
       float* z = Zsm + b * C;
       float m = z[0];
       for (int c = 1; c < C; ++c) m = fmaxf(m, z[c]);
       // p_c = e_c / s; 1 - p_y = (sum_{c != y} e_c) / s (no cancellation)
-      const int y = Ysm[b];
+      const int y = yl;
       float se = 0.f, so = 0.f;
       for (int c = 0; c < C; ++c) {
         const float e = expf(z[c] - m);
@@ -98,12 +159,35 @@ __global__ void __launch_bounds__(kThreads) softreg_round_kernel(const __grid_co
       for (int b = 0; b < B; ++b) l += Lsm[b];
       a.loss_part[static_cast<int64_t>(w) * a.max_tau + s] = l;
     }
-    // weight gradient and update, one thread per input feature k
-    for (int k = tid; k < D; k += kThreads) {
-      for (int c = 0; c < C; ++c) {
-        float g = 0.f;
-        for (int b = 0; b < B; ++b) g = fmaf(Zsm[b * C + c], Xsm[b * D + k], g);
-        Wsm[c * D + k] = fmaf(-a.lr, g, Wsm[c * D + k]);
+    // weight gradient and update: item = (class, 4 input features) (or one
+    // feature when D % 4 != 0)
+    if ((D & 3) == 0) {
+      for (int q = tid; q < C * D4; q += kThreads) {
+        const int c = q / D4, k4 = q - c * D4;
+        float4 g = make_float4(0.f, 0.f, 0.f, 0.f);
+        for (int b = 0; b < B; ++b) {
+          const float d = Zsm[b * C + c];
+          const float4 xv = reinterpret_cast<const float4*>(Xsm + b * D)[k4];
+          g.x = fmaf(d, xv.x, g.x);
+          g.y = fmaf(d, xv.y, g.y);
+          g.z = fmaf(d, xv.z, g.z);
+          g.w = fmaf(d, xv.w, g.w);
+        }
+        float4* wp = reinterpret_cast<float4*>(Wsm + c * D) + k4;
+        float4 wv = *wp;
+        wv.x = fmaf(-a.lr, g.x, wv.x);
+        wv.y = fmaf(-a.lr, g.y, wv.y);
+        wv.z = fmaf(-a.lr, g.z, wv.z);
+        wv.w = fmaf(-a.lr, g.w, wv.w);
+        *wp = wv;
+      }
+    } else {
+      for (int k = tid; k < D; k += kThreads) {
+        for (int c = 0; c < C; ++c) {
+          float g = 0.f;
+          for (int b = 0; b < B; ++b) g = fmaf(Zsm[b * C + c], Xsm[b * D + k], g);
+          Wsm[c * D + k] = fmaf(-a.lr, g, Wsm[c * D + k]);
+        }
       }
     }
     for (int c = tid; c < C; c += kThreads) {
@@ -153,7 +237,7 @@ __global__ void __launch_bounds__(256) softreg_eval_kernel(const __grid_constant
 size_t softreg_smem_bytes(int D, int C, int B) {
   return sizeof(float) * (static_cast<size_t>(C) * D + 32 + static_cast<size_t>(B) * D +
                           static_cast<size_t>(B) * C + B) +
-         sizeof(int) * B;
+         sizeof(int) * B + 8 + sizeof(int64_t) * B;
 }
 
 cudaError_t launch_softreg_round(const SoftregArgs& a, int W, cudaStream_t s) {
