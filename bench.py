@@ -24,6 +24,7 @@ scheme needs to reach the loss BSP ends at.
 from __future__ import annotations
 
 import argparse
+import dataclasses
 import json
 import os
 import subprocess
@@ -55,6 +56,9 @@ def parse():
     ap.add_argument("--no-merge", action="store_true", help="skip the merge microbenchmarks")
     ap.add_argument("--no-cpu", action="store_true", help="skip the CPU oracle baseline")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--samples-per-worker", type=int, default=0,
+                    help="shard rows per worker of the round workload (0: the workload's own; smaller for "
+                         "ncu captures that must stay a few GB on the device)")
     ap.add_argument("--no-side", action="store_true",
                     help="skip the other training workloads (softmax regression, 3072-1024-1024-10 MLP)")
     ap.add_argument("--merge-reps", type=int, default=20)
@@ -386,6 +390,8 @@ def run_gpu(args, rank, world, local_rank):
     dev = torch.device(f"cuda:{local_rank}")
     torch.cuda.set_device(dev)
     w = WORKLOADS[args.workload]
+    if args.samples_per_worker:
+        w = dataclasses.replace(w, samples_per_worker=args.samples_per_worker)
     hbm, tf_burst, tf_sus, peak_kind = peaks()
     T_star, mw, tau = schedule_of(w)
     stream = torch.cuda.current_stream(dev)
@@ -786,6 +792,8 @@ def main():
         args.no_merge = True
     res = run_gpu(args, rank, world, local_rank)
     w = WORKLOADS[args.workload]
+    if args.samples_per_worker:
+        w = dataclasses.replace(w, samples_per_worker=args.samples_per_worker)
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu:
         samples, dt, done = oracle_rounds(w, 6, 15.0)
