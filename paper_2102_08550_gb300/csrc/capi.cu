@@ -146,6 +146,8 @@ struct oscars_ctx {
   int32_t* tau_dev = nullptr;
   int32_t* order_dev = nullptr;         // workers by decreasing tau (launch order of the round kernel)
   int* act_wid = nullptr;  // [max_tau][W]
+  int32_t* stage_slots = nullptr;   // [sum tau] active staging slots s * W + w, step-major
+  int n_stage_slots = 0;
   int* act_src = nullptr;
   int* lane_ids = nullptr;   // [W] 0..W-1
   int* global_src = nullptr; // [W] all = W
@@ -486,6 +488,17 @@ oscars_status build_tables(oscars_ctx* c) {
     if (e == cudaSuccess) e = cudaMemcpy(c->br_src, bs.data(), bs.size() * sizeof(int), cudaMemcpyHostToDevice);
     if (e != cudaSuccess) return cuda_fail(c, e, "branch table upload");
   }
+  std::vector<int32_t> slots;
+  for (int st = 0; st < c->max_tau; ++st)
+    for (int i = 0; i < c->W; ++i)
+      if (c->tau[i] > st) slots.push_back(st * c->W + i);
+  c->n_stage_slots = static_cast<int>(slots.size());
+  if (!dev_alloc(c, &c->stage_slots, slots.size()))
+    return fail(c, OSCARS_ENOMEM, "device allocation failed (staging slots)");
+  {
+    const cudaError_t e = cudaMemcpy(c->stage_slots, slots.data(), slots.size() * sizeof(int32_t), cudaMemcpyHostToDevice);
+    if (e != cudaSuccess) return cuda_fail(c, e, "staging slot upload");
+  }
   if (!dev_alloc(c, &c->act_wid, wid.size()) || !dev_alloc(c, &c->act_src, src.size()) ||
       !dev_alloc(c, &c->loss_part, static_cast<size_t>(c->W) * c->max_tau * std::max(1, c->B / kRowsPerLossChunk)))
     return fail(c, OSCARS_ENOMEM, "device allocation failed (schedule tables)");
@@ -715,6 +728,8 @@ StageArgs stage_args(oscars_ctx* c, int buf, const int32_t* ahead) {
   sa.A0 = c->A0b[buf];
   sa.A0T = c->A0Tb[buf];
   sa.labels = c->labb[buf];
+  sa.slots = c->stage_slots;
+  sa.n_slots = c->n_stage_slots;
   sa.ahead = ahead;
   return sa;
 }
@@ -772,6 +787,8 @@ cudaError_t enqueue_round_mlp(oscars_ctx* c, cudaStream_t st) {
     sa.A0 = c->A0all;
     sa.A0T = c->A0Tall;
     sa.labels = c->labels_all;
+    sa.slots = c->stage_slots;
+    sa.n_slots = c->n_stage_slots;
     ProfScope ps(c, "stage", st);
     if ((e = launch_stage_round(sa, c->tau_dev, c->W, c->max_tau, st)) != cudaSuccess) return e;
   }

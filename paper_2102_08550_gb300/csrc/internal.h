@@ -78,9 +78,12 @@ struct StageArgs {
   __nv_bfloat16* A0T;      // [lanes][D][B]
   int32_t* labels;         // [lanes][B]
   const int32_t* ahead;    // stage_round: null, or tau (the next round: rows from start + tau * B)
+  const int32_t* slots;    // stage_round: the n_slots active slots s * W + w (s < tau[w]), or null (all)
+  int n_slots;
 };
 cudaError_t launch_stage(const StageArgs& a, int n_active, cudaStream_t s);
 // all mini-batches of a round: step s of worker w (s < tau[w]) at slot s * W + w
+// (grid z over a.slots when given, else over all max_tau * W slots)
 cudaError_t launch_stage_round(const StageArgs& a, const int32_t* tau, int W, int max_tau, cudaStream_t s);
 // the same with a launch priority (cudaLaunchAttributePriority)
 cudaError_t launch_stage_round_priority(const StageArgs& a, const int32_t* tau, int W, int max_tau, int priority,

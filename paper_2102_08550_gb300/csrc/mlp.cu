@@ -63,18 +63,23 @@ __global__ void __launch_bounds__(256) stage_kernel(const __grid_constant__ Stag
   stage_tile(a, w, a.start[w] + a.row_add, a.A0 + off, a.A0T + off, a.labels + static_cast<int64_t>(w) * a.B);
 }
 
-// Every mini-batch of a round at once: grid z = step * W + worker; a CTA
-// whose worker has fewer local steps returns at once.  Step s of worker w
-// lands at offset (s * W + w) of the per-step buffers.  A CTA converts 32
-// rows x 128 features: 16-byte loads of fp32 (D % 4 == 0), 8-byte bf16
-// stores of the row-major copy, and the transposed copy assembled in shared
-// memory and written as 32-byte row pieces.
+// Every mini-batch of a round at once: grid z = step * W + worker (or the
+// table of active slots); a CTA whose worker has fewer local steps returns at
+// once.  Step s of worker w lands at offset (s * W + w) of the per-step
+// buffers.  A CTA converts 32 rows x 128 features: the row offsets (cursor
+// arithmetic modulo the shard) once per row, 16-byte loads of fp32 (D % 4 ==
+// 0), all issued before any store, 8-byte bf16 stores of the row-major copy,
+// and the transposed copy through a [row][feature] shared tile whose row
+// stride (65 words) keeps both its writes and its column reads apart in the
+// banks, written as 32-byte pieces of 16 samples.
 constexpr int kStageRows = 32, kStageCols = 128;
+constexpr int kStageLd = kStageCols + 2;   // bf16 row stride of the tile
 
 __global__ void __launch_bounds__(256) stage_round_kernel(const __grid_constant__ StageArgs a, const int32_t* tau,
                                                           int W) {
-  __shared__ __align__(16) __nv_bfloat16 tile[kStageCols][kStageRows + 8];
-  const int z = blockIdx.z;
+  __shared__ __align__(16) __nv_bfloat16 tile[kStageRows][kStageLd];
+  __shared__ int64_t rowoff[kStageRows];
+  const int z = a.slots ? a.slots[blockIdx.z] : static_cast<int>(blockIdx.z);
   const int s = z / W, w = z - s * W;
   if (s >= tau[w]) return;
   const int64_t slot = static_cast<int64_t>(s) * W + w;
@@ -86,6 +91,13 @@ __global__ void __launch_bounds__(256) stage_round_kernel(const __grid_constant_
   const int64_t base = a.start[w] + (static_cast<int64_t>(s) + (a.ahead ? a.ahead[w] : 0)) * a.B;
   const int k0 = blockIdx.x * kStageCols, b0 = blockIdx.y * kStageRows;
   const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;   // 32 x 8
+  if (threadIdx.x < kStageRows) {
+    const int b = b0 + threadIdx.x;
+    const int64_t row = (base + b) % n;
+    rowoff[threadIdx.x] = row * a.D;
+    if (blockIdx.x == 0 && b < a.B) a.labels[slot * a.B + b] = a.y[w][row];
+  }
+  __syncthreads();
   const int k = k0 + tx * 4;
   const bool kok = k < a.D;
   // all of this thread's rows are loaded before any is stored: the shards may
@@ -93,21 +105,19 @@ __global__ void __launch_bounds__(256) stage_round_kernel(const __grid_constant_
   float4 xv[kStageRows / 8];
 #pragma unroll
   for (int i = 0; i < kStageRows / 8; ++i) {
-    const int b = b0 + ty + 8 * i;
+    const int r = ty + 8 * i;
     xv[i] = make_float4(0.f, 0.f, 0.f, 0.f);
-    if (b < a.B && kok) xv[i] = *reinterpret_cast<const float4*>(X + ((base + b) % n) * a.D + k);
+    if (b0 + r < a.B && kok) xv[i] = *reinterpret_cast<const float4*>(X + rowoff[r] + k);
   }
 #pragma unroll
   for (int i = 0; i < kStageRows / 8; ++i) {
     const int r = ty + 8 * i, b = b0 + r;
     const float4 v = xv[i];
-    if (b < a.B && kok)
-      *reinterpret_cast<uint2*>(A0 + static_cast<int64_t>(b) * a.D + k) =
-          make_uint2(pack_bf16x2(v.x, v.y), pack_bf16x2(v.z, v.w));
-    tile[tx * 4 + 0][r] = __float2bfloat16_rn(v.x);
-    tile[tx * 4 + 1][r] = __float2bfloat16_rn(v.y);
-    tile[tx * 4 + 2][r] = __float2bfloat16_rn(v.z);
-    tile[tx * 4 + 3][r] = __float2bfloat16_rn(v.w);
+    const uint32_t lo = pack_bf16x2(v.x, v.y), hi = pack_bf16x2(v.z, v.w);
+    if (b < a.B && kok) *reinterpret_cast<uint2*>(A0 + static_cast<int64_t>(b) * a.D + k) = make_uint2(lo, hi);
+    uint32_t* t = reinterpret_cast<uint32_t*>(&tile[r][tx * 4]);
+    t[0] = lo;
+    t[1] = hi;
   }
   __syncthreads();
   {   // 128 feature rows x 32 samples: two 16-sample pieces per row
@@ -115,15 +125,17 @@ __global__ void __launch_bounds__(256) stage_round_kernel(const __grid_constant_
     const int kk = k0 + kr;
     const int bb = b0 + piece * 16;
     if (kk < a.D && bb < a.B) {
-      const uint4* src = reinterpret_cast<const uint4*>(&tile[kr][piece * 16]);
+      uint32_t p[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const uint32_t e0 = __bfloat16_as_ushort(tile[piece * 16 + 2 * j][kr]);
+        const uint32_t e1 = __bfloat16_as_ushort(tile[piece * 16 + 2 * j + 1][kr]);
+        p[j] = e0 | (e1 << 16);
+      }
       uint4* dst = reinterpret_cast<uint4*>(A0T + static_cast<int64_t>(kk) * a.B + bb);
-      dst[0] = src[0];
-      dst[1] = src[1];
+      dst[0] = make_uint4(p[0], p[1], p[2], p[3]);
+      dst[1] = make_uint4(p[4], p[5], p[6], p[7]);
     }
-  }
-  if (blockIdx.x == 0 && threadIdx.x < kStageRows) {
-    const int b = b0 + threadIdx.x;
-    if (b < a.B) a.labels[slot * a.B + b] = a.y[w][(base + b) % n];
   }
 }
 
@@ -661,7 +673,8 @@ cudaError_t launch_stage_round_priority(const StageArgs& a, const int32_t* tau, 
                                         cudaStream_t s) {
   if (a.D % 4 != 0 || a.B % 16 != 0) return cudaErrorInvalidValue;
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3((a.D + kStageCols - 1) / kStageCols, (a.B + kStageRows - 1) / kStageRows, W * max_tau);
+  cfg.gridDim = dim3((a.D + kStageCols - 1) / kStageCols, (a.B + kStageRows - 1) / kStageRows,
+                     a.slots ? a.n_slots : W * max_tau);
   cfg.blockDim = dim3(256, 1, 1);
   cfg.stream = s;
   cudaLaunchAttribute attr[1];
@@ -674,7 +687,7 @@ cudaError_t launch_stage_round_priority(const StageArgs& a, const int32_t* tau, 
 
 cudaError_t launch_stage_round(const StageArgs& a, const int32_t* tau, int W, int max_tau, cudaStream_t s) {
   if (a.D % 4 != 0 || a.B % 16 != 0) return cudaErrorInvalidValue;
-  dim3 grid((a.D + kStageCols - 1) / kStageCols, (a.B + kStageRows - 1) / kStageRows, W * max_tau);
+  dim3 grid((a.D + kStageCols - 1) / kStageCols, (a.B + kStageRows - 1) / kStageRows, a.slots ? a.n_slots : W * max_tau);
   stage_round_kernel<<<grid, 256, 0, s>>>(a, tau, W);
   return cudaGetLastError();
 }
