@@ -168,6 +168,8 @@ struct oscars_ctx {
   // fp32 W_l of every slot: boxes {32, 128} (loads) and {32, 32} (stores), and
   // the bf16 copy with boxes {64, 32} (stores): the persistent weight gradient
   std::vector<CUtensorMap> mMaster, mMasterSt, mShadowSt;
+  // the last layer's input [lane][B][H] (box {64, 128}) and weights of every slot (box {64, 16})
+  CUtensorMap mHeadIn, mHeadW;
   // per-step input buffers of layer 0 (a round's mini-batches are staged at once)
   int stage_cap = 0;
   __nv_bfloat16* A0all = nullptr;
@@ -583,6 +585,7 @@ HeadArgs head_base(oscars_ctx* c) {
   h.offB = ly.offB;
   h.lr = c->lr;
   h.dlog = c->dlog;
+  h.err = c->err;
   if (c->L >= 2) {
     h.G = c->G[c->L - 2];
     h.GT = c->GT[c->L - 2];
@@ -624,7 +627,10 @@ cudaError_t enqueue_step(oscars_ctx* c, int s, int na, const int* wid, const int
   h.loss_part = c->loss_part;
   h.part_mul = c->max_tau;
   h.part_add = s;
-  if (head_fused_supported(h.H, h.B, h.C)) {
+  if (head_tc_supported(h.H, h.B, h.C)) {
+    ProfScope ps(c, "head_fused", st);
+    if ((e = launch_head_tc(c->mHeadIn, c->mHeadW, h, na, st)) != cudaSuccess) return e;
+  } else if (head_fused_supported(h.H, h.B, h.C)) {
     ProfScope ps(c, "head_fused", st);
     if ((e = launch_head_fused(h, na, st)) != cudaSuccess) return e;
   } else {
@@ -1263,6 +1269,12 @@ oscars_status allocate_mlp(oscars_ctx* c) {
       ok &= make_map(&c->mG[l], c->G[l], ly.out, B, W, ly.out * 2ull, static_cast<uint64_t>(B) * ly.out * 2ull, B);
     }
     if (!ok) return fail(c, OSCARS_ECUDA, "cuTensorMapEncodeTiled failed (or the driver entry point is missing)");
+  }
+  {
+    const Layer& hl = c->layers.back();
+    if (!make_map(&c->mHeadIn, c->A[L - 1], hl.in, B, W, hl.in * 2ull, static_cast<uint64_t>(B) * hl.in * 2ull, 128) ||
+        !make_map(&c->mHeadW, c->shadow + hl.offW, hl.in, hl.out, slots64, hl.in * 2ull, c->P_pad * 2ull, 16))
+      return fail(c, OSCARS_ECUDA, "cuTensorMapEncodeTiled failed (head)");
   }
   return OSCARS_OK;
 }

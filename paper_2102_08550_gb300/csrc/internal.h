@@ -162,8 +162,16 @@ struct HeadArgs {
   __nv_bfloat16* G;           // [lanes][B][H] (head_bwd)
   __nv_bfloat16* GT;          // [lanes][H][B]
   float* gb;                  // [lanes][H]
+  int* err;                   // device error word (bounded waits of the tensor-core head)
 };
 cudaError_t launch_head_fwd(const HeadArgs& a, int n_active, cudaStream_t s);
+// forward + backward of the last layer on the tensor cores (csrc/head_tc.cu):
+// one cluster of H/128 CTAs per active lane; C = 10, 32 <= B <= 128.  mH: the
+// layer input [lane][B][H] bf16, box {64, 128}; mW2: the head weights of every
+// slot [slot][C][H] bf16, box {64, 16}; both with 128-byte swizzle.
+bool head_tc_supported(int H, int B, int C);
+cudaError_t launch_head_tc(const CUtensorMap& mH, const CUtensorMap& mW2, const HeadArgs& a, int n_active,
+                           cudaStream_t s);
 // forward + backward of the last layer in one launch: one cluster of H/128
 // CTAs per active lane (H <= 1024); false if the shape needs the two-kernel path
 bool head_fused_supported(int H, int B, int C);
