@@ -165,6 +165,11 @@ struct oscars_ctx {
   int64_t eval_part_cap = 0;
   // tensor maps per layer
   std::vector<CUtensorMap> mShadow, mShadowMN, mA, mG, mGT, mAT;
+  // G^T [lane][out][B] in boxes of 64 x 64: the MN-major B operand of the input
+  // gradient.  With it (g_rows false: B a multiple of 64 and the tensor-core
+  // head) the row-major output gradients G are neither kept nor written.
+  std::vector<CUtensorMap> mGTmn;
+  bool g_rows = true;
   // fp32 W_l of every slot: boxes {32, 128} (loads) and {32, 32} (stores), and
   // the bf16 copy with boxes {64, 32} (stores): the persistent weight gradient
   std::vector<CUtensorMap> mMaster, mMasterSt, mShadowSt;
@@ -587,7 +592,7 @@ HeadArgs head_base(oscars_ctx* c) {
   h.dlog = c->dlog;
   h.err = c->err;
   if (c->L >= 2) {
-    h.G = c->G[c->L - 2];
+    h.G = c->g_rows ? c->G[c->L - 2] : nullptr;
     h.GT = c->GT[c->L - 2];
     h.gb = c->gb[c->L - 2];
   }
@@ -651,11 +656,13 @@ cudaError_t enqueue_step(oscars_ctx* c, int s, int na, const int* wid, const int
       g.a_z_src = 1;
       g.b_z_src = 0;
       g.hmask = c->A[l];
-      g.out = c->G[l - 1];
+      g.out = c->g_rows ? c->G[l - 1] : nullptr;
+      g.b_mn = c->g_rows ? 0 : 1;
       g.outT = c->GT[l - 1];
       g.gb_out = c->gb[l - 1];
       ProfScope ps(c, "gemm_dh", st);
-      if ((e = launch_gemm(kEpiDh, c->mShadowMN[l], c->mG[l], g, na, st)) != cudaSuccess) return e;
+      if ((e = launch_gemm(kEpiDh, c->mShadowMN[l], c->g_rows ? c->mG[l] : c->mGTmn[l], g, na, st)) != cudaSuccess)
+        return e;
     }
     const CUtensorMap& mX = l == 0 ? c->mAT0s[s] : c->mAT[l];
     if (gemm_dw_supported(ly.out, ly.in, c->B)) {
@@ -1219,6 +1226,10 @@ oscars_status allocate_mlp(oscars_ctx* c) {
   c->A.assign(L, nullptr);
   c->AT.assign(L, nullptr);
   c->G.assign(L, nullptr);
+  {
+    const Layer& hl = c->layers.back();
+    c->g_rows = !(B % 64 == 0 && head_tc_supported(hl.in, B, hl.out));
+  }
   c->GT.assign(L, nullptr);
   c->gb.assign(L, nullptr);
   for (int l = 0; l < L; ++l) {
@@ -1227,7 +1238,7 @@ oscars_status allocate_mlp(oscars_ctx* c) {
       return fail(c, OSCARS_ENOMEM, "device allocation failed (activations)");
     if (l + 1 < L) {
       const size_t gsz = static_cast<size_t>(W) * B * c->dims[l + 1];
-      if (!dev_alloc(c, &c->G[l], gsz) || !dev_alloc(c, &c->GT[l], gsz) ||
+      if ((c->g_rows && !dev_alloc(c, &c->G[l], gsz)) || !dev_alloc(c, &c->GT[l], gsz) ||
           !dev_alloc(c, &c->gb[l], static_cast<size_t>(W) * c->dims[l + 1]))
         return fail(c, OSCARS_ENOMEM, "device allocation failed (gradients)");
     }
@@ -1243,6 +1254,7 @@ oscars_status allocate_mlp(oscars_ctx* c) {
   c->mShadowMN.resize(L);
   c->mA.resize(L);
   c->mG.resize(L);
+  c->mGTmn.resize(L);
   c->mGT.resize(L);
   c->mAT.resize(L);
   const uint64_t slots64 = slots;
@@ -1266,7 +1278,10 @@ oscars_status allocate_mlp(oscars_ctx* c) {
       // MN-major A operand (M = in, K = out) of the input-gradient GEMM
       ok &= make_map(&c->mShadowMN[l], c->shadow + ly.offW, ly.in, ly.out, slots64, ly.in * 2ull, c->P_pad * 2ull, 64);
       // output gradient [lane][B][out]: B operand of the input-gradient GEMM
-      ok &= make_map(&c->mG[l], c->G[l], ly.out, B, W, ly.out * 2ull, static_cast<uint64_t>(B) * ly.out * 2ull, B);
+      if (c->g_rows)
+        ok &= make_map(&c->mG[l], c->G[l], ly.out, B, W, ly.out * 2ull, static_cast<uint64_t>(B) * ly.out * 2ull, B);
+      else   // output gradient^T [lane][out][B], boxes of 64 samples x 64 outputs: the MN-major B operand
+        ok &= make_map(&c->mGTmn[l], c->GT[l], B, ly.out, W, B * 2ull, static_cast<uint64_t>(B) * ly.out * 2ull, 64);
     }
     if (!ok) return fail(c, OSCARS_ECUDA, "cuTensorMapEncodeTiled failed (or the driver entry point is missing)");
   }

@@ -88,7 +88,7 @@ __device__ __forceinline__ void epi_dh_mask(const GemmArgs& a, int wid, int m, i
 
 __device__ __forceinline__ float epi_dh(const GemmArgs& a, int wid, int m, int n0, const float (&v)[32],
                                         const unsigned short (&mk)[32]) {
-  __nv_bfloat16* out = a.out + static_cast<int64_t>(wid) * a.N * a.M;
+  __nv_bfloat16* out = a.out ? a.out + static_cast<int64_t>(wid) * a.N * a.M : nullptr;
   uint32_t pk[16];
   float gsum = 0.f;
 #pragma unroll
@@ -100,8 +100,10 @@ __device__ __forceinline__ float epi_dh(const GemmArgs& a, int wid, int m, int n
     gsum += g0;
     gsum += g1;
     const __nv_bfloat162 p = __floats2bfloat162_rn(g0, g1);
-    out[e0] = p.x;
-    out[e1] = p.y;
+    if (out) {   // the row-major copy only when a consumer reads it K-major
+      out[e0] = p.x;
+      out[e1] = p.y;
+    }
     pk[c >> 1] = *reinterpret_cast<const uint32_t*>(&p);
   }
   uint4* outT = reinterpret_cast<uint4*>(a.outT + (static_cast<int64_t>(wid) * a.M + m) * a.N + n0);
@@ -233,12 +235,20 @@ __global__ void __launch_bounds__(warps_for<EPI>() * 32) gemm_tc_kernel(const __
       } else {
         tma_load_3d(sA + s * kABytes, &mapA, kb * BK, m0, za, &full[s]);
       }
-      tma_load_3d(sB + s * Cfg::kBBytes, &mapB, kb * BK, n0, zb, &full[s]);
+      if (EPI == kEpiDh && a.b_mn) {
+        // B = G read MN-major from G^T [K = out][N = batch]: boxes of 64 N x 64 K, 8 KB apart
+        for (int nb = 0; nb < BN / 64; ++nb)
+          tma_load_3d(sB + s * Cfg::kBBytes + nb * 8192, &mapB, n0 + 64 * nb, kb * BK, zb, &full[s]);
+      } else {
+        tma_load_3d(sB + s * Cfg::kBBytes, &mapB, kb * BK, n0, zb, &full[s]);
+      }
     }
   } else if (warp == 1 && lane == 0) {
     // MMA issuer
-    // A MN-major (transpose-A bit 15) for the input gradient, K-major otherwise
-    constexpr uint32_t idesc = idesc_bf16_f32(BM, BN) | (EPI == kEpiDh ? (1u << 15) : 0u);
+    // A MN-major (transpose-A bit 15) for the input gradient, K-major otherwise;
+    // B MN-major (bit 16) when the input gradient reads G^T
+    const bool bmn = EPI == kEpiDh && a.b_mn;
+    const uint32_t idesc = idesc_bf16_f32(BM, BN) | (EPI == kEpiDh ? (1u << 15) : 0u) | (bmn ? (1u << 16) : 0u);
     for (int kb = 0; kb < nk; ++kb) {
       const int s = kb % stages;
       if (!mbar_wait(&full[s], (kb / stages) & 1, a.err, kDevTimeoutFull)) break;
@@ -250,7 +260,8 @@ __global__ void __launch_bounds__(warps_for<EPI>() * 32) gemm_tc_kernel(const __
         // K-major: 16 K-elements are 32 bytes along a row; MN-major: 16 rows of 128 bytes
         const uint64_t adesc = EPI == kEpiDh ? smem_desc_mn128(a_base + j * 2048, kABytes / 2)
                                              : smem_desc_k128(a_base + j * 32);
-        umma_bf16(tmem, adesc, smem_desc_k128(b_base + j * 32), idesc, (kb | j) != 0 ? 1u : 0u);
+        const uint64_t bdesc = bmn ? smem_desc_mn128(b_base + j * 2048, 8192) : smem_desc_k128(b_base + j * 32);
+        umma_bf16(tmem, adesc, bdesc, idesc, (kb | j) != 0 ? 1u : 0u);
       }
       umma_commit(&empty[s]);
     }

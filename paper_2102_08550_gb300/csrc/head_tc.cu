@@ -376,8 +376,10 @@ __global__ void __launch_bounds__(kHTThreads) head_tc_kernel(const __grid_consta
           gsum += d0;
           gsum += d1;
           const __nv_bfloat162 p = __floats2bfloat162_rn(d0, d1);
-          *h0 = p.x;      // the h tile now holds the bf16 input gradient at (b, f)
-          *h1 = p.y;
+          if (a.G) {      // the h tile now holds the bf16 input gradient at (b, f), for the G rows below
+            *h0 = p.x;
+            *h1 = p.y;
+          }
           pk[j >> 1] = *reinterpret_cast<const uint32_t*>(&p);
         }
         uint4* gt = reinterpret_cast<uint4*>(a.GT + (static_cast<int64_t>(w) * H + k0 + f) * B + b0);
@@ -394,7 +396,7 @@ __global__ void __launch_bounds__(kHTThreads) head_tc_kernel(const __grid_consta
   tc_fence_before();
   __syncthreads();
   if (t < F && ok) a.gb[static_cast<int64_t>(w) * H + k0 + t] = NH == 2 ? gbp[t] : gbp[t] + gbp[F + t];
-  if (ok) {   // G rows: 16-byte chunks of 8 features
+  if (ok && a.G) {   // G rows: 16-byte chunks of 8 features (when a consumer reads G K-major)
     for (int q = t; q < B * (F / 8); q += kHTThreads) {
       const int b = q / (F / 8), j = q % (F / 8);
       *reinterpret_cast<uint4*>(a.G + (static_cast<int64_t>(w) * B + b) * H + k0 + 8 * j) =

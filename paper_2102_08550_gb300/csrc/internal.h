@@ -96,9 +96,10 @@ struct GemmArgs {
   const int* src;     // [n_active]
   int M, N, K;
   int a_z_src, b_z_src;  // TMA z coordinate of A / B: 1 = src slot, 0 = lane id
+  int b_mn;              // kEpiDh: B read MN-major (G^T [lane][K][N] in boxes of 64 N x 64 K; N % 64 == 0)
   int* err;
   // kEpiFwd: out = relu(acc + bias[m]) -> H [lane][N][M], HT [lane][M][N]
-  // kEpiDh : out = acc * (Hmask[lane][n][m] > 0) -> G, GT, gb[lane][m]
+  // kEpiDh : out = acc * (Hmask[lane][n][m] > 0) -> G (if out), GT, gb[lane][m]
   // kEpiDw : W[dst] = W[src] - lr * acc (rows m, cols n < N), shadows, bias
   const float* master;      // fp32 slab base
   float* master_w;          // same slab (written)
