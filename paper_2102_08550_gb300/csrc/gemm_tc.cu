@@ -177,11 +177,29 @@ __device__ __forceinline__ void epi_store(const GemmArgs& a, int m, int n0, cons
   }
 }
 
-template <int BN, int EPI>
+// Split-K (SPLIT > 1, forward and input-gradient epilogues): a cluster of
+// SPLIT CTAs shares one output tile, CTA r multiplying K-blocks [r nk / SPLIT,
+// (r + 1) nk / SPLIT).  Each CTA pushes its fp32 partial rows into the CTA
+// that owns them (rows [r 128 / SPLIT, (r + 1) 128 / SPLIT) belong to CTA r)
+// through distributed shared memory, one cluster barrier follows, and each
+// owner sums the SPLIT partials in rank order and runs the epilogue on its
+// rows.  Used when a launch has too few tiles to fill the GPU (the tail of a
+// round, where one worker with many local steps runs alone).
+constexpr int kRedLd = 4;   // padding of a partial row (floats)
+
+__device__ __forceinline__ void st_dsmem_f32x4(float* local, uint32_t rank, float4 v) {
+  uint32_t remote;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(smem_u32(local)), "r"(rank));
+  asm volatile("st.shared::cluster.v4.f32 [%0], {%1, %2, %3, %4};" ::"r"(remote), "f"(v.x), "f"(v.y), "f"(v.z), "f"(v.w)
+               : "memory");
+}
+
+template <int BN, int EPI, int SPLIT = 1>
 __global__ void __launch_bounds__(warps_for<EPI>() * 32) gemm_tc_kernel(const __grid_constant__ CUtensorMap mapA,
                                                            const __grid_constant__ CUtensorMap mapB,
                                                            const __grid_constant__ GemmArgs a,
                                                            int stages) {
+  static_assert(SPLIT == 1 || EPI == kEpiFwd || EPI == kEpiDh, "split-K serves the forward and input-gradient GEMMs");
   using Cfg = TileCfg<BN>;
   extern __shared__ uint8_t smem_raw[];
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -194,10 +212,13 @@ __global__ void __launch_bounds__(warps_for<EPI>() * 32) gemm_tc_kernel(const __
   float* epi_tiles = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(full) + kBarrierBytes);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int li = blockIdx.z;
+  const int li = blockIdx.z / SPLIT;
+  const int rank = SPLIT > 1 ? static_cast<int>(cluster_ctarank()) : 0;
   const int wid = a.wid ? a.wid[li] : li, src = a.src ? a.src[li] : li;
   const int m0 = blockIdx.x * BM, n0 = blockIdx.y * BN;
-  const int nk = (a.K + BK - 1) / BK;
+  const int nk_all = (a.K + BK - 1) / BK;
+  const int kb0 = rank * nk_all / SPLIT;                 // this CTA's K-blocks [kb0, kb0 + nk)
+  const int nk = (rank + 1) * nk_all / SPLIT - kb0;
 
   if (threadIdx.x == 0) {
     prefetch_tmap(&mapA);
@@ -227,20 +248,21 @@ __global__ void __launch_bounds__(warps_for<EPI>() * 32) gemm_tc_kernel(const __
       const int s = kb % stages;
       if (kb >= stages && !mbar_wait(&empty[s], ((kb / stages) + 1) & 1, a.err, kDevTimeoutEmpty)) break;
       mbar_arrive_expect_tx(&full[s], kABytes + Cfg::kBBytes);
+      const int k = (kb0 + kb) * BK;   // global K coordinate
       if constexpr (EPI == kEpiDh) {
         // A = W^T read MN-major from W [K = out][M = in]: two boxes of 64 M x
         // 64 K, the second 64 M-elements further along (8 KB in shared memory)
-        tma_load_3d(sA + s * kABytes, &mapA, m0, kb * BK, za, &full[s]);
-        tma_load_3d(sA + s * kABytes + kABytes / 2, &mapA, m0 + 64, kb * BK, za, &full[s]);
+        tma_load_3d(sA + s * kABytes, &mapA, m0, k, za, &full[s]);
+        tma_load_3d(sA + s * kABytes + kABytes / 2, &mapA, m0 + 64, k, za, &full[s]);
       } else {
-        tma_load_3d(sA + s * kABytes, &mapA, kb * BK, m0, za, &full[s]);
+        tma_load_3d(sA + s * kABytes, &mapA, k, m0, za, &full[s]);
       }
       if (EPI == kEpiDh && a.b_mn) {
         // B = G read MN-major from G^T [K = out][N = batch]: boxes of 64 N x 64 K, 8 KB apart
         for (int nb = 0; nb < BN / 64; ++nb)
-          tma_load_3d(sB + s * Cfg::kBBytes + nb * 8192, &mapB, n0 + 64 * nb, kb * BK, zb, &full[s]);
+          tma_load_3d(sB + s * Cfg::kBBytes + nb * 8192, &mapB, n0 + 64 * nb, k, zb, &full[s]);
       } else {
-        tma_load_3d(sB + s * Cfg::kBBytes, &mapB, kb * BK, n0, zb, &full[s]);
+        tma_load_3d(sB + s * Cfg::kBBytes, &mapB, k, n0, zb, &full[s]);
       }
     }
   } else if (warp == 1 && lane == 0) {
@@ -268,6 +290,79 @@ __global__ void __launch_bounds__(warps_for<EPI>() * 32) gemm_tc_kernel(const __
     umma_commit(accum);  // arrives once every issued MMA has completed
   }
   __syncwarp();
+
+  if constexpr (SPLIT > 1) {
+    // ---- split-K epilogue (4 warps): push the partial rows to their owners
+    constexpr int R = BM / SPLIT;                   // rows owned per CTA
+    constexpr int ld = BN + kRedLd;
+    float* red = epi_tiles;                         // [SPLIT][R][ld] fp32: the partials of this CTA's rows
+    int acc_ok = mbar_wait(accum, 0, a.err, kDevTimeoutAccum) ? 1 : 0;
+    acc_ok = __all_sync(0xffffffffu, acc_ok);
+    tc_fence_after();
+    const int row = (warp & 3) * 32 + lane;        // accumulator row of this thread
+    const int owner = row / R;
+    float* dst = red + (rank * R + (row - owner * R)) * ld;
+    const uint32_t trow = tmem + (static_cast<uint32_t>((warp & 3) * 32) << 16);
+#pragma unroll 1
+    for (int c0 = 0; c0 < BN; c0 += 32) {
+      float v[32];
+      if (acc_ok) tmem_ld_32x32b_x32(trow + c0, v);
+      else
+#pragma unroll
+        for (int j = 0; j < 32; ++j) v[j] = 0.f;
+#pragma unroll
+      for (int q = 0; q < 8; ++q) {
+        const float4 p4 = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+        if (owner == rank) *reinterpret_cast<float4*>(dst + c0 + 4 * q) = p4;
+        else st_dsmem_f32x4(dst + c0 + 4 * q, owner, p4);
+      }
+    }
+    tc_fence_before();
+    cluster_sync();   // every partial has landed in its owner
+    // own rows: item = (row, 32-column chunk); partials summed in rank order
+    float* gpart = red + SPLIT * R * ld;            // [R][BN / 32] bias-gradient partials (input gradient)
+    for (int it = threadIdx.x; it < R * (BN / 32); it += warps_for<EPI>() * 32) {
+      const int rl = it / (BN / 32), c0 = (it % (BN / 32)) * 32;
+      float v[32];
+#pragma unroll
+      for (int j = 0; j < 32; ++j) v[j] = 0.f;
+#pragma unroll
+      for (int p = 0; p < SPLIT; ++p) {
+        const float* src_row = red + (p * R + rl) * ld + c0;
+#pragma unroll
+        for (int q = 0; q < 8; ++q) {
+          const float4 x = *reinterpret_cast<const float4*>(src_row + 4 * q);
+          v[4 * q] += x.x;
+          v[4 * q + 1] += x.y;
+          v[4 * q + 2] += x.z;
+          v[4 * q + 3] += x.w;
+        }
+      }
+      const int m = m0 + rank * R + rl;
+      if constexpr (EPI == kEpiFwd) {
+        epi_fwd<EPI>(a, wid, src, m, n0 + c0, v);
+      } else {
+        unsigned short mk[32];
+        epi_dh_mask(a, wid, m, n0 + c0, mk);
+        gpart[rl * (BN / 32) + c0 / 32] = epi_dh(a, wid, m, n0 + c0, v, mk);
+      }
+    }
+    if constexpr (EPI == kEpiDh) {
+      __syncthreads();
+      for (int rl = threadIdx.x; rl < R; rl += warps_for<EPI>() * 32) {
+        float g = 0.f;
+        for (int c = 0; c < BN / 32; ++c) g += gpart[rl * (BN / 32) + c];
+        a.gb_out[static_cast<int64_t>(wid) * a.M + m0 + rank * R + rl] = g;
+      }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 2) {
+      tc_fence_after();
+      tmem_dealloc(tmem, Cfg::kTmemCols);
+    }
+    return;
+  }
 
   // epilogue: thread = one accumulator row
   unsigned short mk[32];   // input-gradient mask of the next 32 columns, read while the MMAs run
@@ -348,38 +443,74 @@ size_t smem_floor_for_tmem(uint32_t cols) {
   return per_sm / (max_ctas + 1) - 1024 + 16;
 }
 
-template <int BN, int EPI>
-cudaError_t launch_tile(const CUtensorMap& mA, const CUtensorMap& mB, const GemmArgs& a, int n_active,
-                        cudaStream_t s) {
-  using Cfg = TileCfg<BN>;
-  const int nk = (a.K + BK - 1) / BK;
-  dim3 grid(a.M / BM, (a.N + BN - 1) / BN, n_active);
-  // A grid that fits one CTA per SM gets as many stages as K-blocks, within
-  // ~200 KB of shared memory: the whole K extent of these skinny GEMMs is
-  // then in flight at once.  A larger grid gets stages for ~100 KB, so two
-  // CTAs share each SM and the grid runs in one wave instead of two (the
-  // bytes in flight per SM stay the same).
+int device_sms() {
   static int sms = 0;
   if (sms == 0) {
     int dev = 0;
     cudaGetDevice(&dev);
     if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || sms < 1) sms = 1;
   }
+  return sms;
+}
+
+template <int BN, int EPI, int SPLIT = 1>
+cudaError_t launch_tile(const CUtensorMap& mA, const CUtensorMap& mB, const GemmArgs& a, int n_active,
+                        cudaStream_t s) {
+  using Cfg = TileCfg<BN>;
+  const int nk = ((a.K + BK - 1) / BK + SPLIT - 1) / SPLIT;   // K-blocks of the CTA with the most
+  dim3 grid(a.M / BM, (a.N + BN - 1) / BN, n_active * SPLIT);
+  // A grid that fits one CTA per SM gets as many stages as K-blocks, within
+  // ~200 KB of shared memory: the whole K extent of these skinny GEMMs is
+  // then in flight at once.  A larger grid gets stages for ~100 KB, so two
+  // CTAs share each SM and the grid runs in one wave instead of two (the
+  // bytes in flight per SM stay the same).  A split grid keeps room for the
+  // partial rows its CTAs exchange.
+  const int sms = device_sms();
   const long long ctas = static_cast<long long>(grid.x) * grid.y * grid.z;
-  const int budget = ctas > sms ? 100 * 1024 : 200 * 1024;
+  const size_t red_bytes = SPLIT > 1 ? sizeof(float) * (static_cast<size_t>(BM) * (BN + kRedLd) + BM / SPLIT * (BN / 32))
+                                     : 0;
+  const int budget = SPLIT > 1 ? 150 * 1024 : ctas > sms ? 100 * 1024 : 200 * 1024;
   const int max_stages = static_cast<int>((budget - (EPI == kEpiDw ? 8 * 32 * 33 * 4 : 0)) / Cfg::kStageBytes);
   int stages = nk < max_stages ? nk : (max_stages < 8 ? max_stages : 8);
   if (stages < 2) stages = nk < 2 ? nk : 2;
   constexpr int kWarps = warps_for<EPI>();
   size_t smem = 1024 + static_cast<size_t>(stages) * Cfg::kStageBytes + kBarrierBytes +
-                (EPI == kEpiDw ? sizeof(float) * kWarps * kEpiTileFloats : 0);
+                (EPI == kEpiDw ? sizeof(float) * kWarps * kEpiTileFloats : 0) + red_bytes;
   const size_t floor_b = smem_floor_for_tmem(Cfg::kTmemCols);
   if (smem < floor_b) smem = floor_b;
-  cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<BN, EPI>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<BN, EPI, SPLIT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(smem));
   if (e != cudaSuccess) return e;
-  gemm_tc_kernel<BN, EPI><<<grid, kWarps * 32, smem, s>>>(mA, mB, a, stages);
-  return cudaGetLastError();
+  if constexpr (SPLIT == 1) {
+    gemm_tc_kernel<BN, EPI, 1><<<grid, kWarps * 32, smem, s>>>(mA, mB, a, stages);
+    return cudaGetLastError();
+  } else {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = dim3(kWarps * 32, 1, 1);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = 1;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = SPLIT;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<BN, EPI, SPLIT>, mA, mB, a, stages);
+  }
+}
+
+// K split of a forward or input-gradient launch: 4 or 2 CTAs per tile when
+// the unsplit grid would leave most of the GPU idle and each CTA keeps at
+// least 4 K-blocks
+int split_for(int M, int N, int BN, int K, int n_active) {
+  const long long tiles = static_cast<long long>(M / BM) * ((N + BN - 1) / BN) * n_active;
+  const int nk = (K + BK - 1) / BK;
+  const int sms = device_sms();
+  if (tiles * 4 <= sms && nk >= 16) return 4;
+  if (tiles * 2 <= sms && nk >= 8) return 2;
+  return 1;
 }
 
 }  // namespace
@@ -395,7 +526,10 @@ cudaError_t launch_gemm(int epi, const CUtensorMap& mA, const CUtensorMap& mB, c
   if (epi == kEpiDw) return launch_tile<128, kEpiDw>(mA, mB, a, n_active, s);
   if (epi == kEpiStore) return launch_tile<128, kEpiStore>(mA, mB, a, n_active, s);
   const int bn = gemm_bn_for(epi, a.N);
+  const int split = bn == 128 ? split_for(a.M, a.N, bn, a.K, n_active) : 1;
   if (epi == kEpiFwd) {
+    if (split == 4) return launch_tile<128, kEpiFwd, 4>(mA, mB, a, n_active, s);
+    if (split == 2) return launch_tile<128, kEpiFwd, 2>(mA, mB, a, n_active, s);
     switch (bn) {
       case 32: return launch_tile<32, kEpiFwd>(mA, mB, a, n_active, s);
       case 64: return launch_tile<64, kEpiFwd>(mA, mB, a, n_active, s);
@@ -404,6 +538,8 @@ cudaError_t launch_gemm(int epi, const CUtensorMap& mA, const CUtensorMap& mB, c
       default: return cudaErrorInvalidValue;
     }
   }
+  if (split == 4) return launch_tile<128, kEpiDh, 4>(mA, mB, a, n_active, s);
+  if (split == 2) return launch_tile<128, kEpiDh, 2>(mA, mB, a, n_active, s);
   switch (bn) {
     case 32: return launch_tile<32, kEpiDh>(mA, mB, a, n_active, s);
     case 64: return launch_tile<64, kEpiDh>(mA, mB, a, n_active, s);

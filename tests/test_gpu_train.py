@@ -98,6 +98,8 @@ SMALL = [
     ("2layer", [784, 512, 10], 4, 64, 512, 8),
     ("3layer", [200, 256, 128, 10], 3, 32, 256, 6),       # ragged K tail, middle layer (input-gradient GEMM)
     ("4layer", [96, 128, 256, 128, 10], 5, 128, 512, 4),
+    # two workers, deep K: the forward and input-gradient GEMMs split K over clusters of 4 and 2 CTAs
+    ("split-k", [1024, 512, 512, 10], 2, 64, 256, 4),
 ]
 
 
