@@ -39,7 +39,7 @@
 //     bias;
 //  D  weight gradient of the group's 128 rows over the CTA's own input
 //     columns, dW0[o][k] = sum_b dz0[b][o] X[b][k], on tcgen05 in 32-column
-//     tiles (X^T tiles by TMA into a six-deep ring, the first ones during
+//     tiles (X^T tiles by TMA into a four-deep ring, the first ones during
 //     step F; three TMEM buffers); the epilogue reads the
 //     gradient and the fp32 master from TMEM, applies W0 <- W0 - lr dW0,
 //     stores the master back to TMEM and its bf16 copy into the resident A
@@ -82,7 +82,7 @@ constexpr int kFMaxCluster = 8;
 constexpr int kFBK = 64;               // K-block (bf16 elements, 128 bytes)
 constexpr int kND = 32;                // columns per weight-gradient tile
 constexpr int kNBD = 3;                // weight-gradient TMEM buffers
-constexpr int kNXD = 6;                // X^T tile buffers in shared memory
+constexpr int kNXD = 4;                // X^T tile buffers in shared memory
 constexpr int kTAcc = 512 - kNBD * kND;   // first TMEM column of the accumulators = master columns
 constexpr int kMaxKb = (kTAcc + kFBK - 1) / kFBK;   // resident K-blocks of W0
 constexpr int kW0Blk = kFU * kFBK * 2; // one resident K-block: 128 rows x 64 columns bf16
@@ -132,7 +132,7 @@ struct FCfg {
   static_assert(S == 1 || S == 2, "one or two CTAs per group");
   static_assert(kTAcc + B <= 512, "the forward accumulator must fit the accumulator columns");
   static constexpr int kUPC = kFU / S;                      // units per CTA in steps F (kept) and H
-  static constexpr int kStagesF = 4;
+  static constexpr int kStagesF = 5;
   static constexpr int kBBytes = B * kFBK * 2;              // X tile: B rows x 64 k
   static constexpr int kXtBytes = kND * kFBK * 2;           // X^T tile: 32 rows x 64 k (K padded)
   static constexpr int kDRing = kNXD * kXtBytes;
