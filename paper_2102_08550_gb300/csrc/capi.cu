@@ -613,6 +613,7 @@ cudaError_t enqueue_forward(oscars_ctx* c, const int* wid, const int* src, int n
     g.offB = ly.offB;
     g.out = c->A[l + 1];
     g.outT = c->AT[l + 1];
+    g.pdl = c->profiling ? 0 : 1;   // overlaps its prologue with the previous kernel's tail
     ProfScope ps(c, "gemm_fwd", st);
     cudaError_t e = launch_gemm(kEpiFwd, c->mShadow[l], l == 0 ? c->mA0s[step] : c->mA[l], g, na, st);
     if (e != cudaSuccess) return e;
@@ -633,6 +634,7 @@ cudaError_t enqueue_step(oscars_ctx* c, int s, int na, const int* wid, const int
   h.part_mul = c->max_tau;
   h.part_add = s;
   if (head_tc_supported(h.H, h.B, h.C)) {
+    h.pdl = c->profiling ? 0 : 1;
     ProfScope ps(c, "head_fused", st);
     if ((e = launch_head_tc(c->mHeadIn, c->mHeadW, h, na, st)) != cudaSuccess) return e;
   } else if (head_fused_supported(h.H, h.B, h.C)) {
@@ -658,6 +660,7 @@ cudaError_t enqueue_step(oscars_ctx* c, int s, int na, const int* wid, const int
       g.hmask = c->A[l];
       g.out = c->g_rows ? c->G[l - 1] : nullptr;
       g.b_mn = c->g_rows ? 0 : 1;
+      g.pdl = c->profiling ? 0 : 1;
       g.outT = c->GT[l - 1];
       g.gb_out = c->gb[l - 1];
       ProfScope ps(c, "gemm_dh", st);
@@ -680,6 +683,7 @@ cudaError_t enqueue_step(oscars_ctx* c, int s, int na, const int* wid, const int
       d.offB = ly.offB;
       d.gb = c->gb[l];
       d.err = c->err;
+      d.pdl = c->profiling ? 0 : 1;
       ProfScope ps(c, "gemm_dw_sgd", st);
       if ((e = launch_gemm_dw(c->mGT[l], mX, c->mMaster[l], c->mMasterSt[l], c->mShadowSt[l], d, c->sms, st)) !=
           cudaSuccess)

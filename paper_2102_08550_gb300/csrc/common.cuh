@@ -124,6 +124,17 @@ __device__ __forceinline__ void bar_named(int id, int count) {
   asm volatile("barrier.sync %0, %1;" ::"r"(id), "r"(count) : "memory");
 }
 
+// Programmatic dependent launch.  A kernel launched as a programmatic
+// dependent may start while the previous kernel on its stream finishes;
+// pdl_wait() blocks until that kernel has completed and its memory is
+// visible (a no-op without a programmatic dependency), so a kernel calls it
+// after its prologue (barriers, TMEM, tensor-map prefetch) and before its
+// first global access.  pdl_trigger() lets this kernel's own dependent start
+// its prologue (every CTA of this grid has started by then: no CTA of it can
+// be kept from starting by the dependent's).
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
 __device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(bar)) : "memory");
 }

@@ -106,6 +106,8 @@ __global__ void __launch_bounds__(kDwThreads, 1) gemm_dw_kernel(const __grid_con
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = bars->tmem;
+  pdl_wait();      // the previous kernel's outputs (gradients, bias gradients) are complete
+  pdl_trigger();
 
   if (warp == 0 && lane_id == 0) {
     // ---- TMA producer
@@ -262,8 +264,17 @@ cudaError_t launch_gemm_dw(const CUtensorMap& mA, const CUtensorMap& mB, const C
   if (e != cudaSuccess) return e;
   const int tiles = a.n_active * (a.M / kDwTile) * ((a.N + kDwTile - 1) / kDwTile);
   const int grid = tiles < sms ? tiles : sms;
-  gemm_dw_kernel<<<grid, kDwThreads, kDwSmem, s>>>(mA, mB, mMaster, mMasterSt, mShadowSt, a);
-  return cudaGetLastError();
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid, 1, 1);
+  cfg.blockDim = dim3(kDwThreads, 1, 1);
+  cfg.dynamicSmemBytes = kDwSmem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = a.pdl ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, gemm_dw_kernel, mA, mB, mMaster, mMasterSt, mShadowSt, a);
 }
 
 }  // namespace oscars

@@ -239,6 +239,8 @@ __global__ void __launch_bounds__(warps_for<EPI>() * 32) gemm_tc_kernel(const __
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
+  pdl_wait();      // the previous kernel's outputs (operands, masks, biases) are complete
+  pdl_trigger();
 
   if (warp == 0 && lane == 0) {
     // TMA producer
@@ -481,24 +483,28 @@ cudaError_t launch_tile(const CUtensorMap& mA, const CUtensorMap& mB, const Gemm
   cudaError_t e = cudaFuncSetAttribute(gemm_tc_kernel<BN, EPI, SPLIT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        static_cast<int>(smem));
   if (e != cudaSuccess) return e;
-  if constexpr (SPLIT == 1) {
-    gemm_tc_kernel<BN, EPI, 1><<<grid, kWarps * 32, smem, s>>>(mA, mB, a, stages);
-    return cudaGetLastError();
-  } else {
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = grid;
-    cfg.blockDim = dim3(kWarps * 32, 1, 1);
-    cfg.dynamicSmemBytes = smem;
-    cfg.stream = s;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeClusterDimension;
-    attr[0].val.clusterDim.x = 1;
-    attr[0].val.clusterDim.y = 1;
-    attr[0].val.clusterDim.z = SPLIT;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<BN, EPI, SPLIT>, mA, mB, a, stages);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = dim3(kWarps * 32, 1, 1);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr[2];
+  int n = 0;
+  if (SPLIT > 1) {
+    attr[n].id = cudaLaunchAttributeClusterDimension;
+    attr[n].val.clusterDim.x = 1;
+    attr[n].val.clusterDim.y = 1;
+    attr[n].val.clusterDim.z = SPLIT;
+    ++n;
   }
+  if (a.pdl) {
+    attr[n].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[n].val.programmaticStreamSerializationAllowed = 1;
+    ++n;
+  }
+  cfg.attrs = attr;
+  cfg.numAttrs = n;
+  return cudaLaunchKernelEx(&cfg, gemm_tc_kernel<BN, EPI, SPLIT>, mA, mB, a, stages);
 }
 
 // K split of a forward or input-gradient launch: 4 or 2 CTAs per tile when

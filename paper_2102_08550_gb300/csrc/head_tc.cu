@@ -158,7 +158,10 @@ __global__ void __launch_bounds__(kHTThreads) head_tc_kernel(const __grid_consta
     mbar_init(tma_bar, 1);
     mbar_init(mma_bar, 1);
     fence_barrier_init();
-    // the h and W2 tiles, requested first: everything else of the prologue overlaps them
+  }
+  pdl_wait();      // the layer input (the previous kernel's output) is complete
+  if (t == 0) {
+    // the h and W2 tiles, requested first: the rest of the prologue overlaps them
     mbar_arrive_expect_tx(tma_bar, (F / 64) * (kHTRows * 128 + kHTN * 128));
 #pragma unroll
     for (int q = 0; q < F / 64; ++q) {
@@ -179,6 +182,7 @@ __global__ void __launch_bounds__(kHTThreads) head_tc_kernel(const __grid_consta
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
+  pdl_trigger();
 
   // ---- 1. partial logits
   if (t == 0) {
@@ -432,13 +436,15 @@ cudaError_t launch_head_tc_nh(const CUtensorMap& mH, const CUtensorMap& mW2, con
   cfg.blockDim = dim3(kHTThreads, 1, 1);
   cfg.dynamicSmemBytes = Cfg::kSmem;
   cfg.stream = s;
-  cudaLaunchAttribute attr[1];
+  cudaLaunchAttribute attr[2];
   attr[0].id = cudaLaunchAttributeClusterDimension;
   attr[0].val.clusterDim.x = 1;
   attr[0].val.clusterDim.y = a.H / Cfg::F;
   attr[0].val.clusterDim.z = 1;
+  attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[1].val.programmaticStreamSerializationAllowed = 1;
   cfg.attrs = attr;
-  cfg.numAttrs = 1;
+  cfg.numAttrs = a.pdl ? 2 : 1;
   return cudaLaunchKernelEx(&cfg, head_tc_kernel<NH>, mH, mW2, a);
 }
 

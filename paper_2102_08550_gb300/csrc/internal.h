@@ -97,6 +97,7 @@ struct GemmArgs {
   int M, N, K;
   int a_z_src, b_z_src;  // TMA z coordinate of A / B: 1 = src slot, 0 = lane id
   int b_mn;              // kEpiDh: B read MN-major (G^T [lane][K][N] in boxes of 64 N x 64 K; N % 64 == 0)
+  int pdl;               // launch as a programmatic dependent of the previous kernel on the stream
   int* err;
   // kEpiFwd: out = relu(acc + bias[m]) -> H [lane][N][M], HT [lane][M][N]
   // kEpiDh : out = acc * (Hmask[lane][n][m] > 0) -> G (if out), GT, gb[lane][m]
@@ -132,6 +133,7 @@ struct DwArgs {
   int64_t offB;             // element offset of b_l in a slot
   const float* gb;          // [W][M] bias gradient
   int* err;
+  int pdl;                  // launch as a programmatic dependent of the previous kernel on the stream
 };
 bool gemm_dw_supported(int M, int N, int K);
 // mA: G^T [lane][M][K] bf16, box {64, 128}; mB: X^T [lane][N][K] bf16, box
@@ -164,6 +166,7 @@ struct HeadArgs {
   __nv_bfloat16* GT;          // [lanes][H][B]
   float* gb;                  // [lanes][H]
   int* err;                   // device error word (bounded waits of the tensor-core head)
+  int pdl;                    // tensor-core head: launch as a programmatic dependent
 };
 cudaError_t launch_head_fwd(const HeadArgs& a, int n_active, cudaStream_t s);
 // forward + backward of the last layer on the tensor cores (csrc/head_tc.cu):
