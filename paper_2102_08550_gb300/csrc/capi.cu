@@ -1179,6 +1179,9 @@ oscars_status allocate_cnn(oscars_ctx* c) {
   c->cnn_buf.assign(nbuf, nullptr);
   for (int i = 0; i < nbuf; ++i)
     if (!dev_alloc(c, &c->cnn_buf[i], act)) return fail(c, OSCARS_ENOMEM, "device allocation failed (activations)");
+  // the input buffer's channels past the image's stay zero: the staging kernel writes only the input channels
+  if (cudaMemset(c->cnn_buf[0], 0, act * sizeof(__nv_bfloat16)) != cudaSuccess)
+    return fail(c, OSCARS_ECUDA, "clearing the input buffer failed");
   const size_t tiles = static_cast<size_t>(B) * cnn_tiles_per_image();
   if (!dev_alloc(c, &c->cnn_g, static_cast<size_t>(W) * B * 64) ||
       !dev_alloc(c, &c->cnn_dg, static_cast<size_t>(W) * B * 64) ||

@@ -444,48 +444,68 @@ __global__ void conv_refresh_wt_kernel(const float* master, __nv_bfloat16* wt, i
 }
 
 // ------------------------------------------------------------------ input staging
-// grid (B * 8 tiles, active), 128 threads: one pixel each; the image row of
-// sample b is (start[lane] + s * B + b) mod n[lane] of the lane's shard
-// (fp32 NHWC, Cin channels); channels >= Cin are zero
+// grid (B * 8 tiles, active), 128 threads: the image row of sample b is
+// (start[lane] + s * B + b) mod n[lane] of the lane's shard (fp32 NHWC, Cin
+// channels).  Channels >= Cin stay zero: the buffer is cleared once when the
+// context is built, so only the 16-byte chunks that hold input channels are
+// written (one chunk for Cin <= 8), item = (pixel, chunk) with consecutive
+// threads on consecutive chunks.
 __global__ void __launch_bounds__(kCT) cnn_stage_kernel(const __grid_constant__ CnnStageArgs a) {
   const int tile = blockIdx.x, e = blockIdx.y;
   const int lane = a.wid[e];
-  const int b = tile / kTilesPerImg, pix = (tile % kTilesPerImg) * kTilePix + threadIdx.x;
+  const int b = tile / kTilesPerImg, pix0 = (tile % kTilesPerImg) * kTilePix;
   const int64_t n = a.n[lane];
   const int64_t row = (a.start[lane] + static_cast<int64_t>(a.step) * a.B + b) % n;
-  const float* src = a.x[lane] + row * static_cast<int64_t>(kPix) * a.Cin + static_cast<int64_t>(pix) * a.Cin;
-  float v[kCC];
+  const float* src = a.x[lane] + row * static_cast<int64_t>(kPix) * a.Cin;
+  __nv_bfloat16* dst = a.out + ((static_cast<int64_t>(lane) * a.B + b) * kPix + pix0) * kCC;
+  const int chunks = (a.Cin + 7) / 8;
+  for (int it = threadIdx.x; it < kTilePix * chunks; it += kCT) {
+    const int px = it / chunks, q = it - px * chunks;
+    float v[8];
 #pragma unroll
-  for (int c = 0; c < kCC; ++c) v[c] = c < a.Cin ? src[c] : 0.f;
-  __nv_bfloat16* dst = a.out + ((static_cast<int64_t>(lane) * a.B + b) * kPix + pix) * kCC;
-#pragma unroll
-  for (int q = 0; q < kCC / 8; ++q)
-    *reinterpret_cast<uint4*>(dst + 8 * q) =
-        make_uint4(pack_bf16x2(v[8 * q], v[8 * q + 1]), pack_bf16x2(v[8 * q + 2], v[8 * q + 3]),
-                   pack_bf16x2(v[8 * q + 4], v[8 * q + 5]), pack_bf16x2(v[8 * q + 6], v[8 * q + 7]));
-  if (a.labels && tile == 0 && threadIdx.x < 1) {
-    for (int bb = 0; bb < a.B; ++bb) {
-      const int64_t rr = (a.start[lane] + static_cast<int64_t>(a.step) * a.B + bb) % n;
-      a.labels[static_cast<int64_t>(lane) * a.B + bb] = a.y[lane][rr];
+    for (int j = 0; j < 8; ++j) {
+      const int c = 8 * q + j;
+      v[j] = c < a.Cin ? src[static_cast<int64_t>(pix0 + px) * a.Cin + c] : 0.f;
     }
+    *reinterpret_cast<uint4*>(dst + static_cast<int64_t>(px) * kCC + 8 * q) =
+        make_uint4(pack_bf16x2(v[0], v[1]), pack_bf16x2(v[2], v[3]), pack_bf16x2(v[4], v[5]), pack_bf16x2(v[6], v[7]));
   }
+  if (a.labels && tile % kTilesPerImg == 0 && threadIdx.x == 0)
+    a.labels[static_cast<int64_t>(lane) * a.B + b] = a.y[lane][row];
 }
 
 // ------------------------------------------------------------------ pooling
-// grid (B, active), 256 threads: g[lane][b][c] = sum over the 1024 pixels / 1024
+// grid (B, active), 256 threads: g[lane][b][c] = sum over the 1024 pixels / 1024.
+// Thread t sums channels 8 (t % 8) .. + 8 over pixels t / 8 + 32 i (16-byte
+// loads, a warp reading 512 contiguous bytes), then the 32 partials of each
+// channel group are summed in order.
 __global__ void __launch_bounds__(256) cnn_pool_kernel(const __nv_bfloat16* v, const int* wid, int B, float* g) {
-  __shared__ float part[4][kCC];
+  __shared__ float part[32][kCC + 1];
   const int b = blockIdx.x, lane = wid[blockIdx.y];
-  const int c = threadIdx.x % kCC, grp = threadIdx.x / kCC;
-  const __nv_bfloat16* src = v + (static_cast<int64_t>(lane) * B + b) * kPix * kCC;
-  float s = 0.f;
-  for (int p = grp; p < kPix; p += 4) s += __bfloat162float(src[static_cast<int64_t>(p) * kCC + c]);
-  part[grp][c] = s;
+  const int q = threadIdx.x & 7, p0 = threadIdx.x >> 3;
+  const __nv_bfloat16* src = v + (static_cast<int64_t>(lane) * B + b) * kPix * kCC + 8 * q;
+  float s[8];
+#pragma unroll
+  for (int j = 0; j < 8; ++j) s[j] = 0.f;
+#pragma unroll 4
+  for (int p = p0; p < kPix; p += 32) {
+    const uint4 r = *reinterpret_cast<const uint4*>(src + static_cast<int64_t>(p) * kCC);
+    const __nv_bfloat162* r2 = reinterpret_cast<const __nv_bfloat162*>(&r);
+#pragma unroll
+    for (int j = 0; j < 4; ++j) {
+      const float2 f = __bfloat1622float2(r2[j]);
+      s[2 * j] += f.x;
+      s[2 * j + 1] += f.y;
+    }
+  }
+#pragma unroll
+  for (int j = 0; j < 8; ++j) part[p0][8 * q + j] = s[j];
   __syncthreads();
-  if (threadIdx.x < kCC)
-    g[(static_cast<int64_t>(lane) * B + b) * kCC + threadIdx.x] =
-        (((part[0][threadIdx.x] + part[1][threadIdx.x]) + part[2][threadIdx.x]) + part[3][threadIdx.x]) /
-        static_cast<float>(kPix);
+  if (threadIdx.x < kCC) {
+    float t = 0.f;
+    for (int r = 0; r < 32; ++r) t += part[r][threadIdx.x];
+    g[(static_cast<int64_t>(lane) * B + b) * kCC + threadIdx.x] = t / static_cast<float>(kPix);
+  }
 }
 
 // ------------------------------------------------------------------ head: FC, softmax CE, backward, SGD of the FC
@@ -602,39 +622,50 @@ __global__ void __launch_bounds__(256) cnn_head_loss_kernel(const float* g, cons
 }
 
 // ------------------------------------------------------------------ output gradient of the last block
-// grid (B * 8 tiles, active), 128 threads (pixel): dz = v > 0 ? dg / 1024 : 0,
-// bf16, and per-tile channel sums of the fp32 values
+// grid (B * 8 tiles, active), 128 threads: dz = v > 0 ? dg / 1024 : 0, bf16,
+// and per-tile channel sums of the fp32 values.  Item = (pixel, 16-byte
+// chunk of 8 channels): thread t always has chunk t % 8 (pixels t / 8 + 16 i),
+// so its 8 channel sums stay in registers; the 16 threads of a chunk add
+// theirs in order through shared memory.  dg / 1024 is exact as dg * 2^-10.
 __global__ void __launch_bounds__(kCT) cnn_dzb_kernel(const __nv_bfloat16* v, const float* dg, const int* wid, int B,
                                                       __nv_bfloat16* dz, float* bias_part) {
-  __shared__ float T[kTilePix][kCC + 1];
+  __shared__ float dgs[kCC];
+  __shared__ float T[kCT / 8][kCC + 1];
   const int tile = blockIdx.x, lane = wid[blockIdx.y];
-  const int b = tile / kTilesPerImg, pix = (tile % kTilesPerImg) * kTilePix + threadIdx.x;
-  const int64_t base = ((static_cast<int64_t>(lane) * B + b) * kPix + pix) * kCC;
-  const float* d = dg + (static_cast<int64_t>(lane) * B + b) * kCC;
-  float o[kCC];
+  const int b = tile / kTilesPerImg, pix0 = (tile % kTilesPerImg) * kTilePix;
+  const int64_t base = ((static_cast<int64_t>(lane) * B + b) * kPix + pix0) * kCC;
+  if (threadIdx.x < kCC) dgs[threadIdx.x] = dg[(static_cast<int64_t>(lane) * B + b) * kCC + threadIdx.x] / static_cast<float>(kPix);
+  __syncthreads();
+  const int q = threadIdx.x & 7, p0 = threadIdx.x >> 3;
+  float d[8], sum[8];
 #pragma unroll
-  for (int q = 0; q < kCC / 8; ++q) {
-    const uint4 r = *reinterpret_cast<const uint4*>(v + base + 8 * q);
+  for (int j = 0; j < 8; ++j) {
+    d[j] = dgs[8 * q + j];
+    sum[j] = 0.f;
+  }
+#pragma unroll 4
+  for (int p = p0; p < kTilePix; p += kCT / 8) {
+    const int64_t off = base + static_cast<int64_t>(p) * kCC + 8 * q;
+    const uint4 r = *reinterpret_cast<const uint4*>(v + off);
     const __nv_bfloat162* r2 = reinterpret_cast<const __nv_bfloat162*>(&r);
+    float o[8];
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
       const float2 f = __bfloat1622float2(r2[j]);
-      const int c = 8 * q + 2 * j;
-      o[c] = f.x > 0.f ? d[c] / static_cast<float>(kPix) : 0.f;
-      o[c + 1] = f.y > 0.f ? d[c + 1] / static_cast<float>(kPix) : 0.f;
+      o[2 * j] = f.x > 0.f ? d[2 * j] : 0.f;
+      o[2 * j + 1] = f.y > 0.f ? d[2 * j + 1] : 0.f;
     }
+#pragma unroll
+    for (int j = 0; j < 8; ++j) sum[j] += o[j];
+    *reinterpret_cast<uint4*>(dz + off) = make_uint4(pack_bf16x2(o[0], o[1]), pack_bf16x2(o[2], o[3]),
+                                                     pack_bf16x2(o[4], o[5]), pack_bf16x2(o[6], o[7]));
   }
 #pragma unroll
-  for (int q = 0; q < kCC / 8; ++q)
-    *reinterpret_cast<uint4*>(dz + base + 8 * q) =
-        make_uint4(pack_bf16x2(o[8 * q], o[8 * q + 1]), pack_bf16x2(o[8 * q + 2], o[8 * q + 3]),
-                   pack_bf16x2(o[8 * q + 4], o[8 * q + 5]), pack_bf16x2(o[8 * q + 6], o[8 * q + 7]));
-#pragma unroll
-  for (int c = 0; c < kCC; ++c) T[threadIdx.x][c] = o[c];
+  for (int j = 0; j < 8; ++j) T[p0][8 * q + j] = sum[j];
   __syncthreads();
   if (threadIdx.x < kCC) {
     float s = 0.f;
-    for (int q = 0; q < kTilePix; ++q) s += T[q][threadIdx.x];
+    for (int r = 0; r < kCT / 8; ++r) s += T[r][threadIdx.x];
     bias_part[(static_cast<int64_t>(lane) * B * kTilesPerImg + tile) * kCC + threadIdx.x] = s;
   }
 }
