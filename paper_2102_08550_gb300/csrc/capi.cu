@@ -197,6 +197,7 @@ struct oscars_ctx {
   std::vector<int64_t> cnn_offW, cnn_offB;   // conv layers: stem, then (a, b) of every block
   int64_t cnn_offWf = 0, cnn_offBf = 0;
   int64_t cnn_wt_slot = 0;                   // elements per slot of the transposed copies
+  bool cnn_im2col = false;                   // stem over the im2col input (9 Cin <= 64): weights [64 out][64 k]
   __nv_bfloat16* cnn_wt = nullptr;           // [slot][2 * blocks][9][64 in][64 out]
   std::vector<__nv_bfloat16*> cnn_buf;       // x, s, (u_k, v_k) per block, dz0, dz1, dz2: [W][B][1024][64]
   std::vector<CUtensorMap> cnn_m6, cnn_m4, cnn_m2;   // per buffer: boxes of 6, 4 and 2 image rows
@@ -888,6 +889,7 @@ cudaError_t enqueue_step_cnn(oscars_ctx* c, int s, int na, const int* wid, const
     a.step = s;
     a.B = B;
     a.Cin = c->dims[2];
+    a.im2col = c->cnn_im2col ? 1 : 0;
     a.out = c->cnn_buf[X];
     a.labels = c->labels;
     ProfScope ps(c, "cnn_stage", st);
@@ -907,8 +909,10 @@ cudaError_t enqueue_step_cnn(oscars_ctx* c, int s, int na, const int* wid, const
     a.out = c->cnn_buf[out];
     a.bias_part = bpart;
     a.err = c->err;
+    a.im2col = layer == 0 && c->cnn_im2col ? 1 : 0;
     ProfScope ps(c, mode == 0 ? "conv_fwd" : "conv_dgrad", st);
-    return launch_conv_igemm(mode, c->cnn_m6[in], mode == 0 ? c->cnn_mw[layer] : c->cnn_mwt[layer - 1], a, na,
+    return launch_conv_igemm(mode, a.im2col ? c->cnn_m4[in] : c->cnn_m6[in],
+                             mode == 0 ? c->cnn_mw[layer] : c->cnn_mwt[layer - 1], a, na,
                              conv_ctas_per_worker(B, na, c->sms), st);
   };
   auto wgrad = [&](int layer, int in, int dz) -> cudaError_t {
@@ -919,8 +923,9 @@ cudaError_t enqueue_step_cnn(oscars_ctx* c, int s, int na, const int* wid, const
     a.img_per_chunk = ipc;
     a.part = c->cnn_wpart + layer * wpl;
     a.err = c->err;
+    a.im2col = layer == 0 && c->cnn_im2col ? 1 : 0;
     ProfScope ps(c, "conv_wgrad", st);
-    return launch_conv_wgrad(c->cnn_m4[in], c->cnn_m2[dz], a, na, st);
+    return launch_conv_wgrad(a.im2col ? c->cnn_m2[in] : c->cnn_m4[in], c->cnn_m2[dz], a, na, st);
   };
   // forward
   if ((e = conv(0, 0, X, -1, -1, S, nullptr)) != cudaSuccess) return e;
@@ -993,6 +998,7 @@ cudaError_t enqueue_step_cnn(oscars_ctx* c, int s, int na, const int* wid, const
     a.wt[l] = l >= 1 ? c->cnn_wt + static_cast<int64_t>(l - 1) * 9 * 64 * 64 : nullptr;
     a.offW[l] = c->cnn_offW[l];
     a.offB[l] = c->cnn_offB[l];
+    a.im2col[l] = l == 0 && c->cnn_im2col ? 1 : 0;
   }
   a.master = c->slab;
   a.master_w = c->slab;
@@ -1071,6 +1077,7 @@ oscars_status layout_cnn(oscars_ctx* c, const oscars_config* cfg) {
   c->P = static_cast<int64_t>(C) * 9 * Cin + C + static_cast<int64_t>(c->cnn_blocks) * 2 * (C * 9 * C + C) +
          static_cast<int64_t>(K) * C + K;
   c->cnn_wt_slot = static_cast<int64_t>(2 * c->cnn_blocks) * 9 * 64 * 64;
+  c->cnn_im2col = 9 * Cin <= 64;   // layer 0 then uses the first 64 x 64 of its 64 x 9 x 64 block
   c->cnn_chunks = c->B;   // capacity: at most one image per chunk
   return OSCARS_OK;
 }
@@ -1205,9 +1212,11 @@ oscars_status allocate_cnn(oscars_ctx* c) {
   c->cnn_mw.resize(layers);
   c->cnn_mwt.resize(layers > 1 ? layers - 1 : 1);
   for (int l = 0; l < layers; ++l) {
-    // forward layout [out][tap][in] of every slot: dims {in, tap, out, slot}
-    const uint64_t d[4] = {64, 9, 64, slots};
-    const uint64_t stv[3] = {64 * 2, 9 * 64 * 2, static_cast<uint64_t>(c->P_pad) * 2};
+    // forward layout [out][tap][in] of every slot: dims {in, tap, out, slot};
+    // the im2col stem [out][k]: one tap
+    const uint64_t ntap = l == 0 && c->cnn_im2col ? 1 : 9;
+    const uint64_t d[4] = {64, ntap, 64, slots};
+    const uint64_t stv[3] = {64 * 2, ntap * 64 * 2, static_cast<uint64_t>(c->P_pad) * 2};
     ok &= make_map_box4(&c->cnn_mw[l], c->shadow + c->cnn_offW[l], d, stv, {64, 1, 64, 1});
     if (l >= 1) {
       // transposed [tap][in][out]: dims {out, in, tap, slot}
@@ -1307,11 +1316,14 @@ cudaError_t copy_canonical(oscars_ctx* c, float* padded, const float* canon, boo
     const int Cin = c->dims[2], K = c->dims[4];
     float* dst = const_cast<float*>(canon);
     int64_t co = 0;
-    // stem [64][9][Cin] <-> [64][9][64] (the padded channels stay zero)
-    cudaError_t e = to_padded ? cudaMemcpy2DAsync(padded + c->cnn_offW[0], 64 * sizeof(float), canon, Cin * sizeof(float),
-                                                  Cin * sizeof(float), 64 * 9, cudaMemcpyDefault, s)
-                              : cudaMemcpy2DAsync(dst, Cin * sizeof(float), padded + c->cnn_offW[0], 64 * sizeof(float),
-                                                  Cin * sizeof(float), 64 * 9, cudaMemcpyDefault, s);
+    // stem [64][9][Cin] <-> [64][9][64], or <-> [64][64] with im2col (k = tap * Cin + i);
+    // the padding stays zero
+    const size_t wrow = (c->cnn_im2col ? 9 * Cin : Cin) * sizeof(float);
+    const size_t nrow = c->cnn_im2col ? 64 : 64 * 9;
+    cudaError_t e = to_padded ? cudaMemcpy2DAsync(padded + c->cnn_offW[0], 64 * sizeof(float), canon, wrow, wrow, nrow,
+                                                  cudaMemcpyDefault, s)
+                              : cudaMemcpy2DAsync(dst, wrow, padded + c->cnn_offW[0], 64 * sizeof(float), wrow, nrow,
+                                                  cudaMemcpyDefault, s);
     co = static_cast<int64_t>(64) * 9 * Cin;
     auto seg = [&](int64_t off, int64_t n) -> cudaError_t {
       cudaError_t r = to_padded ? cudaMemcpyAsync(padded + off, canon + co, n * sizeof(float), cudaMemcpyDefault, s)
@@ -1782,6 +1794,7 @@ oscars_status oscars_eval_loss(oscars_ctx* c, const float* x, const int32_t* y, 
       a.step = 0;
       a.B = Bc;
       a.Cin = c->dims[2];
+      a.im2col = c->cnn_im2col ? 1 : 0;
       a.out = c->cnn_buf[0];
       a.labels = c->labels;
       e = launch_cnn_stage(a, 1, c->stream);
@@ -1797,8 +1810,9 @@ oscars_status oscars_eval_loss(oscars_ctx* c, const float* x, const int32_t* y, 
         ca.add = add >= 0 ? c->cnn_buf[add] : nullptr;
         ca.out = c->cnn_buf[out];
         ca.err = c->err;
-        return launch_conv_igemm(0, c->cnn_m6[in], c->cnn_mw[layer], ca, 1, conv_ctas_per_worker(Bc, 1, c->sms),
-                                 c->stream);
+        ca.im2col = layer == 0 && c->cnn_im2col ? 1 : 0;
+        return launch_conv_igemm(0, ca.im2col ? c->cnn_m4[in] : c->cnn_m6[in], c->cnn_mw[layer], ca, 1,
+                                 conv_ctas_per_worker(Bc, 1, c->sms), c->stream);
       };
       if (e == cudaSuccess) e = conv(0, 0, -1, 1);
       for (int k = 0; e == cudaSuccess && k < c->cnn_blocks; ++k) {

@@ -115,9 +115,13 @@ __global__ void __launch_bounds__(kGT, 1) conv_igemm_kernel(const __grid_constan
   tc_fence_after();
   const uint32_t tmem = *tslot;
   constexpr int sgn = MODE == 0 ? 1 : -1;   // the input gradient reads the output gradient at p - off(tap)
+  // im2col stem (forward): one tap of weights, one 4-row box per tile (mIn's
+  // box is {64, 32, 4, 1}), four MMAs
+  const bool one_tap = MODE == 0 && a.im2col;
+  const int nbox = one_tap ? 1 : 3;
   if (t == 0) {
-    mbar_arrive_expect_tx(wfull, kGW);
-    for (int tap = 0; tap < kTaps; ++tap) {
+    mbar_arrive_expect_tx(wfull, one_tap ? kCB : kGW);
+    for (int tap = 0; tap < (one_tap ? 1 : kTaps); ++tap) {
       if (MODE == 0) tma_load_4d(wts + tap * kCB, &mW, 0, tap, 0, slot, wfull);   // {in, tap, out, slot}
       else tma_load_4d(wts + tap * kCB, &mW, 0, 0, tap, slot, wfull);             // {out, in, tap, slot}
     }
@@ -125,14 +129,19 @@ __global__ void __launch_bounds__(kGT, 1) conv_igemm_kernel(const __grid_constan
     for (int k = 0; k < my_tiles; ++k) {
       const int tile = c0 + k * cpw;
       const int img = lane * a.B + tile / kTilesPerImg, y0 = (tile % kTilesPerImg) * kTileRows;
-      for (int dx = 0; dx < 3; ++dx, ++it) {
+      for (int dx = 0; dx < nbox; ++dx, ++it) {
         const int sl = it % kGSlots;
         if (it >= kGSlots && !mbar_wait(&empty[sl], ((it / kGSlots) + 1) & 1, a.err, kDevTimeoutEmpty)) {
           k = my_tiles;
           break;
         }
-        mbar_arrive_expect_tx(&full[sl], kGBox);
-        tma_load_4d(slots + sl * kGBox, &mIn, 0, sgn * (dx - 1), y0 - 1, img, &full[sl]);
+        if (one_tap) {
+          mbar_arrive_expect_tx(&full[sl], kTilePix * kCC * 2);
+          tma_load_4d(slots + sl * kGBox, &mIn, 0, 0, y0, img, &full[sl]);
+        } else {
+          mbar_arrive_expect_tx(&full[sl], kGBox);
+          tma_load_4d(slots + sl * kGBox, &mIn, 0, sgn * (dx - 1), y0 - 1, img, &full[sl]);
+        }
       }
     }
   } else if (t == 32) {
@@ -144,7 +153,7 @@ __global__ void __launch_bounds__(kGT, 1) conv_igemm_kernel(const __grid_constan
       const int buf = k & 1, use = k >> 1;
       if (use >= 1 && !mbar_wait(&acce[buf], (use - 1) & 1, a.err, kDevTimeoutAccum)) break;
       tc_fence_after();
-      for (int dx = 0; dx < 3; ++dx, ++it) {
+      for (int dx = 0; dx < nbox; ++dx, ++it) {
         const int sl = it % kGSlots;
         if (!mbar_wait(&full[sl], (it / kGSlots) & 1, a.err, kDevTimeoutFull)) {
           ok = false;
@@ -152,6 +161,14 @@ __global__ void __launch_bounds__(kGT, 1) conv_igemm_kernel(const __grid_constan
         }
         tc_fence_after();
         const uint32_t sa = smem_u32(slots + sl * kGBox);
+        if (one_tap) {
+#pragma unroll
+          for (int j = 0; j < kCC / 16; ++j)
+            umma_bf16(tmem + buf * kCC, smem_desc_k128(sa + j * 32), smem_desc_k128(smem_u32(wts) + j * 32), idesc,
+                      j != 0 ? 1u : 0u);
+          umma_commit(&empty[sl]);
+          continue;
+        }
 #pragma unroll
         for (int dy = 0; dy < 3; ++dy) {
           const int rowoff = MODE == 0 ? dy : 2 - dy;   // sub-tile of the 6-row box
@@ -327,14 +344,22 @@ __global__ void __launch_bounds__(kWT, 1) conv_wgrad_kernel(const __grid_constan
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tslot;
+  // im2col stem: one 2-row input box per K-block (mIn's box is {64, 32, 2, 1})
+  // and one accumulator, tap 0 in its lower half
+  const int npairs = a.im2col ? 1 : kWPairs;
   if (t == 0) {
     for (int kb = 0; kb < nk; ++kb) {
       const int st = kb % kWStages2;
       if (kb >= kWStages2 && !mbar_wait(&empty[st], ((kb / kWStages2) + 1) & 1, a.err, kDevTimeoutEmpty)) break;
       uint8_t* sa = sm + st * kWStage2;
       const int img = lane * a.B + i0 + kb / (kImg / 2), yr = (kb % (kImg / 2)) * 2;
-      mbar_arrive_expect_tx(&full[st], kWStage2);
-      for (int dx = 0; dx < 3; ++dx) tma_load_4d(sa + dx * kWBox, &mIn, 0, dx - 1, yr - 1, img, &full[st]);
+      if (a.im2col) {
+        mbar_arrive_expect_tx(&full[st], 2 * kWRow + kWTile);
+        tma_load_4d(sa, &mIn, 0, 0, yr, img, &full[st]);
+      } else {
+        mbar_arrive_expect_tx(&full[st], kWStage2);
+        for (int dx = 0; dx < 3; ++dx) tma_load_4d(sa + dx * kWBox, &mIn, 0, dx - 1, yr - 1, img, &full[st]);
+      }
       tma_load_4d(sa + 3 * kWBox, &mDz, 0, 0, yr, img, &full[st]);
     }
   } else if (t == 32) {
@@ -345,6 +370,15 @@ __global__ void __launch_bounds__(kWT, 1) conv_wgrad_kernel(const __grid_constan
       tc_fence_after();
       const uint32_t sa = smem_u32(sm + st * kWStage2);
       const uint32_t sb = sa + 3 * kWBox;
+      if (a.im2col) {
+        // A = the 2-row box (in-channels k); its upper atom (the next row) is not read back
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+          umma_bf16(tmem, smem_desc_mn128(sa + j * 2048, kWRow), smem_desc_mn128(sb + j * 2048, kWTile), idesc,
+                    (kb | j) != 0 ? 1u : 0u);
+        umma_commit(&empty[st]);
+        continue;
+      }
 #pragma unroll
       for (int pr = 0; pr < kWPairs; ++pr) {
         int start, lbo, tap0, tap1;
@@ -364,9 +398,10 @@ __global__ void __launch_bounds__(kWT, 1) conv_wgrad_kernel(const __grid_constan
   // TMEM lane r: row r of each pair's accumulator = (tap of atom r / 64, in-channel r % 64)
   const int r = t;
   const int ci = r & (kCC - 1);
-  for (int pr = 0; pr < kWPairs; ++pr) {
+  for (int pr = 0; pr < npairs; ++pr) {
     int start, lbo, tap0, tap1;
     wgrad_pair(pr, start, lbo, tap0, tap1);
+    if (a.im2col) tap1 = -1;
     const int tap = r < 64 ? tap0 : tap1;
     float lo[32], hi[32];
     tmem_ld_32x32b_x32_pair(tmem + (static_cast<uint32_t>(warp * 32) << 16) + pr * kCC, lo,
@@ -390,7 +425,8 @@ __global__ void __launch_bounds__(kWT, 1) conv_wgrad_kernel(const __grid_constan
 
 // ------------------------------------------------------------------ reduce + SGD of the convolution layers
 // grid (taps * 4, active workers, layers), 256 threads: one tap's 16 in-channel
-// rows x 64 out-channels of one layer; the chunks are summed in chunk order
+// rows x 64 out-channels of one layer; the chunks are summed in chunk order.
+// The im2col stem has one tap (its blocks of taps 1..8 return at once).
 constexpr int kSgdRows = 16;
 __global__ void __launch_bounds__(256) conv_sgd_kernel(const __grid_constant__ ConvSgdArgs a) {
   __shared__ float T[kSgdRows][kCC + 1];   // [in][out]
@@ -398,6 +434,8 @@ __global__ void __launch_bounds__(256) conv_sgd_kernel(const __grid_constant__ C
   const int e = blockIdx.y, layer = blockIdx.z;
   const int lane = a.wid[e], src = a.src[e];
   const int t = threadIdx.x;
+  const int ntap = a.im2col[layer] ? 1 : kTaps;   // the im2col stem: [out][k], one tap
+  if (tap >= ntap) return;
   const float* part = a.part[layer] + (static_cast<int64_t>(lane) * a.n_chunks * kTaps + tap) * kCC * kCC + r0 * kCC;
   const int64_t chunk_stride = static_cast<int64_t>(kTaps) * kCC * kCC;
   for (int q = t; q < kSgdRows * kCC; q += 256) {
@@ -412,7 +450,7 @@ __global__ void __launch_bounds__(256) conv_sgd_kernel(const __grid_constant__ C
   // master / forward copy: [out][tap][in], in fastest
   for (int q = t; q < kSgdRows * kCC; q += 256) {
     const int co = q / kSgdRows, ci = q % kSgdRows;
-    const int64_t off = offW + (static_cast<int64_t>(co) * kTaps + tap) * kCC + r0 + ci;
+    const int64_t off = offW + (static_cast<int64_t>(co) * ntap + tap) * kCC + r0 + ci;
     const float nw = fmaf(-a.lr, T[ci][co], a.master[so + off]);
     a.master_w[dof + off] = nw;
     a.shadow[dof + off] = __float2bfloat16_rn(nw);
@@ -449,7 +487,10 @@ __global__ void conv_refresh_wt_kernel(const float* master, __nv_bfloat16* wt, i
 // channels).  Channels >= Cin stay zero: the buffer is cleared once when the
 // context is built, so only the 16-byte chunks that hold input channels are
 // written (one chunk for Cin <= 8), item = (pixel, chunk) with consecutive
-// threads on consecutive chunks.
+// threads on consecutive chunks.  With im2col (9 Cin <= 64) channel
+// k = tap * Cin + i of pixel (y, x) is x[y + dy - 1][x + dx - 1][i] for
+// tap = 3 dy + dx (zero outside the image): the stem becomes one 64 x 64
+// product per pixel.
 __global__ void __launch_bounds__(kCT) cnn_stage_kernel(const __grid_constant__ CnnStageArgs a) {
   const int tile = blockIdx.x, e = blockIdx.y;
   const int lane = a.wid[e];
@@ -458,14 +499,26 @@ __global__ void __launch_bounds__(kCT) cnn_stage_kernel(const __grid_constant__ 
   const int64_t row = (a.start[lane] + static_cast<int64_t>(a.step) * a.B + b) % n;
   const float* src = a.x[lane] + row * static_cast<int64_t>(kPix) * a.Cin;
   __nv_bfloat16* dst = a.out + ((static_cast<int64_t>(lane) * a.B + b) * kPix + pix0) * kCC;
-  const int chunks = (a.Cin + 7) / 8;
+  const int K = a.im2col ? kTaps * a.Cin : a.Cin;
+  const int chunks = (K + 7) / 8;
   for (int it = threadIdx.x; it < kTilePix * chunks; it += kCT) {
     const int px = it / chunks, q = it - px * chunks;
+    const int y = (pix0 + px) / kImg, x = (pix0 + px) % kImg;
     float v[8];
 #pragma unroll
     for (int j = 0; j < 8; ++j) {
       const int c = 8 * q + j;
-      v[j] = c < a.Cin ? src[static_cast<int64_t>(pix0 + px) * a.Cin + c] : 0.f;
+      float f = 0.f;
+      if (c < K) {
+        if (a.im2col) {
+          const int tap = c / a.Cin, i = c - tap * a.Cin;
+          const int yy = y + tap / 3 - 1, xx = x + tap % 3 - 1;
+          if (yy >= 0 && yy < kImg && xx >= 0 && xx < kImg) f = src[static_cast<int64_t>(yy * kImg + xx) * a.Cin + i];
+        } else {
+          f = src[static_cast<int64_t>(pix0 + px) * a.Cin + c];
+        }
+      }
+      v[j] = f;
     }
     *reinterpret_cast<uint4*>(dst + static_cast<int64_t>(px) * kCC + 8 * q) =
         make_uint4(pack_bf16x2(v[0], v[1]), pack_bf16x2(v[2], v[3]), pack_bf16x2(v[4], v[5]), pack_bf16x2(v[6], v[7]));

@@ -243,12 +243,14 @@ struct ConvArgs {
   __nv_bfloat16* out;          // [lane][B][1024][64]
   float* bias_part;            // input gradient: [lane][cpw][64] per-CTA channel sums, or null
   int* err;
+  int im2col;                  // forward only: 1 = the stem as one 64 x 64 product over the im2col input
 };
 struct WgradArgs {
   const int* wid;
   int B, n_chunks, img_per_chunk;
   float* part;                 // [lane][n_chunks][9][64 in][64 out]
   int* err;
+  int im2col;                  // 1 = the stem over the im2col input: tap 0 of `part` only
 };
 constexpr int kMaxConvLayers = 9;
 struct ConvSgdArgs {
@@ -259,6 +261,7 @@ struct ConvSgdArgs {
   const float* part[kMaxConvLayers];       // per layer, as WgradArgs::part
   const float* bias_part[kMaxConvLayers];  // per layer: [lane][n_tiles][64]
   __nv_bfloat16* wt[kMaxConvLayers];       // per layer: transposed bf16 copy in slot 0, or null
+  int im2col[kMaxConvLayers];              // per layer: 1 = weights [64 out][64 k] (one tap)
   int64_t offW[kMaxConvLayers], offB[kMaxConvLayers];
   const float* master;
   float* master_w;
@@ -273,6 +276,7 @@ struct CnnStageArgs {
   const int64_t* start;        // [W] cursors
   const int* wid;
   int step, B, Cin;
+  int im2col;                  // 1: channel k = tap * Cin + i holds x[y + dy - 1][x + dx - 1][i], tap = 3 dy + dx
   __nv_bfloat16* out;          // [lane][B][1024][64]
   int32_t* labels;             // [lane][B] or null
 };

@@ -4,7 +4,8 @@ conditioning envelope of the oracle (bf16 rounding and ReLU masks amplify
 fp32 summation-order differences), worker losses and eval loss within 1e-3.
 
 Cases: small runs of one and two residual blocks through two rounds (the
-second round starts from the merged model), and the full-size workload
+second round starts from the merged model; 3 input channels take the im2col
+stem, 16 the nine-tap one), and the full-size workload
 (16 workers, batch 32) for one local step of two sampled workers."""
 import dataclasses
 
@@ -49,13 +50,16 @@ def pull(ctx, device):
     return out.cpu().numpy()
 
 
-SMALL = [("1block", 1, 3, 16), ("2blocks", 2, 2, 16)]
+# (name, blocks, workers, batch, input channels): 3 channels take the im2col
+# stem (9 x 3 <= 64 channels), 16 the nine-tap stem
+SMALL = [("1block", 1, 3, 16, 3), ("2blocks", 2, 2, 16, 3), ("1block-cin16", 1, 2, 16, 16)]
 
 
-@pytest.mark.parametrize("name,blocks,W,B", SMALL, ids=[s[0] for s in SMALL])
-def test_cnn_small_two_rounds(cuda_device, name, blocks, W, B):
+@pytest.mark.parametrize("name,blocks,W,B,cin", SMALL, ids=[s[0] for s in SMALL])
+def test_cnn_small_two_rounds(cuda_device, name, blocks, W, B, cin):
     rows = 4 * B
-    w = synth.ConvWorkload(f"cnn-{name}", W, [32 * 32 * 3, 10], B, 0.05, rows, 4, 2, clip=3.0, blocks=blocks)
+    w = synth.ConvWorkload(f"cnn-{name}", W, [32 * 32 * cin, 10], B, 0.05, rows, 4, 2, clip=3.0, blocks=blocks,
+                           in_ch=cin)
     ctx, m, params0 = make_cnn_context(w, cuda_device, rows)
     rounds = 2
     losses, flats = [], []
