@@ -491,7 +491,14 @@ __global__ void conv_refresh_wt_kernel(const float* master, __nv_bfloat16* wt, i
 // k = tap * Cin + i of pixel (y, x) is x[y + dy - 1][x + dx - 1][i] for
 // tap = 3 dy + dx (zero outside the image): the stem becomes one 64 x 64
 // product per pixel.
+// im2col: the tile's 6 source rows (y0 - 1 .. y0 + 4, zero outside the
+// image) are first copied to shared memory with coalesced loads; a table
+// gives each channel k its offset from the centre pixel and its x-offset.
+constexpr int kStageMaxCin = kCC / kTaps;   // 7: the largest input with an im2col stem
+constexpr int kNoTap = 1 << 20;
 __global__ void __launch_bounds__(kCT) cnn_stage_kernel(const __grid_constant__ CnnStageArgs a) {
+  __shared__ float rows[(kTileRows + 2) * kImg * kStageMaxCin];
+  __shared__ int koff[kCC], kdx[kCC];
   const int tile = blockIdx.x, e = blockIdx.y;
   const int lane = a.wid[e];
   const int b = tile / kTilesPerImg, pix0 = (tile % kTilesPerImg) * kTilePix;
@@ -501,30 +508,52 @@ __global__ void __launch_bounds__(kCT) cnn_stage_kernel(const __grid_constant__ 
   __nv_bfloat16* dst = a.out + ((static_cast<int64_t>(lane) * a.B + b) * kPix + pix0) * kCC;
   const int K = a.im2col ? kTaps * a.Cin : a.Cin;
   const int chunks = (K + 7) / 8;
+  if (a.labels && tile % kTilesPerImg == 0 && threadIdx.x == 0)
+    a.labels[static_cast<int64_t>(lane) * a.B + b] = a.y[lane][row];
+  if (a.im2col) {
+    const int Cin = a.Cin, rowel = kImg * Cin, y0 = pix0 / kImg;
+    if (threadIdx.x < kCC) {
+      const int k = threadIdx.x;
+      if (k < K) {
+        const int tap = k / Cin, i = k - tap * Cin, dy = tap / 3, dx = tap % 3;
+        koff[k] = (dy - 1) * rowel + (dx - 1) * Cin + i;
+        kdx[k] = dx - 1;
+      } else {
+        koff[k] = 0;
+        kdx[k] = kNoTap;
+      }
+    }
+    for (int i = threadIdx.x; i < (kTileRows + 2) * rowel; i += kCT) {
+      const int yy = y0 - 1 + i / rowel;
+      rows[i] = yy >= 0 && yy < kImg ? src[static_cast<int64_t>(y0 - 1) * rowel + i] : 0.f;
+    }
+    __syncthreads();
+    for (int it = threadIdx.x; it < kTilePix * chunks; it += kCT) {
+      const int px = it / chunks, q = it - px * chunks;
+      const int x = px % kImg;
+      const int centre = (px / kImg + 1) * rowel + x * Cin;
+      float v[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const int k = 8 * q + j, xx = x + kdx[k];
+        v[j] = xx >= 0 && xx < kImg ? rows[centre + koff[k]] : 0.f;
+      }
+      *reinterpret_cast<uint4*>(dst + static_cast<int64_t>(px) * kCC + 8 * q) =
+          make_uint4(pack_bf16x2(v[0], v[1]), pack_bf16x2(v[2], v[3]), pack_bf16x2(v[4], v[5]), pack_bf16x2(v[6], v[7]));
+    }
+    return;
+  }
   for (int it = threadIdx.x; it < kTilePix * chunks; it += kCT) {
     const int px = it / chunks, q = it - px * chunks;
-    const int y = (pix0 + px) / kImg, x = (pix0 + px) % kImg;
     float v[8];
 #pragma unroll
     for (int j = 0; j < 8; ++j) {
       const int c = 8 * q + j;
-      float f = 0.f;
-      if (c < K) {
-        if (a.im2col) {
-          const int tap = c / a.Cin, i = c - tap * a.Cin;
-          const int yy = y + tap / 3 - 1, xx = x + tap % 3 - 1;
-          if (yy >= 0 && yy < kImg && xx >= 0 && xx < kImg) f = src[static_cast<int64_t>(yy * kImg + xx) * a.Cin + i];
-        } else {
-          f = src[static_cast<int64_t>(pix0 + px) * a.Cin + c];
-        }
-      }
-      v[j] = f;
+      v[j] = c < K ? src[static_cast<int64_t>(pix0 + px) * a.Cin + c] : 0.f;
     }
     *reinterpret_cast<uint4*>(dst + static_cast<int64_t>(px) * kCC + 8 * q) =
         make_uint4(pack_bf16x2(v[0], v[1]), pack_bf16x2(v[2], v[3]), pack_bf16x2(v[4], v[5]), pack_bf16x2(v[6], v[7]));
   }
-  if (a.labels && tile % kTilesPerImg == 0 && threadIdx.x == 0)
-    a.labels[static_cast<int64_t>(lane) * a.B + b] = a.y[lane][row];
 }
 
 // ------------------------------------------------------------------ pooling
