@@ -40,7 +40,9 @@
 //  D  weight gradient of the group's 128 rows over the CTA's own input
 //     columns, dW0[o][k] = sum_b dz0[b][o] X[b][k], on tcgen05 in 32-column
 //     tiles (X^T tiles by TMA into a four-deep ring, the first ones during
-//     step F; three TMEM buffers); the epilogue reads the
+//     step F).  The tiles alternate between two chains, each with its own
+//     issuing thread, TMEM buffer and epilogue warpgroup, so that one chain's
+//     MMA issue overlaps the other's epilogue; the epilogue reads the
 //     gradient and the fp32 master from TMEM, applies W0 <- W0 - lr dW0,
 //     stores the master back to TMEM and its bf16 copy into the resident A
 //     operand.
@@ -62,12 +64,13 @@
 // late ones start as the short workers finish (longest first).
 //
 // Warp roles (384 threads): warp 0 lane 0 issues TMA, warp 1 lane 0 issues
-// tcgen05.mma, warp 2 owns the TMEM allocation (all 512 columns: one CTA per
-// SM), warps 4..11 are the two epilogue warpgroups (each covering the 128
-// TMEM lanes), all warps share the CUDA-core work of step H.
+// tcgen05.mma (in step D with warp 3 lane 0: one chain each), warp 2 owns the
+// TMEM allocation (all 512 columns: one CTA per SM), warps 4..11 are the two
+// epilogue warpgroups (each covering the 128 TMEM lanes), all warps share the
+// CUDA-core work of step H.
 //
 // TMEM columns: [0, kTAcc) fp32 master of the W0 block; [kTAcc, 512) the
-// forward accumulator (B columns) and, in step D, the three 32-column
+// forward accumulator (B columns) and, in step D, the two 32-column
 // weight-gradient buffers (the two uses never overlap in time).
 #include "common.cuh"
 #include "internal.h"
@@ -81,9 +84,9 @@ constexpr int kFC = 10;                // classes
 constexpr int kFMaxCluster = 8;
 constexpr int kFBK = 64;               // K-block (bf16 elements, 128 bytes)
 constexpr int kND = 32;                // columns per weight-gradient tile
-constexpr int kNBD = 3;                // weight-gradient TMEM buffers
+constexpr int kNBD = 2;                // weight-gradient TMEM buffers (one per issuing chain)
 constexpr int kNXD = 4;                // X^T tile buffers in shared memory
-constexpr int kTAcc = 512 - kNBD * kND;   // first TMEM column of the accumulators = master columns
+constexpr int kTAcc = 512 - 3 * kND;   // first TMEM column of the accumulators = master columns
 constexpr int kMaxKb = (kTAcc + kFBK - 1) / kFBK;   // resident K-blocks of W0
 constexpr int kW0Blk = kFU * kFBK * 2; // one resident K-block: 128 rows x 64 columns bf16
 
@@ -630,10 +633,14 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
       if (producer_ok) producer_ok = issue_d(s, pre_d, nD);
       // the first X tiles of the next step's forward, while this step's epilogue runs
       if (producer_ok && s + 1 < tau) producer_ok = issue_f(s + 1, 0, pre_f);
-    } else if (warp == 1 && lane == 0) {
+    } else if ((warp == 1 || warp == 3) && lane == 0) {
+      // two issuing chains: chain e (warp 1: e = 0, warp 3: e = 1) takes the
+      // tiles with running index c = e (mod 2), TMEM buffer e, X^T slots
+      // c % 4 (of its own parity) and epilogue warpgroup e
+      const int e = warp == 1 ? 0 : 1;
       constexpr uint32_t idesc = idesc_bf16_f32(128, kND);
-      for (int tt = 0; tt < nD; ++tt) {
-        const int c = s * nD + tt, buf = c % kNBD, use = c / kNBD, xb = c % kNXD;
+      for (int tt = ((s * nD + e) & 1); tt < nD; tt += 2) {
+        const int c = s * nD + tt, buf = e, use = c / kNBD, xb = c % kNXD;
         if (!mbar_wait(&fullD[xb], (c / kNXD) & 1, a.err, kDevTimeoutFull)) break;
         if (use >= 1 && !mbar_wait(&tfreeD[buf], (use - 1) & 1, a.err, kDevTimeoutAccum)) break;
         tc_fence_after();
@@ -647,13 +654,13 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
         umma_commit(&xfreeD[xb]);
       }
     } else if (warp >= 4) {
-      // the two warpgroups take alternate tiles (a fixed split: a master tile
-      // always belongs to the same warpgroup); a warp covers 32 rows
+      // warpgroup eg drains the tiles of chain eg (its TMEM buffer); a warp
+      // covers 32 rows
       const int quarter = warp & 3, eg = (warp - 4) >> 2;
       const int r = quarter * 32 + lane;
       const uint32_t trow = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
-      for (int tt = eg; tt < nD; tt += 2) {
-        const int c = s * nD + tt, buf = c % kNBD, use = c / kNBD;
+      for (int tt = ((s * nD + eg) & 1); tt < nD; tt += 2) {
+        const int c = s * nD + tt, buf = eg, use = c / kNBD;
         int ok = mbar_wait(&accD[buf], use & 1, a.err, kDevTimeoutAccum) ? 1 : 0;
         ok = __all_sync(0xffffffffu, ok);
         tc_fence_after();
