@@ -25,10 +25,12 @@
 //  F  forward: each CTA computes the partial pre-activation of the group's
 //     128 units over its own input columns on tcgen05 (resident W0; the
 //     first X tiles are prefetched during the previous step).  With S = 2
-//     each CTA keeps 128/S of the units: the epilogue stores each partial
-//     into the shared memory of the CTA that keeps its unit (its own or,
-//     through distributed shared memory, its partner's), and after one
-//     barrier z = (part_0 + part_1) + b0, h = relu(z), bf16;
+//     each CTA keeps 128/S of the units: the epilogue stores its own units'
+//     partials locally and the partner's into an outgoing buffer, which one
+//     bulk copy (async proxy, distributed shared memory) moves into the
+//     partner's incoming buffer, completing on the partner's mbarrier (a
+//     pairwise wait instead of a cluster barrier); then
+//     z = (part_0 + part_1) + b0, h = relu(z), bf16;
 //  H  last layer for the CTA's units: partial logits, summed over the whole
 //     cluster in rank order through distributed shared memory, softmax
 //     cross-entropy; the masked input gradient dz0[b][u] of its units is
@@ -98,11 +100,6 @@ __device__ __forceinline__ void st_dsmem_u32x4(void* local, uint32_t rank, uint4
                : "memory");
 }
 
-__device__ __forceinline__ void st_dsmem_f32x4(float* local, uint32_t rank, float4 v) {
-  st_dsmem_u32x4(local, rank, make_uint4(__float_as_uint(v.x), __float_as_uint(v.y), __float_as_uint(v.z),
-                                         __float_as_uint(v.w)));
-}
-
 __device__ __forceinline__ unsigned long long global_ns() {
   unsigned long long v;
   asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(v));
@@ -168,6 +165,7 @@ struct FCfg {
   static constexpr int kBarBytes = 256;
   static constexpr int kSmem = oBar + kBarBytes + 1024;      // + alignment slack
   static_assert(S == 1 || kUPC * kZs <= B * kHsd, "the incoming partials must fit the h tile they alias");
+  static_assert(S == 1 || 2 * kZBytes <= kFRing, "own and outgoing partials must fit the F ring");
 };
 
 struct FusedArgs {
@@ -200,6 +198,7 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
   uint8_t* dring = sm + Cfg::oRegion;                // X^T tiles of step D
   uint8_t* fring = dring + Cfg::kDRing;              // X tiles of step F
   float* zx = reinterpret_cast<float*>(fring);       // [kUPC][kZs] own partials (S = 2), after the F MMAs
+  float* zout = zx + Cfg::kUPC * Cfg::kZs;           // [kUPC][kZs] the partner's partials, sent by bulk copy
   uint8_t* w0s = sm + Cfg::oW0;                      // resident bf16 W0 block
   uint8_t* dzT = sm + Cfg::oDzT;
   float* hs = reinterpret_cast<float*>(sm + Cfg::oHs);
@@ -227,7 +226,8 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
   uint64_t* xfreeD = fullD + kNXD;             // [kNXD] X^T tile consumed by its MMA
   uint64_t* accD = xfreeD + kNXD;              // [kNBD] TMEM buffer full
   uint64_t* tfreeD = accD + kNBD;              // [kNBD] TMEM buffer drained (128 arrivals)
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(tfreeD + kNBD);
+  uint64_t* pinF = tfreeD + kNBD;              // [1] the partner's partials landed (S = 2)
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(pinF + 1);
 
   const int w = a.order[blockIdx.x];
   const int rank = static_cast<int>(cluster_ctarank());
@@ -267,6 +267,7 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
       mbar_init(&accD[i], 1);
       mbar_init(&tfreeD[i], 128);
     }
+    mbar_init(pinF, 1);
     fence_barrier_init();
     fence_proxy_async_smem();
   }
@@ -359,11 +360,13 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  if (S > 1) cluster_sync();  // every CTA's barriers are initialised before a peer signals them
   if (warp == 0 && lane == 0) producer_ok = issue_f(0, 0, pre_f);
 
   for (int s = 0; s < tau; ++s) {
     if (stamp) a.phase_ts[s * 4 + 0] = global_ns();
     const bool last = s == tau - 1;
+    if (S > 1 && t == 0) mbar_arrive_expect_tx(pinF, Cfg::kZBytes);   // this step's incoming partials
 
     // ------------------------------------------------------------ F: partial forward of the group's units
     if (warp == 0 && lane == 0) {
@@ -403,15 +406,13 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
             for (int j = 0; j < 32; ++j) hs[(c0 + j) * Cfg::kHsd + u] = bf16_round(fmaxf(v[j] + bias, 0.f));
           } else {
             // the partial goes to the CTA that keeps unit u: this one
-            // (own rows) or the partner (its incoming rows)
+            // (own rows) or, through the outgoing buffer, the partner
             const int owner = u / UPC;
-            float* row = (owner == half ? zx : zin) + (u - owner * UPC) * Cfg::kZs + c0;
+            float* row = (owner == half ? zx : zout) + (u - owner * UPC) * Cfg::kZs + c0;
 #pragma unroll
-            for (int q = 0; q < 8; ++q) {
-              const float4 p4 = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
-              if (owner == half) *reinterpret_cast<float4*>(row + 4 * q) = p4;
-              else st_dsmem_f32x4(row + 4 * q, grp * S + owner, p4);
-            }
+            for (int q = 0; q < 8; ++q)
+              *reinterpret_cast<float4*>(row + 4 * q) = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+            fence_proxy_async_smem();   // the outgoing rows are read by the bulk copy
           }
         }
       }
@@ -419,9 +420,12 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
     tc_fence_before();
     __syncthreads();
     if (S > 1) {
+      // the partner's partials of this CTA's units: one bulk copy each way
+      // into the incoming buffer, completing on the receiver's barrier
+      if (t == 0) bulk_copy_to_peer(zin, zout, Cfg::kZBytes, pinF, grp * S + (half ^ 1));
       // both partials of this CTA's units are local now:
       // z = part(half 0) + part(half 1) + b0
-      cluster_sync();
+      mbar_wait(pinF, s & 1, a.err, kDevTimeoutFull);
       constexpr int kZItems = UPC * (B / 4), kZPer = (kZItems + kFT - 1) / kFT;
       float4 zr[kZPer];
 #pragma unroll
