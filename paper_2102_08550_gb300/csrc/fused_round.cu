@@ -431,8 +431,8 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
 #pragma unroll
       for (int k = 0; k < kZPer; ++k) {
         const int q = t + k * kFT;
-        if (q < kZItems) {
-          const int ul = q / (B / 4), b4 = (q % (B / 4)) * 4;
+        if (q < kZItems) {   // item = (unit, 4 samples), consecutive threads on consecutive units
+          const int ul = q % UPC, b4 = (q / UPC) * 4;
           const float4 own = *reinterpret_cast<const float4*>(zx + ul * Cfg::kZs + b4);
           const float4 inc = *reinterpret_cast<const float4*>(zin + ul * Cfg::kZs + b4);
           const float4 p0 = half == 0 ? own : inc, p1 = half == 0 ? inc : own;
@@ -453,7 +453,7 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
       for (int k = 0; k < kZPer; ++k) {
         const int q = t + k * kFT;
         if (q >= kZItems) break;
-        const int ul = q / (B / 4), b4 = (q % (B / 4)) * 4;
+        const int ul = q % UPC, b4 = (q / UPC) * 4;
         const int ug = ku0 + ul;                   // unit within the group
         const float4 z = zr[k];
         const float bias = b0m[ug];
