@@ -505,29 +505,39 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
     // writes (with S = 2 the barrier after the dz0^T exchange does that)
     if (S == 1) cluster_sync();
     else __syncthreads();
-    for (int b = t; b < B; b += kFT) {
-      float z[kFC], e[kFC];
+    // softmax cross-entropy, four threads per row: thread q of the row takes
+    // classes q, q + 4, q + 8 (exponentials and gradients); the row's
+    // exponentials are gathered in every lane of the row and summed in class
+    // order (the arithmetic of one thread per row)
+    static_assert(4 * B <= kFT, "four threads per batch row");
+    if (t < 4 * B) {
+      const int b = t >> 2, q = t & 3, src = lane & ~3;
+      float zq[3], eq[3];
 #pragma unroll
-      for (int c = 0; c < kFC; ++c) z[c] = dz[b * kFC + c];
-      float m = z[0];
+      for (int i = 0; i < 3; ++i) zq[i] = q + 4 * i < kFC ? dz[b * kFC + q + 4 * i] : -INFINITY;
+      float m = fmaxf(fmaxf(zq[0], zq[1]), zq[2]);
+      m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 1));
+      m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 2));
 #pragma unroll
-      for (int c = 1; c < kFC; ++c) m = fmaxf(m, z[c]);
+      for (int i = 0; i < 3; ++i) eq[i] = q + 4 * i < kFC ? expf(zq[i] - m) : 0.f;
       const int y = labs[b];
-      float se = 0.f, so_ = 0.f, zy = 0.f;
+      float se = 0.f, so_ = 0.f;
 #pragma unroll
       for (int c = 0; c < kFC; ++c) {
-        e[c] = expf(z[c] - m);
-        se += e[c];
-        if (c != y) so_ += e[c];
-        else zy = z[c];
+        const float ec = __shfl_sync(0xffffffffu, eq[c >> 2], src | (c & 3));
+        se += ec;
+        if (c != y) so_ += ec;
       }
-      rowloss[b] = m + logf(se) - zy;
+      if (q == (y & 3)) rowloss[b] = m + logf(se) - (y < 4 ? zq[0] : y < 8 ? zq[1] : zq[2]);
       const float inv = 1.0f / static_cast<float>(B);
 #pragma unroll
-      for (int c = 0; c < kFC; ++c) {
-        const float g = (c == y ? -(so_ / se) : e[c] / se) * inv;
-        dz[b * kFC + c] = g;
-        dzb[b * kFC + c] = bf16_round(g);
+      for (int i = 0; i < 3; ++i) {
+        const int c = q + 4 * i;
+        if (c < kFC) {
+          const float g = (c == y ? -(so_ / se) : eq[i] / se) * inv;
+          dz[b * kFC + c] = g;
+          dzb[b * kFC + c] = bf16_round(g);
+        }
       }
     }
     __syncthreads();
