@@ -124,6 +124,12 @@ __device__ __forceinline__ void bar_named(int id, int count) {
   asm volatile("barrier.sync %0, %1;" ::"r"(id), "r"(count) : "memory");
 }
 
+// Arrive on named barrier `id` without waiting (the producer side of a
+// producer/consumer pair whose consumer calls bar_named with the same count).
+__device__ __forceinline__ void bar_arrive_named(int id, int count) {
+  asm volatile("barrier.arrive %0, %1;" ::"r"(id), "r"(count) : "memory");
+}
+
 // Programmatic dependent launch.  A kernel launched as a programmatic
 // dependent may start while the previous kernel on its stream finishes;
 // pdl_wait() blocks until that kernel has completed and its memory is

@@ -225,8 +225,7 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
   uint64_t* fullD = accF + 1;                  // [kNXD] X^T tile landed
   uint64_t* xfreeD = fullD + kNXD;             // [kNXD] X^T tile consumed by its MMA
   uint64_t* accD = xfreeD + kNXD;              // [kNBD] TMEM buffer full
-  uint64_t* tfreeD = accD + kNBD;              // [kNBD] TMEM buffer drained (128 arrivals)
-  uint64_t* pinF = tfreeD + kNBD;              // [1] the partner's partials landed (S = 2)
+  uint64_t* pinF = accD + kNBD;                // [1] the partner's partials landed (S = 2)
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(pinF + 1);
 
   const int w = a.order[blockIdx.x];
@@ -263,10 +262,7 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
       mbar_init(&fullD[i], 1);
       mbar_init(&xfreeD[i], 1);
     }
-    for (int i = 0; i < kNBD; ++i) {
-      mbar_init(&accD[i], 1);
-      mbar_init(&tfreeD[i], 128);
-    }
+    for (int i = 0; i < kNBD; ++i) mbar_init(&accD[i], 1);
     mbar_init(pinF, 1);
     fence_barrier_init();
     fence_proxy_async_smem();
@@ -309,6 +305,8 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
     return true;
   };
   bool producer_ok = true;
+  bool chain_ok = true;    // warps 1 and 3: no wait of this chain has run out
+  int chain_tiles = 0;     // warps 1 and 3: tiles issued by this chain so far
   double loss_sum = 0.0;   // rank 0, thread 0: sum of the 16-row loss chunks, in step and chunk order
 
   // the global model, once: fp32 master block into TMEM and its bf16 copy
@@ -647,25 +645,35 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
       if (producer_ok) producer_ok = issue_d(s, pre_d, nD);
       // the first X tiles of the next step's forward, while this step's epilogue runs
       if (producer_ok && s + 1 < tau) producer_ok = issue_f(s + 1, 0, pre_f);
-    } else if ((warp == 1 || warp == 3) && lane == 0) {
+    } else if (warp == 1 || warp == 3) {
       // two issuing chains: chain e (warp 1: e = 0, warp 3: e = 1) takes the
       // tiles with running index c = e (mod 2), TMEM buffer e, X^T slots
-      // c % 4 (of its own parity) and epilogue warpgroup e
+      // c % 4 (of its own parity) and epilogue warpgroup e.  The warpgroup
+      // hands the drained buffer back through named barrier 1 + e (128
+      // arrivals + this warp: cheaper than an mbarrier wait); every tile is
+      // committed, even after a failed wait, so that the arrivals and the
+      // waits on the named barrier stay paired
       const int e = warp == 1 ? 0 : 1;
       constexpr uint32_t idesc = idesc_bf16_f32(128, kND);
       for (int tt = ((s * nD + e) & 1); tt < nD; tt += 2) {
         const int c = s * nD + tt, buf = e, use = c / kNBD, xb = c % kNXD;
-        if (!mbar_wait(&fullD[xb], (c / kNXD) & 1, a.err, kDevTimeoutFull)) break;
-        if (use >= 1 && !mbar_wait(&tfreeD[buf], (use - 1) & 1, a.err, kDevTimeoutAccum)) break;
+        if (chain_ok) chain_ok = mbar_wait(&fullD[xb], (c / kNXD) & 1, a.err, kDevTimeoutFull);
+        if (use >= 1) bar_named(1 + e, 128 + 32);   // the previous use of the buffer has been read
         tc_fence_after();
-        const uint32_t xa = smem_u32(dring + xb * Cfg::kXtBytes);
-        const uint32_t da = smem_u32(dzT);
-        const uint32_t dcol = tmem + static_cast<uint32_t>(kTAcc + buf * kND);
+        if (lane == 0) {
+          if (chain_ok) {
+            const uint32_t xa = smem_u32(dring + xb * Cfg::kXtBytes);
+            const uint32_t da = smem_u32(dzT);
+            const uint32_t dcol = tmem + static_cast<uint32_t>(kTAcc + buf * kND);
 #pragma unroll
-        for (int j = 0; j < kFBK / 16; ++j)
-          umma_bf16(dcol, smem_desc_k128(da + j * 32), smem_desc_k128(xa + j * 32), idesc, j != 0 ? 1u : 0u);
-        umma_commit(&accD[buf]);
-        umma_commit(&xfreeD[xb]);
+            for (int j = 0; j < kFBK / 16; ++j)
+              umma_bf16(dcol, smem_desc_k128(da + j * 32), smem_desc_k128(xa + j * 32), idesc, j != 0 ? 1u : 0u);
+          }
+          umma_commit(&accD[buf]);
+          umma_commit(&xfreeD[xb]);
+        }
+        __syncwarp();
+        ++chain_tiles;
       }
     } else if (warp >= 4) {
       // warpgroup eg drains the tiles of chain eg (its TMEM buffer); a warp
@@ -683,14 +691,14 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
           float g[32], m[32];
           tmem_ld_32x32b_x32_pair(trow + kTAcc + buf * kND, g, trow + c0, m);
           tc_fence_before();
-          mbar_arrive(&tfreeD[buf]);   // the gradient buffer has been read: the next MMA may reuse it
+          bar_arrive_named(1 + eg, 128 + 32);   // the gradient buffer has been read: the next MMA may reuse it
 #pragma unroll
           for (int j = 0; j < 32; ++j) m[j] = fmaf(-a.lr, g[j], m[j]);
           tmem_st_32x32b_x32(trow + c0, m);
           put_w0_row32(w0s, r, c0, m);
         } else {
           tc_fence_before();
-          mbar_arrive(&tfreeD[buf]);
+          bar_arrive_named(1 + eg, 128 + 32);
         }
       }
       tmem_wait_st();   // the master columns stored above are read again next step
@@ -701,6 +709,8 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
     tc_fence_after();
     if (stamp) a.phase_ts[s * 4 + 3] = global_ns();
   }
+  // the last drain of each chain's buffer pairs with one more wait
+  if ((warp == 1 || warp == 3) && chain_tiles > 0) bar_named(1 + (warp == 1 ? 0 : 1), 128 + 32);
   // the worker's W0 block into its replica slot: each warp moves 32 rows x
   // 32 columns at a time from TMEM through a padded shared tile (the TMA
   // rings are idle now), 4 full 128-byte rows per store instruction
