@@ -155,7 +155,7 @@ struct FCfg {
   static constexpr int oW1m = oWc + kFC * kUPC * 4;          // [C][kUPC] fp32 master head columns
   static constexpr int oPl = oW1m + kFC * kUPC * 4;          // [B][C]
   static constexpr int oDz = oPl + B * kFC * 4;              // [B][C]
-  static constexpr int oDzb = oDz + B * kFC * 4;             // [B][C]
+  static constexpr int oDzb = oDz + B * kFC * 4;             // [C][B] (class-major)
   static constexpr int oGbp = oDzb + B * kFC * 4;            // [kChunks][kUPC]
   static constexpr int oRowLoss = oGbp + kChunks * kUPC * 4;   // [B]
   static constexpr int oB0 = oRowLoss + B * 4;               // [kFU] b0 of the group's units
@@ -534,7 +534,7 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
         if (c < kFC) {
           const float g = (c == y ? -(so_ / se) : eq[i] / se) * inv;
           dz[b * kFC + c] = g;
-          dzb[b * kFC + c] = bf16_round(g);
+          dzb[c * B + b] = bf16_round(g);
         }
       }
     }
@@ -564,18 +564,29 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
     // row, stored here and into the other CTAs of the group
     for (int it = t; it < UPC * Cfg::kChunks; it += kFT) {
       const int u = it % UPC, j = it / UPC;
-      float wc[kFC];
-#pragma unroll
-      for (int c = 0; c < kFC; ++c) wc[c] = wcs[c * UPC + u];
+      // dh[b] = sum over c in class order of dzb[c][b] w[c][u]: the eight
+      // samples of a class are two 16-byte loads of the class-major dzb
       float dv[8];
+#pragma unroll
+      for (int i = 0; i < 8; ++i) dv[i] = 0.f;
+#pragma unroll
+      for (int c = 0; c < kFC; ++c) {
+        const float wc = wcs[c * UPC + u];
+        const float4 d0 = *reinterpret_cast<const float4*>(dzb + c * B + 8 * j);
+        const float4 d1 = *reinterpret_cast<const float4*>(dzb + c * B + 8 * j + 4);
+        dv[0] = fmaf(d0.x, wc, dv[0]);
+        dv[1] = fmaf(d0.y, wc, dv[1]);
+        dv[2] = fmaf(d0.z, wc, dv[2]);
+        dv[3] = fmaf(d0.w, wc, dv[3]);
+        dv[4] = fmaf(d1.x, wc, dv[4]);
+        dv[5] = fmaf(d1.y, wc, dv[5]);
+        dv[6] = fmaf(d1.z, wc, dv[6]);
+        dv[7] = fmaf(d1.w, wc, dv[7]);
+      }
       float gsum = 0.f;
 #pragma unroll
       for (int i = 0; i < 8; ++i) {
-        const int b = 8 * j + i;
-        float dh = 0.f;
-#pragma unroll
-        for (int c = 0; c < kFC; ++c) dh = fmaf(dzb[b * kFC + c], wc[c], dh);
-        dh = hs[b * Cfg::kHsd + u] > 0.f ? dh : 0.f;
+        const float dh = hs[(8 * j + i) * Cfg::kHsd + u] > 0.f ? dv[i] : 0.f;
         dv[i] = dh;
         gsum += dh;
       }
@@ -597,14 +608,18 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
       const int item = q % Cfg::kW1Items, hb = q / Cfg::kW1Items;
       const int c = item / (UPC / 4), u4 = (item % (UPC / 4)) * 4;
       float4 dw = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll 8
-      for (int b = hb * (B / 2); b < (hb + 1) * (B / 2); ++b) {
-        const float g = dzb[b * kFC + c];
-        const float4 hv = *reinterpret_cast<const float4*>(hs + b * Cfg::kHsd + u4);
-        dw.x = fmaf(g, hv.x, dw.x);
-        dw.y = fmaf(g, hv.y, dw.y);
-        dw.z = fmaf(g, hv.z, dw.z);
-        dw.w = fmaf(g, hv.w, dw.w);
+#pragma unroll 2
+      for (int b4 = hb * (B / 2); b4 < (hb + 1) * (B / 2); b4 += 4) {
+        const float4 g4 = *reinterpret_cast<const float4*>(dzb + c * B + b4);   // samples b4 .. b4 + 3
+        const float gk[4] = {g4.x, g4.y, g4.z, g4.w};
+#pragma unroll
+        for (int k = 0; k < 4; ++k) {
+          const float4 hv = *reinterpret_cast<const float4*>(hs + (b4 + k) * Cfg::kHsd + u4);
+          dw.x = fmaf(gk[k], hv.x, dw.x);
+          dw.y = fmaf(gk[k], hv.y, dw.y);
+          dw.z = fmaf(gk[k], hv.z, dw.z);
+          dw.w = fmaf(gk[k], hv.w, dw.w);
+        }
       }
       w1p[hb * Cfg::kW1Items + item] = dw;
     }
