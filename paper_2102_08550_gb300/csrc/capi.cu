@@ -144,7 +144,10 @@ struct oscars_ctx {
   float* loss_dev = nullptr;
   int64_t* cursor = nullptr;
   int32_t* tau_dev = nullptr;
-  int32_t* order_dev = nullptr;         // workers by decreasing tau (launch order of the round kernel)
+  int32_t* order_dev = nullptr;         // workers of the round kernel, cluster by cluster (longest first)
+  int32_t* cl_first_dev = nullptr;      // [n_clusters + 1] first entry of each cluster in order_dev
+  int n_clusters = 0;                   // clusters of the round kernel
+  int fused_max_clusters = 0;           // clusters of the round kernel that fit on the device at once
   int* act_wid = nullptr;  // [max_tau][W]
   int32_t* stage_slots = nullptr;   // [sum tau] active staging slots s * W + w, step-major
   int n_stage_slots = 0;
@@ -513,13 +516,38 @@ oscars_status build_tables(oscars_ctx* c) {
   cudaError_t e = cudaMemcpy(c->act_wid, wid.data(), wid.size() * sizeof(int), cudaMemcpyHostToDevice);
   if (e == cudaSuccess) e = cudaMemcpy(c->act_src, src.data(), src.size() * sizeof(int), cudaMemcpyHostToDevice);
   if (e == cudaSuccess) e = cudaMemcpy(c->tau_dev, c->tau.data(), c->W * sizeof(int32_t), cudaMemcpyHostToDevice);
-  if (e == cudaSuccess) {   // longest first: workers by decreasing tau, ties by index
+  if (e == cudaSuccess) {
+    // Round-kernel clusters: one per worker when they all fit on the device,
+    // else as many as fit, each running its workers one after the other.
+    // Workers by decreasing tau (ties by index) go to the cluster with the
+    // least work so far (longest processing time first; a worker costs its
+    // tau steps plus about half a step of model load).
     std::vector<int32_t> ord(c->W);
     for (int i = 0; i < c->W; ++i) ord[i] = i;
     std::stable_sort(ord.begin(), ord.end(), [&](int32_t x, int32_t y) { return c->tau[x] > c->tau[y]; });
+    const int ncl = c->fused_max_clusters > 0 && c->fused_max_clusters < c->W ? c->fused_max_clusters : c->W;
+    std::vector<std::vector<int32_t>> lists(ncl);
+    std::vector<double> load(ncl, 0.0);
+    for (int32_t wk : ord) {
+      int k = 0;
+      for (int j = 1; j < ncl; ++j)
+        if (load[j] < load[k]) k = j;
+      lists[k].push_back(wk);
+      load[k] += c->tau[wk] + 0.5;
+    }
+    std::vector<int32_t> flat, first(1, 0);
+    for (const auto& l : lists) {
+      flat.insert(flat.end(), l.begin(), l.end());
+      first.push_back(static_cast<int32_t>(flat.size()));
+    }
+    c->n_clusters = ncl;
     if (!c->order_dev && !dev_alloc(c, &c->order_dev, c->W))
       return fail(c, OSCARS_ENOMEM, "device allocation failed (worker order)");
-    e = cudaMemcpy(c->order_dev, ord.data(), c->W * sizeof(int32_t), cudaMemcpyHostToDevice);
+    if (!c->cl_first_dev && !dev_alloc(c, &c->cl_first_dev, c->W + 1))
+      return fail(c, OSCARS_ENOMEM, "device allocation failed (cluster table)");
+    e = cudaMemcpy(c->order_dev, flat.data(), c->W * sizeof(int32_t), cudaMemcpyHostToDevice);
+    if (e == cudaSuccess)
+      e = cudaMemcpy(c->cl_first_dev, first.data(), first.size() * sizeof(int32_t), cudaMemcpyHostToDevice);
   }
   if (e != cudaSuccess) return cuda_fail(c, e, "schedule upload");
   if (c->round_exec) {
@@ -710,6 +738,8 @@ FusedRoundArgs fused_args(oscars_ctx* c) {
   FusedRoundArgs f{};
   f.tau = c->tau_dev;
   f.order = c->order_dev;
+  f.cl_first = c->cl_first_dev;
+  f.n_clusters = c->n_clusters;
   f.W = c->W;
   f.D = c->dims[0];
   f.H = c->dims[1];
@@ -1423,6 +1453,7 @@ oscars_status oscars_create(const oscars_config* cfg, oscars_ctx** out) {
         // a 2-layer bf16 MLP runs each round as one fused launch (flag bit 3: per-layer kernels)
         c->fused = c->model == OSCARS_MODEL_MLP && c->bf16 && !(cfg->flags & 8) && !(cfg->flags & 4) &&
                    fused_round_supported(c->L, c->dims[0], c->L >= 2 ? c->dims[1] : 0, c->C, c->B);
+        if (c->fused) c->fused_max_clusters = fused_round_max_clusters(c->dims[0], c->dims[1], c->B);
         // flag bit 2: bf16 MLP rounds fork into up to 16 concurrent worker branches
         c->n_br = (c->model == OSCARS_MODEL_MLP && c->bf16 && c->L >= 2 && (cfg->flags & 4)) ? std::min(c->W, kMaxBranches) : 1;
         if (st == OSCARS_OK) st = c->model == OSCARS_MODEL_CNN ? allocate_cnn(c) : allocate_mlp(c);

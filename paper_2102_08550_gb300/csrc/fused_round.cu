@@ -170,8 +170,9 @@ struct FCfg {
 
 struct FusedArgs {
   const int32_t* tau;       // [W]
-  const int32_t* order;     // [W] worker of each cluster (decreasing tau)
-  int W, D, H;
+  const int32_t* order;     // [W] workers, cluster by cluster
+  const int32_t* cl_first;  // [clusters + 1] cluster k runs order[cl_first[k] .. cl_first[k + 1])
+  int W, n_clusters, D, H;
   int global_slot;
   float lr;
   const float* master;      // slab read before the first step (the global slot)
@@ -228,7 +229,6 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
   uint64_t* pinF = accD + kNBD;                // [1] the partner's partials landed (S = 2)
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(pinF + 1);
 
-  const int w = a.order[blockIdx.x];
   const int rank = static_cast<int>(cluster_ctarank());
   const int ncl = static_cast<int>(gridDim.y);
   const int grp = rank / S, half = rank % S;    // unit group, column half
@@ -236,7 +236,6 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
   const int ku0 = half * UPC;                   // first kept unit within the group
   const int t = threadIdx.x, warp = t >> 5, lane = t & 31;
   const int D = a.D, H = a.H;
-  const int tau = a.tau[w];
   const int nkF = (D + kFBK - 1) / kFBK;
   const int kb_split = S > 1 ? nkF / 2 : nkF;
   const int kb_begin = half == 0 ? 0 : kb_split, kb_end = half == 0 ? kb_split : nkF;
@@ -248,7 +247,6 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
   const int pre_f = nkf < Cfg::kStagesF ? nkf : Cfg::kStagesF;   // X tiles loaded ahead of a step
   const int pre_d = nD < kNXD ? nD : kNXD;                       // X^T tiles loaded before step D
   const int64_t gso = static_cast<int64_t>(a.global_slot) * a.slot_stride;
-  const int64_t dof = static_cast<int64_t>(w) * a.slot_stride;
 
   if (t == 0) {
     prefetch_tmap(&mX);
@@ -279,486 +277,506 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
-  const bool stamp = a.phase_ts && w == 0 && rank == 0 && t == 0;
-
-  // producer (warp 0 lane 0): X tiles [from, to) of step s's forward; the
-  // ring position of K-block kb of step s is s * nkf + kb
-  auto issue_f = [&](int s, int from, int to) -> bool {
-    for (int kb = from; kb < to; ++kb) {
-      const int c = s * nkf + kb, st = c % Cfg::kStagesF;
-      if (c >= Cfg::kStagesF && !mbar_wait(&emptyF[st], ((c / Cfg::kStagesF) + 1) & 1, a.err, kDevTimeoutEmpty))
-        return false;
-      mbar_arrive_expect_tx(&fullF[st], Cfg::kBBytes);
-      tma_load_4d(fring + st * Cfg::kBBytes, &mX, (kb_begin + kb) * kFBK, 0, w, s, &fullF[st]);
-    }
-    return true;
-  };
-  // X^T tiles [from, to) of step s's weight gradient (ring position s * nD + tile)
-  auto issue_d = [&](int s, int from, int to) -> bool {
-    for (int tt = from; tt < to; ++tt) {
-      const int c = s * nD + tt, xb = c % kNXD, use = c / kNXD;
-      // the buffer's previous tile must have been read by its MMA
-      if (use >= 1 && !mbar_wait(&xfreeD[xb], (use - 1) & 1, a.err, kDevTimeoutEmpty)) return false;
-      mbar_arrive_expect_tx(&fullD[xb], Cfg::kXtBytes);
-      tma_load_4d(dring + xb * Cfg::kXtBytes, &mXT, 0, col_begin + tt * kND, w, s, &fullD[xb]);
-    }
-    return true;
-  };
+  if (S > 1) cluster_sync();  // every CTA's barriers are initialised before a peer signals them
   bool producer_ok = true;
   bool chain_ok = true;    // warps 1 and 3: no wait of this chain has run out
   int chain_tiles = 0;     // warps 1 and 3: tiles issued by this chain so far
-  double loss_sum = 0.0;   // rank 0, thread 0: sum of the 16-row loss chunks, in step and chunk order
+  int sg0 = 0;             // steps this cluster ran for its earlier workers
 
-  // the global model, once: fp32 master block into TMEM and its bf16 copy
-  // into the resident operand (epilogue warps); head columns and biases
-  if (warp >= 4) {
-    const int quarter = warp & 3, eg = (warp - 4) >> 2;
-    const int r = quarter * 32 + lane;
-    const uint32_t trow = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
-    const float* src = a.master + gso + a.offW0 + static_cast<int64_t>(g0 + r) * D + col_begin;
-    // two of the warpgroup's tiles per pass: both tiles' loads are in flight together
-    for (int tt = eg; tt < nD; tt += 4) {
-      float v[2][32];
-#pragma unroll
-      for (int h = 0; h < 2; ++h) {
-        const int c0 = (tt + 2 * h) * kND;
-#pragma unroll
-        for (int q = 0; q < 8; ++q) {
-          const float4 x = c0 + 4 * q < ncols ? *reinterpret_cast<const float4*>(src + c0 + 4 * q)
-                                              : make_float4(0.f, 0.f, 0.f, 0.f);
-          v[h][4 * q] = x.x;
-          v[h][4 * q + 1] = x.y;
-          v[h][4 * q + 2] = x.z;
-          v[h][4 * q + 3] = x.w;
-        }
-      }
-#pragma unroll
-      for (int h = 0; h < 2; ++h) {
-        const int c0 = (tt + 2 * h) * kND;
-        if (tt + 2 * h < nD) {
-          tmem_st_32x32b_x32(trow + c0, v[h]);
-          put_w0_row32(w0s, r, c0, v[h]);
-        }
-      }
-    }
-    tmem_wait_st();
-  } else {
-    for (int q = t; q < kFC * (UPC / 4); q += 128) {
-      const int c = q / (UPC / 4), u4 = (q % (UPC / 4)) * 4;
-      const float4 m = *reinterpret_cast<const float4*>(a.master + gso + a.offW1 + static_cast<int64_t>(c) * H + g0 +
-                                                       ku0 + u4);
-      *reinterpret_cast<float4*>(w1m + c * UPC + u4) = m;
-      *reinterpret_cast<float4*>(wcs + c * UPC + u4) =
-          make_float4(bf16_round(m.x), bf16_round(m.y), bf16_round(m.z), bf16_round(m.w));
-    }
-    for (int u = t; u < kFU; u += 128) b0m[u] = a.master[gso + a.offB0 + g0 + u];
-    if (t < kFC) b1m[t] = a.master[gso + a.offB1 + t];
-  }
-  fence_proxy_async_smem();   // the resident W0 is read by the tensor core
-  tc_fence_before();
-  __syncthreads();
-  tc_fence_after();
-  if (S > 1) cluster_sync();  // every CTA's barriers are initialised before a peer signals them
-  if (warp == 0 && lane == 0) producer_ok = issue_f(0, 0, pre_f);
+  // The cluster's workers, one after the other (when there are more workers
+  // than clusters that fit on the GPU, the host deals them longest first to
+  // the cluster that will be free first).  Ring positions and barrier phases
+  // follow the cluster's running step sg = sg0 + s; the staged inputs are
+  // addressed by the worker and its own step s.
+  for (int wi = a.cl_first[blockIdx.x]; wi < a.cl_first[blockIdx.x + 1]; ++wi) {
+    const int w = a.order[wi];
+    const int tau = a.tau[w];
+    const int64_t dof = static_cast<int64_t>(w) * a.slot_stride;
+    const bool stamp = a.phase_ts && w == 0 && rank == 0 && t == 0;
 
-  for (int s = 0; s < tau; ++s) {
-    if (stamp) a.phase_ts[s * 4 + 0] = global_ns();
-    const bool last = s == tau - 1;
-    if (S > 1 && t == 0) mbar_arrive_expect_tx(pinF, Cfg::kZBytes);   // this step's incoming partials
+    // producer (warp 0 lane 0): X tiles [from, to) of step s's forward; the
+    // ring position of K-block kb of step s is (sg0 + s) * nkf + kb
+    auto issue_f = [&](int s, int from, int to) -> bool {
+      for (int kb = from; kb < to; ++kb) {
+        const int c = (sg0 + s) * nkf + kb, st = c % Cfg::kStagesF;
+        if (c >= Cfg::kStagesF && !mbar_wait(&emptyF[st], ((c / Cfg::kStagesF) + 1) & 1, a.err, kDevTimeoutEmpty))
+          return false;
+        mbar_arrive_expect_tx(&fullF[st], Cfg::kBBytes);
+        tma_load_4d(fring + st * Cfg::kBBytes, &mX, (kb_begin + kb) * kFBK, 0, w, s, &fullF[st]);
+      }
+      return true;
+    };
+    // X^T tiles [from, to) of step s's weight gradient (ring position (sg0 + s) * nD + tile)
+    auto issue_d = [&](int s, int from, int to) -> bool {
+      for (int tt = from; tt < to; ++tt) {
+        const int c = (sg0 + s) * nD + tt, xb = c % kNXD, use = c / kNXD;
+        // the buffer's previous tile must have been read by its MMA
+        if (use >= 1 && !mbar_wait(&xfreeD[xb], (use - 1) & 1, a.err, kDevTimeoutEmpty)) return false;
+        mbar_arrive_expect_tx(&fullD[xb], Cfg::kXtBytes);
+        tma_load_4d(dring + xb * Cfg::kXtBytes, &mXT, 0, col_begin + tt * kND, w, s, &fullD[xb]);
+      }
+      return true;
+    };
+    double loss_sum = 0.0;   // rank 0, thread 0: sum of the 16-row loss chunks, in step and chunk order
 
-    // ------------------------------------------------------------ F: partial forward of the group's units
-    if (warp == 0 && lane == 0) {
-      if (producer_ok) producer_ok = issue_f(s, pre_f, nkf);   // the rest of this step's X tiles
-      if (producer_ok) producer_ok = issue_d(s, 0, pre_d);     // the first X^T tiles of step D
-    } else if (warp == 1 && lane == 0) {
-      constexpr uint32_t idesc = idesc_bf16_f32(128, B);
-      for (int kb = 0; kb < nkf; ++kb) {
-        const int c = s * nkf + kb, st = c % Cfg::kStagesF;
-        if (!mbar_wait(&fullF[st], (c / Cfg::kStagesF) & 1, a.err, kDevTimeoutFull)) break;
-        tc_fence_after();
-        const uint32_t wa = smem_u32(w0s + kb * kW0Blk);
-        const uint32_t xb = smem_u32(fring + st * Cfg::kBBytes);
-#pragma unroll
-        for (int j = 0; j < kFBK / 16; ++j)
-          umma_bf16(tmem + kTAcc, smem_desc_k128(wa + j * 32), smem_desc_k128(xb + j * 32), idesc,
-                    (kb | j) != 0 ? 1u : 0u);
-        umma_commit(&emptyF[st]);
-      }
-      umma_commit(accF);
-    }
-    for (int b = t; b < B; b += kFT) labs[b] = a.labels[(static_cast<int64_t>(s) * a.W + w) * B + b];
-    if (warp >= 4) {   // epilogue F: thread = unit of the group, columns = samples
-      int ok = mbar_wait(accF, s & 1, a.err, kDevTimeoutAccum) ? 1 : 0;
-      ok = __all_sync(0xffffffffu, ok);
-      tc_fence_after();
-      if (ok) {
-        const int quarter = warp & 3, eg = (warp - 4) >> 2;
-        const int u = quarter * 32 + lane;
-        const uint32_t trow = tmem + (static_cast<uint32_t>(quarter * 32) << 16) + kTAcc;
-        for (int c0 = eg * 32; c0 < B; c0 += 64) {
-          float v[32];
-          tmem_ld_32x32b_x32(trow + c0, v);
-          if (S == 1) {
-            const float bias = b0m[u];
-#pragma unroll
-            for (int j = 0; j < 32; ++j) hs[(c0 + j) * Cfg::kHsd + u] = bf16_round(fmaxf(v[j] + bias, 0.f));
-          } else {
-            // the partial goes to the CTA that keeps unit u: this one
-            // (own rows) or, through the outgoing buffer, the partner
-            const int owner = u / UPC;
-            float* row = (owner == half ? zx : zout) + (u - owner * UPC) * Cfg::kZs + c0;
-#pragma unroll
-            for (int q = 0; q < 8; ++q)
-              *reinterpret_cast<float4*>(row + 4 * q) = make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
-            fence_proxy_async_smem();   // the outgoing rows are read by the bulk copy
-          }
-        }
-      }
-    }
-    tc_fence_before();
-    __syncthreads();
-    if (S > 1) {
-      // the partner's partials of this CTA's units: one bulk copy each way
-      // into the incoming buffer, completing on the receiver's barrier
-      if (t == 0) bulk_copy_to_peer(zin, zout, Cfg::kZBytes, pinF, grp * S + (half ^ 1));
-      // both partials of this CTA's units are local now:
-      // z = part(half 0) + part(half 1) + b0
-      mbar_wait(pinF, s & 1, a.err, kDevTimeoutFull);
-      constexpr int kZItems = UPC * (B / 4), kZPer = (kZItems + kFT - 1) / kFT;
-      float4 zr[kZPer];
-#pragma unroll
-      for (int k = 0; k < kZPer; ++k) {
-        const int q = t + k * kFT;
-        if (q < kZItems) {   // item = (unit, 4 samples), consecutive threads on consecutive units
-          const int ul = q % UPC, b4 = (q / UPC) * 4;
-          const float4 own = *reinterpret_cast<const float4*>(zx + ul * Cfg::kZs + b4);
-          const float4 inc = *reinterpret_cast<const float4*>(zin + ul * Cfg::kZs + b4);
-          const float4 p0 = half == 0 ? own : inc, p1 = half == 0 ? inc : own;
-          float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
-          z.x += p0.x;
-          z.y += p0.y;
-          z.z += p0.z;
-          z.w += p0.w;
-          z.x += p1.x;
-          z.y += p1.y;
-          z.z += p1.z;
-          z.w += p1.w;
-          zr[k] = z;
-        }
-      }
-      __syncthreads();   // the incoming partials (aliasing hs) have been read
-#pragma unroll
-      for (int k = 0; k < kZPer; ++k) {
-        const int q = t + k * kFT;
-        if (q >= kZItems) break;
-        const int ul = q % UPC, b4 = (q / UPC) * 4;
-        const int ug = ku0 + ul;                   // unit within the group
-        const float4 z = zr[k];
-        const float bias = b0m[ug];
-        hs[(b4 + 0) * Cfg::kHsd + ul] = bf16_round(fmaxf(z.x + bias, 0.f));
-        hs[(b4 + 1) * Cfg::kHsd + ul] = bf16_round(fmaxf(z.y + bias, 0.f));
-        hs[(b4 + 2) * Cfg::kHsd + ul] = bf16_round(fmaxf(z.z + bias, 0.f));
-        hs[(b4 + 3) * Cfg::kHsd + ul] = bf16_round(fmaxf(z.w + bias, 0.f));
-      }
-      __syncthreads();
-    }
-    if (stamp) a.phase_ts[s * 4 + 1] = global_ns();
-
-    // ------------------------------------------------------------ H: last layer for this CTA's units
-    if (t < 256) {   // partial logits: kTpr threads per row, all classes in registers
-      const int rb = t / Cfg::kTpr, q = t % Cfg::kTpr;
-      float acc[kFC];
-#pragma unroll
-      for (int c = 0; c < kFC; ++c) acc[c] = 0.f;
-      for (int k = 4 * q; k < UPC; k += 4 * Cfg::kTpr) {
-        const float4 hv = *reinterpret_cast<const float4*>(hs + rb * Cfg::kHsd + k);
-#pragma unroll
-        for (int c = 0; c < kFC; ++c) {
-          const float4 wv = *reinterpret_cast<const float4*>(wcs + c * UPC + k);
-          acc[c] = fmaf(hv.x, wv.x, acc[c]);
-          acc[c] = fmaf(hv.y, wv.y, acc[c]);
-          acc[c] = fmaf(hv.z, wv.z, acc[c]);
-          acc[c] = fmaf(hv.w, wv.w, acc[c]);
-        }
-      }
-#pragma unroll
-      for (int c = 0; c < kFC; ++c) {
-        for (int o = Cfg::kTpr / 2; o > 0; o >>= 1) acc[c] += __shfl_xor_sync(0xffffffffu, acc[c], o);
-        if (q == 0) pl[rb * kFC + c] = acc[c];
-      }
-    }
-    cluster_sync();
-    for (int q = t; q < B * kFC; q += kFT) {
-      float part[kFMaxCluster];
-#pragma unroll
-      for (int r = 0; r < kFMaxCluster; ++r) part[r] = r < ncl ? ld_dsmem_f32(pl + q, r) : 0.f;
-      float acc = 0.f;
-#pragma unroll
-      for (int r = 0; r < kFMaxCluster; ++r)
-        if (r < ncl) acc += part[r];
-      dz[q] = acc + b1m[q % kFC];
-    }
-    // the softmax rows below read logits summed by other threads; with S = 1
-    // this barrier also separates the remote reads of pl from the next step's
-    // writes (with S = 2 the barrier after the dz0^T exchange does that)
-    if (S == 1) cluster_sync();
-    else __syncthreads();
-    // softmax cross-entropy, four threads per row: thread q of the row takes
-    // classes q, q + 4, q + 8 (exponentials and gradients); the row's
-    // exponentials are gathered in every lane of the row and summed in class
-    // order (the arithmetic of one thread per row)
-    static_assert(4 * B <= kFT, "four threads per batch row");
-    if (t < 4 * B) {
-      const int b = t >> 2, q = t & 3, src = lane & ~3;
-      float zq[3], eq[3];
-#pragma unroll
-      for (int i = 0; i < 3; ++i) zq[i] = q + 4 * i < kFC ? dz[b * kFC + q + 4 * i] : -INFINITY;
-      float m = fmaxf(fmaxf(zq[0], zq[1]), zq[2]);
-      m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 1));
-      m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 2));
-#pragma unroll
-      for (int i = 0; i < 3; ++i) eq[i] = q + 4 * i < kFC ? expf(zq[i] - m) : 0.f;
-      const int y = labs[b];
-      float se = 0.f, so_ = 0.f;
-#pragma unroll
-      for (int c = 0; c < kFC; ++c) {
-        const float ec = __shfl_sync(0xffffffffu, eq[c >> 2], src | (c & 3));
-        se += ec;
-        if (c != y) so_ += ec;
-      }
-      if (q == (y & 3)) rowloss[b] = m + logf(se) - (y < 4 ? zq[0] : y < 8 ? zq[1] : zq[2]);
-      const float inv = 1.0f / static_cast<float>(B);
-#pragma unroll
-      for (int i = 0; i < 3; ++i) {
-        const int c = q + 4 * i;
-        if (c < kFC) {
-          const float g = (c == y ? -(so_ / se) : eq[i] / se) * inv;
-          dz[b * kFC + c] = g;
-          dzb[c * B + b] = bf16_round(g);
-        }
-      }
-    }
-    __syncthreads();
-    if (rank == 0 && t == 0) {
-      for (int c = 0; c < B / kRowsPerLossChunk; ++c) {
-        float l = 0.f;
-        for (int r = 0; r < kRowsPerLossChunk; ++r) l += rowloss[c * kRowsPerLossChunk + r];
-        loss_sum += static_cast<double>(l);
-      }
-    }
-    if (warp >= 8 && warp < 11) {   // head bias, 8 lanes per class: the same arithmetic in every CTA
-      const int idx = t - 256, c = idx >> 3, j = idx & 7;
-      float g = 0.f;
-      if (c < kFC)
-        for (int b = j; b < B; b += 8) g += dz[b * kFC + c];
-#pragma unroll
-      for (int o = 4; o > 0; o >>= 1) g += __shfl_xor_sync(0xffffffffu, g, o, 8);
-      if (j == 0 && c < kFC) {
-        const float nb = fmaf(-a.lr, g, b1m[c]);
-        b1m[c] = nb;
-        if (last && rank == 0) a.master_w[dof + a.offB1 + c] = nb;
-      }
-    }
-    // masked input gradient dz0[b][u] of this CTA's units: item = (unit, 8
-    // consecutive samples), one 16-byte chunk of the unit's K-major dz0^T
-    // row, stored here and into the other CTAs of the group
-    for (int it = t; it < UPC * Cfg::kChunks; it += kFT) {
-      const int u = it % UPC, j = it / UPC;
-      // dh[b] = sum over c in class order of dzb[c][b] w[c][u]: the eight
-      // samples of a class are two 16-byte loads of the class-major dzb
-      float dv[8];
-#pragma unroll
-      for (int i = 0; i < 8; ++i) dv[i] = 0.f;
-#pragma unroll
-      for (int c = 0; c < kFC; ++c) {
-        const float wc = wcs[c * UPC + u];
-        const float4 d0 = *reinterpret_cast<const float4*>(dzb + c * B + 8 * j);
-        const float4 d1 = *reinterpret_cast<const float4*>(dzb + c * B + 8 * j + 4);
-        dv[0] = fmaf(d0.x, wc, dv[0]);
-        dv[1] = fmaf(d0.y, wc, dv[1]);
-        dv[2] = fmaf(d0.z, wc, dv[2]);
-        dv[3] = fmaf(d0.w, wc, dv[3]);
-        dv[4] = fmaf(d1.x, wc, dv[4]);
-        dv[5] = fmaf(d1.y, wc, dv[5]);
-        dv[6] = fmaf(d1.z, wc, dv[6]);
-        dv[7] = fmaf(d1.w, wc, dv[7]);
-      }
-      float gsum = 0.f;
-#pragma unroll
-      for (int i = 0; i < 8; ++i) {
-        const float dh = hs[(8 * j + i) * Cfg::kHsd + u] > 0.f ? dv[i] : 0.f;
-        dv[i] = dh;
-        gsum += dh;
-      }
-      const uint4 p = make_uint4(pack_bf16x2(dv[0], dv[1]), pack_bf16x2(dv[2], dv[3]), pack_bf16x2(dv[4], dv[5]),
-                                 pack_bf16x2(dv[6], dv[7]));
-      uint8_t* dst = dzT + sw128_offset(ku0 + u, 8 * j);
-      *reinterpret_cast<uint4*>(dst) = p;
-#pragma unroll
-      for (int o = 0; o < S; ++o)
-        if (o != half) st_dsmem_u32x4(dst, grp * S + o, p);
-      gbp[j * UPC + u] = gsum;
-    }
-    fence_proxy_async_smem();   // dz0^T is read by the tensor core next
-    __syncthreads();
-    // head weight gradient of this CTA's columns, item = (class, 4 units),
-    // split over the two halves of the batch (partials in the idle F ring)
-    float4* w1p = reinterpret_cast<float4*>(fring);   // [2][kW1Items]
-    for (int q = t; q < 2 * Cfg::kW1Items; q += kFT) {
-      const int item = q % Cfg::kW1Items, hb = q / Cfg::kW1Items;
-      const int c = item / (UPC / 4), u4 = (item % (UPC / 4)) * 4;
-      float4 dw = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll 2
-      for (int b4 = hb * (B / 2); b4 < (hb + 1) * (B / 2); b4 += 4) {
-        const float4 g4 = *reinterpret_cast<const float4*>(dzb + c * B + b4);   // samples b4 .. b4 + 3
-        const float gk[4] = {g4.x, g4.y, g4.z, g4.w};
-#pragma unroll
-        for (int k = 0; k < 4; ++k) {
-          const float4 hv = *reinterpret_cast<const float4*>(hs + (b4 + k) * Cfg::kHsd + u4);
-          dw.x = fmaf(gk[k], hv.x, dw.x);
-          dw.y = fmaf(gk[k], hv.y, dw.y);
-          dw.z = fmaf(gk[k], hv.z, dw.z);
-          dw.w = fmaf(gk[k], hv.w, dw.w);
-        }
-      }
-      w1p[hb * Cfg::kW1Items + item] = dw;
-    }
-    if (t < UPC) {   // b0 of this CTA's units (chunk sums in chunk order)
-      float g = 0.f;
-#pragma unroll
-      for (int r = 0; r < Cfg::kChunks; ++r) g += gbp[r * UPC + t];
-      const float nb = fmaf(-a.lr, g, b0m[ku0 + t]);
-      b0m[ku0 + t] = nb;
-      if (last) a.master_w[dof + a.offB0 + g0 + ku0 + t] = nb;
-    }
-    __syncthreads();
-    // SGD of the head-weight columns: first half + second half of the batch
-    for (int item = t; item < Cfg::kW1Items; item += kFT) {
-      const int c = item / (UPC / 4), u4 = (item % (UPC / 4)) * 4;
-      const float4 d0 = w1p[item], d1 = w1p[Cfg::kW1Items + item];
-      const float4 dw = make_float4(d0.x + d1.x, d0.y + d1.y, d0.z + d1.z, d0.w + d1.w);
-      const float4 o = *reinterpret_cast<const float4*>(w1m + c * UPC + u4);
-      float4 nw;
-      nw.x = fmaf(-a.lr, dw.x, o.x);
-      nw.y = fmaf(-a.lr, dw.y, o.y);
-      nw.z = fmaf(-a.lr, dw.z, o.z);
-      nw.w = fmaf(-a.lr, dw.w, o.w);
-      *reinterpret_cast<float4*>(w1m + c * UPC + u4) = nw;
-      *reinterpret_cast<float4*>(wcs + c * UPC + u4) =
-          make_float4(bf16_round(nw.x), bf16_round(nw.y), bf16_round(nw.z), bf16_round(nw.w));
-      if (last)
-        *reinterpret_cast<float4*>(a.master_w + dof + a.offW1 + static_cast<int64_t>(c) * H + g0 + ku0 + u4) = nw;
-    }
-    if (S > 1) {
-      cluster_sync();             // the partner's dz0^T rows have landed
-      fence_proxy_async_smem();
-    }
-    if (stamp) a.phase_ts[s * 4 + 2] = global_ns();
-
-    // ------------------------------------------------------------ D: weight gradient + SGD of own W0 block
-    if (warp == 0 && lane == 0) {
-      if (producer_ok) producer_ok = issue_d(s, pre_d, nD);
-      // the first X tiles of the next step's forward, while this step's epilogue runs
-      if (producer_ok && s + 1 < tau) producer_ok = issue_f(s + 1, 0, pre_f);
-    } else if (warp == 1 || warp == 3) {
-      // two issuing chains: chain e (warp 1: e = 0, warp 3: e = 1) takes the
-      // tiles with running index c = e (mod 2), TMEM buffer e, X^T slots
-      // c % 4 (of its own parity) and epilogue warpgroup e.  The warpgroup
-      // hands the drained buffer back through named barrier 1 + e (128
-      // arrivals + this warp: cheaper than an mbarrier wait); every tile is
-      // committed, even after a failed wait, so that the arrivals and the
-      // waits on the named barrier stay paired
-      const int e = warp == 1 ? 0 : 1;
-      constexpr uint32_t idesc = idesc_bf16_f32(128, kND);
-      for (int tt = ((s * nD + e) & 1); tt < nD; tt += 2) {
-        const int c = s * nD + tt, buf = e, use = c / kNBD, xb = c % kNXD;
-        if (chain_ok) chain_ok = mbar_wait(&fullD[xb], (c / kNXD) & 1, a.err, kDevTimeoutFull);
-        if (use >= 1) bar_named(1 + e, 128 + 32);   // the previous use of the buffer has been read
-        tc_fence_after();
-        if (lane == 0) {
-          if (chain_ok) {
-            const uint32_t xa = smem_u32(dring + xb * Cfg::kXtBytes);
-            const uint32_t da = smem_u32(dzT);
-            const uint32_t dcol = tmem + static_cast<uint32_t>(kTAcc + buf * kND);
-#pragma unroll
-            for (int j = 0; j < kFBK / 16; ++j)
-              umma_bf16(dcol, smem_desc_k128(da + j * 32), smem_desc_k128(xa + j * 32), idesc, j != 0 ? 1u : 0u);
-          }
-          umma_commit(&accD[buf]);
-          umma_commit(&xfreeD[xb]);
-        }
-        __syncwarp();
-        ++chain_tiles;
-      }
-    } else if (warp >= 4) {
-      // warpgroup eg drains the tiles of chain eg (its TMEM buffer); a warp
-      // covers 32 rows
+    // the global model, once per worker: fp32 master block into TMEM and its bf16 copy
+    // into the resident operand (epilogue warps); head columns and biases
+    if (warp >= 4) {
       const int quarter = warp & 3, eg = (warp - 4) >> 2;
       const int r = quarter * 32 + lane;
       const uint32_t trow = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
-      for (int tt = ((s * nD + eg) & 1); tt < nD; tt += 2) {
-        const int c = s * nD + tt, buf = eg, use = c / kNBD;
-        int ok = mbar_wait(&accD[buf], use & 1, a.err, kDevTimeoutAccum) ? 1 : 0;
-        ok = __all_sync(0xffffffffu, ok);
-        tc_fence_after();
-        if (ok) {
-          const int c0 = tt * kND;
-          float g[32], m[32];
-          tmem_ld_32x32b_x32_pair(trow + kTAcc + buf * kND, g, trow + c0, m);
-          tc_fence_before();
-          bar_arrive_named(1 + eg, 128 + 32);   // the gradient buffer has been read: the next MMA may reuse it
-#pragma unroll
-          for (int j = 0; j < 32; ++j) m[j] = fmaf(-a.lr, g[j], m[j]);
-          tmem_st_32x32b_x32(trow + c0, m);
-          put_w0_row32(w0s, r, c0, m);
-        } else {
-          tc_fence_before();
-          bar_arrive_named(1 + eg, 128 + 32);
+      const float* src = a.master + gso + a.offW0 + static_cast<int64_t>(g0 + r) * D + col_begin;
+      // two of the warpgroup's tiles per pass: both tiles' loads are in flight together
+      for (int tt = eg; tt < nD; tt += 4) {
+        float v[2][32];
+  #pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          const int c0 = (tt + 2 * h) * kND;
+  #pragma unroll
+          for (int q = 0; q < 8; ++q) {
+            const float4 x = c0 + 4 * q < ncols ? *reinterpret_cast<const float4*>(src + c0 + 4 * q)
+                                                : make_float4(0.f, 0.f, 0.f, 0.f);
+            v[h][4 * q] = x.x;
+            v[h][4 * q + 1] = x.y;
+            v[h][4 * q + 2] = x.z;
+            v[h][4 * q + 3] = x.w;
+          }
+        }
+  #pragma unroll
+        for (int h = 0; h < 2; ++h) {
+          const int c0 = (tt + 2 * h) * kND;
+          if (tt + 2 * h < nD) {
+            tmem_st_32x32b_x32(trow + c0, v[h]);
+            put_w0_row32(w0s, r, c0, v[h]);
+          }
         }
       }
-      tmem_wait_st();   // the master columns stored above are read again next step
+      tmem_wait_st();
+    } else {
+      for (int q = t; q < kFC * (UPC / 4); q += 128) {
+        const int c = q / (UPC / 4), u4 = (q % (UPC / 4)) * 4;
+        const float4 m = *reinterpret_cast<const float4*>(a.master + gso + a.offW1 + static_cast<int64_t>(c) * H + g0 +
+                                                         ku0 + u4);
+        *reinterpret_cast<float4*>(w1m + c * UPC + u4) = m;
+        *reinterpret_cast<float4*>(wcs + c * UPC + u4) =
+            make_float4(bf16_round(m.x), bf16_round(m.y), bf16_round(m.z), bf16_round(m.w));
+      }
+      for (int u = t; u < kFU; u += 128) b0m[u] = a.master[gso + a.offB0 + g0 + u];
+      if (t < kFC) b1m[t] = a.master[gso + a.offB1 + t];
     }
-    fence_proxy_async_smem();   // the resident W0 written here is read by the tensor core next step
+    fence_proxy_async_smem();   // the resident W0 is read by the tensor core
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    if (stamp) a.phase_ts[s * 4 + 3] = global_ns();
+    if (warp == 0 && lane == 0) producer_ok = issue_f(0, 0, pre_f);
+
+    for (int s = 0; s < tau; ++s) {
+      if (stamp) a.phase_ts[s * 4 + 0] = global_ns();
+      const bool last = s == tau - 1;
+      const int sg = sg0 + s;
+      if (S > 1 && t == 0) mbar_arrive_expect_tx(pinF, Cfg::kZBytes);   // this step's incoming partials
+
+      // ------------------------------------------------------------ F: partial forward of the group's units
+      if (warp == 0 && lane == 0) {
+        if (producer_ok) producer_ok = issue_f(s, pre_f, nkf);   // the rest of this step's X tiles
+        if (producer_ok) producer_ok = issue_d(s, 0, pre_d);     // the first X^T tiles of step D
+      } else if (warp == 1 && lane == 0) {
+        constexpr uint32_t idesc = idesc_bf16_f32(128, B);
+        for (int kb = 0; kb < nkf; ++kb) {
+          const int c = sg * nkf + kb, st = c % Cfg::kStagesF;
+          if (!mbar_wait(&fullF[st], (c / Cfg::kStagesF) & 1, a.err, kDevTimeoutFull)) break;
+          tc_fence_after();
+          const uint32_t wa = smem_u32(w0s + kb * kW0Blk);
+          const uint32_t xb = smem_u32(fring + st * Cfg::kBBytes);
+  #pragma unroll
+          for (int j = 0; j < kFBK / 16; ++j)
+            umma_bf16(tmem + kTAcc, smem_desc_k128(wa + j * 32), smem_desc_k128(xb + j * 32), idesc,
+                      (kb | j) != 0 ? 1u : 0u);
+          umma_commit(&emptyF[st]);
+        }
+        umma_commit(accF);
+      }
+      for (int b = t; b < B; b += kFT) labs[b] = a.labels[(static_cast<int64_t>(s) * a.W + w) * B + b];
+      if (warp >= 4) {   // epilogue F: thread = unit of the group, columns = samples
+        int ok = mbar_wait(accF, sg & 1, a.err, kDevTimeoutAccum) ? 1 : 0;
+        ok = __all_sync(0xffffffffu, ok);
+        tc_fence_after();
+        if (ok) {
+          const int quarter = warp & 3, eg = (warp - 4) >> 2;
+          const int u = quarter * 32 + lane;
+          const uint32_t trow = tmem + (static_cast<uint32_t>(quarter * 32) << 16) + kTAcc;
+          for (int c0 = eg * 32; c0 < B; c0 += 64) {
+            float v[32];
+            tmem_ld_32x32b_x32(trow + c0, v);
+            if (S == 1) {
+              const float bias = b0m[u];
+  #pragma unroll
+              for (int j = 0; j < 32; ++j) hs[(c0 + j) * Cfg::kHsd + u] = bf16_round(fmaxf(v[j] + bias, 0.f));
+            } else {
+              // the partial goes to the CTA that keeps unit u: this one
+              // (own rows) or, through the outgoing buffer, the partner
+              const int owner = u / UPC;
+              float* row = (owner == half ? zx : zout) + (u - owner * UPC) * Cfg::kZs + c0;
+  #pragma unroll
+              for (int q = 0; q < 8; ++q)
+                *reinterpret_cast<float4*>(row + 4 * q) =
+                    make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+              fence_proxy_async_smem();   // the outgoing rows are read by the bulk copy
+            }
+          }
+        }
+      }
+      tc_fence_before();
+      __syncthreads();
+      if (S > 1) {
+        // the partner's partials of this CTA's units: one bulk copy each way
+        // into the incoming buffer, completing on the receiver's barrier
+        if (t == 0) bulk_copy_to_peer(zin, zout, Cfg::kZBytes, pinF, grp * S + (half ^ 1));
+        // both partials of this CTA's units are local now:
+        // z = part(half 0) + part(half 1) + b0
+        mbar_wait(pinF, sg & 1, a.err, kDevTimeoutFull);
+        constexpr int kZItems = UPC * (B / 4), kZPer = (kZItems + kFT - 1) / kFT;
+        float4 zr[kZPer];
+  #pragma unroll
+        for (int k = 0; k < kZPer; ++k) {
+          const int q = t + k * kFT;
+          if (q < kZItems) {   // item = (unit, 4 samples), consecutive threads on consecutive units
+            const int ul = q % UPC, b4 = (q / UPC) * 4;
+            const float4 own = *reinterpret_cast<const float4*>(zx + ul * Cfg::kZs + b4);
+            const float4 inc = *reinterpret_cast<const float4*>(zin + ul * Cfg::kZs + b4);
+            const float4 p0 = half == 0 ? own : inc, p1 = half == 0 ? inc : own;
+            float4 z = make_float4(0.f, 0.f, 0.f, 0.f);
+            z.x += p0.x;
+            z.y += p0.y;
+            z.z += p0.z;
+            z.w += p0.w;
+            z.x += p1.x;
+            z.y += p1.y;
+            z.z += p1.z;
+            z.w += p1.w;
+            zr[k] = z;
+          }
+        }
+        __syncthreads();   // the incoming partials (aliasing hs) have been read
+  #pragma unroll
+        for (int k = 0; k < kZPer; ++k) {
+          const int q = t + k * kFT;
+          if (q >= kZItems) break;
+          const int ul = q % UPC, b4 = (q / UPC) * 4;
+          const int ug = ku0 + ul;                   // unit within the group
+          const float4 z = zr[k];
+          const float bias = b0m[ug];
+          hs[(b4 + 0) * Cfg::kHsd + ul] = bf16_round(fmaxf(z.x + bias, 0.f));
+          hs[(b4 + 1) * Cfg::kHsd + ul] = bf16_round(fmaxf(z.y + bias, 0.f));
+          hs[(b4 + 2) * Cfg::kHsd + ul] = bf16_round(fmaxf(z.z + bias, 0.f));
+          hs[(b4 + 3) * Cfg::kHsd + ul] = bf16_round(fmaxf(z.w + bias, 0.f));
+        }
+        __syncthreads();
+      }
+      if (stamp) a.phase_ts[s * 4 + 1] = global_ns();
+
+      // ------------------------------------------------------------ H: last layer for this CTA's units
+      if (t < 256) {   // partial logits: kTpr threads per row, all classes in registers
+        const int rb = t / Cfg::kTpr, q = t % Cfg::kTpr;
+        float acc[kFC];
+  #pragma unroll
+        for (int c = 0; c < kFC; ++c) acc[c] = 0.f;
+        for (int k = 4 * q; k < UPC; k += 4 * Cfg::kTpr) {
+          const float4 hv = *reinterpret_cast<const float4*>(hs + rb * Cfg::kHsd + k);
+  #pragma unroll
+          for (int c = 0; c < kFC; ++c) {
+            const float4 wv = *reinterpret_cast<const float4*>(wcs + c * UPC + k);
+            acc[c] = fmaf(hv.x, wv.x, acc[c]);
+            acc[c] = fmaf(hv.y, wv.y, acc[c]);
+            acc[c] = fmaf(hv.z, wv.z, acc[c]);
+            acc[c] = fmaf(hv.w, wv.w, acc[c]);
+          }
+        }
+  #pragma unroll
+        for (int c = 0; c < kFC; ++c) {
+          for (int o = Cfg::kTpr / 2; o > 0; o >>= 1) acc[c] += __shfl_xor_sync(0xffffffffu, acc[c], o);
+          if (q == 0) pl[rb * kFC + c] = acc[c];
+        }
+      }
+      cluster_sync();
+      for (int q = t; q < B * kFC; q += kFT) {
+        float part[kFMaxCluster];
+  #pragma unroll
+        for (int r = 0; r < kFMaxCluster; ++r) part[r] = r < ncl ? ld_dsmem_f32(pl + q, r) : 0.f;
+        float acc = 0.f;
+  #pragma unroll
+        for (int r = 0; r < kFMaxCluster; ++r)
+          if (r < ncl) acc += part[r];
+        dz[q] = acc + b1m[q % kFC];
+      }
+      // the softmax rows below read logits summed by other threads; with S = 1
+      // this barrier also separates the remote reads of pl from the next step's
+      // writes (with S = 2 the barrier after the dz0^T exchange does that)
+      if (S == 1) cluster_sync();
+      else __syncthreads();
+      // softmax cross-entropy, four threads per row: thread q of the row takes
+      // classes q, q + 4, q + 8 (exponentials and gradients); the row's
+      // exponentials are gathered in every lane of the row and summed in class
+      // order (the arithmetic of one thread per row)
+      static_assert(4 * B <= kFT, "four threads per batch row");
+      if (t < 4 * B) {
+        const int b = t >> 2, q = t & 3, src = lane & ~3;
+        float zq[3], eq[3];
+  #pragma unroll
+        for (int i = 0; i < 3; ++i) zq[i] = q + 4 * i < kFC ? dz[b * kFC + q + 4 * i] : -INFINITY;
+        float m = fmaxf(fmaxf(zq[0], zq[1]), zq[2]);
+        m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 1));
+        m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 2));
+  #pragma unroll
+        for (int i = 0; i < 3; ++i) eq[i] = q + 4 * i < kFC ? expf(zq[i] - m) : 0.f;
+        const int y = labs[b];
+        float se = 0.f, so_ = 0.f;
+  #pragma unroll
+        for (int c = 0; c < kFC; ++c) {
+          const float ec = __shfl_sync(0xffffffffu, eq[c >> 2], src | (c & 3));
+          se += ec;
+          if (c != y) so_ += ec;
+        }
+        if (q == (y & 3)) rowloss[b] = m + logf(se) - (y < 4 ? zq[0] : y < 8 ? zq[1] : zq[2]);
+        const float inv = 1.0f / static_cast<float>(B);
+  #pragma unroll
+        for (int i = 0; i < 3; ++i) {
+          const int c = q + 4 * i;
+          if (c < kFC) {
+            const float g = (c == y ? -(so_ / se) : eq[i] / se) * inv;
+            dz[b * kFC + c] = g;
+            dzb[c * B + b] = bf16_round(g);
+          }
+        }
+      }
+      __syncthreads();
+      if (rank == 0 && t == 0) {
+        for (int c = 0; c < B / kRowsPerLossChunk; ++c) {
+          float l = 0.f;
+          for (int r = 0; r < kRowsPerLossChunk; ++r) l += rowloss[c * kRowsPerLossChunk + r];
+          loss_sum += static_cast<double>(l);
+        }
+      }
+      if (warp >= 8 && warp < 11) {   // head bias, 8 lanes per class: the same arithmetic in every CTA
+        const int idx = t - 256, c = idx >> 3, j = idx & 7;
+        float g = 0.f;
+        if (c < kFC)
+          for (int b = j; b < B; b += 8) g += dz[b * kFC + c];
+  #pragma unroll
+        for (int o = 4; o > 0; o >>= 1) g += __shfl_xor_sync(0xffffffffu, g, o, 8);
+        if (j == 0 && c < kFC) {
+          const float nb = fmaf(-a.lr, g, b1m[c]);
+          b1m[c] = nb;
+          if (last && rank == 0) a.master_w[dof + a.offB1 + c] = nb;
+        }
+      }
+      // masked input gradient dz0[b][u] of this CTA's units: item = (unit, 8
+      // consecutive samples), one 16-byte chunk of the unit's K-major dz0^T
+      // row, stored here and into the other CTAs of the group
+      for (int it = t; it < UPC * Cfg::kChunks; it += kFT) {
+        const int u = it % UPC, j = it / UPC;
+        // dh[b] = sum over c in class order of dzb[c][b] w[c][u]: the eight
+        // samples of a class are two 16-byte loads of the class-major dzb
+        float dv[8];
+  #pragma unroll
+        for (int i = 0; i < 8; ++i) dv[i] = 0.f;
+  #pragma unroll
+        for (int c = 0; c < kFC; ++c) {
+          const float wc = wcs[c * UPC + u];
+          const float4 d0 = *reinterpret_cast<const float4*>(dzb + c * B + 8 * j);
+          const float4 d1 = *reinterpret_cast<const float4*>(dzb + c * B + 8 * j + 4);
+          dv[0] = fmaf(d0.x, wc, dv[0]);
+          dv[1] = fmaf(d0.y, wc, dv[1]);
+          dv[2] = fmaf(d0.z, wc, dv[2]);
+          dv[3] = fmaf(d0.w, wc, dv[3]);
+          dv[4] = fmaf(d1.x, wc, dv[4]);
+          dv[5] = fmaf(d1.y, wc, dv[5]);
+          dv[6] = fmaf(d1.z, wc, dv[6]);
+          dv[7] = fmaf(d1.w, wc, dv[7]);
+        }
+        float gsum = 0.f;
+  #pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          const float dh = hs[(8 * j + i) * Cfg::kHsd + u] > 0.f ? dv[i] : 0.f;
+          dv[i] = dh;
+          gsum += dh;
+        }
+        const uint4 p = make_uint4(pack_bf16x2(dv[0], dv[1]), pack_bf16x2(dv[2], dv[3]), pack_bf16x2(dv[4], dv[5]),
+                                   pack_bf16x2(dv[6], dv[7]));
+        uint8_t* dst = dzT + sw128_offset(ku0 + u, 8 * j);
+        *reinterpret_cast<uint4*>(dst) = p;
+  #pragma unroll
+        for (int o = 0; o < S; ++o)
+          if (o != half) st_dsmem_u32x4(dst, grp * S + o, p);
+        gbp[j * UPC + u] = gsum;
+      }
+      fence_proxy_async_smem();   // dz0^T is read by the tensor core next
+      __syncthreads();
+      // head weight gradient of this CTA's columns, item = (class, 4 units),
+      // split over the two halves of the batch (partials in the idle F ring)
+      float4* w1p = reinterpret_cast<float4*>(fring);   // [2][kW1Items]
+      for (int q = t; q < 2 * Cfg::kW1Items; q += kFT) {
+        const int item = q % Cfg::kW1Items, hb = q / Cfg::kW1Items;
+        const int c = item / (UPC / 4), u4 = (item % (UPC / 4)) * 4;
+        float4 dw = make_float4(0.f, 0.f, 0.f, 0.f);
+  #pragma unroll 2
+        for (int b4 = hb * (B / 2); b4 < (hb + 1) * (B / 2); b4 += 4) {
+          const float4 g4 = *reinterpret_cast<const float4*>(dzb + c * B + b4);   // samples b4 .. b4 + 3
+          const float gk[4] = {g4.x, g4.y, g4.z, g4.w};
+  #pragma unroll
+          for (int k = 0; k < 4; ++k) {
+            const float4 hv = *reinterpret_cast<const float4*>(hs + (b4 + k) * Cfg::kHsd + u4);
+            dw.x = fmaf(gk[k], hv.x, dw.x);
+            dw.y = fmaf(gk[k], hv.y, dw.y);
+            dw.z = fmaf(gk[k], hv.z, dw.z);
+            dw.w = fmaf(gk[k], hv.w, dw.w);
+          }
+        }
+        w1p[hb * Cfg::kW1Items + item] = dw;
+      }
+      if (t < UPC) {   // b0 of this CTA's units (chunk sums in chunk order)
+        float g = 0.f;
+  #pragma unroll
+        for (int r = 0; r < Cfg::kChunks; ++r) g += gbp[r * UPC + t];
+        const float nb = fmaf(-a.lr, g, b0m[ku0 + t]);
+        b0m[ku0 + t] = nb;
+        if (last) a.master_w[dof + a.offB0 + g0 + ku0 + t] = nb;
+      }
+      __syncthreads();
+      // SGD of the head-weight columns: first half + second half of the batch
+      for (int item = t; item < Cfg::kW1Items; item += kFT) {
+        const int c = item / (UPC / 4), u4 = (item % (UPC / 4)) * 4;
+        const float4 d0 = w1p[item], d1 = w1p[Cfg::kW1Items + item];
+        const float4 dw = make_float4(d0.x + d1.x, d0.y + d1.y, d0.z + d1.z, d0.w + d1.w);
+        const float4 o = *reinterpret_cast<const float4*>(w1m + c * UPC + u4);
+        float4 nw;
+        nw.x = fmaf(-a.lr, dw.x, o.x);
+        nw.y = fmaf(-a.lr, dw.y, o.y);
+        nw.z = fmaf(-a.lr, dw.z, o.z);
+        nw.w = fmaf(-a.lr, dw.w, o.w);
+        *reinterpret_cast<float4*>(w1m + c * UPC + u4) = nw;
+        *reinterpret_cast<float4*>(wcs + c * UPC + u4) =
+            make_float4(bf16_round(nw.x), bf16_round(nw.y), bf16_round(nw.z), bf16_round(nw.w));
+        if (last)
+          *reinterpret_cast<float4*>(a.master_w + dof + a.offW1 + static_cast<int64_t>(c) * H + g0 + ku0 + u4) = nw;
+      }
+      if (S > 1) {
+        cluster_sync();             // the partner's dz0^T rows have landed
+        fence_proxy_async_smem();
+      }
+      if (stamp) a.phase_ts[s * 4 + 2] = global_ns();
+
+      // ------------------------------------------------------------ D: weight gradient + SGD of own W0 block
+      if (warp == 0 && lane == 0) {
+        if (producer_ok) producer_ok = issue_d(s, pre_d, nD);
+        // the first X tiles of the next step's forward, while this step's epilogue runs
+        if (producer_ok && s + 1 < tau) producer_ok = issue_f(s + 1, 0, pre_f);
+      } else if (warp == 1 || warp == 3) {
+        // two issuing chains: chain e (warp 1: e = 0, warp 3: e = 1) takes the
+        // tiles with running index c = e (mod 2), TMEM buffer e, X^T slots
+        // c % 4 (of its own parity) and epilogue warpgroup e.  The warpgroup
+        // hands the drained buffer back through named barrier 1 + e (128
+        // arrivals + this warp: cheaper than an mbarrier wait); every tile is
+        // committed, even after a failed wait, so that the arrivals and the
+        // waits on the named barrier stay paired
+        const int e = warp == 1 ? 0 : 1;
+        constexpr uint32_t idesc = idesc_bf16_f32(128, kND);
+        for (int tt = ((sg * nD + e) & 1); tt < nD; tt += 2) {
+          const int c = sg * nD + tt, buf = e, use = c / kNBD, xb = c % kNXD;
+          if (chain_ok) chain_ok = mbar_wait(&fullD[xb], (c / kNXD) & 1, a.err, kDevTimeoutFull);
+          if (use >= 1) bar_named(1 + e, 128 + 32);   // the previous use of the buffer has been read
+          tc_fence_after();
+          if (lane == 0) {
+            if (chain_ok) {
+              const uint32_t xa = smem_u32(dring + xb * Cfg::kXtBytes);
+              const uint32_t da = smem_u32(dzT);
+              const uint32_t dcol = tmem + static_cast<uint32_t>(kTAcc + buf * kND);
+  #pragma unroll
+              for (int j = 0; j < kFBK / 16; ++j)
+                umma_bf16(dcol, smem_desc_k128(da + j * 32), smem_desc_k128(xa + j * 32), idesc, j != 0 ? 1u : 0u);
+            }
+            umma_commit(&accD[buf]);
+            umma_commit(&xfreeD[xb]);
+          }
+          __syncwarp();
+          ++chain_tiles;
+        }
+      } else if (warp >= 4) {
+        // warpgroup eg drains the tiles of chain eg (its TMEM buffer); a warp
+        // covers 32 rows
+        const int quarter = warp & 3, eg = (warp - 4) >> 2;
+        const int r = quarter * 32 + lane;
+        const uint32_t trow = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
+        for (int tt = ((sg * nD + eg) & 1); tt < nD; tt += 2) {
+          const int c = sg * nD + tt, buf = eg, use = c / kNBD;
+          int ok = mbar_wait(&accD[buf], use & 1, a.err, kDevTimeoutAccum) ? 1 : 0;
+          ok = __all_sync(0xffffffffu, ok);
+          tc_fence_after();
+          if (ok) {
+            const int c0 = tt * kND;
+            float g[32], m[32];
+            tmem_ld_32x32b_x32_pair(trow + kTAcc + buf * kND, g, trow + c0, m);
+            tc_fence_before();
+            bar_arrive_named(1 + eg, 128 + 32);   // the gradient buffer has been read: the next MMA may reuse it
+  #pragma unroll
+            for (int j = 0; j < 32; ++j) m[j] = fmaf(-a.lr, g[j], m[j]);
+            tmem_st_32x32b_x32(trow + c0, m);
+            put_w0_row32(w0s, r, c0, m);
+          } else {
+            tc_fence_before();
+            bar_arrive_named(1 + eg, 128 + 32);
+          }
+        }
+        tmem_wait_st();   // the master columns stored above are read again next step
+      }
+      fence_proxy_async_smem();   // the resident W0 written here is read by the tensor core next step
+      tc_fence_before();
+      __syncthreads();
+      tc_fence_after();
+      if (stamp) a.phase_ts[s * 4 + 3] = global_ns();
+    }
+    // the worker's W0 block into its replica slot: each warp moves 32 rows x
+    // 32 columns at a time from TMEM through a padded shared tile (the TMA
+    // rings are idle now), 4 full 128-byte rows per store instruction
+    if (warp >= 4) {
+      const int quarter = warp & 3, eg = (warp - 4) >> 2;
+      const uint32_t trow = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
+      float* T = reinterpret_cast<float*>(sm + Cfg::oRegion) + (warp - 4) * 32 * 36;
+      float* dst = a.master_w + dof + a.offW0 + static_cast<int64_t>(g0 + quarter * 32) * D + col_begin;
+      const int cq = (lane & 7) * 4;
+      for (int tt = eg; tt < nD; tt += 2) {
+        const int c0 = tt * kND;
+        float m[32];
+        tmem_ld_32x32b_x32(trow + c0, m);
+  #pragma unroll
+        for (int q = 0; q < 8; ++q)
+          *reinterpret_cast<float4*>(T + lane * 36 + 4 * q) =
+              make_float4(m[4 * q], m[4 * q + 1], m[4 * q + 2], m[4 * q + 3]);
+        __syncwarp();
+        if (c0 + cq < ncols) {
+  #pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            const int rr = 4 * i + (lane >> 3);
+            *reinterpret_cast<float4*>(dst + static_cast<int64_t>(rr) * D + c0 + cq) =
+                *reinterpret_cast<const float4*>(T + rr * 36 + cq);
+          }
+        }
+        __syncwarp();
+      }
+    }
+    // round bookkeeping of this worker: mean loss over its steps and the data cursor
+    if (rank == 0 && t == 0) {
+      a.loss_out[w] = static_cast<float>(loss_sum / (static_cast<double>(B) * tau));
+      if (a.cursor) a.cursor[w] = (a.cursor[w] + static_cast<int64_t>(tau) * B) % a.shard_n[w];
+    }
+    // the write-back has read TMEM and the shared tile before the next worker's model goes in
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    sg0 += tau;
   }
   // the last drain of each chain's buffer pairs with one more wait
   if ((warp == 1 || warp == 3) && chain_tiles > 0) bar_named(1 + (warp == 1 ? 0 : 1), 128 + 32);
-  // the worker's W0 block into its replica slot: each warp moves 32 rows x
-  // 32 columns at a time from TMEM through a padded shared tile (the TMA
-  // rings are idle now), 4 full 128-byte rows per store instruction
-  if (warp >= 4) {
-    const int quarter = warp & 3, eg = (warp - 4) >> 2;
-    const uint32_t trow = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
-    float* T = reinterpret_cast<float*>(sm + Cfg::oRegion) + (warp - 4) * 32 * 36;
-    float* dst = a.master_w + dof + a.offW0 + static_cast<int64_t>(g0 + quarter * 32) * D + col_begin;
-    const int cq = (lane & 7) * 4;
-    for (int tt = eg; tt < nD; tt += 2) {
-      const int c0 = tt * kND;
-      float m[32];
-      tmem_ld_32x32b_x32(trow + c0, m);
-#pragma unroll
-      for (int q = 0; q < 8; ++q)
-        *reinterpret_cast<float4*>(T + lane * 36 + 4 * q) = make_float4(m[4 * q], m[4 * q + 1], m[4 * q + 2], m[4 * q + 3]);
-      __syncwarp();
-      if (c0 + cq < ncols) {
-#pragma unroll
-        for (int i = 0; i < 8; ++i) {
-          const int rr = 4 * i + (lane >> 3);
-          *reinterpret_cast<float4*>(dst + static_cast<int64_t>(rr) * D + c0 + cq) =
-              *reinterpret_cast<const float4*>(T + rr * 36 + cq);
-        }
-      }
-      __syncwarp();
-    }
-  }
-  // round bookkeeping of this worker: mean loss over its steps and the data cursor
-  if (rank == 0 && t == 0) {
-    a.loss_out[w] = static_cast<float>(loss_sum / (static_cast<double>(B) * tau));
-    if (a.cursor) a.cursor[w] = (a.cursor[w] + static_cast<int64_t>(tau) * B) % a.shard_n[w];
-  }
   tc_fence_before();
   __syncthreads();
   if (warp == 2) {
@@ -775,7 +793,7 @@ cudaError_t launch_bs(const CUtensorMap& mX, const CUtensorMap& mXT, const Fused
                                        Cfg::kSmem);
   if (e != cudaSuccess) return e;
   cudaLaunchConfig_t cfg = {};
-  cfg.gridDim = dim3(a.W, S * (a.H / kFU), 1);
+  cfg.gridDim = dim3(a.n_clusters, S * (a.H / kFU), 1);
   cfg.blockDim = dim3(kFT, 1, 1);
   cfg.dynamicSmemBytes = Cfg::kSmem;
   cfg.stream = s;
@@ -822,11 +840,48 @@ bool fused_round_supported(int L, int D, int H, int C, int B) {
 
 int fused_round_xt_rows(int) { return kND; }
 
+namespace {
+template <int B, int S>
+int max_clusters_bs(int H) {
+  using Cfg = FCfg<B, S>;
+  if (cudaFuncSetAttribute(fused_mlp2_round_kernel<B, S>, cudaFuncAttributeMaxDynamicSharedMemorySize, Cfg::kSmem) !=
+      cudaSuccess)
+    return 0;
+  cudaLaunchConfig_t cfg = {};
+  const int ncl = S * (H / kFU);
+  cfg.gridDim = dim3(1, ncl, 1);
+  cfg.blockDim = dim3(kFT, 1, 1);
+  cfg.dynamicSmemBytes = Cfg::kSmem;
+  cudaLaunchAttribute attr;
+  attr.id = cudaLaunchAttributeClusterDimension;
+  attr.val.clusterDim.x = 1;
+  attr.val.clusterDim.y = ncl;
+  attr.val.clusterDim.z = 1;
+  cfg.attrs = &attr;
+  cfg.numAttrs = 1;
+  int n = 0;
+  if (cudaOccupancyMaxActiveClusters(&n, fused_mlp2_round_kernel<B, S>, &cfg) != cudaSuccess) {
+    cudaGetLastError();
+    return 0;
+  }
+  return n;
+}
+}  // namespace
+
+int fused_round_max_clusters(int D, int H, int B) {
+  const int S = split_for(D, H);
+  if (B == 32) return S == 2 ? max_clusters_bs<32, 2>(H) : max_clusters_bs<32, 1>(H);
+  if (B == 64) return S == 2 ? max_clusters_bs<64, 2>(H) : max_clusters_bs<64, 1>(H);
+  return 0;
+}
+
 cudaError_t launch_fused_round(const CUtensorMap& mX, const CUtensorMap& mXT, const FusedRoundArgs& r, cudaStream_t s) {
   FusedArgs a;
   a.tau = r.tau;
   a.order = r.order;
+  a.cl_first = r.cl_first;
   a.W = r.W;
+  a.n_clusters = r.n_clusters;
   a.D = r.D;
   a.H = r.H;
   a.global_slot = r.global_slot;

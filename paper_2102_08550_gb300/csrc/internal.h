@@ -185,8 +185,9 @@ cudaError_t launch_head_bwd(const HeadArgs& a, int n_active, cudaStream_t s);
 // ---------------------------------------------------------------- fused round (2-layer MLP)
 struct FusedRoundArgs {
   const int32_t* tau;
-  const int32_t* order;           // [W] workers by decreasing tau (cluster launch order)
-  int W, D, H, B;
+  const int32_t* order;           // [W] workers, cluster by cluster (longest first)
+  const int32_t* cl_first;        // [n_clusters + 1] cluster k runs order[cl_first[k] .. cl_first[k + 1])
+  int W, n_clusters, D, H, B;
   int global_slot;
   float lr;
   const float* master;
@@ -206,6 +207,8 @@ struct FusedRoundArgs {
 // worker, the worker's model resident on chip for the round)
 bool fused_round_supported(int L, int D, int H, int C, int B);
 int fused_round_xt_rows(int B);   // rows of the X^T box the kernel loads
+// clusters of the round kernel that fit on the device at once (0 if unknown)
+int fused_round_max_clusters(int D, int H, int B);
 // mX: staged inputs {D, B, W, steps} box {64, B}; mXT: staged transposed
 // inputs {B, D, W, steps} box {64, fused_round_xt_rows(B)}; both bf16,
 // 128-byte swizzle
