@@ -61,12 +61,13 @@
 // The staging of the next round into the other input buffer runs beside
 // the kernel at a lower launch priority, on the SMs its clusters leave free.
 //
-// Clusters are launched in order of decreasing tau (a table maps cluster to
-// worker): when fewer clusters fit on the GPU than there are workers, the
-// late ones start as the short workers finish (longest first).
+// The grid has one cluster per worker, or as many clusters as fit on the GPU
+// at once when there are more workers; a table gives each cluster its
+// workers, which it runs one after the other (the host deals them by
+// decreasing tau to the cluster with the least work so far).
 //
 // Warp roles (384 threads): warp 0 lane 0 issues TMA, warp 1 lane 0 issues
-// tcgen05.mma (in step D with warp 3 lane 0: one chain each), warp 2 owns the
+// tcgen05.mma (in step D warps 1 and 3 issue one chain each), warp 2 owns the
 // TMEM allocation (all 512 columns: one CTA per SM), warps 4..11 are the two
 // epilogue warpgroups (each covering the 128 TMEM lanes), all warps share the
 // CUDA-core work of step H.
