@@ -192,6 +192,8 @@ struct FusedArgs {
 template <int B, int S>
 __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_constant__ CUtensorMap mX,
                                                                  const __grid_constant__ CUtensorMap mXT,
+                                                                 const __grid_constant__ CUtensorMap mW0f,
+                                                                 const __grid_constant__ CUtensorMap mW0b,
                                                                  const __grid_constant__ FusedArgs a) {
   using Cfg = FCfg<B, S>;
   constexpr int UPC = Cfg::kUPC;
@@ -228,7 +230,8 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
   uint64_t* xfreeD = fullD + kNXD;             // [kNXD] X^T tile consumed by its MMA
   uint64_t* accD = xfreeD + kNXD;              // [kNBD] TMEM buffer full
   uint64_t* pinF = accD + kNBD;                // [1] the partner's partials landed (S = 2)
-  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(pinF + 1);
+  uint64_t* ldW = pinF + 1;                    // [1] model tiles landed (prologue)
+  uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(ldW + 1);
 
   const int rank = static_cast<int>(cluster_ctarank());
   const int ncl = static_cast<int>(gridDim.y);
@@ -252,6 +255,8 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
   if (t == 0) {
     prefetch_tmap(&mX);
     prefetch_tmap(&mXT);
+    prefetch_tmap(&mW0f);
+    prefetch_tmap(&mW0b);
     for (int i = 0; i < Cfg::kStagesF; ++i) {
       mbar_init(&fullF[i], 1);
       mbar_init(&emptyF[i], 1);
@@ -263,6 +268,7 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
     }
     for (int i = 0; i < kNBD; ++i) mbar_init(&accD[i], 1);
     mbar_init(pinF, 1);
+    mbar_init(ldW, 1);
     fence_barrier_init();
     fence_proxy_async_smem();
   }
@@ -283,6 +289,7 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
   bool chain_ok = true;    // warps 1 and 3: no wait of this chain has run out
   int chain_tiles = 0;     // warps 1 and 3: tiles issued by this chain so far
   int sg0 = 0;             // steps this cluster ran for its earlier workers
+  int ld_phase = 0;        // completed phases of ldW
 
   // The cluster's workers, one after the other (when there are more workers
   // than clusters that fit on the GPU, the host deals them longest first to
@@ -320,40 +327,14 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
     };
     double loss_sum = 0.0;   // rank 0, thread 0: sum of the 16-row loss chunks, in step and chunk order
 
-    // the global model, once per worker: fp32 master block into TMEM and its bf16 copy
-    // into the resident operand (epilogue warps); head columns and biases
-    if (warp >= 4) {
-      const int quarter = warp & 3, eg = (warp - 4) >> 2;
-      const int r = quarter * 32 + lane;
-      const uint32_t trow = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
-      const float* src = a.master + gso + a.offW0 + static_cast<int64_t>(g0 + r) * D + col_begin;
-      // two of the warpgroup's tiles per pass: both tiles' loads are in flight together
-      for (int tt = eg; tt < nD; tt += 4) {
-        float v[2][32];
-  #pragma unroll
-        for (int h = 0; h < 2; ++h) {
-          const int c0 = (tt + 2 * h) * kND;
-  #pragma unroll
-          for (int q = 0; q < 8; ++q) {
-            const float4 x = c0 + 4 * q < ncols ? *reinterpret_cast<const float4*>(src + c0 + 4 * q)
-                                                : make_float4(0.f, 0.f, 0.f, 0.f);
-            v[h][4 * q] = x.x;
-            v[h][4 * q + 1] = x.y;
-            v[h][4 * q + 2] = x.z;
-            v[h][4 * q + 3] = x.w;
-          }
-        }
-  #pragma unroll
-        for (int h = 0; h < 2; ++h) {
-          const int c0 = (tt + 2 * h) * kND;
-          if (tt + 2 * h < nD) {
-            tmem_st_32x32b_x32(trow + c0, v[h]);
-            put_w0_row32(w0s, r, c0, v[h]);
-          }
-        }
-      }
-      tmem_wait_st();
-    } else {
+    // the global model, once per worker.  Warps 0-3: head columns and
+    // biases.  The fp32 master block comes by TMA in tiles of 128 rows x 32
+    // columns, up to kMaxKb at a time, into the resident-operand area (not in
+    // use yet); the epilogue warps move each row to TMEM.  Then the bf16
+    // operand itself comes by TMA from the global slot's bf16 copy (the
+    // round-to-nearest bf16 of the same values).  Columns past D are zero (TMA
+    // fill).
+    if (warp < 4) {
       for (int q = t; q < kFC * (UPC / 4); q += 128) {
         const int c = q / (UPC / 4), u4 = (q % (UPC / 4)) * 4;
         const float4 m = *reinterpret_cast<const float4*>(a.master + gso + a.offW1 + static_cast<int64_t>(c) * H + g0 +
@@ -365,6 +346,42 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
       for (int u = t; u < kFU; u += 128) b0m[u] = a.master[gso + a.offB0 + g0 + u];
       if (t < kFC) b1m[t] = a.master[gso + a.offB1 + t];
     }
+    for (int tb = 0; tb < nD; tb += kMaxKb) {
+      const int nb = nD - tb < kMaxKb ? nD - tb : kMaxKb;
+      if (t == 0) {
+        mbar_arrive_expect_tx(ldW, nb * kW0Blk);   // an fp32 tile has the size of a bf16 K-block
+        for (int i = 0; i < nb; ++i) tma_load_3d(w0s + i * kW0Blk, &mW0f, col_begin + (tb + i) * kND, g0, 0, ldW);
+      }
+      if (warp >= 4) {
+        const int quarter = warp & 3, eg = (warp - 4) >> 2;
+        const int r = quarter * 32 + lane;
+        const uint32_t trow = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
+        mbar_wait(ldW, ld_phase & 1, a.err, kDevTimeoutFull);
+        for (int i = eg; i < nb; i += 2) {
+          // row r of the tile: 128 bytes, 16-byte chunk q at (q ^ (r & 7))
+          const uint8_t* row = w0s + i * kW0Blk + r * 128;
+          float v[32];
+#pragma unroll
+          for (int q = 0; q < 8; ++q) {
+            const float4 x = *reinterpret_cast<const float4*>(row + ((q ^ (r & 7)) << 4));
+            v[4 * q] = x.x;
+            v[4 * q + 1] = x.y;
+            v[4 * q + 2] = x.z;
+            v[4 * q + 3] = x.w;
+          }
+          tmem_st_32x32b_x32(trow + (tb + i) * kND, v);
+        }
+        tmem_wait_st();
+      }
+      ++ld_phase;
+      __syncthreads();   // the tiles have been read before the area is written again
+    }
+    if (t == 0) {
+      mbar_arrive_expect_tx(ldW, nkf * kW0Blk);
+      for (int j = 0; j < nkf; ++j) tma_load_3d(w0s + j * kW0Blk, &mW0b, col_begin + j * kFBK, g0, 0, ldW);
+    }
+    mbar_wait(ldW, ld_phase & 1, a.err, kDevTimeoutFull);
+    ++ld_phase;
     fence_proxy_async_smem();   // the resident W0 is read by the tensor core
     tc_fence_before();
     __syncthreads();
@@ -389,7 +406,7 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
           tc_fence_after();
           const uint32_t wa = smem_u32(w0s + kb * kW0Blk);
           const uint32_t xb = smem_u32(fring + st * Cfg::kBBytes);
-  #pragma unroll
+#pragma unroll
           for (int j = 0; j < kFBK / 16; ++j)
             umma_bf16(tmem + kTAcc, smem_desc_k128(wa + j * 32), smem_desc_k128(xb + j * 32), idesc,
                       (kb | j) != 0 ? 1u : 0u);
@@ -411,14 +428,14 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
             tmem_ld_32x32b_x32(trow + c0, v);
             if (S == 1) {
               const float bias = b0m[u];
-  #pragma unroll
+#pragma unroll
               for (int j = 0; j < 32; ++j) hs[(c0 + j) * Cfg::kHsd + u] = bf16_round(fmaxf(v[j] + bias, 0.f));
             } else {
               // the partial goes to the CTA that keeps unit u: this one
               // (own rows) or, through the outgoing buffer, the partner
               const int owner = u / UPC;
               float* row = (owner == half ? zx : zout) + (u - owner * UPC) * Cfg::kZs + c0;
-  #pragma unroll
+#pragma unroll
               for (int q = 0; q < 8; ++q)
                 *reinterpret_cast<float4*>(row + 4 * q) =
                     make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
@@ -438,7 +455,7 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
         mbar_wait(pinF, sg & 1, a.err, kDevTimeoutFull);
         constexpr int kZItems = UPC * (B / 4), kZPer = (kZItems + kFT - 1) / kFT;
         float4 zr[kZPer];
-  #pragma unroll
+#pragma unroll
         for (int k = 0; k < kZPer; ++k) {
           const int q = t + k * kFT;
           if (q < kZItems) {   // item = (unit, 4 samples), consecutive threads on consecutive units
@@ -459,7 +476,7 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
           }
         }
         __syncthreads();   // the incoming partials (aliasing hs) have been read
-  #pragma unroll
+#pragma unroll
         for (int k = 0; k < kZPer; ++k) {
           const int q = t + k * kFT;
           if (q >= kZItems) break;
@@ -480,11 +497,11 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
       if (t < 256) {   // partial logits: kTpr threads per row, all classes in registers
         const int rb = t / Cfg::kTpr, q = t % Cfg::kTpr;
         float acc[kFC];
-  #pragma unroll
+#pragma unroll
         for (int c = 0; c < kFC; ++c) acc[c] = 0.f;
         for (int k = 4 * q; k < UPC; k += 4 * Cfg::kTpr) {
           const float4 hv = *reinterpret_cast<const float4*>(hs + rb * Cfg::kHsd + k);
-  #pragma unroll
+#pragma unroll
           for (int c = 0; c < kFC; ++c) {
             const float4 wv = *reinterpret_cast<const float4*>(wcs + c * UPC + k);
             acc[c] = fmaf(hv.x, wv.x, acc[c]);
@@ -493,7 +510,7 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
             acc[c] = fmaf(hv.w, wv.w, acc[c]);
           }
         }
-  #pragma unroll
+#pragma unroll
         for (int c = 0; c < kFC; ++c) {
           for (int o = Cfg::kTpr / 2; o > 0; o >>= 1) acc[c] += __shfl_xor_sync(0xffffffffu, acc[c], o);
           if (q == 0) pl[rb * kFC + c] = acc[c];
@@ -502,10 +519,10 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
       cluster_sync();
       for (int q = t; q < B * kFC; q += kFT) {
         float part[kFMaxCluster];
-  #pragma unroll
+#pragma unroll
         for (int r = 0; r < kFMaxCluster; ++r) part[r] = r < ncl ? ld_dsmem_f32(pl + q, r) : 0.f;
         float acc = 0.f;
-  #pragma unroll
+#pragma unroll
         for (int r = 0; r < kFMaxCluster; ++r)
           if (r < ncl) acc += part[r];
         dz[q] = acc + b1m[q % kFC];
@@ -523,16 +540,16 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
       if (t < 4 * B) {
         const int b = t >> 2, q = t & 3, src = lane & ~3;
         float zq[3], eq[3];
-  #pragma unroll
+#pragma unroll
         for (int i = 0; i < 3; ++i) zq[i] = q + 4 * i < kFC ? dz[b * kFC + q + 4 * i] : -INFINITY;
         float m = fmaxf(fmaxf(zq[0], zq[1]), zq[2]);
         m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 1));
         m = fmaxf(m, __shfl_xor_sync(0xffffffffu, m, 2));
-  #pragma unroll
+#pragma unroll
         for (int i = 0; i < 3; ++i) eq[i] = q + 4 * i < kFC ? expf(zq[i] - m) : 0.f;
         const int y = labs[b];
         float se = 0.f, so_ = 0.f;
-  #pragma unroll
+#pragma unroll
         for (int c = 0; c < kFC; ++c) {
           const float ec = __shfl_sync(0xffffffffu, eq[c >> 2], src | (c & 3));
           se += ec;
@@ -540,7 +557,7 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
         }
         if (q == (y & 3)) rowloss[b] = m + logf(se) - (y < 4 ? zq[0] : y < 8 ? zq[1] : zq[2]);
         const float inv = 1.0f / static_cast<float>(B);
-  #pragma unroll
+#pragma unroll
         for (int i = 0; i < 3; ++i) {
           const int c = q + 4 * i;
           if (c < kFC) {
@@ -563,7 +580,7 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
         float g = 0.f;
         if (c < kFC)
           for (int b = j; b < B; b += 8) g += dz[b * kFC + c];
-  #pragma unroll
+#pragma unroll
         for (int o = 4; o > 0; o >>= 1) g += __shfl_xor_sync(0xffffffffu, g, o, 8);
         if (j == 0 && c < kFC) {
           const float nb = fmaf(-a.lr, g, b1m[c]);
@@ -579,9 +596,9 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
         // dh[b] = sum over c in class order of dzb[c][b] w[c][u]: the eight
         // samples of a class are two 16-byte loads of the class-major dzb
         float dv[8];
-  #pragma unroll
+#pragma unroll
         for (int i = 0; i < 8; ++i) dv[i] = 0.f;
-  #pragma unroll
+#pragma unroll
         for (int c = 0; c < kFC; ++c) {
           const float wc = wcs[c * UPC + u];
           const float4 d0 = *reinterpret_cast<const float4*>(dzb + c * B + 8 * j);
@@ -596,7 +613,7 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
           dv[7] = fmaf(d1.w, wc, dv[7]);
         }
         float gsum = 0.f;
-  #pragma unroll
+#pragma unroll
         for (int i = 0; i < 8; ++i) {
           const float dh = hs[(8 * j + i) * Cfg::kHsd + u] > 0.f ? dv[i] : 0.f;
           dv[i] = dh;
@@ -606,7 +623,7 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
                                    pack_bf16x2(dv[6], dv[7]));
         uint8_t* dst = dzT + sw128_offset(ku0 + u, 8 * j);
         *reinterpret_cast<uint4*>(dst) = p;
-  #pragma unroll
+#pragma unroll
         for (int o = 0; o < S; ++o)
           if (o != half) st_dsmem_u32x4(dst, grp * S + o, p);
         gbp[j * UPC + u] = gsum;
@@ -620,11 +637,11 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
         const int item = q % Cfg::kW1Items, hb = q / Cfg::kW1Items;
         const int c = item / (UPC / 4), u4 = (item % (UPC / 4)) * 4;
         float4 dw = make_float4(0.f, 0.f, 0.f, 0.f);
-  #pragma unroll 2
+#pragma unroll 2
         for (int b4 = hb * (B / 2); b4 < (hb + 1) * (B / 2); b4 += 4) {
           const float4 g4 = *reinterpret_cast<const float4*>(dzb + c * B + b4);   // samples b4 .. b4 + 3
           const float gk[4] = {g4.x, g4.y, g4.z, g4.w};
-  #pragma unroll
+#pragma unroll
           for (int k = 0; k < 4; ++k) {
             const float4 hv = *reinterpret_cast<const float4*>(hs + (b4 + k) * Cfg::kHsd + u4);
             dw.x = fmaf(gk[k], hv.x, dw.x);
@@ -637,7 +654,7 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
       }
       if (t < UPC) {   // b0 of this CTA's units (chunk sums in chunk order)
         float g = 0.f;
-  #pragma unroll
+#pragma unroll
         for (int r = 0; r < Cfg::kChunks; ++r) g += gbp[r * UPC + t];
         const float nb = fmaf(-a.lr, g, b0m[ku0 + t]);
         b0m[ku0 + t] = nb;
@@ -692,7 +709,7 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
               const uint32_t xa = smem_u32(dring + xb * Cfg::kXtBytes);
               const uint32_t da = smem_u32(dzT);
               const uint32_t dcol = tmem + static_cast<uint32_t>(kTAcc + buf * kND);
-  #pragma unroll
+#pragma unroll
               for (int j = 0; j < kFBK / 16; ++j)
                 umma_bf16(dcol, smem_desc_k128(da + j * 32), smem_desc_k128(xa + j * 32), idesc, j != 0 ? 1u : 0u);
             }
@@ -719,7 +736,7 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
             tmem_ld_32x32b_x32_pair(trow + kTAcc + buf * kND, g, trow + c0, m);
             tc_fence_before();
             bar_arrive_named(1 + eg, 128 + 32);   // the gradient buffer has been read: the next MMA may reuse it
-  #pragma unroll
+#pragma unroll
             for (int j = 0; j < 32; ++j) m[j] = fmaf(-a.lr, g[j], m[j]);
             tmem_st_32x32b_x32(trow + c0, m);
             put_w0_row32(w0s, r, c0, m);
@@ -749,13 +766,13 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
         const int c0 = tt * kND;
         float m[32];
         tmem_ld_32x32b_x32(trow + c0, m);
-  #pragma unroll
+#pragma unroll
         for (int q = 0; q < 8; ++q)
           *reinterpret_cast<float4*>(T + lane * 36 + 4 * q) =
               make_float4(m[4 * q], m[4 * q + 1], m[4 * q + 2], m[4 * q + 3]);
         __syncwarp();
         if (c0 + cq < ncols) {
-  #pragma unroll
+#pragma unroll
           for (int i = 0; i < 8; ++i) {
             const int rr = 4 * i + (lane >> 3);
             *reinterpret_cast<float4*>(dst + static_cast<int64_t>(rr) * D + c0 + cq) =
@@ -787,8 +804,8 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
 }
 
 template <int B, int S>
-cudaError_t launch_bs(const CUtensorMap& mX, const CUtensorMap& mXT, const FusedArgs& a, int priority,
-                      cudaStream_t s) {
+cudaError_t launch_bs(const CUtensorMap& mX, const CUtensorMap& mXT, const CUtensorMap& mW0f, const CUtensorMap& mW0b,
+                      const FusedArgs& a, int priority, cudaStream_t s) {
   using Cfg = FCfg<B, S>;
   cudaError_t e = cudaFuncSetAttribute(fused_mlp2_round_kernel<B, S>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        Cfg::kSmem);
@@ -812,7 +829,7 @@ cudaError_t launch_bs(const CUtensorMap& mX, const CUtensorMap& mXT, const Fused
   }
   cfg.attrs = attr;
   cfg.numAttrs = n;
-  return cudaLaunchKernelEx(&cfg, fused_mlp2_round_kernel<B, S>, mX, mXT, a);
+  return cudaLaunchKernelEx(&cfg, fused_mlp2_round_kernel<B, S>, mX, mXT, mW0f, mW0b, a);
 }
 
 // two CTAs per unit group when the cluster stays within 8 CTAs and the input
@@ -876,7 +893,8 @@ int fused_round_max_clusters(int D, int H, int B) {
   return 0;
 }
 
-cudaError_t launch_fused_round(const CUtensorMap& mX, const CUtensorMap& mXT, const FusedRoundArgs& r, cudaStream_t s) {
+cudaError_t launch_fused_round(const CUtensorMap& mX, const CUtensorMap& mXT, const CUtensorMap& mW0f,
+                               const CUtensorMap& mW0b, const FusedRoundArgs& r, cudaStream_t s) {
   FusedArgs a;
   a.tau = r.tau;
   a.order = r.order;
@@ -903,9 +921,11 @@ cudaError_t launch_fused_round(const CUtensorMap& mX, const CUtensorMap& mXT, co
   a.shard_n = r.shard_n;
   const int S = split_for(r.D, r.H);
   if (r.B == 32)
-    return S == 2 ? launch_bs<32, 2>(mX, mXT, a, r.priority, s) : launch_bs<32, 1>(mX, mXT, a, r.priority, s);
+    return S == 2 ? launch_bs<32, 2>(mX, mXT, mW0f, mW0b, a, r.priority, s)
+                  : launch_bs<32, 1>(mX, mXT, mW0f, mW0b, a, r.priority, s);
   if (r.B == 64)
-    return S == 2 ? launch_bs<64, 2>(mX, mXT, a, r.priority, s) : launch_bs<64, 1>(mX, mXT, a, r.priority, s);
+    return S == 2 ? launch_bs<64, 2>(mX, mXT, mW0f, mW0b, a, r.priority, s)
+                  : launch_bs<64, 1>(mX, mXT, mW0f, mW0b, a, r.priority, s);
   return cudaErrorInvalidValue;
 }
 
