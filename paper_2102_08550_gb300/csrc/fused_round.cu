@@ -14,7 +14,9 @@
 // the forward GEMM, in shared memory (K-major, 128-byte swizzled K-blocks).
 // Its head-weight columns, its b0 entries and a private copy of the head
 // bias (updated identically by every CTA) live in shared memory.  The model
-// is read from the global slot once, before the first step, and the worker's
+// is read from the global slot once, before the first step (the W0 block by
+// TMA: fp32 tiles staged in shared memory on their way to TMEM, the bf16
+// operand from the global slot's bf16 copy), and the worker's
 // replica is written once, after the last step (the W0 block through a
 // per-warp shared-memory transpose, so that every store instruction writes
 // whole 128-byte lines).  Per step only the mini-batch (staged bf16 X and X^T
