@@ -336,6 +336,9 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
     // operand itself comes by TMA from the global slot's bf16 copy (the
     // round-to-nearest bf16 of the same values).  Columns past D are zero (TMA
     // fill).
+    // the first X tiles of step 0 go out first (the F ring is free: the
+    // previous worker's write-back has read it before the last barrier)
+    if (warp == 0 && lane == 0) producer_ok = issue_f(0, 0, pre_f);
     if (warp < 4) {
       for (int q = t; q < kFC * (UPC / 4); q += 128) {
         const int c = q / (UPC / 4), u4 = (q % (UPC / 4)) * 4;
@@ -388,7 +391,6 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    if (warp == 0 && lane == 0) producer_ok = issue_f(0, 0, pre_f);
 
     for (int s = 0; s < tau; ++s) {
       if (stamp) a.phase_ts[s * 4 + 0] = global_ns();
