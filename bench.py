@@ -29,6 +29,7 @@ import json
 import os
 import subprocess
 import sys
+import tempfile
 import time
 
 ROOT = os.path.dirname(os.path.abspath(__file__))
@@ -102,7 +103,9 @@ class ClockSampler:
     def __init__(self, index: int):
         self.index = index
         self.proc = None
-        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_{os.getpid()}.csv")
+        # raw samples (the JSON line carries their summary); OSCARS_CLOCK_LOG_DIR keeps them elsewhere
+        log_dir = os.environ.get("OSCARS_CLOCK_LOG_DIR", tempfile.gettempdir())
+        self.path = os.path.join(log_dir, f"oscars_clocks_{os.getpid()}.csv")
 
     def __enter__(self):
         if self.index < 0:                # sampling off
