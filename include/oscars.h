@@ -366,6 +366,24 @@ oscars_status oscars_partition_sizes(const int64_t* weight, int32_t n, int64_t t
                                      int64_t* sizes);
 
 /*
+ * oscars_round_clusters - the worker lists of the one-launch round kernel
+ * (one thread-block cluster per worker, the worker's model on chip; Eq. 4,
+ * "otherwise" branch) when fewer of its clusters fit on the device than there
+ * are workers.  tau[n] (host, >= 1): the local steps of each worker this
+ * round; max_clusters: the clusters that fit at once (<= 0 or >= n: one
+ * cluster per worker).  Workers by decreasing tau (ties by index) go, one at
+ * a time, to the cluster with the least work so far (ties to the lower
+ * cluster), a worker costing tau + 1/2 (its steps and about half a step of
+ * model load): longest processing time first.  order[n] (host) receives the
+ * workers cluster by cluster, first[] (host, room for n + 1) the start of
+ * each cluster's run in order plus the end, *clusters their number; a
+ * cluster runs its workers one after the other.  Errors: EINVAL (NULL,
+ * n < 1, a tau < 1).
+ */
+oscars_status oscars_round_clusters(const int32_t* tau, int32_t n, int32_t max_clusters, int32_t* order,
+                                    int32_t* first, int32_t* clusters);
+
+/*
  * oscars_merge - the server update of Eq. 4 (first branch) on caller buffers,
  * without a context: x_g[p] <- x_g[p] + server_lr * sum_k w[k] * deltas[k][p]
  * for p < P.  x_g: device, P fp32, updated in place.  deltas: host array of W

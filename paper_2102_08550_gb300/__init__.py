@@ -80,6 +80,8 @@ _SIGS = {
     "oscars_policy_local_steps": (c_int32, [c_int32, POINTER(c_int64), c_int32, c_int64, c_int32, c_int32,
                                             POINTER(c_int32), POINTER(c_int64)]),
     "oscars_partition_sizes": (c_int32, [POINTER(c_int64), c_int32, c_int64, c_int64, POINTER(c_int64)]),
+    "oscars_round_clusters": (c_int32, [POINTER(c_int32), c_int32, c_int32, POINTER(c_int32), POINTER(c_int32),
+                                        POINTER(c_int32)]),
     "oscars_train": (c_int32, [c_void_p, c_int32, c_void_p, c_void_p, c_int64, c_float, POINTER(OscarsRoundLog),
                                POINTER(c_int32)]),
     "oscars_merge": (c_int32, [c_void_p, POINTER(c_void_p), POINTER(c_float), c_int32, c_int64, c_float, c_void_p]),
@@ -150,6 +152,14 @@ def oscars_partition_sizes(weight: Sequence[int], total: int, unit: int = 1):
     out = (c_int64 * n)()
     _check(lib().oscars_partition_sizes(_arr(c_int64, weight), n, total, unit, out))
     return list(out)
+
+
+def oscars_round_clusters(tau: Sequence[int], max_clusters: int):
+    """Worker lists of the one-launch round kernel: a list of workers per cluster."""
+    n = len(tau)
+    order, first, ncl = (c_int32 * n)(), (c_int32 * (n + 1))(), c_int32()
+    _check(lib().oscars_round_clusters(_arr(c_int32, tau), n, max_clusters, order, first, ctypes.byref(ncl)))
+    return [list(order[first[k]:first[k + 1]]) for k in range(ncl.value)]
 
 
 def oscars_train(ctx: int, rounds: int, eval_x_ptr: Optional[int] = None, eval_y_ptr: Optional[int] = None,

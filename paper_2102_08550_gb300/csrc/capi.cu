@@ -525,28 +525,14 @@ oscars_status build_tables(oscars_ctx* c) {
   if (e == cudaSuccess) e = cudaMemcpy(c->tau_dev, c->tau.data(), c->W * sizeof(int32_t), cudaMemcpyHostToDevice);
   if (e == cudaSuccess) {
     // Round-kernel clusters: one per worker when they all fit on the device,
-    // else as many as fit, each running its workers one after the other.
-    // Workers by decreasing tau (ties by index) go to the cluster with the
-    // least work so far (longest processing time first; a worker costs its
-    // tau steps plus about half a step of model load).
-    std::vector<int32_t> ord(c->W);
-    for (int i = 0; i < c->W; ++i) ord[i] = i;
-    std::stable_sort(ord.begin(), ord.end(), [&](int32_t x, int32_t y) { return c->tau[x] > c->tau[y]; });
-    const int ncl = c->fused_max_clusters > 0 && c->fused_max_clusters < c->W ? c->fused_max_clusters : c->W;
-    std::vector<std::vector<int32_t>> lists(ncl);
-    std::vector<double> load(ncl, 0.0);
-    for (int32_t wk : ord) {
-      int k = 0;
-      for (int j = 1; j < ncl; ++j)
-        if (load[j] < load[k]) k = j;
-      lists[k].push_back(wk);
-      load[k] += c->tau[wk] + 0.5;
-    }
-    std::vector<int32_t> flat, first(1, 0);
-    for (const auto& l : lists) {
-      flat.insert(flat.end(), l.begin(), l.end());
-      first.push_back(static_cast<int32_t>(flat.size()));
-    }
+    // else as many as fit, each running its workers one after the other
+    // (longest processing time first: oscars_round_clusters)
+    std::vector<int32_t> flat(c->W), first(static_cast<size_t>(c->W) + 1);
+    int32_t ncl = 0;
+    if (oscars_round_clusters(c->tau.data(), c->W, c->fused_max_clusters, flat.data(), first.data(), &ncl) !=
+        OSCARS_OK)
+      return fail(c, OSCARS_EINVAL, "round cluster plan");
+    first.resize(static_cast<size_t>(ncl) + 1);
     c->n_clusters = ncl;
     if (!c->order_dev && !dev_alloc(c, &c->order_dev, c->W))
       return fail(c, OSCARS_ENOMEM, "device allocation failed (worker order)");

@@ -193,6 +193,37 @@ oscars_status oscars_partition_sizes(const int64_t* weight, int32_t n, int64_t t
   return OSCARS_OK;
 }
 
+oscars_status oscars_round_clusters(const int32_t* tau, int32_t n, int32_t max_clusters, int32_t* order,
+                                    int32_t* first, int32_t* clusters) {
+  if (!tau || !order || !first || !clusters || n < 1) return OSCARS_EINVAL;
+  for (int i = 0; i < n; ++i)
+    if (tau[i] < 1) return OSCARS_EINVAL;
+  std::vector<int32_t> ord(n);
+  for (int i = 0; i < n; ++i) ord[i] = i;
+  std::stable_sort(ord.begin(), ord.end(), [&](int32_t x, int32_t y) { return tau[x] > tau[y]; });
+  const int ncl = max_clusters > 0 && max_clusters < n ? max_clusters : n;
+  // longest processing time first: each worker to the cluster with the least
+  // work so far (a worker costs tau + 1/2: its steps and about half a step of
+  // model load; half-integers are exact in a double)
+  std::vector<std::vector<int32_t>> lists(ncl);
+  std::vector<double> load(ncl, 0.0);
+  for (int32_t w : ord) {
+    int k = 0;
+    for (int j = 1; j < ncl; ++j)
+      if (load[j] < load[k]) k = j;
+    lists[k].push_back(w);
+    load[k] += tau[w] + 0.5;
+  }
+  int at = 0;
+  first[0] = 0;
+  for (int k = 0; k < ncl; ++k) {
+    for (int32_t w : lists[k]) order[at++] = w;
+    first[k + 1] = at;
+  }
+  *clusters = ncl;
+  return OSCARS_OK;
+}
+
 const char* oscars_status_string(int32_t s) {
   switch (s) {
     case OSCARS_OK: return "OSCARS_OK";
