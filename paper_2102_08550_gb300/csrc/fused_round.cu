@@ -2,7 +2,7 @@
 // ReLU units -> 10 classes) in ONE launch (Eq. 4, "otherwise" branch: each
 // worker runs tau_i SGD steps from the global model).
 //
-// One thread-block cluster serves one worker.  The hidden units come in
+// One thread-block cluster serves one worker at a time.  The hidden units come in
 // groups of 128 (one tensor-core tile of rows); each group is served by S
 // CTAs (S = 1 or 2) that split the INPUT dimension: CTA h of the group owns
 // input columns [c_h, c_{h+1}) of the group's 128 rows of W0 (a split on a
