@@ -85,16 +85,26 @@ def peaks():
     return 6800.0, 1900.0, 1700.0, "fallback"
 
 
-def schedule_of(w):
-    from oracle import schedule as S  # schedule inputs only; not timed
-    t = S.iteration_ticks(synth.speeds(w), w.ticks_per_unit)
-    return S.schedule(t, w.M)
+# how the GPU arm keeps timed rounds from reusing L2 (the same string in both
+# arms, so that their config dicts are identical)
+L2_NOTE = "GPU arm: L2 flushed between timed rounds (512 MB write)"
+L2_NOTE_MERGE = "inputs larger than L2 (6.8 and 13.6 GB per launch)"
 
 
-def workload_config(w, l2):
+def library_schedule(w):
+    """T*, max wait and tau of the library's own scheduler (Algorithm 1 in
+    the C ABI), for the workload's speeds."""
+    import paper_2102_08550_gb300 as P
+    t = P.oscars_iteration_ticks(synth.speeds(w).tolist(), w.ticks_per_unit)
+    T, mw, tau = P.oscars_schedule_solve(t, w.M)
+    return int(T), int(mw), np.asarray(tau, np.int64)
+
+
+def workload_config(w, l2=L2_NOTE):
+    speeds = "speeds {" + ", ".join(f"{v:g}" for v in w.speeds) + "}" if w.speeds else "lognormal(0,0.5) speeds"
     return {"workload": f"{w.name} (W={w.num_workers}, dims={'-'.join(map(str, w.dims))}, batch={w.batch}, "
-                        f"M={w.M}, lognormal(0,0.5) speeds)",
-            "W": w.num_workers, "dims": w.dims, "batch": w.batch, "M": w.M, "lr": w.lr,
+                        f"M={w.M}, {speeds})",
+            "W": w.num_workers, "batch": w.batch, "M": w.M, "lr": w.lr,
             "samples_per_worker": w.samples_per_worker, "l2": l2}
 
 
@@ -185,6 +195,9 @@ def algorithmic_work(w, tau):
     add("head_bwd", n * 4 * B * H * C,
         n * (B * H * 2 + C * H * (2 + 4 + 4 + 2) + 2 * B * H * 2 + H * 4 + B * C * 4 + C * 8))
     add("stage", 0.0, n * B * (d[0] * 4 + 2 * d[0] * 2 + 8))
+    # the fused last layer of the per-layer path does the head's forward and
+    # backward in one launch
+    fl["head_fused"], by["head_fused"] = fl["head_fwd"] + fl["head_bwd"], by["head_fwd"] + by["head_bwd"]
     # the one-launch round of a 2-layer model does all of the above per step
     # and keeps each worker's model on chip for the round: its work is the sum
     # of the parts, its compulsory bytes the global model read once (the
@@ -231,6 +244,11 @@ def alu_peak_tflops():
 
 
 def roofline_of(name, ms_per_launch, launches_per_round, flops, bytes_, hbm, tflops, peak_kind, workload=None):
+    """Roofline of one kernel class from its algorithmic work per launch and
+    its measured duration per launch.  ``bound`` is the roof that binds at
+    that work (the larger of flops / bf16 peak and bytes / HBM peak);
+    tensor-core kernels also report ``tensor_frac`` (their FLOP rate over the
+    bf16 peak) beside an HBM bound, and ``hbm_frac`` beside a tensor bound."""
     f = flops.get(name, 0.0) / launches_per_round
     b = bytes_.get(name, 0.0) / launches_per_round
     t = ms_per_launch / 1e3
@@ -247,16 +265,19 @@ def roofline_of(name, ms_per_launch, launches_per_round, flops, bytes_, hbm, tfl
     t_mem = b / (hbm * 1e9)
     tr = NCU_TRAFFIC.get((name, workload))
     traffic = tr[0] if tr else None
+    tensor_frac = f / t / 1e12 / tflops if name in TENSOR_KERNELS and f > 0.0 else None
     if t_flop >= t_mem:
         ach = f / t / 1e12
         return {"kernel": name, "bound": "tensor", "achieved": ach, "peak": tflops, "unit": "TFLOP/s",
-                "frac": ach / tflops, "peak_kind": f"{peak_kind} bf16 dense (sustained)", "flops_per_launch": f,
-                "bytes_per_launch": b, "ms_per_launch": ms_per_launch, "traffic": traffic}
+                "frac": ach / tflops, "peak_kind": f"{peak_kind} bf16 dense (burst)", "flops_per_launch": f,
+                "bytes_per_launch": b, "ms_per_launch": ms_per_launch, "traffic": traffic,
+                "traffic_source": tr[1] if tr else None, "hbm_frac": b / t / 1e9 / hbm}
     ach = b / t / 1e9
     return {"kernel": name, "bound": "hbm", "achieved": ach, "peak": hbm, "unit": "GB/s", "frac": ach / hbm,
             "peak_kind": f"{peak_kind} HBM copy", "flops_per_launch": f, "bytes_per_launch": b,
             "ms_per_launch": ms_per_launch, "traffic": traffic,
-            "traffic_source": tr[1] if tr else None}
+            "traffic_source": tr[1] if tr else None, "tensor_frac": tensor_frac,
+            "tensor_peak": tflops if tensor_frac is not None else None}
 
 
 def max_over_ranks(ms: float, world: int, device) -> float:
@@ -282,8 +303,6 @@ def measure_rounds(w, steps, warmup, dev, world=1, local_rank=0, flush=None, clo
     import torch
     import paper_2102_08550_gb300 as P
     hbm, tf_burst, tf_sus, peak_kind = peaks()
-    T_star, mw, tau = schedule_of(w)
-    samples_per_round = int(np.sum(tau)) * w.batch
     shards = [synth.shard_t(w, k, dev) for k in range(w.num_workers)]
     layers0 = synth.init_layers_np(w)
     init = torch.from_numpy(synth.flatten_layers(layers0)).to(dev)
@@ -295,6 +314,10 @@ def measure_rounds(w, steps, warmup, dev, world=1, local_rank=0, flush=None, clo
                                stream=stream.cuda_stream, flags=flags)
 
     ctx = make()
+    sch = ctx.schedule()                 # what the library runs: its own Algorithm 1
+    tau = np.asarray(sch["tau"], np.int64)
+    T_star = sch["T_star"]
+    samples_per_round = int(np.sum(tau)) * w.batch
     if flush is None:
         flush = torch.empty(512 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)   # > L2 (129 MB)
 
@@ -344,20 +367,20 @@ def measure_rounds(w, steps, warmup, dev, world=1, local_rank=0, flush=None, clo
     kernels = {}
     tot = sum(x[0] for x in prof.values())
     for k, (ms, cnt) in prof.items():
-        r = roofline_of(k, ms / cnt, cnt / prof_rounds, flops, bytes_, hbm, tf_sus, peak_kind)
+        r = roofline_of(k, ms / cnt, cnt / prof_rounds, flops, bytes_, hbm, tf_burst, peak_kind)
         kernels[k] = {"ms_per_round": ms / prof_rounds, "launches_per_round": cnt / prof_rounds,
                       "share": ms / tot, "bound": r["bound"], "frac": r["frac"]}
         if k in TENSOR_KERNELS and flops.get(k, 0.0) > 0.0:   # tensor-core work: its fraction of the tensor peak
             tf = flops[k] / (ms / prof_rounds / 1e3) / 1e12
             kernels[k]["tflops"] = tf
-            kernels[k]["tensor_frac"] = tf / tf_sus
-    gemm = [k for k in kernels if k.startswith("gemm_")]
+            kernels[k]["tensor_frac"] = tf / tf_burst
+    gemm = [k for k in kernels if k.startswith("gemm_") or k == "head_fused"]
     if gemm:                            # the grouped worker GEMMs together
         g_ms = sum(prof[k][0] for k in gemm) / prof_rounds
-        g_tf = sum(flops[k] for k in gemm) / (g_ms / 1e3) / 1e12
+        g_tf = sum(flops.get(k, 0.0) for k in gemm) / (g_ms / 1e3) / 1e12
         kernels["all_gemms"] = {"ms_per_round": g_ms, "share": g_ms * prof_rounds / tot, "tflops": g_tf,
-                                "tensor_frac": g_tf / tf_sus}
-    roof = roofline_of(dom, prof[dom][0] / prof[dom][1], prof[dom][1] / prof_rounds, flops, bytes_, hbm, tf_sus,
+                                "tensor_frac": g_tf / tf_burst}
+    roof = roofline_of(dom, prof[dom][0] / prof[dom][1], prof[dom][1] / prof_rounds, flops, bytes_, hbm, tf_burst,
                        peak_kind, w.name)
     return {"value": value, "ms_per_step": total_ms / steps, "roofline": roof, "kernels": kernels,
             "gpu_launches": int(round(launches_per_round * steps)), "clocks": clk.summary() if clock else None,
@@ -365,7 +388,7 @@ def measure_rounds(w, steps, warmup, dev, world=1, local_rank=0, flush=None, clo
 
 
 # kernel classes whose FLOPs run on the tensor cores (tcgen05)
-TENSOR_KERNELS = ("gemm_fwd", "gemm_dh", "gemm_dw_sgd", "fused_round")
+TENSOR_KERNELS = ("gemm_fwd", "gemm_dh", "gemm_dw_sgd", "head_fused", "fused_round")
 
 # the training workloads measured beside the headline (absolute samples/s and
 # the roofline of their dominant kernel)
@@ -377,10 +400,16 @@ def run_side_workloads(args, dev):
     out = {}
     for w in SIDE_WORKLOADS:
         r = measure_rounds(w, max(20, args.steps), max(3, args.warmup), dev, clock=False, prof_rounds=3)
+        e2e = None
+        if not args.no_e2e:
+            shards = [synth.shard_t(w, k, dev) for k in range(w.num_workers)]
+            e2e = run_e2e(args, shards, w, np.asarray(r["tau"]), dev, torch.cuda.current_stream(dev))
+            del shards
         out[w.name] = {"metric": "simulated-worker samples/s", "value": r["value"], "unit": UNIT,
-                       "ms_per_round": r["ms_per_step"], "config": workload_config(w, "flushed between timed rounds"),
+                       "ms_per_round": r["ms_per_step"], "config": workload_config(w),
                        "dtype": "bf16 (fp32 master, fp32 accumulate)" if w.bf16 else "f32",
-                       "roofline": r["roofline"], "kernels": r["kernels"], "samples_per_round": r["samples_per_round"]}
+                       "roofline": r["roofline"], "kernels": r["kernels"], "samples_per_round": r["samples_per_round"],
+                       "e2e": e2e}
         torch.cuda.empty_cache()
     return out
 
@@ -396,7 +425,6 @@ def run_gpu(args, rank, world, local_rank):
     if args.samples_per_worker:
         w = dataclasses.replace(w, samples_per_worker=args.samples_per_worker)
     hbm, tf_burst, tf_sus, peak_kind = peaks()
-    T_star, mw, tau = schedule_of(w)
     stream = torch.cuda.current_stream(dev)
     res = measure_rounds(w, args.steps, args.warmup, dev, world, local_rank)
 
@@ -404,7 +432,7 @@ def run_gpu(args, rank, world, local_rank):
     e2e = None
     if not args.no_e2e:
         shards = [synth.shard_t(w, k, dev) for k in range(w.num_workers)]
-        e2e = run_e2e(args, shards, w, tau, dev, stream, world)
+        e2e = run_e2e(args, shards, w, np.asarray(res["tau"]), dev, stream, world)
         del shards
         torch.cuda.empty_cache()
 
@@ -425,7 +453,7 @@ def run_e2e(args, shards, w, tau, dev, stream, world=1):
     host = [(x.cpu().pin_memory(), y.cpu().pin_memory()) for x, y in shards]
     layers0 = synth.init_layers_np(w)
     init = torch.from_numpy(synth.flatten_layers(layers0)).pin_memory()
-    ctx = P.OscarsContext(num_workers=w.num_workers, dims=w.dims, batch=w.batch, lr=w.lr,
+    ctx = P.OscarsContext(num_workers=w.num_workers, dims=w.dims, batch=w.batch, lr=w.lr, bf16=w.bf16,
                           speed=synth.speeds(w).tolist(), M=w.M, shards=host, init_params=init,
                           stream=stream.cuda_stream)
     # warm-up: one full pass over every shard.  The first touch of each
@@ -451,11 +479,8 @@ def run_e2e(args, shards, w, tau, dev, stream, world=1):
     return {"value": whole_job_rate(samples * steps, world, dt * 1e3), "unit": UNIT, "h2d_bytes_per_step": h2d,
             "d2h_bytes_per_step": 4 * w.num_workers, "steps": steps, "warmup_rounds": epoch,
             "first_pass_value": first_pass,
-            "note": "host wall clock around one oscars_train call; shards in pinned host memory read by the "
-                    "staging kernel each round (host->device), local steps + merge, every round's per-worker "
-                    "losses copied to pinned host memory and read by the host (rounds pipelined one deep in the "
-                    "library); timed after one warm-up pass over every shard (first_pass_value: that pass, "
-                    "including the first touch of every pinned page)"}
+            "note": "one oscars_train call, host wall clock; shards in pinned host memory, read by the staging "
+                    "kernel; losses read back every round"}
 
 
 def merge_workloads(args):
@@ -466,6 +491,15 @@ def merge_workloads(args):
         Pn, W = (int(v) for v in item.split(":"))
         out.append(synth.MergeWorkload(f"merge-P{Pn}-W{W}", W, Pn, 1e-3, 8, "localsteps"))
     return out
+
+
+# DRAM bytes per algorithmic byte of the merge kernel, from ncu captures of
+# smaller launches of the same kernel with the same worker count (the
+# full-size launches are too large to capture; traffic grows in proportion to
+# P): (dram__bytes_read.sum + dram__bytes_write.sum) / ((W + 2) * P * 4).
+MERGE_TRAFFIC = {
+    64: (0.99621, "profiles/merge_vec4_P4M_W64.md (P = 4M, scaled by P)"),
+}
 
 
 def run_merge(args, dev, stream, hbm, peak_kind):
@@ -496,14 +530,40 @@ def run_merge(args, dev, stream, hbm, peak_kind):
         med = ts[len(ts) // 2]
         alg = (W + 2) * Pn * 4.0
         gbs = alg / (med / 1e3) / 1e9
+        tr = MERGE_TRAFFIC.get(W)
         res[m.name] = {"GB/s": gbs, "frac": gbs / hbm, "ms_median": med, "ms_min": ts[0],
                        "bytes_per_launch": alg, "weight_rule": m.weight_rule,
-                       "peak": hbm, "peak_kind": f"{peak_kind} HBM copy", "bound": "hbm", "traffic": None,
-                       "l2": "inputs larger than L2"}
+                       "peak": hbm, "peak_kind": f"{peak_kind} HBM copy", "bound": "hbm",
+                       "traffic": tr[0] * alg if tr else None, "traffic_source": tr[1] if tr else None,
+                       "launches": args.merge_reps, "l2": L2_NOTE_MERGE}
         ctx.close()
         del deltas
         torch.cuda.empty_cache()
     return res
+
+
+def merge_cpu_baseline(m, dev, budget_s=8.0):
+    """The oracle merge (fp64 sum in worker order) on the host cores over a
+    bounded prefix of the parameter vector: GB/s of (W + 2) * P_sample * 4
+    algorithmic bytes.  The inputs are drawn on the GPU (untimed)."""
+    from oracle import merge as omerge
+    from oracle import schedule as S
+    n = 1 << 20 if m.num_workers > 16 else 1 << 22
+    xg = synth.merge_xg_t(m, 0, n, dev).cpu().numpy()
+    deltas = [synth.merge_delta_t(m, k, 0, n, dev).cpu().numpy() for k in range(m.num_workers)]
+    w = S.merge_weights(m.weight_rule, synth.merge_taus(m))
+    omerge.merge_deltas(xg, deltas, w, m.server_lr)          # warm-up
+    t0 = time.perf_counter()
+    reps = 0
+    while True:
+        omerge.merge_deltas(xg, deltas, w, m.server_lr)
+        reps += 1
+        if time.perf_counter() - t0 > budget_s:
+            break
+    dt = time.perf_counter() - t0
+    return {"value": (m.num_workers + 2) * n * 4.0 * reps / dt / 1e9, "unit": "GB/s", "cores": cores_used(),
+            "kind": "oracle", "sample": f"{reps} merges of the first {n} of {m.num_params} parameters, "
+                                        f"W={m.num_workers} (numpy fp64)"}
 
 
 # ------------------------------------------------------------------ CPU oracle
@@ -657,16 +717,13 @@ def run_cnn(args, dev):
     roofline of its convolution kernels."""
     import torch
     import paper_2102_08550_gb300 as P
-    from oracle import schedule as S   # schedule inputs only; not timed
     w = synth.CFG6
     hbm, tf_burst, tf_sus, peak_kind = peaks()
-    t = S.iteration_ticks(synth.speeds(w), w.ticks_per_unit)
-    T_star, mw, tau = S.schedule(t, w.M)
+    T_star, mw, tau = library_schedule(w)
     samples_per_round = int(np.sum(tau)) * w.batch
     shards = [synth.shard_t(w, k, dev) for k in range(w.num_workers)]
-    from oracle import conv as oconv
-    m = oconv.CNN(w.height, w.width, w.in_ch, w.ch, w.blocks, w.dims[-1])
-    init = torch.from_numpy(m.flatten(synth.init_cnn_np(w))).to(dev)
+    # canonical layout: the tensors one after the other
+    init = torch.from_numpy(np.concatenate([p.reshape(-1) for p in synth.init_cnn_np(w)]).astype(np.float32)).to(dev)
     stream = torch.cuda.current_stream(dev)
 
     def make(flags=0):
@@ -742,11 +799,62 @@ def run_reference(args):
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
             "steps": done, "warmup": args.warmup, "ms_per_step": dt / done * 1e3, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64 (bf16 operand emulation)", "data": "synthetic",
-            "config": workload_config(w, "n/a (CPU)"),
+            "config": workload_config(w),
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": cores_used(), "kind": "oracle",
                              "sample": f"{done} Oscars rounds of {w.name} (numpy fp64, BLAS threads = all cores)"},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line))
+
+
+def training_cpu_baseline(w, rounds, budget_s):
+    samples, dt, done = oracle_rounds(w, rounds, budget_s)
+    return {"value": samples / dt, "unit": UNIT, "cores": cores_used(), "kind": "oracle",
+            "sample": f"{done} Oscars rounds of {w.name} (numpy fp64" +
+                      (" with bf16 operand emulation)" if w.bf16 else ")")}
+
+
+ROOF_KEYS = ("kernel", "bound", "achieved", "peak", "unit", "frac", "traffic", "ms_per_launch", "tensor_frac",
+             "hbm_frac")
+
+
+def config_records(res, cpus):
+    """Every workload of the run by name: its throughput, the roofline of its
+    dominant kernel, its oracle baseline and (training) its end-to-end rate."""
+    roof, cpu, e2e = {}, {}, {}
+    for name, r in (res.get("workloads") or {}).items():
+        roof[name] = {k: r["roofline"].get(k) for k in ROOF_KEYS if r["roofline"].get(k) is not None}
+        roof[name]["samples_per_s"] = r["value"]
+        if r.get("e2e"):
+            e2e[name] = {k: r["e2e"][k] for k in ("value", "unit", "h2d_bytes_per_step", "d2h_bytes_per_step")}
+    for name, m in (res.get("merge") or {}).items():
+        roof[name] = {"kernel": "merge_vec4", "bound": "hbm", "achieved": m["GB/s"], "peak": m["peak"],
+                      "unit": "GB/s", "frac": m["frac"], "traffic": m["traffic"], "ms_per_launch": m["ms_median"]}
+    for name, c in cpus.items():
+        cpu[name] = c
+    return roof, cpu, e2e
+
+
+def result_line(args, world, w, res, cpu, cpus):
+    roof, cpu_cfg, e2e_cfg = config_records(res, cpus)
+    top_roof = dict(res["roofline"])
+    head = {k: top_roof.get(k) for k in ROOF_KEYS if top_roof.get(k) is not None}
+    head["samples_per_s"] = res["value"]
+    top_roof["configs"] = {w.name: head, **roof}
+    cpu_line = dict(cpu) if cpu else None
+    if cpu_line is not None:
+        cpu_line["configs"] = {w.name: dict(cpu), **cpu_cfg}
+    e2e_line = dict(res["e2e"]) if res["e2e"] else None
+    if e2e_line is not None:
+        e2e_line["configs"] = {w.name: {k: res["e2e"][k] for k in ("value", "unit", "h2d_bytes_per_step",
+                                                                  "d2h_bytes_per_step")}, **e2e_cfg}
+    return {"metric": METRIC, "value": res["value"], "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": res["ms_per_step"], "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16 (fp32 master, fp32 accumulate)",
+            "data": "synthetic (seeded Gaussian-mixture shards, random-init MLP)",
+            "config": workload_config(w), "roofline": top_roof, "cpu_baseline": cpu_line, "e2e": e2e_line,
+            "gpu_launches": res["gpu_launches"], "clocks": res["clocks"], "merge": res["merge"],
+            "kernels": res["kernels"], "samples_per_round": res["samples_per_round"],
+            "T_star": res["T_star"], "tau": res["tau"], "workloads": res["workloads"]}
 
 
 def main():
@@ -797,22 +905,19 @@ def main():
     w = WORKLOADS[args.workload]
     if args.samples_per_worker:
         w = dataclasses.replace(w, samples_per_worker=args.samples_per_worker)
-    cpu = None
+    cpu, cpus = None, {}
     if rank == 0 and world == 1 and not args.no_cpu:
-        samples, dt, done = oracle_rounds(w, 6, 15.0)
-        cpu = {"value": samples / dt, "unit": UNIT, "cores": cores_used(), "kind": "oracle",
-               "sample": f"{done} Oscars rounds of {w.name} (numpy fp64 with bf16 operand emulation)"}
+        cpu = training_cpu_baseline(w, 6, 10.0)
+        if res["workloads"]:
+            cpus[synth.CFG1.name] = training_cpu_baseline(synth.CFG1, 20, 4.0)
+            cpus[synth.CFG3.name] = training_cpu_baseline(synth.CFG3, 1, 30.0)
+        if res["merge"]:
+            import torch
+            dev = torch.device(f"cuda:{local_rank}")
+            for m in merge_workloads(args):
+                cpus[m.name] = merge_cpu_baseline(m, dev)
     if rank == 0:
-        line = {"metric": METRIC, "value": res["value"], "unit": UNIT, "n_gpus": world, "steps": args.steps,
-                "warmup": args.warmup, "ms_per_step": res["ms_per_step"], "higher_is_better": True,
-                "scaling": "weak", "vs_baseline": None, "dtype": "bf16 (fp32 master, fp32 accumulate)",
-                "data": "synthetic (seeded Gaussian-mixture shards, random-init MLP)",
-                "config": workload_config(w, "flushed between timed rounds (512 MB write)"),
-                "roofline": res["roofline"], "cpu_baseline": cpu, "e2e": res["e2e"],
-                "gpu_launches": res["gpu_launches"], "clocks": res["clocks"], "merge": res["merge"],
-                "kernels": res["kernels"], "samples_per_round": res["samples_per_round"],
-                "T_star": res["T_star"], "tau": res["tau"], "workloads": res["workloads"]}
-        print(json.dumps(line))
+        print(json.dumps(result_line(args, world, w, res, cpu, cpus)))
     if world > 1:
         import torch
         torch.distributed.barrier()

@@ -98,7 +98,9 @@ typedef struct {
   int32_t num_layers;   /* L >= 1 (MLP); 1 for FLAT                              */
   const int32_t* dims;  /* host, L+1 entries: input, hidden..., classes.  FLAT:  */
                         /* dims[0] = P.  MLP: classes <= 32                      */
-  int32_t batch;        /* B, mini-batch rows per local step (MLP)               */
+  int32_t batch;        /* B, mini-batch rows per local step (MLP); fp32        */
+                        /* softmax regression: 1..512, bf16 MLP: multiple of 32 */
+                        /* up to 256                                            */
   float lr;             /* eta of Eq. 4                                          */
   float server_lr;      /* eta_s of the delta-form merge; 1.0 = Eq. 4's average  */
   int32_t weight_rule;  /* oscars_weight_rule                                    */
@@ -419,12 +421,14 @@ oscars_status oscars_gemm_bf16_nt(const void* A, const void* B, float* C, int32_
  *
  * params_in / params_out: device, classes*dim + classes fp32 each, canonical
  * layout (W [classes][dim], then b [classes]); they may be the same buffer.
- * x: device [n][dim] fp32; y: device [n] int32 labels in [0, classes).
- * Step s uses rows (cursor + s*batch + b) mod n, b < batch.
+ * x: device [n][dim] fp32 (any alignment; with dim % 4 == 0 and x 16-byte
+ * aligned the rows are read as 16-byte vectors); y: device [n] int32 labels
+ * in [0, classes).  Step s uses rows (cursor + s*batch + b) mod n, b < batch.
  * loss_out: device, 1 float: the mean mini-batch loss over the tau steps.
  * Ordered on `stream`.  1 <= tau <= 16320 (the scratch holds one loss
  * partial per step); larger tau, classes outside [2, 32] or bad pointers give
- * EINVAL, shapes whose weights plus one batch exceed shared memory ENOTSUP.
+ * EINVAL; batch > 512, or shapes whose weights plus one batch exceed shared
+ * memory, ENOTSUP.
  * The first call on a device looks up the scratch address (once per device);
  * make that first call before any stream capture.  Every call shares the one
  * scratch array and leaves its contents behind; each call writes all it reads

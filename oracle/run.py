@@ -80,6 +80,7 @@ class RoundRecord:
     idle: np.ndarray                 # idle ticks of each worker this round (Eq. 1)
     x_g: Optional[np.ndarray] = None # global model after the merge (flat, fp32)
     eval_loss: Optional[float] = None
+    replicas: Optional[list] = None  # the pushed models (flat), when asked for
 
 
 @dataclass
@@ -132,7 +133,8 @@ def local_steps(state: OscarsState, worker: int, shard, batch: int, lr: float, r
 
 
 def run_round(state: OscarsState, shards, batch: int, lr: float, rnd: Callable,
-              weight_rule: str = "uniform", server_lr: float = 1.0, weights=None) -> RoundRecord:
+              weight_rule: str = "uniform", server_lr: float = 1.0, weights=None,
+              keep_replicas: bool = False) -> RoundRecord:
     W = len(shards)
     models, wl = [], np.zeros(W)
     for i in range(W):
@@ -144,18 +146,21 @@ def run_round(state: OscarsState, shards, batch: int, lr: float, rnd: Callable,
     idle = state.T_star - state.tau.astype(np.int64) * state.t_iter     # = mod(T*, t_i) under Algorithm 1
     state.clock += state.tau.astype(np.int64) * state.t_iter + idle
     state.idle += idle
-    return RoundRecord(state.tau.copy(), state.T_star, wl, idle, x_new)
+    return RoundRecord(state.tau.copy(), state.T_star, wl, idle, x_new,
+                       replicas=models if keep_replicas else None)
 
 
 def run(dims, layers0, shards, speeds=None, t_iter=None, M: int = 8, rounds: int = 1,
         batch: int = 32, lr: float = 0.05, bf16: bool = True, weight_rule: str = "uniform",
         server_lr: float = 1.0, mode: int = _sched.CAPPED, tau_override=None,
-        eval_set=None, ticks_per_unit: int = 1000, target_loss=None, t_per_round=None, model=None):
+        eval_set=None, ticks_per_unit: int = 1000, target_loss=None, t_per_round=None, model=None,
+        keep_replicas: bool = False):
     """Run ``rounds`` rounds; returns (final state, [RoundRecord]).  With an
     eval set and a target loss, stop after the first round whose eval loss
     is at or below the target.  ``t_per_round[r]`` (optional): iteration
     times in force from round r on (drifting speeds), re-solved with
-    Algorithm 1 before that round."""
+    Algorithm 1 before that round.  ``keep_replicas``: every record also
+    holds the W pushed models of its round."""
     if t_iter is None:
         t_iter = t_per_round[0] if t_per_round is not None else _sched.iteration_ticks(speeds, ticks_per_unit)
     rnd = _bf16.round_bf16 if bf16 else _bf16.identity
@@ -164,7 +169,7 @@ def run(dims, layers0, shards, speeds=None, t_iter=None, M: int = 8, rounds: int
     for r in range(rounds):
         if t_per_round is not None and r > 0:
             reschedule(state, t_per_round[r], M, mode)
-        rec = run_round(state, shards, batch, lr, rnd, weight_rule, server_lr)
+        rec = run_round(state, shards, batch, lr, rnd, weight_rule, server_lr, keep_replicas=keep_replicas)
         if eval_set is not None:
             rec.eval_loss = state.model.loss_of(state.x_g, eval_set[0], eval_set[1], rnd)
         records.append(rec)

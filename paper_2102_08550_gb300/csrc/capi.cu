@@ -1136,6 +1136,7 @@ oscars_status validate_and_layout(oscars_ctx* c, const oscars_config* cfg) {
   if (c->C < 2 || c->C > kMaxClasses) return fail(c, OSCARS_ENOTSUP, "classes must be in [2, 32]");
   if (!(c->lr == c->lr)) return fail(c, OSCARS_EINVAL, "lr is NaN");
   if (c->L == 1 && !c->bf16) {
+    if (c->B > kSoftregMaxBatch) return fail(c, OSCARS_ENOTSUP, "softmax regression: batch must be <= 512");
     if (softreg_smem_bytes(c->dims[0], c->C, c->B) > 220 * 1024)
       return fail(c, OSCARS_ENOTSUP, "softmax regression: weights plus one batch must fit in shared memory");
   } else if (c->bf16 && c->L >= 2) {

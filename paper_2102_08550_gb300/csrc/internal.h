@@ -50,6 +50,9 @@ struct SoftregArgs {
 };
 cudaError_t launch_softreg_round(const SoftregArgs& a, int W, cudaStream_t s);
 size_t softreg_smem_bytes(int D, int C, int B);
+// the round kernel gives each mini-batch row one thread for its row offset,
+// label and softmax: B must not exceed its block size
+constexpr int kSoftregMaxBatch = 512;
 
 struct SoftregEvalArgs {
   const float* master;  // global slot

@@ -14,8 +14,16 @@
 // In MLP mode the same pass also writes the bf16 operand copy of x_g.
 //
 // Grid: persistent, (SM count) x (resident CTAs per SM) blocks of 256
-// threads striding over 16-byte chunks; each thread keeps 8 independent
-// 16-byte loads in flight per group of 8 workers.
+// threads striding over 16-byte chunks; each thread keeps 16 independent
+// 16-byte loads in flight per group of 16 workers.
+//
+// Alignment: the vector kernel needs every buffer at the same offset modulo
+// 16 bytes.  When they share one offset that is not 0, the first (up to 3)
+// elements are peeled off to the scalar kernel and the vector kernel starts
+// at the first 16-byte boundary; only buffers with different offsets fall
+// back to the scalar kernel for the whole vector.
+#include <atomic>
+
 #include "common.cuh"
 #include "internal.h"
 
@@ -84,14 +92,18 @@ __global__ void __launch_bounds__(kThreads) merge_vec4_kernel(const __grid_const
   }
 }
 
-// Any alignment: one element per thread and iteration, elements [begin, P).
+// Any alignment: one element per thread and iteration, over the elements
+// [0, head) and [tail, P) (the peeled head and the tail of the vector
+// kernel, or head = tail = 0 for the whole vector).
 template <bool kReplica>
 __global__ void __launch_bounds__(kThreads) merge_scalar_kernel(const __grid_constant__ MergeArgs a,
                                                                 float* __restrict__ x_g,
-                                                                int64_t begin, int64_t P, float eta,
+                                                                int64_t head, int64_t tail, int64_t P, float eta,
                                                                 __nv_bfloat16* __restrict__ shadow) {
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
-  for (int64_t p = begin + static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; p < P; p += stride) {
+  const int64_t count = head + (P - tail);
+  for (int64_t q = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; q < count; q += stride) {
+    const int64_t p = q < head ? q : tail + (q - head);
     const float x = x_g[p];
     float acc = 0.f;
     for (int k = 0; k < a.W; ++k) {
@@ -104,16 +116,23 @@ __global__ void __launch_bounds__(kThreads) merge_scalar_kernel(const __grid_con
   }
 }
 
-int g_sm_count = 0;
+constexpr int kMaxDevices = 64;
+std::atomic<int> g_sm_count[kMaxDevices];
 
+// SM count of the current device (queried once per device)
 int sm_count() {
-  if (g_sm_count == 0) {
-    int dev = 0;
-    cudaGetDevice(&dev);
-    cudaDeviceGetAttribute(&g_sm_count, cudaDevAttrMultiProcessorCount, dev);
-    if (g_sm_count <= 0) g_sm_count = 1;
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0) return 1;
+  if (dev >= kMaxDevices) {
+    int n = 0;
+    return cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess && n > 0 ? n : 1;
   }
-  return g_sm_count;
+  int n = g_sm_count[dev].load(std::memory_order_relaxed);
+  if (n == 0) {
+    if (cudaDeviceGetAttribute(&n, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess || n <= 0) n = 1;
+    g_sm_count[dev].store(n, std::memory_order_relaxed);
+  }
+  return n;
 }
 
 }  // namespace
@@ -121,35 +140,48 @@ int sm_count() {
 cudaError_t launch_merge(const MergeArgs& a, float* x_g, int64_t P, float eta, bool replica,
                          cudaStream_t s, __nv_bfloat16* shadow) {
   if (P <= 0) return cudaSuccess;
-  bool aligned = (reinterpret_cast<uintptr_t>(x_g) & 15) == 0 && (reinterpret_cast<uintptr_t>(shadow) & 7) == 0;
-  for (int k = 0; k < a.W && aligned; ++k) aligned = (reinterpret_cast<uintptr_t>(a.src[k]) & 15) == 0;
+  // elements before the first 16-byte boundary of x_g; the vector kernel
+  // runs from there when every buffer has the same offset modulo 16 bytes
+  // (and the bf16 copy, two bytes per element, is then 8-byte aligned)
+  const uintptr_t off = reinterpret_cast<uintptr_t>(x_g) & 15;
+  bool vec = (off & 3) == 0;
+  int64_t head = vec ? static_cast<int64_t>((16 - off) & 15) / 4 : 0;
+  if (head > P) head = P;
+  for (int k = 0; k < a.W && vec; ++k) vec = (reinterpret_cast<uintptr_t>(a.src[k]) & 15) == off;
+  if (vec && shadow) vec = (reinterpret_cast<uintptr_t>(shadow + head) & 7) == 0;
   const int ctas_per_sm = 2048 / kThreads;
-  const int64_t n4 = aligned ? P / 4 : 0;
+  const int64_t n4 = vec ? (P - head) / 4 : 0;
+  if (n4 == 0) head = 0;
   if (n4 > 0) {
+    MergeArgs av = a;   // the same buffers from the first 16-byte boundary on
+    for (int k = 0; k < a.W; ++k) av.src[k] = a.src[k] + head;
+    float* xv = x_g + head;
+    __nv_bfloat16* sv = shadow ? shadow + head : nullptr;
     int64_t blocks = static_cast<int64_t>(sm_count()) * ctas_per_sm;
     const int64_t need = (n4 + kThreads - 1) / kThreads;
     if (need < blocks) blocks = need;
     const unsigned nb = static_cast<unsigned>(blocks);
     if (replica && shadow)
-      merge_vec4_kernel<true, true><<<nb, kThreads, 0, s>>>(a, x_g, n4, eta, shadow);
+      merge_vec4_kernel<true, true><<<nb, kThreads, 0, s>>>(av, xv, n4, eta, sv);
     else if (replica)
-      merge_vec4_kernel<true, false><<<nb, kThreads, 0, s>>>(a, x_g, n4, eta, nullptr);
+      merge_vec4_kernel<true, false><<<nb, kThreads, 0, s>>>(av, xv, n4, eta, nullptr);
     else if (shadow)
-      merge_vec4_kernel<false, true><<<nb, kThreads, 0, s>>>(a, x_g, n4, eta, shadow);
+      merge_vec4_kernel<false, true><<<nb, kThreads, 0, s>>>(av, xv, n4, eta, sv);
     else
-      merge_vec4_kernel<false, false><<<nb, kThreads, 0, s>>>(a, x_g, n4, eta, nullptr);
+      merge_vec4_kernel<false, false><<<nb, kThreads, 0, s>>>(av, xv, n4, eta, nullptr);
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
   }
-  const int64_t begin = n4 * 4;
-  if (begin < P) {
+  const int64_t tail = head + n4 * 4;
+  if (head > 0 || tail < P) {
     int64_t blocks = static_cast<int64_t>(sm_count()) * ctas_per_sm;
-    const int64_t need = (P - begin + kThreads - 1) / kThreads;
+    const int64_t need = (head + (P - tail) + kThreads - 1) / kThreads;
     if (need < blocks) blocks = need;
+    const unsigned nb = static_cast<unsigned>(blocks);
     if (replica)
-      merge_scalar_kernel<true><<<static_cast<unsigned>(blocks), kThreads, 0, s>>>(a, x_g, begin, P, eta, shadow);
+      merge_scalar_kernel<true><<<nb, kThreads, 0, s>>>(a, x_g, head, tail, P, eta, shadow);
     else
-      merge_scalar_kernel<false><<<static_cast<unsigned>(blocks), kThreads, 0, s>>>(a, x_g, begin, P, eta, shadow);
+      merge_scalar_kernel<false><<<nb, kThreads, 0, s>>>(a, x_g, head, tail, P, eta, shadow);
     return cudaGetLastError();
   }
   return cudaSuccess;

@@ -82,6 +82,7 @@ extern "C" oscars_status oscars_softreg_steps_noalloc(const float* params_in, fl
   if (!params_in || !params_out || !x || !y || !loss_out) return OSCARS_EINVAL;
   if (n < 1 || cursor < 0 || dim < 1 || batch < 1 || classes < 2 || classes > kMaxClasses) return OSCARS_EINVAL;
   if (tau < 1 || tau > kMaxSteps) return OSCARS_EINVAL;   // beyond the fixed scratch
+  if (batch > kSoftregMaxBatch) return OSCARS_ENOTSUP;
   if (softreg_smem_bytes(dim, classes, batch) > 220 * 1024) return OSCARS_ENOTSUP;
   void* base = nullptr;
   if (scratch_address(&base) != cudaSuccess) return OSCARS_ECUDA;

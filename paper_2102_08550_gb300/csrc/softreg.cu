@@ -22,6 +22,7 @@ namespace {
 
 constexpr int kThreads = 512;
 constexpr int kWarps = kThreads / 32;
+static_assert(kSoftregMaxBatch <= kThreads, "one thread per mini-batch row");
 
 __device__ __forceinline__ float warp_sum(float v) {
 #pragma unroll
@@ -59,10 +60,11 @@ __global__ void __launch_bounds__(kThreads) softreg_round_kernel(const __grid_co
   const int64_t n = a.shard_n[w];
   const int64_t cur = a.cursor[w];
   const float invB = 1.0f / static_cast<float>(B);
-  // with D % 4 == 0 and a mini-batch of at most kPrefetch float4 per thread,
-  // step s + 1's rows are loaded into registers while step s computes
+  // with D % 4 == 0, a 16-byte aligned shard and a mini-batch of at most
+  // kPrefetch float4 per thread, step s + 1's rows are loaded into registers
+  // while step s computes (otherwise rows are read one float at a time)
   const int D4 = D / 4;
-  const bool vec = (D & 3) == 0 && B * D4 <= kPrefetch * kThreads;
+  const bool vec = (D & 3) == 0 && (reinterpret_cast<uintptr_t>(X) & 15) == 0 && B * D4 <= kPrefetch * kThreads;
   float4 pf[kPrefetch];
   auto fetch = [&](int s) {   // rows of step s into registers (row offsets already in Rsm)
 #pragma unroll

@@ -122,6 +122,9 @@ def _cfg(**kw):
     (dict(dims=[8, 128, 40]), P.OSCARS_ENOTSUP),      # more than 32 classes
     (dict(batch=48), P.OSCARS_ENOTSUP),
     (dict(), P.OSCARS_EINVAL),                        # valid shape but NULL shards
+    (dict(dims=[64, 10], bf16=0, batch=513), P.OSCARS_ENOTSUP),    # fp32 softmax regression: batch > 512
+    (dict(dims=[64, 10], bf16=0, batch=512), P.OSCARS_EINVAL),     # batch 512 passes; NULL shards
+    (dict(dims=[4096, 10], bf16=0, batch=32), P.OSCARS_ENOTSUP),   # weights + batch beyond shared memory
 ])
 def test_create_rejects_before_device_work(oscars_lib, change, status):
     cfg, keep = _cfg(**change)

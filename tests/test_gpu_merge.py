@@ -14,8 +14,15 @@ from tests.gpu_util import PARAM_RTOL, rel_maxabs
 pytestmark = pytest.mark.gpu
 
 
+# offset: elements before every buffer.  With (Pn + offset) % 4 == 0 all the
+# buffers share one misalignment (the vector kernel after a peeled scalar
+# head: (5, 4099, 1), (17, 777, 3), (5, 7, 1), (9, 4095, 1) with no tail, and
+# (5, 3, 1) where the head is all of P); otherwise the delta rows are
+# misaligned differently and the scalar kernel takes the whole vector
+# ((4, 1001, 1)).
 @pytest.mark.parametrize("W,Pn,offset", [(1, 1, 0), (1, 7, 0), (3, 1023, 0), (8, 4096, 0), (5, 4099, 1),
-                                           (64, 10001, 0), (17, 777, 3), (256, 513, 0)])
+                                           (64, 10001, 0), (17, 777, 3), (256, 513, 0), (5, 3, 1), (5, 7, 1),
+                                           (9, 4095, 1), (4, 1001, 1)])
 def test_merge_small(cuda_device, W, Pn, offset):
     rng = np.random.default_rng(W * 1000 + Pn)
     xg = rng.standard_normal(Pn).astype(np.float32)
