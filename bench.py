@@ -499,6 +499,7 @@ def merge_workloads(args):
 # P): (dram__bytes_read.sum + dram__bytes_write.sum) / ((W + 2) * P * 4).
 MERGE_TRAFFIC = {
     64: (0.99621, "profiles/merge_vec4_P4M_W64.md (P = 4M, scaled by P)"),
+    8: (0.98790, "profiles/merge_vec4_P32M_W8.md (P = 32M, scaled by P)"),
 }
 
 

@@ -9,7 +9,8 @@ Here the oracle stands in for the GPU path:
   under a third perturbation seed) stays inside the bound;
 * each planted mistake of ``tests.oracle_mutants`` (stale bf16 operand after
   step 0, bias update skipped, one sample dropped per mini-batch, cursor one
-  batch ahead) lands outside it, on the 784-512-10 workload with 16 workers
+  batch ahead) lands outside it by at least a factor 2, on the 784-512-10
+  workload with 16 workers
   and on a small 3-layer shape, in every round checked.
 """
 import numpy as np
@@ -24,7 +25,7 @@ from tests.gpu_util import ENV_FACTOR, PARAM_RTOL, envelope, per_tensor_errors, 
 CASES = {
     # name: (workload, rounds, rows per shard)
     "mlp-784-512-10-W16": (synth.CFG2, 2, 2 * 6 * 64 + 64),
-    "small-3layer": (synth.TrainWorkload("small-3layer", 3, [200, 256, 128, 10], 32, 0.05, 256, 6, 3), 3, 256),
+    "small-3layer": (synth.TrainWorkload("small-3layer", 3, [200, 256, 128, 10], 32, 0.05, 512, 6, 3), 3, 512),
 }
 
 
@@ -68,4 +69,4 @@ def test_planted_mistake_lands_outside(case, mutant):
         got = run()
     for r, (g, x, b) in enumerate(zip(got, ref, bound)):
         e = np.asarray(per_tensor_errors(g, x, w.dims))
-        assert np.any(e > 4.0 * b), (name, mutant, r, (e / b).tolist())
+        assert np.any(e > 2.0 * b), (name, mutant, r, (e / b).tolist())
