@@ -881,7 +881,8 @@ cudaError_t enqueue_round_softreg(oscars_ctx* c, cudaStream_t st) {
   cudaError_t e;
   {
     ProfScope ps(c, "softreg_round", st);
-    e = launch_softreg_round(a, c->W, st);
+    e = softreg_cluster_supported(a.D, a.C, a.B) ? launch_softreg_cluster_round(a, c->W, st)
+                                                 : launch_softreg_round(a, c->W, st);
   }
   if (e != cudaSuccess) return e;
   ProfScope ps(c, "round_bookkeeping", st);

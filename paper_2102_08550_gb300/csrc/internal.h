@@ -53,6 +53,12 @@ size_t softreg_smem_bytes(int D, int C, int B);
 // the round kernel gives each mini-batch row one thread for its row offset,
 // label and softmax: B must not exceed its block size
 constexpr int kSoftregMaxBatch = 512;
+// the same round with each worker on a cluster of 8 CTAs splitting the input
+// columns (B <= 256 and a column slice plus one batch slice in shared memory)
+bool softreg_cluster_supported(int D, int C, int B);
+int softreg_cluster_cols(int D);
+size_t softreg_cluster_smem_bytes(int D, int C, int B);
+cudaError_t launch_softreg_cluster_round(const SoftregArgs& a, int W, cudaStream_t s);
 
 struct SoftregEvalArgs {
   const float* master;  // global slot

@@ -2,12 +2,15 @@
 // cross-entropy): Eq. 4, "otherwise" branch, x <- x - lr * g(x) with g the
 // mean mini-batch gradient.
 //
-// One CTA per worker runs the worker's whole round: it pulls the global
+// Each worker's whole round runs in one launch: the worker pulls the global
 // model into shared memory (the pull of the parameter-server description,
 // fused: nothing is copied through HBM), runs tau_i SGD steps on successive
 // mini-batches of its shard with the weights resident in shared memory, and
 // writes the result to the worker's replica (the push).  Workers never
-// exchange data inside a round, so the round is one launch.
+// exchange data inside a round.  Two kernels: softreg_cluster_round_kernel
+// puts each worker on a cluster of 8 CTAs that split the input columns (the
+// round kernel of a context, batch <= 256); softreg_round_kernel puts each
+// worker on one CTA (larger batches, and the allocation-free entry point).
 //
 // Per step: logits z[b][c] = sum_k x[b][k] W[c][k] + bias[c] (warp-level dot
 // products), p = softmax(z), loss_b = logsumexp(z_b) - z_b[y_b],
@@ -204,6 +207,214 @@ __global__ void __launch_bounds__(kThreads) softreg_round_kernel(const __grid_co
   for (int i = tid; i < C; i += kThreads) dst[a.offB + i] = bsm[i];
 }
 
+// The same round with each worker on a cluster of kCl CTAs that split the
+// input columns: CTA r owns columns [r * Dc, min(D, (r + 1) * Dc)) (Dc a
+// multiple of 4) of W and of every mini-batch row, so a step's work and the
+// shared memory it needs are divided by kCl.  Per step each CTA computes the
+// partial logits of the whole mini-batch over its columns; after one cluster
+// barrier every CTA sums the kCl partials in rank order (distributed shared
+// memory loads) and adds the bias, and runs the softmax cross-entropy of every
+// row itself (identical arithmetic in every CTA); then it updates its own
+// columns of W, and its private copy of the bias (the same update in every
+// CTA; rank 0 writes it back).  The partial logits are double-buffered by
+// step parity: a CTA rewrites a buffer two steps later, after a barrier that
+// every reader of the buffer has passed.
+constexpr int kCl = 8;
+constexpr int kClThreads = 256;
+// columns per CTA: D / kCl rounded up to a multiple of 4
+__host__ __device__ inline int cluster_cols(int D) { return ((D + kCl - 1) / kCl + 3) / 4 * 4; }
+constexpr int kClPrefetch = 8;   // float4 items of the next step's rows held per thread
+
+__global__ void __launch_bounds__(kClThreads) softreg_cluster_round_kernel(const __grid_constant__ SoftregArgs a) {
+  extern __shared__ __align__(16) float sm[];
+  const int D = a.D, C = a.C, B = a.B;
+  const int Dc = cluster_cols(D);
+  const int rank = static_cast<int>(cluster_ctarank());
+  const int c0 = rank * Dc;
+  const int nc = D - c0 < Dc ? (D - c0 > 0 ? D - c0 : 0) : Dc;   // this CTA's columns (may be 0)
+  float* Wsm = sm;                       // [C][Dc]
+  float* bsm = Wsm + C * Dc;             // [32]
+  float* Xsm = bsm + 32;                 // [B][Dc]
+  float* Psm = Xsm + B * Dc;             // [2][B][C] partial logits, by step parity
+  float* Zsm = Psm + 2 * B * C;          // [B][C] logits, then dz
+  float* Lsm = Zsm + B * C;              // [B]
+  int* Ysm = reinterpret_cast<int*>(Lsm + B);   // [B]
+  int64_t* Rsm = reinterpret_cast<int64_t*>((reinterpret_cast<uintptr_t>(Ysm + B) + 7) & ~uintptr_t(7));  // [B]
+
+  const int w = blockIdx.y;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int tau = a.tau[w];
+  const float* gsrc = a.master + static_cast<int64_t>(a.global_slot) * a.slot_stride;
+  float* dst = a.master_out + static_cast<int64_t>(w) * a.slot_stride;
+  const float* X = a.shard_x[w];
+  const int32_t* Y = a.shard_y[w];
+  const int64_t n = a.shard_n[w];
+  const int64_t cur = a.cursor[w];
+  const float invB = 1.0f / static_cast<float>(B);
+  const int nc4 = nc / 4;
+
+  // pull: this CTA's columns of the global model, and the whole bias
+  for (int i = tid; i < C * Dc; i += kClThreads) {
+    const int c = i / Dc, k = i - c * Dc;
+    Wsm[i] = k < nc ? gsrc[a.offW + static_cast<int64_t>(c) * D + c0 + k] : 0.f;
+  }
+  for (int i = tid; i < C; i += kClThreads) bsm[i] = gsrc[a.offB + i];
+
+  // rows of step s: (cursor + s*B + b) mod n; this CTA's columns of each,
+  // as 16-byte loads when every row's slice is 16-byte aligned
+  const bool vec = (D & 3) == 0 && (reinterpret_cast<uintptr_t>(X) & 15) == 0 && B * nc4 <= kClPrefetch * kClThreads;
+  float4 pf[kClPrefetch];
+  auto row_offsets = [&](int s) {
+    if (tid < B) {
+      const int64_t r = (cur + static_cast<int64_t>(s) * B + tid) % n;
+      Rsm[tid] = r * D + c0;
+      Ysm[tid] = Y[r];
+    }
+  };
+  auto fetch = [&]() {
+#pragma unroll
+    for (int j = 0; j < kClPrefetch; ++j) {
+      const int i = tid + j * kClThreads;
+      if (i < B * nc4) {
+        const int b = i / nc4, k4 = i - b * nc4;
+        pf[j] = *reinterpret_cast<const float4*>(X + Rsm[b] + 4 * k4);
+      }
+    }
+  };
+  if (vec && tau > 0) {
+    row_offsets(0);
+    __syncthreads();
+    fetch();
+  }
+
+  for (int s = 0; s < tau; ++s) {
+    float* Pp = Psm + (s & 1) * B * C;
+    __syncthreads();   // the previous step is done with Xsm and Zsm
+    int yl = 0;
+    if (vec) {
+      if (tid < B) yl = Ysm[tid];
+#pragma unroll
+      for (int j = 0; j < kClPrefetch; ++j) {
+        const int i = tid + j * kClThreads;
+        if (i < B * nc4) {
+          const int b = i / nc4, k4 = i - b * nc4;
+          reinterpret_cast<float4*>(Xsm + b * Dc)[k4] = pf[j];
+        }
+      }
+      if (s + 1 < tau) row_offsets(s + 1);
+      __syncthreads();
+      if (s + 1 < tau) fetch();
+    } else {
+      row_offsets(s);
+      __syncthreads();
+      for (int i = tid; i < B * nc; i += kClThreads) {
+        const int b = i / nc, k = i - b * nc;
+        Xsm[b * Dc + k] = X[Rsm[b] + k];
+      }
+      if (tid < B) yl = Ysm[tid];
+      __syncthreads();
+    }
+    // partial logits over this CTA's columns: one thread per (row, class)
+    for (int q = tid; q < B * C; q += kClThreads) {
+      const int b = q / C, c = q - b * C;
+      const float* xr = Xsm + b * Dc;
+      const float* wr = Wsm + c * Dc;
+      float acc = 0.f;
+      if ((nc & 3) == 0) {
+        for (int k4 = 0; k4 < nc4; ++k4) {
+          const float4 xv = reinterpret_cast<const float4*>(xr)[k4];
+          const float4 wv = reinterpret_cast<const float4*>(wr)[k4];
+          acc = fmaf(xv.x, wv.x, acc);
+          acc = fmaf(xv.y, wv.y, acc);
+          acc = fmaf(xv.z, wv.z, acc);
+          acc = fmaf(xv.w, wv.w, acc);
+        }
+      } else {
+        for (int k = 0; k < nc; ++k) acc = fmaf(xr[k], wr[k], acc);
+      }
+      Pp[q] = acc;
+    }
+    cluster_sync();
+    // logits: the partials of every CTA in rank order, then the bias
+    for (int q = tid; q < B * C; q += kClThreads) {
+      float part[kCl];
+#pragma unroll
+      for (int r = 0; r < kCl; ++r) part[r] = ld_dsmem_f32(Pp + q, r);
+      float acc = 0.f;
+#pragma unroll
+      for (int r = 0; r < kCl; ++r) acc += part[r];
+      Zsm[q] = acc + bsm[q % C];
+    }
+    __syncthreads();
+    // softmax cross-entropy, one thread per row
+    if (tid < B) {
+      float* z = Zsm + tid * C;
+      float m = z[0];
+      for (int c = 1; c < C; ++c) m = fmaxf(m, z[c]);
+      const int y = yl;
+      float se = 0.f, so = 0.f;
+      for (int c = 0; c < C; ++c) {
+        const float e = expf(z[c] - m);
+        se += e;
+        if (c != y) so += e;
+      }
+      Lsm[tid] = m + logf(se) - z[y];
+      for (int c = 0; c < C; ++c) z[c] = (c == y ? -(so / se) : expf(z[c] - m) / se) * invB;
+    }
+    __syncthreads();
+    if (rank == 0 && warp == 0) {   // the step's loss: rows summed in order
+      if (lane == 0) {
+        float l = 0.f;
+        for (int b = 0; b < B; ++b) l += Lsm[b];
+        a.loss_part[static_cast<int64_t>(w) * a.max_tau + s] = l;
+      }
+    }
+    // weight gradient and update of this CTA's columns: item = (class, 4 columns)
+    if ((nc & 3) == 0) {
+      for (int q = tid; q < C * nc4; q += kClThreads) {
+        const int c = q / nc4, k4 = q - c * nc4;
+        float4 g = make_float4(0.f, 0.f, 0.f, 0.f);
+        for (int b = 0; b < B; ++b) {
+          const float d = Zsm[b * C + c];
+          const float4 xv = reinterpret_cast<const float4*>(Xsm + b * Dc)[k4];
+          g.x = fmaf(d, xv.x, g.x);
+          g.y = fmaf(d, xv.y, g.y);
+          g.z = fmaf(d, xv.z, g.z);
+          g.w = fmaf(d, xv.w, g.w);
+        }
+        float4* wp = reinterpret_cast<float4*>(Wsm + c * Dc) + k4;
+        float4 wv = *wp;
+        wv.x = fmaf(-a.lr, g.x, wv.x);
+        wv.y = fmaf(-a.lr, g.y, wv.y);
+        wv.z = fmaf(-a.lr, g.z, wv.z);
+        wv.w = fmaf(-a.lr, g.w, wv.w);
+        *wp = wv;
+      }
+    } else {
+      for (int q = tid; q < C * nc; q += kClThreads) {
+        const int c = q / nc, k = q - c * nc;
+        float g = 0.f;
+        for (int b = 0; b < B; ++b) g = fmaf(Zsm[b * C + c], Xsm[b * Dc + k], g);
+        Wsm[c * Dc + k] = fmaf(-a.lr, g, Wsm[c * Dc + k]);
+      }
+    }
+    for (int c = tid; c < C; c += kClThreads) {   // the bias, the same update in every CTA
+      float g = 0.f;
+      for (int b = 0; b < B; ++b) g += Zsm[b * C + c];
+      bsm[c] = fmaf(-a.lr, g, bsm[c]);
+    }
+  }
+  __syncthreads();
+  // push: this CTA's columns into the replica (rank 0 also the bias)
+  for (int i = tid; i < C * nc; i += kClThreads) {
+    const int c = i / nc, k = i - c * nc;
+    dst[a.offW + static_cast<int64_t>(c) * D + c0 + k] = Wsm[c * Dc + k];
+  }
+  if (rank == 0)
+    for (int i = tid; i < C; i += kClThreads) dst[a.offB + i] = bsm[i];
+  cluster_sync();   // no CTA leaves while a peer may still read its partial logits
+}
+
 // Mean cross-entropy of the global model: one warp per sample, partial sums
 // per block (summed afterwards in a fixed order).
 __global__ void __launch_bounds__(256) softreg_eval_kernel(const __grid_constant__ SoftregEvalArgs a) {
@@ -249,6 +460,38 @@ cudaError_t launch_softreg_round(const SoftregArgs& a, int W, cudaStream_t s) {
   if (e != cudaSuccess) return e;
   softreg_round_kernel<<<W, kThreads, smem, s>>>(a);
   return cudaGetLastError();
+}
+
+int softreg_cluster_cols(int D) { return cluster_cols(D); }
+
+size_t softreg_cluster_smem_bytes(int D, int C, int B) {
+  const size_t Dc = static_cast<size_t>(softreg_cluster_cols(D));
+  return sizeof(float) * (C * Dc + 32 + static_cast<size_t>(B) * Dc + 3 * static_cast<size_t>(B) * C + B) +
+         sizeof(int) * B + 8 + sizeof(int64_t) * B;
+}
+
+bool softreg_cluster_supported(int D, int C, int B) {
+  return B <= kClThreads && softreg_cluster_smem_bytes(D, C, B) <= 200 * 1024;
+}
+
+cudaError_t launch_softreg_cluster_round(const SoftregArgs& a, int W, cudaStream_t s) {
+  const size_t smem = softreg_cluster_smem_bytes(a.D, a.C, a.B);
+  cudaError_t e = cudaFuncSetAttribute(softreg_cluster_round_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       static_cast<int>(smem));
+  if (e != cudaSuccess) return e;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(kCl, W, 1);
+  cfg.blockDim = dim3(kClThreads, 1, 1);
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr;
+  attr.id = cudaLaunchAttributeClusterDimension;
+  attr.val.clusterDim.x = kCl;
+  attr.val.clusterDim.y = 1;
+  attr.val.clusterDim.z = 1;
+  cfg.attrs = &attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, softreg_cluster_round_kernel, a);
 }
 
 cudaError_t launch_softreg_eval(const SoftregEvalArgs& a, int blocks, cudaStream_t s) {

@@ -217,6 +217,24 @@ def test_mlp_3072_1024_1024_10_w32_every_worker(cuda_device):
         i += 1
 
 
+SOFTREG_SHAPES = [
+    # name, D, C, B, rows: the cluster kernel's column split (8 CTAs per worker)
+    ("d18-c10", 18, 10, 20, 100),      # some CTAs own no column, one owns 2
+    ("d785-c10", 785, 10, 32, 128),    # D % 4 != 0: one float at a time
+    ("d64-c32-b256", 64, 32, 256, 600),  # the largest batch and class count of the cluster kernel
+]
+
+
+@pytest.mark.parametrize("name,D,C,B,rows", SOFTREG_SHAPES, ids=[s[0] for s in SOFTREG_SHAPES])
+def test_softmax_regression_shapes(cuda_device, name, D, C, B, rows):
+    """fp32 softmax regression with each worker on a cluster that splits the
+    input columns: ragged and empty column slices, scalar row loads, shards
+    that wrap; three rounds, strict 1e-5 against the oracle."""
+    w = synth.TrainWorkload(f"softreg-{name}", 3, [D, C], B, 0.05, rows, 4, 3, bf16=False,
+                            speeds=[1.0, 2.0, 1.5])
+    run_both(w, 3, cuda_device, rows=rows)
+
+
 def test_softmax_regression_batch_512(cuda_device):
     """The largest batch of the fp32 round kernel (one thread per row): three
     rounds, shards that wrap, strict 1e-5 against the oracle."""
