@@ -160,6 +160,24 @@ __device__ __forceinline__ void bulk_copy_to_peer(void* dst, const void* src, ui
                : "memory");
 }
 
+// Address of the same shared-memory offset as `local` in CTA `rank` of the
+// cluster (a shared::cluster address).
+__device__ __forceinline__ uint32_t cluster_addr(const void* local, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(smem_u32(local)), "r"(rank));
+  return r;
+}
+
+// Asynchronous 16-byte store into another CTA's shared memory (both
+// addresses from cluster_addr, of the same CTA): the bytes complete on that
+// CTA's mbarrier `remote_bar`, whose waiter then sees the data.
+__device__ __forceinline__ void st_async_v4(uint32_t remote_addr, uint4 v, uint32_t remote_bar) {
+  asm volatile("st.async.shared::cluster.mbarrier::complete_tx::bytes.v4.b32 [%0], {%1, %2, %3, %4}, [%5];" ::"r"(
+                   remote_addr),
+               "r"(v.x), "r"(v.y), "r"(v.z), "r"(v.w), "r"(remote_bar)
+               : "memory");
+}
+
 __device__ __forceinline__ void prefetch_tmap(const CUtensorMap* map) {
   asm volatile("prefetch.tensormap [%0];" ::"l"(reinterpret_cast<uint64_t>(map)) : "memory");
 }

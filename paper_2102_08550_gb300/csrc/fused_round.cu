@@ -28,19 +28,22 @@
 //     128 units over its own input columns on tcgen05 (resident W0; the
 //     first X tiles are prefetched during the previous step).  With S = 2
 //     each CTA keeps 128/S of the units: the epilogue stores its own units'
-//     partials locally and the partner's into an outgoing buffer, which one
-//     bulk copy (async proxy, distributed shared memory) moves into the
-//     partner's incoming buffer, completing on the partner's mbarrier (a
-//     pairwise wait instead of a cluster barrier); then
+//     partials locally and writes the partner's straight into the partner's
+//     incoming buffer with asynchronous 16-byte stores (st.async, distributed
+//     shared memory) that complete on the partner's mbarrier (a pairwise
+//     wait instead of a cluster barrier); then
 //     z = (part_0 + part_1) + b0, h = relu(z), bf16;
-//  H  last layer for the CTA's units: partial logits, summed over the whole
-//     cluster in rank order through distributed shared memory, softmax
+//  H  last layer for the CTA's units: partial logits (double-buffered by
+//     step parity), summed over the whole cluster in rank order through
+//     distributed shared memory after one cluster barrier, softmax
 //     cross-entropy; the masked input gradient dz0[b][u] of its units is
 //     written (as bf16, 16-byte chunks of 8 samples) into the
-//     128-byte-swizzled K-major dz0^T tile of every CTA of its group (the A
-//     operand of step D); bias gradient and SGD
-//     of b0 (own units), of the head weights (own columns) and of the head
-//     bias;
+//     128-byte-swizzled K-major dz0^T tile (the A operand of step D); bias
+//     gradient and SGD of b0 (own units), of the head weights (own columns)
+//     and of the head bias.  With S = 2, once the CTA has read h for the
+//     last time in the step, its dz0^T rows go to the partner with st.async,
+//     completing on the partner's mbarrier, which the partner's MMA issuers
+//     wait on before step D (a pairwise wait, no cluster barrier);
 //  D  weight gradient of the group's 128 rows over the CTA's own input
 //     columns, dW0[o][k] = sum_b dz0[b][o] X[b][k], on tcgen05 in 32-column
 //     tiles (X^T tiles by TMA into a four-deep ring, the first ones during
@@ -53,9 +56,15 @@
 //
 // Ownership: a CTA rewrites only its own block of W0, its own b0 entries and
 // head-weight columns, and its private head bias, so its next step reads its
-// own writes; what it reads from other CTAs (partials, dz0 rows, logits) is
-// ordered by cluster barriers, and a buffer that other CTAs read is not
-// rewritten before a later barrier has proved those reads done.
+// own writes.  The logits it reads from other CTAs follow the cluster
+// barrier of the step; each buffer of partial logits is rewritten two steps
+// later, after the next step's barrier, which every reader has passed.  The
+// partner's partials and dz0 rows arrive on mbarriers (expected bytes set at
+// the start of each step).  The incoming partials land in the h tile: the
+// partner writes them in its next forward epilogue, which follows its step
+// D, which waits for this CTA's dz0 rows, which this CTA sends only after its
+// last read of h; so they never overwrite h in use.  A final cluster barrier
+// keeps every CTA resident until no peer can read its partial logits.
 // Generic-proxy writes that the tensor core reads are fenced with
 // fence.proxy.async.  Arithmetic and rounding points are those of the
 // per-layer path (the pair's two partial sums are added in rank order).
@@ -94,14 +103,6 @@ constexpr int kNXD = 4;                // X^T tile buffers in shared memory
 constexpr int kTAcc = 512 - 3 * kND;   // first TMEM column of the accumulators = master columns
 constexpr int kMaxKb = (kTAcc + kFBK - 1) / kFBK;   // resident K-blocks of W0
 constexpr int kW0Blk = kFU * kFBK * 2; // one resident K-block: 128 rows x 64 columns bf16
-
-__device__ __forceinline__ void st_dsmem_u32x4(void* local, uint32_t rank, uint4 v) {
-  uint32_t remote;
-  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(remote) : "r"(smem_u32(local)), "r"(rank));
-  asm volatile("st.shared::cluster.v4.u32 [%0], {%1, %2, %3, %4};" ::"r"(remote), "r"(v.x), "r"(v.y), "r"(v.z),
-               "r"(v.w)
-               : "memory");
-}
 
 __device__ __forceinline__ unsigned long long global_ns() {
   unsigned long long v;
@@ -142,6 +143,8 @@ struct FCfg {
   static constexpr int kFRing = kStagesF * kBBytes;
   static constexpr int kZs = B + 4;                         // row stride of the partial z exchange (floats)
   static constexpr int kZBytes = S > 1 ? kUPC * kZs * 4 : 0;  // own partials (the incoming ones alias hs)
+  static constexpr int kZTx = kUPC * B * 4;                 // partial bytes the partner sends per step
+  static constexpr int kDzTx = kUPC * B * 2;                // dz0^T bytes the partner sends per step
   static constexpr int kRegion = kDRing + (kFRing > kZBytes ? kFRing : kZBytes);   // D ring | F ring or z
   static constexpr int kDzT = kFU * 128;                    // dz0^T tile: 128 rows x 64 k (batch padded)
   static constexpr int kTpr = 256 / B;                      // threads per row, partial logits
@@ -156,8 +159,8 @@ struct FCfg {
   static constexpr int oHs = oDzT + kDzT;                    // [B][kHsd] float
   static constexpr int oWc = oHs + B * kHsd * 4;             // [C][kUPC] float (bf16 operand)
   static constexpr int oW1m = oWc + kFC * kUPC * 4;          // [C][kUPC] fp32 master head columns
-  static constexpr int oPl = oW1m + kFC * kUPC * 4;          // [B][C]
-  static constexpr int oDz = oPl + B * kFC * 4;              // [B][C]
+  static constexpr int oPl = oW1m + kFC * kUPC * 4;          // [2][B][C] partial logits by step parity
+  static constexpr int oDz = oPl + 2 * B * kFC * 4;          // [B][C]
   static constexpr int oDzb = oDz + B * kFC * 4;             // [C][B] (class-major)
   static constexpr int oGbp = oDzb + B * kFC * 4;            // [kChunks][kUPC]
   static constexpr int oRowLoss = oGbp + kChunks * kUPC * 4;   // [B]
@@ -168,7 +171,7 @@ struct FCfg {
   static constexpr int kBarBytes = 256;
   static constexpr int kSmem = oBar + kBarBytes + 1024;      // + alignment slack
   static_assert(S == 1 || kUPC * kZs <= B * kHsd, "the incoming partials must fit the h tile they alias");
-  static_assert(S == 1 || 2 * kZBytes <= kFRing, "own and outgoing partials must fit the F ring");
+  static_assert(S == 1 || kZBytes <= kFRing, "own partials must fit the F ring");
 };
 
 struct FusedArgs {
@@ -204,7 +207,6 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
   uint8_t* dring = sm + Cfg::oRegion;                // X^T tiles of step D
   uint8_t* fring = dring + Cfg::kDRing;              // X tiles of step F
   float* zx = reinterpret_cast<float*>(fring);       // [kUPC][kZs] own partials (S = 2), after the F MMAs
-  float* zout = zx + Cfg::kUPC * Cfg::kZs;           // [kUPC][kZs] the partner's partials, sent by bulk copy
   uint8_t* w0s = sm + Cfg::oW0;                      // resident bf16 W0 block
   uint8_t* dzT = sm + Cfg::oDzT;
   float* hs = reinterpret_cast<float*>(sm + Cfg::oHs);
@@ -232,7 +234,8 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
   uint64_t* xfreeD = fullD + kNXD;             // [kNXD] X^T tile consumed by its MMA
   uint64_t* accD = xfreeD + kNXD;              // [kNBD] TMEM buffer full
   uint64_t* pinF = accD + kNBD;                // [1] the partner's partials landed (S = 2)
-  uint64_t* ldW = pinF + 1;                    // [1] model tiles landed (prologue)
+  uint64_t* dzin = pinF + 1;                   // [1] the partner's dz0^T rows landed (S = 2)
+  uint64_t* ldW = dzin + 1;                    // [1] model tiles landed (prologue)
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(ldW + 1);
 
   const int rank = static_cast<int>(cluster_ctarank());
@@ -253,6 +256,7 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
   const int pre_f = nkf < Cfg::kStagesF ? nkf : Cfg::kStagesF;   // X tiles loaded ahead of a step
   const int pre_d = nD < kNXD ? nD : kNXD;                       // X^T tiles loaded before step D
   const int64_t gso = static_cast<int64_t>(a.global_slot) * a.slot_stride;
+  const int partner = grp * S + (half ^ 1);     // S = 2: the other CTA of the group
 
   if (t == 0) {
     prefetch_tmap(&mX);
@@ -270,6 +274,7 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
     }
     for (int i = 0; i < kNBD; ++i) mbar_init(&accD[i], 1);
     mbar_init(pinF, 1);
+    mbar_init(dzin, 1);
     mbar_init(ldW, 1);
     fence_barrier_init();
     fence_proxy_async_smem();
@@ -396,7 +401,10 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
       if (stamp) a.phase_ts[s * 4 + 0] = global_ns();
       const bool last = s == tau - 1;
       const int sg = sg0 + s;
-      if (S > 1 && t == 0) mbar_arrive_expect_tx(pinF, Cfg::kZBytes);   // this step's incoming partials
+      if (S > 1 && t == 0) {   // what the partner sends this step: its partials and its dz0^T rows
+        mbar_arrive_expect_tx(pinF, Cfg::kZTx);
+        mbar_arrive_expect_tx(dzin, Cfg::kDzTx);
+      }
 
       // ------------------------------------------------------------ F: partial forward of the group's units
       if (warp == 0 && lane == 0) {
@@ -436,14 +444,22 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
               for (int j = 0; j < 32; ++j) hs[(c0 + j) * Cfg::kHsd + u] = bf16_round(fmaxf(v[j] + bias, 0.f));
             } else {
               // the partial goes to the CTA that keeps unit u: this one
-              // (own rows) or, through the outgoing buffer, the partner
+              // (own rows) or the partner (its incoming buffer)
               const int owner = u / UPC;
-              float* row = (owner == half ? zx : zout) + (u - owner * UPC) * Cfg::kZs + c0;
+              const int off = (u - owner * UPC) * Cfg::kZs + c0;
+              if (owner == half) {
 #pragma unroll
-              for (int q = 0; q < 8; ++q)
-                *reinterpret_cast<float4*>(row + 4 * q) =
-                    make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
-              fence_proxy_async_smem();   // the outgoing rows are read by the bulk copy
+                for (int q = 0; q < 8; ++q)
+                  *reinterpret_cast<float4*>(zx + off + 4 * q) =
+                      make_float4(v[4 * q], v[4 * q + 1], v[4 * q + 2], v[4 * q + 3]);
+              } else {   // 16-byte asynchronous stores, counted on the partner's barrier
+                const uint32_t dst = cluster_addr(zin + off, partner), bar = cluster_addr(pinF, partner);
+#pragma unroll
+                for (int q = 0; q < 8; ++q)
+                  st_async_v4(dst + 16 * q, make_uint4(__float_as_uint(v[4 * q]), __float_as_uint(v[4 * q + 1]),
+                                                       __float_as_uint(v[4 * q + 2]), __float_as_uint(v[4 * q + 3])),
+                              bar);
+              }
             }
           }
         }
@@ -451,10 +467,8 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
       tc_fence_before();
       __syncthreads();
       if (S > 1) {
-        // the partner's partials of this CTA's units: one bulk copy each way
-        // into the incoming buffer, completing on the receiver's barrier
-        if (t == 0) bulk_copy_to_peer(zin, zout, Cfg::kZBytes, pinF, grp * S + (half ^ 1));
-        // both partials of this CTA's units are local now:
+        // both partials of this CTA's units are local once the partner's
+        // stores have landed:
         // z = part(half 0) + part(half 1) + b0
         mbar_wait(pinF, sg & 1, a.err, kDevTimeoutFull);
         constexpr int kZItems = UPC * (B / 4), kZPer = (kZItems + kFT - 1) / kFT;
@@ -498,6 +512,7 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
       if (stamp) a.phase_ts[s * 4 + 1] = global_ns();
 
       // ------------------------------------------------------------ H: last layer for this CTA's units
+      float* plb = pl + (sg & 1) * B * kFC;   // this step's partial logits (read by every CTA)
       if (t < 256) {   // partial logits: kTpr threads per row, all classes in registers
         const int rb = t / Cfg::kTpr, q = t % Cfg::kTpr;
         float acc[kFC];
@@ -517,25 +532,21 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
 #pragma unroll
         for (int c = 0; c < kFC; ++c) {
           for (int o = Cfg::kTpr / 2; o > 0; o >>= 1) acc[c] += __shfl_xor_sync(0xffffffffu, acc[c], o);
-          if (q == 0) pl[rb * kFC + c] = acc[c];
+          if (q == 0) plb[rb * kFC + c] = acc[c];
         }
       }
       cluster_sync();
       for (int q = t; q < B * kFC; q += kFT) {
         float part[kFMaxCluster];
 #pragma unroll
-        for (int r = 0; r < kFMaxCluster; ++r) part[r] = r < ncl ? ld_dsmem_f32(pl + q, r) : 0.f;
+        for (int r = 0; r < kFMaxCluster; ++r) part[r] = r < ncl ? ld_dsmem_f32(plb + q, r) : 0.f;
         float acc = 0.f;
 #pragma unroll
         for (int r = 0; r < kFMaxCluster; ++r)
           if (r < ncl) acc += part[r];
         dz[q] = acc + b1m[q % kFC];
       }
-      // the softmax rows below read logits summed by other threads; with S = 1
-      // this barrier also separates the remote reads of pl from the next step's
-      // writes (with S = 2 the barrier after the dz0^T exchange does that)
-      if (S == 1) cluster_sync();
-      else __syncthreads();
+      __syncthreads();   // the softmax rows below read logits summed by other threads
       // softmax cross-entropy, four threads per row: thread q of the row takes
       // classes q, q + 4, q + 8 (exponentials and gradients); the row's
       // exponentials are gathered in every lane of the row and summed in class
@@ -594,7 +605,7 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
       }
       // masked input gradient dz0[b][u] of this CTA's units: item = (unit, 8
       // consecutive samples), one 16-byte chunk of the unit's K-major dz0^T
-      // row, stored here and into the other CTAs of the group
+      // row
       for (int it = t; it < UPC * Cfg::kChunks; it += kFT) {
         const int u = it % UPC, j = it / UPC;
         // dh[b] = sum over c in class order of dzb[c][b] w[c][u]: the eight
@@ -625,11 +636,7 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
         }
         const uint4 p = make_uint4(pack_bf16x2(dv[0], dv[1]), pack_bf16x2(dv[2], dv[3]), pack_bf16x2(dv[4], dv[5]),
                                    pack_bf16x2(dv[6], dv[7]));
-        uint8_t* dst = dzT + sw128_offset(ku0 + u, 8 * j);
-        *reinterpret_cast<uint4*>(dst) = p;
-#pragma unroll
-        for (int o = 0; o < S; ++o)
-          if (o != half) st_dsmem_u32x4(dst, grp * S + o, p);
+        *reinterpret_cast<uint4*>(dzT + sw128_offset(ku0 + u, 8 * j)) = p;
         gbp[j * UPC + u] = gsum;
       }
       fence_proxy_async_smem();   // dz0^T is read by the tensor core next
@@ -665,6 +672,13 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
         if (last) a.master_w[dof + a.offB0 + g0 + ku0 + t] = nb;
       }
       __syncthreads();
+      if (S > 1) {   // h is not read again this step: this CTA's dz0^T rows to the partner
+        const uint32_t dst = cluster_addr(dzT, partner), bar = cluster_addr(dzin, partner);
+        for (int it = t; it < UPC * Cfg::kChunks; it += kFT) {
+          const uint32_t off = sw128_offset(ku0 + it / Cfg::kChunks, 8 * (it % Cfg::kChunks));
+          st_async_v4(dst + off, *reinterpret_cast<const uint4*>(dzT + off), bar);
+        }
+      }
       // SGD of the head-weight columns: first half + second half of the batch
       for (int item = t; item < Cfg::kW1Items; item += kFT) {
         const int c = item / (UPC / 4), u4 = (item % (UPC / 4)) * 4;
@@ -681,10 +695,6 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
             make_float4(bf16_round(nw.x), bf16_round(nw.y), bf16_round(nw.z), bf16_round(nw.w));
         if (last)
           *reinterpret_cast<float4*>(a.master_w + dof + a.offW1 + static_cast<int64_t>(c) * H + g0 + ku0 + u4) = nw;
-      }
-      if (S > 1) {
-        cluster_sync();             // the partner's dz0^T rows have landed
-        fence_proxy_async_smem();
       }
       if (stamp) a.phase_ts[s * 4 + 2] = global_ns();
 
@@ -703,6 +713,10 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
         // waits on the named barrier stay paired
         const int e = warp == 1 ? 0 : 1;
         constexpr uint32_t idesc = idesc_bf16_f32(128, kND);
+        if (S > 1) {   // the partner's dz0^T rows (st.async) have landed before the tensor core reads them
+          if (chain_ok) chain_ok = mbar_wait(dzin, sg & 1, a.err, kDevTimeoutFull);
+          fence_proxy_async_smem();
+        }
         for (int tt = ((sg * nD + e) & 1); tt < nD; tt += 2) {
           const int c = sg * nD + tt, buf = e, use = c / kNBD, xb = c % kNXD;
           if (chain_ok) chain_ok = mbar_wait(&fullD[xb], (c / kNXD) & 1, a.err, kDevTimeoutFull);
@@ -799,6 +813,7 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
   }
   // the last drain of each chain's buffer pairs with one more wait
   if ((warp == 1 || warp == 3) && chain_tiles > 0) bar_named(1 + (warp == 1 ? 0 : 1), 128 + 32);
+  cluster_sync();   // peers may still read this CTA's partial logits of the last step
   tc_fence_before();
   __syncthreads();
   if (warp == 2) {
