@@ -117,6 +117,11 @@ __device__ __forceinline__ uint32_t sw128_offset(int row, int k) {
                                (k & 7) * 2);
 }
 
+// one bf16 value (round to nearest even) at a byte address of shared memory
+__device__ __forceinline__ void st_bf16(uint8_t* p, float v) {
+  *reinterpret_cast<__nv_bfloat16*>(p) = __float2bfloat16_rn(v);
+}
+
 // bf16 copy of columns [c0, c0 + 32) of row r (c0 a multiple of 32) into the
 // resident W0 operand: four 16-byte chunks of one swizzled 128-byte row
 __device__ __forceinline__ void put_w0_row32(uint8_t* w0s, int r, int c0, const float (&v)[32]) {
@@ -151,6 +156,18 @@ struct FCfg {
   static constexpr int kHsd = kUPC + 4 * kTpr;              // padded row stride of the float h tile
   static constexpr int kChunks = B / 8;                     // 8-sample chunks of a dz0^T row
   static constexpr int kW1Items = kFC * (kUPC / 4);         // (class, 4 units) items of the head update
+  // the last layer's three products on the tensor core (batch 64, two CTAs
+  // per group): operand tiles of 128-byte K-major rows in the forward X ring,
+  // which is idle between the forward's partial sums and step D
+  static constexpr bool kTCH = B == 64 && S == 2;
+  static constexpr int tH = 0;                               // h [b][u]: logits A (rows b)
+  static constexpr int tHT = 8192;                           // h^T [u][b]: head-gradient A (rows u)
+  static constexpr int tW1 = 16384;                          // W1 [c][u]: logits B (16 rows)
+  static constexpr int tW1T = 18432;                         // W1^T [u][c]: input-gradient A (K = 16 classes)
+  static constexpr int tDz = 26624;                          // dz1 [b][c]: input-gradient B (K = 16 classes)
+  static constexpr int tDzT = 34816;                         // dz1^T [c][b]: head-gradient B (16 rows)
+  static_assert(!kTCH || (kUPC == 64 && tDzT + 16 * 128 <= kFRing && tW1T + 128 * 128 <= kFRing),
+                "the head's operand tiles (and the 128-row reads of the A tiles) fit the F ring");
   static_assert(2 * kW1Items * 16 <= kStagesF * B * kFBK * 2, "head-update partials must fit the F ring");
   // shared memory carve-up (bytes, from a 1024-aligned base)
   static constexpr int oRegion = 0;
@@ -235,7 +252,9 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
   uint64_t* accD = xfreeD + kNXD;              // [kNBD] TMEM buffer full
   uint64_t* pinF = accD + kNBD;                // [1] the partner's partials landed (S = 2)
   uint64_t* dzin = pinF + 1;                   // [1] the partner's dz0^T rows landed (S = 2)
-  uint64_t* ldW = dzin + 1;                    // [1] model tiles landed (prologue)
+  uint64_t* accH1 = dzin + 1;                  // [1] partial logits (tensor-core head)
+  uint64_t* accH2 = accH1 + 1;                 // [1] input gradient and head-weight gradient (tensor-core head)
+  uint64_t* ldW = accH2 + 1;                   // [1] model tiles landed (prologue)
   uint32_t* tmem_slot = reinterpret_cast<uint32_t*>(ldW + 1);
 
   const int rank = static_cast<int>(cluster_ctarank());
@@ -275,6 +294,8 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
     for (int i = 0; i < kNBD; ++i) mbar_init(&accD[i], 1);
     mbar_init(pinF, 1);
     mbar_init(dzin, 1);
+    mbar_init(accH1, 1);
+    mbar_init(accH2, 1);
     mbar_init(ldW, 1);
     fence_barrier_init();
     fence_proxy_async_smem();
@@ -502,10 +523,43 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
           const int ug = ku0 + ul;                   // unit within the group
           const float4 z = zr[k];
           const float bias = b0m[ug];
-          hs[(b4 + 0) * Cfg::kHsd + ul] = bf16_round(fmaxf(z.x + bias, 0.f));
-          hs[(b4 + 1) * Cfg::kHsd + ul] = bf16_round(fmaxf(z.y + bias, 0.f));
-          hs[(b4 + 2) * Cfg::kHsd + ul] = bf16_round(fmaxf(z.z + bias, 0.f));
-          hs[(b4 + 3) * Cfg::kHsd + ul] = bf16_round(fmaxf(z.w + bias, 0.f));
+          const float h0 = bf16_round(fmaxf(z.x + bias, 0.f)), h1 = bf16_round(fmaxf(z.y + bias, 0.f));
+          const float h2 = bf16_round(fmaxf(z.z + bias, 0.f)), h3 = bf16_round(fmaxf(z.w + bias, 0.f));
+          hs[(b4 + 0) * Cfg::kHsd + ul] = h0;
+          hs[(b4 + 1) * Cfg::kHsd + ul] = h1;
+          hs[(b4 + 2) * Cfg::kHsd + ul] = h2;
+          hs[(b4 + 3) * Cfg::kHsd + ul] = h3;
+          if constexpr (Cfg::kTCH) {   // h as the tensor core reads it, both ways
+            st_bf16(fring + Cfg::tH + sw128_offset(b4 + 0, ul), h0);
+            st_bf16(fring + Cfg::tH + sw128_offset(b4 + 1, ul), h1);
+            st_bf16(fring + Cfg::tH + sw128_offset(b4 + 2, ul), h2);
+            st_bf16(fring + Cfg::tH + sw128_offset(b4 + 3, ul), h3);
+            *reinterpret_cast<uint2*>(fring + Cfg::tHT + sw128_offset(ul, b4)) =
+                make_uint2(pack_bf16x2(h0, h1), pack_bf16x2(h2, h3));
+          }
+        }
+        if constexpr (Cfg::kTCH) {
+          // this CTA's head columns (bf16 values) as the tensor core reads
+          // them: W1 [c][u] (rows c < 10) and W1^T [u][c] (classes 10..15
+          // zero: they multiply the zero classes of dz1)
+          for (int it = t; it < kFC * (UPC / 8) + UPC * 2; it += kFT) {
+            if (it < kFC * (UPC / 8)) {
+              const int c = it / (UPC / 8), u8 = (it % (UPC / 8)) * 8;
+              const float* w = wcs + c * UPC + u8;
+              *reinterpret_cast<uint4*>(fring + Cfg::tW1 + sw128_offset(c, u8)) =
+                  make_uint4(pack_bf16x2(w[0], w[1]), pack_bf16x2(w[2], w[3]), pack_bf16x2(w[4], w[5]),
+                             pack_bf16x2(w[6], w[7]));
+            } else {
+              const int i2 = it - kFC * (UPC / 8), u = i2 >> 1, c8 = (i2 & 1) * 8;
+              float w[8];
+#pragma unroll
+              for (int i = 0; i < 8; ++i) w[i] = c8 + i < kFC ? wcs[(c8 + i) * UPC + u] : 0.f;
+              *reinterpret_cast<uint4*>(fring + Cfg::tW1T + sw128_offset(u, c8)) =
+                  make_uint4(pack_bf16x2(w[0], w[1]), pack_bf16x2(w[2], w[3]), pack_bf16x2(w[4], w[5]),
+                             pack_bf16x2(w[6], w[7]));
+            }
+          }
+          fence_proxy_async_smem();   // the tiles are read by the tensor core
         }
         __syncthreads();
       }
@@ -513,7 +567,31 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
 
       // ------------------------------------------------------------ H: last layer for this CTA's units
       float* plb = pl + (sg & 1) * B * kFC;   // this step's partial logits (read by every CTA)
-      if (t < 256) {   // partial logits: kTpr threads per row, all classes in registers
+      if constexpr (Cfg::kTCH) {
+        // partial logits plb[b][c] = sum over this CTA's units of h[b][u] W1[c][u]:
+        // M = 128 (rows b < 64 used), N = 16 (classes < 10 used), K = 64 units
+        if (warp == 1 && lane == 0) {
+          tc_fence_after();
+          constexpr uint32_t idesc = idesc_bf16_f32(128, 16);
+          const uint32_t ha = smem_u32(fring + Cfg::tH), wb = smem_u32(fring + Cfg::tW1);
+#pragma unroll
+          for (int j = 0; j < kFBK / 16; ++j)
+            umma_bf16(tmem + kTAcc + 64, smem_desc_k128(ha + j * 32), smem_desc_k128(wb + j * 32), idesc, j != 0 ? 1u : 0u);
+          umma_commit(accH1);
+        } else if (warp == 4 || warp == 5) {   // lanes 0..63: one sample each
+          int ok = mbar_wait(accH1, sg & 1, a.err, kDevTimeoutAccum) ? 1 : 0;
+          ok = __all_sync(0xffffffffu, ok);
+          tc_fence_after();
+          if (ok) {
+            float v[16];
+            tmem_ld_32x32b_x16(tmem + (static_cast<uint32_t>((warp & 3) * 32) << 16) + kTAcc + 64, v);
+            const int b = (warp & 3) * 32 + lane;
+#pragma unroll
+            for (int c = 0; c < kFC; ++c) plb[b * kFC + c] = v[c];
+          }
+          tc_fence_before();
+        }
+      } else if (t < 256) {   // partial logits: kTpr threads per row, all classes in registers
         const int rb = t / Cfg::kTpr, q = t % Cfg::kTpr;
         float acc[kFC];
 #pragma unroll
@@ -573,16 +651,26 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
         if (q == (y & 3)) rowloss[b] = m + logf(se) - (y < 4 ? zq[0] : y < 8 ? zq[1] : zq[2]);
         const float inv = 1.0f / static_cast<float>(B);
 #pragma unroll
-        for (int i = 0; i < 3; ++i) {
+        for (int i = 0; i < 4; ++i) {
           const int c = q + 4 * i;
-          if (c < kFC) {
-            const float g = (c == y ? -(so_ / se) : eq[i] / se) * inv;
+          if (i < 3 && c < kFC) {
+            const float g = (c == y ? -(so_ / se) : eq[i < 3 ? i : 2] / se) * inv;
             dz[b * kFC + c] = g;
-            dzb[c * B + b] = bf16_round(g);
+            if constexpr (Cfg::kTCH) {   // dz1 as the tensor core reads it, both ways
+              st_bf16(fring + Cfg::tDz + sw128_offset(b, c), g);
+              st_bf16(fring + Cfg::tDzT + sw128_offset(c, b), g);
+            } else {
+              dzb[c * B + b] = bf16_round(g);
+            }
+          } else if (Cfg::kTCH) {
+            st_bf16(fring + Cfg::tDz + sw128_offset(b, c), 0.f);   // classes 10..15 of the K = 16 operand
           }
         }
       }
+      if constexpr (Cfg::kTCH) fence_proxy_async_smem();   // the dz1 tiles are read by the tensor core
+      tc_fence_before();
       __syncthreads();
+      tc_fence_after();
       if (rank == 0 && t == 0) {
         for (int c = 0; c < B / kRowsPerLossChunk; ++c) {
           float l = 0.f;
@@ -603,75 +691,73 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
           if (last && rank == 0) a.master_w[dof + a.offB1 + c] = nb;
         }
       }
-      // masked input gradient dz0[b][u] of this CTA's units: item = (unit, 8
-      // consecutive samples), one 16-byte chunk of the unit's K-major dz0^T
-      // row
-      for (int it = t; it < UPC * Cfg::kChunks; it += kFT) {
-        const int u = it % UPC, j = it / UPC;
-        // dh[b] = sum over c in class order of dzb[c][b] w[c][u]: the eight
-        // samples of a class are two 16-byte loads of the class-major dzb
-        float dv[8];
+      if constexpr (Cfg::kTCH) {
+        // the input gradient dh^T[u][b] = sum_c W1^T[u][c] dz1[b][c] (M = 128
+        // with rows u < 64 used, N = 64 samples, K = 16 classes) and the
+        // head-weight gradient dW1^T[u][c] = sum_b h^T[u][b] dz1^T[c][b]
+        // (N = 16 with classes < 10 used, K = 64 samples), one commit
+        if (warp == 1 && lane == 0) {
+          umma_bf16(tmem + kTAcc, smem_desc_k128(smem_u32(fring + Cfg::tW1T)), smem_desc_k128(smem_u32(fring + Cfg::tDz)),
+                    idesc_bf16_f32(128, B), 0u);
+          constexpr uint32_t idesc = idesc_bf16_f32(128, 16);
+          const uint32_t ha = smem_u32(fring + Cfg::tHT), gb = smem_u32(fring + Cfg::tDzT);
 #pragma unroll
-        for (int i = 0; i < 8; ++i) dv[i] = 0.f;
+          for (int j = 0; j < kFBK / 16; ++j)
+            umma_bf16(tmem + kTAcc + 64, smem_desc_k128(ha + j * 32), smem_desc_k128(gb + j * 32), idesc, j != 0 ? 1u : 0u);
+          umma_commit(accH2);
+        } else if (warp == 4 || warp == 5) {
+          // unit u = (warp & 3) * 32 + lane: its masked dz0 row (bf16 into the
+          // K-major dz0^T tile, the A operand of step D) and its b0 (the sum
+          // of the fp32 masked gradient)
+          int ok = mbar_wait(accH2, sg & 1, a.err, kDevTimeoutAccum) ? 1 : 0;
+          ok = __all_sync(0xffffffffu, ok);
+          tc_fence_after();
+          const int u = (warp & 3) * 32 + lane;
+          const uint32_t trow = tmem + (static_cast<uint32_t>((warp & 3) * 32) << 16) + kTAcc;
+          float gsum = 0.f;
+          if (ok) {
+            for (int c0 = 0; c0 < B; c0 += 32) {
+              float v[32];
+              tmem_ld_32x32b_x32(trow + c0, v);
 #pragma unroll
-        for (int c = 0; c < kFC; ++c) {
-          const float wc = wcs[c * UPC + u];
-          const float4 d0 = *reinterpret_cast<const float4*>(dzb + c * B + 8 * j);
-          const float4 d1 = *reinterpret_cast<const float4*>(dzb + c * B + 8 * j + 4);
-          dv[0] = fmaf(d0.x, wc, dv[0]);
-          dv[1] = fmaf(d0.y, wc, dv[1]);
-          dv[2] = fmaf(d0.z, wc, dv[2]);
-          dv[3] = fmaf(d0.w, wc, dv[3]);
-          dv[4] = fmaf(d1.x, wc, dv[4]);
-          dv[5] = fmaf(d1.y, wc, dv[5]);
-          dv[6] = fmaf(d1.z, wc, dv[6]);
-          dv[7] = fmaf(d1.w, wc, dv[7]);
-        }
-        float gsum = 0.f;
+              for (int i = 0; i < 32; ++i) {
+                const float dh = hs[(c0 + i) * Cfg::kHsd + u] > 0.f ? v[i] : 0.f;
+                v[i] = dh;
+                gsum += dh;
+              }
 #pragma unroll
-        for (int i = 0; i < 8; ++i) {
-          const float dh = hs[(8 * j + i) * Cfg::kHsd + u] > 0.f ? dv[i] : 0.f;
-          dv[i] = dh;
-          gsum += dh;
-        }
-        const uint4 p = make_uint4(pack_bf16x2(dv[0], dv[1]), pack_bf16x2(dv[2], dv[3]), pack_bf16x2(dv[4], dv[5]),
-                                   pack_bf16x2(dv[6], dv[7]));
-        *reinterpret_cast<uint4*>(dzT + sw128_offset(ku0 + u, 8 * j)) = p;
-        gbp[j * UPC + u] = gsum;
-      }
-      fence_proxy_async_smem();   // dz0^T is read by the tensor core next
-      __syncthreads();
-      // head weight gradient of this CTA's columns, item = (class, 4 units),
-      // split over the two halves of the batch (partials in the idle F ring)
-      float4* w1p = reinterpret_cast<float4*>(fring);   // [2][kW1Items]
-      for (int q = t; q < 2 * Cfg::kW1Items; q += kFT) {
-        const int item = q % Cfg::kW1Items, hb = q / Cfg::kW1Items;
-        const int c = item / (UPC / 4), u4 = (item % (UPC / 4)) * 4;
-        float4 dw = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll 2
-        for (int b4 = hb * (B / 2); b4 < (hb + 1) * (B / 2); b4 += 4) {
-          const float4 g4 = *reinterpret_cast<const float4*>(dzb + c * B + b4);   // samples b4 .. b4 + 3
-          const float gk[4] = {g4.x, g4.y, g4.z, g4.w};
-#pragma unroll
-          for (int k = 0; k < 4; ++k) {
-            const float4 hv = *reinterpret_cast<const float4*>(hs + (b4 + k) * Cfg::kHsd + u4);
-            dw.x = fmaf(gk[k], hv.x, dw.x);
-            dw.y = fmaf(gk[k], hv.y, dw.y);
-            dw.z = fmaf(gk[k], hv.z, dw.z);
-            dw.w = fmaf(gk[k], hv.w, dw.w);
+              for (int k = 0; k < 4; ++k)
+                *reinterpret_cast<uint4*>(dzT + sw128_offset(ku0 + u, c0 + 8 * k)) =
+                    make_uint4(pack_bf16x2(v[8 * k], v[8 * k + 1]), pack_bf16x2(v[8 * k + 2], v[8 * k + 3]),
+                               pack_bf16x2(v[8 * k + 4], v[8 * k + 5]), pack_bf16x2(v[8 * k + 6], v[8 * k + 7]));
+            }
           }
-        }
-        w1p[hb * Cfg::kW1Items + item] = dw;
-      }
-      if (t < UPC) {   // b0 of this CTA's units (chunk sums in chunk order)
-        float g = 0.f;
+          const float nb = fmaf(-a.lr, gsum, b0m[ku0 + u]);
+          b0m[ku0 + u] = nb;
+          if (last) a.master_w[dof + a.offB0 + g0 + ku0 + u] = nb;
+          tc_fence_before();
+        } else if (warp == 8 || warp == 9) {
+          // SGD of the head-weight column of unit u = (warp & 3) * 32 + lane
+          int ok = mbar_wait(accH2, sg & 1, a.err, kDevTimeoutAccum) ? 1 : 0;
+          ok = __all_sync(0xffffffffu, ok);
+          tc_fence_after();
+          const int u = (warp & 3) * 32 + lane;
+          if (ok) {
+            float v[16];
+            tmem_ld_32x32b_x16(tmem + (static_cast<uint32_t>((warp & 3) * 32) << 16) + kTAcc + 64, v);
 #pragma unroll
-        for (int r = 0; r < Cfg::kChunks; ++r) g += gbp[r * UPC + t];
-        const float nb = fmaf(-a.lr, g, b0m[ku0 + t]);
-        b0m[ku0 + t] = nb;
-        if (last) a.master_w[dof + a.offB0 + g0 + ku0 + t] = nb;
-      }
-      __syncthreads();
+            for (int c = 0; c < kFC; ++c) {
+              const float nw = fmaf(-a.lr, v[c], w1m[c * UPC + u]);
+              w1m[c * UPC + u] = nw;
+              wcs[c * UPC + u] = bf16_round(nw);
+              if (last) a.master_w[dof + a.offW1 + static_cast<int64_t>(c) * H + g0 + ku0 + u] = nw;
+            }
+          }
+          tc_fence_before();
+        }
+        fence_proxy_async_smem();   // dz0^T is read by the tensor core next
+        __syncthreads();
+        tc_fence_after();
       if (S > 1) {   // h is not read again this step: this CTA's dz0^T rows to the partner
         const uint32_t dst = cluster_addr(dzT, partner), bar = cluster_addr(dzin, partner);
         for (int it = t; it < UPC * Cfg::kChunks; it += kFT) {
@@ -679,22 +765,100 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
           st_async_v4(dst + off, *reinterpret_cast<const uint4*>(dzT + off), bar);
         }
       }
-      // SGD of the head-weight columns: first half + second half of the batch
-      for (int item = t; item < Cfg::kW1Items; item += kFT) {
-        const int c = item / (UPC / 4), u4 = (item % (UPC / 4)) * 4;
-        const float4 d0 = w1p[item], d1 = w1p[Cfg::kW1Items + item];
-        const float4 dw = make_float4(d0.x + d1.x, d0.y + d1.y, d0.z + d1.z, d0.w + d1.w);
-        const float4 o = *reinterpret_cast<const float4*>(w1m + c * UPC + u4);
-        float4 nw;
-        nw.x = fmaf(-a.lr, dw.x, o.x);
-        nw.y = fmaf(-a.lr, dw.y, o.y);
-        nw.z = fmaf(-a.lr, dw.z, o.z);
-        nw.w = fmaf(-a.lr, dw.w, o.w);
-        *reinterpret_cast<float4*>(w1m + c * UPC + u4) = nw;
-        *reinterpret_cast<float4*>(wcs + c * UPC + u4) =
-            make_float4(bf16_round(nw.x), bf16_round(nw.y), bf16_round(nw.z), bf16_round(nw.w));
-        if (last)
-          *reinterpret_cast<float4*>(a.master_w + dof + a.offW1 + static_cast<int64_t>(c) * H + g0 + ku0 + u4) = nw;
+      } else {
+        // masked input gradient dz0[b][u] of this CTA's units: item = (unit, 8
+        // consecutive samples), one 16-byte chunk of the unit's K-major dz0^T
+        // row
+        for (int it = t; it < UPC * Cfg::kChunks; it += kFT) {
+          const int u = it % UPC, j = it / UPC;
+          // dh[b] = sum over c in class order of dzb[c][b] w[c][u]: the eight
+          // samples of a class are two 16-byte loads of the class-major dzb
+          float dv[8];
+#pragma unroll
+          for (int i = 0; i < 8; ++i) dv[i] = 0.f;
+#pragma unroll
+          for (int c = 0; c < kFC; ++c) {
+            const float wc = wcs[c * UPC + u];
+            const float4 d0 = *reinterpret_cast<const float4*>(dzb + c * B + 8 * j);
+            const float4 d1 = *reinterpret_cast<const float4*>(dzb + c * B + 8 * j + 4);
+            dv[0] = fmaf(d0.x, wc, dv[0]);
+            dv[1] = fmaf(d0.y, wc, dv[1]);
+            dv[2] = fmaf(d0.z, wc, dv[2]);
+            dv[3] = fmaf(d0.w, wc, dv[3]);
+            dv[4] = fmaf(d1.x, wc, dv[4]);
+            dv[5] = fmaf(d1.y, wc, dv[5]);
+            dv[6] = fmaf(d1.z, wc, dv[6]);
+            dv[7] = fmaf(d1.w, wc, dv[7]);
+          }
+          float gsum = 0.f;
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            const float dh = hs[(8 * j + i) * Cfg::kHsd + u] > 0.f ? dv[i] : 0.f;
+            dv[i] = dh;
+            gsum += dh;
+          }
+          const uint4 p = make_uint4(pack_bf16x2(dv[0], dv[1]), pack_bf16x2(dv[2], dv[3]), pack_bf16x2(dv[4], dv[5]),
+                                     pack_bf16x2(dv[6], dv[7]));
+          *reinterpret_cast<uint4*>(dzT + sw128_offset(ku0 + u, 8 * j)) = p;
+          gbp[j * UPC + u] = gsum;
+        }
+        fence_proxy_async_smem();   // dz0^T is read by the tensor core next
+        __syncthreads();
+        // head weight gradient of this CTA's columns, item = (class, 4 units),
+        // split over the two halves of the batch (partials in the idle F ring)
+        float4* w1p = reinterpret_cast<float4*>(fring);   // [2][kW1Items]
+        for (int q = t; q < 2 * Cfg::kW1Items; q += kFT) {
+          const int item = q % Cfg::kW1Items, hb = q / Cfg::kW1Items;
+          const int c = item / (UPC / 4), u4 = (item % (UPC / 4)) * 4;
+          float4 dw = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll 2
+          for (int b4 = hb * (B / 2); b4 < (hb + 1) * (B / 2); b4 += 4) {
+            const float4 g4 = *reinterpret_cast<const float4*>(dzb + c * B + b4);   // samples b4 .. b4 + 3
+            const float gk[4] = {g4.x, g4.y, g4.z, g4.w};
+#pragma unroll
+            for (int k = 0; k < 4; ++k) {
+              const float4 hv = *reinterpret_cast<const float4*>(hs + (b4 + k) * Cfg::kHsd + u4);
+              dw.x = fmaf(gk[k], hv.x, dw.x);
+              dw.y = fmaf(gk[k], hv.y, dw.y);
+              dw.z = fmaf(gk[k], hv.z, dw.z);
+              dw.w = fmaf(gk[k], hv.w, dw.w);
+            }
+          }
+          w1p[hb * Cfg::kW1Items + item] = dw;
+        }
+        if (t < UPC) {   // b0 of this CTA's units (chunk sums in chunk order)
+          float g = 0.f;
+#pragma unroll
+          for (int r = 0; r < Cfg::kChunks; ++r) g += gbp[r * UPC + t];
+          const float nb = fmaf(-a.lr, g, b0m[ku0 + t]);
+          b0m[ku0 + t] = nb;
+          if (last) a.master_w[dof + a.offB0 + g0 + ku0 + t] = nb;
+        }
+        __syncthreads();
+        if (S > 1) {   // h is not read again this step: this CTA's dz0^T rows to the partner
+          const uint32_t dst = cluster_addr(dzT, partner), bar = cluster_addr(dzin, partner);
+          for (int it = t; it < UPC * Cfg::kChunks; it += kFT) {
+            const uint32_t off = sw128_offset(ku0 + it / Cfg::kChunks, 8 * (it % Cfg::kChunks));
+            st_async_v4(dst + off, *reinterpret_cast<const uint4*>(dzT + off), bar);
+          }
+        }
+        // SGD of the head-weight columns: first half + second half of the batch
+        for (int item = t; item < Cfg::kW1Items; item += kFT) {
+          const int c = item / (UPC / 4), u4 = (item % (UPC / 4)) * 4;
+          const float4 d0 = w1p[item], d1 = w1p[Cfg::kW1Items + item];
+          const float4 dw = make_float4(d0.x + d1.x, d0.y + d1.y, d0.z + d1.z, d0.w + d1.w);
+          const float4 o = *reinterpret_cast<const float4*>(w1m + c * UPC + u4);
+          float4 nw;
+          nw.x = fmaf(-a.lr, dw.x, o.x);
+          nw.y = fmaf(-a.lr, dw.y, o.y);
+          nw.z = fmaf(-a.lr, dw.z, o.z);
+          nw.w = fmaf(-a.lr, dw.w, o.w);
+          *reinterpret_cast<float4*>(w1m + c * UPC + u4) = nw;
+          *reinterpret_cast<float4*>(wcs + c * UPC + u4) =
+              make_float4(bf16_round(nw.x), bf16_round(nw.y), bf16_round(nw.z), bf16_round(nw.w));
+          if (last)
+            *reinterpret_cast<float4*>(a.master_w + dof + a.offW1 + static_cast<int64_t>(c) * H + g0 + ku0 + u4) = nw;
+        }
       }
       if (stamp) a.phase_ts[s * 4 + 2] = global_ns();
 
