@@ -162,12 +162,13 @@ struct FCfg {
   static constexpr bool kTCH = B == 64 && S == 2;
   static constexpr int tH = 0;                               // h [b][u]: logits A (rows b)
   static constexpr int tHT = 8192;                           // h^T [u][b]: head-gradient A (rows u)
-  static constexpr int tW1 = 16384;                          // W1 [c][u]: logits B (16 rows)
-  static constexpr int tW1T = 18432;                         // W1^T [u][c]: input-gradient A (K = 16 classes)
-  static constexpr int tDz = 26624;                          // dz1 [b][c]: input-gradient B (K = 16 classes)
-  static constexpr int tDzT = 34816;                         // dz1^T [c][b]: head-gradient B (16 rows)
+  static constexpr int tW1 = 18432;                          // W1 [c][u]: logits B (16 rows)
+  static constexpr int tW1T = 20480;                         // W1^T [u][c]: input-gradient A (K = 16 classes)
+  static constexpr int tDz = 28672;                          // dz1 [b][c]: input-gradient B (K = 16 classes)
+  static constexpr int tDzT = 36864;                         // dz1^T [c][b]: head-gradient B (16 rows)
   static_assert(!kTCH || (kUPC == 64 && tDzT + 16 * 128 <= kFRing && tW1T + 128 * 128 <= kFRing),
                 "the head's operand tiles (and the 128-row reads of the A tiles) fit the F ring");
+  static_assert(!kTCH || tW1 >= kZBytes, "the head-column tiles, written during the pair wait, clear the own partials");
   static_assert(2 * kW1Items * 16 <= kStagesF * B * kFBK * 2, "head-update partials must fit the F ring");
   // shared memory carve-up (bytes, from a 1024-aligned base)
   static constexpr int oRegion = 0;
@@ -488,6 +489,29 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
       tc_fence_before();
       __syncthreads();
       if (S > 1) {
+        if constexpr (Cfg::kTCH) {
+          // while the partner's partials are on their way: this CTA's head
+          // columns (bf16 values) as the tensor core reads them, W1 [c][u]
+          // (rows c < 10) and W1^T [u][c] (classes 10..15 zero: they multiply
+          // the zero classes of dz1), clear of the own partials in the F ring
+          for (int it = t; it < kFC * (UPC / 8) + UPC * 2; it += kFT) {
+            if (it < kFC * (UPC / 8)) {
+              const int c = it / (UPC / 8), u8 = (it % (UPC / 8)) * 8;
+              const float* w = wcs + c * UPC + u8;
+              *reinterpret_cast<uint4*>(fring + Cfg::tW1 + sw128_offset(c, u8)) =
+                  make_uint4(pack_bf16x2(w[0], w[1]), pack_bf16x2(w[2], w[3]), pack_bf16x2(w[4], w[5]),
+                             pack_bf16x2(w[6], w[7]));
+            } else {
+              const int i2 = it - kFC * (UPC / 8), u = i2 >> 1, c8 = (i2 & 1) * 8;
+              float w[8];
+#pragma unroll
+              for (int i = 0; i < 8; ++i) w[i] = c8 + i < kFC ? wcs[(c8 + i) * UPC + u] : 0.f;
+              *reinterpret_cast<uint4*>(fring + Cfg::tW1T + sw128_offset(u, c8)) =
+                  make_uint4(pack_bf16x2(w[0], w[1]), pack_bf16x2(w[2], w[3]), pack_bf16x2(w[4], w[5]),
+                             pack_bf16x2(w[6], w[7]));
+            }
+          }
+        }
         // both partials of this CTA's units are local once the partner's
         // stores have landed:
         // z = part(half 0) + part(half 1) + b0
@@ -538,29 +562,7 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
                 make_uint2(pack_bf16x2(h0, h1), pack_bf16x2(h2, h3));
           }
         }
-        if constexpr (Cfg::kTCH) {
-          // this CTA's head columns (bf16 values) as the tensor core reads
-          // them: W1 [c][u] (rows c < 10) and W1^T [u][c] (classes 10..15
-          // zero: they multiply the zero classes of dz1)
-          for (int it = t; it < kFC * (UPC / 8) + UPC * 2; it += kFT) {
-            if (it < kFC * (UPC / 8)) {
-              const int c = it / (UPC / 8), u8 = (it % (UPC / 8)) * 8;
-              const float* w = wcs + c * UPC + u8;
-              *reinterpret_cast<uint4*>(fring + Cfg::tW1 + sw128_offset(c, u8)) =
-                  make_uint4(pack_bf16x2(w[0], w[1]), pack_bf16x2(w[2], w[3]), pack_bf16x2(w[4], w[5]),
-                             pack_bf16x2(w[6], w[7]));
-            } else {
-              const int i2 = it - kFC * (UPC / 8), u = i2 >> 1, c8 = (i2 & 1) * 8;
-              float w[8];
-#pragma unroll
-              for (int i = 0; i < 8; ++i) w[i] = c8 + i < kFC ? wcs[(c8 + i) * UPC + u] : 0.f;
-              *reinterpret_cast<uint4*>(fring + Cfg::tW1T + sw128_offset(u, c8)) =
-                  make_uint4(pack_bf16x2(w[0], w[1]), pack_bf16x2(w[2], w[3]), pack_bf16x2(w[4], w[5]),
-                             pack_bf16x2(w[6], w[7]));
-            }
-          }
-          fence_proxy_async_smem();   // the tiles are read by the tensor core
-        }
+        if constexpr (Cfg::kTCH) fence_proxy_async_smem();   // the h tiles are read by the tensor core
         __syncthreads();
       }
       if (stamp) a.phase_ts[s * 4 + 1] = global_ns();
@@ -614,15 +616,28 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
         }
       }
       cluster_sync();
-      for (int q = t; q < B * kFC; q += kFT) {
-        float part[kFMaxCluster];
-#pragma unroll
-        for (int r = 0; r < kFMaxCluster; ++r) part[r] = r < ncl ? ld_dsmem_f32(plb + q, r) : 0.f;
-        float acc = 0.f;
+      // logits: the partials of every CTA of the cluster in rank order, then
+      // the bias; four consecutive logits per thread (16-byte remote loads)
+      static_assert((B * kFC) % 4 == 0 && (Cfg::oPl % 16) == 0, "16-byte items of the partial logits");
+      for (int q4 = t; q4 < B * kFC / 4; q4 += kFT) {
+        float4 part[kFMaxCluster];
 #pragma unroll
         for (int r = 0; r < kFMaxCluster; ++r)
-          if (r < ncl) acc += part[r];
-        dz[q] = acc + b1m[q % kFC];
+          part[r] = r < ncl ? ld_dsmem_f32x4(plb + 4 * q4, r) : make_float4(0.f, 0.f, 0.f, 0.f);
+        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+        for (int r = 0; r < kFMaxCluster; ++r)
+          if (r < ncl) {
+            acc.x += part[r].x;
+            acc.y += part[r].y;
+            acc.z += part[r].z;
+            acc.w += part[r].w;
+          }
+        const int q = 4 * q4;
+        dz[q] = acc.x + b1m[q % kFC];
+        dz[q + 1] = acc.y + b1m[(q + 1) % kFC];
+        dz[q + 2] = acc.z + b1m[(q + 2) % kFC];
+        dz[q + 3] = acc.w + b1m[(q + 3) % kFC];
       }
       __syncthreads();   // the softmax rows below read logits summed by other threads
       // softmax cross-entropy, four threads per row: thread q of the row takes
@@ -757,7 +772,6 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
         }
         fence_proxy_async_smem();   // dz0^T is read by the tensor core next
         __syncthreads();
-        tc_fence_after();
       if (S > 1) {   // h is not read again this step: this CTA's dz0^T rows to the partner
         const uint32_t dst = cluster_addr(dzT, partner), bar = cluster_addr(dzin, partner);
         for (int it = t; it < UPC * Cfg::kChunks; it += kFT) {
