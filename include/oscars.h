@@ -308,6 +308,22 @@ oscars_status oscars_profile_reset(oscars_ctx* ctx);
  */
 int32_t oscars_phase_times(oscars_ctx* ctx, int32_t cap, double* us);
 
+/*
+ * oscars_check_wait_timeout - exercise the failure path of the kernels'
+ * bounded waits.  Every wait of a kernel in this library on an mbarrier (a
+ * TMA stage, a tensor-core accumulator, a peer CTA's data) gives up after a
+ * fixed number of polls, records a code in the context's device error word
+ * and lets the kernel end, and the next call that reads results reports
+ * OSCARS_ETIMEOUT.  This call runs that path on purpose: one GPU thread waits
+ * `polls` polls (1 .. 2^20) on an mbarrier that nothing completes, on the
+ * context's stream, then the host reads and clears the error word as after a
+ * round.  It returns OSCARS_ETIMEOUT when the path works; the context stays
+ * usable.  Not a step of the method (the paper assumes steady workers and
+ * has no failure model).  Errors: EINVAL (NULL, polls out of range), ESTATE
+ * (FLAT mode: no kernel error word), ECUDA.
+ */
+oscars_status oscars_check_wait_timeout(oscars_ctx* ctx, int32_t polls);
+
 /* oscars_num_params - P of the context (canonical layout). */
 oscars_status oscars_num_params(const oscars_ctx* ctx, int64_t* P);
 

@@ -70,6 +70,7 @@ _SIGS = {
                                         POINTER(c_int64), POINTER(c_int32)]),
     "oscars_merge_weights": (c_int32, [c_int32, POINTER(c_int32), c_int32, POINTER(c_float)]),
     "oscars_read_replica": (c_int32, [c_void_p, c_int32, c_void_p]),
+    "oscars_check_wait_timeout": (c_int32, [c_void_p, c_int32]),
     "oscars_gemm_bf16_nt": (c_int32, [c_void_p, c_void_p, c_void_p, c_int32, c_int32, c_int32, c_void_p]),
     "oscars_profile_read": (c_int32, [c_void_p, c_int32, POINTER(ctypes.c_char_p), POINTER(c_double),
                                       POINTER(c_int32)]),
@@ -262,6 +263,12 @@ def oscars_eval_loss(ctx: int, x_ptr: int, y_ptr: int, n: int) -> float:
 
 def oscars_read_replica(ctx: int, k: int, dst_ptr: int):
     _check(lib().oscars_read_replica(c_void_p(ctx), k, c_void_p(dst_ptr)), c_void_p(ctx))
+
+
+def oscars_check_wait_timeout(ctx: int, polls: int):
+    """Run the kernels' bounded-wait failure path once (raises OscarsError
+    with OSCARS_ETIMEOUT when the path works)."""
+    _check(lib().oscars_check_wait_timeout(c_void_p(ctx), polls), c_void_p(ctx))
 
 
 def oscars_gemm_bf16_nt(a_ptr: int, b_ptr: int, c_ptr: int, M: int, N: int, K: int, stream: Optional[int] = None):

@@ -1928,6 +1928,15 @@ oscars_status oscars_eval_loss(oscars_ctx* c, const float* x, const int32_t* y, 
   return check_err_word(c);
 }
 
+oscars_status oscars_check_wait_timeout(oscars_ctx* c, int32_t polls) {
+  if (!c || polls < 1 || polls > (1 << 20)) return OSCARS_EINVAL;
+  if (!c->err) return fail(c, OSCARS_ESTATE, "the context has no kernel error word (FLAT mode)");
+  cudaError_t e = launch_wait_selfcheck(c->err, static_cast<uint32_t>(polls), c->stream);
+  if (e == cudaSuccess) e = cudaStreamSynchronize(c->stream);
+  if (e != cudaSuccess) return cuda_fail(c, e, "wait self-check");
+  return check_err_word(c);
+}
+
 oscars_status oscars_read_replica(oscars_ctx* c, int32_t k, float* dst) {
   if (!c || !dst) return OSCARS_EINVAL;
   if (!slotted(c)) return fail(c, OSCARS_ESTATE, "replicas exist in MLP and CNN mode only");

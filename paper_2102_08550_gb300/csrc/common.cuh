@@ -20,6 +20,7 @@ enum DevErr : int {
   kDevTimeoutFull = 1,   // MMA issuer gave up waiting for a TMA stage
   kDevTimeoutEmpty = 2,  // producer gave up waiting for a free stage
   kDevTimeoutAccum = 3,  // epilogue gave up waiting for the accumulator
+  kDevTimeoutCheck = 4,  // the self-check's wait ran out (as it must)
 };
 
 // ~2^22 polls with a short back-off: well over a second of waiting.
@@ -60,9 +61,10 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
 }
 
 // Bounded wait for the completion of phase `parity`.  Returns false (and
-// records `code` in *err) when the limit runs out.
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, int* err, int code) {
-  for (uint32_t i = 0; i < kSpinLimit; ++i) {
+// records `code` in *err) when `limit` polls have run out.
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, int* err, int code,
+                                          uint32_t limit = kSpinLimit) {
+  for (uint32_t i = 0; i < limit; ++i) {
     if (mbar_try_wait(bar, parity)) return true;
     if (i > 64) __nanosleep(64);
   }

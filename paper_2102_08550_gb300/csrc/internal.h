@@ -25,6 +25,10 @@ struct MergeArgs {
 cudaError_t launch_merge(const MergeArgs& a, float* x_g, int64_t P, float eta, bool replica,
                          cudaStream_t s, __nv_bfloat16* shadow = nullptr);
 
+// one thread waits `polls` polls on an mbarrier nothing completes, then
+// records its timeout code in *err (the bounded-wait failure path)
+cudaError_t launch_wait_selfcheck(int* err, uint32_t polls, cudaStream_t s);
+
 // ---------------------------------------------------------------- scheduler (host)
 int iteration_ticks(const double* speed, int n, int64_t Q, int64_t* t, const char** why);
 int schedule_solve(const int64_t* t, int n, int64_t M, int mode, int64_t* T_star,

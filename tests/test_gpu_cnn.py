@@ -5,8 +5,8 @@ fp32 summation-order differences), worker losses and eval loss within 1e-3.
 
 Cases: small runs of one and two residual blocks through two rounds (the
 second round starts from the merged model; 3 input channels take the im2col
-stem, 16 the nine-tap one), and the full-size workload
-(16 workers, batch 32) for one local step of two sampled workers."""
+stem, 16 the nine-tap one), and the full-size workload (16 workers, batch
+32) for one full round: every worker's replica and the merged model."""
 import dataclasses
 
 import numpy as np
@@ -90,29 +90,40 @@ def test_cnn_small_two_rounds(cuda_device, name, blocks, W, B, cin):
     assert abs(ge - oe) <= LOSS_RTOL * abs(oe), (ge, oe)
 
 
-def test_cnn_full_size_one_step_sampled(cuda_device):
-    """The 16-worker, batch-32 workload: one local step per worker, the
-    replicas of the first and the last worker against the oracle."""
+def test_cnn_full_size_one_round_every_worker(cuda_device):
+    """The 16-worker, batch-32 workload for one full round of its schedule (71
+    worker-steps, tau up to 6): every worker's pushed replica and the merged
+    model against the oracle (conditioning envelope per tensor), the schedule
+    exact and the worker losses within 1e-3."""
     w = synth.CFG6
-    rows = 2 * w.batch
+    t, T, mw, tau = oracle_schedule(w)
+    rows = int(tau.max()) * w.batch
     ctx, m, params0 = make_cnn_context(w, cuda_device, rows)
-    ctx.set_local_steps([1] * w.num_workers)
-    _, loss = ctx.local_steps()
-    t, _, _, _ = oracle_schedule(w)
-    for k in (0, w.num_workers - 1):
+    tau_g, loss = ctx.local_steps()
+    assert tau_g == tau.tolist()
+    reps = []
+    for k in range(w.num_workers):
         out = torch.empty(ctx.P, dtype=torch.float32, device=cuda_device)
         ctx.read_replica(k, out)
         torch.cuda.synchronize()
-        got = out.cpu().numpy()
-        Xk, yk = synth.shard_np(w, k, n=rows)
-
-        def worker_run():
-            state = orun.init_state(None, params0, t, w.M, tau_override=[1] * w.num_workers, model=m)
-            layers, l = orun.local_steps(state, k, (Xk, yk), w.batch, w.lr, obf16.round_bf16)
-            return m.flatten(layers), l
-        ref, lref = worker_run()
-        env = envelope(lambda: [worker_run()[0]], None, [ref], errors=lambda f, r: cnn_errors(m, f, r))[0]
-        assert_within(cnn_errors(m, got, ref), env, f"worker {k}")
-        assert abs(loss[k] - lref) <= LOSS_RTOL * abs(lref)
+        reps.append(out.cpu().numpy())
     ctx.push_merge()
+    merged = pull(ctx, cuda_device)
+    sch = ctx.schedule()
     ctx.close()
+    assert sch["T_star"] == T
+    shards_h = [synth.shard_np(w, k, n=rows) for k in range(w.num_workers)]
+
+    def oracle_run():
+        _, recs = orun.run(None, params0, shards_h, t_iter=t, M=w.M, rounds=1, batch=w.batch, lr=w.lr,
+                           bf16=True, model=m, keep_replicas=True)
+        return recs[0]
+
+    def flats(rec):
+        return [*rec.replicas, rec.x_g]
+    rec = oracle_run()
+    env = envelope(lambda: flats(oracle_run()), None, flats(rec), errors=lambda f, r: cnn_errors(m, f, r))
+    np.testing.assert_allclose(loss, rec.worker_loss, rtol=LOSS_RTOL)
+    for k in range(w.num_workers):
+        assert_within(cnn_errors(m, reps[k], rec.replicas[k]), env[k], f"worker {k} (tau {int(tau[k])})")
+    assert_within(cnn_errors(m, merged, rec.x_g), env[-1], "merged")

@@ -242,6 +242,30 @@ def test_softmax_regression_batch_512(cuda_device):
     run_both(w, 3, cuda_device, rows=1300)
 
 
+def test_bounded_wait_runs_out_and_context_stays_usable(cuda_device):
+    """A kernel wait that runs out (an mbarrier that nothing completes, 1000
+    polls) records its code in the context's error word: the host reports
+    ETIMEOUT and clears the word, and the next rounds run and match those of
+    a fresh context bit for bit (no fault, no hang, the GPU stays usable)."""
+    w = synth.TrainWorkload("wait-check", 2, [128, 128, 10], 32, 0.05, 64, 4, 1)
+    shards = device_shards(w, cuda_device, n=64)
+    a, _ = make_context(w, shards, cuda_device)
+    with pytest.raises(P.OscarsError) as e:
+        P.oscars_check_wait_timeout(a.handle, 1000)
+    assert e.value.status == P.OSCARS_ETIMEOUT
+    with pytest.raises(P.OscarsError) as e:
+        P.oscars_check_wait_timeout(a.handle, 0)
+    assert e.value.status == P.OSCARS_EINVAL
+    b, _ = make_context(w, shards, cuda_device)
+    for ctx in (a, b):
+        for _ in range(2):
+            ctx.local_steps()          # reads the error word: it must be clear again
+            ctx.push_merge()
+    np.testing.assert_array_equal(pull_flat(a, cuda_device), pull_flat(b, cuda_device))
+    a.close()
+    b.close()
+
+
 def test_create_out_of_device_memory(cuda_device):
     """A model whose W + 1 parameter slots cannot fit in device memory
     (65 x 8.6 GB): oscars_create returns ENOMEM, creates nothing, and leaves
