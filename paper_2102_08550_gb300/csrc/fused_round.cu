@@ -45,8 +45,9 @@
 //     completing on the partner's mbarrier, which the partner's MMA issuers
 //     wait on before step D (a pairwise wait, no cluster barrier);
 //  D  weight gradient of the group's 128 rows over the CTA's own input
-//     columns, dW0[o][k] = sum_b dz0[b][o] X[b][k], on tcgen05 in 32-column
-//     tiles (X^T tiles by TMA into a four-deep ring, the first ones during
+//     columns, dW0[o][k] = sum_b dz0[b][o] X[b][k], on tcgen05 in 48-column
+//     tiles (the last one 16 or 32 columns; X^T tiles of 48 rows by TMA into
+//     a four-deep ring, two slots per issuing chain, the first ones during
 //     step F).  The tiles alternate between two chains, each with its own
 //     issuing thread, TMEM buffer and epilogue warpgroup, so that one chain's
 //     MMA issue overlaps the other's epilogue; the epilogue reads the
@@ -83,9 +84,10 @@
 // epilogue warpgroups (each covering the 128 TMEM lanes), all warps share the
 // CUDA-core work of step H.
 //
-// TMEM columns: [0, kTAcc) fp32 master of the W0 block; [kTAcc, 512) the
-// forward accumulator (B columns) and, in step D, the two 32-column
-// weight-gradient buffers (the two uses never overlap in time).
+// TMEM columns: [0, kTAcc) fp32 master of the W0 block (416 columns); [kTAcc,
+// 512) the forward accumulator (B columns), the last layer's accumulators
+// and, in step D, the two 48-column weight-gradient buffers (the uses never
+// overlap in time).
 #include "common.cuh"
 #include "internal.h"
 
@@ -97,10 +99,11 @@ constexpr int kFU = 128;               // hidden units per group (tensor-core ro
 constexpr int kFC = 10;                // classes
 constexpr int kFMaxCluster = 8;
 constexpr int kFBK = 64;               // K-block (bf16 elements, 128 bytes)
-constexpr int kND = 32;                // columns per weight-gradient tile
+constexpr int kND = 32;                // columns per fp32 model tile (the load and the write-back)
+constexpr int kDT = 48;                // columns per weight-gradient tile
 constexpr int kNBD = 2;                // weight-gradient TMEM buffers (one per issuing chain)
-constexpr int kNXD = 4;                // X^T tile buffers in shared memory
-constexpr int kTAcc = 512 - 3 * kND;   // first TMEM column of the accumulators = master columns
+constexpr int kNXD = 4;                // X^T tile buffers in shared memory (even: two per issuing chain)
+constexpr int kTAcc = 512 - kNBD * kDT;   // first TMEM column of the accumulators = master columns (416)
 constexpr int kMaxKb = (kTAcc + kFBK - 1) / kFBK;   // resident K-blocks of W0
 constexpr int kW0Blk = kFU * kFBK * 2; // one resident K-block: 128 rows x 64 columns bf16
 
@@ -122,16 +125,18 @@ __device__ __forceinline__ void st_bf16(uint8_t* p, float v) {
   *reinterpret_cast<__nv_bfloat16*>(p) = __float2bfloat16_rn(v);
 }
 
-// bf16 copy of columns [c0, c0 + 32) of row r (c0 a multiple of 32) into the
-// resident W0 operand: four 16-byte chunks of one swizzled 128-byte row
-__device__ __forceinline__ void put_w0_row32(uint8_t* w0s, int r, int c0, const float (&v)[32]) {
-  uint8_t* blk = w0s + (c0 / kFBK) * kW0Blk;
-  const int k0 = c0 % kFBK;
+// bf16 copy of columns [c0, c0 + N) of row r (c0 a multiple of 8) into the
+// resident W0 operand: one 16-byte chunk of a swizzled 128-byte row per 8
+// columns, each in the K-block of its columns
+template <int N>
+__device__ __forceinline__ void put_w0_cols(uint8_t* w0s, int r, int c0, const float (&v)[N]) {
 #pragma unroll
-  for (int i = 0; i < 4; ++i)
-    *reinterpret_cast<uint4*>(blk + sw128_offset(r, k0 + 8 * i)) =
+  for (int i = 0; i < N / 8; ++i) {
+    const int col = c0 + 8 * i;
+    *reinterpret_cast<uint4*>(w0s + (col / kFBK) * kW0Blk + sw128_offset(r, col % kFBK)) =
         make_uint4(pack_bf16x2(v[8 * i], v[8 * i + 1]), pack_bf16x2(v[8 * i + 2], v[8 * i + 3]),
                    pack_bf16x2(v[8 * i + 4], v[8 * i + 5]), pack_bf16x2(v[8 * i + 6], v[8 * i + 7]));
+  }
 }
 
 // Per-shape configuration (all sizes known at compile time).
@@ -141,9 +146,9 @@ struct FCfg {
   static_assert(S == 1 || S == 2, "one or two CTAs per group");
   static_assert(kTAcc + B <= 512, "the forward accumulator must fit the accumulator columns");
   static constexpr int kUPC = kFU / S;                      // units per CTA in steps F (kept) and H
-  static constexpr int kStagesF = 5;
+  static constexpr int kStagesF = 4;
   static constexpr int kBBytes = B * kFBK * 2;              // X tile: B rows x 64 k
-  static constexpr int kXtBytes = kND * kFBK * 2;           // X^T tile: 32 rows x 64 k (K padded)
+  static constexpr int kXtBytes = kDT * kFBK * 2;           // X^T tile: 48 rows x 64 k (K padded)
   static constexpr int kDRing = kNXD * kXtBytes;
   static constexpr int kFRing = kStagesF * kBBytes;
   static constexpr int kZs = B + 4;                         // row stride of the partial z exchange (floats)
@@ -158,16 +163,20 @@ struct FCfg {
   static constexpr int kW1Items = kFC * (kUPC / 4);         // (class, 4 units) items of the head update
   // the last layer's three products on the tensor core (batch 64, two CTAs
   // per group): operand tiles of 128-byte K-major rows in the forward X ring,
-  // which is idle between the forward's partial sums and step D
+  // which is idle between the forward's partial sums and step D.  An A tile
+  // holds 64 used rows; the MMA (M = 128) also reads the next 64 rows, which
+  // feed accumulator lanes nobody reads and may lie past the ring, in the
+  // resident W0 area that follows it.  dz1 takes h's slot once the logits
+  // MMA has completed.
   static constexpr bool kTCH = B == 64 && S == 2;
   static constexpr int tH = 0;                               // h [b][u]: logits A (rows b)
   static constexpr int tHT = 8192;                           // h^T [u][b]: head-gradient A (rows u)
+  static constexpr int tDzT = 16384;                         // dz1^T [c][b]: head-gradient B (16 rows)
   static constexpr int tW1 = 18432;                          // W1 [c][u]: logits B (16 rows)
   static constexpr int tW1T = 20480;                         // W1^T [u][c]: input-gradient A (K = 16 classes)
-  static constexpr int tDz = 28672;                          // dz1 [b][c]: input-gradient B (K = 16 classes)
-  static constexpr int tDzT = 36864;                         // dz1^T [c][b]: head-gradient B (16 rows)
-  static_assert(!kTCH || (kUPC == 64 && tDzT + 16 * 128 <= kFRing && tW1T + 128 * 128 <= kFRing),
-                "the head's operand tiles (and the 128-row reads of the A tiles) fit the F ring");
+  static constexpr int tDz = 0;                              // dz1 [b][c]: input-gradient B (K = 16 classes)
+  static_assert(!kTCH || (kUPC == 64 && tW1T + 64 * 128 <= kFRing && tDzT + 16 * 128 <= tW1),
+                "the head's operand tiles fit the F ring");
   static_assert(!kTCH || tW1 >= kZBytes, "the head-column tiles, written during the pair wait, clear the own partials");
   static_assert(2 * kW1Items * 16 <= kStagesF * B * kFBK * 2, "head-update partials must fit the F ring");
   // shared memory carve-up (bytes, from a 1024-aligned base)
@@ -272,9 +281,11 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
   const int col_end = half == S - 1 ? D : kb_end * kFBK;
   const int ncols = col_end - col_begin;        // a multiple of 8
   const int nkf = kb_end - kb_begin;
-  const int nD = (ncols + kND - 1) / kND;
+  const int nD = (ncols + kND - 1) / kND;        // 32-column model tiles (load, write-back)
+  const int nT = (ncols + kDT - 1) / kDT;        // 48-column weight-gradient tiles
+  const int ncols16 = (ncols + 15) & ~15;        // columns the weight-gradient epilogue updates
   const int pre_f = nkf < Cfg::kStagesF ? nkf : Cfg::kStagesF;   // X tiles loaded ahead of a step
-  const int pre_d = nD < kNXD ? nD : kNXD;                       // X^T tiles loaded before step D
+  const int pre_d = nT < kNXD ? nT : kNXD;                       // X^T tiles loaded before step D
   const int64_t gso = static_cast<int64_t>(a.global_slot) * a.slot_stride;
   const int partner = grp * S + (half ^ 1);     // S = 2: the other CTA of the group
 
@@ -343,14 +354,14 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
       }
       return true;
     };
-    // X^T tiles [from, to) of step s's weight gradient (ring position (sg0 + s) * nD + tile)
+    // X^T tiles [from, to) of step s's weight gradient (ring position (sg0 + s) * nT + tile)
     auto issue_d = [&](int s, int from, int to) -> bool {
       for (int tt = from; tt < to; ++tt) {
-        const int c = (sg0 + s) * nD + tt, xb = c % kNXD, use = c / kNXD;
+        const int c = (sg0 + s) * nT + tt, xb = c % kNXD, use = c / kNXD;
         // the buffer's previous tile must have been read by its MMA
         if (use >= 1 && !mbar_wait(&xfreeD[xb], (use - 1) & 1, a.err, kDevTimeoutEmpty)) return false;
         mbar_arrive_expect_tx(&fullD[xb], Cfg::kXtBytes);
-        tma_load_4d(dring + xb * Cfg::kXtBytes, &mXT, 0, col_begin + tt * kND, w, s, &fullD[xb]);
+        tma_load_4d(dring + xb * Cfg::kXtBytes, &mXT, 0, col_begin + tt * kDT, w, s, &fullD[xb]);
       }
       return true;
     };
@@ -878,7 +889,7 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
 
       // ------------------------------------------------------------ D: weight gradient + SGD of own W0 block
       if (warp == 0 && lane == 0) {
-        if (producer_ok) producer_ok = issue_d(s, pre_d, nD);
+        if (producer_ok) producer_ok = issue_d(s, pre_d, nT);
         // the first X tiles of the next step's forward, while this step's epilogue runs
         if (producer_ok && s + 1 < tau) producer_ok = issue_f(s + 1, 0, pre_f);
       } else if (warp == 1 || warp == 3) {
@@ -890,13 +901,13 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
         // committed, even after a failed wait, so that the arrivals and the
         // waits on the named barrier stay paired
         const int e = warp == 1 ? 0 : 1;
-        constexpr uint32_t idesc = idesc_bf16_f32(128, kND);
+        constexpr uint32_t idesc = idesc_bf16_f32(128, kDT);
         if (S > 1) {   // the partner's dz0^T rows (st.async) have landed before the tensor core reads them
           if (chain_ok) chain_ok = mbar_wait(dzin, sg & 1, a.err, kDevTimeoutFull);
           fence_proxy_async_smem();
         }
-        for (int tt = ((sg * nD + e) & 1); tt < nD; tt += 2) {
-          const int c = sg * nD + tt, buf = e, use = c / kNBD, xb = c % kNXD;
+        for (int tt = ((sg * nT + e) & 1); tt < nT; tt += 2) {
+          const int c = sg * nT + tt, buf = e, use = c / kNBD, xb = c % kNXD;
           if (chain_ok) chain_ok = mbar_wait(&fullD[xb], (c / kNXD) & 1, a.err, kDevTimeoutFull);
           if (use >= 1) bar_named(1 + e, 128 + 32);   // the previous use of the buffer has been read
           tc_fence_after();
@@ -904,7 +915,7 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
             if (chain_ok) {
               const uint32_t xa = smem_u32(dring + xb * Cfg::kXtBytes);
               const uint32_t da = smem_u32(dzT);
-              const uint32_t dcol = tmem + static_cast<uint32_t>(kTAcc + buf * kND);
+              const uint32_t dcol = tmem + static_cast<uint32_t>(kTAcc + buf * kDT);
 #pragma unroll
               for (int j = 0; j < kFBK / 16; ++j)
                 umma_bf16(dcol, smem_desc_k128(da + j * 32), smem_desc_k128(xa + j * 32), idesc, j != 0 ? 1u : 0u);
@@ -921,21 +932,43 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
         const int quarter = warp & 3, eg = (warp - 4) >> 2;
         const int r = quarter * 32 + lane;
         const uint32_t trow = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
-        for (int tt = ((sg * nD + eg) & 1); tt < nD; tt += 2) {
-          const int c = sg * nD + tt, buf = eg, use = c / kNBD;
+        for (int tt = ((sg * nT + eg) & 1); tt < nT; tt += 2) {
+          const int c = sg * nT + tt, buf = eg, use = c / kNBD;
           int ok = mbar_wait(&accD[buf], use & 1, a.err, kDevTimeoutAccum) ? 1 : 0;
           ok = __all_sync(0xffffffffu, ok);
           tc_fence_after();
           if (ok) {
-            const int c0 = tt * kND;
-            float g[32], m[32];
-            tmem_ld_32x32b_x32_pair(trow + kTAcc + buf * kND, g, trow + c0, m);
+            // the tile's columns up to the input's end rounded to 16 (the
+            // padding columns past the input are zero in the master and in
+            // X^T): 32 and/or 16 columns, the same for the whole warp
+            const int c0 = tt * kDT;
+            const int nc = ncols16 - c0 < kDT ? ncols16 - c0 : kDT;
+            const bool has32 = nc >= 32, has16 = (nc & 16) != 0;
+            const int c16 = c0 + (has32 ? 32 : 0);
+            const uint32_t gcol = trow + kTAcc + buf * kDT;
+            // the gradient first: once it is in registers the buffer goes back
+            // to the issuing chain; the master columns are this thread's own
+            float g[32], g16[16];
+            if (has32) tmem_ld_32x32b_x32(gcol, g);
+            if (has16) tmem_ld_32x32b_x16(gcol + (has32 ? 32 : 0), g16);
             tc_fence_before();
             bar_arrive_named(1 + eg, 128 + 32);   // the gradient buffer has been read: the next MMA may reuse it
+            if (has32) {
+              float m[32];
+              tmem_ld_32x32b_x32(trow + c0, m);
 #pragma unroll
-            for (int j = 0; j < 32; ++j) m[j] = fmaf(-a.lr, g[j], m[j]);
-            tmem_st_32x32b_x32(trow + c0, m);
-            put_w0_row32(w0s, r, c0, m);
+              for (int j = 0; j < 32; ++j) m[j] = fmaf(-a.lr, g[j], m[j]);
+              tmem_st_32x32b_x32(trow + c0, m);
+              put_w0_cols<32>(w0s, r, c0, m);
+            }
+            if (has16) {
+              float m16[16];
+              tmem_ld_32x32b_x16(trow + c16, m16);
+#pragma unroll
+              for (int j = 0; j < 16; ++j) m16[j] = fmaf(-a.lr, g16[j], m16[j]);
+              tmem_st_32x32b_x16(trow + c16, m16);
+              put_w0_cols<16>(w0s, r, c16, m16);
+            }
           } else {
             tc_fence_before();
             bar_arrive_named(1 + eg, 128 + 32);
@@ -1053,7 +1086,7 @@ bool fused_round_supported(int L, int D, int H, int C, int B) {
   return smem <= 227 * 1024;
 }
 
-int fused_round_xt_rows(int) { return kND; }
+int fused_round_xt_rows(int) { return kDT; }
 
 namespace {
 template <int B, int S>

@@ -5,9 +5,13 @@ interleavings.
 Actors: the X^T producer, two MMA-issuing threads and two epilogue
 warpgroups.  Tile c (the cluster's running tile index) belongs to chain
 e = c % 2: its MMA is issued by chain e's thread into TMEM buffer e and
-committed to accD[e] and xfreeD[c % 4]; warpgroup e waits accD[e], reads the
+committed to accD[e] and xfreeD[c % K]; warpgroup e waits accD[e], reads the
 buffer and hands it back by a named barrier that chain e's thread waits on
-before the tile c + 2.  X^T tile c goes to ring slot c % 4 (fullD / xfreeD).
+before the tile c + 2.  X^T tile c goes to ring slot c % K (fullD / xfreeD),
+K = 4 in the kernel.  The ring depth must be even: with K = 3 a slot
+alternates between the chains, and a chain can start its parity wait for a
+slot's phase k while the other chain's phase k - 1 has not landed, which the
+parity test would take for complete; the model catches that.
 
 The checks: every mbarrier parity wait targets the phase in progress or the
 one just completed (a barrier two phases ahead or behind would make the
@@ -20,7 +24,7 @@ import random
 
 import pytest
 
-KNXD = 4
+KNXD_KERNEL = 4
 
 
 class _Bar:
@@ -34,7 +38,7 @@ def _wait(bar, k):
     return bar.n == k + 1
 
 
-def _run(nD, tau, seed, nbuf=2, acc_index=lambda c, nbuf: c % nbuf):
+def _run(nD, tau, seed, nbuf=2, acc_index=lambda c, nbuf: c % nbuf, KNXD=KNXD_KERNEL):
     rnd = random.Random(seed)
     fullD = [_Bar() for _ in range(KNXD)]
     xfree = [_Bar() for _ in range(KNXD)]
@@ -98,11 +102,12 @@ def _run(nD, tau, seed, nbuf=2, acc_index=lambda c, nbuf: c % nbuf):
         assert len(pend[b]) == (1 if used else 0)
 
 
-@pytest.mark.parametrize("nD", [1, 2, 3, 5, 12, 13])
+@pytest.mark.parametrize("knxd", [KNXD_KERNEL, 2, 6])
+@pytest.mark.parametrize("nD", [1, 2, 3, 5, 8, 9, 12, 13])
 @pytest.mark.parametrize("tau", [1, 2, 7])
-def test_two_chain_step_d_protocol(nD, tau):
+def test_two_chain_step_d_protocol(nD, tau, knxd):
     for seed in range(40):
-        _run(nD, tau, seed)
+        _run(nD, tau, seed, KNXD=knxd)
 
 
 def test_three_buffers_in_turn_with_one_barrier_per_buffer_is_caught():
@@ -110,6 +115,18 @@ def test_three_buffers_in_turn_with_one_barrier_per_buffer_is_caught():
     for seed in range(40):
         try:
             _run(13, 7, seed, nbuf=3)
+        except AssertionError:
+            failures += 1
+    assert failures > 0
+
+
+def test_odd_ring_depth_is_caught():
+    """Three X^T slots shared by two chains: some interleaving makes a parity
+    wait two phases ahead of its barrier."""
+    failures = 0
+    for seed in range(40):
+        try:
+            _run(5, 2, seed, KNXD=3)
         except AssertionError:
             failures += 1
     assert failures > 0
