@@ -146,7 +146,10 @@ struct FCfg {
   static_assert(S == 1 || S == 2, "one or two CTAs per group");
   static_assert(kTAcc + B <= 512, "the forward accumulator must fit the accumulator columns");
   static constexpr int kUPC = kFU / S;                      // units per CTA in steps F (kept) and H
-  static constexpr int kStagesF = 4;
+  // the last layer's three products on the tensor core (batch 64, two CTAs
+  // per group; see the operand tiles below)
+  static constexpr bool kTCH = B == 64 && S == 2;
+  static constexpr int kStagesF = kTCH ? 5 : 4;
   static constexpr int kBBytes = B * kFBK * 2;              // X tile: B rows x 64 k
   static constexpr int kXtBytes = kDT * kFBK * 2;           // X^T tile: 48 rows x 64 k (K padded)
   static constexpr int kDRing = kNXD * kXtBytes;
@@ -168,7 +171,6 @@ struct FCfg {
   // feed accumulator lanes nobody reads and may lie past the ring, in the
   // resident W0 area that follows it.  dz1 takes h's slot once the logits
   // MMA has completed.
-  static constexpr bool kTCH = B == 64 && S == 2;
   static constexpr int tH = 0;                               // h [b][u]: logits A (rows b)
   static constexpr int tHT = 8192;                           // h^T [u][b]: head-gradient A (rows u)
   static constexpr int tDzT = 16384;                         // dz1^T [c][b]: head-gradient B (16 rows)
@@ -183,21 +185,24 @@ struct FCfg {
   static constexpr int oRegion = 0;
   static constexpr int oW0 = (oRegion + kRegion + 1023) / 1024 * 1024;
   static constexpr int oDzT = oW0 + kMaxKb * kW0Blk;
+  // the float h tile (CUDA-core last layer), which also receives the
+  // partner's partials; with the tensor-core last layer only the latter
+  static constexpr int kHsBytes = kTCH ? kZBytes : B * kHsd * 4;
   static constexpr int oHs = oDzT + kDzT;                    // [B][kHsd] float
-  static constexpr int oWc = oHs + B * kHsd * 4;             // [C][kUPC] float (bf16 operand)
+  static constexpr int oWc = oHs + kHsBytes;                 // [C][kUPC] float (bf16 operand)
   static constexpr int oW1m = oWc + kFC * kUPC * 4;          // [C][kUPC] fp32 master head columns
   static constexpr int oPl = oW1m + kFC * kUPC * 4;          // [2][B][C] partial logits by step parity
   static constexpr int oDz = oPl + 2 * B * kFC * 4;          // [B][C]
-  static constexpr int oDzb = oDz + B * kFC * 4;             // [C][B] (class-major)
-  static constexpr int oGbp = oDzb + B * kFC * 4;            // [kChunks][kUPC]
-  static constexpr int oRowLoss = oGbp + kChunks * kUPC * 4;   // [B]
+  static constexpr int oDzb = oDz + B * kFC * 4;             // [C][B] (class-major; CUDA-core last layer)
+  static constexpr int oGbp = oDzb + (kTCH ? 0 : B * kFC * 4);   // [kChunks][kUPC] (CUDA-core last layer)
+  static constexpr int oRowLoss = oGbp + (kTCH ? 0 : kChunks * kUPC * 4);   // [B]
   static constexpr int oB0 = oRowLoss + B * 4;               // [kFU] b0 of the group's units
   static constexpr int oB1 = oB0 + kFU * 4;                  // [16] head bias (private copy)
   static constexpr int oLab = oB1 + 16 * 4;                  // [B] int
   static constexpr int oBar = (oLab + B * 4 + 15) / 16 * 16;
   static constexpr int kBarBytes = 256;
   static constexpr int kSmem = oBar + kBarBytes + 1024;      // + alignment slack
-  static_assert(S == 1 || kUPC * kZs <= B * kHsd, "the incoming partials must fit the h tile they alias");
+  static_assert(S == 1 || kUPC * kZs * 4 <= kHsBytes, "the incoming partials must fit the h tile they alias");
   static_assert(S == 1 || kZBytes <= kFRing, "own partials must fit the F ring");
 };
 
@@ -560,11 +565,12 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
           const float bias = b0m[ug];
           const float h0 = bf16_round(fmaxf(z.x + bias, 0.f)), h1 = bf16_round(fmaxf(z.y + bias, 0.f));
           const float h2 = bf16_round(fmaxf(z.z + bias, 0.f)), h3 = bf16_round(fmaxf(z.w + bias, 0.f));
-          hs[(b4 + 0) * Cfg::kHsd + ul] = h0;
-          hs[(b4 + 1) * Cfg::kHsd + ul] = h1;
-          hs[(b4 + 2) * Cfg::kHsd + ul] = h2;
-          hs[(b4 + 3) * Cfg::kHsd + ul] = h3;
-          if constexpr (Cfg::kTCH) {   // h as the tensor core reads it, both ways
+          if constexpr (!Cfg::kTCH) {
+            hs[(b4 + 0) * Cfg::kHsd + ul] = h0;
+            hs[(b4 + 1) * Cfg::kHsd + ul] = h1;
+            hs[(b4 + 2) * Cfg::kHsd + ul] = h2;
+            hs[(b4 + 3) * Cfg::kHsd + ul] = h3;
+          } else {   // h as the tensor core reads it, both ways (the only copy)
             st_bf16(fring + Cfg::tH + sw128_offset(b4 + 0, ul), h0);
             st_bf16(fring + Cfg::tH + sw128_offset(b4 + 1, ul), h1);
             st_bf16(fring + Cfg::tH + sw128_offset(b4 + 2, ul), h2);
@@ -745,9 +751,21 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
             for (int c0 = 0; c0 < B; c0 += 32) {
               float v[32];
               tmem_ld_32x32b_x32(trow + c0, v);
+              // ReLU mask from unit u's row of the bf16 h^T tile: h >= 0, so
+              // h > 0 exactly when its bf16 bits are not zero
+              uint32_t hb[16];
+#pragma unroll
+              for (int k = 0; k < 4; ++k) {
+                const uint4 q = *reinterpret_cast<const uint4*>(fring + Cfg::tHT + sw128_offset(u, c0 + 8 * k));
+                hb[4 * k] = q.x;
+                hb[4 * k + 1] = q.y;
+                hb[4 * k + 2] = q.z;
+                hb[4 * k + 3] = q.w;
+              }
 #pragma unroll
               for (int i = 0; i < 32; ++i) {
-                const float dh = hs[(c0 + i) * Cfg::kHsd + u] > 0.f ? v[i] : 0.f;
+                const uint32_t bits = (hb[i >> 1] >> ((i & 1) * 16)) & 0xFFFFu;
+                const float dh = bits != 0u ? v[i] : 0.f;
                 v[i] = dh;
                 gsum += dh;
               }
