@@ -309,6 +309,27 @@ oscars_status oscars_profile_reset(oscars_ctx* ctx);
 int32_t oscars_phase_times(oscars_ctx* ctx, int32_t cap, double* us);
 
 /*
+ * oscars_check_padding - look for writes where no kernel should write, in
+ * place of a memory checker: the layout pads each weight and bias of a slot
+ * to 64 elements, and that padding must stay zero in the fp32 slab and in
+ * its bf16 copy; 256 guard words after each of the two hold a byte pattern
+ * written at creation.  *bad (host) receives the number of padding values
+ * that are not zero (MLP mode) plus the guard words that changed (MLP and
+ * CNN).  Synchronises the stream and copies both slabs to the host: meant
+ * for tests and debugging, not for a training loop.  Not a step of the
+ * method.  Errors: EINVAL (NULL), ESTATE (FLAT mode), ENOMEM, ECUDA.
+ */
+oscars_status oscars_check_padding(oscars_ctx* ctx, int64_t* bad);
+
+/*
+ * oscars_debug_slab - the device address of the context's fp32 slab and its
+ * slot stride in floats (slot k < W is worker k's replica, slot W the global
+ * model; each tensor starts on a 64-element boundary), for tests of the
+ * layout.  Writing through it changes the model.  Errors: EINVAL (NULL).
+ */
+oscars_status oscars_debug_slab(const oscars_ctx* ctx, float** slab, int64_t* slot_stride);
+
+/*
  * oscars_check_wait_timeout - exercise the failure path of the kernels'
  * bounded waits.  Every wait of a kernel in this library on an mbarrier (a
  * TMA stage, a tensor-core accumulator, a peer CTA's data) gives up after a

@@ -71,6 +71,8 @@ _SIGS = {
     "oscars_merge_weights": (c_int32, [c_int32, POINTER(c_int32), c_int32, POINTER(c_float)]),
     "oscars_read_replica": (c_int32, [c_void_p, c_int32, c_void_p]),
     "oscars_check_wait_timeout": (c_int32, [c_void_p, c_int32]),
+    "oscars_check_padding": (c_int32, [c_void_p, POINTER(c_int64)]),
+    "oscars_debug_slab": (c_int32, [c_void_p, POINTER(c_void_p), POINTER(c_int64)]),
     "oscars_gemm_bf16_nt": (c_int32, [c_void_p, c_void_p, c_void_p, c_int32, c_int32, c_int32, c_void_p]),
     "oscars_profile_read": (c_int32, [c_void_p, c_int32, POINTER(ctypes.c_char_p), POINTER(c_double),
                                       POINTER(c_int32)]),
@@ -263,6 +265,21 @@ def oscars_eval_loss(ctx: int, x_ptr: int, y_ptr: int, n: int) -> float:
 
 def oscars_read_replica(ctx: int, k: int, dst_ptr: int):
     _check(lib().oscars_read_replica(c_void_p(ctx), k, c_void_p(dst_ptr)), c_void_p(ctx))
+
+
+def oscars_check_padding(ctx: int) -> int:
+    """Padding values that are not zero plus changed guard words (0 when no
+    kernel wrote outside its tensors)."""
+    bad = c_int64()
+    _check(lib().oscars_check_padding(c_void_p(ctx), ctypes.byref(bad)), c_void_p(ctx))
+    return bad.value
+
+
+def oscars_debug_slab(ctx: int):
+    """(device address of the fp32 slab, slot stride in floats)."""
+    p, st = c_void_p(), c_int64()
+    _check(lib().oscars_debug_slab(c_void_p(ctx), ctypes.byref(p), ctypes.byref(st)))
+    return p.value, st.value
 
 
 def oscars_check_wait_timeout(ctx: int, polls: int):

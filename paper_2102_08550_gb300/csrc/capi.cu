@@ -338,6 +338,11 @@ void prof_after_replay(oscars_ctx* c, const std::vector<oscars_ctx::ProfEntry>& 
   prof_collect(c);   // read now: the next replay records the same events again
 }
 
+// guard words after the model slab and after its bf16 copy: a byte pattern
+// written at creation that no kernel writes (oscars_check_padding reads it)
+constexpr size_t kGuardWords = 256;
+constexpr int kGuardByte = 0xA5;
+
 template <typename T>
 bool dev_alloc(oscars_ctx* c, T** p, size_t count) {
   void* q = nullptr;
@@ -1176,8 +1181,10 @@ oscars_status allocate_common(oscars_ctx* c) {
   }
   const int W = c->W;
   const size_t slots = static_cast<size_t>(W) + 1;
-  if (!dev_alloc(c, &c->slab, slots * c->P_pad)) return fail(c, OSCARS_ENOMEM, "device allocation failed (model slab)");
+  if (!dev_alloc(c, &c->slab, slots * c->P_pad + kGuardWords))
+    return fail(c, OSCARS_ENOMEM, "device allocation failed (model slab)");
   cudaMemset(c->slab, 0, slots * c->P_pad * sizeof(float));
+  cudaMemset(c->slab + slots * c->P_pad, kGuardByte, kGuardWords * sizeof(float));
   if (!dev_alloc(c, &c->cursor, W) || !dev_alloc(c, &c->tau_dev, W) || !dev_alloc(c, &c->loss_dev, std::max(W, 1)) ||
       !dev_alloc(c, &c->dx_tab, W) || !dev_alloc(c, &c->dy_tab, W) || !dev_alloc(c, &c->dn_tab, W) ||
       !dev_alloc(c, &c->err, 1) || !dev_alloc(c, &c->lane_ids, W) || !dev_alloc(c, &c->global_src, W) ||
@@ -1202,9 +1209,10 @@ oscars_status allocate_cnn(oscars_ctx* c) {
   const int W = c->W, B = c->B;
   const size_t slots = static_cast<size_t>(W) + 1;
   const int layers = 1 + 2 * c->cnn_blocks;
-  if (!dev_alloc(c, &c->shadow, slots * c->P_pad) || !dev_alloc(c, &c->cnn_wt, slots * c->cnn_wt_slot))
+  if (!dev_alloc(c, &c->shadow, slots * c->P_pad + kGuardWords) || !dev_alloc(c, &c->cnn_wt, slots * c->cnn_wt_slot))
     return fail(c, OSCARS_ENOMEM, "device allocation failed (bf16 weights)");
   cudaMemset(c->shadow, 0, slots * c->P_pad * sizeof(__nv_bfloat16));
+  cudaMemset(c->shadow + slots * c->P_pad, kGuardByte, kGuardWords * sizeof(__nv_bfloat16));
   cudaMemset(c->cnn_wt, 0, slots * c->cnn_wt_slot * sizeof(__nv_bfloat16));
   const size_t act = static_cast<size_t>(W) * B * 1024 * 64;
   const int nbuf = 2 + 2 * c->cnn_blocks + 3;
@@ -1262,8 +1270,10 @@ oscars_status allocate_mlp(oscars_ctx* c) {
   const size_t slots = static_cast<size_t>(W) + 1;
   if (L == 1 && !c->bf16) return OSCARS_OK;
 
-  if (!dev_alloc(c, &c->shadow, slots * c->P_pad)) return fail(c, OSCARS_ENOMEM, "device allocation failed (bf16 shadow)");
+  if (!dev_alloc(c, &c->shadow, slots * c->P_pad + kGuardWords))
+    return fail(c, OSCARS_ENOMEM, "device allocation failed (bf16 shadow)");
   cudaMemset(c->shadow, 0, slots * c->P_pad * sizeof(__nv_bfloat16));
+  cudaMemset(c->shadow + slots * c->P_pad, kGuardByte, kGuardWords * sizeof(__nv_bfloat16));
   c->A.assign(L, nullptr);
   c->AT.assign(L, nullptr);
   c->G.assign(L, nullptr);
@@ -1926,6 +1936,57 @@ oscars_status oscars_eval_loss(oscars_ctx* c, const float* x, const int32_t* y, 
   if (e == cudaSuccess) e = cudaMemcpy(loss, c->loss_dev, sizeof(float), cudaMemcpyDeviceToHost);
   if (e != cudaSuccess) return cuda_fail(c, e, "eval");
   return check_err_word(c);
+}
+
+oscars_status oscars_debug_slab(const oscars_ctx* c, float** slab, int64_t* slot_stride) {
+  if (!c || !slab || !slot_stride) return OSCARS_EINVAL;
+  *slab = c->slab;
+  *slot_stride = c->P_pad;
+  return OSCARS_OK;
+}
+
+oscars_status oscars_check_padding(oscars_ctx* c, int64_t* bad) {
+  if (!c || !bad) return OSCARS_EINVAL;
+  if (!slotted(c)) return fail(c, OSCARS_ESTATE, "the padding check needs an MLP or CNN context");
+  try {
+    const size_t slots = static_cast<size_t>(c->W) + 1, n = slots * c->P_pad;
+    std::vector<uint32_t> f(n + kGuardWords);
+    cudaError_t e = cudaStreamSynchronize(c->stream);
+    if (e == cudaSuccess) e = cudaMemcpy(f.data(), c->slab, f.size() * sizeof(uint32_t), cudaMemcpyDeviceToHost);
+    std::vector<uint16_t> h;
+    if (e == cudaSuccess && c->shadow) {
+      h.resize(n + kGuardWords);
+      e = cudaMemcpy(h.data(), c->shadow, h.size() * sizeof(uint16_t), cudaMemcpyDeviceToHost);
+    }
+    if (e != cudaSuccess) return cuda_fail(c, e, "padding check");
+    int64_t count = 0;
+    const uint32_t g32 = 0x01010101u * kGuardByte;
+    const uint16_t g16 = static_cast<uint16_t>(0x0101u * kGuardByte);
+    for (size_t i = n; i < f.size(); ++i) count += f[i] != g32;
+    for (size_t i = n; i < h.size(); ++i) count += h[i] != g16;
+    if (c->model == OSCARS_MODEL_MLP) {
+      // the gaps between a slot's tensors and its tail (the layout pads each
+      // W_l and b_l to 64 elements); the value bits of -0.0 count as set
+      for (size_t k = 0; k < slots; ++k) {
+        const size_t base = k * c->P_pad;
+        for (size_t l = 0; l < c->layers.size(); ++l) {
+          const Layer& ly = c->layers[l];
+          const int64_t end = l + 1 < c->layers.size() ? c->layers[l + 1].offW : c->P_pad;
+          const int64_t gaps[2][2] = {{ly.offW + static_cast<int64_t>(ly.in) * ly.out, ly.offB},
+                                      {ly.offB + ly.out, end}};
+          for (const auto& g : gaps)
+            for (int64_t i = g[0]; i < g[1]; ++i) {
+              count += f[base + i] != 0u;
+              if (!h.empty()) count += h[base + i] != 0u;
+            }
+        }
+      }
+    }
+    *bad = count;
+    return OSCARS_OK;
+  } catch (const std::bad_alloc&) {
+    return fail(c, OSCARS_ENOMEM, "host allocation failed");
+  }
 }
 
 oscars_status oscars_check_wait_timeout(oscars_ctx* c, int32_t polls) {
