@@ -31,6 +31,11 @@ namespace {
 int64_t round_up(int64_t x, int64_t m) { return (x + m - 1) / m * m; }
 
 constexpr int kMaxBranches = 16;
+// blocks of the per-layer round's staging when it reads host-resident shards
+// (16 KB of rows in flight per block; 48 to 76 blocks measured within 2% of
+// one another on the 3072-1024-1024-10 MLP with 32 workers, 128 and the full
+// grid up to 25% slower per round)
+constexpr int kHostStageBlocks = 64;
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
                                   const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
@@ -185,8 +190,13 @@ struct oscars_ctx {
   int32_t* labels_all = nullptr;
   std::vector<CUtensorMap> mA0s, mAT0s;
   bool fused = false;                   // whole-round kernel (2-layer MLP)
-  // the one-launch round stages the next round while the current one runs:
-  // two input buffers, used alternately (index `parity` holds the next round)
+  bool ahead_mlp = false;               // per-layer bf16 MLP round that stages the next round beside it
+  bool shards_host = false;             // some shard's samples live in host memory
+  int cur_buf = 0;                      // ahead_mlp: the input buffer the round being enqueued reads
+  std::vector<CUtensorMap> mA0p[2], mAT0p[2];   // ahead_mlp: per-step maps of each input buffer
+  // the one-launch round (and ahead_mlp) stages the next round while the
+  // current one runs: two input buffers, used alternately (index `parity`
+  // holds the next round)
   __nv_bfloat16* A0b[2] = {};
   __nv_bfloat16* A0Tb[2] = {};
   int32_t* labb[2] = {};
@@ -435,14 +445,27 @@ oscars_status ensure_stage_buffers(oscars_ctx* c) {
   if (c->fused && (c->flags & 16) &&
       !dev_alloc(c, &c->phase_ts, static_cast<size_t>(cap) * 4))   // stamps of every step (flag bit 4)
     return fail(c, OSCARS_ENOMEM, "device allocation failed (phase stamps)");
-  if (c->fused) {
-    const uint64_t per_b = static_cast<uint64_t>(per) * 2;
+  if (c->fused || c->ahead_mlp) {
     c->A0b[0] = c->A0all;
     c->A0Tb[0] = c->A0Tall;
     c->labb[0] = c->labels_all;
     if (!dev_alloc(c, &c->A0b[1], per * cap) || !dev_alloc(c, &c->A0Tb[1], per * cap) ||
         !dev_alloc(c, &c->labb[1], static_cast<size_t>(W) * B * cap))
       return fail(c, OSCARS_ENOMEM, "device allocation failed (second input buffer)");
+  }
+  if (c->ahead_mlp) {   // the per-step maps of both input buffers
+    for (int b = 0; b < 2; ++b) {
+      c->mA0p[b].resize(cap);
+      c->mAT0p[b].resize(cap);
+      for (int s = 0; s < cap; ++s)
+        if (!make_map(&c->mA0p[b][s], c->A0b[b] + per * s, D, B, W, D * 2ull, static_cast<uint64_t>(B) * D * 2ull, B) ||
+            !make_map(&c->mAT0p[b][s], c->A0Tb[b] + per * s, B, D, W, B * 2ull, static_cast<uint64_t>(B) * D * 2ull,
+                      128))
+          return fail(c, OSCARS_ECUDA, "cuTensorMapEncodeTiled failed (per-step inputs)");
+    }
+  }
+  if (c->fused) {
+    const uint64_t per_b = static_cast<uint64_t>(per) * 2;
     for (int i = 0; i < 2; ++i)
       if (!make_map4(&c->mX4b[i], c->A0b[i], D, B, W, cap, D * 2ull, static_cast<uint64_t>(B) * D * 2ull, per_b, B) ||
           !make_map4(&c->mXT4b[i], c->A0Tb[i], B, D, W, cap, B * 2ull, static_cast<uint64_t>(B) * D * 2ull, per_b,
@@ -626,6 +649,16 @@ HeadArgs head_base(oscars_ctx* c) {
   return h;
 }
 
+// the staged layer-0 inputs of local step `step` (and their labels): the
+// input buffer of the round being enqueued when rounds stage ahead
+const CUtensorMap& step_inputs(oscars_ctx* c, int step) {
+  return c->ahead_mlp ? c->mA0p[c->cur_buf][step] : c->mA0s[step];
+}
+const CUtensorMap& step_inputs_t(oscars_ctx* c, int step) {
+  return c->ahead_mlp ? c->mAT0p[c->cur_buf][step] : c->mAT0s[step];
+}
+const int32_t* step_labels(oscars_ctx* c) { return c->ahead_mlp ? c->labb[c->cur_buf] : c->labels_all; }
+
 // forward layers 0..L-2 for `na` lanes (training step or evaluation)
 cudaError_t enqueue_forward(oscars_ctx* c, const int* wid, const int* src, int na, cudaStream_t st, int step = 0) {
   for (int l = 0; l + 1 < c->L; ++l) {
@@ -642,7 +675,7 @@ cudaError_t enqueue_forward(oscars_ctx* c, const int* wid, const int* src, int n
     g.outT = c->AT[l + 1];
     g.pdl = c->profiling ? 0 : 1;   // overlaps its prologue with the previous kernel's tail
     ProfScope ps(c, "gemm_fwd", st);
-    cudaError_t e = launch_gemm(kEpiFwd, c->mShadow[l], l == 0 ? c->mA0s[step] : c->mA[l], g, na, st);
+    cudaError_t e = launch_gemm(kEpiFwd, c->mShadow[l], l == 0 ? step_inputs(c, step) : c->mA[l], g, na, st);
     if (e != cudaSuccess) return e;
   }
   return cudaSuccess;
@@ -656,7 +689,7 @@ cudaError_t enqueue_step(oscars_ctx* c, int s, int na, const int* wid, const int
   HeadArgs h = head_base(c);
   h.wid = wid;
   h.src = src;
-  h.labels = c->labels_all + static_cast<size_t>(s) * c->W * c->B;
+  h.labels = step_labels(c) + static_cast<size_t>(s) * c->W * c->B;
   h.loss_part = c->loss_part;
   h.part_mul = c->max_tau;
   h.part_add = s;
@@ -694,7 +727,7 @@ cudaError_t enqueue_step(oscars_ctx* c, int s, int na, const int* wid, const int
       if ((e = launch_gemm(kEpiDh, c->mShadowMN[l], c->g_rows ? c->mG[l] : c->mGTmn[l], g, na, st)) != cudaSuccess)
         return e;
     }
-    const CUtensorMap& mX = l == 0 ? c->mAT0s[s] : c->mAT[l];
+    const CUtensorMap& mX = l == 0 ? step_inputs_t(c, s) : c->mAT[l];
     if (gemm_dw_supported(ly.out, ly.in, c->B)) {
       DwArgs d{};
       d.wid = wid;
@@ -862,6 +895,57 @@ cudaError_t enqueue_round_mlp(oscars_ctx* c, cudaStream_t st) {
   if ((e = launch_loss_finalize(c->loss_part, c->tau_dev, c->W, c->max_tau, nc, c->B, c->loss_dev, st)) != cudaSuccess)
     return e;
   return launch_cursor_advance(c->cursor, c->tau_dev, c->dn_tab, c->B, c->W, st);
+}
+
+// per-layer round from input buffer `buf` (staged earlier) and, beside it
+// on the side stream at the lowest launch priority, the staging of the next
+// round into the other buffer followed by the cursor advance (as the
+// one-launch round does): with shards in host memory the next round's rows
+// cross the host link while this round computes.  While profiling,
+// everything runs in sequence on `st`.
+cudaError_t enqueue_round_mlp_ahead(oscars_ctx* c, int buf, cudaStream_t st) {
+  cudaError_t e;
+  c->cur_buf = buf;
+  const StageArgs sa = stage_args(c, buf ^ 1, c->tau_dev);
+  auto steps = [&](cudaStream_t s0) -> cudaError_t {
+    for (int s = 0; s < c->br_max_tau[0]; ++s) {
+      cudaError_t r = enqueue_step(c, s, c->br_na[s], c->br_wid + static_cast<size_t>(s) * c->W,
+                                   c->br_src + static_cast<size_t>(s) * c->W, s0);
+      if (r != cudaSuccess) return r;
+    }
+    return cudaSuccess;
+  };
+  // from host memory every load waits a round trip over the host link: a
+  // grid of kHostStageBlocks blocks striding over the tiles keeps enough rows
+  // in flight and leaves the SMs to the round's GEMMs (the full grid of one
+  // block per tile fills every SM between GEMM waves); from device memory the
+  // full grid is done soonest
+  auto stage_next = [&](cudaStream_t s0) {
+    return c->shards_host
+               ? launch_stage_round_strided(sa, c->tau_dev, c->W, c->max_tau, kHostStageBlocks, c->prio_least, s0)
+               : launch_stage_round_priority(sa, c->tau_dev, c->W, c->max_tau, c->prio_least, s0);
+  };
+  const int nc = c->B / kRowsPerLossChunk;
+  if (c->profiling) {
+    if ((e = steps(st)) != cudaSuccess) return e;
+    {
+      ProfScope ps(c, "stage", st);
+      if ((e = stage_next(st)) != cudaSuccess) return e;
+    }
+    ProfScope ps(c, "round_bookkeeping", st);
+    if ((e = launch_loss_finalize(c->loss_part, c->tau_dev, c->W, c->max_tau, nc, c->B, c->loss_dev, st)) != cudaSuccess)
+      return e;
+    return launch_cursor_advance(c->cursor, c->tau_dev, c->dn_tab, c->B, c->W, st);
+  }
+  if ((e = cudaEventRecord(c->side_fork, st)) != cudaSuccess) return e;
+  if ((e = cudaStreamWaitEvent(c->side, c->side_fork, 0)) != cudaSuccess) return e;
+  if ((e = stage_next(c->side)) != cudaSuccess) return e;
+  if ((e = launch_cursor_advance(c->cursor, c->tau_dev, c->dn_tab, c->B, c->W, c->side)) != cudaSuccess) return e;
+  if ((e = cudaEventRecord(c->side_join, c->side)) != cudaSuccess) return e;
+  if ((e = steps(st)) != cudaSuccess) return e;
+  if ((e = launch_loss_finalize(c->loss_part, c->tau_dev, c->W, c->max_tau, nc, c->B, c->loss_dev, st)) != cudaSuccess)
+    return e;
+  return cudaStreamWaitEvent(st, c->side_join, 0);
 }
 
 cudaError_t enqueue_round_softreg(oscars_ctx* c, cudaStream_t st) {
@@ -1450,6 +1534,7 @@ oscars_status oscars_create(const oscars_config* cfg, oscars_ctx** out) {
             st = fail(c, OSCARS_EINVAL, "bf16 MLP: shard " + std::to_string(i) + " samples must be 16-byte aligned");
           else {
             c->shard_x.push_back(cfg->shard_x[i]);
+            if (is_host_ptr(cfg->shard_x[i])) c->shards_host = true;
             c->shard_y.push_back(cfg->shard_y[i]);
             c->shard_n.push_back(cfg->shard_n[i]);
           }
@@ -1461,6 +1546,9 @@ oscars_status oscars_create(const oscars_config* cfg, oscars_ctx** out) {
         if (c->fused) c->fused_max_clusters = fused_round_max_clusters(c->dims[0], c->dims[1], c->B);
         // flag bit 2: bf16 MLP rounds fork into up to 16 concurrent worker branches
         c->n_br = (c->model == OSCARS_MODEL_MLP && c->bf16 && c->L >= 2 && (cfg->flags & 4)) ? std::min(c->W, kMaxBranches) : 1;
+        // the per-layer round stages the next round beside the current one
+        // (not with concurrent worker branches)
+        c->ahead_mlp = c->model == OSCARS_MODEL_MLP && c->bf16 && c->L >= 2 && !c->fused && c->n_br == 1;
         if (st == OSCARS_OK) st = c->model == OSCARS_MODEL_CNN ? allocate_cnn(c) : allocate_mlp(c);
         if (st == OSCARS_OK) st = build_tables(c);
         if (st == OSCARS_OK) {
@@ -1485,7 +1573,7 @@ oscars_status oscars_create(const oscars_config* cfg, oscars_ctx** out) {
         }
         if (st == OSCARS_OK && c->n_br > 1 && cudaEventCreateWithFlags(&c->br_fork, cudaEventDisableTiming) != cudaSuccess)
           st = fail(c, OSCARS_ECUDA, "event creation failed");
-        if (st == OSCARS_OK && c->fused &&
+        if (st == OSCARS_OK && (c->fused || c->ahead_mlp) &&
             (cudaDeviceGetStreamPriorityRange(&c->prio_least, &c->prio_greatest) != cudaSuccess ||
              cudaStreamCreateWithFlags(&c->side, cudaStreamNonBlocking) != cudaSuccess ||
              cudaEventCreateWithFlags(&c->side_fork, cudaEventDisableTiming) != cudaSuccess ||
@@ -1530,9 +1618,13 @@ oscars_status oscars_local_steps(oscars_ctx* c, int32_t* tau_out, float* loss_ou
   if (c->pending) return fail(c, OSCARS_ESTATE, "the previous round has not been merged");
   try {
     cudaError_t e = cudaSuccess;
-    if (c->fused) {
-      // the one-launch round: the first round (or the first after tau changed)
-      // stages its own mini-batches; every round stages the next one
+    if (c->fused || c->ahead_mlp) {
+      // the one-launch round (or the per-layer round): the first round (or
+      // the first after tau changed or an evaluation) stages its own
+      // mini-batches; every round stages the next one
+      auto enqueue_ahead = [&](int b, cudaStream_t s0) {
+        return c->fused ? enqueue_round_fused_ahead(c, b, s0) : enqueue_round_mlp_ahead(c, b, s0);
+      };
       const int buf = c->parity;
       if (!c->staged) {
         c->profiling = (c->flags & 2) != 0;
@@ -1545,7 +1637,7 @@ oscars_status oscars_local_steps(oscars_ctx* c, int32_t* tau_out, float* loss_ou
       }
       if (c->flags & 1) {
         c->profiling = (c->flags & 2) != 0;
-        e = enqueue_round_fused_ahead(c, buf, c->stream);
+        e = enqueue_ahead(buf, c->stream);
         c->profiling = false;
       } else {
         if (!c->ahead_exec[buf]) {
@@ -1554,7 +1646,7 @@ oscars_status oscars_local_steps(oscars_ctx* c, int32_t* tau_out, float* loss_ou
           c->prof_sink = &c->prof_ahead_graph[buf];   // empty: this parity's graph does not exist yet
           e = cudaStreamBeginCapture(c->cap, cudaStreamCaptureModeThreadLocal);
           if (e == cudaSuccess) {
-            cudaError_t e2 = enqueue_round_fused_ahead(c, buf, c->cap);
+            cudaError_t e2 = enqueue_ahead(buf, c->cap);
             e = cudaStreamEndCapture(c->cap, &g);
             if (e2 != cudaSuccess) e = e2;
           }
@@ -1917,6 +2009,7 @@ oscars_status oscars_eval_loss(oscars_ctx* c, const float* x, const int32_t* y, 
       sa.A0T = c->AT[0];
       sa.labels = c->labels;
       e = launch_stage(sa, na, c->stream);
+      c->cur_buf = 0;   // the evaluation stages its rows into the first input buffer
       if (e == cudaSuccess) e = enqueue_forward(c, c->lane_ids, c->global_src, na, c->stream);
       if (e == cudaSuccess) {
         HeadArgs h = head_base(c);

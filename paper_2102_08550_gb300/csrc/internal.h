@@ -99,6 +99,9 @@ cudaError_t launch_stage(const StageArgs& a, int n_active, cudaStream_t s);
 // (grid z over a.slots when given, else over all max_tau * W slots)
 cudaError_t launch_stage_round(const StageArgs& a, const int32_t* tau, int W, int max_tau, cudaStream_t s);
 // the same with a launch priority (cudaLaunchAttributePriority)
+// the same staging from `blocks` blocks striding over the tiles (bounded footprint beside other kernels)
+cudaError_t launch_stage_round_strided(const StageArgs& a, const int32_t* tau, int W, int max_tau, int blocks,
+                                       int priority, cudaStream_t s);
 cudaError_t launch_stage_round_priority(const StageArgs& a, const int32_t* tau, int W, int max_tau, int priority,
                                         cudaStream_t s);
 

@@ -75,11 +75,12 @@ __global__ void __launch_bounds__(256) stage_kernel(const __grid_constant__ Stag
 constexpr int kStageRows = 32, kStageCols = 128;
 constexpr int kStageLd = kStageCols + 2;   // bf16 row stride of the tile
 
-__global__ void __launch_bounds__(256) stage_round_kernel(const __grid_constant__ StageArgs a, const int32_t* tau,
-                                                          int W) {
-  __shared__ __align__(16) __nv_bfloat16 tile[kStageRows][kStageLd];
-  __shared__ int64_t rowoff[kStageRows];
-  const int z = a.slots ? a.slots[blockIdx.z] : static_cast<int>(blockIdx.z);
+// One tile of one (step, worker) slot: rows [by * kStageRows, +kStageRows)
+// and features [bx * kStageCols, +kStageCols) of the slot's mini-batch.
+__device__ __forceinline__ void stage_round_tile(const StageArgs& a, const int32_t* tau, int W, int bx, int by,
+                                                 int bz, __nv_bfloat16 (&tile)[kStageRows][kStageLd],
+                                                 int64_t (&rowoff)[kStageRows]) {
+  const int z = a.slots ? a.slots[bz] : bz;
   const int s = z / W, w = z - s * W;
   if (s >= tau[w]) return;
   const int64_t slot = static_cast<int64_t>(s) * W + w;
@@ -89,13 +90,13 @@ __global__ void __launch_bounds__(256) stage_round_kernel(const __grid_constant_
   const float* X = a.x[w];
   const int64_t n = a.n[w];
   const int64_t base = a.start[w] + (static_cast<int64_t>(s) + (a.ahead ? a.ahead[w] : 0)) * a.B;
-  const int k0 = blockIdx.x * kStageCols, b0 = blockIdx.y * kStageRows;
+  const int k0 = bx * kStageCols, b0 = by * kStageRows;
   const int tx = threadIdx.x & 31, ty = threadIdx.x >> 5;   // 32 x 8
   if (threadIdx.x < kStageRows) {
     const int b = b0 + threadIdx.x;
     const int64_t row = (base + b) % n;
     rowoff[threadIdx.x] = row * a.D;
-    if (blockIdx.x == 0 && b < a.B) a.labels[slot * a.B + b] = a.y[w][row];
+    if (bx == 0 && b < a.B) a.labels[slot * a.B + b] = a.y[w][row];
   }
   __syncthreads();
   const int k = k0 + tx * 4;
@@ -136,6 +137,30 @@ __global__ void __launch_bounds__(256) stage_round_kernel(const __grid_constant_
       dst[0] = make_uint4(p[0], p[1], p[2], p[3]);
       dst[1] = make_uint4(p[4], p[5], p[6], p[7]);
     }
+  }
+}
+
+__global__ void __launch_bounds__(256) stage_round_kernel(const __grid_constant__ StageArgs a, const int32_t* tau,
+                                                          int W) {
+  __shared__ __align__(16) __nv_bfloat16 tile[kStageRows][kStageLd];
+  __shared__ int64_t rowoff[kStageRows];
+  stage_round_tile(a, tau, W, blockIdx.x, blockIdx.y, blockIdx.z, tile, rowoff);
+}
+
+// The same tiles from a fixed number of blocks striding over them: a staging
+// that runs beside other kernels keeps a bounded footprint (each block fits
+// beside the GEMM blocks of an SM) while its loads stay in flight.
+__global__ void __launch_bounds__(256) stage_round_strided_kernel(const __grid_constant__ StageArgs a,
+                                                                  const int32_t* tau, int W, int nx, int ny,
+                                                                  int nz) {
+  __shared__ __align__(16) __nv_bfloat16 tile[kStageRows][kStageLd];
+  __shared__ int64_t rowoff[kStageRows];
+  const int64_t total = static_cast<int64_t>(nx) * ny * nz;
+  for (int64_t lin = blockIdx.x; lin < total; lin += gridDim.x) {
+    const int bx = static_cast<int>(lin % nx), by = static_cast<int>((lin / nx) % ny);
+    const int bz = static_cast<int>(lin / (static_cast<int64_t>(nx) * ny));
+    stage_round_tile(a, tau, W, bx, by, bz, tile, rowoff);
+    __syncthreads();   // the tile and the row offsets are rewritten by the next one
   }
 }
 
@@ -683,6 +708,23 @@ cudaError_t launch_stage_round_priority(const StageArgs& a, const int32_t* tau, 
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   return cudaLaunchKernelEx(&cfg, stage_round_kernel, a, tau, W);
+}
+
+cudaError_t launch_stage_round_strided(const StageArgs& a, const int32_t* tau, int W, int max_tau, int blocks,
+                                       int priority, cudaStream_t s) {
+  if (a.D % 4 != 0 || a.B % 16 != 0 || blocks < 1) return cudaErrorInvalidValue;
+  const int nx = (a.D + kStageCols - 1) / kStageCols, ny = (a.B + kStageRows - 1) / kStageRows;
+  const int nz = a.slots ? a.n_slots : W * max_tau;
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(static_cast<unsigned>(blocks), 1, 1);
+  cfg.blockDim = dim3(256, 1, 1);
+  cfg.stream = s;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributePriority;
+  attr[0].val.priority = priority;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, stage_round_strided_kernel, a, tau, W, nx, ny, nz);
 }
 
 cudaError_t launch_stage_round(const StageArgs& a, const int32_t* tau, int W, int max_tau, cudaStream_t s) {

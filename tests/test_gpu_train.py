@@ -307,10 +307,15 @@ def test_protocol_errors(cuda_device):
     ctx.close()
 
 
-@pytest.mark.parametrize("dims", [[784, 512, 10], [256, 128, 128, 10]], ids=["fused", "per-layer"])
+@pytest.mark.parametrize("dims", [[784, 512, 10], [256, 128, 128, 10], [1024, 256, 128, 10]],
+                         ids=["fused", "per-layer", "per-layer-strided"])
 def test_pinned_host_shards_match_device_shards(cuda_device, dims):
     """Shards in pinned host memory (read over the host link by the staging
-    kernel) give bit-identical rounds to the same shards in device memory."""
+    kernel) give bit-identical rounds to the same shards in device memory.
+    The per-layer path stages host rows from a fixed number of blocks
+    striding over the tiles; at 1024 inputs a round has more tiles (8 feature
+    blocks x 2 row blocks x every (step, worker) slot) than blocks, so each
+    block stages several."""
     w = synth.TrainWorkload("host-shards", 3, dims, 64, 0.05, 256, 6, 2)
     dev_shards = device_shards(w, cuda_device, n=256)
     host_shards = [(x.cpu().pin_memory(), y.cpu().pin_memory()) for x, y in dev_shards]
@@ -512,16 +517,23 @@ def test_train_without_eval_matches_round_by_round(cuda_device, dims):
     b.close()
 
 
-def test_round_kernel_restaging_between_rounds(cuda_device):
-    """The one-launch round stages the next round's mini-batches while it
-    runs.  Between rounds: an evaluation (which reuses the first input
-    buffer), a tau override, new iteration times (Algorithm 1 again) and a
-    plain round; the staged data must follow every change.  Against the
-    oracle driven through the same changes."""
+@pytest.mark.parametrize("dims,kernel,host", [([784, 512, 10], "fused_round", False),
+                                              ([256, 256, 128, 10], "gemm_dw_sgd", False),
+                                              ([512, 256, 128, 10], "gemm_dw_sgd", True)],
+                         ids=["one-launch", "per-layer", "per-layer-host-shards"])
+def test_round_kernel_restaging_between_rounds(cuda_device, dims, kernel, host):
+    """Both round paths stage the next round's mini-batches while the current
+    round runs (from host-resident shards, the per-layer path with a fixed
+    number of blocks striding over the tiles).  Between rounds: an evaluation
+    (which reuses the first input buffer), a tau override, new iteration
+    times (Algorithm 1 again) and a plain round; the staged data must follow
+    every change.  Against the oracle driven through the same changes."""
     from oracle import schedule as osched
-    w = synth.TrainWorkload("restage", 4, [784, 512, 10], 64, 0.05, 1024, 8, 1)
-    ctx, layers0 = make_context(w, device_shards(w, cuda_device, n=w.samples_per_worker), cuda_device,
-                                flags=P.FLAG_PROFILE)
+    w = synth.TrainWorkload("restage", 4, dims, 64, 0.05, 1024, 8, 1)
+    shards = device_shards(w, cuda_device, n=w.samples_per_worker)
+    if host:
+        shards = [(x.cpu().pin_memory(), y.cpu().pin_memory()) for x, y in shards]
+    ctx, layers0 = make_context(w, shards, cuda_device, flags=P.FLAG_PROFILE)
     Xe, ye = synth.eval_np(w, n=128)
     ex, ey = torch.from_numpy(Xe).to(cuda_device), torch.from_numpy(ye).to(cuda_device)
     t0 = oracle_schedule(w)[0]
@@ -540,7 +552,7 @@ def test_round_kernel_restaging_between_rounds(cuda_device):
             ctx.set_local_steps([2, 1, 3, 1])
         elif op == "ticks":
             ctx.set_iteration_ticks(t_new.tolist())
-    assert "fused_round" in ctx.profile()
+    assert kernel in ctx.profile()
     ctx.close()
 
     def oracle_run():
