@@ -498,8 +498,8 @@ def merge_workloads(args):
 # full-size launches are too large to capture; traffic grows in proportion to
 # P): (dram__bytes_read.sum + dram__bytes_write.sum) / ((W + 2) * P * 4).
 MERGE_TRAFFIC = {
-    64: (0.99621, "profiles/merge_vec4_P4M_W64.md (P = 4M, scaled by P)"),
-    8: (0.98790, "profiles/merge_vec4_P32M_W8.md (P = 32M, scaled by P)"),
+    64: (0.99694, "profiles/merge_vec4_P4M_W64.md (P = 4M, scaled by P)"),
+    8: (0.98816, "profiles/merge_vec4_P32M_W8.md (P = 32M, scaled by P)"),
 }
 
 

@@ -13,9 +13,10 @@
 //
 // In MLP mode the same pass also writes the bf16 operand copy of x_g.
 //
-// Grid: persistent, (SM count) x (resident CTAs per SM) blocks of 256
-// threads striding over 16-byte chunks; each thread keeps 16 independent
-// 16-byte loads in flight per group of 16 workers.
+// Grid: persistent, (SM count) x 3 blocks of 224 threads striding over
+// 16-byte chunks; each thread keeps 16 independent 16-byte loads in flight
+// per group of 16 workers (the rest in groups of 8, 4, 2 and 1), still
+// summing in worker order.
 //
 // Alignment: the vector kernel needs every buffer at the same offset modulo
 // 16 bytes.  When they share one offset that is not 0, the first (up to 3)
@@ -31,56 +32,67 @@ namespace oscars {
 
 namespace {
 
-constexpr int kThreads = 256;
+// 7 warps and 3 resident blocks per SM: the launch bounds cap a thread at 96
+// registers, enough for 16 float4 loads in flight (without the cap the
+// compiler picks 32 registers for full occupancy and the loads of a thread
+// run one after the other); 672 threads per SM cover the 407 K-parameter
+// model of the 784-512-10 MLP in one wave
+constexpr int kThreads = 224;
+constexpr int kMinBlocks = 3;
 constexpr int kGroup = 16;   // replica loads in flight per thread before the first is used
 
 __device__ __forceinline__ float4 ld_stream4(const float4* p) { return __ldcs(p); }
 
+// Workers [k, k + G) of 16-byte chunk i added to acc in worker order: all G
+// loads are issued before the first is used, so a thread keeps G of them in
+// flight (the kernel's launch bounds leave it the registers for 16).
+template <int G, bool kReplica>
+__device__ __forceinline__ void merge_group(const MergeArgs& a, int k, int64_t i, const float4& x, float4& acc) {
+  float4 v[G];
+#pragma unroll
+  for (int j = 0; j < G; ++j) v[j] = ld_stream4(reinterpret_cast<const float4*>(a.src[k + j]) + i);
+#pragma unroll
+  for (int j = 0; j < G; ++j) {
+    const float w = a.w[k + j];
+    if (kReplica) {
+      acc.x = fmaf(w, v[j].x - x.x, acc.x);
+      acc.y = fmaf(w, v[j].y - x.y, acc.y);
+      acc.z = fmaf(w, v[j].z - x.z, acc.z);
+      acc.w = fmaf(w, v[j].w - x.w, acc.w);
+    } else {
+      acc.x = fmaf(w, v[j].x, acc.x);
+      acc.y = fmaf(w, v[j].y, acc.y);
+      acc.z = fmaf(w, v[j].z, acc.z);
+      acc.w = fmaf(w, v[j].w, acc.w);
+    }
+  }
+}
+
 template <bool kReplica, bool kShadow>
-__global__ void __launch_bounds__(kThreads) merge_vec4_kernel(const __grid_constant__ MergeArgs a,
-                                                              float* __restrict__ x_g, int64_t n4,
-                                                              float eta, __nv_bfloat16* __restrict__ shadow) {
+__global__ void __launch_bounds__(kThreads, kMinBlocks) merge_vec4_kernel(const __grid_constant__ MergeArgs a,
+                                                                          float* __restrict__ x_g, int64_t n4,
+                                                                          float eta, __nv_bfloat16* __restrict__ shadow) {
   float4* xg4 = reinterpret_cast<float4*>(x_g);
   const int64_t stride = static_cast<int64_t>(gridDim.x) * blockDim.x;
   for (int64_t i = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n4; i += stride) {
     const float4 x = __ldcs(xg4 + i);
     float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
     int k = 0;
-    for (; k + kGroup <= a.W; k += kGroup) {
-      float4 v[kGroup];
-#pragma unroll
-      for (int j = 0; j < kGroup; ++j) v[j] = ld_stream4(reinterpret_cast<const float4*>(a.src[k + j]) + i);
-#pragma unroll
-      for (int j = 0; j < kGroup; ++j) {
-        const float w = a.w[k + j];
-        if (kReplica) {
-          acc.x = fmaf(w, v[j].x - x.x, acc.x);
-          acc.y = fmaf(w, v[j].y - x.y, acc.y);
-          acc.z = fmaf(w, v[j].z - x.z, acc.z);
-          acc.w = fmaf(w, v[j].w - x.w, acc.w);
-        } else {
-          acc.x = fmaf(w, v[j].x, acc.x);
-          acc.y = fmaf(w, v[j].y, acc.y);
-          acc.z = fmaf(w, v[j].z, acc.z);
-          acc.w = fmaf(w, v[j].w, acc.w);
-        }
-      }
+    for (; k + kGroup <= a.W; k += kGroup) merge_group<kGroup, kReplica>(a, k, i, x, acc);
+    // the rest in groups of 8, 4, 2 and 1, still in worker order
+    if (k + 8 <= a.W) {
+      merge_group<8, kReplica>(a, k, i, x, acc);
+      k += 8;
     }
-    for (; k < a.W; ++k) {
-      const float4 v = ld_stream4(reinterpret_cast<const float4*>(a.src[k]) + i);
-      const float w = a.w[k];
-      if (kReplica) {
-        acc.x = fmaf(w, v.x - x.x, acc.x);
-        acc.y = fmaf(w, v.y - x.y, acc.y);
-        acc.z = fmaf(w, v.z - x.z, acc.z);
-        acc.w = fmaf(w, v.w - x.w, acc.w);
-      } else {
-        acc.x = fmaf(w, v.x, acc.x);
-        acc.y = fmaf(w, v.y, acc.y);
-        acc.z = fmaf(w, v.z, acc.z);
-        acc.w = fmaf(w, v.w, acc.w);
-      }
+    if (k + 4 <= a.W) {
+      merge_group<4, kReplica>(a, k, i, x, acc);
+      k += 4;
     }
+    if (k + 2 <= a.W) {
+      merge_group<2, kReplica>(a, k, i, x, acc);
+      k += 2;
+    }
+    if (k < a.W) merge_group<1, kReplica>(a, k, i, x, acc);
     float4 out;
     out.x = fmaf(eta, acc.x, x.x);
     out.y = fmaf(eta, acc.y, x.y);
@@ -149,7 +161,7 @@ cudaError_t launch_merge(const MergeArgs& a, float* x_g, int64_t P, float eta, b
   if (head > P) head = P;
   for (int k = 0; k < a.W && vec; ++k) vec = (reinterpret_cast<uintptr_t>(a.src[k]) & 15) == off;
   if (vec && shadow) vec = (reinterpret_cast<uintptr_t>(shadow + head) & 7) == 0;
-  const int ctas_per_sm = 2048 / kThreads;
+  const int ctas_per_sm = kMinBlocks;
   const int64_t n4 = vec ? (P - head) / 4 : 0;
   if (n4 == 0) head = 0;
   if (n4 > 0) {
