@@ -317,19 +317,30 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
     fence_barrier_init();
     fence_proxy_async_smem();
   }
+  // thread 0: fp32 tiles [tb, tb + kMaxKb) of the global model's W0 block
+  // (the same for every worker of the cluster) by TMA into the
+  // resident-operand area, completing on ldW.  Columns past D are zero (TMA
+  // fill); every byte of the area that the tensor core reads later comes by
+  // TMA or from the weight-gradient epilogue, so it needs no clearing.
+  auto issue_w0f = [&](int tb) {
+    const int nb = nD - tb < kMaxKb ? nD - tb : kMaxKb;
+    mbar_arrive_expect_tx(ldW, nb * kW0Blk);   // an fp32 tile has the size of a bf16 K-block
+    for (int i = 0; i < nb; ++i) tma_load_3d(w0s + i * kW0Blk, &mW0f, col_begin + (tb + i) * kND, g0, 0, ldW);
+  };
+  if (t == 0) issue_w0f(0);   // the first worker's first tiles are in flight during the set-up
   if (warp == 2) {
     tmem_alloc(tmem_slot, 512);
     tmem_relinquish();
   }
-  // zero the dz0^T tile (its K padding must stay zero for B < 64) and the
-  // resident W0 (columns past the CTA's own stay zero)
+  // zero the dz0^T tile (its K padding must stay zero for B < 64)
   for (int i = t; i < Cfg::kDzT / 16; i += kFT) reinterpret_cast<uint4*>(dzT)[i] = make_uint4(0, 0, 0, 0);
-  for (int i = t; i < kMaxKb * kW0Blk / 16; i += kFT) reinterpret_cast<uint4*>(w0s)[i] = make_uint4(0, 0, 0, 0);
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *tmem_slot;
-  if (S > 1) cluster_sync();  // every CTA's barriers are initialised before a peer signals them
+  // every CTA's barriers are initialised before a peer signals them: the
+  // arrival here, the wait before the first step
+  if (S > 1) cluster_arrive();
   bool producer_ok = true;
   bool chain_ok = true;    // warps 1 and 3: no wait of this chain has run out
   int chain_tiles = 0;     // warps 1 and 3: tiles issued by this chain so far
@@ -396,10 +407,7 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
     }
     for (int tb = 0; tb < nD; tb += kMaxKb) {
       const int nb = nD - tb < kMaxKb ? nD - tb : kMaxKb;
-      if (t == 0) {
-        mbar_arrive_expect_tx(ldW, nb * kW0Blk);   // an fp32 tile has the size of a bf16 K-block
-        for (int i = 0; i < nb; ++i) tma_load_3d(w0s + i * kW0Blk, &mW0f, col_begin + (tb + i) * kND, g0, 0, ldW);
-      }
+      if (t == 0 && (tb > 0 || wi != a.cl_first[blockIdx.x])) issue_w0f(tb);
       if (warp >= 4) {
         const int quarter = warp & 3, eg = (warp - 4) >> 2;
         const int r = quarter * 32 + lane;
@@ -434,6 +442,7 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
+    if (S > 1 && wi == a.cl_first[blockIdx.x]) cluster_wait();
 
     for (int s = 0; s < tau; ++s) {
       if (stamp) a.phase_ts[s * 4 + 0] = global_ns();
@@ -1042,6 +1051,8 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
   }
   // the last drain of each chain's buffer pairs with one more wait
   if ((warp == 1 || warp == 3) && chain_tiles > 0) bar_named(1 + (warp == 1 ? 0 : 1), 128 + 32);
+  // (a cluster without workers still completes the set-up barrier)
+  if (S > 1 && a.cl_first[blockIdx.x] == a.cl_first[blockIdx.x + 1]) cluster_wait();
   cluster_sync();   // peers may still read this CTA's partial logits of the last step
   tc_fence_before();
   __syncthreads();
