@@ -201,7 +201,7 @@ struct oscars_ctx {
   __nv_bfloat16* A0Tb[2] = {};
   int32_t* labb[2] = {};
   CUtensorMap mX4b[2], mXT4b[2];
-  CUtensorMap mW0f, mW0b;               // the global slot's W0 (fp32 and its bf16 copy) for the round kernel
+  CUtensorMap mW0f;                     // the global slot's fp32 W0 for the round kernel
   int parity = 0;
   bool staged = false;                  // A0b[parity] holds the mini-batches of the next round
   cudaGraphExec_t ahead_exec[2] = {};   // round graphs, one per parity
@@ -471,11 +471,10 @@ oscars_status ensure_stage_buffers(oscars_ctx* c) {
           !make_map4(&c->mXT4b[i], c->A0Tb[i], B, D, W, cap, B * 2ull, static_cast<uint64_t>(B) * D * 2ull, per_b,
                      fused_round_xt_rows(B)))
         return fail(c, OSCARS_ECUDA, "cuTensorMapEncodeTiled failed (fused round inputs)");
-    // the global slot's W0: fp32 tiles of 128 rows x 32 columns, bf16 K-blocks of 128 rows x 64
+    // the global slot's W0: fp32 tiles of 128 rows x 32 columns
     const int64_t gw0 = static_cast<int64_t>(W) * c->P_pad + c->layers[0].offW;
     const uint64_t H = static_cast<uint64_t>(c->dims[1]);
-    if (!make_map_f32(&c->mW0f, c->slab + gw0, D, H, 1, D * 4ull, D * H * 4ull, 128) ||
-        !make_map(&c->mW0b, c->shadow + gw0, D, H, 1, D * 2ull, D * H * 2ull, 128))
+    if (!make_map_f32(&c->mW0f, c->slab + gw0, D, H, 1, D * 4ull, D * H * 4ull, 128))
       return fail(c, OSCARS_ECUDA, "cuTensorMapEncodeTiled failed (fused round model)");
   }
   // step 0 doubles as the single-step buffers (evaluation)
@@ -831,7 +830,7 @@ cudaError_t enqueue_round_fused_ahead(oscars_ctx* c, int buf, cudaStream_t st) {
   if (c->profiling) {
     {
       ProfScope ps(c, "fused_round", st);
-      if ((e = launch_fused_round(c->mX4b[buf], c->mXT4b[buf], c->mW0f, c->mW0b, f, st)) != cudaSuccess) return e;
+      if ((e = launch_fused_round(c->mX4b[buf], c->mXT4b[buf], c->mW0f, f, st)) != cudaSuccess) return e;
     }
     {
       ProfScope ps(c, "stage", st);
@@ -843,7 +842,7 @@ cudaError_t enqueue_round_fused_ahead(oscars_ctx* c, int buf, cudaStream_t st) {
   if ((e = cudaEventRecord(c->side_fork, st)) != cudaSuccess) return e;
   if ((e = cudaStreamWaitEvent(c->side, c->side_fork, 0)) != cudaSuccess) return e;
   f.priority = c->prio_greatest;
-  if ((e = launch_fused_round(c->mX4b[buf], c->mXT4b[buf], c->mW0f, c->mW0b, f, st)) != cudaSuccess) return e;
+  if ((e = launch_fused_round(c->mX4b[buf], c->mXT4b[buf], c->mW0f, f, st)) != cudaSuccess) return e;
   if ((e = launch_stage_round_priority(sa, c->tau_dev, c->W, c->max_tau, c->prio_least, c->side)) != cudaSuccess)
     return e;
   if ((e = launch_cursor_advance(c->cursor, c->tau_dev, c->dn_tab, c->B, c->W, c->side)) != cudaSuccess) return e;

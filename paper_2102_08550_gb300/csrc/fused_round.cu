@@ -230,7 +230,6 @@ template <int B, int S>
 __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_constant__ CUtensorMap mX,
                                                                  const __grid_constant__ CUtensorMap mXT,
                                                                  const __grid_constant__ CUtensorMap mW0f,
-                                                                 const __grid_constant__ CUtensorMap mW0b,
                                                                  const __grid_constant__ FusedArgs a) {
   using Cfg = FCfg<B, S>;
   constexpr int UPC = Cfg::kUPC;
@@ -298,7 +297,6 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
     prefetch_tmap(&mX);
     prefetch_tmap(&mXT);
     prefetch_tmap(&mW0f);
-    prefetch_tmap(&mW0b);
     for (int i = 0; i < Cfg::kStagesF; ++i) {
       mbar_init(&fullF[i], 1);
       mbar_init(&emptyF[i], 1);
@@ -386,10 +384,9 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
     // the global model, once per worker.  Warps 0-3: head columns and
     // biases.  The fp32 master block comes by TMA in tiles of 128 rows x 32
     // columns, up to kMaxKb at a time, into the resident-operand area (not in
-    // use yet); the epilogue warps move each row to TMEM.  Then the bf16
-    // operand itself comes by TMA from the global slot's bf16 copy (the
-    // round-to-nearest bf16 of the same values).  Columns past D are zero (TMA
-    // fill).
+    // use yet); the epilogue warps move each row to TMEM.  Then they write the
+    // bf16 operand, rounded from the master in TMEM.  Columns past D are zero
+    // (TMA fill).
     // the first X tiles of step 0 go out first (the F ring is free: the
     // previous worker's write-back has read it before the last barrier)
     if (warp == 0 && lane == 0) producer_ok = issue_f(0, 0, pre_f);
@@ -430,14 +427,31 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
         tmem_wait_st();
       }
       ++ld_phase;
+      tc_fence_before();
       __syncthreads();   // the tiles have been read before the area is written again
+      tc_fence_after();
     }
-    if (t == 0) {
-      mbar_arrive_expect_tx(ldW, nkf * kW0Blk);
-      for (int j = 0; j < nkf; ++j) tma_load_3d(w0s + j * kW0Blk, &mW0b, col_begin + j * kFBK, g0, 0, ldW);
+    // the bf16 operand: the round-to-nearest bf16 of the fp32 master just
+    // stored (the global model), K-block by K-block from TMEM into the
+    // resident-operand area; columns past the CTA's last 32-column tile are
+    // zero
+    if (warp >= 4) {
+      const int quarter = warp & 3, eg = (warp - 4) >> 2;
+      const int r = quarter * 32 + lane;
+      const uint32_t trow = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
+      for (int j = eg; j < nkf; j += 2) {   // 2j < nD always
+        float v0[32], v1[32];
+        if (2 * j + 1 < nD) {
+          tmem_ld_32x32b_x32_pair(trow + 2 * j * kND, v0, trow + (2 * j + 1) * kND, v1);
+        } else {
+          tmem_ld_32x32b_x32(trow + 2 * j * kND, v0);
+#pragma unroll
+          for (int i = 0; i < 32; ++i) v1[i] = 0.f;
+        }
+        put_w0_cols<32>(w0s, r, j * kFBK, v0);
+        put_w0_cols<32>(w0s, r, j * kFBK + 32, v1);
+      }
     }
-    mbar_wait(ldW, ld_phase & 1, a.err, kDevTimeoutFull);
-    ++ld_phase;
     fence_proxy_async_smem();   // the resident W0 is read by the tensor core
     tc_fence_before();
     __syncthreads();
@@ -1063,8 +1077,8 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
 }
 
 template <int B, int S>
-cudaError_t launch_bs(const CUtensorMap& mX, const CUtensorMap& mXT, const CUtensorMap& mW0f, const CUtensorMap& mW0b,
-                      const FusedArgs& a, int priority, cudaStream_t s) {
+cudaError_t launch_bs(const CUtensorMap& mX, const CUtensorMap& mXT, const CUtensorMap& mW0f, const FusedArgs& a,
+                      int priority, cudaStream_t s) {
   using Cfg = FCfg<B, S>;
   cudaError_t e = cudaFuncSetAttribute(fused_mlp2_round_kernel<B, S>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        Cfg::kSmem);
@@ -1088,7 +1102,7 @@ cudaError_t launch_bs(const CUtensorMap& mX, const CUtensorMap& mXT, const CUten
   }
   cfg.attrs = attr;
   cfg.numAttrs = n;
-  return cudaLaunchKernelEx(&cfg, fused_mlp2_round_kernel<B, S>, mX, mXT, mW0f, mW0b, a);
+  return cudaLaunchKernelEx(&cfg, fused_mlp2_round_kernel<B, S>, mX, mXT, mW0f, a);
 }
 
 // two CTAs per unit group when the cluster stays within 8 CTAs and the input
@@ -1153,7 +1167,7 @@ int fused_round_max_clusters(int D, int H, int B) {
 }
 
 cudaError_t launch_fused_round(const CUtensorMap& mX, const CUtensorMap& mXT, const CUtensorMap& mW0f,
-                               const CUtensorMap& mW0b, const FusedRoundArgs& r, cudaStream_t s) {
+                               const FusedRoundArgs& r, cudaStream_t s) {
   FusedArgs a;
   a.tau = r.tau;
   a.order = r.order;
@@ -1180,11 +1194,11 @@ cudaError_t launch_fused_round(const CUtensorMap& mX, const CUtensorMap& mXT, co
   a.shard_n = r.shard_n;
   const int S = split_for(r.D, r.H);
   if (r.B == 32)
-    return S == 2 ? launch_bs<32, 2>(mX, mXT, mW0f, mW0b, a, r.priority, s)
-                  : launch_bs<32, 1>(mX, mXT, mW0f, mW0b, a, r.priority, s);
+    return S == 2 ? launch_bs<32, 2>(mX, mXT, mW0f, a, r.priority, s)
+                  : launch_bs<32, 1>(mX, mXT, mW0f, a, r.priority, s);
   if (r.B == 64)
-    return S == 2 ? launch_bs<64, 2>(mX, mXT, mW0f, mW0b, a, r.priority, s)
-                  : launch_bs<64, 1>(mX, mXT, mW0f, mW0b, a, r.priority, s);
+    return S == 2 ? launch_bs<64, 2>(mX, mXT, mW0f, a, r.priority, s)
+                  : launch_bs<64, 1>(mX, mXT, mW0f, a, r.priority, s);
   return cudaErrorInvalidValue;
 }
 
