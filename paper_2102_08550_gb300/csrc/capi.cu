@@ -100,15 +100,16 @@ bool make_map_box4(CUtensorMap* m, const void* base, const uint64_t (&d)[4], con
 
 // 3-D fp32 tensor map, boxes of 32 x box_y x 1 (128-byte rows), 128-byte swizzle
 bool make_map_f32(CUtensorMap* m, const void* base, uint64_t dx, uint64_t dy, uint64_t dz, uint64_t stride_y,
-                  uint64_t stride_z, uint32_t box_y) {
+                  uint64_t stride_z, uint32_t box_y, uint32_t box_x = 32,
+                  CUtensorMapSwizzle swz = CU_TENSOR_MAP_SWIZZLE_128B) {
   EncodeTiledFn f = encode_fn();
   if (!f) return false;
   cuuint64_t dims[3] = {dx, dy, dz};
   cuuint64_t strides[2] = {stride_y, stride_z};
-  cuuint32_t box[3] = {32, box_y, 1};
+  cuuint32_t box[3] = {box_x, box_y, 1};
   cuuint32_t es[3] = {1, 1, 1};
   return f(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, const_cast<void*>(base), dims, strides, box, es,
-           CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+           CU_TENSOR_MAP_INTERLEAVE_NONE, swz, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
@@ -202,6 +203,7 @@ struct oscars_ctx {
   int32_t* labb[2] = {};
   CUtensorMap mX4b[2], mXT4b[2];
   CUtensorMap mW0f;                     // the global slot's fp32 W0 for the round kernel
+  CUtensorMap mRep32, mRep16;           // every replica slot's W0 (the round kernel's last-step stores)
   int parity = 0;
   bool staged = false;                  // A0b[parity] holds the mini-batches of the next round
   cudaGraphExec_t ahead_exec[2] = {};   // round graphs, one per parity
@@ -474,7 +476,14 @@ oscars_status ensure_stage_buffers(oscars_ctx* c) {
     // the global slot's W0: fp32 tiles of 128 rows x 32 columns
     const int64_t gw0 = static_cast<int64_t>(W) * c->P_pad + c->layers[0].offW;
     const uint64_t H = static_cast<uint64_t>(c->dims[1]);
-    if (!make_map_f32(&c->mW0f, c->slab + gw0, D, H, 1, D * 4ull, D * H * 4ull, 128))
+    // every replica slot's W0, for the last step's stores: boxes of 32 rows
+    // x 32 (swizzled) and x 16 columns
+    const int64_t rw0 = c->layers[0].offW;
+    const uint64_t slots = static_cast<uint64_t>(W);
+    if (!make_map_f32(&c->mW0f, c->slab + gw0, D, H, 1, D * 4ull, D * H * 4ull, 128) ||
+        !make_map_f32(&c->mRep32, c->slab + rw0, D, H, slots, D * 4ull, static_cast<uint64_t>(c->P_pad) * 4ull, 32) ||
+        !make_map_f32(&c->mRep16, c->slab + rw0, D, H, slots, D * 4ull, static_cast<uint64_t>(c->P_pad) * 4ull, 32, 16,
+                      CU_TENSOR_MAP_SWIZZLE_NONE))
       return fail(c, OSCARS_ECUDA, "cuTensorMapEncodeTiled failed (fused round model)");
   }
   // step 0 doubles as the single-step buffers (evaluation)
@@ -830,7 +839,7 @@ cudaError_t enqueue_round_fused_ahead(oscars_ctx* c, int buf, cudaStream_t st) {
   if (c->profiling) {
     {
       ProfScope ps(c, "fused_round", st);
-      if ((e = launch_fused_round(c->mX4b[buf], c->mXT4b[buf], c->mW0f, f, st)) != cudaSuccess) return e;
+      if ((e = launch_fused_round(c->mX4b[buf], c->mXT4b[buf], c->mW0f, c->mRep32, c->mRep16, f, st)) != cudaSuccess) return e;
     }
     {
       ProfScope ps(c, "stage", st);
@@ -842,7 +851,7 @@ cudaError_t enqueue_round_fused_ahead(oscars_ctx* c, int buf, cudaStream_t st) {
   if ((e = cudaEventRecord(c->side_fork, st)) != cudaSuccess) return e;
   if ((e = cudaStreamWaitEvent(c->side, c->side_fork, 0)) != cudaSuccess) return e;
   f.priority = c->prio_greatest;
-  if ((e = launch_fused_round(c->mX4b[buf], c->mXT4b[buf], c->mW0f, f, st)) != cudaSuccess) return e;
+  if ((e = launch_fused_round(c->mX4b[buf], c->mXT4b[buf], c->mW0f, c->mRep32, c->mRep16, f, st)) != cudaSuccess) return e;
   if ((e = launch_stage_round_priority(sa, c->tau_dev, c->W, c->max_tau, c->prio_least, c->side)) != cudaSuccess)
     return e;
   if ((e = launch_cursor_advance(c->cursor, c->tau_dev, c->dn_tab, c->B, c->W, c->side)) != cudaSuccess) return e;

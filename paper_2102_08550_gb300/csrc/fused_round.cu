@@ -99,13 +99,19 @@ constexpr int kFU = 128;               // hidden units per group (tensor-core ro
 constexpr int kFC = 10;                // classes
 constexpr int kFMaxCluster = 8;
 constexpr int kFBK = 64;               // K-block (bf16 elements, 128 bytes)
-constexpr int kND = 32;                // columns per fp32 model tile (the load and the write-back)
+constexpr int kND = 32;                // columns per fp32 model tile (the load)
+// replica staging of the last step, per epilogue warp: two 32 x 32 fp32
+// boxes and two 32 x 16 boxes (1024-byte aligned for the swizzled ones)
+constexpr int kStg32 = 32 * 32 * 4, kStg16 = 32 * 16 * 4;
+constexpr int kStgBytes = 2 * kStg32 + 2 * kStg16;
 constexpr int kDT = 48;                // columns per weight-gradient tile
 constexpr int kNBD = 2;                // weight-gradient TMEM buffers (one per issuing chain)
 constexpr int kNXD = 4;                // X^T tile buffers in shared memory (even: two per issuing chain)
 constexpr int kTAcc = 512 - kNBD * kDT;   // first TMEM column of the accumulators = master columns (416)
 constexpr int kMaxKb = (kTAcc + kFBK - 1) / kFBK;   // resident K-blocks of W0
 constexpr int kW0Blk = kFU * kFBK * 2; // one resident K-block: 128 rows x 64 columns bf16
+static_assert((kFT / 32 - 4) * kStgBytes <= kMaxKb * kW0Blk && kStgBytes % 1024 == 0 && kStg32 % 1024 == 0,
+              "the replica staging of the epilogue warps fits the resident-operand area, 1024-byte aligned");
 
 __device__ __forceinline__ unsigned long long global_ns() {
   unsigned long long v;
@@ -230,6 +236,8 @@ template <int B, int S>
 __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_constant__ CUtensorMap mX,
                                                                  const __grid_constant__ CUtensorMap mXT,
                                                                  const __grid_constant__ CUtensorMap mW0f,
+                                                                 const __grid_constant__ CUtensorMap mRep32,
+                                                                 const __grid_constant__ CUtensorMap mRep16,
                                                                  const __grid_constant__ FusedArgs a) {
   using Cfg = FCfg<B, S>;
   constexpr int UPC = Cfg::kUPC;
@@ -285,7 +293,7 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
   const int col_end = half == S - 1 ? D : kb_end * kFBK;
   const int ncols = col_end - col_begin;        // a multiple of 8
   const int nkf = kb_end - kb_begin;
-  const int nD = (ncols + kND - 1) / kND;        // 32-column model tiles (load, write-back)
+  const int nD = (ncols + kND - 1) / kND;        // 32-column model tiles (load)
   const int nT = (ncols + kDT - 1) / kDT;        // 48-column weight-gradient tiles
   const int ncols16 = (ncols + 15) & ~15;        // columns the weight-gradient epilogue updates
   const int pre_f = nkf < Cfg::kStagesF ? nkf : Cfg::kStagesF;   // X tiles loaded ahead of a step
@@ -297,6 +305,8 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
     prefetch_tmap(&mX);
     prefetch_tmap(&mXT);
     prefetch_tmap(&mW0f);
+    prefetch_tmap(&mRep32);
+    prefetch_tmap(&mRep16);
     for (int i = 0; i < Cfg::kStagesF; ++i) {
       mbar_init(&fullF[i], 1);
       mbar_init(&emptyF[i], 1);
@@ -388,7 +398,7 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
     // bf16 operand, rounded from the master in TMEM.  Columns past D are zero
     // (TMA fill).
     // the first X tiles of step 0 go out first (the F ring is free: the
-    // previous worker's write-back has read it before the last barrier)
+    // previous worker's last forward has consumed it before the last barrier)
     if (warp == 0 && lane == 0) producer_ok = issue_f(0, 0, pre_f);
     if (warp < 4) {
       for (int q = t; q < kFC * (UPC / 4); q += 128) {
@@ -973,6 +983,13 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
         const int quarter = warp & 3, eg = (warp - 4) >> 2;
         const int r = quarter * 32 + lane;
         const uint32_t trow = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
+        // the last step's updated master goes to the worker's replica slot by
+        // TMA stores from two staging buffers per warp in the resident-operand
+        // area (not read again by this worker once the step's forward has
+        // run): 32 columns as a 128-byte-swizzled 32 x 32 box, 16 columns as
+        // a plain 32 x 16 box
+        uint8_t* stg = w0s + (warp - 4) * kStgBytes;
+        int nst = 0;   // tiles this warp has stored
         for (int tt = ((sg * nT + eg) & 1); tt < nT; tt += 2) {
           const int c = sg * nT + tt, buf = eg, use = c / kNBD;
           int ok = mbar_wait(&accD[buf], use & 1, a.err, kDevTimeoutAccum) ? 1 : 0;
@@ -994,21 +1011,51 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
             if (has16) tmem_ld_32x32b_x16(gcol + (has32 ? 32 : 0), g16);
             tc_fence_before();
             bar_arrive_named(1 + eg, 128 + 32);   // the gradient buffer has been read: the next MMA may reuse it
+            uint8_t* st32 = stg + (nst & 1) * kStg32;
+            uint8_t* st16 = stg + 2 * kStg32 + (nst & 1) * kStg16;
+            if (last) {   // the store of two tiles ago has read this buffer pair
+              if (lane == 0 && nst >= 2) bulk_wait_read_but_one();
+              __syncwarp();
+            }
             if (has32) {
               float m[32];
               tmem_ld_32x32b_x32(trow + c0, m);
 #pragma unroll
               for (int j = 0; j < 32; ++j) m[j] = fmaf(-a.lr, g[j], m[j]);
-              tmem_st_32x32b_x32(trow + c0, m);
-              put_w0_cols<32>(w0s, r, c0, m);
+              if (!last) {
+                tmem_st_32x32b_x32(trow + c0, m);
+                put_w0_cols<32>(w0s, r, c0, m);
+              } else {   // row `lane`: 16-byte chunk q at (q ^ (lane & 7))
+#pragma unroll
+                for (int q = 0; q < 8; ++q)
+                  *reinterpret_cast<float4*>(st32 + lane * 128 + ((q ^ (lane & 7)) << 4)) =
+                      make_float4(m[4 * q], m[4 * q + 1], m[4 * q + 2], m[4 * q + 3]);
+              }
             }
             if (has16) {
               float m16[16];
               tmem_ld_32x32b_x16(trow + c16, m16);
 #pragma unroll
               for (int j = 0; j < 16; ++j) m16[j] = fmaf(-a.lr, g16[j], m16[j]);
-              tmem_st_32x32b_x16(trow + c16, m16);
-              put_w0_cols<16>(w0s, r, c16, m16);
+              if (!last) {
+                tmem_st_32x32b_x16(trow + c16, m16);
+                put_w0_cols<16>(w0s, r, c16, m16);
+              } else {
+#pragma unroll
+                for (int q = 0; q < 4; ++q)
+                  *reinterpret_cast<float4*>(st16 + lane * 64 + q * 16) =
+                      make_float4(m16[4 * q], m16[4 * q + 1], m16[4 * q + 2], m16[4 * q + 3]);
+              }
+            }
+            if (last) {
+              fence_proxy_async_smem();   // the staged rows are read by the TMA store
+              __syncwarp();
+              if (lane == 0) {
+                if (has32) tma_store_3d(&mRep32, st32, col_begin + c0, g0 + quarter * 32, w);
+                if (has16) tma_store_3d(&mRep16, st16, col_begin + c16, g0 + quarter * 32, w);
+                bulk_commit_group();
+              }
+              ++nst;
             }
           } else {
             tc_fence_before();
@@ -1016,6 +1063,8 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
           }
         }
         tmem_wait_st();   // the master columns stored above are read again next step
+        // the staging buffers are read before the next worker's model comes in
+        if (last && lane == 0) bulk_wait_read_all();
       }
       fence_proxy_async_smem();   // the resident W0 written here is read by the tensor core next step
       tc_fence_before();
@@ -1023,41 +1072,14 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
       tc_fence_after();
       if (stamp) a.phase_ts[s * 4 + 3] = global_ns();
     }
-    // the worker's W0 block into its replica slot: each warp moves 32 rows x
-    // 32 columns at a time from TMEM through a padded shared tile (the TMA
-    // rings are idle now), 4 full 128-byte rows per store instruction
-    if (warp >= 4) {
-      const int quarter = warp & 3, eg = (warp - 4) >> 2;
-      const uint32_t trow = tmem + (static_cast<uint32_t>(quarter * 32) << 16);
-      float* T = reinterpret_cast<float*>(sm + Cfg::oRegion) + (warp - 4) * 32 * 36;
-      float* dst = a.master_w + dof + a.offW0 + static_cast<int64_t>(g0 + quarter * 32) * D + col_begin;
-      const int cq = (lane & 7) * 4;
-      for (int tt = eg; tt < nD; tt += 2) {
-        const int c0 = tt * kND;
-        float m[32];
-        tmem_ld_32x32b_x32(trow + c0, m);
-#pragma unroll
-        for (int q = 0; q < 8; ++q)
-          *reinterpret_cast<float4*>(T + lane * 36 + 4 * q) =
-              make_float4(m[4 * q], m[4 * q + 1], m[4 * q + 2], m[4 * q + 3]);
-        __syncwarp();
-        if (c0 + cq < ncols) {
-#pragma unroll
-          for (int i = 0; i < 8; ++i) {
-            const int rr = 4 * i + (lane >> 3);
-            *reinterpret_cast<float4*>(dst + static_cast<int64_t>(rr) * D + c0 + cq) =
-                *reinterpret_cast<const float4*>(T + rr * 36 + cq);
-          }
-        }
-        __syncwarp();
-      }
-    }
-    // round bookkeeping of this worker: mean loss over its steps and the data cursor
+    // round bookkeeping of this worker (its W0 block went to its replica slot
+    // by TMA stores in the last step): mean loss over its steps and the data
+    // cursor
     if (rank == 0 && t == 0) {
       a.loss_out[w] = static_cast<float>(loss_sum / (static_cast<double>(B) * tau));
       if (a.cursor) a.cursor[w] = (a.cursor[w] + static_cast<int64_t>(tau) * B) % a.shard_n[w];
     }
-    // the write-back has read TMEM and the shared tile before the next worker's model goes in
+    // the last step has read TMEM before the next worker's model goes in
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -1065,6 +1087,8 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
   }
   // the last drain of each chain's buffer pairs with one more wait
   if ((warp == 1 || warp == 3) && chain_tiles > 0) bar_named(1 + (warp == 1 ? 0 : 1), 128 + 32);
+  // every replica store has completed before the kernel ends
+  if (warp >= 4 && lane == 0) bulk_wait_all();
   // (a cluster without workers still completes the set-up barrier)
   if (S > 1 && a.cl_first[blockIdx.x] == a.cl_first[blockIdx.x + 1]) cluster_wait();
   cluster_sync();   // peers may still read this CTA's partial logits of the last step
@@ -1077,8 +1101,8 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
 }
 
 template <int B, int S>
-cudaError_t launch_bs(const CUtensorMap& mX, const CUtensorMap& mXT, const CUtensorMap& mW0f, const FusedArgs& a,
-                      int priority, cudaStream_t s) {
+cudaError_t launch_bs(const CUtensorMap& mX, const CUtensorMap& mXT, const CUtensorMap& mW0f, const CUtensorMap& mRep32,
+                      const CUtensorMap& mRep16, const FusedArgs& a, int priority, cudaStream_t s) {
   using Cfg = FCfg<B, S>;
   cudaError_t e = cudaFuncSetAttribute(fused_mlp2_round_kernel<B, S>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        Cfg::kSmem);
@@ -1102,7 +1126,7 @@ cudaError_t launch_bs(const CUtensorMap& mX, const CUtensorMap& mXT, const CUten
   }
   cfg.attrs = attr;
   cfg.numAttrs = n;
-  return cudaLaunchKernelEx(&cfg, fused_mlp2_round_kernel<B, S>, mX, mXT, mW0f, a);
+  return cudaLaunchKernelEx(&cfg, fused_mlp2_round_kernel<B, S>, mX, mXT, mW0f, mRep32, mRep16, a);
 }
 
 // two CTAs per unit group when the cluster stays within 8 CTAs and the input
@@ -1167,7 +1191,8 @@ int fused_round_max_clusters(int D, int H, int B) {
 }
 
 cudaError_t launch_fused_round(const CUtensorMap& mX, const CUtensorMap& mXT, const CUtensorMap& mW0f,
-                               const FusedRoundArgs& r, cudaStream_t s) {
+                               const CUtensorMap& mRep32, const CUtensorMap& mRep16, const FusedRoundArgs& r,
+                               cudaStream_t s) {
   FusedArgs a;
   a.tau = r.tau;
   a.order = r.order;
@@ -1194,11 +1219,11 @@ cudaError_t launch_fused_round(const CUtensorMap& mX, const CUtensorMap& mXT, co
   a.shard_n = r.shard_n;
   const int S = split_for(r.D, r.H);
   if (r.B == 32)
-    return S == 2 ? launch_bs<32, 2>(mX, mXT, mW0f, a, r.priority, s)
-                  : launch_bs<32, 1>(mX, mXT, mW0f, a, r.priority, s);
+    return S == 2 ? launch_bs<32, 2>(mX, mXT, mW0f, mRep32, mRep16, a, r.priority, s)
+                  : launch_bs<32, 1>(mX, mXT, mW0f, mRep32, mRep16, a, r.priority, s);
   if (r.B == 64)
-    return S == 2 ? launch_bs<64, 2>(mX, mXT, mW0f, a, r.priority, s)
-                  : launch_bs<64, 1>(mX, mXT, mW0f, a, r.priority, s);
+    return S == 2 ? launch_bs<64, 2>(mX, mXT, mW0f, mRep32, mRep16, a, r.priority, s)
+                  : launch_bs<64, 1>(mX, mXT, mW0f, mRep32, mRep16, a, r.priority, s);
   return cudaErrorInvalidValue;
 }
 

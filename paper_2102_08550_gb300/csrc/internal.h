@@ -228,9 +228,12 @@ int fused_round_max_clusters(int D, int H, int B);
 // mX: staged inputs {D, B, W, steps} box {64, B}; mXT: staged transposed
 // inputs {B, D, W, steps} box {64, fused_round_xt_rows(B)}; both bf16,
 // 128-byte swizzle.  mW0f: the global slot's W0 {D, H, 1} fp32, box
-// {32, 128}, 128-byte swizzle (the kernel rounds its own bf16 operand)
+// {32, 128}, 128-byte swizzle (the kernel rounds its own bf16 operand).
+// mRep32 / mRep16: W0 of every replica slot {D, H, slots} fp32, box
+// {32, 32} with 128-byte swizzle / {16, 32} without (the last step's stores)
 cudaError_t launch_fused_round(const CUtensorMap& mX, const CUtensorMap& mXT, const CUtensorMap& mW0f,
-                               const FusedRoundArgs& a, cudaStream_t s);
+                               const CUtensorMap& mRep32, const CUtensorMap& mRep16, const FusedRoundArgs& a,
+                               cudaStream_t s);
 
 // loss[w] = sum_{s < tau[w]} sum_c part[(w*max_tau + s)*nc + c] / (B * tau[w])
 cudaError_t launch_loss_finalize(const float* part, const int32_t* tau, int W, int max_tau,
