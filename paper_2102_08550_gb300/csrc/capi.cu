@@ -265,6 +265,9 @@ struct oscars_ctx {
   // losses and one event per slot (rounds pipelined one deep)
   float* train_loss_host = nullptr;
   cudaEvent_t train_done[2] = {nullptr, nullptr};
+  // oscars_train with staged-ahead rounds: the round from input buffer b, the
+  // loss copy into host slot h and the merge, captured as one graph [b][h]
+  cudaGraphExec_t train_exec[2][2] = {};
 };
 
 namespace {
@@ -368,6 +371,14 @@ bool dev_alloc(oscars_ctx* c, T** p, size_t count) {
   return true;
 }
 
+void destroy_train_graphs(oscars_ctx* c) {
+  for (auto& row : c->train_exec)
+    for (auto& g : row) {
+      if (g) cudaGraphExecDestroy(g);
+      g = nullptr;
+    }
+}
+
 void free_all(oscars_ctx* c) {
   for (auto& p : c->prof_pending)
     if (!p.graph_owned) {
@@ -398,6 +409,7 @@ void free_all(oscars_ctx* c) {
     if (g) cudaGraphExecDestroy(g);
     g = nullptr;
   }
+  destroy_train_graphs(c);
   for (void* p : c->allocs) cudaFree(p);
   c->allocs.clear();
   if (c->cap) cudaStreamDestroy(c->cap);
@@ -597,6 +609,7 @@ oscars_status build_tables(oscars_ctx* c) {
     cudaGraphExecDestroy(c->merge_exec);
     c->merge_exec = nullptr;
   }
+  destroy_train_graphs(c);
   return ensure_stage_buffers(c);
 }
 
@@ -614,6 +627,29 @@ cudaError_t refresh_global_shadows(oscars_ctx* c, cudaStream_t s, bool plain_don
     if (e != cudaSuccess) return e;
   }
   return cudaSuccess;
+}
+
+// Eq. 4, first branch, over the workers' replica slots: x_g += eta sum_k
+// w_k (x^k - x_g) with the weights w, the bf16 copy of x_g in the same pass
+// (and, for the CNN, its transposed copies)
+cudaError_t enqueue_replica_merge(oscars_ctx* c, const float* w, cudaStream_t st) {
+  MergeArgs a;
+  std::memset(&a, 0, sizeof(a));
+  a.W = c->W;
+  for (int k = 0; k < c->W; ++k) {
+    a.w[k] = w[k];
+    a.src[k] = c->slab + static_cast<int64_t>(k) * c->P_pad;
+  }
+  const int64_t g = static_cast<int64_t>(c->W) * c->P_pad;
+  cudaError_t r;
+  {
+    ProfScope ps(c, "merge", st);
+    r = launch_merge(a, c->slab + g, c->P_pad, c->server_lr, true, st, c->shadow ? c->shadow + g : nullptr);
+  }
+  if (r != cudaSuccess) return r;
+  if (c->model != OSCARS_MODEL_CNN) return cudaSuccess;   // no transposed copies to refresh
+  ProfScope ps(c, "shadow_refresh", st);
+  return refresh_global_shadows(c, st, true);
 }
 
 GemmArgs gemm_base(oscars_ctx* c, const int* wid, const int* src) {
@@ -1489,6 +1525,36 @@ cudaError_t copy_canonical(oscars_ctx* c, float* padded, const float* canon, boo
   return cudaSuccess;
 }
 
+// the round from input buffer b (staged by the round before) with, beside
+// it, the staging of the next round into the other buffer
+cudaError_t enqueue_ahead(oscars_ctx* c, int b, cudaStream_t s0) {
+  return c->fused ? enqueue_round_fused_ahead(c, b, s0) : enqueue_round_mlp_ahead(c, b, s0);
+}
+
+// the first staged-ahead round (or the first after tau changed or an
+// evaluation) stages its own mini-batches into buffer b first
+cudaError_t stage_own_round(oscars_ctx* c, int b) {
+  c->profiling = (c->flags & 2) != 0;
+  cudaError_t e;
+  {
+    ProfScope ps(c, "stage", c->stream);
+    e = launch_stage_round(stage_args(c, b, nullptr), c->tau_dev, c->W, c->max_tau, c->stream);
+  }
+  c->profiling = false;
+  return e;
+}
+
+// the simulated clocks after an enqueued round: every worker reaches the
+// barrier T*, idle for T* minus its busy time
+void advance_clocks(oscars_ctx* c) {
+  for (int i = 0; i < c->W; ++i) {
+    const int64_t busy = static_cast<int64_t>(c->tau[i]) * c->t_iter[i];
+    c->clock[i] += c->barrier;
+    c->idle[i] += c->barrier - busy;
+  }
+  ++c->rounds_run;
+}
+
 bool is_host_ptr(const void* p) {
   cudaPointerAttributes at;
   if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
@@ -1627,25 +1693,13 @@ oscars_status oscars_local_steps(oscars_ctx* c, int32_t* tau_out, float* loss_ou
   try {
     cudaError_t e = cudaSuccess;
     if (c->fused || c->ahead_mlp) {
-      // the one-launch round (or the per-layer round): the first round (or
-      // the first after tau changed or an evaluation) stages its own
-      // mini-batches; every round stages the next one
-      auto enqueue_ahead = [&](int b, cudaStream_t s0) {
-        return c->fused ? enqueue_round_fused_ahead(c, b, s0) : enqueue_round_mlp_ahead(c, b, s0);
-      };
+      // the one-launch round (or the per-layer round): every round stages
+      // the next one
       const int buf = c->parity;
-      if (!c->staged) {
-        c->profiling = (c->flags & 2) != 0;
-        {
-          ProfScope ps(c, "stage", c->stream);
-          e = launch_stage_round(stage_args(c, buf, nullptr), c->tau_dev, c->W, c->max_tau, c->stream);
-        }
-        c->profiling = false;
-        if (e != cudaSuccess) return cuda_fail(c, e, "local steps launch");
-      }
+      if (!c->staged && (e = stage_own_round(c, buf)) != cudaSuccess) return cuda_fail(c, e, "local steps launch");
       if (c->flags & 1) {
         c->profiling = (c->flags & 2) != 0;
-        e = enqueue_ahead(buf, c->stream);
+        e = enqueue_ahead(c, buf, c->stream);
         c->profiling = false;
       } else {
         if (!c->ahead_exec[buf]) {
@@ -1654,7 +1708,7 @@ oscars_status oscars_local_steps(oscars_ctx* c, int32_t* tau_out, float* loss_ou
           c->prof_sink = &c->prof_ahead_graph[buf];   // empty: this parity's graph does not exist yet
           e = cudaStreamBeginCapture(c->cap, cudaStreamCaptureModeThreadLocal);
           if (e == cudaSuccess) {
-            cudaError_t e2 = enqueue_ahead(buf, c->cap);
+            cudaError_t e2 = enqueue_ahead(c, buf, c->cap);
             e = cudaStreamEndCapture(c->cap, &g);
             if (e2 != cudaSuccess) e = e2;
           }
@@ -1699,13 +1753,8 @@ oscars_status oscars_local_steps(oscars_ctx* c, int32_t* tau_out, float* loss_ou
       if (e == cudaSuccess) prof_after_replay(c, c->prof_round_graph);
     }
     if (e != cudaSuccess) return cuda_fail(c, e, "local steps launch");
-    for (int i = 0; i < c->W; ++i) {
-      const int64_t busy = static_cast<int64_t>(c->tau[i]) * c->t_iter[i];
-      c->clock[i] += c->barrier;
-      c->idle[i] += c->barrier - busy;
-    }
+    advance_clocks(c);
     c->pending = true;
-    ++c->rounds_run;
     if (tau_out) std::memcpy(tau_out, c->tau.data(), c->W * sizeof(int32_t));
     if (loss_out) {
       e = cudaStreamSynchronize(c->stream);
@@ -1748,18 +1797,7 @@ oscars_status oscars_push_merge(oscars_ctx* c, const float* const* deltas, const
   if (!deltas) {
     if (!slotted(c) || !c->pending)
       return fail(c, OSCARS_ESTATE, "push_merge without deltas needs pending local steps");
-    for (int k = 0; k < c->W; ++k) a.src[k] = c->slab + static_cast<int64_t>(k) * c->P_pad;
-    auto enqueue = [&](cudaStream_t st) -> cudaError_t {
-      cudaError_t r;
-      {
-        ProfScope ps(c, "merge", st);
-        r = launch_merge(a, xg, c->P_pad, eta, true, st, c->shadow ? c->shadow + static_cast<int64_t>(c->W) * c->P_pad : nullptr);
-      }
-      if (r != cudaSuccess) return r;
-      if (c->model != OSCARS_MODEL_CNN) return cudaSuccess;   // no transposed copies to refresh
-      ProfScope ps(c, "shadow_refresh", st);
-      return refresh_global_shadows(c, st, true);
-    };
+    auto enqueue = [&](cudaStream_t st) { return enqueue_replica_merge(c, a.w, st); };
     if (c->flags & 1) {
       e = enqueue(c->stream);
     } else {
@@ -2168,6 +2206,41 @@ namespace {
 // of its W losses into a pinned host slot, push + merge) is enqueued before
 // the host waits for round r - 1 and reads that round's losses, so the host
 // work of one round overlaps the device work of the next.
+// One round of oscars_train with staged-ahead rounds (graphs on, no
+// profiling): the round, the copy of its per-worker losses into host slot
+// `slot` and the merge under the context's rule as one graph launch.  The
+// graph for (input buffer, slot) is captured once; the merge weights follow
+// tau, so a schedule change drops it.
+oscars_status train_round_graph(oscars_ctx* c, int slot) {
+  if (c->pending) return fail(c, OSCARS_ESTATE, "the previous round has not been merged");
+  const int buf = c->parity;
+  cudaError_t e = cudaSuccess;
+  if (!c->staged) e = stage_own_round(c, buf);
+  if (e == cudaSuccess && !c->train_exec[buf][slot]) {
+    std::vector<float> w(c->W);
+    merge_weights(c->rule, c->tau.data(), c->W, w.data());
+    cudaGraph_t g = nullptr;
+    e = cudaStreamBeginCapture(c->cap, cudaStreamCaptureModeThreadLocal);
+    if (e == cudaSuccess) {
+      cudaError_t e2 = enqueue_ahead(c, buf, c->cap);
+      if (e2 == cudaSuccess)
+        e2 = cudaMemcpyAsync(c->train_loss_host + slot * c->W, c->loss_dev, c->W * sizeof(float),
+                             cudaMemcpyDeviceToHost, c->cap);
+      if (e2 == cudaSuccess) e2 = enqueue_replica_merge(c, w.data(), c->cap);
+      e = cudaStreamEndCapture(c->cap, &g);
+      if (e2 != cudaSuccess) e = e2;
+    }
+    if (e == cudaSuccess) e = cudaGraphInstantiateWithFlags(&c->train_exec[buf][slot], g, 0);
+    if (g) cudaGraphDestroy(g);
+  }
+  if (e == cudaSuccess) e = cudaGraphLaunch(c->train_exec[buf][slot], c->stream);
+  if (e != cudaSuccess) return cuda_fail(c, e, "train round launch");
+  c->staged = true;
+  c->parity = buf ^ 1;
+  advance_clocks(c);   // merged in the same launch: nothing is left pending
+  return OSCARS_OK;
+}
+
 oscars_status train_pipelined(oscars_ctx* c, int32_t rounds, oscars_round_log* log, int32_t* rounds_done) {
   if (!c->train_loss_host) {
     cudaError_t e = cudaHostAlloc(&c->train_loss_host, 2 * sizeof(float) * c->W, cudaHostAllocDefault);
@@ -2190,10 +2263,16 @@ oscars_status train_pipelined(oscars_ctx* c, int32_t rounds, oscars_round_log* l
     if (rounds_done) *rounds_done = r + 1;
     return OSCARS_OK;
   };
+  const bool one_graph = (c->fused || c->ahead_mlp) && !(c->flags & 3);
   for (int32_t r = 0; r < rounds; ++r) {
-    oscars_status st = oscars_local_steps(c, nullptr, nullptr);
-    if (st == OSCARS_OK) st = oscars_losses_async(c, c->train_loss_host + (r & 1) * c->W);
-    if (st == OSCARS_OK) st = oscars_push_merge(c, nullptr, nullptr);
+    oscars_status st = OSCARS_OK;
+    if (one_graph) {
+      st = train_round_graph(c, r & 1);
+    } else {
+      st = oscars_local_steps(c, nullptr, nullptr);
+      if (st == OSCARS_OK) st = oscars_losses_async(c, c->train_loss_host + (r & 1) * c->W);
+      if (st == OSCARS_OK) st = oscars_push_merge(c, nullptr, nullptr);
+    }
     if (st != OSCARS_OK) return st;
     if (log) {
       log[r].ticks = *std::max_element(c->clock.begin(), c->clock.end());

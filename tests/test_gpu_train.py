@@ -517,6 +517,44 @@ def test_train_without_eval_matches_round_by_round(cuda_device, dims):
     b.close()
 
 
+@pytest.mark.parametrize("dims", [[784, 512, 10], [256, 256, 128, 10]], ids=["one-launch", "per-layer"])
+def test_train_follows_schedule_changes(cuda_device, dims):
+    """oscars_train runs each round, its loss copy and its merge as one cached
+    graph launch; between calls a tau override, an evaluation (which reuses
+    the first input buffer) and new iteration times (Algorithm 1 again, new
+    merge weights) must reach the next call's rounds.  Against the same
+    rounds run one call at a time, bit for bit."""
+    w = synth.TrainWorkload("train-sched", 4, dims, 64, 0.05, 1024, 8, 1)
+    shards = device_shards(w, cuda_device, n=w.samples_per_worker)
+    Xe, ye = synth.eval_np(w, n=128)
+    ex, ey = torch.from_numpy(Xe).to(cuda_device), torch.from_numpy(ye).to(cuda_device)
+    t_new = (oracle_schedule(w)[0][::-1]).copy()
+    a, _ = make_context(w, shards, cuda_device, weight_rule=P.W_LOCALSTEPS)
+    b, _ = make_context(w, shards, cuda_device, weight_rule=P.W_LOCALSTEPS)
+    logs = []
+    plan = [("train", 2), ("tau", [2, 1, 3, 1]), ("train", 2), ("eval", None), ("ticks", t_new), ("train", 3)]
+    for op, arg in plan:
+        if op == "train":
+            logs += a.train(arg)
+            for k in range(arg):
+                _, loss = b.local_steps()
+                b.push_merge()
+                assert logs[len(logs) - arg + k]["worker_loss"] == pytest.approx(
+                    float(np.mean(np.asarray(loss, np.float64))), rel=1e-6)
+        elif op == "tau":
+            a.set_local_steps(arg)
+            b.set_local_steps(arg)
+        elif op == "eval":
+            assert a.eval_loss(ex, ey) == b.eval_loss(ex, ey)
+        else:
+            a.set_iteration_ticks(arg.tolist())
+            b.set_iteration_ticks(arg.tolist())
+    np.testing.assert_array_equal(a.schedule()["clock"], b.schedule()["clock"])
+    np.testing.assert_array_equal(pull_flat(a, cuda_device), pull_flat(b, cuda_device))
+    a.close()
+    b.close()
+
+
 @pytest.mark.parametrize("dims,kernel,host", [([784, 512, 10], "fused_round", False),
                                               ([256, 256, 128, 10], "gemm_dw_sgd", False),
                                               ([512, 256, 128, 10], "gemm_dw_sgd", True)],
