@@ -489,10 +489,14 @@ __global__ void __launch_bounds__(kFT, 1) fused_mlp2_round_kernel(const __grid_c
           tc_fence_after();
           const uint32_t wa = smem_u32(w0s + kb * kW0Blk);
           const uint32_t xb = smem_u32(fring + st * Cfg::kBBytes);
+          // K slices of 16 wholly past the input's end (zero in both
+          // operands) are not issued
+          const int kleft = D - (kb_begin + kb) * kFBK;
 #pragma unroll
           for (int j = 0; j < kFBK / 16; ++j)
-            umma_bf16(tmem + kTAcc, smem_desc_k128(wa + j * 32), smem_desc_k128(xb + j * 32), idesc,
-                      (kb | j) != 0 ? 1u : 0u);
+            if (j * 16 < kleft)
+              umma_bf16(tmem + kTAcc, smem_desc_k128(wa + j * 32), smem_desc_k128(xb + j * 32), idesc,
+                        (kb | j) != 0 ? 1u : 0u);
           umma_commit(&emptyF[st]);
         }
         umma_commit(accF);
