@@ -15,12 +15,12 @@
 // Its head-weight columns, its b0 entries and a private copy of the head
 // bias (updated identically by every CTA) live in shared memory.  The model
 // is read from the global slot once, before the first step (the W0 block by
-// TMA: fp32 tiles staged in shared memory on their way to TMEM, the bf16
-// operand from the global slot's bf16 copy), and the worker's
-// replica is written once, after the last step (the W0 block through a
-// per-warp shared-memory transpose, so that every store instruction writes
-// whole 128-byte lines).  Per step only the mini-batch (staged bf16 X and X^T
-// tiles, by TMA) and the labels come from global memory.
+// TMA: fp32 tiles staged in shared memory on their way to TMEM; the bf16
+// operand is then rounded from TMEM), and the worker's replica is written
+// once, in the last step (the weight-gradient epilogue stages the updated W0
+// columns in shared memory and TMA stores them).  Per step only the
+// mini-batch (staged bf16 X and X^T tiles, by TMA) and the labels come from
+// global memory.
 //
 // Every step of the worker runs inside the cluster:
 //
@@ -53,7 +53,7 @@
 //     MMA issue overlaps the other's epilogue; the epilogue reads the
 //     gradient and the fp32 master from TMEM, applies W0 <- W0 - lr dW0,
 //     stores the master back to TMEM and its bf16 copy into the resident A
-//     operand.
+//     operand (in the worker's last step: into the replica slot instead).
 //
 // Ownership: a CTA rewrites only its own block of W0, its own b0 entries and
 // head-weight columns, and its private head bias, so its next step reads its
