@@ -218,7 +218,7 @@ def algorithmic_work(w, tau):
 # ncu capture of the kernel as it stands, with the profile summary that holds
 # it; a kernel missing here reports traffic null.
 NCU_TRAFFIC = {
-    ("fused_round", "mlp-784-512-10-W16"): (16.001024e6, "profiles/fused_round_mlp784-512-10_W16.md"),
+    ("fused_round", "mlp-784-512-10-W16"): (15.999488e6, "profiles/fused_round_mlp784-512-10_W16.md"),
 }
 
 
