@@ -1011,17 +1011,11 @@ cudaError_t enqueue_round_softreg(oscars_ctx* c, cudaStream_t st) {
   a.cursor = c->cursor;
   a.loss_part = c->loss_part;
   a.max_tau = c->max_tau;
-  cudaError_t e;
-  {
-    ProfScope ps(c, "softreg_round", st);
-    e = softreg_cluster_supported(a.D, a.C, a.B) ? launch_softreg_cluster_round(a, c->W, st)
-                                                 : launch_softreg_round(a, c->W, st);
-  }
-  if (e != cudaSuccess) return e;
-  ProfScope ps(c, "round_bookkeeping", st);
-  if ((e = launch_loss_finalize(c->loss_part, c->tau_dev, c->W, c->max_tau, 1, c->B, c->loss_dev, st)) != cudaSuccess)
-    return e;
-  return launch_cursor_advance(c->cursor, c->tau_dev, c->dn_tab, c->B, c->W, st);
+  a.loss_out = c->loss_dev;   // the round's bookkeeping in the same launch
+  a.cursor_next = c->cursor;
+  ProfScope ps(c, "softreg_round", st);
+  return softreg_cluster_supported(a.D, a.C, a.B) ? launch_softreg_cluster_round(a, c->W, st)
+                                                  : launch_softreg_round(a, c->W, st);
 }
 
 // one local step of the convolutional worker for the `na` active workers
@@ -2206,23 +2200,24 @@ namespace {
 // of its W losses into a pinned host slot, push + merge) is enqueued before
 // the host waits for round r - 1 and reads that round's losses, so the host
 // work of one round overlaps the device work of the next.
-// One round of oscars_train with staged-ahead rounds (graphs on, no
-// profiling): the round, the copy of its per-worker losses into host slot
-// `slot` and the merge under the context's rule as one graph launch.  The
-// graph for (input buffer, slot) is captured once; the merge weights follow
-// tau, so a schedule change drops it.
+// One round of oscars_train (graphs on, no profiling): the round, the copy
+// of its per-worker losses into host slot `slot` and the merge under the
+// context's rule as one graph launch.  The graph for (input buffer of a
+// staged-ahead round, slot) is captured once; the merge weights follow tau,
+// so a schedule change drops it.
 oscars_status train_round_graph(oscars_ctx* c, int slot) {
   if (c->pending) return fail(c, OSCARS_ESTATE, "the previous round has not been merged");
-  const int buf = c->parity;
+  const bool ahead = c->fused || c->ahead_mlp;
+  const int buf = ahead ? c->parity : 0;
   cudaError_t e = cudaSuccess;
-  if (!c->staged) e = stage_own_round(c, buf);
+  if (ahead && !c->staged) e = stage_own_round(c, buf);
   if (e == cudaSuccess && !c->train_exec[buf][slot]) {
     std::vector<float> w(c->W);
     merge_weights(c->rule, c->tau.data(), c->W, w.data());
     cudaGraph_t g = nullptr;
     e = cudaStreamBeginCapture(c->cap, cudaStreamCaptureModeThreadLocal);
     if (e == cudaSuccess) {
-      cudaError_t e2 = enqueue_ahead(c, buf, c->cap);
+      cudaError_t e2 = ahead ? enqueue_ahead(c, buf, c->cap) : enqueue_round(c, c->cap);
       if (e2 == cudaSuccess)
         e2 = cudaMemcpyAsync(c->train_loss_host + slot * c->W, c->loss_dev, c->W * sizeof(float),
                              cudaMemcpyDeviceToHost, c->cap);
@@ -2235,8 +2230,10 @@ oscars_status train_round_graph(oscars_ctx* c, int slot) {
   }
   if (e == cudaSuccess) e = cudaGraphLaunch(c->train_exec[buf][slot], c->stream);
   if (e != cudaSuccess) return cuda_fail(c, e, "train round launch");
-  c->staged = true;
-  c->parity = buf ^ 1;
+  if (ahead) {
+    c->staged = true;
+    c->parity = buf ^ 1;
+  }
   advance_clocks(c);   // merged in the same launch: nothing is left pending
   return OSCARS_OK;
 }
@@ -2263,7 +2260,7 @@ oscars_status train_pipelined(oscars_ctx* c, int32_t rounds, oscars_round_log* l
     if (rounds_done) *rounds_done = r + 1;
     return OSCARS_OK;
   };
-  const bool one_graph = (c->fused || c->ahead_mlp) && !(c->flags & 3);
+  const bool one_graph = !(c->flags & 3);
   for (int32_t r = 0; r < rounds; ++r) {
     oscars_status st = OSCARS_OK;
     if (one_graph) {

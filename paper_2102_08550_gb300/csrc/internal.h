@@ -51,6 +51,10 @@ struct SoftregArgs {
   const int64_t* cursor;        // [W]
   float* loss_part;             // [W][max_tau]  (sum of per-sample losses of one step)
   int max_tau;
+  // round bookkeeping in the same launch (null: not done): the worker's mean
+  // loss over its steps, and its cursor advanced by tau * B (mod the shard)
+  float* loss_out = nullptr;    // [W]
+  int64_t* cursor_next = nullptr;   // [W], may be `cursor` itself
 };
 cudaError_t launch_softreg_round(const SoftregArgs& a, int W, cudaStream_t s);
 size_t softreg_smem_bytes(int D, int C, int B);

@@ -37,6 +37,18 @@ __device__ __forceinline__ float warp_sum(float v) {
 // previous step computes (the next step's rows are loaded ahead)
 constexpr int kPrefetch = 16;
 
+// Round bookkeeping of worker w at the end of its round: the mean loss over
+// its tau steps (the step partials summed in step order in double, divided
+// by B tau) and the data cursor advanced by tau mini-batches.
+__device__ __forceinline__ void finish_worker(const SoftregArgs& a, int w, int tau, int64_t cur, int64_t n) {
+  if (a.loss_out) {
+    double sum = 0.0;
+    for (int st = 0; st < tau; ++st) sum += a.loss_part[static_cast<int64_t>(w) * a.max_tau + st];
+    a.loss_out[w] = static_cast<float>(sum / (static_cast<double>(a.B) * tau));
+  }
+  if (a.cursor_next) a.cursor_next[w] = (cur + static_cast<int64_t>(tau) * a.B) % n;
+}
+
 __global__ void __launch_bounds__(kThreads) softreg_round_kernel(const __grid_constant__ SoftregArgs a) {
   extern __shared__ __align__(16) float sm[];
   const int D = a.D, C = a.C, B = a.B;
@@ -205,6 +217,7 @@ __global__ void __launch_bounds__(kThreads) softreg_round_kernel(const __grid_co
   // push: replica <- shared memory
   for (int i = tid; i < C * D; i += kThreads) dst[a.offW + i] = Wsm[i];
   for (int i = tid; i < C; i += kThreads) dst[a.offB + i] = bsm[i];
+  if (tid == 0) finish_worker(a, w, tau, cur, n);   // the thread that wrote the loss partials
 }
 
 // The same round with each worker on a cluster of kCl CTAs that split the
@@ -413,6 +426,8 @@ __global__ void __launch_bounds__(kClThreads) softreg_cluster_round_kernel(const
   if (rank == 0)
     for (int i = tid; i < C; i += kClThreads) dst[a.offB + i] = bsm[i];
   cluster_sync();   // no CTA leaves while a peer may still read its partial logits
+  // every CTA has read the cursor; rank 0's thread 0 wrote the loss partials
+  if (rank == 0 && tid == 0) finish_worker(a, w, tau, cur, n);
 }
 
 // Mean cross-entropy of the global model: one warp per sample, partial sums

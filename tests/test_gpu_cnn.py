@@ -127,3 +127,23 @@ def test_cnn_full_size_one_round_every_worker(cuda_device):
     for k in range(w.num_workers):
         assert_within(cnn_errors(m, reps[k], rec.replicas[k]), env[k], f"worker {k} (tau {int(tau[k])})")
     assert_within(cnn_errors(m, merged, rec.x_g), env[-1], "merged")
+
+
+def test_cnn_train_matches_round_by_round(cuda_device):
+    """oscars_train runs each round of the convolutional worker, its loss
+    copy and its merge (with the transposed-copy refresh) as one graph
+    launch; the models and per-round losses are those of the same rounds run
+    one call at a time, bit for bit."""
+    B = 16
+    rows = 6 * B
+    w = synth.ConvWorkload("cnn-train", 2, [32 * 32 * 3, 10], B, 0.05, rows, 4, 2, clip=3.0, blocks=1, in_ch=3)
+    a, _, _ = make_cnn_context(w, cuda_device, rows)
+    b, _, _ = make_cnn_context(w, cuda_device, rows)
+    log = a.train(3)
+    for r in range(3):
+        _, loss = b.local_steps()
+        b.push_merge()
+        assert log[r]["worker_loss"] == pytest.approx(float(np.mean(np.asarray(loss, np.float64))), rel=1e-6)
+    np.testing.assert_array_equal(pull(a, cuda_device), pull(b, cuda_device))
+    a.close()
+    b.close()

@@ -495,12 +495,15 @@ def test_losses_async_matches_synchronous_read(cuda_device):
     ctx.close()
 
 
-@pytest.mark.parametrize("dims", [[784, 512, 10], [256, 256, 128, 10]], ids=["one-launch", "per-layer"])
-def test_train_without_eval_matches_round_by_round(cuda_device, dims):
-    """oscars_train without evaluation pipelines its rounds one deep; the
-    models and per-round losses must be those of the same rounds run one
-    call at a time (bit for bit: the same kernels in the same order)."""
-    w = synth.TrainWorkload("train-pipe", 4, dims, 64, 0.05, 512, 8, 5)
+@pytest.mark.parametrize("dims,bf16,B", [([784, 512, 10], True, 64), ([256, 256, 128, 10], True, 64),
+                                         ([784, 10], False, 32)],
+                         ids=["one-launch", "per-layer", "softmax-regression"])
+def test_train_without_eval_matches_round_by_round(cuda_device, dims, bf16, B):
+    """oscars_train without evaluation pipelines its rounds one deep, each
+    round, its loss copy and its merge one graph launch; the models and
+    per-round losses must be those of the same rounds run one call at a time
+    (bit for bit: the same kernels in the same order)."""
+    w = synth.TrainWorkload("train-pipe", 4, dims, B, 0.05, 512, 8, 5, bf16=bf16)
     shards = device_shards(w, cuda_device, n=512)
     a, _ = make_context(w, shards, cuda_device)
     log = a.train(5)
