@@ -520,6 +520,25 @@ def test_train_without_eval_matches_round_by_round(cuda_device, dims, bf16, B):
     b.close()
 
 
+@pytest.mark.parametrize("ref_flags,flags", [(0, P.FLAG_NO_GRAPH), (0, P.FLAG_PROFILE),
+                                             (P.FLAG_BRANCHES, P.FLAG_BRANCHES | P.FLAG_NO_GRAPH)],
+                         ids=["no-graph", "profile", "branches"])
+def test_train_graph_matches_other_launch_modes(cuda_device, ref_flags, flags):
+    """oscars_train launches each round, its loss copy and its merge as one
+    graph; without graphs or while profiling it runs the three calls in
+    sequence instead, and must train the same model bit for bit (also with
+    the workers' kernels on concurrent stream branches)."""
+    w = synth.TrainWorkload("train-modes", 4, [256, 256, 128, 10], 64, 0.05, 512, 8, 5)
+    shards = device_shards(w, cuda_device, n=512)
+    a, _ = make_context(w, shards, cuda_device, flags=ref_flags)
+    b, _ = make_context(w, shards, cuda_device, flags=flags)
+    la, lb = a.train(4), b.train(4)
+    assert [r["worker_loss"] for r in la] == [r["worker_loss"] for r in lb]
+    np.testing.assert_array_equal(pull_flat(a, cuda_device), pull_flat(b, cuda_device))
+    a.close()
+    b.close()
+
+
 @pytest.mark.parametrize("dims", [[784, 512, 10], [256, 256, 128, 10]], ids=["one-launch", "per-layer"])
 def test_train_follows_schedule_changes(cuda_device, dims):
     """oscars_train runs each round, its loss copy and its merge as one cached
