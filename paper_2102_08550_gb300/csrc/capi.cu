@@ -265,15 +265,6 @@ struct oscars_ctx {
   // losses and one event per slot (rounds pipelined one deep)
   float* train_loss_host = nullptr;
   cudaEvent_t train_done[2] = {nullptr, nullptr};
-  // oscars_train with staged-ahead rounds: the round from input buffer b, the
-  // loss copy into host slot h and the merge, captured as one graph [b][h]
-  cudaGraphExec_t train_exec[2][2] = {};
-  // oscars_train's graph rounds alternate between two device loss buffers
-  // (loss_dev, loss_train) so that each round's loss copy to the host runs on
-  // its own stream, off the path of the next round
-  float* loss_train = nullptr;
-  cudaStream_t loss_side = nullptr;
-  cudaEvent_t loss_fork = nullptr;
 };
 
 namespace {
@@ -377,14 +368,6 @@ bool dev_alloc(oscars_ctx* c, T** p, size_t count) {
   return true;
 }
 
-void destroy_train_graphs(oscars_ctx* c) {
-  for (auto& row : c->train_exec)
-    for (auto& g : row) {
-      if (g) cudaGraphExecDestroy(g);
-      g = nullptr;
-    }
-}
-
 void free_all(oscars_ctx* c) {
   for (auto& p : c->prof_pending)
     if (!p.graph_owned) {
@@ -407,10 +390,6 @@ void free_all(oscars_ctx* c) {
     if (e) cudaEventDestroy(e);
     e = nullptr;
   }
-  if (c->loss_fork) cudaEventDestroy(c->loss_fork);
-  c->loss_fork = nullptr;
-  if (c->loss_side) cudaStreamDestroy(c->loss_side);
-  c->loss_side = nullptr;
   if (c->train_loss_host) cudaFreeHost(c->train_loss_host);
   c->train_loss_host = nullptr;
   if (c->round_exec) cudaGraphExecDestroy(c->round_exec);
@@ -419,7 +398,6 @@ void free_all(oscars_ctx* c) {
     if (g) cudaGraphExecDestroy(g);
     g = nullptr;
   }
-  destroy_train_graphs(c);
   for (void* p : c->allocs) cudaFree(p);
   c->allocs.clear();
   if (c->cap) cudaStreamDestroy(c->cap);
@@ -619,7 +597,6 @@ oscars_status build_tables(oscars_ctx* c) {
     cudaGraphExecDestroy(c->merge_exec);
     c->merge_exec = nullptr;
   }
-  destroy_train_graphs(c);
   return ensure_stage_buffers(c);
 }
 
@@ -2210,54 +2187,6 @@ namespace {
 // of its W losses into a pinned host slot, push + merge) is enqueued before
 // the host waits for round r - 1 and reads that round's losses, so the host
 // work of one round overlaps the device work of the next.
-// One round of oscars_train (graphs on, no profiling): the round, the copy
-// of its per-worker losses into host slot `slot` and the merge under the
-// context's rule as one graph launch.  The graph for (input buffer of a
-// staged-ahead round, slot) is captured once; the merge weights follow tau,
-// so a schedule change drops it.
-oscars_status train_round_graph(oscars_ctx* c, int slot) {
-  if (c->pending) return fail(c, OSCARS_ESTATE, "the previous round has not been merged");
-  const bool ahead = c->fused || c->ahead_mlp;
-  const int buf = ahead ? c->parity : 0;
-  cudaError_t e = cudaSuccess;
-  if (ahead && !c->staged) e = stage_own_round(c, buf);
-  float* loss = slot ? c->loss_train : c->loss_dev;   // this round's loss buffer
-  if (e == cudaSuccess && !c->train_exec[buf][slot]) {
-    std::vector<float> w(c->W);
-    merge_weights(c->rule, c->tau.data(), c->W, w.data());
-    cudaGraph_t g = nullptr;
-    float* const keep = c->loss_dev;
-    c->loss_dev = loss;   // the round's kernels write their losses here
-    e = cudaStreamBeginCapture(c->cap, cudaStreamCaptureModeThreadLocal);
-    if (e == cudaSuccess) {
-      cudaError_t e2 = ahead ? enqueue_ahead(c, buf, c->cap) : enqueue_round(c, c->cap);
-      if (e2 == cudaSuccess) e2 = enqueue_replica_merge(c, w.data(), c->cap);
-      e = cudaStreamEndCapture(c->cap, &g);
-      if (e2 != cudaSuccess) e = e2;
-    }
-    c->loss_dev = keep;
-    if (e == cudaSuccess) e = cudaGraphInstantiateWithFlags(&c->train_exec[buf][slot], g, 0);
-    if (g) cudaGraphDestroy(g);
-  }
-  if (e == cudaSuccess) e = cudaGraphLaunch(c->train_exec[buf][slot], c->stream);
-  // the loss copy follows this round's graph on its own stream: the next
-  // round does not wait for it.  The host reads the slot after this copy, and
-  // the buffer is written again two rounds later, after the host's wait for
-  // this round.
-  if (e == cudaSuccess) e = cudaEventRecord(c->loss_fork, c->stream);
-  if (e == cudaSuccess) e = cudaStreamWaitEvent(c->loss_side, c->loss_fork, 0);
-  if (e == cudaSuccess)
-    e = cudaMemcpyAsync(c->train_loss_host + slot * c->W, loss, c->W * sizeof(float), cudaMemcpyDeviceToHost,
-                        c->loss_side);
-  if (e != cudaSuccess) return cuda_fail(c, e, "train round launch");
-  if (ahead) {
-    c->staged = true;
-    c->parity = buf ^ 1;
-  }
-  advance_clocks(c);   // merged in the same launch: nothing is left pending
-  return OSCARS_OK;
-}
-
 oscars_status train_pipelined(oscars_ctx* c, int32_t rounds, oscars_round_log* log, int32_t* rounds_done) {
   if (!c->train_loss_host) {
     cudaError_t e = cudaHostAlloc(&c->train_loss_host, 2 * sizeof(float) * c->W, cudaHostAllocDefault);
@@ -2267,13 +2196,7 @@ oscars_status train_pipelined(oscars_ctx* c, int32_t rounds, oscars_round_log* l
     }
     for (auto& ev : c->train_done)
       if ((e = cudaEventCreateWithFlags(&ev, cudaEventDisableTiming)) != cudaSuccess) return cuda_fail(c, e, "train event");
-    if ((e = cudaEventCreateWithFlags(&c->loss_fork, cudaEventDisableTiming)) != cudaSuccess)
-      return cuda_fail(c, e, "train event");
-    if ((e = cudaStreamCreateWithFlags(&c->loss_side, cudaStreamNonBlocking)) != cudaSuccess)
-      return cuda_fail(c, e, "train stream");
   }
-  if (!c->loss_train && !dev_alloc(c, &c->loss_train, std::max(c->W, 1)))
-    return fail(c, OSCARS_ENOMEM, "device allocation failed (train losses)");
   auto finish = [&](int32_t r) -> oscars_status {
     const cudaError_t e = cudaEventSynchronize(c->train_done[r & 1]);
     if (e != cudaSuccess) return cuda_fail(c, e, "train round");
@@ -2286,37 +2209,21 @@ oscars_status train_pipelined(oscars_ctx* c, int32_t rounds, oscars_round_log* l
     if (rounds_done) *rounds_done = r + 1;
     return OSCARS_OK;
   };
-  const bool one_graph = !(c->flags & 3);
   for (int32_t r = 0; r < rounds; ++r) {
-    oscars_status st = OSCARS_OK;
-    if (one_graph) {
-      st = train_round_graph(c, r & 1);
-    } else {
-      st = oscars_local_steps(c, nullptr, nullptr);
-      if (st == OSCARS_OK) st = oscars_losses_async(c, c->train_loss_host + (r & 1) * c->W);
-      if (st == OSCARS_OK) st = oscars_push_merge(c, nullptr, nullptr);
-    }
+    oscars_status st = oscars_local_steps(c, nullptr, nullptr);
+    if (st == OSCARS_OK) st = oscars_losses_async(c, c->train_loss_host + (r & 1) * c->W);
+    if (st == OSCARS_OK) st = oscars_push_merge(c, nullptr, nullptr);
     if (st != OSCARS_OK) return st;
     if (log) {
       log[r].ticks = *std::max_element(c->clock.begin(), c->clock.end());
       log[r].barrier = c->barrier;
       log[r].eval_loss = std::numeric_limits<float>::quiet_NaN();
     }
-    // a round is done for the host once its losses are in the host slot
-    const cudaError_t e = cudaEventRecord(c->train_done[r & 1], one_graph ? c->loss_side : c->stream);
+    const cudaError_t e = cudaEventRecord(c->train_done[r & 1], c->stream);
     if (e != cudaSuccess) return cuda_fail(c, e, "train event");
     if (r >= 1 && (st = finish(r - 1)) != OSCARS_OK) return st;
   }
-  oscars_status st = finish(rounds - 1);
-  if (st == OSCARS_OK && one_graph) {
-    // the last round's losses stay readable where the single-round calls
-    // keep them, and its merge has finished
-    cudaError_t e = cudaSuccess;
-    if ((rounds - 1) & 1)
-      e = cudaMemcpyAsync(c->loss_dev, c->loss_train, c->W * sizeof(float), cudaMemcpyDeviceToDevice, c->stream);
-    if (e == cudaSuccess) e = cudaStreamSynchronize(c->stream);
-    if (e != cudaSuccess) st = cuda_fail(c, e, "train round");
-  }
+  const oscars_status st = finish(rounds - 1);
   // the kernels' error word is sticky: one read after the last round reports
   // a bounded wait that ran out in any of them
   return st == OSCARS_OK ? check_err_word(c) : st;

@@ -130,10 +130,10 @@ def test_cnn_full_size_one_round_every_worker(cuda_device):
 
 
 def test_cnn_train_matches_round_by_round(cuda_device):
-    """oscars_train runs each round of the convolutional worker, its loss
-    copy and its merge (with the transposed-copy refresh) as one graph
-    launch; the models and per-round losses are those of the same rounds run
-    one call at a time, bit for bit."""
+    """oscars_train pipelines the rounds of the convolutional worker and their
+    merges (with the transposed-copy refresh); the models and per-round
+    losses are those of the same rounds run one call at a time, bit for
+    bit."""
     B = 16
     rows = 6 * B
     w = synth.ConvWorkload("cnn-train", 2, [32 * 32 * 3, 10], B, 0.05, rows, 4, 2, clip=3.0, blocks=1, in_ch=3)

@@ -499,10 +499,9 @@ def test_losses_async_matches_synchronous_read(cuda_device):
                                          ([784, 10], False, 32)],
                          ids=["one-launch", "per-layer", "softmax-regression"])
 def test_train_without_eval_matches_round_by_round(cuda_device, dims, bf16, B):
-    """oscars_train without evaluation pipelines its rounds one deep, each
-    round, its loss copy and its merge one graph launch; the models and
-    per-round losses must be those of the same rounds run one call at a time
-    (bit for bit: the same kernels in the same order)."""
+    """oscars_train without evaluation pipelines its rounds one deep; the
+    models and per-round losses must be those of the same rounds run one
+    call at a time (bit for bit: the same kernels in the same order)."""
     w = synth.TrainWorkload("train-pipe", 4, dims, B, 0.05, 512, 8, 5, bf16=bf16)
     shards = device_shards(w, cuda_device, n=512)
     a, _ = make_context(w, shards, cuda_device)
@@ -523,11 +522,10 @@ def test_train_without_eval_matches_round_by_round(cuda_device, dims, bf16, B):
 @pytest.mark.parametrize("ref_flags,flags", [(0, P.FLAG_NO_GRAPH), (0, P.FLAG_PROFILE),
                                              (P.FLAG_BRANCHES, P.FLAG_BRANCHES | P.FLAG_NO_GRAPH)],
                          ids=["no-graph", "profile", "branches"])
-def test_train_graph_matches_other_launch_modes(cuda_device, ref_flags, flags):
-    """oscars_train launches each round, its loss copy and its merge as one
-    graph; without graphs or while profiling it runs the three calls in
-    sequence instead, and must train the same model bit for bit (also with
-    the workers' kernels on concurrent stream branches)."""
+def test_train_matches_other_launch_modes(cuda_device, ref_flags, flags):
+    """oscars_train with its rounds and merges launched as CUDA graphs must
+    train the same model bit for bit as without graphs or while profiling
+    (also with the workers' kernels on concurrent stream branches)."""
     w = synth.TrainWorkload("train-modes", 4, [256, 256, 128, 10], 64, 0.05, 512, 8, 5)
     shards = device_shards(w, cuda_device, n=512)
     a, _ = make_context(w, shards, cuda_device, flags=ref_flags)
@@ -541,11 +539,11 @@ def test_train_graph_matches_other_launch_modes(cuda_device, ref_flags, flags):
 
 @pytest.mark.parametrize("dims", [[784, 512, 10], [256, 256, 128, 10]], ids=["one-launch", "per-layer"])
 def test_train_follows_schedule_changes(cuda_device, dims):
-    """oscars_train runs each round, its loss copy and its merge as one cached
-    graph launch; between calls a tau override, an evaluation (which reuses
-    the first input buffer) and new iteration times (Algorithm 1 again, new
-    merge weights) must reach the next call's rounds.  Against the same
-    rounds run one call at a time, bit for bit."""
+    """oscars_train pipelines its rounds through cached round and merge
+    graphs; between calls a tau override, an evaluation (which reuses the
+    first input buffer) and new iteration times (Algorithm 1 again, new merge
+    weights) must reach the next call's rounds.  Against the same rounds run
+    one call at a time, bit for bit."""
     w = synth.TrainWorkload("train-sched", 4, dims, 64, 0.05, 1024, 8, 1)
     shards = device_shards(w, cuda_device, n=w.samples_per_worker)
     Xe, ye = synth.eval_np(w, n=128)
