@@ -1782,7 +1782,8 @@ oscars_status oscars_push_merge(oscars_ctx* c, const float* const* deltas, const
     if (c->flags & 1) {
       e = enqueue(c->stream);
     } else {
-      // the weights and buffers of a replica-mode merge never change: one graph
+      // the buffers of a replica-mode merge never change and its weights only
+      // with the schedule, which drops the graph: one graph
       if (!c->merge_exec || c->rule == OSCARS_W_EXPLICIT) {
         if (c->merge_exec) cudaGraphExecDestroy(c->merge_exec);
         c->merge_exec = nullptr;
