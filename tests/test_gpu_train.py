@@ -307,16 +307,19 @@ def test_protocol_errors(cuda_device):
     ctx.close()
 
 
-@pytest.mark.parametrize("dims", [[784, 512, 10], [256, 128, 128, 10], [1024, 256, 128, 10]],
-                         ids=["fused", "per-layer", "per-layer-strided"])
-def test_pinned_host_shards_match_device_shards(cuda_device, dims):
+@pytest.mark.parametrize("dims,B", [([784, 512, 10], 64), ([256, 128, 128, 10], 64), ([1024, 256, 128, 10], 64),
+                                    ([1000, 256, 128, 10], 32)],
+                         ids=["fused", "per-layer", "per-layer-strided", "per-layer-strided-ragged"])
+def test_pinned_host_shards_match_device_shards(cuda_device, dims, B):
     """Shards in pinned host memory (read over the host link by the staging
     kernel) give bit-identical rounds to the same shards in device memory.
     The per-layer path stages host rows from a fixed number of blocks
     striding over the tiles; at 1024 inputs a round has more tiles (8 feature
     blocks x 2 row blocks x every (step, worker) slot) than blocks, so each
-    block stages several."""
-    w = synth.TrainWorkload("host-shards", 3, dims, 64, 0.05, 256, 6, 2)
+    block stages several; at 1000 inputs the last feature block of every slot
+    holds 104 of 128 columns (the batch of a bf16 MLP is a multiple of the
+    32-row block, so row blocks are always whole)."""
+    w = synth.TrainWorkload("host-shards", 3, dims, B, 0.05, 256, 6, 2)
     dev_shards = device_shards(w, cuda_device, n=256)
     host_shards = [(x.cpu().pin_memory(), y.cpu().pin_memory()) for x, y in dev_shards]
     outs = []
